@@ -1,0 +1,293 @@
+/*
+ * kvg.h — C ABI of libkvg: byte-exact KV-state graft and GQA decode attention
+ * on one GB300 (sm_103a).
+ *
+ * The operations follow the problem statement of "Byte-Exact KV-State
+ * Grafting" (arxiv 2607.14431):
+ *   - deposit: a computed KV state is captured once, with its positions, as a
+ *     persistent block (Sec. 3.3, deposit step of the flywheel; Sec. 4.4);
+ *   - graft: the block is installed into a fresh context at the positions it
+ *     was captured at, [0, N), and new queries are computed on top at
+ *     [N, N+q) (Sec. 3.2, "position consistency");
+ *   - relocate: optionally the block is re-based to another absolute offset,
+ *     which re-rotates its keys and is not byte-exact (Sec. 4.2);
+ *   - decode: attention of a new query over the grafted context (Sec. 3.2,
+ *     Sec. 4.3);
+ *   - digest: SHA-256 of raw bytes, the paper's byte-exactness test (Sec. 3.2)
+ *     and its per-block integrity check (Sec. 4.11).
+ *
+ * Conventions for every call:
+ *   - No exceptions cross the ABI and nothing aborts the process: each call
+ *     returns a kvg_status.  Arguments are checked on the host before any GPU
+ *     work is enqueued; a call that fails a host check changes no state.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *     stream).  GPU work is enqueued on it and the call returns without
+ *     waiting unless a flag asks for it.  Errors that only the GPU can see
+ *     (a digest mismatch, a failed device-side bounds check) are recorded in
+ *     the cache's device status word and reported by kvg_sync().
+ *   - Element type: bf16 only (raw 16-bit patterns).  Sizes are in elements
+ *     unless a name ends in _bytes.
+ *   - Ownership: stores, caches and their device memory belong to the
+ *     library; buffers passed in (k, v, q, out, positions) belong to the
+ *     caller and must stay valid until the enqueued work completes.
+ *   - Threads: a store or cache must not be used from two host threads at
+ *     once.  Different caches are independent.
+ */
+#ifndef KVG_H
+#define KVG_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum kvg_status {
+    KVG_OK = 0,
+    KVG_ERR_ARG = -1,          /* bad argument or unsupported geometry */
+    KVG_ERR_OOM = -2,          /* device or pinned-host allocation failed */
+    KVG_ERR_CUDA = -3,         /* a CUDA runtime call failed */
+    KVG_ERR_NOT_FOUND = -4,    /* no such block id */
+    KVG_ERR_CAPACITY = -5,     /* not enough free pages, slots or store bytes */
+    KVG_ERR_POSITION = -6,     /* position tag + delta outside [0, 2^31) */
+    KVG_ERR_DIGEST = -7,       /* a page digest did not match the stored one */
+    KVG_ERR_FORMAT = -8,       /* serialized block header or layout invalid */
+    KVG_ERR_TIMEOUT = -9,      /* kvg_sync gave up waiting */
+    KVG_ERR_DEVICE_CHECK = -10 /* a kernel's own bounds/wait check failed */
+} kvg_status;
+
+enum { KVG_RESIDENCY_HBM = 0, KVG_RESIDENCY_PINNED_HOST = 1 };
+enum { KVG_ROPE_HALF = 0, KVG_ROPE_INTERLEAVED = 1 };
+enum { KVG_GRAFT_VERIFY = 1u, KVG_GRAFT_SYNC = 2u };
+enum { KVG_SHA256_PLAIN = 0, KVG_SHA256_PAGED = 1 };
+
+/* Leaf size of the two-level page digest (bytes). */
+#define KVG_DIGEST_LEAF_BYTES 4096
+/* Most page indices a graft report lists. */
+#define KVG_REPORT_MAX_PAGES 64
+
+/* KV geometry shared by a store and the caches it grafts into.
+ * A page holds page_size consecutive token slots of every KV head:
+ * bf16 [n_kv_heads][page_size][head_dim] per layer and per K or V, so
+ * page_bytes = 2 * n_kv_heads * page_size * head_dim.
+ * Supported: head_dim in {64, 128, 256}; page_size >= 1; page_bytes a
+ * multiple of 16.  rope_theta / rope_style only matter for relocation:
+ * the rotation pairs dimension i with i + head_dim/2 (KVG_ROPE_HALF) or
+ * 2i with 2i+1 (KVG_ROPE_INTERLEAVED) at frequency rope_theta^(-2i/head_dim). */
+typedef struct kvg_dims {
+    int32_t n_layers;
+    int32_t n_kv_heads;
+    int32_t head_dim;
+    int32_t page_size;
+    double rope_theta;
+    int32_t rope_style;
+    int32_t reserved;
+} kvg_dims;
+
+typedef struct kvg_store kvg_store;
+typedef struct kvg_cache kvg_cache;
+
+/* ---------------------------------------------------------------- store -- */
+
+/* A store holds serialized blocks (the paper's persistent artifacts, Sec. 3.3,
+ * Sec. 4.4) in HBM or in pinned host memory, up to capacity_bytes.  Block ids
+ * are 0, 1, 2, ... in deposit/import order.  Pinned-host stores are carved
+ * from 1 GiB (or larger, for larger blocks) page-locked slabs allocated on
+ * demand; a block never straddles two slabs.
+ * device: CUDA ordinal used for HBM stores and for the store's kernels. */
+kvg_status kvg_store_create(const kvg_dims *dims, int32_t residency, uint64_t capacity_bytes,
+                            int32_t device, kvg_store **out);
+void kvg_store_destroy(kvg_store *store);
+
+/* Serialized block layout (little-endian), one contiguous region:
+ *   [0, 256)      header: magic "KVGBLK01", u32 version = 1, u32 header bytes
+ *                 = 256, i32 n_layers, n_kv_heads, head_dim, page_size,
+ *                 i64 n_tokens, i64 n_pages, f64 rope_theta, i32 rope_style,
+ *                 i32 dtype (1 = bf16), u64 positions_offset, digests_offset,
+ *                 pages_offset, total_bytes; at byte 96 the 32-byte block
+ *                 digest; the rest zero.
+ *   positions     int32 [n_tokens] position tags (offset 256)
+ *   digests       [n_layers][2][n_pages][32] page digests (256-aligned)
+ *   pages         bf16 [n_layers][2][n_pages][n_kv_heads][page_size][head_dim]
+ *                 (4096-aligned), kv 0 = K, 1 = V; token t of the block is row
+ *                 t % page_size of page t / page_size; rows past n_tokens in
+ *                 the last page are zero.
+ * Page digest = SHA-256 over the concatenated SHA-256 digests of the page's
+ * consecutive 4096-byte leaves (the last leaf may be shorter).  Block digest =
+ * SHA-256 over the position tags (int32 LE) followed by all page digests. */
+typedef struct kvg_block_info {
+    int64_t n_tokens;
+    int64_t n_pages;           /* pages per layer per K/V */
+    int32_t residency;
+    int32_t reserved;
+    const void *bytes;         /* device pointer (HBM store) or host pointer */
+    uint64_t total_bytes;
+    uint64_t positions_offset;
+    uint64_t digests_offset;
+    uint64_t pages_offset;
+    uint8_t block_digest[32];  /* read back from the block header (synchronous) */
+} kvg_block_info;
+
+/* Describes block `block_id`.  Synchronizes the device (it reads the header
+ * the deposit kernels wrote).  KVG_ERR_NOT_FOUND for an unknown id. */
+kvg_status kvg_store_block_info(kvg_store *store, uint64_t block_id, kvg_block_info *out);
+
+/* Copies a serialized block (host memory, e.g. read from a block file) into
+ * the store.  The header is validated against the store's geometry
+ * (KVG_ERR_FORMAT); with KVG_GRAFT_VERIFY every page digest and the block
+ * digest are recomputed on the GPU and compared (KVG_ERR_DIGEST; the block is
+ * then not added).  Synchronous.  This is how a block file moves between
+ * machines (Sec. 4.11). */
+kvg_status kvg_store_import(kvg_store *store, const void *bytes, uint64_t n_bytes, uint32_t flags,
+                            uint64_t *block_id_out);
+
+/* Copies block `block_id`'s serialized bytes to host memory `dst` (capacity
+ * dst_bytes >= total_bytes).  Synchronous. */
+kvg_status kvg_store_export(kvg_store *store, uint64_t block_id, void *dst, uint64_t dst_bytes);
+
+/* ---------------------------------------------------------------- cache -- */
+
+/* A paged KV cache on `device`: pool bf16 [n_layers][2][n_pages][n_kv_heads]
+ * [page_size][head_dim] (one page id names the same token rows in every
+ * layer), and per sequence a page table, per-page fill counts, position tags
+ * per slot and a slot high-water mark.  The pool is not initialised.
+ * Free pages are handed out from the front of an ordered free list,
+ * initially 0, 1, ..., n_pages-1; a released sequence's pages go to its back
+ * in page-table order.  max_slots bounds one sequence's slots. */
+kvg_status kvg_cache_create(const kvg_dims *dims, int32_t n_pages, int32_t max_seqs,
+                            int32_t max_slots, int32_t device, kvg_cache **out);
+void kvg_cache_destroy(kvg_cache *cache);
+
+/* Replaces the free-list order by the permutation order[0..n_pages).  Only
+ * while every page is free (KVG_ERR_ARG otherwise).  Physical placement never
+ * changes any result: attention reduces in logical token order. */
+kvg_status kvg_cache_set_free_order(kvg_cache *cache, const int32_t *order, int32_t n_pages);
+
+/* Device-side layout, for inspection and for interop with other kernels. */
+typedef struct kvg_cache_view {
+    void *pool;            /* bf16 [L][2][n_pages][Hkv][P][D] */
+    int32_t *page_table;   /* int32 [max_seqs][max_pages], -1 = no page */
+    int32_t *page_fill;    /* int32 [max_seqs][max_pages], valid rows (a prefix) */
+    int32_t *positions;    /* int32 [max_seqs][max_slots], -1 = unwritten */
+    uint64_t pool_bytes;
+    uint64_t page_bytes;
+    int32_t n_pages;
+    int32_t max_seqs;
+    int32_t max_slots;
+    int32_t max_pages;     /* ceil(max_slots / page_size) */
+} kvg_cache_view;
+kvg_status kvg_cache_view_get(const kvg_cache *cache, kvg_cache_view *out);
+
+/* Host-side bookkeeping of sequence `seq`: slot high-water mark and pages held. */
+kvg_status kvg_cache_seq_info(const kvg_cache *cache, int32_t seq, int32_t *n_slots,
+                              int32_t *n_pages);
+
+/* Fresh write (the "fresh" arm the graft must reproduce, Sec. 3.2): rows
+ * t = 0..n-1 of k and v (device, bf16 [n_layers][n][n_kv_heads][head_dim],
+ * post-RoPE as a prefill produced them) and positions (device int32 [n]) go
+ * to slots s = n_slots + t of `seq`, allocating pages as needed.
+ * KVG_ERR_CAPACITY if slots or pages run out (nothing is written). */
+kvg_status kvg_cache_append(kvg_cache *cache, int32_t seq, const void *k, const void *v,
+                            const int32_t *positions, int32_t n, void *stream);
+
+/* Returns the sequence's pages to the free list and clears its page table,
+ * fills and position tags. */
+kvg_status kvg_cache_release(kvg_cache *cache, int32_t seq, void *stream);
+
+/* ----------------------------------------------------------- deposit -- */
+
+/* Captures slots [slot0, slot0+n) of `seq` (slot0 a multiple of page_size,
+ * slot0 + n <= n_slots) with their position tags into a new block of `store`
+ * (layout above), computing every page digest and the block digest on the
+ * GPU.  Sec. 3.3 deposit; the block is byte-identical to one built from the
+ * same rows anywhere else.  KVG_ERR_CAPACITY if the store is full. */
+kvg_status kvg_deposit(kvg_store *store, const kvg_cache *cache, int32_t seq, int32_t slot0,
+                       int32_t n, void *stream, uint64_t *block_id_out);
+
+/* -------------------------------------------------------------- graft -- */
+
+typedef struct kvg_graft_report {
+    int32_t seq;
+    int32_t n_pages_checked;   /* pages hashed (L * 2 * n_pages) */
+    int32_t n_mismatch;        /* pages whose digest differed */
+    int32_t n_listed;
+    int32_t mismatch_pages[KVG_REPORT_MAX_PAGES]; /* index (l * 2 + kv) * n_pages + j */
+} kvg_graft_report;
+
+/* Own-position graft (Sec. 3.2): installs block `block_id` into sequence
+ * `seq` at slot dst_slot, which must be the sequence's next page boundary
+ * (ceil(n_slots / page_size) * page_size; pass -1 for that).  The block's
+ * pages are copied whole into freshly allocated cache pages, its position
+ * tags are written to the slots, and n_slots becomes dst_slot + n_tokens.
+ * The graft is a byte copy: restored rows equal the deposited rows bit for
+ * bit, so attention over them equals attention over the same rows written
+ * fresh.
+ * delta != 0 re-bases the block (Sec. 4.2): position tags become tag + delta,
+ * and each valid key row is rotated by delta positions (fp32 arithmetic on a
+ * host-fp64 cos/sin table, rounded to bf16 RNE); value rows and padding rows
+ * are copied unchanged.  delta == 0 is the pure copy.
+ * Blocks of a pinned-host store are read by the GPU directly from host memory.
+ * flags: KVG_GRAFT_VERIFY hashes every page the graft read (delta != 0: the
+ * store's pages; delta == 0: the restored cache pages) and compares with the
+ * stored digests; KVG_GRAFT_SYNC waits for completion, fills `report`
+ * (nullable) and returns KVG_ERR_DIGEST on a mismatch.  Without SYNC a
+ * mismatch surfaces at the next kvg_sync().
+ * Errors (no state change): KVG_ERR_NOT_FOUND, KVG_ERR_ARG (geometry or
+ * dst_slot), KVG_ERR_CAPACITY (pages or slots), KVG_ERR_POSITION. */
+kvg_status kvg_graft(kvg_store *store, uint64_t block_id, kvg_cache *cache, int32_t seq,
+                     int32_t dst_slot, int64_t delta, uint32_t flags, void *stream,
+                     kvg_graft_report *report);
+
+/* ------------------------------------------------------------- decode -- */
+
+/* Decode attention of one query token per sequence (Sec. 3.2, Sec. 4.3):
+ * for batch row b (sequence seq_ids[b], host array), query head h and KV head
+ * g = h / (n_q_heads / n_kv_heads):
+ *     o[h] = sum_t softmax_t(scale * q[h] . k_t[g]) v_t[g]
+ * over every valid row of the sequence (pages in logical order, rows below
+ * their fill), accumulated in fp32 and rounded to bf16 (RNE).  An empty
+ * sequence gives o = 0.
+ * q, out: device bf16 [n_layers_run][B][n_q_heads][head_dim] where
+ * layer >= 0 runs that layer only (n_layers_run = 1) and layer == -1 runs all
+ * layers in one launch.  The reduction order depends only on the logical
+ * token index, never on physical page placement, so results are bitwise
+ * reproducible and identical for grafted and freshly written rows.
+ * n_q_heads must be a multiple of n_kv_heads with group size in {1, 2, 4, 8}
+ * and group * head_dim <= 512.  B <= 4096. */
+kvg_status kvg_decode_attention(kvg_cache *cache, int32_t layer, const int32_t *seq_ids,
+                                int32_t B, const void *q, int32_t n_q_heads, void *out,
+                                float scale, void *stream);
+
+/* ------------------------------------------------------------- digest -- */
+
+/* SHA-256 (FIPS 180-4) on the GPU.
+ * KVG_SHA256_PLAIN: out[32] = SHA-256 of bytes[0, n) (one serial chain).
+ * KVG_SHA256_PAGED: n must be a multiple of page_bytes; out[32 * i] = the
+ *   two-level digest of page i = bytes[i * page_bytes, (i+1) * page_bytes).
+ * bytes and out are device pointers (or pinned host memory the GPU can
+ * reach).  Uses the library's per-device scratch (leaf digests). */
+kvg_status kvg_digest(const void *bytes, uint64_t n, int32_t mode, uint64_t page_bytes,
+                      uint8_t *out, void *stream);
+
+/* --------------------------------------------------------------- misc -- */
+
+/* Waits (up to timeout_s seconds, polling) for `stream`, then reads and clears
+ * the cache's device status word.  Returns KVG_ERR_TIMEOUT if the stream is
+ * still busy, KVG_ERR_DIGEST after a failed verification (report, nullable,
+ * gets the details), KVG_ERR_DEVICE_CHECK if a kernel's own check failed. */
+kvg_status kvg_sync(kvg_cache *cache, void *stream, double timeout_s, kvg_graft_report *report);
+
+const char *kvg_status_string(kvg_status status);
+
+/* Human-readable detail of the last failed call on this host thread (empty if
+ * none); valid until the next call on the thread. */
+const char *kvg_last_error(void);
+
+/* Library version, e.g. 0x000100 for 0.1.0. */
+uint32_t kvg_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVG_H */

@@ -1,0 +1,245 @@
+// common.cuh — internal declarations shared by the libkvg translation units:
+// device status word, kernel parameter blocks, inline-PTX helpers for
+// mbarriers and bulk (TMA, non-tensor) copies, and the launchers each .cu
+// exports to the host runtime.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "kvg.h"
+
+namespace kvg {
+
+// ---------------------------------------------------------------- limits --
+constexpr int kMaxPagesPerLaunch = 1024;  // page ids carried in kernel params
+constexpr int kMaxBatchPerLaunch = 256;   // decode rows carried in kernel params
+constexpr int kMaxHalfDim = 128;          // head_dim <= 256
+constexpr uint64_t kLeafBytes = KVG_DIGEST_LEAF_BYTES;
+
+// Device status word of a cache (or of a library-level scratch).  Kernels
+// record the first error code they see; digest checks count mismatches and
+// list the first KVG_REPORT_MAX_PAGES page indices.
+struct DevStatus {
+    int32_t err;           // 0 or a kvg_status (negative)
+    int32_t err_detail;    // kernel-specific detail of the first error
+    int32_t n_mismatch;
+    int32_t n_checked;
+    int32_t seq;
+    int32_t pad[3];
+    int32_t list[KVG_REPORT_MAX_PAGES];
+};
+
+struct PageList {
+    int32_t n;
+    int32_t pid[kMaxPagesPerLaunch];
+};
+
+// ------------------------------------------------------------ graft copy --
+// One launch copies n_units = n_layers * 2 * npb pages (block page order
+// (l * 2 + kv) * npb + j) from `src` (contiguous block pages) into the pool
+// pages named by pids, optionally rotating the valid key rows.
+struct GraftParams {
+    const uint8_t *src;        // block pages region (device or host-mapped)
+    uint8_t *pool;             // cache pool
+    uint64_t page_bytes;
+    int64_t pool_pages;        // n_pages of the pool (stride between (l,kv) planes)
+    int32_t n_layers;
+    int32_t npb;               // pages of this launch per (l, kv)
+    int32_t page_base;         // block page index of the first page of this launch
+    int32_t block_pages;       // block pages per (l, kv) (stride of src planes)
+    int32_t chunk_bytes;       // unit of work: divides page_bytes, multiple of 16
+    int32_t rotate;            // 0 copy, 1 half-split rotation, 2 interleaved rotation
+    int32_t n_kv_heads, page_size, head_dim;
+    int64_t n_tokens;          // block tokens (rows >= n_tokens are padding)
+    float cosv[kMaxHalfDim];
+    float sinv[kMaxHalfDim];
+    // metadata written by the same launch
+    const int32_t *src_pos;    // block position tags (this launch's tokens start at page_base*P)
+    int32_t *dst_pos;          // positions row of the sequence + dst slot of page_base
+    int32_t *table_row;        // page_table row + first page index of this launch
+    int32_t *fill_row;         // page_fill row + first page index of this launch
+    int64_t delta;
+    PageList pids;
+};
+
+// ---------------------------------------------------------------- append --
+struct AppendParams {
+    const uint16_t *k, *v;     // [L][n][Hkv][D]
+    const int32_t *pos;        // [n]
+    uint8_t *pool;
+    int64_t pool_pages;
+    int32_t n_layers, n_kv_heads, page_size, head_dim;
+    int32_t n;                 // rows of this launch
+    int32_t row0;              // first row of this launch within k/v/pos
+    int32_t slot0;             // slot of row0
+    int32_t page0;             // page index (within the sequence) of pids.pid[0]
+    int32_t n_rows_total;      // rows of the whole k/v arrays (their token stride)
+    int32_t *pos_row;          // positions row of the sequence
+    int32_t *table_row;        // page_table row
+    int32_t *fill_row;         // page_fill row
+    PageList pids;             // pages touched: page0 .. page0 + n - 1
+};
+
+// --------------------------------------------------------------- deposit --
+struct GatherParams {
+    const uint8_t *pool;
+    uint8_t *dst;              // block pages region
+    uint64_t page_bytes;
+    int64_t pool_pages;
+    int32_t n_layers, npb, page_base, block_pages;
+    int32_t n_kv_heads, page_size, head_dim;
+    int64_t n_tokens;          // rows >= n_tokens are written as zero
+    const int32_t *src_pos;    // positions row + slot0
+    int32_t *dst_pos;          // block positions
+    PageList pids;
+};
+
+struct HeaderParams {
+    uint8_t *dst;
+    uint8_t bytes[256];
+};
+
+// ---------------------------------------------------------------- digest --
+// Address of page p: contiguous (pid == nullptr): base + p * page_bytes;
+// cache pages: base + ((p / npb) * plane_pages + pid[p % npb]) * page_bytes.
+struct PageSource {
+    const uint8_t *base;
+    uint64_t page_bytes;
+    const int32_t *pid;
+    int32_t npb;
+    int64_t plane_pages;
+};
+
+// --------------------------------------------------------------- decode --
+struct BatchRows {
+    int32_t seq[kMaxBatchPerLaunch];
+    int32_t npages[kMaxBatchPerLaunch];
+};
+
+struct DecodeParams {
+    const uint8_t *pool;
+    int64_t pool_pages;
+    int32_t n_kv_heads, page_size, n_q_heads;
+    int32_t layer0, n_layers_run, B;
+    int32_t n_splits, pages_per_split;
+    const int32_t *page_table;
+    const int32_t *page_fill;
+    int32_t max_pages;
+    const __nv_bfloat16 *q;    // [Lrun][B][Hq][D] (this launch's rows)
+    int32_t q_row_stride_b;    // rows of the full batch (B of the whole call)
+    int32_t b0;                // first batch row of this launch
+    float qscale;              // softmax scale * log2(e)
+    float *part_o;             // [Lrun][B][Hkv][S][G][D]
+    float2 *part_ml;           // [Lrun][B][Hkv][S][G]
+    DevStatus *status;
+    BatchRows rows;
+};
+
+struct CombineParams {
+    const float *part_o;
+    const float2 *part_ml;
+    __nv_bfloat16 *out;        // [Lrun][B][Hq][D]
+    int32_t n_kv_heads, n_q_heads, n_splits, B, q_row_stride_b, b0;
+};
+
+// -------------------------------------------------------------- launchers --
+cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s);
+cudaError_t launch_append(const AppendParams &p, int n_sm, cudaStream_t s);
+cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s);
+cudaError_t launch_write_header(const HeaderParams &p, cudaStream_t s);
+cudaError_t launch_reset_seq(int32_t *table_row, int32_t *fill_row, int32_t max_pages,
+                             int32_t *pos_row, int32_t max_slots, cudaStream_t s);
+
+// leaf digests (8 uint32 words per leaf, host order of the hash state)
+cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_t *leaf_words,
+                                 int n_sm, cudaStream_t s);
+// page digests from leaf digests; writes out (nullable, 32 bytes per page) and
+// compares with expected (nullable), recording mismatches in status.
+cudaError_t launch_sha256_pages(const uint32_t *leaf_words, int64_t n_pages, int64_t leaves_per_page,
+                                uint8_t *out, const uint8_t *expected, DevStatus *status,
+                                int32_t seq, cudaStream_t s);
+// SHA-256 of seg0 || seg1 (one thread); expected (nullable) compared like above.
+cudaError_t launch_sha256_serial(const uint8_t *seg0, uint64_t n0, const uint8_t *seg1, uint64_t n1,
+                                 uint8_t *out, const uint8_t *expected, DevStatus *status,
+                                 cudaStream_t s);
+
+cudaError_t launch_decode(int head_dim, int group, const DecodeParams &p, cudaStream_t s);
+cudaError_t launch_combine(int head_dim, int group, const CombineParams &p, int n_layers_run,
+                           int B, cudaStream_t s);
+bool decode_supported(int head_dim, int group);
+size_t decode_smem_bytes(int head_dim);
+
+// ------------------------------------------------------------ PTX helpers --
+#ifdef __CUDACC__
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
+                 : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t global_timer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Bounded wait on an mbarrier phase: gives up after ~2 s of wall time and
+// returns false (the caller records KVG_ERR_DEVICE_CHECK and unwinds).
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 0;; ++it) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((it & 255u) == 255u && global_timer_ns() - t0 > 2000000000ull) return false;
+    }
+}
+
+// Bulk (non-tensor) asynchronous copy global -> this CTA's shared memory,
+// completing `bytes` of transaction count on `bar`.  dst/src 16-byte aligned,
+// bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes,
+                                         uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+            "r"(smem_addr(dst)),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void record_error(DevStatus *st, int32_t code, int32_t detail) {
+    if (st && atomicCAS(&st->err, 0, code) == 0) st->err_detail = detail;
+}
+#endif
+
+}  // namespace kvg

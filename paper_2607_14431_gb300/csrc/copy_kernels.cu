@@ -1,0 +1,296 @@
+// copy_kernels.cu — the byte-moving kernels of the graft path.
+//
+//  graft_kernel<ROT>: own-position graft (Sec. 3.2) copies block pages into
+//    the cache pages a sequence was given; with ROT != 0 the valid key rows
+//    are re-based by an offset (Sec. 4.2) on the way.  Work unit = one chunk
+//    of one page; the grid strides over all units so a single launch covers
+//    every layer, K and V.  Loads and stores are 16-byte vectors with the
+//    streaming cache hint (the data is touched once).
+//  append_kernel: the "fresh" write of prefill-shaped rows into slots.
+//  gather_kernel: deposit, cache pages -> block pages, zeroing padding rows.
+#include "common.cuh"
+
+namespace kvg {
+
+namespace {
+
+constexpr int kCopyThreads = 512;
+constexpr int kCopyUnroll = 8;
+
+__device__ __forceinline__ void copy_chunk(uint8_t *__restrict__ dst, const uint8_t *__restrict__ src,
+                                           int bytes) {
+    const uint4 *s = reinterpret_cast<const uint4 *>(src);
+    uint4 *d = reinterpret_cast<uint4 *>(dst);
+    const int nvec = bytes >> 4;
+    for (int base = threadIdx.x; base < nvec; base += kCopyThreads * kCopyUnroll) {
+        uint4 r[kCopyUnroll];
+#pragma unroll
+        for (int u = 0; u < kCopyUnroll; ++u) {
+            const int i = base + u * kCopyThreads;
+            if (i < nvec) r[u] = __ldcs(s + i);
+        }
+#pragma unroll
+        for (int u = 0; u < kCopyUnroll; ++u) {
+            const int i = base + u * kCopyThreads;
+            if (i < nvec) __stcs(d + i, r[u]);
+        }
+    }
+}
+
+__device__ __forceinline__ void unpack8(const uint4 &v, float *f) {
+    const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 t = __bfloat1622float2(h[i]);
+        f[2 * i] = t.x;
+        f[2 * i + 1] = t.y;
+    }
+}
+
+__device__ __forceinline__ uint4 pack8(const float *f) {
+    uint4 v;
+    __nv_bfloat162 *h = reinterpret_cast<__nv_bfloat162 *>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+    return v;
+}
+
+// Rotation of the pair (a, b) by the angle whose cosine/sine are (c, s):
+// a' = a c - b s, b' = a s + b c, in fp32 with a fixed operation order.
+__device__ __forceinline__ void rot(float a, float b, float c, float s, float &ra, float &rb) {
+    ra = __fmaf_rn(a, c, __fmul_rn(-b, s));
+    rb = __fmaf_rn(a, s, __fmul_rn(b, c));
+}
+
+// Key chunk re-based by delta: rows of head_dim elements; half-split pairs
+// (i, i + D/2) live in two 16-byte vectors of the same row, interleaved pairs
+// (2i, 2i+1) inside one vector.  Rows whose token index is >= n_tokens are
+// padding and are copied unchanged.
+template <int ROT>
+__device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const uint8_t *__restrict__ src,
+                                             int bytes, int64_t first_row_in_page,
+                                             int64_t page_token0, const GraftParams &p) {
+    const int D = p.head_dim;
+    const int vec_per_row = D >> 3;
+    const int rows = bytes / (2 * D);
+    const uint4 *s4 = reinterpret_cast<const uint4 *>(src);
+    uint4 *d4 = reinterpret_cast<uint4 *>(dst);
+    if (ROT == 1) {
+        const int half_vecs = vec_per_row >> 1;
+        const int n_items = rows * half_vecs;
+        for (int it = threadIdx.x; it < n_items; it += kCopyThreads) {
+            const int rr = it / half_vecs;
+            const int c = it - rr * half_vecs;
+            const int64_t row_in_page = first_row_in_page + rr;
+            const int64_t tok = page_token0 + (row_in_page % p.page_size);
+            const int lo_i = rr * vec_per_row + c;
+            const int hi_i = lo_i + half_vecs;
+            const uint4 lo = __ldcs(s4 + lo_i);
+            const uint4 hi = __ldcs(s4 + hi_i);
+            if (tok < p.n_tokens) {
+                float a[8], b[8], ra[8], rb[8];
+                unpack8(lo, a);
+                unpack8(hi, b);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) rot(a[e], b[e], p.cosv[c * 8 + e], p.sinv[c * 8 + e], ra[e], rb[e]);
+                __stcs(d4 + lo_i, pack8(ra));
+                __stcs(d4 + hi_i, pack8(rb));
+            } else {
+                __stcs(d4 + lo_i, lo);
+                __stcs(d4 + hi_i, hi);
+            }
+        }
+    } else {
+        const int n_items = rows * vec_per_row;
+        for (int it = threadIdx.x; it < n_items; it += kCopyThreads) {
+            const int rr = it / vec_per_row;
+            const int c = it - rr * vec_per_row;
+            const int64_t row_in_page = first_row_in_page + rr;
+            const int64_t tok = page_token0 + (row_in_page % p.page_size);
+            const uint4 x = __ldcs(s4 + it);
+            if (tok < p.n_tokens) {
+                float f[8], g[8];
+                unpack8(x, f);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int i = c * 4 + e;
+                    rot(f[2 * e], f[2 * e + 1], p.cosv[i], p.sinv[i], g[2 * e], g[2 * e + 1]);
+                }
+                __stcs(d4 + it, pack8(g));
+            } else {
+                __stcs(d4 + it, x);
+            }
+        }
+    }
+}
+
+template <int ROT>
+__global__ void __launch_bounds__(kCopyThreads) graft_kernel(const GraftParams p) {
+    const int64_t P = p.page_size;
+    // metadata: position tags, page table and fill counts of this launch's pages
+    {
+        const int64_t tok0 = (int64_t)p.page_base * P;
+        int64_t n_meta = (int64_t)p.npb * P;
+        if (tok0 + n_meta > p.n_tokens) n_meta = p.n_tokens - tok0;
+        const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+        const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+        for (int64_t t = gtid; t < n_meta; t += gsz)
+            p.dst_pos[t] = (int32_t)((int64_t)p.src_pos[t] + p.delta);
+        for (int64_t j = gtid; j < p.npb; j += gsz) {
+            p.table_row[j] = p.pids.pid[j];
+            int64_t f = p.n_tokens - (tok0 + j * P);
+            p.fill_row[j] = (int32_t)(f < P ? f : P);
+        }
+    }
+    const uint64_t page_bytes = p.page_bytes;
+    const int cpp = (int)(page_bytes / (uint64_t)p.chunk_bytes);
+    const int64_t n_units = (int64_t)p.n_layers * 2 * p.npb * cpp;
+    const int row_bytes = 2 * p.head_dim;
+    for (int64_t unit = blockIdx.x; unit < n_units; unit += gridDim.x) {
+        const int64_t page_u = unit / cpp;
+        const int chunk = (int)(unit - page_u * cpp);
+        const int64_t lkv = page_u / p.npb;
+        const int jj = (int)(page_u - lkv * p.npb);
+        const uint64_t off = (uint64_t)chunk * (uint64_t)p.chunk_bytes;
+        const uint8_t *src = p.src + ((uint64_t)lkv * p.block_pages + p.page_base + jj) * page_bytes + off;
+        uint8_t *dst = p.pool + ((uint64_t)lkv * p.pool_pages + p.pids.pid[jj]) * page_bytes + off;
+        if (ROT == 0 || (lkv & 1)) {
+            copy_chunk(dst, src, p.chunk_bytes);
+        } else {
+            rotate_chunk<ROT>(dst, src, p.chunk_bytes, (int64_t)(off / row_bytes),
+                              (int64_t)(p.page_base + jj) * P, p);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
+    const int D = p.head_dim;
+    const int vpr = D >> 3;  // 16-byte vectors per row
+    const int64_t per_kv = (int64_t)p.n_layers * p.n * p.n_kv_heads * vpr;
+    const int64_t total = 2 * per_kv;
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+    const int64_t P = p.page_size;
+    for (int64_t t = gtid; t < p.n; t += gsz) p.pos_row[p.slot0 + t] = p.pos[p.row0 + t];
+    for (int64_t i = gtid; i < p.pids.n; i += gsz) {
+        const int64_t pg = p.page0 + i;
+        p.table_row[pg] = p.pids.pid[i];
+        const int64_t f = (int64_t)p.slot0 + p.n - pg * P;
+        p.fill_row[pg] = (int32_t)(f < P ? f : P);
+    }
+    for (int64_t idx = gtid; idx < total; idx += gsz) {
+        const int kv = idx >= per_kv;
+        int64_t r = idx - kv * per_kv;
+        const int c = (int)(r % vpr);
+        r /= vpr;
+        const int h = (int)(r % p.n_kv_heads);
+        r /= p.n_kv_heads;
+        const int t = (int)(r % p.n);
+        const int l = (int)(r / p.n);
+        const uint16_t *srcbase = kv ? p.v : p.k;
+        const uint4 val = __ldcs(reinterpret_cast<const uint4 *>(
+            srcbase + (((int64_t)l * p.n_rows_total + p.row0 + t) * p.n_kv_heads + h) * D) + c);
+        const int64_t s = (int64_t)p.slot0 + t;
+        const int64_t pg = s / P;
+        const int pid = p.pids.pid[pg - p.page0];
+        const int64_t row = s - pg * P;
+        uint16_t *dst = reinterpret_cast<uint16_t *>(p.pool) +
+                        ((((int64_t)l * 2 + kv) * p.pool_pages + pid) * p.n_kv_heads + h) * P * D + row * D;
+        __stcs(reinterpret_cast<uint4 *>(dst) + c, val);
+    }
+}
+
+__global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
+    const int64_t P = p.page_size;
+    const int64_t D = p.head_dim;
+    const int64_t vpp = (int64_t)(p.page_bytes >> 4);
+    const int64_t total = (int64_t)p.n_layers * 2 * p.npb * vpp;
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+    const int64_t tok0 = (int64_t)p.page_base * P;
+    int64_t n_meta = (int64_t)p.npb * P;
+    if (tok0 + n_meta > p.n_tokens) n_meta = p.n_tokens - tok0;
+    for (int64_t t = gtid; t < n_meta; t += gsz) p.dst_pos[t] = p.src_pos[t];
+    for (int64_t idx = gtid; idx < total; idx += gsz) {
+        const int64_t page_u = idx / vpp;
+        const int64_t off = idx - page_u * vpp;
+        const int64_t lkv = page_u / p.npb;
+        const int64_t jj = page_u - lkv * p.npb;
+        const int64_t row = ((off * 16) / (2 * D)) % P;
+        const int64_t tok = (p.page_base + jj) * P + row;
+        uint4 val = make_uint4(0, 0, 0, 0);
+        if (tok < p.n_tokens) {
+            const uint4 *src = reinterpret_cast<const uint4 *>(
+                p.pool + ((uint64_t)lkv * p.pool_pages + p.pids.pid[jj]) * p.page_bytes);
+            val = __ldcs(src + off);
+        }
+        uint4 *dst = reinterpret_cast<uint4 *>(
+            p.dst + ((uint64_t)lkv * p.block_pages + p.page_base + jj) * p.page_bytes);
+        dst[off] = val;
+    }
+}
+
+__global__ void write_header_kernel(const HeaderParams p) {
+    const int i = threadIdx.x;
+    if (i < 64) reinterpret_cast<uint32_t *>(p.dst)[i] = reinterpret_cast<const uint32_t *>(p.bytes)[i];
+}
+
+__global__ void reset_seq_kernel(int32_t *table_row, int32_t *fill_row, int32_t max_pages,
+                                 int32_t *pos_row, int32_t max_slots) {
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t j = gtid; j < max_pages; j += gsz) {
+        table_row[j] = -1;
+        fill_row[j] = 0;
+    }
+    for (int64_t s = gtid; s < max_slots; s += gsz) pos_row[s] = -1;
+}
+
+int grid_for(int64_t work_items, int per_block, int n_sm, int waves) {
+    int64_t g = (work_items + per_block - 1) / per_block;
+    const int64_t cap = (int64_t)n_sm * waves;
+    if (g > cap) g = cap;
+    if (g < 1) g = 1;
+    return (int)g;
+}
+
+}  // namespace
+
+cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s) {
+    const int64_t units = (int64_t)p.n_layers * 2 * p.npb * (int64_t)(p.page_bytes / p.chunk_bytes);
+    const int grid = grid_for(units, 1, n_sm, 4);
+    if (p.rotate == 0)
+        graft_kernel<0><<<grid, kCopyThreads, 0, s>>>(p);
+    else if (p.rotate == 1)
+        graft_kernel<1><<<grid, kCopyThreads, 0, s>>>(p);
+    else
+        graft_kernel<2><<<grid, kCopyThreads, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append(const AppendParams &p, int n_sm, cudaStream_t s) {
+    const int64_t items = 2ll * p.n_layers * p.n * p.n_kv_heads * (p.head_dim / 8);
+    append_kernel<<<grid_for(items, 256, n_sm, 8), 256, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s) {
+    const int64_t items = 2ll * p.n_layers * p.npb * (int64_t)(p.page_bytes / 16);
+    gather_kernel<<<grid_for(items, 256, n_sm, 8), 256, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_write_header(const HeaderParams &p, cudaStream_t s) {
+    write_header_kernel<<<1, 64, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_reset_seq(int32_t *table_row, int32_t *fill_row, int32_t max_pages,
+                             int32_t *pos_row, int32_t max_slots, cudaStream_t s) {
+    const int64_t items = max_pages > max_slots ? max_pages : max_slots;
+    reset_seq_kernel<<<grid_for(items, 256, 152, 1), 256, 0, s>>>(table_row, fill_row, max_pages,
+                                                                   pos_row, max_slots);
+    return cudaGetLastError();
+}
+
+}  // namespace kvg

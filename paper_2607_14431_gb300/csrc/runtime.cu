@@ -1,0 +1,927 @@
+// runtime.cu — host side of libkvg: the C ABI declared in include/kvg.h.
+//
+// Owns stores (serialized blocks in HBM or pinned-host slabs), caches (page
+// pool, device page tables, host mirror of the free list and of each
+// sequence's pages), per-object scratch (leaf digests, split-K partials) and
+// device status words.  Every call validates its arguments on the host before
+// it enqueues anything, then plans launches for the kernels in
+// copy_kernels.cu, sha256_kernels.cu and attn_kernels.cu.
+#include <algorithm>
+#include <cstdarg>
+#include <chrono>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <deque>
+#include <mutex>
+#include <string>
+#include <thread>
+#include <vector>
+
+#include "common.cuh"
+
+using namespace kvg;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+kvg_status fail(kvg_status st, const char *fmt, ...) __attribute__((format(printf, 2, 3)));
+kvg_status fail(kvg_status st, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return st;
+}
+
+kvg_status cuda_fail(cudaError_t e, const char *where) {
+    return fail(KVG_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+#define KVG_CUDA(call)                                      \
+    do {                                                    \
+        cudaError_t e_ = (call);                            \
+        if (e_ != cudaSuccess) return cuda_fail(e_, #call); \
+    } while (0)
+
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard() {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+uint64_t round_up(uint64_t x, uint64_t m) { return (x + m - 1) / m * m; }
+
+int sm_count(int dev) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 1;
+    return n;
+}
+
+bool dims_valid(const kvg_dims &d) {
+    if (d.n_layers <= 0 || d.n_kv_heads <= 0 || d.page_size <= 0) return false;
+    if (d.head_dim != 64 && d.head_dim != 128 && d.head_dim != 256) return false;
+    if (d.rope_style != KVG_ROPE_HALF && d.rope_style != KVG_ROPE_INTERLEAVED) return false;
+    const uint64_t pb = 2ull * d.n_kv_heads * d.page_size * d.head_dim;
+    return pb % 16 == 0 && pb <= (1ull << 31);
+}
+
+bool same_geometry(const kvg_dims &a, const kvg_dims &b) {
+    return a.n_layers == b.n_layers && a.n_kv_heads == b.n_kv_heads && a.head_dim == b.head_dim &&
+           a.page_size == b.page_size;
+}
+
+uint64_t page_bytes_of(const kvg_dims &d) { return 2ull * d.n_kv_heads * d.page_size * d.head_dim; }
+
+struct BlockLayout {
+    int64_t n_tokens, n_pages;
+    uint64_t pos_off, dig_off, pages_off, total;
+};
+
+BlockLayout layout_for(const kvg_dims &d, int64_t n_tokens) {
+    BlockLayout b;
+    b.n_tokens = n_tokens;
+    b.n_pages = (n_tokens + d.page_size - 1) / d.page_size;
+    b.pos_off = 256;
+    b.dig_off = round_up(b.pos_off + 4ull * n_tokens, 256);
+    b.pages_off = round_up(b.dig_off + (uint64_t)d.n_layers * 2 * b.n_pages * 32, 4096);
+    b.total = b.pages_off + (uint64_t)d.n_layers * 2 * b.n_pages * page_bytes_of(d);
+    return b;
+}
+
+void build_header(uint8_t h[256], const kvg_dims &d, const BlockLayout &b) {
+    memset(h, 0, 256);
+    memcpy(h, "KVGBLK01", 8);
+    uint32_t u32;
+    int32_t i32;
+    int64_t i64;
+    uint64_t u64;
+    double f64;
+    u32 = 1; memcpy(h + 8, &u32, 4);
+    u32 = 256; memcpy(h + 12, &u32, 4);
+    i32 = d.n_layers; memcpy(h + 16, &i32, 4);
+    i32 = d.n_kv_heads; memcpy(h + 20, &i32, 4);
+    i32 = d.head_dim; memcpy(h + 24, &i32, 4);
+    i32 = d.page_size; memcpy(h + 28, &i32, 4);
+    i64 = b.n_tokens; memcpy(h + 32, &i64, 8);
+    i64 = b.n_pages; memcpy(h + 40, &i64, 8);
+    f64 = d.rope_theta; memcpy(h + 48, &f64, 8);
+    i32 = d.rope_style; memcpy(h + 56, &i32, 4);
+    i32 = 1; memcpy(h + 60, &i32, 4);
+    u64 = b.pos_off; memcpy(h + 64, &u64, 8);
+    u64 = b.dig_off; memcpy(h + 72, &u64, 8);
+    u64 = b.pages_off; memcpy(h + 80, &u64, 8);
+    u64 = b.total; memcpy(h + 88, &u64, 8);
+}
+
+// Chunk of a page that one CTA copies: <= 64 KiB, divides the page, whole rows.
+int32_t copy_chunk_bytes(const kvg_dims &d) {
+    uint64_t c = page_bytes_of(d);
+    const uint64_t row = 2ull * d.head_dim;
+    while (c > 65536 && c % 2 == 0 && (c / 2) % row == 0 && (c / 2) % 16 == 0) c /= 2;
+    return (int32_t)c;
+}
+
+// Growable device scratch.  Growing frees the old buffer (cudaFree waits for
+// the device), so work still using it has finished.
+struct Scratch {
+    void *ptr = nullptr;
+    size_t cap = 0;
+    cudaError_t ensure(size_t bytes) {
+        if (bytes <= cap) return cudaSuccess;
+        if (ptr) cudaFree(ptr);
+        ptr = nullptr;
+        cap = 0;
+        size_t want = std::max(bytes, (size_t)1 << 20);
+        cudaError_t e = cudaMalloc(&ptr, want);
+        if (e != cudaSuccess) return e;
+        cap = want;
+        return cudaSuccess;
+    }
+    void release() {
+        if (ptr) cudaFree(ptr);
+        ptr = nullptr;
+        cap = 0;
+    }
+};
+
+}  // namespace
+
+// ------------------------------------------------------------------- store --
+
+struct kvg_store {
+    kvg_dims dims;
+    int32_t residency = KVG_RESIDENCY_HBM;
+    uint64_t capacity = 0;
+    uint64_t reserved_bytes = 0;  // slab bytes allocated so far
+    int device = 0;
+    int n_sm = 1;
+    struct Slab {
+        uint8_t *host = nullptr;  // pinned-host slabs
+        uint8_t *dev = nullptr;   // device-accessible address
+        uint64_t size = 0, used = 0;
+    };
+    std::vector<Slab> slabs;
+    struct Blk {
+        uint8_t *dev;   // device-accessible start of the serialized block
+        uint8_t *host;  // host address (pinned-host store) or nullptr
+        BlockLayout lay;
+        int64_t min_pos, max_pos;
+    };
+    std::vector<Blk> blocks;
+    Scratch leaf;
+    DevStatus *status = nullptr;
+};
+
+static kvg_status store_alloc(kvg_store *s, uint64_t bytes, uint8_t **dev, uint8_t **host) {
+    for (auto &sl : s->slabs) {
+        const uint64_t at = round_up(sl.used, 4096);
+        if (at + bytes <= sl.size) {
+            *dev = sl.dev + at;
+            *host = sl.host ? sl.host + at : nullptr;
+            sl.used = at + bytes;
+            return KVG_OK;
+        }
+    }
+    const uint64_t slab = std::max<uint64_t>(bytes, 1ull << 30);
+    if (s->reserved_bytes + slab > s->capacity) {
+        if (s->reserved_bytes + bytes > s->capacity)
+            return fail(KVG_ERR_CAPACITY, "store full: %llu of %llu bytes reserved, block needs %llu",
+                        (unsigned long long)s->reserved_bytes, (unsigned long long)s->capacity,
+                        (unsigned long long)bytes);
+    }
+    const uint64_t size = std::min<uint64_t>(slab, s->capacity - s->reserved_bytes);
+    kvg_store::Slab sl;
+    sl.size = size;
+    if (s->residency == KVG_RESIDENCY_HBM) {
+        cudaError_t e = cudaMalloc(&sl.dev, size);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(KVG_ERR_OOM, "cudaMalloc(%llu): %s", (unsigned long long)size, cudaGetErrorString(e));
+        }
+    } else {
+        cudaError_t e = cudaHostAlloc(reinterpret_cast<void **>(&sl.host), size,
+                                      cudaHostAllocMapped | cudaHostAllocPortable);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(KVG_ERR_OOM, "cudaHostAlloc(%llu): %s", (unsigned long long)size, cudaGetErrorString(e));
+        }
+        e = cudaHostGetDevicePointer(reinterpret_cast<void **>(&sl.dev), sl.host, 0);
+        if (e != cudaSuccess) {
+            cudaFreeHost(sl.host);
+            return cuda_fail(e, "cudaHostGetDevicePointer");
+        }
+    }
+    s->reserved_bytes += size;
+    sl.used = bytes;
+    *dev = sl.dev;
+    *host = sl.host;
+    s->slabs.push_back(sl);
+    return KVG_OK;
+}
+
+extern "C" kvg_status kvg_store_create(const kvg_dims *dims, int32_t residency, uint64_t capacity_bytes,
+                                       int32_t device, kvg_store **out) {
+    if (!dims || !out) return fail(KVG_ERR_ARG, "null argument");
+    *out = nullptr;
+    if (!dims_valid(*dims)) return fail(KVG_ERR_ARG, "unsupported geometry");
+    if (residency != KVG_RESIDENCY_HBM && residency != KVG_RESIDENCY_PINNED_HOST)
+        return fail(KVG_ERR_ARG, "bad residency %d", residency);
+    int ndev = 0;
+    KVG_CUDA(cudaGetDeviceCount(&ndev));
+    if (device < 0 || device >= ndev) return fail(KVG_ERR_ARG, "bad device %d", device);
+    DeviceGuard g(device);
+    if (!g.ok) return fail(KVG_ERR_CUDA, "cudaSetDevice(%d) failed", device);
+    kvg_store *s = new kvg_store();
+    s->dims = *dims;
+    s->residency = residency;
+    s->capacity = capacity_bytes;
+    s->device = device;
+    s->n_sm = sm_count(device);
+    cudaError_t e = cudaMalloc(&s->status, sizeof(DevStatus));
+    if (e != cudaSuccess) {
+        delete s;
+        return cuda_fail(e, "cudaMalloc(status)");
+    }
+    cudaMemset(s->status, 0, sizeof(DevStatus));
+    *out = s;
+    return KVG_OK;
+}
+
+extern "C" void kvg_store_destroy(kvg_store *s) {
+    if (!s) return;
+    DeviceGuard g(s->device);
+    cudaDeviceSynchronize();
+    for (auto &sl : s->slabs) {
+        if (sl.host)
+            cudaFreeHost(sl.host);
+        else if (sl.dev)
+            cudaFree(sl.dev);
+    }
+    s->leaf.release();
+    if (s->status) cudaFree(s->status);
+    delete s;
+}
+
+extern "C" kvg_status kvg_store_block_info(kvg_store *s, uint64_t id, kvg_block_info *out) {
+    if (!s || !out) return fail(KVG_ERR_ARG, "null argument");
+    if (id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)id);
+    DeviceGuard g(s->device);
+    const auto &b = s->blocks[id];
+    memset(out, 0, sizeof *out);
+    out->n_tokens = b.lay.n_tokens;
+    out->n_pages = b.lay.n_pages;
+    out->residency = s->residency;
+    out->bytes = b.host ? (const void *)b.host : (const void *)b.dev;
+    out->total_bytes = b.lay.total;
+    out->positions_offset = b.lay.pos_off;
+    out->digests_offset = b.lay.dig_off;
+    out->pages_offset = b.lay.pages_off;
+    KVG_CUDA(cudaDeviceSynchronize());
+    if (b.host)
+        memcpy(out->block_digest, b.host + 96, 32);
+    else
+        KVG_CUDA(cudaMemcpy(out->block_digest, b.dev + 96, 32, cudaMemcpyDeviceToHost));
+    return KVG_OK;
+}
+
+// Hashes every page of a block (contiguous pages region) and its block digest
+// against `expected` digests (nullable: then writes them), on stream st.
+static kvg_status hash_block(kvg_store *s, uint8_t *blk_dev, const BlockLayout &lay, bool verify,
+                             cudaStream_t st) {
+    const kvg_dims &d = s->dims;
+    const uint64_t pb = page_bytes_of(d);
+    const int64_t m = (int64_t)((pb + kLeafBytes - 1) / kLeafBytes);
+    const int64_t n_pages = (int64_t)d.n_layers * 2 * lay.n_pages;
+    KVG_CUDA(s->leaf.ensure((size_t)n_pages * m * 32));
+    PageSource src{blk_dev + lay.pages_off, pb, nullptr, 1, 0};
+    uint32_t *leaf = static_cast<uint32_t *>(s->leaf.ptr);
+    KVG_CUDA(launch_sha256_leaves(src, n_pages, leaf, s->n_sm, st));
+    uint8_t *dig = blk_dev + lay.dig_off;
+    KVG_CUDA(launch_sha256_pages(leaf, n_pages, m, verify ? nullptr : dig, verify ? dig : nullptr,
+                                 s->status, -1, st));
+    KVG_CUDA(launch_sha256_serial(blk_dev + lay.pos_off, 4ull * lay.n_tokens, dig,
+                                  (uint64_t)n_pages * 32, verify ? nullptr : blk_dev + 96,
+                                  verify ? blk_dev + 96 : nullptr, s->status, st));
+    return KVG_OK;
+}
+
+static void minmax_positions(const int32_t *pos, int64_t n, int64_t *mn, int64_t *mx) {
+    int64_t a = INT64_MAX, b = INT64_MIN;
+    for (int64_t i = 0; i < n; ++i) {
+        a = std::min<int64_t>(a, pos[i]);
+        b = std::max<int64_t>(b, pos[i]);
+    }
+    *mn = n ? a : 0;
+    *mx = n ? b : 0;
+}
+
+extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t n_bytes, uint32_t flags,
+                                       uint64_t *block_id_out) {
+    if (!s || !bytes || !block_id_out) return fail(KVG_ERR_ARG, "null argument");
+    const uint8_t *h = static_cast<const uint8_t *>(bytes);
+    if (n_bytes < 256 || memcmp(h, "KVGBLK01", 8) != 0) return fail(KVG_ERR_FORMAT, "bad magic");
+    uint32_t ver, hb;
+    int32_t L, Hkv, D, P, style, dtype;
+    int64_t n_tok, n_pg;
+    uint64_t po, dof, pgo, tot;
+    memcpy(&ver, h + 8, 4);
+    memcpy(&hb, h + 12, 4);
+    memcpy(&L, h + 16, 4);
+    memcpy(&Hkv, h + 20, 4);
+    memcpy(&D, h + 24, 4);
+    memcpy(&P, h + 28, 4);
+    memcpy(&n_tok, h + 32, 8);
+    memcpy(&n_pg, h + 40, 8);
+    memcpy(&style, h + 56, 4);
+    memcpy(&dtype, h + 60, 4);
+    memcpy(&po, h + 64, 8);
+    memcpy(&dof, h + 72, 8);
+    memcpy(&pgo, h + 80, 8);
+    memcpy(&tot, h + 88, 8);
+    const kvg_dims &d = s->dims;
+    if (ver != 1 || hb != 256 || dtype != 1) return fail(KVG_ERR_FORMAT, "unsupported version/dtype");
+    if (L != d.n_layers || Hkv != d.n_kv_heads || D != d.head_dim || P != d.page_size)
+        return fail(KVG_ERR_FORMAT, "geometry differs from the store's");
+    if (n_tok <= 0 || n_tok > (1ll << 31)) return fail(KVG_ERR_FORMAT, "bad n_tokens");
+    const BlockLayout lay = layout_for(d, n_tok);
+    if (n_pg != lay.n_pages || po != lay.pos_off || dof != lay.dig_off || pgo != lay.pages_off ||
+        tot != lay.total || n_bytes < tot)
+        return fail(KVG_ERR_FORMAT, "layout fields inconsistent");
+    DeviceGuard g(s->device);
+    uint8_t *dev = nullptr, *host = nullptr;
+    kvg_status st = store_alloc(s, lay.total, &dev, &host);
+    if (st != KVG_OK) return st;
+    if (host)
+        memcpy(host, h, lay.total);
+    else
+        KVG_CUDA(cudaMemcpy(dev, h, lay.total, cudaMemcpyHostToDevice));
+    if (flags & KVG_GRAFT_VERIFY) {
+        KVG_CUDA(cudaMemset(s->status, 0, sizeof(DevStatus)));
+        st = hash_block(s, dev, lay, true, 0);
+        if (st != KVG_OK) return st;
+        KVG_CUDA(cudaDeviceSynchronize());
+        DevStatus hs;
+        KVG_CUDA(cudaMemcpy(&hs, s->status, sizeof hs, cudaMemcpyDeviceToHost));
+        KVG_CUDA(cudaMemset(s->status, 0, sizeof(DevStatus)));
+        if (hs.n_mismatch)
+            return fail(KVG_ERR_DIGEST, "import: %d digest mismatches (block not added)", hs.n_mismatch);
+    }
+    kvg_store::Blk b{dev, host, lay, 0, 0};
+    minmax_positions(reinterpret_cast<const int32_t *>(h + lay.pos_off), n_tok, &b.min_pos, &b.max_pos);
+    s->blocks.push_back(b);
+    *block_id_out = s->blocks.size() - 1;
+    return KVG_OK;
+}
+
+extern "C" kvg_status kvg_store_export(kvg_store *s, uint64_t id, void *dst, uint64_t dst_bytes) {
+    if (!s || !dst) return fail(KVG_ERR_ARG, "null argument");
+    if (id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)id);
+    const auto &b = s->blocks[id];
+    if (dst_bytes < b.lay.total) return fail(KVG_ERR_CAPACITY, "destination too small");
+    DeviceGuard g(s->device);
+    KVG_CUDA(cudaDeviceSynchronize());
+    if (b.host)
+        memcpy(dst, b.host, b.lay.total);
+    else
+        KVG_CUDA(cudaMemcpy(dst, b.dev, b.lay.total, cudaMemcpyDeviceToHost));
+    return KVG_OK;
+}
+
+// ------------------------------------------------------------------- cache --
+
+struct kvg_cache {
+    kvg_dims dims;
+    int32_t n_pages = 0, max_seqs = 0, max_slots = 0, max_pages = 0;
+    int device = 0, n_sm = 1;
+    uint64_t page_bytes = 0;
+    uint8_t *pool = nullptr;
+    int32_t *page_table = nullptr, *page_fill = nullptr, *positions = nullptr;
+    DevStatus *status = nullptr;
+    std::deque<int32_t> free_list;
+    std::vector<std::vector<int32_t>> seq_pages;
+    std::vector<int32_t> n_slots;
+    Scratch leaf, part_o, part_ml;
+};
+
+extern "C" kvg_status kvg_cache_create(const kvg_dims *dims, int32_t n_pages, int32_t max_seqs,
+                                       int32_t max_slots, int32_t device, kvg_cache **out) {
+    if (!dims || !out) return fail(KVG_ERR_ARG, "null argument");
+    *out = nullptr;
+    if (!dims_valid(*dims)) return fail(KVG_ERR_ARG, "unsupported geometry");
+    if (n_pages <= 0 || max_seqs <= 0 || max_slots <= 0) return fail(KVG_ERR_ARG, "bad sizes");
+    int ndev = 0;
+    KVG_CUDA(cudaGetDeviceCount(&ndev));
+    if (device < 0 || device >= ndev) return fail(KVG_ERR_ARG, "bad device %d", device);
+    DeviceGuard g(device);
+    if (!g.ok) return fail(KVG_ERR_CUDA, "cudaSetDevice(%d) failed", device);
+    kvg_cache *c = new kvg_cache();
+    c->dims = *dims;
+    c->n_pages = n_pages;
+    c->max_seqs = max_seqs;
+    c->max_slots = max_slots;
+    c->max_pages = (max_slots + dims->page_size - 1) / dims->page_size;
+    c->device = device;
+    c->n_sm = sm_count(device);
+    c->page_bytes = page_bytes_of(*dims);
+    const uint64_t pool_bytes = (uint64_t)dims->n_layers * 2 * n_pages * c->page_bytes;
+    auto cleanup = [&](kvg_status st) {
+        kvg_cache_destroy(c);
+        return st;
+    };
+    cudaError_t e = cudaMalloc(&c->pool, pool_bytes);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        c->pool = nullptr;
+        return cleanup(fail(KVG_ERR_OOM, "pool cudaMalloc(%llu): %s", (unsigned long long)pool_bytes,
+                            cudaGetErrorString(e)));
+    }
+    const size_t tbl = (size_t)max_seqs * c->max_pages * 4;
+    const size_t pos = (size_t)max_seqs * max_slots * 4;
+    if (cudaMalloc(&c->page_table, tbl) != cudaSuccess || cudaMalloc(&c->page_fill, tbl) != cudaSuccess ||
+        cudaMalloc(&c->positions, pos) != cudaSuccess || cudaMalloc(&c->status, sizeof(DevStatus)) != cudaSuccess) {
+        cudaGetLastError();
+        return cleanup(fail(KVG_ERR_OOM, "cache tables allocation failed"));
+    }
+    if (cudaMemset(c->page_table, 0xFF, tbl) != cudaSuccess || cudaMemset(c->page_fill, 0, tbl) != cudaSuccess ||
+        cudaMemset(c->positions, 0xFF, pos) != cudaSuccess ||
+        cudaMemset(c->status, 0, sizeof(DevStatus)) != cudaSuccess)
+        return cleanup(fail(KVG_ERR_CUDA, "cache tables init failed"));
+    for (int32_t i = 0; i < n_pages; ++i) c->free_list.push_back(i);
+    c->seq_pages.assign(max_seqs, {});
+    c->n_slots.assign(max_seqs, 0);
+    if (cudaDeviceSynchronize() != cudaSuccess) return cleanup(fail(KVG_ERR_CUDA, "init sync failed"));
+    *out = c;
+    return KVG_OK;
+}
+
+extern "C" void kvg_cache_destroy(kvg_cache *c) {
+    if (!c) return;
+    DeviceGuard g(c->device);
+    cudaDeviceSynchronize();
+    if (c->pool) cudaFree(c->pool);
+    if (c->page_table) cudaFree(c->page_table);
+    if (c->page_fill) cudaFree(c->page_fill);
+    if (c->positions) cudaFree(c->positions);
+    if (c->status) cudaFree(c->status);
+    c->leaf.release();
+    c->part_o.release();
+    c->part_ml.release();
+    delete c;
+}
+
+extern "C" kvg_status kvg_cache_set_free_order(kvg_cache *c, const int32_t *order, int32_t n) {
+    if (!c || !order) return fail(KVG_ERR_ARG, "null argument");
+    if (n != c->n_pages || (int32_t)c->free_list.size() != c->n_pages)
+        return fail(KVG_ERR_ARG, "free order needs every page free and n == n_pages");
+    std::vector<char> seen(n, 0);
+    for (int32_t i = 0; i < n; ++i) {
+        if (order[i] < 0 || order[i] >= n || seen[order[i]]) return fail(KVG_ERR_ARG, "not a permutation");
+        seen[order[i]] = 1;
+    }
+    c->free_list.assign(order, order + n);
+    return KVG_OK;
+}
+
+extern "C" kvg_status kvg_cache_view_get(const kvg_cache *c, kvg_cache_view *v) {
+    if (!c || !v) return fail(KVG_ERR_ARG, "null argument");
+    v->pool = c->pool;
+    v->page_table = c->page_table;
+    v->page_fill = c->page_fill;
+    v->positions = c->positions;
+    v->pool_bytes = (uint64_t)c->dims.n_layers * 2 * c->n_pages * c->page_bytes;
+    v->page_bytes = c->page_bytes;
+    v->n_pages = c->n_pages;
+    v->max_seqs = c->max_seqs;
+    v->max_slots = c->max_slots;
+    v->max_pages = c->max_pages;
+    return KVG_OK;
+}
+
+extern "C" kvg_status kvg_cache_seq_info(const kvg_cache *c, int32_t seq, int32_t *n_slots, int32_t *n_pages) {
+    if (!c) return fail(KVG_ERR_ARG, "null argument");
+    if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d", seq);
+    if (n_slots) *n_slots = c->n_slots[seq];
+    if (n_pages) *n_pages = (int32_t)c->seq_pages[seq].size();
+    return KVG_OK;
+}
+
+static std::vector<int32_t> take_pages(kvg_cache *c, int64_t n) {
+    std::vector<int32_t> v;
+    v.reserve(n);
+    for (int64_t i = 0; i < n; ++i) {
+        v.push_back(c->free_list.front());
+        c->free_list.pop_front();
+    }
+    return v;
+}
+
+extern "C" kvg_status kvg_cache_append(kvg_cache *c, int32_t seq, const void *k, const void *v,
+                                       const int32_t *positions, int32_t n, void *stream) {
+    if (!c) return fail(KVG_ERR_ARG, "null cache");
+    if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d", seq);
+    if (n < 0) return fail(KVG_ERR_ARG, "negative n");
+    if (n == 0) return KVG_OK;
+    if (!k || !v || !positions) return fail(KVG_ERR_ARG, "null buffer");
+    if ((reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(v)) & 15)
+        return fail(KVG_ERR_ARG, "k/v must be 16-byte aligned");
+    const int64_t P = c->dims.page_size;
+    const int64_t s0 = c->n_slots[seq];
+    if (s0 + n > c->max_slots) return fail(KVG_ERR_CAPACITY, "append past max_slots");
+    const int64_t have = (int64_t)c->seq_pages[seq].size();
+    const int64_t need = (s0 + n + P - 1) / P - have;
+    if (need > (int64_t)c->free_list.size()) return fail(KVG_ERR_CAPACITY, "out of free pages");
+    DeviceGuard g(c->device);
+    auto got = take_pages(c, std::max<int64_t>(need, 0));
+    auto &sp = c->seq_pages[seq];
+    sp.insert(sp.end(), got.begin(), got.end());
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int64_t rows_per_launch = (int64_t)(kMaxPagesPerLaunch - 1) * P;
+    for (int64_t row0 = 0; row0 < n; row0 += rows_per_launch) {
+        const int64_t nr = std::min<int64_t>(rows_per_launch, n - row0);
+        const int64_t s = s0 + row0;
+        AppendParams p{};
+        p.k = static_cast<const uint16_t *>(k);
+        p.v = static_cast<const uint16_t *>(v);
+        p.pos = positions;
+        p.pool = c->pool;
+        p.pool_pages = c->n_pages;
+        p.n_layers = c->dims.n_layers;
+        p.n_kv_heads = c->dims.n_kv_heads;
+        p.page_size = (int32_t)P;
+        p.head_dim = c->dims.head_dim;
+        p.n = (int32_t)nr;
+        p.row0 = (int32_t)row0;
+        p.slot0 = (int32_t)s;
+        p.page0 = (int32_t)(s / P);
+        p.n_rows_total = n;
+        p.pos_row = c->positions + (int64_t)seq * c->max_slots;
+        p.table_row = c->page_table + (int64_t)seq * c->max_pages;
+        p.fill_row = c->page_fill + (int64_t)seq * c->max_pages;
+        const int64_t last = (s + nr - 1) / P;
+        p.pids.n = (int32_t)(last - p.page0 + 1);
+        for (int32_t i = 0; i < p.pids.n; ++i) p.pids.pid[i] = sp[p.page0 + i];
+        KVG_CUDA(launch_append(p, c->n_sm, st));
+    }
+    c->n_slots[seq] = (int32_t)(s0 + n);
+    return KVG_OK;
+}
+
+extern "C" kvg_status kvg_cache_release(kvg_cache *c, int32_t seq, void *stream) {
+    if (!c) return fail(KVG_ERR_ARG, "null cache");
+    if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d", seq);
+    DeviceGuard g(c->device);
+    for (int32_t pid : c->seq_pages[seq]) c->free_list.push_back(pid);
+    c->seq_pages[seq].clear();
+    c->n_slots[seq] = 0;
+    KVG_CUDA(launch_reset_seq(c->page_table + (int64_t)seq * c->max_pages,
+                              c->page_fill + (int64_t)seq * c->max_pages, c->max_pages,
+                              c->positions + (int64_t)seq * c->max_slots, c->max_slots,
+                              static_cast<cudaStream_t>(stream)));
+    return KVG_OK;
+}
+
+// ----------------------------------------------------------------- deposit --
+
+extern "C" kvg_status kvg_deposit(kvg_store *s, const kvg_cache *cc, int32_t seq, int32_t slot0, int32_t n,
+                                  void *stream, uint64_t *block_id_out) {
+    kvg_cache *c = const_cast<kvg_cache *>(cc);
+    if (!s || !c || !block_id_out) return fail(KVG_ERR_ARG, "null argument");
+    if (!same_geometry(s->dims, c->dims)) return fail(KVG_ERR_ARG, "store and cache geometry differ");
+    if (s->device != c->device) return fail(KVG_ERR_ARG, "store and cache on different devices");
+    if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d", seq);
+    const int64_t P = c->dims.page_size;
+    if (n <= 0 || slot0 < 0 || slot0 % P || (int64_t)slot0 + n > c->n_slots[seq])
+        return fail(KVG_ERR_ARG, "bad range [%d, %d) of %d slots", slot0, slot0 + n, c->n_slots[seq]);
+    DeviceGuard g(s->device);
+    const BlockLayout lay = layout_for(s->dims, n);
+    uint8_t *dev = nullptr, *host = nullptr;
+    kvg_status stt = store_alloc(s, lay.total, &dev, &host);
+    if (stt != KVG_OK) return stt;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    HeaderParams hp;
+    hp.dst = dev;
+    build_header(hp.bytes, s->dims, lay);
+    KVG_CUDA(launch_write_header(hp, st));
+    const auto &sp = c->seq_pages[seq];
+    const int64_t j_first = slot0 / P;
+    for (int64_t base = 0; base < lay.n_pages; base += kMaxPagesPerLaunch) {
+        GatherParams p{};
+        p.pool = c->pool;
+        p.dst = dev + lay.pages_off;
+        p.page_bytes = c->page_bytes;
+        p.pool_pages = c->n_pages;
+        p.n_layers = c->dims.n_layers;
+        p.npb = (int32_t)std::min<int64_t>(kMaxPagesPerLaunch, lay.n_pages - base);
+        p.page_base = (int32_t)base;
+        p.block_pages = (int32_t)lay.n_pages;
+        p.n_kv_heads = c->dims.n_kv_heads;
+        p.page_size = (int32_t)P;
+        p.head_dim = c->dims.head_dim;
+        p.n_tokens = n;
+        p.src_pos = c->positions + (int64_t)seq * c->max_slots + slot0 + base * P;
+        p.dst_pos = reinterpret_cast<int32_t *>(dev + lay.pos_off) + base * P;
+        p.pids.n = p.npb;
+        for (int32_t i = 0; i < p.npb; ++i) p.pids.pid[i] = sp[j_first + base + i];
+        KVG_CUDA(launch_gather(p, s->n_sm, st));
+    }
+    stt = hash_block(s, dev, lay, false, st);
+    if (stt != KVG_OK) return stt;
+    KVG_CUDA(cudaStreamSynchronize(st));
+    kvg_store::Blk b{dev, host, lay, 0, 0};
+    std::vector<int32_t> pos(n);
+    if (host)
+        memcpy(pos.data(), host + lay.pos_off, 4ull * n);
+    else
+        KVG_CUDA(cudaMemcpy(pos.data(), dev + lay.pos_off, 4ull * n, cudaMemcpyDeviceToHost));
+    minmax_positions(pos.data(), n, &b.min_pos, &b.max_pos);
+    s->blocks.push_back(b);
+    *block_id_out = s->blocks.size() - 1;
+    return KVG_OK;
+}
+
+// ------------------------------------------------------------------- graft --
+
+static kvg_status read_status(kvg_cache *c, kvg_graft_report *report) {
+    DevStatus hs;
+    KVG_CUDA(cudaMemcpy(&hs, c->status, sizeof hs, cudaMemcpyDeviceToHost));
+    KVG_CUDA(cudaMemset(c->status, 0, sizeof(DevStatus)));
+    if (report) {
+        report->seq = hs.seq;
+        report->n_mismatch = hs.n_mismatch;
+        report->n_listed = std::min(hs.n_mismatch, (int32_t)KVG_REPORT_MAX_PAGES);
+        for (int i = 0; i < report->n_listed; ++i) report->mismatch_pages[i] = hs.list[i];
+    }
+    if (hs.err == KVG_ERR_DIGEST || hs.n_mismatch)
+        return fail(KVG_ERR_DIGEST, "digest mismatch on %d page(s) (seq %d)", hs.n_mismatch, hs.seq);
+    if (hs.err) return fail((kvg_status)hs.err, "device check failed (detail %d)", hs.err_detail);
+    return KVG_OK;
+}
+
+extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t dst_slot,
+                                int64_t delta, uint32_t flags, void *stream, kvg_graft_report *report) {
+    if (!s || !c) return fail(KVG_ERR_ARG, "null argument");
+    if (block_id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)block_id);
+    if (!same_geometry(s->dims, c->dims)) return fail(KVG_ERR_ARG, "store and cache geometry differ");
+    if (s->device != c->device) return fail(KVG_ERR_ARG, "store and cache on different devices");
+    if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d", seq);
+    if (flags & ~(uint32_t)(KVG_GRAFT_VERIFY | KVG_GRAFT_SYNC)) return fail(KVG_ERR_ARG, "unknown flags");
+    const auto &blk = s->blocks[block_id];
+    const int64_t P = c->dims.page_size;
+    const int64_t boundary = (c->n_slots[seq] + P - 1) / P * P;
+    const int64_t dst = dst_slot < 0 ? boundary : dst_slot;
+    if (dst != boundary) return fail(KVG_ERR_ARG, "dst_slot %d is not the next page boundary %lld", dst_slot, (long long)boundary);
+    const int64_t n = blk.lay.n_tokens, npb = blk.lay.n_pages;
+    if (dst + n > c->max_slots) return fail(KVG_ERR_CAPACITY, "graft past max_slots");
+    if (npb > (int64_t)c->free_list.size()) return fail(KVG_ERR_CAPACITY, "out of free pages");
+    if (blk.min_pos + delta < 0 || blk.max_pos + delta >= (1ll << 31))
+        return fail(KVG_ERR_POSITION, "position tags + delta leave [0, 2^31)");
+    DeviceGuard g(c->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    auto pids = take_pages(c, npb);
+    auto &sp = c->seq_pages[seq];
+    const int64_t jdst = dst / P;
+    sp.insert(sp.end(), pids.begin(), pids.end());
+    c->n_slots[seq] = (int32_t)(dst + n);
+
+    GraftParams p{};
+    p.src = blk.dev + blk.lay.pages_off;
+    p.pool = c->pool;
+    p.page_bytes = c->page_bytes;
+    p.pool_pages = c->n_pages;
+    p.n_layers = c->dims.n_layers;
+    p.block_pages = (int32_t)npb;
+    p.chunk_bytes = copy_chunk_bytes(c->dims);
+    p.n_kv_heads = c->dims.n_kv_heads;
+    p.page_size = (int32_t)P;
+    p.head_dim = c->dims.head_dim;
+    p.n_tokens = n;
+    p.delta = delta;
+    p.rotate = 0;
+    if (delta != 0) {
+        const kvg_dims &sd = s->dims;
+        p.rotate = sd.rope_style == KVG_ROPE_HALF ? 1 : 2;
+        const int half = sd.head_dim / 2;
+        for (int i = 0; i < half; ++i) {
+            const double w = std::pow(sd.rope_theta, -2.0 * i / sd.head_dim);
+            const double a = (double)delta * w;
+            p.cosv[i] = (float)std::cos(a);
+            p.sinv[i] = (float)std::sin(a);
+        }
+    }
+    const int32_t *bpos = reinterpret_cast<const int32_t *>(blk.dev + blk.lay.pos_off);
+    for (int64_t base = 0; base < npb; base += kMaxPagesPerLaunch) {
+        p.npb = (int32_t)std::min<int64_t>(kMaxPagesPerLaunch, npb - base);
+        p.page_base = (int32_t)base;
+        p.src_pos = bpos + base * P;
+        p.dst_pos = c->positions + (int64_t)seq * c->max_slots + dst + base * P;
+        p.table_row = c->page_table + (int64_t)seq * c->max_pages + jdst + base;
+        p.fill_row = c->page_fill + (int64_t)seq * c->max_pages + jdst + base;
+        p.pids.n = p.npb;
+        for (int32_t i = 0; i < p.npb; ++i) p.pids.pid[i] = pids[base + i];
+        KVG_CUDA(launch_graft_copy(p, c->n_sm, st));
+    }
+    if (flags & KVG_GRAFT_VERIFY) {
+        const uint64_t pb = c->page_bytes;
+        const int64_t m = (int64_t)((pb + kLeafBytes - 1) / kLeafBytes);
+        const int64_t n_pages = (int64_t)c->dims.n_layers * 2 * npb;
+        KVG_CUDA(c->leaf.ensure((size_t)n_pages * m * 32));
+        PageSource src;
+        if (delta == 0)
+            src = PageSource{c->pool, pb, c->page_table + (int64_t)seq * c->max_pages + jdst, (int32_t)npb,
+                             (int64_t)c->n_pages};
+        else
+            src = PageSource{blk.dev + blk.lay.pages_off, pb, nullptr, 1, 0};
+        uint32_t *leaf = static_cast<uint32_t *>(c->leaf.ptr);
+        KVG_CUDA(launch_sha256_leaves(src, n_pages, leaf, c->n_sm, st));
+        KVG_CUDA(launch_sha256_pages(leaf, n_pages, m, nullptr, blk.dev + blk.lay.dig_off, c->status, seq, st));
+    }
+    if (report) {
+        memset(report, 0, sizeof *report);
+        report->seq = seq;
+        report->n_pages_checked = (flags & KVG_GRAFT_VERIFY) ? (int32_t)(c->dims.n_layers * 2 * npb) : 0;
+    }
+    if (flags & KVG_GRAFT_SYNC) {
+        KVG_CUDA(cudaStreamSynchronize(st));
+        const int32_t checked = report ? report->n_pages_checked : 0;
+        kvg_status r = read_status(c, report);
+        if (report) report->n_pages_checked = checked;
+        return r;
+    }
+    return KVG_OK;
+}
+
+// ------------------------------------------------------------------ decode --
+
+static int split_target_waves() {
+    static int w = [] {
+        const char *e = getenv("KVG_SPLIT_WAVES");
+        int v = e ? atoi(e) : 0;
+        return v > 0 ? v : 16;
+    }();
+    return w;
+}
+
+extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
+                                           const void *q, int32_t n_q_heads, void *out, float scale,
+                                           void *stream) {
+    if (!c || !seq_ids || !q || !out) return fail(KVG_ERR_ARG, "null argument");
+    const kvg_dims &d = c->dims;
+    if (layer < -1 || layer >= d.n_layers) return fail(KVG_ERR_ARG, "bad layer %d", layer);
+    if (B <= 0 || B > 4096) return fail(KVG_ERR_ARG, "B must be in [1, 4096]");
+    if (n_q_heads <= 0 || n_q_heads % d.n_kv_heads) return fail(KVG_ERR_ARG, "n_q_heads must be a multiple of n_kv_heads");
+    const int G = n_q_heads / d.n_kv_heads;
+    if (!decode_supported(d.head_dim, G)) return fail(KVG_ERR_ARG, "unsupported head_dim %d / group %d", d.head_dim, G);
+    if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out)) & 15)
+        return fail(KVG_ERR_ARG, "q/out must be 16-byte aligned");
+    int64_t max_np = 0, total_np = 0;
+    for (int32_t b = 0; b < B; ++b) {
+        if (seq_ids[b] < 0 || seq_ids[b] >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq id %d", seq_ids[b]);
+        const int64_t np = (int64_t)c->seq_pages[seq_ids[b]].size();
+        max_np = std::max(max_np, np);
+        total_np += np;
+    }
+    DeviceGuard g(c->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int Lrun = layer < 0 ? d.n_layers : 1;
+    const int layer0 = layer < 0 ? 0 : layer;
+    // pages per split: about split_target_waves() CTAs per SM over the whole call
+    const int64_t work = (int64_t)Lrun * d.n_kv_heads * total_np;
+    const int64_t target = (int64_t)c->n_sm * split_target_waves();
+    int64_t pps = std::max<int64_t>(1, (work + target - 1) / target);
+    if (max_np == 0) pps = 1;
+    const int64_t S = std::max<int64_t>(1, (max_np + pps - 1) / pps);
+    const int64_t bchunk = std::min<int64_t>(B, kMaxBatchPerLaunch);
+    const size_t units = (size_t)Lrun * bchunk * d.n_kv_heads * S * G;
+    KVG_CUDA(c->part_o.ensure(units * d.head_dim * sizeof(float)));
+    KVG_CUDA(c->part_ml.ensure(units * sizeof(float2)));
+    for (int64_t b0 = 0; b0 < B; b0 += kMaxBatchPerLaunch) {
+        const int32_t nb = (int32_t)std::min<int64_t>(kMaxBatchPerLaunch, B - b0);
+        DecodeParams p{};
+        p.pool = c->pool;
+        p.pool_pages = c->n_pages;
+        p.n_kv_heads = d.n_kv_heads;
+        p.page_size = d.page_size;
+        p.n_q_heads = n_q_heads;
+        p.layer0 = layer0;
+        p.n_layers_run = Lrun;
+        p.B = nb;
+        p.n_splits = (int32_t)S;
+        p.pages_per_split = (int32_t)pps;
+        p.page_table = c->page_table;
+        p.page_fill = c->page_fill;
+        p.max_pages = c->max_pages;
+        p.q = static_cast<const __nv_bfloat16 *>(q);
+        p.q_row_stride_b = B;
+        p.b0 = (int32_t)b0;
+        p.qscale = scale * 1.4426950408889634f;
+        p.part_o = static_cast<float *>(c->part_o.ptr);
+        p.part_ml = static_cast<float2 *>(c->part_ml.ptr);
+        p.status = c->status;
+        for (int32_t i = 0; i < nb; ++i) {
+            p.rows.seq[i] = seq_ids[b0 + i];
+            p.rows.npages[i] = (int32_t)c->seq_pages[seq_ids[b0 + i]].size();
+        }
+        KVG_CUDA(launch_decode(d.head_dim, G, p, st));
+        CombineParams cp{};
+        cp.part_o = p.part_o;
+        cp.part_ml = p.part_ml;
+        cp.out = static_cast<__nv_bfloat16 *>(out);
+        cp.n_kv_heads = d.n_kv_heads;
+        cp.n_q_heads = n_q_heads;
+        cp.n_splits = (int32_t)S;
+        cp.B = nb;
+        cp.q_row_stride_b = B;
+        cp.b0 = (int32_t)b0;
+        KVG_CUDA(launch_combine(d.head_dim, G, cp, Lrun, nb, st));
+    }
+    return KVG_OK;
+}
+
+// ------------------------------------------------------------------ digest --
+
+namespace {
+std::mutex g_digest_mu;
+Scratch g_digest_leaf[64];
+DevStatus *g_digest_status[64] = {};
+}  // namespace
+
+extern "C" kvg_status kvg_digest(const void *bytes, uint64_t n, int32_t mode, uint64_t page_bytes, uint8_t *out,
+                                 void *stream) {
+    if (!out || (n && !bytes)) return fail(KVG_ERR_ARG, "null argument");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int dev = 0;
+    KVG_CUDA(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= 64) return fail(KVG_ERR_ARG, "device ordinal out of range");
+    if (mode == KVG_SHA256_PLAIN) {
+        KVG_CUDA(launch_sha256_serial(static_cast<const uint8_t *>(bytes), n, nullptr, 0, out, nullptr, nullptr, st));
+        return KVG_OK;
+    }
+    if (mode != KVG_SHA256_PAGED) return fail(KVG_ERR_ARG, "bad mode %d", mode);
+    if (page_bytes == 0 || n % page_bytes) return fail(KVG_ERR_ARG, "n must be a multiple of page_bytes");
+    if (page_bytes % 16 || reinterpret_cast<uintptr_t>(bytes) % 16)
+        return fail(KVG_ERR_ARG, "paged mode needs 16-byte aligned pages");
+    const int64_t n_pages = (int64_t)(n / page_bytes);
+    const int64_t m = (int64_t)((page_bytes + kLeafBytes - 1) / kLeafBytes);
+    std::lock_guard<std::mutex> lk(g_digest_mu);
+    if (!g_digest_status[dev]) {
+        KVG_CUDA(cudaMalloc(&g_digest_status[dev], sizeof(DevStatus)));
+        KVG_CUDA(cudaMemset(g_digest_status[dev], 0, sizeof(DevStatus)));
+    }
+    KVG_CUDA(g_digest_leaf[dev].ensure((size_t)n_pages * m * 32));
+    PageSource src{static_cast<const uint8_t *>(bytes), page_bytes, nullptr, 1, 0};
+    uint32_t *leaf = static_cast<uint32_t *>(g_digest_leaf[dev].ptr);
+    KVG_CUDA(launch_sha256_leaves(src, n_pages, leaf, sm_count(dev), st));
+    KVG_CUDA(launch_sha256_pages(leaf, n_pages, m, out, nullptr, g_digest_status[dev], -1, st));
+    return KVG_OK;
+}
+
+// -------------------------------------------------------------------- misc --
+
+extern "C" kvg_status kvg_sync(kvg_cache *c, void *stream, double timeout_s, kvg_graft_report *report) {
+    if (!c) return fail(KVG_ERR_ARG, "null cache");
+    DeviceGuard g(c->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const auto t0 = std::chrono::steady_clock::now();
+    for (;;) {
+        cudaError_t e = cudaStreamQuery(st);
+        if (e == cudaSuccess) break;
+        if (e != cudaErrorNotReady) return cuda_fail(e, "cudaStreamQuery");
+        const double el = std::chrono::duration<double>(std::chrono::steady_clock::now() - t0).count();
+        if (el > timeout_s) return fail(KVG_ERR_TIMEOUT, "stream still busy after %.3f s", el);
+        std::this_thread::sleep_for(std::chrono::microseconds(50));
+    }
+    if (report) memset(report, 0, sizeof *report);
+    return read_status(c, report);
+}
+
+extern "C" const char *kvg_status_string(kvg_status s) {
+    switch (s) {
+        case KVG_OK: return "ok";
+        case KVG_ERR_ARG: return "invalid argument";
+        case KVG_ERR_OOM: return "out of memory";
+        case KVG_ERR_CUDA: return "CUDA error";
+        case KVG_ERR_NOT_FOUND: return "block not found";
+        case KVG_ERR_CAPACITY: return "capacity exceeded";
+        case KVG_ERR_POSITION: return "position out of range";
+        case KVG_ERR_DIGEST: return "digest mismatch";
+        case KVG_ERR_FORMAT: return "bad block format";
+        case KVG_ERR_TIMEOUT: return "timeout";
+        case KVG_ERR_DEVICE_CHECK: return "device-side check failed";
+    }
+    return "unknown status";
+}
+
+extern "C" const char *kvg_last_error(void) { return g_last_error.c_str(); }
+
+extern "C" uint32_t kvg_version(void) { return 0x000100u; }

@@ -1,0 +1,323 @@
+// sha256_kernels.cu — SHA-256 (FIPS 180-4) on the GPU for page digests.
+//
+// The digest of a page is SHA-256 over the concatenated SHA-256 digests of its
+// consecutive 4096-byte leaves.  A leaf is a serial Merkle-Damgard chain, so
+// the natural mapping is one thread per leaf (65 compressions for a 4 KB
+// leaf); a second kernel hashes each page's leaf digests with one thread per
+// page.  Integer-ALU bound: ~1.7k simple integer ops per 64-byte block.
+#include "common.cuh"
+
+namespace kvg {
+
+namespace {
+
+// FIPS 180-4 sec. 4.2.2 round constants and sec. 5.3.3 initial hash value.
+__constant__ uint32_t kK[64] = {
+    0x428a2f98u, 0x71374491u, 0xb5c0fbcfu, 0xe9b5dba5u, 0x3956c25bu, 0x59f111f1u, 0x923f82a4u,
+    0xab1c5ed5u, 0xd807aa98u, 0x12835b01u, 0x243185beu, 0x550c7dc3u, 0x72be5d74u, 0x80deb1feu,
+    0x9bdc06a7u, 0xc19bf174u, 0xe49b69c1u, 0xefbe4786u, 0x0fc19dc6u, 0x240ca1ccu, 0x2de92c6fu,
+    0x4a7484aau, 0x5cb0a9dcu, 0x76f988dau, 0x983e5152u, 0xa831c66du, 0xb00327c8u, 0xbf597fc7u,
+    0xc6e00bf3u, 0xd5a79147u, 0x06ca6351u, 0x14292967u, 0x27b70a85u, 0x2e1b2138u, 0x4d2c6dfcu,
+    0x53380d13u, 0x650a7354u, 0x766a0abbu, 0x81c2c92eu, 0x92722c85u, 0xa2bfe8a1u, 0xa81a664bu,
+    0xc24b8b70u, 0xc76c51a3u, 0xd192e819u, 0xd6990624u, 0xf40e3585u, 0x106aa070u, 0x19a4c116u,
+    0x1e376c08u, 0x2748774cu, 0x34b0bcb5u, 0x391c0cb3u, 0x4ed8aa4au, 0x5b9cca4fu, 0x682e6ff3u,
+    0x748f82eeu, 0x78a5636fu, 0x84c87814u, 0x8cc70208u, 0x90befffau, 0xa4506cebu, 0xbef9a3f7u,
+    0xc67178f2u};
+__constant__ uint32_t kH0[8] = {0x6a09e667u, 0xbb67ae85u, 0x3c6ef372u, 0xa54ff53au,
+                                0x510e527fu, 0x9b05688cu, 0x1f83d9abu, 0x5be0cd19u};
+
+__device__ __forceinline__ uint32_t rotr(uint32_t x, int n) { return __funnelshift_r(x, x, n); }
+
+__device__ __forceinline__ uint32_t bswap(uint32_t x) { return __byte_perm(x, 0, 0x0123); }
+
+// One compression of the 16-word block w (FIPS 180-4 sec. 6.2.2), with the
+// message schedule kept as a rolling 16-word window.
+__device__ __forceinline__ void compress(uint32_t st[8], uint32_t w[16]) {
+    uint32_t a = st[0], b = st[1], c = st[2], d = st[3], e = st[4], f = st[5], g = st[6], h = st[7];
+#pragma unroll
+    for (int t = 0; t < 64; ++t) {
+        uint32_t wt;
+        if (t < 16) {
+            wt = w[t];
+        } else {
+            const uint32_t w15 = w[(t - 15) & 15], w2 = w[(t - 2) & 15];
+            const uint32_t s0 = rotr(w15, 7) ^ rotr(w15, 18) ^ (w15 >> 3);
+            const uint32_t s1 = rotr(w2, 17) ^ rotr(w2, 19) ^ (w2 >> 10);
+            wt = w[t & 15] = w[t & 15] + s0 + w[(t - 7) & 15] + s1;
+        }
+        const uint32_t S1 = rotr(e, 6) ^ rotr(e, 11) ^ rotr(e, 25);
+        const uint32_t ch = (e & f) ^ (~e & g);
+        const uint32_t T1 = h + S1 + ch + kK[t] + wt;
+        const uint32_t S0 = rotr(a, 2) ^ rotr(a, 13) ^ rotr(a, 22);
+        const uint32_t maj = (a & b) ^ (a & c) ^ (b & c);
+        const uint32_t T2 = S0 + maj;
+        h = g;
+        g = f;
+        f = e;
+        e = d + T1;
+        d = c;
+        c = b;
+        b = a;
+        a = T1 + T2;
+    }
+    st[0] += a;
+    st[1] += b;
+    st[2] += c;
+    st[3] += d;
+    st[4] += e;
+    st[5] += f;
+    st[6] += g;
+    st[7] += h;
+}
+
+__device__ __forceinline__ void init_state(uint32_t st[8]) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) st[i] = kH0[i];
+}
+
+// Final block(s) for a message whose last `rem` (< 64) bytes start at `tail`
+// and whose total length is `total_bytes`.
+__device__ void finish(uint32_t st[8], const uint8_t *tail, int rem, uint64_t total_bytes) {
+    uint32_t w[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) w[i] = 0;
+    for (int k = 0; k < rem; ++k) w[k >> 2] |= (uint32_t)tail[k] << (24 - 8 * (k & 3));
+    w[rem >> 2] |= 0x80u << (24 - 8 * (rem & 3));
+    const uint64_t bits = total_bytes * 8ull;
+    if (rem < 56) {
+        w[14] = (uint32_t)(bits >> 32);
+        w[15] = (uint32_t)bits;
+        compress(st, w);
+    } else {
+        compress(st, w);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) w[i] = 0;
+        w[14] = (uint32_t)(bits >> 32);
+        w[15] = (uint32_t)bits;
+        compress(st, w);
+    }
+}
+
+__device__ __forceinline__ const uint8_t *page_addr(const PageSource &s, int64_t p) {
+    if (!s.pid) return s.base + (uint64_t)p * s.page_bytes;
+    const int64_t plane = p / s.npb;
+    const int64_t j = p - plane * s.npb;
+    return s.base + ((uint64_t)plane * s.plane_pages + (uint64_t)s.pid[j]) * s.page_bytes;
+}
+
+__global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src, int64_t n_pages,
+                                                            int64_t leaves_per_page,
+                                                            uint32_t *__restrict__ out) {
+    const int64_t n_leaves = n_pages * leaves_per_page;
+    for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < n_leaves;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t p = idx / leaves_per_page;
+        const int64_t i = idx - p * leaves_per_page;
+        uint64_t len = src.page_bytes - (uint64_t)i * kLeafBytes;
+        if (len > kLeafBytes) len = kLeafBytes;
+        const uint8_t *leaf = page_addr(src, p) + (uint64_t)i * kLeafBytes;
+        const uint4 *v = reinterpret_cast<const uint4 *>(leaf);
+        uint32_t st[8];
+        init_state(st);
+        const int nfull = (int)(len >> 6);
+        for (int blk = 0; blk < nfull; ++blk) {
+            uint32_t w[16];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint4 x = __ldg(v + 4 * blk + q);
+                w[4 * q + 0] = bswap(x.x);
+                w[4 * q + 1] = bswap(x.y);
+                w[4 * q + 2] = bswap(x.z);
+                w[4 * q + 3] = bswap(x.w);
+            }
+            compress(st, w);
+        }
+        const int rem = (int)(len & 63);
+        if (rem == 0) {
+            uint32_t w[16];
+#pragma unroll
+            for (int q = 0; q < 16; ++q) w[q] = 0;
+            w[0] = 0x80000000u;
+            const uint64_t bits = len * 8ull;
+            w[14] = (uint32_t)(bits >> 32);
+            w[15] = (uint32_t)bits;
+            compress(st, w);
+        } else {
+            finish(st, leaf + (len & ~63ull), rem, len);
+        }
+        uint4 *o = reinterpret_cast<uint4 *>(out + idx * 8);
+        o[0] = make_uint4(st[0], st[1], st[2], st[3]);
+        o[1] = make_uint4(st[4], st[5], st[6], st[7]);
+    }
+}
+
+// Page digest from its leaf digests: the message is the leaf digests' bytes,
+// i.e. (big-endian) exactly the 8 state words of each leaf in order.
+__global__ void __launch_bounds__(128) sha256_pages_kernel(const uint32_t *__restrict__ leaf_words,
+                                                           int64_t n_pages, int64_t m,
+                                                           uint8_t *__restrict__ out,
+                                                           const uint8_t *__restrict__ expected,
+                                                           DevStatus *status, int32_t seq) {
+    const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (p >= n_pages) return;
+    const uint32_t *lw = leaf_words + p * m * 8;
+    uint32_t st[8];
+    init_state(st);
+    const int64_t nwords = m * 8;
+    const int64_t nfull = nwords / 16;
+    for (int64_t blk = 0; blk < nfull; ++blk) {
+        uint32_t w[16];
+        const uint4 *v = reinterpret_cast<const uint4 *>(lw + blk * 16);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const uint4 x = v[q];
+            w[4 * q + 0] = x.x;
+            w[4 * q + 1] = x.y;
+            w[4 * q + 2] = x.z;
+            w[4 * q + 3] = x.w;
+        }
+        compress(st, w);
+    }
+    {
+        uint32_t w[16];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) w[q] = 0;
+        const int remw = (int)(nwords - nfull * 16);  // 0 or 8
+        for (int q = 0; q < remw; ++q) w[q] = lw[nfull * 16 + q];
+        w[remw] = 0x80000000u;
+        const uint64_t bits = (uint64_t)m * 32ull * 8ull;
+        w[14] = (uint32_t)(bits >> 32);
+        w[15] = (uint32_t)bits;
+        compress(st, w);
+    }
+    uint8_t dg[32];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        dg[4 * k + 0] = (uint8_t)(st[k] >> 24);
+        dg[4 * k + 1] = (uint8_t)(st[k] >> 16);
+        dg[4 * k + 2] = (uint8_t)(st[k] >> 8);
+        dg[4 * k + 3] = (uint8_t)st[k];
+    }
+    if (out) {
+#pragma unroll
+        for (int k = 0; k < 32; ++k) out[p * 32 + k] = dg[k];
+    }
+    if (expected) {
+        bool same = true;
+#pragma unroll
+        for (int k = 0; k < 32; ++k) same &= dg[k] == expected[p * 32 + k];
+        if (!same) {
+            const int slot = atomicAdd(&status->n_mismatch, 1);
+            if (slot < KVG_REPORT_MAX_PAGES) status->list[slot] = (int32_t)p;
+            status->seq = seq;
+            atomicCAS(&status->err, 0, (int32_t)KVG_ERR_DIGEST);
+        }
+    }
+}
+
+// Streaming single-thread hasher for seg0 || seg1 of arbitrary lengths.
+struct Stream {
+    uint32_t st[8];
+    uint32_t w[16];
+    int fill;  // bytes in w
+    uint64_t total;
+
+    __device__ void init() {
+        init_state(st);
+        fill = 0;
+        total = 0;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) w[i] = 0;
+    }
+    __device__ void byte(uint8_t x) {
+        w[fill >> 2] |= (uint32_t)x << (24 - 8 * (fill & 3));
+        if (++fill == 64) {
+            compress(st, w);
+            fill = 0;
+#pragma unroll
+            for (int i = 0; i < 16; ++i) w[i] = 0;
+        }
+    }
+    __device__ void feed(const uint8_t *ptr, uint64_t n) {
+        total += n;
+        uint64_t k = 0;
+        while (k < n && (fill != 0 || (reinterpret_cast<uintptr_t>(ptr + k) & 3))) byte(ptr[k++]);
+        while (n - k >= 64) {
+            const uint32_t *q = reinterpret_cast<const uint32_t *>(ptr + k);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) w[i] = bswap(q[i]);
+            compress(st, w);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) w[i] = 0;
+            k += 64;
+        }
+        while (k < n) byte(ptr[k++]);
+    }
+    __device__ void final(uint8_t out[32]) {
+        const uint64_t bits = total * 8ull;
+        byte(0x80);
+        while (fill != 56) byte(0);
+        for (int i = 7; i >= 0; --i) byte((uint8_t)(bits >> (8 * i)));
+        for (int k = 0; k < 8; ++k) {
+            out[4 * k + 0] = (uint8_t)(st[k] >> 24);
+            out[4 * k + 1] = (uint8_t)(st[k] >> 16);
+            out[4 * k + 2] = (uint8_t)(st[k] >> 8);
+            out[4 * k + 3] = (uint8_t)st[k];
+        }
+    }
+};
+
+__global__ void sha256_serial_kernel(const uint8_t *seg0, uint64_t n0, const uint8_t *seg1,
+                                     uint64_t n1, uint8_t *out, const uint8_t *expected,
+                                     DevStatus *status) {
+    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+    Stream s;
+    s.init();
+    if (n0) s.feed(seg0, n0);
+    if (n1) s.feed(seg1, n1);
+    uint8_t dg[32];
+    s.final(dg);
+    if (out)
+        for (int k = 0; k < 32; ++k) out[k] = dg[k];
+    if (expected) {
+        bool same = true;
+        for (int k = 0; k < 32; ++k) same &= dg[k] == expected[k];
+        if (!same) {
+            atomicAdd(&status->n_mismatch, 1);
+            atomicCAS(&status->err, 0, (int32_t)KVG_ERR_DIGEST);
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_t *leaf_words,
+                                 int n_sm, cudaStream_t s) {
+    const int64_t m = (int64_t)((src.page_bytes + kLeafBytes - 1) / kLeafBytes);
+    const int64_t n = n_pages * m;
+    if (n == 0) return cudaSuccess;
+    int64_t grid = (n + 127) / 128;
+    const int64_t cap = (int64_t)n_sm * 16;
+    if (grid > cap) grid = cap;
+    sha256_leaves_kernel<<<(int)grid, 128, 0, s>>>(src, n_pages, m, leaf_words);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sha256_pages(const uint32_t *leaf_words, int64_t n_pages, int64_t leaves_per_page,
+                                uint8_t *out, const uint8_t *expected, DevStatus *status,
+                                int32_t seq, cudaStream_t s) {
+    if (n_pages == 0) return cudaSuccess;
+    sha256_pages_kernel<<<(int)((n_pages + 127) / 128), 128, 0, s>>>(leaf_words, n_pages,
+                                                                     leaves_per_page, out,
+                                                                     expected, status, seq);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sha256_serial(const uint8_t *seg0, uint64_t n0, const uint8_t *seg1, uint64_t n1,
+                                 uint8_t *out, const uint8_t *expected, DevStatus *status,
+                                 cudaStream_t s) {
+    sha256_serial_kernel<<<1, 32, 0, s>>>(seg0, n0, seg1, n1, out, expected, status);
+    return cudaGetLastError();
+}
+
+}  // namespace kvg

@@ -1,0 +1,338 @@
+"""GPU parity: the CUDA library (through its C ABI) against the CPU oracle on
+the same seeded inputs.  Graft, page tables, positions, block bytes and
+digests must match bit for bit; decode attention within 1e-2 max-abs of the
+fp64 oracle (bf16 out, fp32 accumulate); relocated keys within 2e-2 of the
+fp64 rotation; grafted-vs-fresh attention outputs SHA-256-identical."""
+import hashlib
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import kvg_synth as syn
+from kvg_testlib import (CANARY, append, compare_decode, decode, dev_view, dims_for, fill_canary,
+                         geometry, need_gpu, oracle_dims, pool_u16, tables, to_dev, u16)
+
+pytestmark = pytest.mark.gpu
+
+HBM_CAP = 8 << 30
+
+
+def _kv(w, n, seed):
+    k, v = syn.kv_rows(w, n, seed)
+    return syn.as_u16(k), syn.as_u16(v)
+
+
+def _slots(w, n):
+    return (-(-n // w.page_size) + 2) * w.page_size
+
+
+def _sha(a: np.ndarray) -> bytes:
+    return hashlib.sha256(np.ascontiguousarray(a).tobytes()).digest()
+
+
+# ------------------------------------------------------------------- digests
+
+NIST = [b"", b"abc", b"abcdbcdecdefdefgefghfghighijhijkijkljklmklmnlmnomnopnopq", b"a" * 1_000_000,
+        bytes(range(256)) * 3 + b"xyz"]
+
+
+@pytest.mark.parametrize("msg", NIST, ids=["empty", "abc", "448bit", "million_a", "odd_len"])
+def test_digest_plain_matches_hashlib(msg):
+    kvg = need_gpu()
+    buf = torch.frombuffer(bytearray(msg or b"\0"), dtype=torch.uint8).cuda()
+    out = torch.zeros(32, dtype=torch.uint8, device="cuda")
+    kvg.kvg_digest(buf.data_ptr(), len(msg), kvg.KVG_SHA256_PLAIN, 0, out.data_ptr())
+    torch.cuda.synchronize()
+    assert bytes(out.cpu().numpy()) == hashlib.sha256(msg).digest()
+
+
+@pytest.mark.parametrize("page_bytes,n_pages", [(4096, 7), (262144, 5), (10000, 3), (64, 9), (65552, 2)])
+def test_digest_paged_matches_oracle(oracle, page_bytes, n_pages):
+    kvg = need_gpu()
+    rng = np.random.default_rng(page_bytes)
+    data = rng.integers(0, 256, page_bytes * n_pages, dtype=np.uint8)
+    d = torch.from_numpy(data).cuda()
+    out = torch.zeros(32 * n_pages, dtype=torch.uint8, device="cuda")
+    kvg.kvg_digest(d.data_ptr(), data.size, kvg.KVG_SHA256_PAGED, page_bytes, out.data_ptr())
+    torch.cuda.synchronize()
+    assert np.array_equal(out.cpu().numpy().reshape(n_pages, 32), oracle.page_digests(data, page_bytes))
+
+
+# ------------------------------------------------------------ graft parity
+
+CASES = [("tiny", 256, 0), ("tiny", 250, 37), ("d128", 1000, 700), ("d256", 700, 300), ("g4", 333, 100)]
+
+
+def _build_both(kvg, oracle, w, nb, nf, residency=0, style=0, seed=1, copies=1):
+    """Deposits an nb-token block from a freshly written sequence and grafts
+    it (then appends nf fresh tokens) into a canary-filled cache, on both
+    sides.  Returns everything the tests compare."""
+    k, v = _kv(w, nb + nf, seed)
+    max_slots = _slots(w, nb + nf)
+    n_pages = (max_slots // w.page_size + 3) * copies
+    dims = dims_for(kvg, w, style)
+    src = kvg.Cache(dims, n_pages, 2, max_slots)
+    kvg.kvg_cache_set_free_order(src.h, syn.permutation(n_pages, seed + 7))
+    append(kvg, src, 0, k[:, :nb], v[:, :nb], syn.positions(0, nb))
+    store = kvg.Store(dims, residency, HBM_CAP)
+    bid = kvg.kvg_deposit(store.h, src.h, 0, 0, nb)
+    dst = kvg.Cache(dims, n_pages, 3, max_slots)
+    fill_canary(dst)
+    od = oracle_dims(oracle, w, style)
+    oblk = oracle.block_from_kv(od, k[:, :nb], v[:, :nb], syn.positions(0, nb))
+    ocache = oracle.OracleCache(od, n_pages, 3, max_slots, fill=CANARY)
+    return dict(k=k, v=v, src=src, store=store, bid=bid, dst=dst, oblk=oblk, ocache=ocache,
+                n_pages=n_pages, max_slots=max_slots, dims=dims)
+
+
+@pytest.mark.parametrize("geo,nb,nf", CASES)
+def test_deposit_graft_append_bit_exact(oracle, geo, nb, nf):
+    kvg = need_gpu()
+    w = geometry(geo)
+    s = _build_both(kvg, oracle, w, nb, nf)
+    # deposit: the serialized block equals the oracle's byte for byte
+    assert kvg.kvg_store_export(s["store"].h, s["bid"]) == s["oblk"].serialize()
+    info = kvg.kvg_store_block_info(s["store"].h, s["bid"])
+    assert bytes(info.block_digest) == s["oblk"].block_digest
+    rep = kvg.kvg_graft_report()
+    kvg.kvg_graft(s["store"].h, s["bid"], s["dst"].h, 1, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC,
+                  report=rep)
+    assert rep.n_mismatch == 0 and rep.n_pages_checked == w.n_layers * 2 * s["oblk"].n_pages
+    append(kvg, s["dst"], 1, s["k"][:, nb:], s["v"][:, nb:], syn.positions(nb, nf))
+    oc = s["ocache"]
+    oc.graft(1, s["oblk"])
+    oc.append(1, s["k"][:, nb:], s["v"][:, nb:], syn.positions(nb, nf))
+    assert np.array_equal(pool_u16(s["dst"], w), oc.pool)
+    pt, pf, ps = tables(s["dst"])
+    assert np.array_equal(pt, oc.page_table) and np.array_equal(pf, oc.page_fill)
+    assert np.array_equal(ps, oc.positions)
+    assert kvg.kvg_cache_seq_info(s["dst"].h, 1) == (nb + nf, int((oc.page_table[1] >= 0).sum()))
+
+
+@pytest.mark.parametrize("geo,nb,nf", [("tiny", 250, 37), ("d256", 700, 300)])
+def test_pinned_host_store_graft_bit_exact(oracle, geo, nb, nf):
+    kvg = need_gpu()
+    w = geometry(geo)
+    s = _build_both(kvg, oracle, w, nb, nf, residency=kvg.KVG_RESIDENCY_PINNED_HOST, seed=3)
+    assert kvg.kvg_store_export(s["store"].h, s["bid"]) == s["oblk"].serialize()
+    kvg.kvg_graft(s["store"].h, s["bid"], s["dst"].h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+    s["ocache"].graft(0, s["oblk"])
+    assert np.array_equal(pool_u16(s["dst"], w), s["ocache"].pool)
+
+
+# ----------------------------------------------------------- decode parity
+
+@pytest.mark.parametrize("geo,nb,nf", CASES)
+def test_decode_matches_oracle_and_grafted_equals_fresh(oracle, geo, nb, nf):
+    kvg = need_gpu()
+    w = geometry(geo)
+    s = _build_both(kvg, oracle, w, nb, nf, seed=11)
+    kvg.kvg_graft(s["store"].h, s["bid"], s["dst"].h, 2, -1, 0, kvg.KVG_GRAFT_SYNC)
+    append(kvg, s["dst"], 2, s["k"][:, nb:], s["v"][:, nb:], syn.positions(nb, nf))
+    q = syn.as_u16(syn.queries(w, w.n_layers, 1, 11))
+    o = decode(kvg, s["dst"], w, [2], q)
+    scale = 1.0 / math.sqrt(w.head_dim)
+    for l in range(w.n_layers):
+        ref = oracle.gqa_decode(q[l, 0], s["k"][l], s["v"][l], scale)
+        compare_decode(oracle, o[l, 0], ref)
+    # the same rows written fresh into differently placed pages: identical bytes
+    fresh = kvg.Cache(s["dims"], s["n_pages"], 1, s["max_slots"])
+    kvg.kvg_cache_set_free_order(fresh.h, syn.permutation(s["n_pages"], 99))
+    append(kvg, fresh, 0, s["k"], s["v"], syn.positions(0, nb + nf))
+    of = decode(kvg, fresh, w, [0], q)
+    assert _sha(of) == _sha(o)
+    # run-to-run bitwise determinism
+    for _ in range(3):
+        assert _sha(decode(kvg, s["dst"], w, [2], q)) == _sha(o)
+    # one layer at a time is within tolerance too
+    for l in range(w.n_layers):
+        ol = decode(kvg, s["dst"], w, [2], q[l:l + 1], layer=l)
+        compare_decode(oracle, ol[0, 0], oracle.gqa_decode(q[l, 0], s["k"][l], s["v"][l], scale))
+
+
+def test_decode_closed_forms(oracle):
+    kvg = need_gpu()
+    w = geometry("d128")
+    dims = dims_for(kvg, w)
+    cache = kvg.Cache(dims, 16, 4, 512)
+    scale = 1 / math.sqrt(w.head_dim)
+    # one token: the softmax weight is exactly 1, so o is v0 bit for bit
+    k, v = _kv(w, 1, 21)
+    append(kvg, cache, 0, k, v, syn.positions(0, 1))
+    q = syn.as_u16(syn.queries(w, w.n_layers, 1, 21))
+    o = decode(kvg, cache, w, [0], q)
+    G = w.group
+    for l in range(w.n_layers):
+        for h in range(w.n_q_heads):
+            assert np.array_equal(o[l, 0, h], v[l, 0, h // G])
+    # every value row equal: o equals that row
+    n = 300
+    k2, _ = _kv(w, n, 22)
+    row = syn.as_u16(syn.normal_bf16((w.n_layers, 1, w.n_kv_heads, w.head_dim), 23))
+    v2 = np.repeat(row, n, axis=1)
+    append(kvg, cache, 1, k2, v2, syn.positions(0, n))
+    o2 = decode(kvg, cache, w, [1], q)
+    for l in range(w.n_layers):
+        for h in range(w.n_q_heads):
+            assert np.array_equal(o2[l, 0, h], row[l, 0, h // G])
+    # empty sequence: zeros; a batch mixing empty and non-empty rows
+    o3 = decode(kvg, cache, w, [3, 0, 1], np.repeat(q, 3, axis=1))
+    assert not o3[:, 0].any()
+    assert np.array_equal(o3[:, 1], o[:, 0])
+
+
+def test_decode_batch_ragged_vs_oracle(oracle):
+    kvg = need_gpu()
+    w = geometry("d256")
+    dims = dims_for(kvg, w)
+    lens = [1, 63, 64, 65, 500, 1111]
+    max_slots = _slots(w, max(lens))
+    cache = kvg.Cache(dims, sum(-(-n // w.page_size) for n in lens) + 4, len(lens), max_slots)
+    kvs = []
+    for i, n in enumerate(lens):
+        k, v = _kv(w, n, 30 + i)
+        kvs.append((k, v))
+        append(kvg, cache, i, k, v, syn.positions(0, n))
+    order = [5, 0, 3, 1, 4, 2]
+    q = syn.as_u16(syn.queries(w, w.n_layers, len(order), 31))
+    o = decode(kvg, cache, w, order, q)
+    for bi, sq in enumerate(order):
+        k, v = kvs[sq]
+        for l in range(w.n_layers):
+            compare_decode(oracle, o[l, bi], oracle.gqa_decode(q[l, bi], k[l], v[l], 1 / math.sqrt(w.head_dim)))
+
+
+# --------------------------------------------------------------- relocation
+
+def _logical_k(pool, pt, w, seq, n):
+    out = np.zeros((w.n_layers, n, w.n_kv_heads, w.head_dim), np.uint16)
+    for t in range(n):
+        j, r = divmod(t, w.page_size)
+        out[:, t] = pool[:, 0, pt[seq, j], :, r, :]
+    return out
+
+
+@pytest.mark.parametrize("geo,style", [("tiny", 0), ("d128", 0), ("d128", 1), ("d256", 0)])
+def test_relocated_graft_within_tolerance(oracle, geo, style):
+    kvg = need_gpu()
+    w = geometry(geo)
+    nb = 200 if geo != "d128" else 333
+    s = _build_both(kvg, oracle, w, nb, 0, style=style, seed=41, copies=3)
+    # own position through the relocation entry with delta = 0 is the pure copy
+    kvg.kvg_graft(s["store"].h, s["bid"], s["dst"].h, 0, -1, 0, kvg.KVG_GRAFT_SYNC)
+    s["ocache"].graft(0, s["oblk"])
+    for i, delta in enumerate([1, 4096, 100000]):
+        seq = 1 + (i % 2)
+        if i == 2:
+            kvg.kvg_cache_release(s["dst"].h, 1)
+            s["ocache"].release(1)
+        kvg.kvg_graft(s["store"].h, s["bid"], s["dst"].h, seq, -1, delta,
+                      kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+        s["ocache"].graft(seq, s["oblk"], delta=delta)
+        pool = pool_u16(s["dst"], w)
+        pt, pf, ps = tables(s["dst"])
+        oc = s["ocache"]
+        assert np.array_equal(pt, oc.page_table) and np.array_equal(pf, oc.page_fill)
+        assert np.array_equal(ps, oc.positions)
+        # values, padding rows and untouched pages: bit-exact
+        assert np.array_equal(pool[:, 1], oc.pool[:, 1])
+        kg = _logical_k(pool, pt, w, seq, nb)
+        k64 = np.stack([oracle.rope_rotate_rows(s["k"][l, :nb], delta, w.rope_theta, style)
+                        for l in range(w.n_layers)])
+        err = np.abs(oracle.bf16_to_f64(kg) - k64).max()
+        assert err <= 2e-2, err
+        # bytes outside the valid key rows equal the oracle's
+        mask = np.ones(pool.shape[:3] + pool.shape[3:], bool)[:, 0]
+        for t in range(nb):
+            j, r = divmod(t, w.page_size)
+            mask[:, pt[seq, j], :, r, :] = False
+        assert np.array_equal(pool[:, 0][mask], oc.pool[:, 0][mask])
+
+
+def test_relocated_decode_is_delta_invariant_within_tolerance(oracle):
+    # keys re-based by delta and the query rotated by delta: the fp64 oracle is
+    # delta-invariant; the GPU output stays within tolerance of it
+    kvg = need_gpu()
+    w = geometry("d128")
+    nb = 512
+    s = _build_both(kvg, oracle, w, nb, 0, seed=43, copies=3)
+    q0 = syn.as_u16(syn.queries(w, w.n_layers, 1, 43))
+    scale = 1 / math.sqrt(w.head_dim)
+    ref = [oracle.gqa_decode(q0[l, 0], s["k"][l], s["v"][l], scale) for l in range(w.n_layers)]
+    for seq, delta in enumerate([0, 1, 4096]):
+        kvg.kvg_graft(s["store"].h, s["bid"], s["dst"].h, seq, -1, delta, kvg.KVG_GRAFT_SYNC)
+        qd = np.stack([oracle.rope_rotate_rows_bf16(q0[l], delta, w.rope_theta, 0) for l in range(w.n_layers)])
+        o = decode(kvg, s["dst"], w, [seq], qd)
+        for l in range(w.n_layers):
+            compare_decode(oracle, o[l, 0], ref[l])
+
+
+# ------------------------------------------------------- integrity & errors
+
+def test_verify_detects_a_flipped_byte(oracle):
+    kvg = need_gpu()
+    w = geometry("d128")
+    s = _build_both(kvg, oracle, w, 300, 0, seed=51, copies=3)
+    blob = bytearray(kvg.kvg_store_export(s["store"].h, s["bid"]))
+    info = kvg.kvg_store_block_info(s["store"].h, s["bid"])
+    npb = info.n_pages
+    bad_page = (1 * 2 + 1) * npb + 2  # layer 1, V, page 2
+    blob[info.pages_offset + bad_page * s["dims"].n_kv_heads * w.page_size * w.head_dim * 2 + 100] ^= 0x10
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_store_import(s["store"].h, bytes(blob), kvg.KVG_GRAFT_VERIFY)
+    assert e.value.status == kvg.KVG_ERR_DIGEST
+    bid2 = kvg.kvg_store_import(s["store"].h, bytes(blob), 0)
+    rep = kvg.kvg_graft_report()
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_graft(s["store"].h, bid2, s["dst"].h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC,
+                      report=rep)
+    assert e.value.status == kvg.KVG_ERR_DIGEST
+    assert rep.n_mismatch == 1 and rep.mismatch_pages[0] == bad_page and rep.seq == 0
+    # asynchronous form: the mismatch surfaces at kvg_sync
+    kvg.kvg_graft(s["store"].h, bid2, s["dst"].h, 1, -1, 0, kvg.KVG_GRAFT_VERIFY)
+    rep2 = kvg.kvg_graft_report()
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_sync(s["dst"].h, None, 10.0, rep2)
+    assert e.value.status == kvg.KVG_ERR_DIGEST and rep2.mismatch_pages[0] == bad_page
+    # the intact block verifies and imports cleanly
+    good = kvg.kvg_store_export(s["store"].h, s["bid"])
+    bid3 = kvg.kvg_store_import(s["store"].h, good, kvg.KVG_GRAFT_VERIFY)
+    assert kvg.kvg_store_export(s["store"].h, bid3) == good
+    kvg.kvg_sync(s["dst"].h)
+
+
+def test_host_checks_reject_bad_calls(oracle):
+    kvg = need_gpu()
+    w = geometry("tiny")
+    s = _build_both(kvg, oracle, w, 40, 0, seed=61)
+    st, dst = s["store"].h, s["dst"].h
+    E = kvg.KvgError
+    with pytest.raises(E) as e:
+        kvg.kvg_graft(st, 99, dst, 0)
+    assert e.value.status == kvg.KVG_ERR_NOT_FOUND
+    with pytest.raises(E) as e:
+        kvg.kvg_graft(st, s["bid"], dst, 0, 16)  # not the next page boundary (0)
+    assert e.value.status == kvg.KVG_ERR_ARG
+    with pytest.raises(E) as e:
+        kvg.kvg_graft(st, s["bid"], dst, 0, -1, -5)  # positions 0.. + delta < 0
+    assert e.value.status == kvg.KVG_ERR_POSITION
+    with pytest.raises(E) as e:
+        kvg.kvg_graft(st, s["bid"], dst, 0, -1, 2**31 - 20)
+    assert e.value.status == kvg.KVG_ERR_POSITION
+    assert kvg.kvg_cache_seq_info(dst, 0) == (0, 0)  # failed calls changed nothing
+    small = kvg.Cache(s["dims"], 2, 1, 64)
+    with pytest.raises(E) as e:
+        kvg.kvg_graft(st, s["bid"], small.h, 0)  # 3 pages needed, 2 exist
+    assert e.value.status == kvg.KVG_ERR_CAPACITY
+    with pytest.raises(E) as e:
+        kvg.kvg_deposit(st, s["src"].h, 0, 8, 10)  # slot0 not page-aligned
+    assert e.value.status == kvg.KVG_ERR_ARG
+    q = torch.zeros((w.n_layers, 1, 3, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(E) as e:
+        kvg.kvg_decode_attention(dst, -1, [0], q.data_ptr(), 3, q.data_ptr(), 0.1)
+    assert e.value.status == kvg.KVG_ERR_ARG
+    with pytest.raises(E) as e:
+        kvg.kvg_cache_set_free_order(s["src"].h, list(range(s["n_pages"])))  # pages in use
+    assert e.value.status == kvg.KVG_ERR_ARG
