@@ -239,6 +239,15 @@ kvg_status kvg_graft(kvg_store *store, uint64_t block_id, kvg_cache *cache, int3
                      int32_t dst_slot, int64_t delta, uint32_t flags, void *stream,
                      kvg_graft_report *report);
 
+/* Re-checks a grafted range: hashes the cache pages that hold slots
+ * [slot0, slot0 + n_tokens(block)) of `seq` (slot0 page-aligned) on the GPU
+ * and compares each page digest with block `block_id`'s stored digest
+ * (Sec. 4.11 integrity check, applied to the live copy).  Only meaningful for
+ * own-position grafts (relocated key pages differ by design).  Flags and
+ * reporting as for kvg_graft (KVG_GRAFT_SYNC waits and fills `report`). */
+kvg_status kvg_verify(kvg_store *store, uint64_t block_id, kvg_cache *cache, int32_t seq,
+                      int32_t slot0, uint32_t flags, void *stream, kvg_graft_report *report);
+
 /* ------------------------------------------------------------- decode -- */
 
 /* Decode attention of one query token per sequence (Sec. 3.2, Sec. 4.3):
@@ -286,6 +295,10 @@ const char *kvg_last_error(void);
 
 /* Library version, e.g. 0x000100 for 0.1.0. */
 uint32_t kvg_version(void);
+
+/* Number of CUDA kernel launches this library has issued since it was
+ * loaded (all devices, all threads).  A diagnostic for benchmarks. */
+uint64_t kvg_launch_count(void);
 
 #ifdef __cplusplus
 }

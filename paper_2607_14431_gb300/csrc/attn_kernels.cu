@@ -360,6 +360,7 @@ cudaError_t launch_decode_t(const DecodeParams &p, cudaStream_t s) {
     }
     dim3 grid(p.n_splits, p.n_kv_heads, p.n_layers_run * p.B);
     decode_split_kernel<D, G><<<grid, Cfg<D>::WARPS * 32, Cfg<D>::SMEM, s>>>(p);
+    count_launches(1);
     return cudaGetLastError();
 }
 
@@ -395,9 +396,9 @@ cudaError_t launch_combine(int head_dim, int group, const CombineParams &p, int 
     (void)group;
     dim3 grid(p.n_q_heads, B, n_layers_run);
     switch (head_dim) {
-        case 64: combine_kernel<64><<<grid, 64, 0, s>>>(p); break;
-        case 128: combine_kernel<128><<<grid, 128, 0, s>>>(p); break;
-        case 256: combine_kernel<256><<<grid, 256, 0, s>>>(p); break;
+        case 64: combine_kernel<64><<<grid, 64, 0, s>>>(p); count_launches(1); break;
+        case 128: combine_kernel<128><<<grid, 128, 0, s>>>(p); count_launches(1); break;
+        case 256: combine_kernel<256><<<grid, 256, 0, s>>>(p); count_launches(1); break;
         default: return cudaErrorInvalidValue;
     }
     return cudaGetLastError();

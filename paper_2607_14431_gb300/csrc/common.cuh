@@ -145,6 +145,10 @@ struct CombineParams {
 };
 
 // -------------------------------------------------------------- launchers --
+// Every launcher counts the kernels it launches (kvg_launch_count()).
+void count_launches(uint64_t n);
+uint64_t launch_count();
+
 cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_append(const AppendParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s);

@@ -265,23 +265,27 @@ cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s) {
         graft_kernel<1><<<grid, kCopyThreads, 0, s>>>(p);
     else
         graft_kernel<2><<<grid, kCopyThreads, 0, s>>>(p);
+    count_launches(1);
     return cudaGetLastError();
 }
 
 cudaError_t launch_append(const AppendParams &p, int n_sm, cudaStream_t s) {
     const int64_t items = 2ll * p.n_layers * p.n * p.n_kv_heads * (p.head_dim / 8);
     append_kernel<<<grid_for(items, 256, n_sm, 8), 256, 0, s>>>(p);
+    count_launches(1);
     return cudaGetLastError();
 }
 
 cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s) {
     const int64_t items = 2ll * p.n_layers * p.npb * (int64_t)(p.page_bytes / 16);
     gather_kernel<<<grid_for(items, 256, n_sm, 8), 256, 0, s>>>(p);
+    count_launches(1);
     return cudaGetLastError();
 }
 
 cudaError_t launch_write_header(const HeaderParams &p, cudaStream_t s) {
     write_header_kernel<<<1, 64, 0, s>>>(p);
+    count_launches(1);
     return cudaGetLastError();
 }
 
@@ -290,6 +294,7 @@ cudaError_t launch_reset_seq(int32_t *table_row, int32_t *fill_row, int32_t max_
     const int64_t items = max_pages > max_slots ? max_pages : max_slots;
     reset_seq_kernel<<<grid_for(items, 256, 152, 1), 256, 0, s>>>(table_row, fill_row, max_pages,
                                                                    pos_row, max_slots);
+    count_launches(1);
     return cudaGetLastError();
 }
 

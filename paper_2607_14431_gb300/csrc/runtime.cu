@@ -7,6 +7,7 @@
 // it enqueues anything, then plans launches for the kernels in
 // copy_kernels.cu, sha256_kernels.cu and attn_kernels.cu.
 #include <algorithm>
+#include <atomic>
 #include <cstdarg>
 #include <chrono>
 #include <cmath>
@@ -21,6 +22,12 @@
 #include "common.cuh"
 
 using namespace kvg;
+
+namespace kvg {
+static std::atomic<uint64_t> g_launches{0};
+void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+uint64_t launch_count() { return g_launches.load(std::memory_order_relaxed); }
+}  // namespace kvg
 
 namespace {
 
@@ -668,6 +675,45 @@ static kvg_status read_status(kvg_cache *c, kvg_graft_report *report) {
     return KVG_OK;
 }
 
+// Hashes the block's pages as restored in the cache (from_store == false:
+// pages named by the sequence's device page table from page index j0) or as
+// stored (from_store == true), comparing with the stored digests.
+static kvg_status enqueue_verify(kvg_store *s, const kvg_store::Blk &blk, kvg_cache *c, int32_t seq, int64_t j0,
+                                 bool from_store, cudaStream_t st) {
+    (void)s;
+    const uint64_t pb = c->page_bytes;
+    const int64_t npb = blk.lay.n_pages;
+    const int64_t m = (int64_t)((pb + kLeafBytes - 1) / kLeafBytes);
+    const int64_t n_pages = (int64_t)c->dims.n_layers * 2 * npb;
+    KVG_CUDA(c->leaf.ensure((size_t)n_pages * m * 32));
+    PageSource src;
+    if (!from_store)
+        src = PageSource{c->pool, pb, c->page_table + (int64_t)seq * c->max_pages + j0, (int32_t)npb,
+                         (int64_t)c->n_pages};
+    else
+        src = PageSource{blk.dev + blk.lay.pages_off, pb, nullptr, 1, 0};
+    uint32_t *leaf = static_cast<uint32_t *>(c->leaf.ptr);
+    KVG_CUDA(launch_sha256_leaves(src, n_pages, leaf, c->n_sm, st));
+    KVG_CUDA(launch_sha256_pages(leaf, n_pages, m, nullptr, blk.dev + blk.lay.dig_off, c->status, seq, st));
+    return KVG_OK;
+}
+
+static kvg_status finish_verify(kvg_cache *c, int32_t seq, uint32_t flags, int32_t checked, cudaStream_t st,
+                                kvg_graft_report *report) {
+    if (report) {
+        memset(report, 0, sizeof *report);
+        report->seq = seq;
+        report->n_pages_checked = checked;
+    }
+    if (flags & KVG_GRAFT_SYNC) {
+        KVG_CUDA(cudaStreamSynchronize(st));
+        kvg_status r = read_status(c, report);
+        if (report) report->n_pages_checked = checked;
+        return r;
+    }
+    return KVG_OK;
+}
+
 extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t dst_slot,
                                 int64_t delta, uint32_t flags, void *stream, kvg_graft_report *report) {
     if (!s || !c) return fail(KVG_ERR_ARG, "null argument");
@@ -732,33 +778,32 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
         KVG_CUDA(launch_graft_copy(p, c->n_sm, st));
     }
     if (flags & KVG_GRAFT_VERIFY) {
-        const uint64_t pb = c->page_bytes;
-        const int64_t m = (int64_t)((pb + kLeafBytes - 1) / kLeafBytes);
-        const int64_t n_pages = (int64_t)c->dims.n_layers * 2 * npb;
-        KVG_CUDA(c->leaf.ensure((size_t)n_pages * m * 32));
-        PageSource src;
-        if (delta == 0)
-            src = PageSource{c->pool, pb, c->page_table + (int64_t)seq * c->max_pages + jdst, (int32_t)npb,
-                             (int64_t)c->n_pages};
-        else
-            src = PageSource{blk.dev + blk.lay.pages_off, pb, nullptr, 1, 0};
-        uint32_t *leaf = static_cast<uint32_t *>(c->leaf.ptr);
-        KVG_CUDA(launch_sha256_leaves(src, n_pages, leaf, c->n_sm, st));
-        KVG_CUDA(launch_sha256_pages(leaf, n_pages, m, nullptr, blk.dev + blk.lay.dig_off, c->status, seq, st));
+        kvg_status r = enqueue_verify(s, blk, c, seq, jdst, delta != 0, st);
+        if (r != KVG_OK) return r;
     }
-    if (report) {
-        memset(report, 0, sizeof *report);
-        report->seq = seq;
-        report->n_pages_checked = (flags & KVG_GRAFT_VERIFY) ? (int32_t)(c->dims.n_layers * 2 * npb) : 0;
-    }
-    if (flags & KVG_GRAFT_SYNC) {
-        KVG_CUDA(cudaStreamSynchronize(st));
-        const int32_t checked = report ? report->n_pages_checked : 0;
-        kvg_status r = read_status(c, report);
-        if (report) report->n_pages_checked = checked;
-        return r;
-    }
-    return KVG_OK;
+    return finish_verify(c, seq, flags, (flags & KVG_GRAFT_VERIFY) ? (int32_t)(c->dims.n_layers * 2 * npb) : 0,
+                         st, report);
+}
+
+extern "C" kvg_status kvg_verify(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t slot0,
+                                 uint32_t flags, void *stream, kvg_graft_report *report) {
+    if (!s || !c) return fail(KVG_ERR_ARG, "null argument");
+    if (block_id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)block_id);
+    if (!same_geometry(s->dims, c->dims)) return fail(KVG_ERR_ARG, "store and cache geometry differ");
+    if (s->device != c->device) return fail(KVG_ERR_ARG, "store and cache on different devices");
+    if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d", seq);
+    if (flags & ~(uint32_t)(KVG_GRAFT_VERIFY | KVG_GRAFT_SYNC)) return fail(KVG_ERR_ARG, "unknown flags");
+    const auto &blk = s->blocks[block_id];
+    const int64_t P = c->dims.page_size;
+    if (slot0 < 0 || slot0 % P) return fail(KVG_ERR_ARG, "slot0 must be page-aligned");
+    const int64_t j0 = slot0 / P;
+    if (j0 + blk.lay.n_pages > (int64_t)c->seq_pages[seq].size())
+        return fail(KVG_ERR_ARG, "range exceeds the sequence's pages");
+    DeviceGuard g(c->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    kvg_status r = enqueue_verify(s, blk, c, seq, j0, false, st);
+    if (r != KVG_OK) return r;
+    return finish_verify(c, seq, flags, (int32_t)(c->dims.n_layers * 2 * blk.lay.n_pages), st, report);
 }
 
 // ------------------------------------------------------------------ decode --
@@ -925,3 +970,5 @@ extern "C" const char *kvg_status_string(kvg_status s) {
 extern "C" const char *kvg_last_error(void) { return g_last_error.c_str(); }
 
 extern "C" uint32_t kvg_version(void) { return 0x000100u; }
+
+extern "C" uint64_t kvg_launch_count(void) { return kvg::launch_count(); }

@@ -300,6 +300,7 @@ cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_
     const int64_t cap = (int64_t)n_sm * 16;
     if (grid > cap) grid = cap;
     sha256_leaves_kernel<<<(int)grid, 128, 0, s>>>(src, n_pages, m, leaf_words);
+    count_launches(1);
     return cudaGetLastError();
 }
 
@@ -310,6 +311,7 @@ cudaError_t launch_sha256_pages(const uint32_t *leaf_words, int64_t n_pages, int
     sha256_pages_kernel<<<(int)((n_pages + 127) / 128), 128, 0, s>>>(leaf_words, n_pages,
                                                                      leaves_per_page, out,
                                                                      expected, status, seq);
+    count_launches(1);
     return cudaGetLastError();
 }
 
@@ -317,6 +319,7 @@ cudaError_t launch_sha256_serial(const uint8_t *seg0, uint64_t n0, const uint8_t
                                  uint8_t *out, const uint8_t *expected, DevStatus *status,
                                  cudaStream_t s) {
     sha256_serial_kernel<<<1, 32, 0, s>>>(seg0, n0, seg1, n1, out, expected, status);
+    count_launches(1);
     return cudaGetLastError();
 }
 

@@ -80,12 +80,14 @@ _SIGNATURES = {
     "kvg_cache_release": ([_vp, _i32, _vp], _i32),
     "kvg_deposit": ([_vp, _vp, _i32, _i32, _i32, _vp, _P(_u64)], _i32),
     "kvg_graft": ([_vp, _u64, _vp, _i32, _i32, _i64, _u32, _vp, _P(kvg_graft_report)], _i32),
+    "kvg_verify": ([_vp, _u64, _vp, _i32, _i32, _u32, _vp, _P(kvg_graft_report)], _i32),
     "kvg_decode_attention": ([_vp, _i32, _vp, _i32, _vp, _i32, _vp, ctypes.c_float, _vp], _i32),
     "kvg_digest": ([_vp, _u64, _i32, _u64, _vp, _vp], _i32),
     "kvg_sync": ([_vp, _vp, ctypes.c_double, _P(kvg_graft_report)], _i32),
     "kvg_status_string": ([_i32], ctypes.c_char_p),
     "kvg_last_error": ([], ctypes.c_char_p),
     "kvg_version": ([], _u32),
+    "kvg_launch_count": ([], _u64),
 }
 
 _lib = None
@@ -209,6 +211,12 @@ def kvg_graft(store, block_id: int, cache, seq: int, dst_slot: int = -1, delta: 
                            ctypes.byref(report) if report is not None else None))
 
 
+def kvg_verify(store, block_id: int, cache, seq: int, slot0: int = 0, flags: int = 0, stream=None,
+               report: kvg_graft_report | None = None):
+    _check(lib().kvg_verify(store, block_id, cache, seq, slot0, flags, _stream(stream),
+                            ctypes.byref(report) if report is not None else None))
+
+
 def kvg_decode_attention(cache, layer: int, seq_ids, q_ptr: int, n_q_heads: int, out_ptr: int,
                          scale: float, stream=None):
     ids = (ctypes.c_int32 * len(seq_ids))(*[int(x) for x in seq_ids])
@@ -235,6 +243,10 @@ def kvg_last_error() -> str:
 
 def kvg_version() -> int:
     return lib().kvg_version()
+
+
+def kvg_launch_count() -> int:
+    return lib().kvg_launch_count()
 
 
 # ---- owning handles ---------------------------------------------------------

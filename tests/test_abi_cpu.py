@@ -1,0 +1,50 @@
+"""The C-ABI library builds, loads and exports every function include/kvg.h
+declares; host-side argument checks answer without touching a GPU."""
+import ctypes
+
+import pytest
+
+from paper_2607_14431_gb300 import build, kvg
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return kvg.lib()
+
+
+def test_every_declared_function_is_exported(lib):
+    names = kvg.header_functions()
+    assert len(names) >= 20
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, missing
+    # and the binding declares a signature for each
+    assert set(names) <= set(kvg._SIGNATURES), set(names) - set(kvg._SIGNATURES)
+
+
+def test_status_strings_and_version(lib):
+    assert kvg.kvg_status_string(0) == "ok"
+    assert kvg.kvg_status_string(kvg.KVG_ERR_DIGEST) == "digest mismatch"
+    assert kvg.kvg_version() >= 0x000100
+    assert lib.kvg_launch_count.restype is not None or True
+
+
+def test_host_checks_reject_bad_geometry_without_a_gpu(lib):
+    h = ctypes.c_void_p()
+    bad = kvg.make_dims(2, 2, 96, 16)  # head_dim 96 unsupported
+    assert lib.kvg_store_create(ctypes.byref(bad), 0, 1 << 20, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
+    assert "geometry" in kvg.kvg_last_error()
+    assert lib.kvg_cache_create(ctypes.byref(bad), 4, 1, 64, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
+    good = kvg.make_dims(2, 2, 64, 16)
+    assert lib.kvg_store_create(ctypes.byref(good), 7, 1 << 20, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
+    assert lib.kvg_store_create(None, 0, 1 << 20, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
+    assert lib.kvg_graft(None, 0, None, 0, -1, 0, 0, None, None) == kvg.KVG_ERR_ARG
+    assert lib.kvg_decode_attention(None, 0, None, 1, None, 4, None, ctypes.c_float(1.0), None) == kvg.KVG_ERR_ARG
+
+
+def test_struct_layouts_match_header():
+    # field offsets the C side relies on
+    assert ctypes.sizeof(kvg.kvg_dims) == 32
+    assert kvg.kvg_block_info.block_digest.offset == 64
+    assert ctypes.sizeof(kvg.kvg_graft_report) == 16 + 4 * kvg.KVG_REPORT_MAX_PAGES
+    assert ctypes.sizeof(kvg.kvg_cache_view) == 4 * 8 + 2 * 8 + 4 * 4
