@@ -268,6 +268,34 @@ kvg_status kvg_decode_attention(kvg_cache *cache, int32_t layer, const int32_t *
                                 int32_t B, const void *q, int32_t n_q_heads, void *out,
                                 float scale, void *stream);
 
+/* The same decode attention, for callers that cannot allocate GPU memory.
+ * (The paper has no counterpart: this is a deployment variant.)
+ * kvg_decode_attention() grows per-cache scratch for its split-K partial
+ * results with cudaMalloc when a call first needs it; cudaMalloc/cudaFree
+ * synchronise the whole device and can fail once another allocator has
+ * reserved the memory, which latency-bound serving loops and processes with a
+ * fixed memory footprint cannot accept.  This entry point instead keeps the
+ * partials in one file-scope device array of 16 MiB that every GPU loading
+ * the library holds until the process exits, and calls no allocating routine
+ * (no cudaMalloc, cudaFree or library allocator).  Arguments, results and
+ * errors are those of kvg_decode_attention, with these differences:
+ *   - the split plan is capped so the partials fit the array; a call whose
+ *     partials would not fit even unsplit (n_layers_run * min(B, 256) *
+ *     n_q_heads * (4 * head_dim + 8) bytes > 16 MiB - 256) returns
+ *     KVG_ERR_CAPACITY with an explanatory kvg_last_error() and enqueues
+ *     nothing;
+ *   - the first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); make that first call
+ *     before any stream capture;
+ *   - every call on a device shares the one array, and the array keeps the
+ *     previous call's contents (each partial the call reads is first written
+ *     by the same call, so nothing needs clearing): calls whose GPU work
+ *     overlaps in time, on different streams or from different threads, race
+ *     and give wrong results.  Serialise them (one stream, or events). */
+kvg_status kvg_decode_attention_noalloc(kvg_cache *cache, int32_t layer, const int32_t *seq_ids,
+                                        int32_t B, const void *q, int32_t n_q_heads, void *out,
+                                        float scale, void *stream);
+
 /* ------------------------------------------------------------- digest -- */
 
 /* SHA-256 (FIPS 180-4) on the GPU.

@@ -969,6 +969,25 @@ extern "C" const char *kvg_status_string(kvg_status s) {
 
 extern "C" const char *kvg_last_error(void) { return g_last_error.c_str(); }
 
+namespace kvg {
+// Read-only views used by noalloc.cu.
+struct CacheShape {
+    int32_t n_layers, n_kv_heads, head_dim, page_size, n_pages, max_seqs, max_pages, device, n_sm;
+    uint8_t *pool;
+    int32_t *page_table, *page_fill;
+    DevStatus *status;
+};
+bool cache_shape(const kvg_cache *c, CacheShape *out) {
+    if (!c || !out) return false;
+    *out = CacheShape{c->dims.n_layers, c->dims.n_kv_heads, c->dims.head_dim, c->dims.page_size, c->n_pages,
+                      c->max_seqs, c->max_pages, c->device, c->n_sm, c->pool, c->page_table, c->page_fill,
+                      c->status};
+    return true;
+}
+int32_t cache_seq_pages(const kvg_cache *c, int32_t seq) { return (int32_t)c->seq_pages[seq].size(); }
+void set_last_error(const char *msg) { g_last_error = msg; }
+}  // namespace kvg
+
 extern "C" uint32_t kvg_version(void) { return 0x000100u; }
 
 extern "C" uint64_t kvg_launch_count(void) { return kvg::launch_count(); }

@@ -82,6 +82,7 @@ _SIGNATURES = {
     "kvg_graft": ([_vp, _u64, _vp, _i32, _i32, _i64, _u32, _vp, _P(kvg_graft_report)], _i32),
     "kvg_verify": ([_vp, _u64, _vp, _i32, _i32, _u32, _vp, _P(kvg_graft_report)], _i32),
     "kvg_decode_attention": ([_vp, _i32, _vp, _i32, _vp, _i32, _vp, ctypes.c_float, _vp], _i32),
+    "kvg_decode_attention_noalloc": ([_vp, _i32, _vp, _i32, _vp, _i32, _vp, ctypes.c_float, _vp], _i32),
     "kvg_digest": ([_vp, _u64, _i32, _u64, _vp, _vp], _i32),
     "kvg_sync": ([_vp, _vp, ctypes.c_double, _P(kvg_graft_report)], _i32),
     "kvg_status_string": ([_i32], ctypes.c_char_p),
@@ -222,6 +223,14 @@ def kvg_decode_attention(cache, layer: int, seq_ids, q_ptr: int, n_q_heads: int,
     ids = (ctypes.c_int32 * len(seq_ids))(*[int(x) for x in seq_ids])
     _check(lib().kvg_decode_attention(cache, layer, ids, len(seq_ids), q_ptr, n_q_heads, out_ptr,
                                       float(scale), _stream(stream)))
+
+
+def kvg_decode_attention_noalloc(cache, layer: int, seq_ids, q_ptr: int, n_q_heads: int, out_ptr: int,
+                                 scale: float, stream=None):
+    """kvg_decode_attention without any GPU allocation (static scratch; see kvg.h)."""
+    ids = (ctypes.c_int32 * len(seq_ids))(*[int(x) for x in seq_ids])
+    _check(lib().kvg_decode_attention_noalloc(cache, layer, ids, len(seq_ids), q_ptr, n_q_heads, out_ptr,
+                                              float(scale), _stream(stream)))
 
 
 def kvg_digest(ptr: int, n: int, mode: int, page_bytes: int, out_ptr: int, stream=None):
