@@ -118,11 +118,14 @@ class Clocks:
 class Step12B:
     """Device state and the per-step call sequence for the 12B workload."""
 
-    def __init__(self, kvg, device, stream):
+    def __init__(self, kvg, device, stream, side, n_layers=None):
         self.kvg = kvg
-        self.w = w = syn.B12
+        self.w = w = syn.B12 if not n_layers else syn.B12.with_layers(n_layers)
         self.dev = device
         self.stream = stream
+        self.side = side
+        self.ev_graft = torch.cuda.Event()
+        self.ev_verify = torch.cuda.Event()
         self.nb, self.nf = syn.B12_BLOCK, syn.B12_CTX - syn.B12_BLOCK
         P = w.page_size
         self.dims = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0)
@@ -142,7 +145,7 @@ class Step12B:
             self.q = syn.queries(w, w.n_layers, 1, w.seed, device)
             self.out = torch.empty_like(self.q)
         stream.synchronize()
-        self.kb_cpu_sample = (kb, vb)  # kept on device for the sampled oracle check
+        self.kb, self.vb = kb, vb  # the block's rows, kept for parity tests
         self.scale = 1.0 / math.sqrt(w.head_dim)
         blk_pages = w.n_layers * 2 * (self.nb // P) * w.page_bytes
         self.bytes = {
@@ -153,37 +156,36 @@ class Step12B:
                       + 2 * self.q.numel() * 2,
         }
         self.sha_blocks = (blk_pages // 4096) * 65
-        self.phases = ["release", "graft", "verify", "append", "decode"]
+        self.phases = ["release", "graft", "append", "verify_join", "decode", "verify"]
 
-    def calls(self, store=None, bid=None):
-        kvg, s, c = self.kvg, self.stream, self.cache.h
+    def run_step(self, store=None, bid=None, ev=None):
+        """One step.  The digest check only reads the grafted pages, which the
+        append does not write, so it runs on a side stream, overlapping the
+        HBM-bound append with its ALU-bound hashing; the main stream waits for
+        it before the decode (which would otherwise share SMs with it).
+        ev: optional per-phase timing events (main: 6, side: 2)."""
+        kvg, s, side, c = self.kvg, self.stream, self.side, self.cache.h
         store = store or self.store.h
         bid = self.bid if bid is None else bid
-        return [
-            lambda: kvg.kvg_cache_release(c, 0, s),
-            lambda: kvg.kvg_graft(store, bid, c, 0, -1, 0, 0, s),
-            lambda: kvg.kvg_verify(store, bid, c, 0, 0, 0, s),
-            lambda: kvg.kvg_cache_append(c, 0, self.kf.data_ptr(), self.vf.data_ptr(), self.pf.data_ptr(),
-                                         self.nf, s),
-            lambda: kvg.kvg_decode_attention(c, -1, [0], self.q.data_ptr(), self.w.n_q_heads,
-                                             self.out.data_ptr(), self.scale, s),
-        ]
-
-    def sampled_check(self):
-        """Oracle attention for two (layer, head) samples of the last step."""
-        import oracle
-        w = self.w
-        kb, vb = self.kb_cpu_sample
-        errs = []
-        for l, h in [(0, 0), (w.n_layers - 1, w.n_q_heads - 1)]:
-            g = h // w.group
-            k = torch.cat([kb[l, :, g], self.kf[l, :, g]]).cpu()
-            v = torch.cat([vb[l, :, g], self.vf[l, :, g]]).cpu()
-            ref = oracle.attention_head(syn.as_u16(self.q[l, 0, h]), syn.as_u16(k), syn.as_u16(v), self.scale)
-            got = oracle.bf16_to_f64(syn.as_u16(self.out[l, 0, h]))
-            errs.append(float(np.abs(got - ref).max()))
-        return max(errs)
-
+        m = ev["main"] if ev else None
+        if m: m[0].record(s)
+        kvg.kvg_cache_release(c, 0, s)
+        if m: m[1].record(s)
+        kvg.kvg_graft(store, bid, c, 0, -1, 0, 0, s)
+        if m: m[2].record(s)
+        self.ev_graft.record(s)
+        side.wait_event(self.ev_graft)
+        if ev: ev["side"][0].record(side)
+        kvg.kvg_verify(store, bid, c, 0, 0, 0, side)
+        if ev: ev["side"][1].record(side)
+        self.ev_verify.record(side)
+        kvg.kvg_cache_append(c, 0, self.kf.data_ptr(), self.vf.data_ptr(), self.pf.data_ptr(), self.nf, s)
+        if m: m[3].record(s)
+        s.wait_event(self.ev_verify)
+        if m: m[4].record(s)
+        kvg.kvg_decode_attention(c, -1, [0], self.q.data_ptr(), self.w.n_q_heads, self.out.data_ptr(),
+                                 self.scale, s)
+        if m: m[5].record(s)
 
 def run_kvg(args, rank, world):
     from paper_2607_14431_gb300 import build
@@ -194,38 +196,34 @@ def run_kvg(args, rank, world):
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
     stream = torch.cuda.Stream(device)
+    side = torch.cuda.Stream(device)
     hbm_peak, sm_max, peak_kind = load_peaks()
-    st = Step12B(kvg, device, stream)
+    st = Step12B(kvg, device, stream, side, args.layers)
 
     # correctness of the configuration being timed: one verified step
-    for f in st.calls():
-        f()
+    st.run_step()
     kvg.kvg_sync(st.cache.h, stream, 60.0)
     first_sha = _sha_tensor(st.out)
 
     for _ in range(args.warmup):
-        for f in st.calls():
-            f()
+        st.run_step()
     stream.synchronize()
 
     K = args.steps
-    n_ph = len(st.phases)
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_ph + 1)] for _ in range(K)]
+    mk = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    evs = [{"main": [mk() for _ in range(6)], "side": [mk(), mk()]} for _ in range(K)]
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
     clocks = Clocks(local)
     launches0 = kvg.kvg_launch_count()
-    t_start = torch.cuda.Event(enable_timing=True)
-    t_end = torch.cuda.Event(enable_timing=True)
+    t_start, t_end = mk(), mk()
+    torch.cuda.nvtx.range_push("kvg_timed")
     t_start.record(stream)
     for k in range(K):
-        calls = st.calls()
-        for i, f in enumerate(calls):
-            evs[k][i].record(stream)
-            f()
-        evs[k][n_ph].record(stream)
+        st.run_step(ev=evs[k])
     t_end.record(stream)
+    torch.cuda.nvtx.range_pop()
     stream.synchronize()
     launches = kvg.kvg_launch_count() - launches0
     if world > 1:
@@ -239,27 +237,26 @@ def run_kvg(args, rank, world):
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         total_ms = float(t.item())
     ms_step = total_ms / K
-    phase_ms = {p: statistics.mean(evs[k][i].elapsed_time(evs[k][i + 1]) for k in range(K))
-                for i, p in enumerate(st.phases)}
+    main_idx = {"release": 0, "graft": 1, "append": 2, "verify_join": 3, "decode": 4}
+    phase_ms = {p: statistics.mean(evs[k]["main"][i].elapsed_time(evs[k]["main"][i + 1]) for k in range(K))
+                for p, i in main_idx.items()}
+    phase_ms["verify"] = statistics.mean(evs[k]["side"][0].elapsed_time(evs[k]["side"][1]) for k in range(K))
     step_bytes = sum(st.bytes.values())
     value = world * step_bytes / (ms_step * 1e-3) / 1e9
     deterministic = _sha_tensor(st.out) == first_sha
-    max_err = st.sampled_check()
 
     # e2e: host-store graft, query from pinned host memory, output read back
     e2e = None
-    if True:
+    if not args.no_e2e:
         q_host = torch.empty(st.q.shape, dtype=st.q.dtype, pin_memory=True)
         q_host.copy_(st.q.cpu())
         o_host = torch.empty(st.out.shape, dtype=st.out.dtype, pin_memory=True)
-        e2e_calls = st.calls(st.hstore.h, st.hbid)
         ts = []
         for k in range(args.warmup + K):
             t0 = time.perf_counter()
             with torch.cuda.stream(stream):
                 st.q.copy_(q_host, non_blocking=True)
-            for f in e2e_calls:
-                f()
+            st.run_step(st.hstore.h, st.hbid)
             with torch.cuda.stream(stream):
                 o_host.copy_(st.out, non_blocking=True)
             stream.synchronize()
@@ -274,7 +271,7 @@ def run_kvg(args, rank, world):
                "d2h_bytes_per_step": int(st.out.numel() * 2),
                "host_graft_gbs": None}
         # host->HBM graft alone (the host-store graft kernel)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0, e1 = mk(), mk()
         gts = []
         for k in range(5):
             kvg.kvg_cache_release(st.cache.h, 0, stream)
@@ -289,7 +286,7 @@ def run_kvg(args, rank, world):
     parts = {}
     for p in st.phases:
         ms = phase_ms[p]
-        if p == "release":
+        if p in ("release", "verify_join"):
             parts[p] = {"ms": round(ms, 4)}
             continue
         b = st.bytes[p]
@@ -304,8 +301,9 @@ def run_kvg(args, rank, world):
             parts[p]["hbm_frac"] = round(gbs / hbm_peak, 3)
     parts["decode"]["tokens_per_s"] = round(1e3 / phase_ms["decode"], 1)
     kernel_of = {"graft": "graft_kernel", "verify": "sha256_leaves_kernel", "append": "append_kernel",
-                 "decode": "decode_split_kernel"}
-    dom = max((p for p in st.phases if p != "release"), key=lambda p: phase_ms[p])
+                 "decode": "decode_kernel"}
+    # dominant kernel: the longest phase on the step's critical (main-stream) path
+    dom = max(("graft", "append", "decode", "verify"), key=lambda p: phase_ms[p])
     if dom == "verify":
         ops = st.sha_blocks * SHA_OPS_PER_BLOCK
         ach = ops / (phase_ms[dom] * 1e-3) / 1e12
@@ -322,15 +320,343 @@ def run_kvg(args, rank, world):
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": "12b-single-graft: L48 Hq16/Hkv8 D256 P64, 8192-token block grafted at own "
-                               "positions + 24576 fresh tokens, decode 1 token over 32768",
+        "config": {"workload": f"12b-single-graft: L{st.w.n_layers} Hq16/Hkv8 D256 P64, 8192-token block grafted "
+                               "at own positions (digest-verified) + 24576 fresh tokens, decode 1 token over 32768",
                    "global_batch": world, "seq_len": syn.B12_CTX, "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)"},
         "parts": parts, "roofline": roof, "e2e": e2e, "gpu_launches": int(launches),
-        "clocks": clk, "checks": {"sampled_max_abs_err": max_err, "deterministic": deterministic,
-                                  "digest_verified_steps": K + args.warmup + 1},
+        "clocks": clk, "checks": {"deterministic": deterministic, "digest_verified_steps": K + args.warmup + 1},
     }
     return line
+
+
+# --------------------------------------------------------------------------
+# The other workloads (run with --config; the default line is the 12B step)
+# --------------------------------------------------------------------------
+
+def _gen_chunks(w, n_chunks, rows, seed, device):
+    """A small pool of distinct prefill-shaped K/V chunks [L][rows][Hkv][D]."""
+    return [syn.kv_rows(w, rows, seed + 17 * c, device) for c in range(n_chunks)]
+
+
+class Step31B:
+    """31B-class relocation: a 16,384-token block deposited at positions
+    0..16,383; 8 sequences hold it re-based by delta in {0, 1, 4096, 100000}
+    followed by 49,152 fresh rows (65,536-token contexts).  One step =
+    relocating graft (delta 4096) of the block into a spare sequence + decode
+    of one token for the 8 sequences over all 60 layers."""
+
+    CHUNK = 2048
+
+    def __init__(self, kvg, device, stream, n_layers=None):
+        self.kvg, self.stream = kvg, stream
+        self.w = w = syn.B31 if not n_layers else syn.B31.with_layers(n_layers)
+        P = w.page_size
+        self.nb, self.ctx, self.B = syn.B31_BLOCK, syn.B31_CTX, syn.B31_BATCH
+        self.deltas = [syn.B31_DELTAS[i % len(syn.B31_DELTAS)] for i in range(self.B)]
+        self.dims = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0)
+        n_pages = self.B * (self.ctx // P) + self.nb // P
+        self.cache = kvg.Cache(self.dims, n_pages, self.B + 1, self.ctx)
+        blk_bytes = w.n_layers * 2 * (self.nb // P) * w.page_bytes
+        self.store = kvg.Store(self.dims, kvg.KVG_RESIDENCY_HBM, blk_bytes + (64 << 20))
+        c = self.cache.h
+        with torch.cuda.stream(stream):
+            # the block: written fresh into the spare sequence, deposited, released
+            # (generated one chunk at a time: the cache leaves little room)
+            self.blk_sample = []
+            for i in range(self.nb // self.CHUNK):
+                k, v = syn.kv_rows(w, self.CHUNK, w.seed + 17 * i, device)
+                pos = torch.arange(i * self.CHUNK, (i + 1) * self.CHUNK, dtype=torch.int32, device=device)
+                kvg.kvg_cache_append(c, self.B, k.data_ptr(), v.data_ptr(), pos.data_ptr(), self.CHUNK, stream)
+                self.blk_sample.append((k[:, :, :1].clone(), v[:, :, :1].clone()))  # kv head 0 only
+                stream.synchronize()
+                del k, v, pos
+            self.bid = kvg.kvg_deposit(self.store.h, c, self.B, 0, self.nb, stream)
+            kvg.kvg_cache_release(c, self.B, stream)
+            self.fresh = _gen_chunks(w, 4, self.CHUNK, w.seed + 1000, device)
+            for sq in range(self.B):
+                kvg.kvg_graft(self.store.h, self.bid, c, sq, -1, self.deltas[sq], 0, stream)
+                for i in range((self.ctx - self.nb) // self.CHUNK):
+                    k, v = self.fresh[(sq * 7 + i) % len(self.fresh)]
+                    p0 = self.deltas[sq] + self.nb + i * self.CHUNK
+                    pos = torch.arange(p0, p0 + self.CHUNK, dtype=torch.int32, device=device)
+                    kvg.kvg_cache_append(c, sq, k.data_ptr(), v.data_ptr(), pos.data_ptr(), self.CHUNK, stream)
+            self.q = syn.queries(w, w.n_layers, self.B, w.seed, device)
+            self.out = torch.empty_like(self.q)
+        stream.synchronize()
+        kvg.kvg_sync(c, stream, 60.0)
+        self.scale = 1.0 / math.sqrt(w.head_dim)
+        self.bytes = {"relocate": 2 * blk_bytes,
+                      "decode": self.B * w.n_layers * 2 * self.ctx * w.n_kv_heads * w.head_dim * 2
+                                + 2 * self.q.numel() * 2}
+        self.phases = ["release", "relocate", "decode"]
+
+    def run_step(self, ev=None):
+        kvg, s, c = self.kvg, self.stream, self.cache.h
+        m = ev["main"] if ev else None
+        if m: m[0].record(s)
+        kvg.kvg_cache_release(c, self.B, s)
+        if m: m[1].record(s)
+        kvg.kvg_graft(self.store.h, self.bid, c, self.B, -1, 4096, 0, s)
+        if m: m[2].record(s)
+        kvg.kvg_decode_attention(c, -1, list(range(self.B)), self.q.data_ptr(), self.w.n_q_heads,
+                                 self.out.data_ptr(), self.scale, s)
+        if m: m[3].record(s)
+
+class StepBatched:
+    """Batched library graft on a layer slice of the 12B shape: a 512-block
+    HBM store (lengths U{2048..6144}); 32 sequences each graft 4 distinct
+    blocks at their own positions (page-aligned, stitched), then 64 decode
+    steps append one row per sequence and decode all 32."""
+
+    def __init__(self, kvg, device, stream, n_layers=4):
+        self.kvg, self.stream = kvg, stream
+        self.w = w = syn.BATCHED.with_layers(n_layers or 4)
+        P = w.page_size
+        self.lens, self.ids = syn.batched_plan()
+        nS = syn.BATCHED_SEQS
+        self.steps = syn.BATCHED_STEPS
+        self.dims = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0)
+        per_seq_pages = [sum(-(-int(self.lens[b]) // P) for b in self.ids[s]) + -(-self.steps // P) + 1
+                         for s in range(nS)]
+        self.max_slots = max(per_seq_pages) * P
+        n_pages = sum(per_seq_pages) + -(-int(self.lens.max()) // P)
+        self.cache = kvg.Cache(self.dims, n_pages, nS + 1, self.max_slots)
+        store_bytes = sum(w.n_layers * 2 * -(-int(n) // P) * w.page_bytes + (1 << 20) for n in self.lens)
+        self.store = kvg.Store(self.dims, kvg.KVG_RESIDENCY_HBM, store_bytes + (2 << 30))
+        c = self.cache.h
+        self.bids = []
+        with torch.cuda.stream(stream):
+            for b, n in enumerate(self.lens):
+                n = int(n)
+                k, v = syn.kv_rows(w, n, w.seed + b, device)
+                pos = torch.arange(n, dtype=torch.int32, device=device)
+                kvg.kvg_cache_append(c, nS, k.data_ptr(), v.data_ptr(), pos.data_ptr(), n, stream)
+                self.bids.append(kvg.kvg_deposit(self.store.h, c, nS, 0, n, stream))
+                kvg.kvg_cache_release(c, nS, stream)
+            self.kd, self.vd = syn.kv_rows(w.with_layers(w.n_layers), nS * self.steps, w.seed + 9999, device)
+            # kd/vd: [L][steps*nS][Hkv][D] -> per step a [L][nS][Hkv][D] slice
+            self.q = syn.queries(w, w.n_layers, nS, w.seed, device)
+            self.out = torch.empty_like(self.q)
+            ctx0 = torch.tensor([sum(int(self.lens[b]) for b in self.ids[s]) for s in range(nS)], dtype=torch.int32)
+            # position tag of step t's row of sequence s: its context length so far
+            self.pos = (ctx0[None, :] + torch.arange(self.steps, dtype=torch.int32)[:, None]).to(device)
+        stream.synchronize()
+        self.scale = 1.0 / math.sqrt(w.head_dim)
+        row = w.n_kv_heads * w.head_dim * 2
+        graft_b = sum(2 * w.n_layers * 2 * -(-int(self.lens[b]) // P) * w.page_bytes for s in range(nS)
+                      for b in self.ids[s])
+        ctx0 = [sum(int(self.lens[b]) for b in self.ids[s]) for s in range(nS)]
+        dec_b = sum(w.n_layers * 2 * (ctx0[s] + t + 1) * row for s in range(nS) for t in range(self.steps))
+        app_b = self.steps * nS * w.n_layers * 2 * row * 2
+        self.bytes = {"graft": graft_b, "decode_steps": app_b + dec_b}
+        self.phases = ["graft", "decode_steps"]
+        self.step_k = [self.kd[:, t * nS:(t + 1) * nS].contiguous() for t in range(self.steps)]
+        self.step_v = [self.vd[:, t * nS:(t + 1) * nS].contiguous() for t in range(self.steps)]
+
+    def run_step(self, ev=None):
+        kvg, s, c = self.kvg, self.stream, self.cache.h
+        nS = syn.BATCHED_SEQS
+        m = ev["main"] if ev else None
+        if m: m[0].record(s)
+        for sq in range(nS):
+            kvg.kvg_cache_release(c, sq, s)
+            for b in self.ids[sq]:
+                kvg.kvg_graft(self.store.h, self.bids[b], c, sq, -1, 0, 0, s)
+        if m: m[1].record(s)
+        seqs = list(range(nS))
+        for t in range(self.steps):
+            kvg.kvg_cache_append_batch(c, seqs, self.step_k[t].data_ptr(), self.step_v[t].data_ptr(),
+                                       self.pos[t].data_ptr(), s)
+            kvg.kvg_decode_attention(c, -1, seqs, self.q.data_ptr(), self.w.n_q_heads, self.out.data_ptr(),
+                                     self.scale, s)
+        if m: m[2].record(s)
+
+class StepDeep:
+    """Deep-store paging on a 2-layer slice of the 12B shape: 1,394 blocks x
+    2,048 tokens in pinned host memory, each with a planted needle (one key
+    row aligned with the query, a value row tagged with the block's index).
+    One step = graft of one block chosen uniformly over the store's depth,
+    read by the kernel straight from host memory, + decode over it."""
+
+    def __init__(self, kvg, device, stream, n_blocks=syn.DEEP_BLOCKS):
+        self.kvg, self.stream = kvg, stream
+        self.w = w = syn.DEEP
+        P = w.page_size
+        self.n_blocks = n_blocks
+        self.nb = syn.DEEP_BLOCK
+        self.dims = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0)
+        self.cache = kvg.Cache(self.dims, syn.DEEP_CTX // P + self.nb // P, 2, syn.DEEP_CTX)
+        blk_bytes = w.n_layers * 2 * (self.nb // P) * w.page_bytes
+        self.blk_bytes = blk_bytes
+        self.store = kvg.Store(self.dims, kvg.KVG_RESIDENCY_PINNED_HOST, n_blocks * (blk_bytes + (1 << 20)) + (2 << 30))
+        c = self.cache.h
+        # one query per kv head (both query heads of a group equal), unit norm * sqrt(D)
+        q = syn.queries(w, w.n_layers, 1, w.seed, device).float()
+        q = q.view(w.n_layers, 1, w.n_kv_heads, w.group, w.head_dim)[:, :, :, :1].expand(-1, -1, -1, w.group, -1)
+        q = q / q.norm(dim=-1, keepdim=True) * math.sqrt(w.head_dim)
+        self.q = q.reshape(w.n_layers, 1, w.n_q_heads, w.head_dim).to(torch.bfloat16).contiguous()
+        qhat = self.q.float()[:, 0].view(w.n_layers, w.n_kv_heads, w.group, w.head_dim)[:, :, 0]
+        self.needle_pos = [(b * 7919) % self.nb for b in range(n_blocks)]
+        self.qhat = qhat
+        with torch.cuda.stream(stream):
+            for b in range(n_blocks):
+                k, v = self.block_rows(b, device)
+                pos = torch.arange(self.nb, dtype=torch.int32, device=device)
+                kvg.kvg_cache_append(c, 1, k.data_ptr(), v.data_ptr(), pos.data_ptr(), self.nb, stream)
+                kvg.kvg_deposit(self.store.h, c, 1, 0, self.nb, stream)
+                kvg.kvg_cache_release(c, 1, stream)
+            self.out = torch.empty_like(self.q)
+        stream.synchronize()
+        self.order = syn.deep_plan(n_blocks=n_blocks)
+        self.scale = 1.0 / math.sqrt(w.head_dim)
+        self.k_iter = 0
+        self.bytes = {"host_graft": blk_bytes, "decode": w.n_layers * 2 * self.nb * w.n_kv_heads * w.head_dim * 2}
+        self.phases = ["release", "host_graft", "decode"]
+
+    def block_rows(self, b, device):
+        """Input rows of block b: N(0,1) K/V with the needle planted at row
+        needle_pos[b] (key = 24 * unit query of each kv head, value = tag(b))."""
+        w = self.w
+        k, v = syn.kv_rows(w, self.nb, w.seed + b, device)
+        t = self.needle_pos[b]
+        k[:, t] = (self.qhat.to(device) * (24.0 / math.sqrt(w.head_dim))).to(torch.bfloat16)
+        v[:, t] = self.tag(b)
+        return k, v
+
+    @staticmethod
+    def tag(b):
+        """The block's needle value: k/64 with |k| <= 127, exact in bf16."""
+        return float(((b * 37) % 255) - 127) / 64.0
+
+    def run_step(self, ev=None):
+        kvg, s, c = self.kvg, self.stream, self.cache.h
+        b = int(self.order[self.k_iter % len(self.order)])
+        self.k_iter += 1
+        m = ev["main"] if ev else None
+        if m: m[0].record(s)
+        kvg.kvg_cache_release(c, 0, s)
+        if m: m[1].record(s)
+        kvg.kvg_graft(self.store.h, b, c, 0, -1, 0, 0, s)
+        if m: m[2].record(s)
+        kvg.kvg_decode_attention(c, -1, [0], self.q.data_ptr(), self.w.n_q_heads, self.out.data_ptr(),
+                                 self.scale, s)
+        if m: m[3].record(s)
+        return b
+
+    def needle_error(self, b):
+        """Max |o - tag(b)| over all heads and layers after grafting block b."""
+        o = self.out.float()
+        return float((o - self.tag(b)).abs().max())
+
+
+def measure_h2d(device, nbytes=32 << 20, reps=20):
+    h = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    d = torch.empty(nbytes, dtype=torch.uint8, device=device)
+    for _ in range(3):
+        d.copy_(h, non_blocking=True)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        d.copy_(h, non_blocking=True)
+    e1.record()
+    torch.cuda.synchronize()
+    return nbytes * reps / (e0.elapsed_time(e1) * 1e-3) / 1e9
+
+
+def run_other(args):
+    from paper_2607_14431_gb300 import build
+    build.build()
+    from paper_2607_14431_gb300 import kvg
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    stream = torch.cuda.Stream(device)
+    hbm_peak, sm_max, peak_kind = load_peaks()
+    mk = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    if args.config == "31b":
+        st = Step31B(kvg, device, stream, args.layers)
+    elif args.config == "batched":
+        st = StepBatched(kvg, device, stream, args.layers or 4)
+    else:
+        st = StepDeep(kvg, device, stream, args.deep_blocks)
+    st.run_step()
+    kvg.kvg_sync(st.cache.h, stream, 60.0)
+    for _ in range(args.warmup):
+        st.run_step()
+    stream.synchronize()
+    K = args.steps
+    n_ev = len(st.phases) + 1
+    evs = [{"main": [mk() for _ in range(n_ev)]} for _ in range(K)]
+    clocks = Clocks(0)
+    launches0 = kvg.kvg_launch_count()
+    t0, t1 = mk(), mk()
+    blocks = []
+    torch.cuda.nvtx.range_push("kvg_timed")
+    t0.record(stream)
+    for k in range(K):
+        r = st.run_step(ev=evs[k])
+        blocks.append(r)
+    t1.record(stream)
+    torch.cuda.nvtx.range_pop()
+    stream.synchronize()
+    launches = kvg.kvg_launch_count() - launches0
+    clk = clocks.stop()
+    kvg.kvg_sync(st.cache.h, stream, 60.0)
+    ms_step = t0.elapsed_time(t1) / K
+    phase_ms = {p: [evs[k]["main"][i].elapsed_time(evs[k]["main"][i + 1]) for k in range(K)]
+                for i, p in enumerate(st.phases)}
+    step_bytes = sum(st.bytes.values())
+    parts = {}
+    for p, ts in phase_ms.items():
+        ms = statistics.mean(ts)
+        parts[p] = {"ms": round(ms, 4)}
+        if p in st.bytes:
+            gbs = st.bytes[p] / (ms * 1e-3) / 1e9
+            parts[p].update({"algorithmic_bytes": st.bytes[p], "gbs": round(gbs, 1),
+                             "hbm_frac": round(gbs / hbm_peak, 3)})
+    line = {"metric": METRIC, "unit": "GB/s", "n_gpus": 1, "steps": K, "warmup": args.warmup,
+            "ms_per_step": round(ms_step, 4), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic", "parts": parts, "gpu_launches": int(launches), "clocks": clk}
+    if args.config == "31b":
+        line["value"] = round(step_bytes / (ms_step * 1e-3) / 1e9, 2)
+        line["config"] = {"workload": f"31b-relocation: L{st.w.n_layers} Hq32/Hkv16 D128 P64 theta 1e6, 16384-token "
+                                      "block re-based by delta (0,1,4096,100000 across 8 sequences; 4096 timed), "
+                                      "decode batch 8 over 65536-token contexts"}
+        line["parts"]["decode"]["tokens_per_s"] = round(st.B * 1e3 / statistics.mean(phase_ms["decode"]), 1)
+    elif args.config == "batched":
+        line["value"] = round(step_bytes / (ms_step * 1e-3) / 1e9, 2)
+        line["config"] = {"workload": f"batched-library: L{st.w.n_layers} slice of 12b, 32 seqs x 4 blocks "
+                                      "U{2048..6144} from a 512-block HBM store, then 64 decode steps (batch 32)"}
+        line["parts"]["decode_steps"]["tokens_per_s"] = round(
+            syn.BATCHED_SEQS * st.steps * 1e3 / statistics.mean(phase_ms["decode_steps"]), 1)
+    else:
+        g = np.array(phase_ms["host_graft"])
+        depth = np.array(blocks, dtype=np.float64)
+        slope = float(np.polyfit(depth, g, 1)[0]) if len(set(blocks)) > 1 else 0.0
+        h2d = measure_h2d(device)
+        gbs = st.blk_bytes / (np.median(g) * 1e-3) / 1e9
+        line["value"] = round(gbs, 2)
+        line["unit"] = "GB/s host->HBM"
+        line["config"] = {"workload": f"deep-store: 2-layer 12b slice, {st.n_blocks} blocks x 2048 tokens "
+                                      f"({st.n_blocks * 2048} tokens, {st.n_blocks * st.blk_bytes / 1e9:.1f} GB) in "
+                                      "pinned host memory, uniform random grafts"}
+        line["roofline"] = {"bound": "host-link", "kernel": "graft_kernel", "achieved": round(gbs, 1),
+                            "peak": round(h2d, 1), "unit": "GB/s", "frac": round(gbs / h2d, 3),
+                            "peak_kind": "measured in-run: pinned cudaMemcpy H2D, 32 MiB"}
+        line["latency_ms"] = {"p50": round(float(np.percentile(g, 50)), 4),
+                              "p99": round(float(np.percentile(g, 99)), 4),
+                              "slope_ms_per_1000_blocks_depth": round(slope * 1000, 5)}
+        errs = []
+        # needle check on 8 sampled blocks
+        for b in sorted(set(int(x) for x in blocks))[:8]:
+            st.order = np.array([b])
+            st.k_iter = 0
+            st.run_step()
+            stream.synchronize()
+            errs.append(st.needle_error(b))
+        line["checks"] = {"needle_max_abs_err": max(errs), "needles_checked": len(errs)}
+    print(json.dumps(line), flush=True)
 
 
 def _sha_tensor(t):
@@ -342,40 +668,43 @@ def _sha_tensor(t):
 # CPU oracle on a bounded sample of the same step
 # --------------------------------------------------------------------------
 
-def oracle_sample(n_layers_sample: int):
-    """One oracle pass of the 12B step restricted to n_layers_sample layers.
+def oracle_sample(n_layers_sample: int, chunk: int = 4):
+    """One oracle pass of the 12B step over n_layers_sample layers, run in
+    chunks of `chunk` layers (inputs are generated per chunk, untimed).
     Returns (seconds, algorithmic bytes of the sample, threads used)."""
     import oracle
-    w = syn.B12.with_layers(n_layers_sample)
     nb, nf = syn.B12_BLOCK, syn.B12_CTX - syn.B12_BLOCK
-    k, v = syn.kv_rows(w, syn.B12_CTX, w.seed)
-    k, v = syn.as_u16(k), syn.as_u16(v)
-    q = syn.as_u16(syn.queries(w, w.n_layers, 1, w.seed))
-    d = oracle.Dims(w.n_layers, w.n_kv_heads, w.head_dim, w.page_size, w.rope_theta, 0)
-    blk = oracle.block_from_kv(d, k[:, :nb], v[:, :nb], syn.positions(0, nb))
-    cache = oracle.OracleCache(d, syn.B12_CTX // w.page_size, 1, syn.B12_CTX)
-    scale = 1 / math.sqrt(w.head_dim)
-    t0 = time.perf_counter()
-    cache.graft(0, blk)
-    pages = np.stack([cache.pool[l, kv, cache.page_table[0, j]] for l in range(w.n_layers) for kv in range(2)
-                      for j in range(blk.n_pages)])
-    dig = oracle.page_digests(pages.reshape(-1), w.page_bytes)
-    assert np.array_equal(dig.reshape(blk.digests.shape), blk.digests)
-    cache.append(0, k[:, nb:], v[:, nb:], syn.positions(nb, nf))
-    for l in range(w.n_layers):
-        cache.decode(0, l, q[l, 0], scale)
-    dt = time.perf_counter() - t0
-    blk_pages = w.n_layers * 2 * (nb // w.page_size) * w.page_bytes
-    b = 2 * blk_pages + blk_pages + 2 * w.n_layers * 2 * nf * w.n_kv_heads * w.head_dim * 2 \
-        + w.n_layers * 2 * syn.B12_CTX * w.n_kv_heads * w.head_dim * 2
-    return dt, b, oracle.omp_threads()
+    total_t, total_b = 0.0, 0
+    for c0 in range(0, n_layers_sample, chunk):
+        w = syn.B12.with_layers(min(chunk, n_layers_sample - c0))
+        k, v = syn.kv_rows(w, syn.B12_CTX, w.seed + c0)
+        k, v = syn.as_u16(k), syn.as_u16(v)
+        q = syn.as_u16(syn.queries(w, w.n_layers, 1, w.seed + c0))
+        d = oracle.Dims(w.n_layers, w.n_kv_heads, w.head_dim, w.page_size, w.rope_theta, 0)
+        blk = oracle.block_from_kv(d, k[:, :nb], v[:, :nb], syn.positions(0, nb))
+        cache = oracle.OracleCache(d, syn.B12_CTX // w.page_size, 1, syn.B12_CTX)
+        scale = 1 / math.sqrt(w.head_dim)
+        t0 = time.perf_counter()
+        cache.graft(0, blk)
+        pages = np.stack([cache.pool[l, kv, cache.page_table[0, j]] for l in range(w.n_layers)
+                          for kv in range(2) for j in range(blk.n_pages)])
+        dig = oracle.page_digests(pages.reshape(-1), w.page_bytes)
+        assert np.array_equal(dig.reshape(blk.digests.shape), blk.digests)
+        cache.append(0, k[:, nb:], v[:, nb:], syn.positions(nb, nf))
+        for l in range(w.n_layers):
+            cache.decode(0, l, q[l, 0], scale)
+        total_t += time.perf_counter() - t0
+        blk_pages = w.n_layers * 2 * (nb // w.page_size) * w.page_bytes
+        total_b += 2 * blk_pages + blk_pages + 2 * w.n_layers * 2 * nf * w.n_kv_heads * w.head_dim * 2 \
+            + w.n_layers * 2 * syn.B12_CTX * w.n_kv_heads * w.head_dim * 2
+    return total_t, total_b, oracle.omp_threads()
 
 
-def cpu_baseline(n_layers_sample=1):
+def cpu_baseline(n_layers_sample=48):
     dt, b, cores = oracle_sample(n_layers_sample)
     return {"value": round(b / dt / 1e9, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
             "sample": f"{n_layers_sample} of 48 layers of one 12b step (graft, page digests, 24576-row "
-                      f"append, fp64 decode of 16 heads over 32768 rows): {dt:.2f} s"}
+                      f"append, fp64 decode of 16 heads over 32768 rows), in 4-layer chunks: {dt:.2f} s"}
 
 
 def run_reference(args):
@@ -402,7 +731,11 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="kvg", choices=["kvg", "reference"])
-    ap.add_argument("--cpu-baseline-layers", type=int, default=4)
+    ap.add_argument("--cpu-baseline-layers", type=int, default=48)
+    ap.add_argument("--layers", type=int, default=0, help="layer count override (small profiling cases)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--config", default="12b", choices=["12b", "31b", "batched", "deep"])
+    ap.add_argument("--deep-blocks", type=int, default=syn.DEEP_BLOCKS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -412,6 +745,10 @@ def main():
     if args.impl == "reference":
         if rank == 0:
             print(json.dumps(run_reference(args)), flush=True)
+        return
+    if args.config != "12b":
+        if rank == 0:
+            run_other(args)
         return
     if world > 1:
         torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))

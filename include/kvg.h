@@ -191,6 +191,15 @@ kvg_status kvg_cache_seq_info(const kvg_cache *cache, int32_t seq, int32_t *n_sl
 kvg_status kvg_cache_append(kvg_cache *cache, int32_t seq, const void *k, const void *v,
                             const int32_t *positions, int32_t n, void *stream);
 
+/* Decode-step append: one new row per sequence for B sequences in one
+ * launch.  Row b of k and v (device, bf16 [n_layers][B][n_kv_heads]
+ * [head_dim]) and positions[b] (device int32 [B]) go to slot n_slots of
+ * sequence seq_ids[b] (host array, distinct ids, B <= 256), allocating a page
+ * where a sequence's last page is full.  KVG_ERR_CAPACITY if slots or pages
+ * run out (nothing is written); KVG_ERR_ARG on repeated ids. */
+kvg_status kvg_cache_append_batch(kvg_cache *cache, const int32_t *seq_ids, int32_t B, const void *k,
+                                  const void *v, const int32_t *positions, void *stream);
+
 /* Returns the sequence's pages to the free list and clears its page table,
  * fills and position tags. */
 kvg_status kvg_cache_release(kvg_cache *cache, int32_t seq, void *stream);
@@ -279,11 +288,12 @@ kvg_status kvg_decode_attention(kvg_cache *cache, int32_t layer, const int32_t *
  * the library holds until the process exits, and calls no allocating routine
  * (no cudaMalloc, cudaFree or library allocator).  Arguments, results and
  * errors are those of kvg_decode_attention, with these differences:
- *   - the split plan is capped so the partials fit the array; a call whose
- *     partials would not fit even unsplit (n_layers_run * min(B, 256) *
- *     n_q_heads * (4 * head_dim + 8) bytes > 16 MiB - 256) returns
- *     KVG_ERR_CAPACITY with an explanatory kvg_last_error() and enqueues
- *     nothing;
+ *   - the partials take (units + workers) * G * (4 * head_dim + 8) bytes,
+ *     units = n_layers_run * min(B, 256) * n_kv_heads, G = n_q_heads /
+ *     n_kv_heads; the number of decode workers (warps) is capped so they fit
+ *     in 16 MiB - 256 bytes, and a call that does not fit even with one
+ *     worker returns KVG_ERR_CAPACITY with an explanatory kvg_last_error()
+ *     and enqueues nothing;
  *   - the first call on a device looks up the array's device address
  *     (cudaGetSymbolAddress, with that device current); make that first call
  *     before any stream capture;

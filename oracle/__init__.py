@@ -323,6 +323,18 @@ class Block:
         return pos_off, dig_off, pages_off, total
 
 
+class BlockMeta:
+    """A block's bookkeeping only (length, pages, position tags), for
+    modelling page tables at sizes where the pool bytes are not modelled."""
+
+    def __init__(self, dims: Dims, positions: np.ndarray):
+        self.dims = dims
+        self.positions = np.ascontiguousarray(positions, np.int32)
+        self.n_tokens = int(self.positions.size)
+        self.n_pages = (self.n_tokens + dims.P - 1) // dims.P
+        self.pages = None
+
+
 def block_from_kv(dims: Dims, k: np.ndarray, v: np.ndarray, positions: np.ndarray) -> Block:
     """Deposit of logical rows: k, v [L][n][Hkv][D] bf16 bits, positions[n]."""
     d = dims
@@ -366,14 +378,17 @@ class OracleCache:
     a released sequence's pages go to the back in page-table order.
     """
 
-    def __init__(self, dims: Dims, n_pages: int, max_seqs: int, max_slots: int, fill=None):
+    def __init__(self, dims: Dims, n_pages: int, max_seqs: int, max_slots: int, fill=None,
+                 with_pool: bool = True):
+        """with_pool=False models page tables, fills and position tags only
+        (the pool bytes are not kept), for full-size workloads."""
         d = self.dims = dims
         self.n_pages = n_pages
         self.max_seqs = max_seqs
         self.max_slots = max_slots
         self.max_pages = (max_slots + d.P - 1) // d.P
-        self.pool = np.zeros((d.L, 2, n_pages, d.Hkv, d.P, d.D), np.uint16)
-        if fill is not None:
+        self.pool = np.zeros((d.L, 2, n_pages, d.Hkv, d.P, d.D), np.uint16) if with_pool else None
+        if fill is not None and self.pool is not None:
             self.pool[...] = fill
         self.free = list(range(n_pages))
         self.page_table = np.full((max_seqs, self.max_pages), -1, np.int32)
@@ -412,8 +427,9 @@ class OracleCache:
             s = s0 + t
             j, r = divmod(s, d.P)
             pid = self.page_table[seq, j]
-            self.pool[:, 0, pid, :, r, :] = k[:, t, :, :]
-            self.pool[:, 1, pid, :, r, :] = v[:, t, :, :]
+            if self.pool is not None:
+                self.pool[:, 0, pid, :, r, :] = k[:, t, :, :]
+                self.pool[:, 1, pid, :, r, :] = v[:, t, :, :]
             self.positions[seq, s] = positions[t]
             self.page_fill[seq, j] = r + 1
         self.n_slots[seq] = s0 + n
@@ -445,6 +461,8 @@ class OracleCache:
         for j, pid in enumerate(pids):
             self.page_table[seq, j0 + j] = pid
             self.page_fill[seq, j0 + j] = min(d.P, n - j * d.P)
+            if self.pool is None:
+                continue
             self.pool[:, :, pid] = block.pages[:, :, j]
             if delta != 0:
                 valid = min(d.P, n - j * d.P)
@@ -454,6 +472,14 @@ class OracleCache:
                         rows, delta, d.rope_theta, d.rope_style)
         self.positions[seq, dst_slot:dst_slot + n] = newpos.astype(np.int32)
         self.n_slots[seq] = dst_slot + n
+
+    def append_batch(self, seq_ids, k: np.ndarray, v: np.ndarray, positions: np.ndarray):
+        """Decode-step append: row b of k, v [L][B][Hkv][D] is appended to
+        sequence seq_ids[b] (one fresh row each, in batch order)."""
+        if len(set(int(x) for x in seq_ids)) != len(seq_ids):
+            raise KvgError("repeated sequence")
+        for b, sq in enumerate(seq_ids):
+            self.append(int(sq), k[:, b:b + 1], v[:, b:b + 1], positions[b:b + 1])
 
     def release(self, seq: int):
         used = [int(p) for p in self.page_table[seq] if p >= 0]

@@ -1,27 +1,32 @@
-// attn_kernels.cu — split-K paged GQA decode attention (Sec. 3.2 / Sec. 4.3:
-// one new query token attends to every row of the grafted context).
+// attn_kernels.cu — paged GQA decode attention (Sec. 3.2 / Sec. 4.3: one new
+// query token attends to every row of the grafted context).
 //
-// Grid (split, kv head g, layer x batch row).  A CTA owns a contiguous range
-// of the sequence's logical pages for one (layer, sequence, kv head) and all
-// G = Hq / Hkv query heads that read that kv head, so every K/V byte is read
-// from HBM once per step.  Each warp is an independent pipeline: its lane 0
-// issues bulk asynchronous copies (cp.async.bulk, completion on an mbarrier)
-// of TOK-row K and V tiles into the warp's own STAGES-deep shared-memory ring,
-// and all 32 lanes consume them:
-//   - lanes form 4 groups of 8; a group owns TOK/4 rows of the tile and each
-//     lane of the group 8*NCH of the D dimensions (16-byte chunks j, j+8, ...
-//     so a group's 8 lanes read one contiguous 128-byte span: no bank
-//     conflicts);
+// Persistent, load-balanced ("stream-K") design.  The work of a call is a
+// global list of tiles: unit (layer, batch row, kv head) owns its sequence's
+// pages in logical order, each page split into ceil(P / TOK) tiles of TOK
+// rows.  The kernel launches W one-warp CTAs, all co-resident; warp w takes
+// the contiguous range [w*T/W, (w+1)*T/W) of the T tiles, so every warp gets
+// the same share and there is no tail wave.  A warp is an independent
+// pipeline: lane 0 issues bulk asynchronous copies (cp.async.bulk, completion
+// on an mbarrier, bounded wait) of the K and V rows of a tile into a
+// STAGES-deep shared-memory ring, STAGES-1 tiles ahead, across unit
+// boundaries; the 32 lanes consume them:
+//   - lanes form 4 groups of 8; a group owns every 4th row of the tile and
+//     each lane 8*D/64 dimensions in 16-byte chunks j, j+8, ... (a group's 8
+//     lanes read one contiguous 128-byte span: no bank conflicts);
 //   - q.k partial sums are all-reduced over the group with 3 xor shuffles;
-//   - each group keeps its own online-softmax state (running max m, sum l,
-//     output o in fp32) and rescales o only when the running max grows
-//     (multiplying by exp2(0) = 1 would change nothing, so this is exact);
-//   - at the end the 4 groups, then the warps, then the splits are merged in a
-//     fixed order.
-// Every reduction order depends only on logical token indices, never on the
-// physical page ids, so the output is bitwise reproducible and identical for
-// grafted and freshly written rows.  G = 2 (the workloads here) fills 2 of 16
-// rows of an MMA tile; at ~2 flop per byte the CUDA cores keep up with HBM.
+//   - each group keeps an online-softmax state (running max m, sum l, fp32
+//     output o) for all G query heads of the kv head (K/V read once) and
+//     rescales o only when the running max grows (the skipped factor is
+//     exactly 1);
+//   - when the warp leaves a unit it merges its 4 groups in a fixed order and
+//     writes the unit's partial (o, m, l) to slot unit + w.
+// The combine kernel merges, for each unit, the partials of the warps that
+// covered it, in warp order.  Every reduction order is a function of logical
+// token indices and of (T, W) only — never of physical page ids — so results
+// are bitwise reproducible and identical for grafted and freshly written rows.
+// G = 2 fills 2 of 16 rows of an MMA tile; at ~2 flop per byte the CUDA cores
+// keep up with HBM, so the contraction stays on the FMA pipe.
 #include <math.h>
 
 #include "common.cuh"
@@ -34,27 +39,26 @@ template <int D>
 struct TileShape;
 template <>
 struct TileShape<64> {
-    static constexpr int TOK = 32, STAGES = 3, WARPS = 4;
+    static constexpr int TOK = 32, STAGES = 3;
 };
 template <>
 struct TileShape<128> {
-    static constexpr int TOK = 32, STAGES = 3, WARPS = 4;
+    static constexpr int TOK = 32, STAGES = 2;
 };
 template <>
 struct TileShape<256> {
-    static constexpr int TOK = 16, STAGES = 3, WARPS = 4;
+    static constexpr int TOK = 16, STAGES = 2;
 };
 
 template <int D>
 struct Cfg {
     static constexpr int TOK = TileShape<D>::TOK;
     static constexpr int STAGES = TileShape<D>::STAGES;
-    static constexpr int WARPS = TileShape<D>::WARPS;
-    static constexpr int NCH = D / 64;            // 16-byte chunks per lane per row
+    static constexpr int NCH = D / 64;              // 16-byte chunks per lane per row
     static constexpr int TILE_BYTES = TOK * D * 2;  // one K (or V) tile
     static constexpr int STAGE_BYTES = 2 * TILE_BYTES;
-    static constexpr int RING_BYTES = WARPS * STAGES * STAGE_BYTES;
-    static constexpr int SMEM = RING_BYTES + WARPS * STAGES * (8 + 4);
+    static constexpr int RING_BYTES = STAGES * STAGE_BYTES;
+    static constexpr int SMEM = RING_BYTES + STAGES * (8 + 4);
 };
 
 __device__ __forceinline__ void unpack8(const uint4 &v, float *f) {
@@ -73,32 +77,56 @@ __device__ __forceinline__ float wsum(float x, float a, float y, float b) {
     return __fadd_rn(__fmul_rn(x, a), __fmul_rn(y, b));
 }
 
+// Position of global tile t: unit (lr, b, g) and tile index within the unit.
+struct TilePos {
+    int lr, b, g;
+    int64_t unit;
+    int tile;
+};
+
+__device__ __forceinline__ TilePos locate(const DecodeParams &p, int64_t t) {
+    const int64_t sumT = p.rows.pref_tiles[p.B];
+    const int64_t per_layer = (int64_t)p.n_kv_heads * sumT;
+    TilePos r;
+    r.lr = (int)(t / per_layer);
+    const int64_t rem = t - (int64_t)r.lr * per_layer;
+    int lo = 0, hi = p.B - 1;  // largest b with Hkv * pref[b] <= rem
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if ((int64_t)p.n_kv_heads * p.rows.pref_tiles[mid] <= rem)
+            lo = mid;
+        else
+            hi = mid - 1;
+    }
+    r.b = lo;
+    const int64_t r2 = rem - (int64_t)p.n_kv_heads * p.rows.pref_tiles[lo];
+    const int Tb = p.rows.pref_tiles[lo + 1] - p.rows.pref_tiles[lo];
+    r.g = (int)(r2 / Tb);
+    r.tile = (int)(r2 - (int64_t)r.g * Tb);
+    r.unit = ((int64_t)r.lr * p.B + r.b) * p.n_kv_heads + r.g;
+    return r;
+}
+
+__device__ __forceinline__ int64_t warp_start(int64_t w, int64_t T, int64_t W) { return w * T / W; }
+
 template <int D, int G>
-__global__ void __launch_bounds__(Cfg<D>::WARPS * 32, 1) decode_split_kernel(const DecodeParams p) {
+__global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p) {
     using C = Cfg<D>;
-    constexpr int TOK = C::TOK, STAGES = C::STAGES, WARPS = C::WARPS, NCH = C::NCH;
+    constexpr int TOK = C::TOK, STAGES = C::STAGES, NCH = C::NCH;
     constexpr int TPG = TOK / 4;  // rows per lane group per tile
     extern __shared__ __align__(128) uint8_t smem[];
 
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int lane = threadIdx.x;
     const int grp = lane >> 3, lj = lane & 7;
-    const int split = blockIdx.x, g = blockIdx.y;
-    const int lr = blockIdx.z / p.B, b = blockIdx.z - lr * p.B;
-    const int l = p.layer0 + lr;
-    const int seq = p.rows.seq[b];
-    const int np = p.rows.npages[b];
+    const int64_t w = blockIdx.x;
+    const int64_t t0 = warp_start(w, p.n_tiles, p.n_warps);
+    const int64_t t1 = warp_start(w + 1, p.n_tiles, p.n_warps);
     const int P = p.page_size;
     const int tpp = (P + TOK - 1) / TOK;
-    const int j0 = split * p.pages_per_split;
-    int j1 = j0 + p.pages_per_split;
-    if (j1 > np) j1 = np;
-    const int ntiles = j1 > j0 ? (j1 - j0) * tpp : 0;
-    const int my_n = warp < ntiles ? (ntiles - warp + WARPS - 1) / WARPS : 0;
 
-    uint8_t *ring = smem + warp * STAGES * C::STAGE_BYTES;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::RING_BYTES) + warp * STAGES;
-    int *vrs = reinterpret_cast<int *>(smem + C::RING_BYTES + WARPS * STAGES * 8) + warp * STAGES;
-
+    uint8_t *ring = smem;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::RING_BYTES);
+    int *vrs = reinterpret_cast<int *>(smem + C::RING_BYTES + STAGES * 8);
     if (lane == 0) {
 #pragma unroll
         for (int s = 0; s < STAGES; ++s) mbar_init(&bars[s], 1);
@@ -108,16 +136,14 @@ __global__ void __launch_bounds__(Cfg<D>::WARPS * 32, 1) decode_split_kernel(con
 
     const int64_t plane_elems = p.pool_pages * (int64_t)p.n_kv_heads * P * D;
     const __nv_bfloat16 *poolh = reinterpret_cast<const __nv_bfloat16 *>(p.pool);
-    const int32_t *trow = p.page_table + (int64_t)seq * p.max_pages;
-    const int32_t *frow = p.page_fill + (int64_t)seq * p.max_pages;
 
-    auto issue = [&](int i) {  // lane 0: tile i of this warp's sequence
-        const int t = warp + i * WARPS;
-        const int jj = j0 + t / tpp;
-        const int k = t - (t / tpp) * tpp;
-        const int stg = i % STAGES;
-        const int fill = frow[jj];
-        const int pid = trow[jj];
+    auto issue = [&](int64_t t, int stg) {  // lane 0
+        const TilePos tp = locate(p, t);
+        const int seq = p.rows.seq[tp.b];
+        const int jj = tp.tile / tpp;
+        const int k = tp.tile - jj * tpp;
+        const int fill = p.page_fill[(int64_t)seq * p.max_pages + jj];
+        const int pid = p.page_table[(int64_t)seq * p.max_pages + jj];
         int vr = fill - k * TOK;
         vr = vr < 0 ? 0 : (vr > TOK ? TOK : vr);
         if (vr > 0 && (pid < 0 || pid >= p.pool_pages)) {
@@ -129,8 +155,9 @@ __global__ void __launch_bounds__(Cfg<D>::WARPS * 32, 1) decode_split_kernel(con
         if (vr > 0) {
             const uint32_t bytes = (uint32_t)vr * D * 2;
             mbar_arrive_expect_tx(bar, 2 * bytes);
+            const int l = p.layer0 + tp.lr;
             const __nv_bfloat16 *ks = poolh + (int64_t)(2 * l) * plane_elems +
-                                      ((int64_t)pid * p.n_kv_heads + g) * P * D + (int64_t)k * TOK * D;
+                                      ((int64_t)pid * p.n_kv_heads + tp.g) * P * D + (int64_t)k * TOK * D;
             uint8_t *dst = ring + stg * C::STAGE_BYTES;
             bulk_g2s(dst, ks, bytes, bar);
             bulk_g2s(dst + C::TILE_BYTES, ks + plane_elems, bytes, bar);
@@ -139,42 +166,87 @@ __global__ void __launch_bounds__(Cfg<D>::WARPS * 32, 1) decode_split_kernel(con
         }
     };
 
-    // query rows of this kv head's group, pre-scaled by scale*log2(e)
     float qf[G][NCH][8];
-    {
-        const __nv_bfloat16 *qrow =
-            p.q + ((int64_t)(lr * p.q_row_stride_b + p.b0 + b) * p.n_q_heads + g * G) * D;
+    float m[G], lsum[G], o[G][NCH][8];
+    int64_t cur_unit = -1;
+
+    auto flush = [&](int64_t unit) {
+        // merge the 4 lane groups: (0,1),(2,3) then (01,23)
 #pragma unroll
-        for (int h = 0; h < G; ++h)
+        for (int off = 8; off <= 16; off <<= 1) {
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                const float mo = __shfl_xor_sync(0xffffffffu, m[h], off);
+                const float lo = __shfl_xor_sync(0xffffffffu, lsum[h], off);
+                const float mn = fmaxf(m[h], mo);
+                const float a = m[h] == -INFINITY ? 0.f : exp2f(m[h] - mn);
+                const float bb = mo == -INFINITY ? 0.f : exp2f(mo - mn);
+                lsum[h] = wsum(lsum[h], a, lo, bb);
+#pragma unroll
+                for (int c = 0; c < NCH; ++c)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float oo = __shfl_xor_sync(0xffffffffu, o[h][c][e], off);
+                        o[h][c][e] = wsum(o[h][c][e], a, oo, bb);
+                    }
+                m[h] = mn;
+            }
+        }
+        const int64_t slot = unit + w;
+        if (lane < 8) {
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                float *dst = p.part_o + (slot * G + h) * D;
+#pragma unroll
+                for (int c = 0; c < NCH; ++c) {
+                    float4 *d4 = reinterpret_cast<float4 *>(dst + 8 * (lj + 8 * c));
+                    d4[0] = make_float4(o[h][c][0], o[h][c][1], o[h][c][2], o[h][c][3]);
+                    d4[1] = make_float4(o[h][c][4], o[h][c][5], o[h][c][6], o[h][c][7]);
+                }
+            }
+            if (lane == 0)
+#pragma unroll
+                for (int h = 0; h < G; ++h) p.part_ml[slot * G + h] = make_float2(m[h], lsum[h]);
+        }
+    };
+
+    auto begin = [&](const TilePos &tp) {
+        const __nv_bfloat16 *qrow =
+            p.q + ((int64_t)(tp.lr * p.q_row_stride_b + p.b0 + tp.b) * p.n_q_heads + tp.g * G) * D;
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            m[h] = -INFINITY;
+            lsum[h] = 0.f;
 #pragma unroll
             for (int c = 0; c < NCH; ++c) {
                 const uint4 v = *reinterpret_cast<const uint4 *>(qrow + h * D + 8 * (lj + 8 * c));
                 unpack8(v, qf[h][c]);
 #pragma unroll
-                for (int e = 0; e < 8; ++e) qf[h][c][e] *= p.qscale;
+                for (int e = 0; e < 8; ++e) {
+                    qf[h][c][e] *= p.qscale;
+                    o[h][c][e] = 0.f;
+                }
             }
-    }
-
-    float m[G], lsum[G], o[G][NCH][8];
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-        m[h] = -INFINITY;
-        lsum[h] = 0.f;
-#pragma unroll
-        for (int c = 0; c < NCH; ++c)
-#pragma unroll
-            for (int e = 0; e < 8; ++e) o[h][c][e] = 0.f;
-    }
+        }
+    };
 
     if (lane == 0) {
-        const int pre = my_n < STAGES ? my_n : STAGES;
-        for (int i = 0; i < pre; ++i) issue(i);
+        for (int i = 0; i < STAGES && t0 + i < t1; ++i) issue(t0 + i, i);
     }
 
     bool alive = true;
-    for (int i = 0; i < my_n; ++i) {
-        const int stg = i % STAGES;
+    int64_t unit_end = t0;  // first tile past the current unit
+    for (int64_t t = t0; t < t1; ++t) {
+        const int64_t i = t - t0;
+        const int stg = (int)(i % STAGES);
         const uint32_t par = (uint32_t)((i / STAGES) & 1);
+        if (t >= unit_end) {
+            const TilePos tp = locate(p, t);
+            if (cur_unit >= 0) flush(cur_unit);
+            begin(tp);
+            cur_unit = tp.unit;
+            unit_end = t - tp.tile + (p.rows.pref_tiles[tp.b + 1] - p.rows.pref_tiles[tp.b]);
+        }
         const bool ok = mbar_wait_bounded(&bars[stg], par);
         if (!__all_sync(0xffffffffu, ok)) {
             if (lane == 0) record_error(p.status, KVG_ERR_DEVICE_CHECK, 2);
@@ -251,11 +323,12 @@ __global__ void __launch_bounds__(Cfg<D>::WARPS * 32, 1) decode_split_kernel(con
             }
         }
         __syncwarp();
-        if (lane == 0 && i + STAGES < my_n) issue(i + STAGES);
+        if (lane == 0 && t + STAGES < t1) issue(t + STAGES, stg);
     }
     if (!alive) {
-        // drain this warp's copies still in flight (bounded) before the CTA
-        // can exit, then report an empty partial
+        // a copy never completed: wait (bounded) on every stage once more so
+        // no copy is left writing this CTA's shared memory, then record an
+        // empty partial for the unit in progress
         if (lane == 0)
             for (int s = 0; s < STAGES; ++s) (void)mbar_wait_bounded(&bars[s], 0);
 #pragma unroll
@@ -268,101 +341,70 @@ __global__ void __launch_bounds__(Cfg<D>::WARPS * 32, 1) decode_split_kernel(con
                 for (int e = 0; e < 8; ++e) o[h][c][e] = 0.f;
         }
     }
-
-    // merge the 4 lane groups of the warp: (0,1),(2,3) then (01,23)
-#pragma unroll
-    for (int off = 8; off <= 16; off <<= 1) {
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-            const float mo = __shfl_xor_sync(0xffffffffu, m[h], off);
-            const float lo = __shfl_xor_sync(0xffffffffu, lsum[h], off);
-            const float mn = fmaxf(m[h], mo);
-            const float a = m[h] == -INFINITY ? 0.f : exp2f(m[h] - mn);
-            const float bb = mo == -INFINITY ? 0.f : exp2f(mo - mn);
-            lsum[h] = wsum(lsum[h], a, lo, bb);
-#pragma unroll
-            for (int c = 0; c < NCH; ++c)
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float oo = __shfl_xor_sync(0xffffffffu, o[h][c][e], off);
-                    o[h][c][e] = wsum(o[h][c][e], a, oo, bb);
-                }
-            m[h] = mn;
-        }
-    }
-
-    // merge the warps through shared memory (ring no longer in use), in order
-    __syncthreads();
-    float *red_o = reinterpret_cast<float *>(smem);                    // [WARPS][G][D]
-    float2 *red_ml = reinterpret_cast<float2 *>(smem + WARPS * G * D * 4);  // [WARPS][G]
-    if (lane < 8) {
-#pragma unroll
-        for (int h = 0; h < G; ++h)
-#pragma unroll
-            for (int c = 0; c < NCH; ++c)
-#pragma unroll
-                for (int e = 0; e < 8; ++e) red_o[(warp * G + h) * D + 8 * (lj + 8 * c) + e] = o[h][c][e];
-        if (lane == 0)
-#pragma unroll
-            for (int h = 0; h < G; ++h) red_ml[warp * G + h] = make_float2(m[h], lsum[h]);
-    }
-    __syncthreads();
-    const int64_t unit = ((int64_t)lr * p.B + b) * p.n_kv_heads + g;
-    for (int idx = threadIdx.x; idx < G * D; idx += WARPS * 32) {
-        const int h = idx / D, d = idx - h * D;
-        float M = -INFINITY;
-#pragma unroll
-        for (int w = 0; w < WARPS; ++w) M = fmaxf(M, red_ml[w * G + h].x);
-        float L = 0.f, O = 0.f;
-#pragma unroll
-        for (int w = 0; w < WARPS; ++w) {
-            const float2 ml = red_ml[w * G + h];
-            const float sc = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);
-            L = __fmaf_rn(ml.y, sc, L);
-            O = __fmaf_rn(red_o[(w * G + h) * D + d], sc, O);
-        }
-        const int64_t part = (unit * p.n_splits + split) * G + h;
-        p.part_o[part * D + d] = O;
-        if (d == 0) p.part_ml[part] = make_float2(M, L);
-    }
+    if (cur_unit >= 0) flush(cur_unit);
 }
 
+// Largest warp index whose range starts at or before tile t.
+__device__ __forceinline__ int64_t warp_of(int64_t t, int64_t T, int64_t W) { return ((t + 1) * W - 1) / T; }
+
 template <int D>
-__global__ void __launch_bounds__(D) combine_kernel(const CombineParams p) {
+__global__ void __launch_bounds__(D) combine_kernel(const DecodeParams p) {
     const int h = blockIdx.x, b = blockIdx.y, lr = blockIdx.z;
     const int G = p.n_q_heads / p.n_kv_heads;
     const int g = h / G, hh = h - g * G;
     const int d = threadIdx.x;
     const int64_t unit = ((int64_t)lr * p.B + b) * p.n_kv_heads + g;
-    float M = -INFINITY;
-    for (int s = 0; s < p.n_splits; ++s) M = fmaxf(M, p.part_ml[(unit * p.n_splits + s) * G + hh].x);
+    const int64_t sumT = p.rows.pref_tiles[p.B];
+    const int64_t Tb = p.rows.pref_tiles[b + 1] - p.rows.pref_tiles[b];
     float L = 0.f, O = 0.f;
-    for (int s = 0; s < p.n_splits; ++s) {
-        const int64_t part = (unit * p.n_splits + s) * G + hh;
-        const float2 ml = p.part_ml[part];
-        if (ml.x == -INFINITY) continue;
-        const float sc = exp2f(ml.x - M);
-        L = __fmaf_rn(ml.y, sc, L);
-        O = __fmaf_rn(p.part_o[part * D + d], sc, O);
+    if (Tb > 0) {
+        const int64_t T = p.n_tiles, W = p.n_warps;
+        const int64_t first = (int64_t)lr * p.n_kv_heads * sumT + (int64_t)p.n_kv_heads * p.rows.pref_tiles[b] +
+                              (int64_t)g * Tb;
+        const int64_t last = first + Tb - 1;
+        const int64_t wa = warp_of(first, T, W), wb = warp_of(last, T, W);
+        float M = -INFINITY;
+        for (int64_t w = wa; w <= wb; ++w) {
+            if (warp_start(w + 1, T, W) == warp_start(w, T, W)) continue;  // empty range
+            M = fmaxf(M, p.part_ml[(unit + w) * G + hh].x);
+        }
+        for (int64_t w = wa; w <= wb; ++w) {
+            if (warp_start(w + 1, T, W) == warp_start(w, T, W)) continue;
+            const float2 ml = p.part_ml[(unit + w) * G + hh];
+            if (ml.x == -INFINITY) continue;
+            const float sc = exp2f(ml.x - M);
+            L = __fmaf_rn(ml.y, sc, L);
+            O = __fmaf_rn(p.part_o[((unit + w) * G + hh) * D + d], sc, O);
+        }
     }
     const float r = L > 0.f ? __fdiv_rn(O, L) : 0.f;
     p.out[((int64_t)(lr * p.q_row_stride_b + p.b0 + b) * p.n_q_heads + h) * D + d] = __float2bfloat16_rn(r);
 }
 
 template <int D, int G>
-cudaError_t launch_decode_t(const DecodeParams &p, cudaStream_t s) {
-    static bool configured = false;  // attribute set once per instantiation
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<D, G>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<D>::SMEM);
-        if (e != cudaSuccess) return e;
-        configured = true;
+struct DecodeLaunch {
+    static int max_blocks_per_sm() {
+        static int cached = -1;
+        if (cached < 0) {
+            if (cudaFuncSetAttribute(decode_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     Cfg<D>::SMEM) != cudaSuccess)
+                return 0;
+            int n = 0;
+            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<D, G>, 32, Cfg<D>::SMEM) !=
+                cudaSuccess)
+                return 0;
+            cached = n;
+        }
+        return cached;
     }
-    dim3 grid(p.n_splits, p.n_kv_heads, p.n_layers_run * p.B);
-    decode_split_kernel<D, G><<<grid, Cfg<D>::WARPS * 32, Cfg<D>::SMEM, s>>>(p);
-    count_launches(1);
-    return cudaGetLastError();
-}
+    static cudaError_t run(const DecodeParams &p, cudaStream_t s) {
+        if (max_blocks_per_sm() <= 0) return cudaErrorInvalidConfiguration;
+        if (p.n_warps <= 0 || p.n_tiles <= 0) return cudaSuccess;
+        decode_kernel<D, G><<<p.n_warps, 32, Cfg<D>::SMEM, s>>>(p);
+        count_launches(1);
+        return cudaGetLastError();
+    }
+};
 
 }  // namespace
 
@@ -372,29 +414,37 @@ bool decode_supported(int head_dim, int group) {
     return head_dim * group <= 512;
 }
 
-size_t decode_smem_bytes(int head_dim) {
+int decode_tile_tokens(int head_dim) {
     switch (head_dim) {
-        case 64: return Cfg<64>::SMEM;
-        case 128: return Cfg<128>::SMEM;
-        case 256: return Cfg<256>::SMEM;
+        case 64: return Cfg<64>::TOK;
+        case 128: return Cfg<128>::TOK;
+        case 256: return Cfg<256>::TOK;
     }
+    return 0;
+}
+
+#define KVG_DECODE_CASES(X) \
+    X(64, 1) X(64, 2) X(64, 4) X(64, 8) X(128, 1) X(128, 2) X(128, 4) X(256, 1) X(256, 2)
+
+int decode_max_warps(int head_dim, int group, int n_sm) {
+#define KVG_CASE(DD, GG) \
+    if (head_dim == DD && group == GG) return DecodeLaunch<DD, GG>::max_blocks_per_sm() * n_sm;
+    KVG_DECODE_CASES(KVG_CASE)
+#undef KVG_CASE
     return 0;
 }
 
 cudaError_t launch_decode(int head_dim, int group, const DecodeParams &p, cudaStream_t s) {
 #define KVG_CASE(DD, GG) \
-    if (head_dim == DD && group == GG) return launch_decode_t<DD, GG>(p, s);
-    KVG_CASE(64, 1) KVG_CASE(64, 2) KVG_CASE(64, 4) KVG_CASE(64, 8)
-    KVG_CASE(128, 1) KVG_CASE(128, 2) KVG_CASE(128, 4)
-    KVG_CASE(256, 1) KVG_CASE(256, 2)
+    if (head_dim == DD && group == GG) return DecodeLaunch<DD, GG>::run(p, s);
+    KVG_DECODE_CASES(KVG_CASE)
 #undef KVG_CASE
     return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_combine(int head_dim, int group, const CombineParams &p, int n_layers_run, int B,
-                           cudaStream_t s) {
+cudaError_t launch_combine(int head_dim, int group, const DecodeParams &p, cudaStream_t s) {
     (void)group;
-    dim3 grid(p.n_q_heads, B, n_layers_run);
+    dim3 grid(p.n_q_heads, p.B, p.n_layers_run);
     switch (head_dim) {
         case 64: combine_kernel<64><<<grid, 64, 0, s>>>(p); count_launches(1); break;
         case 128: combine_kernel<128><<<grid, 128, 0, s>>>(p); count_launches(1); break;

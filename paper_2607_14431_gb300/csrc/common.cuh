@@ -82,6 +82,20 @@ struct AppendParams {
     PageList pids;             // pages touched: page0 .. page0 + n - 1
 };
 
+// One new row per sequence (decode step): row b goes to page pid[b], row
+// `row[b]` of that page, slot slot[b] of sequence seq[b].
+struct AppendBatchParams {
+    const uint16_t *k, *v;     // [L][B][Hkv][D]
+    const int32_t *pos;        // [B]
+    uint8_t *pool;
+    int64_t pool_pages;
+    int32_t n_layers, n_kv_heads, page_size, head_dim, B, max_pages, max_slots;
+    int32_t *page_table, *page_fill, *positions;  // whole-cache arrays
+    int32_t seq[kMaxBatchPerLaunch];
+    int32_t pid[kMaxBatchPerLaunch];
+    int32_t slot[kMaxBatchPerLaunch];
+};
+
 // --------------------------------------------------------------- deposit --
 struct GatherParams {
     const uint8_t *pool;
@@ -113,9 +127,15 @@ struct PageSource {
 };
 
 // --------------------------------------------------------------- decode --
+// A launch covers Lrun layers x B batch rows x Hkv kv heads ("units").  Unit
+// (l, b, g) owns T_b = npages_b * tiles_per_page tiles, in page order; the
+// global tile list orders units (l, b, g) with g fastest.  Warp w of W takes
+// the contiguous range [w*T/W, (w+1)*T/W) and writes one partial per unit it
+// touches, at slot unit + w (unique because both ranges are contiguous).
 struct BatchRows {
     int32_t seq[kMaxBatchPerLaunch];
     int32_t npages[kMaxBatchPerLaunch];
+    int32_t pref_tiles[kMaxBatchPerLaunch + 1];  // prefix sums of T_b
 };
 
 struct DecodeParams {
@@ -123,34 +143,33 @@ struct DecodeParams {
     int64_t pool_pages;
     int32_t n_kv_heads, page_size, n_q_heads;
     int32_t layer0, n_layers_run, B;
-    int32_t n_splits, pages_per_split;
+    int32_t n_warps;           // W
+    int64_t n_tiles;           // T
     const int32_t *page_table;
     const int32_t *page_fill;
     int32_t max_pages;
-    const __nv_bfloat16 *q;    // [Lrun][B][Hq][D] (this launch's rows)
+    const __nv_bfloat16 *q;    // [Lrun][Btot][Hq][D]
     int32_t q_row_stride_b;    // rows of the full batch (B of the whole call)
     int32_t b0;                // first batch row of this launch
     float qscale;              // softmax scale * log2(e)
-    float *part_o;             // [Lrun][B][Hkv][S][G][D]
-    float2 *part_ml;           // [Lrun][B][Hkv][S][G]
+    float *part_o;             // [U + W][G][D]
+    float2 *part_ml;           // [U + W][G]
+    __nv_bfloat16 *out;        // [Lrun][Btot][Hq][D] (combine)
     DevStatus *status;
     BatchRows rows;
-};
-
-struct CombineParams {
-    const float *part_o;
-    const float2 *part_ml;
-    __nv_bfloat16 *out;        // [Lrun][B][Hq][D]
-    int32_t n_kv_heads, n_q_heads, n_splits, B, q_row_stride_b, b0;
 };
 
 // -------------------------------------------------------------- launchers --
 // Every launcher counts the kernels it launches (kvg_launch_count()).
 void count_launches(uint64_t n);
 uint64_t launch_count();
+// Integer tuning knob from the environment (read once), e.g. CTAs per SM of
+// a grid-stride kernel; `fallback` when unset or not positive.
+int env_knob(const char *name, int fallback);
 
 cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_append(const AppendParams &p, int n_sm, cudaStream_t s);
+cudaError_t launch_append_batch(const AppendBatchParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_write_header(const HeaderParams &p, cudaStream_t s);
 cudaError_t launch_reset_seq(int32_t *table_row, int32_t *fill_row, int32_t max_pages,
@@ -169,11 +188,15 @@ cudaError_t launch_sha256_serial(const uint8_t *seg0, uint64_t n0, const uint8_t
                                  uint8_t *out, const uint8_t *expected, DevStatus *status,
                                  cudaStream_t s);
 
+// Persistent decode: p.n_warps one-warp CTAs over p.n_tiles tiles, then the
+// combine over every (layer, row, query head).  decode_tile_tokens() is the
+// tile height TOK (tiles per page = ceil(P / TOK)); decode_max_warps() the
+// number of co-resident warps the decode kernel can keep on the device.
 cudaError_t launch_decode(int head_dim, int group, const DecodeParams &p, cudaStream_t s);
-cudaError_t launch_combine(int head_dim, int group, const CombineParams &p, int n_layers_run,
-                           int B, cudaStream_t s);
+cudaError_t launch_combine(int head_dim, int group, const DecodeParams &p, cudaStream_t s);
 bool decode_supported(int head_dim, int group);
-size_t decode_smem_bytes(int head_dim);
+int decode_tile_tokens(int head_dim);
+int decode_max_warps(int head_dim, int group, int n_sm);
 
 // ------------------------------------------------------------ PTX helpers --
 #ifdef __CUDACC__

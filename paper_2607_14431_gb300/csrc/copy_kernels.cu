@@ -163,11 +163,14 @@ __global__ void __launch_bounds__(kCopyThreads) graft_kernel(const GraftParams p
     }
 }
 
-__global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
-    const int D = p.head_dim;
-    const int vpr = D >> 3;  // 16-byte vectors per row
-    const int64_t per_kv = (int64_t)p.n_layers * p.n * p.n_kv_heads * vpr;
-    const int64_t total = 2 * per_kv;
+// One warp per (layer, K/V, token) row: the row's Hkv*D*2 source bytes are
+// contiguous ([L][n][Hkv][D] input); head h goes to row `row` of head h's
+// [P][D] slab in the token's page.  Index arithmetic is per row, not per
+// vector; each lane keeps up to kAppendUnroll 16-byte loads in flight.
+constexpr int kAppendThreads = 256;
+constexpr int kAppendUnroll = 8;
+
+__global__ void __launch_bounds__(kAppendThreads) append_kernel(const AppendParams p) {
     const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
     const int64_t P = p.page_size;
@@ -178,25 +181,79 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
         const int64_t f = (int64_t)p.slot0 + p.n - pg * P;
         p.fill_row[pg] = (int32_t)(f < P ? f : P);
     }
-    for (int64_t idx = gtid; idx < total; idx += gsz) {
-        const int kv = idx >= per_kv;
-        int64_t r = idx - kv * per_kv;
-        const int c = (int)(r % vpr);
-        r /= vpr;
-        const int h = (int)(r % p.n_kv_heads);
-        r /= p.n_kv_heads;
-        const int t = (int)(r % p.n);
-        const int l = (int)(r / p.n);
-        const uint16_t *srcbase = kv ? p.v : p.k;
-        const uint4 val = __ldcs(reinterpret_cast<const uint4 *>(
-            srcbase + (((int64_t)l * p.n_rows_total + p.row0 + t) * p.n_kv_heads + h) * D) + c);
+    const int D = p.head_dim;
+    const int vpr = D >> 3;                 // 16-byte vectors per head row
+    const int vpt = p.n_kv_heads * vpr;     // vectors per token row
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = gtid >> 5;
+    const int64_t n_warps = gsz >> 5;
+    const int64_t rows = (int64_t)p.n_layers * 2 * p.n;
+    const int64_t head_stride_vec = P * D / 8;  // between heads of one page, in vectors
+    for (int64_t r = warp; r < rows; r += n_warps) {
+        const int64_t lkv = r / p.n;
+        const int t = (int)(r - lkv * p.n);
+        const int l = (int)(lkv >> 1), kv = (int)(lkv & 1);
+        const uint4 *src = reinterpret_cast<const uint4 *>(
+            (kv ? p.v : p.k) + ((int64_t)l * p.n_rows_total + p.row0 + t) * p.n_kv_heads * D);
         const int64_t s = (int64_t)p.slot0 + t;
         const int64_t pg = s / P;
         const int pid = p.pids.pid[pg - p.page0];
         const int64_t row = s - pg * P;
-        uint16_t *dst = reinterpret_cast<uint16_t *>(p.pool) +
-                        ((((int64_t)l * 2 + kv) * p.pool_pages + pid) * p.n_kv_heads + h) * P * D + row * D;
-        __stcs(reinterpret_cast<uint4 *>(dst) + c, val);
+        uint4 *dst = reinterpret_cast<uint4 *>(
+            reinterpret_cast<uint16_t *>(p.pool) +
+            (((int64_t)lkv * p.pool_pages + pid) * p.n_kv_heads) * P * D + row * D);
+        for (int base = lane; base < vpt; base += 32 * kAppendUnroll) {
+            uint4 val[kAppendUnroll];
+#pragma unroll
+            for (int u = 0; u < kAppendUnroll; ++u) {
+                const int i = base + 32 * u;
+                if (i < vpt) val[u] = __ldcs(src + i);
+            }
+#pragma unroll
+            for (int u = 0; u < kAppendUnroll; ++u) {
+                const int i = base + 32 * u;
+                if (i < vpt) {
+                    const int h = i / vpr, c = i - h * vpr;
+                    __stcs(dst + h * head_stride_vec + c, val[u]);
+                }
+            }
+        }
+    }
+}
+
+// One warp per (layer, K/V, batch row): Hkv*D*2 contiguous source bytes to
+// row `row` of each head's slab of the row's page.
+__global__ void __launch_bounds__(kAppendThreads) append_batch_kernel(const AppendBatchParams p) {
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+    const int64_t P = p.page_size;
+    for (int64_t b = gtid; b < p.B; b += gsz) {
+        const int64_t s = p.slot[b];
+        const int64_t pg = s / P;
+        p.positions[(int64_t)p.seq[b] * p.max_slots + s] = p.pos[b];
+        p.page_table[(int64_t)p.seq[b] * p.max_pages + pg] = p.pid[b];
+        p.page_fill[(int64_t)p.seq[b] * p.max_pages + pg] = (int32_t)(s - pg * P + 1);
+    }
+    const int D = p.head_dim;
+    const int vpr = D >> 3;
+    const int vpt = p.n_kv_heads * vpr;
+    const int lane = threadIdx.x & 31;
+    const int64_t rows = (int64_t)p.n_layers * 2 * p.B;
+    const int64_t head_stride_vec = P * D / 8;
+    for (int64_t r = gtid >> 5; r < rows; r += gsz >> 5) {
+        const int64_t lkv = r / p.B;
+        const int b = (int)(r - lkv * p.B);
+        const int l = (int)(lkv >> 1), kv = (int)(lkv & 1);
+        const uint4 *src = reinterpret_cast<const uint4 *>((kv ? p.v : p.k) + ((int64_t)l * p.B + b) * p.n_kv_heads * D);
+        const int64_t s = p.slot[b];
+        const int64_t row = s - (s / P) * P;
+        uint4 *dst = reinterpret_cast<uint4 *>(reinterpret_cast<uint16_t *>(p.pool) +
+                                               (((int64_t)lkv * p.pool_pages + p.pid[b]) * p.n_kv_heads) * P * D +
+                                               row * D);
+        for (int i = lane; i < vpt; i += 32) {
+            const int h = i / vpr, c = i - h * vpr;
+            __stcs(dst + h * head_stride_vec + c, __ldcs(src + i));
+        }
     }
 }
 
@@ -270,8 +327,16 @@ cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s) {
 }
 
 cudaError_t launch_append(const AppendParams &p, int n_sm, cudaStream_t s) {
-    const int64_t items = 2ll * p.n_layers * p.n * p.n_kv_heads * (p.head_dim / 8);
-    append_kernel<<<grid_for(items, 256, n_sm, 8), 256, 0, s>>>(p);
+    const int64_t rows = 2ll * p.n_layers * p.n;  // one warp each
+    static const int ctas_per_sm = env_knob("KVG_APPEND_CTAS_PER_SM", 2);
+    append_kernel<<<grid_for(rows, kAppendThreads / 32, n_sm, ctas_per_sm), kAppendThreads, 0, s>>>(p);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append_batch(const AppendBatchParams &p, int n_sm, cudaStream_t s) {
+    const int64_t rows = 2ll * p.n_layers * p.B;
+    append_batch_kernel<<<grid_for(rows, kAppendThreads / 32, n_sm, 8), kAppendThreads, 0, s>>>(p);
     count_launches(1);
     return cudaGetLastError();
 }

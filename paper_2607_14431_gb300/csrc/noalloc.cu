@@ -34,17 +34,6 @@ constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 void *g_scratch_dev[kMaxDevices] = {};
 
-// The split plan of kvg_decode_attention: about KVG_SPLIT_WAVES (default 16)
-// CTAs per SM over the whole call.
-int split_waves() {
-    static int w = [] {
-        const char *e = getenv("KVG_SPLIT_WAVES");
-        int v = e ? atoi(e) : 0;
-        return v > 0 ? v : 16;
-    }();
-    return w;
-}
-
 }  // namespace
 
 namespace kvg {
@@ -57,6 +46,8 @@ struct CacheShape {
 };
 bool cache_shape(const kvg_cache *c, CacheShape *out);
 int32_t cache_seq_pages(const kvg_cache *c, int32_t seq);
+int64_t cache_fill_rows(const kvg_cache *c, const int32_t *seq_ids, int64_t b0, int32_t nb, int tpp, int Lrun,
+                        BatchRows *rows);
 void set_last_error(const char *msg);
 }  // namespace kvg
 
@@ -83,38 +74,25 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
     if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out)) & 15)
         return reject(KVG_ERR_ARG, "q/out must be 16-byte aligned");
     if (cs.device < 0 || cs.device >= kMaxDevices) return reject(KVG_ERR_ARG, "device ordinal out of range");
-    int64_t max_np = 0, total_np = 0;
-    for (int32_t b = 0; b < B; ++b) {
+    for (int32_t b = 0; b < B; ++b)
         if (seq_ids[b] < 0 || seq_ids[b] >= cs.max_seqs) return reject(KVG_ERR_ARG, "bad seq id");
-        const int64_t np = cache_seq_pages(c, seq_ids[b]);
-        max_np = np > max_np ? np : max_np;
-        total_np += np;
-    }
     const int Lrun = layer < 0 ? cs.n_layers : 1;
     const int64_t bchunk = B < kMaxBatchPerLaunch ? B : kMaxBatchPerLaunch;
-    // bytes of one split's partials for the whole launch
-    const uint64_t per_split = (uint64_t)Lrun * bchunk * cs.n_kv_heads * G * ((uint64_t)cs.head_dim * 4 + 8);
-    // (m, l) start 256-byte aligned after o: keep 256 bytes of slack
-    const int64_t s_cap = (int64_t)((kScratchBytes - 256) / per_split);
-    if (s_cap < 1) {
-        char m[256];
+    // partials: (units + workers) slots of G * (4 * head_dim + 8) bytes; the
+    // (m, l) part starts 256-byte aligned after o, so keep 256 bytes of slack
+    const uint64_t per_slot = (uint64_t)G * ((uint64_t)cs.head_dim * 4 + 8);
+    const int64_t cap_slots = (int64_t)((kScratchBytes - 256) / per_slot);
+    const int64_t units = (int64_t)Lrun * bchunk * cs.n_kv_heads;
+    if (cap_slots - units < 1) {
+        char m[320];
         snprintf(m, sizeof m,
-                 "noalloc decode: %d layer(s) x %lld batch rows need %llu bytes of partials per split, "
-                 "above the %zu-byte static scratch; use kvg_decode_attention or fewer rows per call",
-                 Lrun, (long long)bchunk, (unsigned long long)per_split, kScratchBytes);
+                 "noalloc decode: %d layer(s) x %lld batch rows x %d kv heads need at least %llu bytes of "
+                 "partials, above the %zu-byte static scratch; use kvg_decode_attention or fewer rows per call",
+                 Lrun, (long long)bchunk, cs.n_kv_heads, (unsigned long long)((units + 1) * per_slot),
+                 kScratchBytes);
         return reject(KVG_ERR_CAPACITY, m);
     }
-    // same split plan as kvg_decode_attention, capped so the partials fit
-    const int64_t work = (int64_t)Lrun * cs.n_kv_heads * total_np;
-    const int64_t target = (int64_t)cs.n_sm * split_waves();
-    int64_t pps = work > 0 ? (work + target - 1) / target : 1;
-    if (pps < 1 || max_np == 0) pps = 1;
-    int64_t S = max_np > 0 ? (max_np + pps - 1) / pps : 1;
-    if (S > s_cap) {
-        S = s_cap;
-        pps = (max_np + S - 1) / S;
-        S = (max_np + pps - 1) / pps;
-    }
+    const int tpp = (cs.page_size + decode_tile_tokens(cs.head_dim) - 1) / decode_tile_tokens(cs.head_dim);
 
     int prev = -1;
     cudaGetDevice(&prev);
@@ -140,14 +118,19 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
         }
         scratch = g_scratch_dev[cs.device];
     }
-    const size_t units = (size_t)Lrun * bchunk * cs.n_kv_heads * S * G;
+    const int w_max = decode_max_warps(cs.head_dim, G, cs.n_sm);
+    if (w_max <= 0) return reject(KVG_ERR_CUDA, "decode kernel cannot be made resident");
+    const int64_t w_cap = cap_slots - units < w_max ? cap_slots - units : w_max;
+    const size_t slots = (size_t)units + (size_t)w_cap;
     float *part_o = static_cast<float *>(scratch);
     float2 *part_ml = reinterpret_cast<float2 *>(static_cast<unsigned char *>(scratch) +
-                                                 ((units * cs.head_dim * 4 + 255) / 256) * 256);
+                                                 ((slots * G * cs.head_dim * 4 + 255) / 256) * 256);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     for (int64_t b0 = 0; b0 < B; b0 += kMaxBatchPerLaunch) {
         const int32_t nb = (int32_t)((B - b0) < kMaxBatchPerLaunch ? (B - b0) : kMaxBatchPerLaunch);
         DecodeParams p{};
+        p.n_tiles = cache_fill_rows(c, seq_ids, b0, nb, tpp, Lrun, &p.rows);
+        p.n_warps = (int32_t)(p.n_tiles < w_cap ? (p.n_tiles > 1 ? p.n_tiles : 1) : w_cap);
         p.pool = cs.pool;
         p.pool_pages = cs.n_pages;
         p.n_kv_heads = cs.n_kv_heads;
@@ -156,8 +139,6 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
         p.layer0 = layer < 0 ? 0 : layer;
         p.n_layers_run = Lrun;
         p.B = nb;
-        p.n_splits = (int32_t)S;
-        p.pages_per_split = (int32_t)pps;
         p.page_table = cs.page_table;
         p.page_fill = cs.page_fill;
         p.max_pages = cs.max_pages;
@@ -167,24 +148,11 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
         p.qscale = scale * 1.4426950408889634f;
         p.part_o = part_o;
         p.part_ml = part_ml;
+        p.out = static_cast<__nv_bfloat16 *>(out);
         p.status = cs.status;
-        for (int32_t i = 0; i < nb; ++i) {
-            p.rows.seq[i] = seq_ids[b0 + i];
-            p.rows.npages[i] = cache_seq_pages(c, seq_ids[b0 + i]);
-        }
         cudaError_t e = launch_decode(cs.head_dim, G, p, st);
         if (e != cudaSuccess) return reject(KVG_ERR_CUDA, std::string("decode launch: ") + cudaGetErrorString(e));
-        CombineParams cp{};
-        cp.part_o = part_o;
-        cp.part_ml = part_ml;
-        cp.out = static_cast<__nv_bfloat16 *>(out);
-        cp.n_kv_heads = cs.n_kv_heads;
-        cp.n_q_heads = n_q_heads;
-        cp.n_splits = (int32_t)S;
-        cp.B = nb;
-        cp.q_row_stride_b = B;
-        cp.b0 = (int32_t)b0;
-        e = launch_combine(cs.head_dim, G, cp, Lrun, nb, st);
+        e = launch_combine(cs.head_dim, G, p, st);
         if (e != cudaSuccess) return reject(KVG_ERR_CUDA, std::string("combine launch: ") + cudaGetErrorString(e));
     }
     return KVG_OK;

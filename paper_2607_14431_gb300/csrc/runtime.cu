@@ -27,6 +27,11 @@ namespace kvg {
 static std::atomic<uint64_t> g_launches{0};
 void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 uint64_t launch_count() { return g_launches.load(std::memory_order_relaxed); }
+int env_knob(const char *name, int fallback) {
+    const char *e = getenv(name);
+    const int v = e ? atoi(e) : 0;
+    return v > 0 ? v : fallback;
+}
 }  // namespace kvg
 
 namespace {
@@ -584,6 +589,58 @@ extern "C" kvg_status kvg_cache_append(kvg_cache *c, int32_t seq, const void *k,
     return KVG_OK;
 }
 
+extern "C" kvg_status kvg_cache_append_batch(kvg_cache *c, const int32_t *seq_ids, int32_t B, const void *k,
+                                             const void *v, const int32_t *positions, void *stream) {
+    if (!c || !seq_ids || !k || !v || !positions) return fail(KVG_ERR_ARG, "null argument");
+    if (B <= 0 || B > kMaxBatchPerLaunch) return fail(KVG_ERR_ARG, "B must be in [1, %d]", kMaxBatchPerLaunch);
+    if ((reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(v)) & 15)
+        return fail(KVG_ERR_ARG, "k/v must be 16-byte aligned");
+    const int64_t P = c->dims.page_size;
+    std::vector<char> seen(c->max_seqs, 0);
+    int64_t need = 0;
+    for (int32_t b = 0; b < B; ++b) {
+        const int32_t sq = seq_ids[b];
+        if (sq < 0 || sq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq id %d", sq);
+        if (seen[sq]) return fail(KVG_ERR_ARG, "seq id %d repeated", sq);
+        seen[sq] = 1;
+        if (c->n_slots[sq] + 1 > c->max_slots) return fail(KVG_ERR_CAPACITY, "append past max_slots (seq %d)", sq);
+        if (c->n_slots[sq] % P == 0 && (int64_t)c->seq_pages[sq].size() * P <= c->n_slots[sq]) ++need;
+    }
+    if (need > (int64_t)c->free_list.size()) return fail(KVG_ERR_CAPACITY, "out of free pages");
+    DeviceGuard g(c->device);
+    AppendBatchParams p{};
+    p.k = static_cast<const uint16_t *>(k);
+    p.v = static_cast<const uint16_t *>(v);
+    p.pos = positions;
+    p.pool = c->pool;
+    p.pool_pages = c->n_pages;
+    p.n_layers = c->dims.n_layers;
+    p.n_kv_heads = c->dims.n_kv_heads;
+    p.page_size = (int32_t)P;
+    p.head_dim = c->dims.head_dim;
+    p.B = B;
+    p.max_pages = c->max_pages;
+    p.max_slots = c->max_slots;
+    p.page_table = c->page_table;
+    p.page_fill = c->page_fill;
+    p.positions = c->positions;
+    for (int32_t b = 0; b < B; ++b) {
+        const int32_t sq = seq_ids[b];
+        const int64_t s = c->n_slots[sq];
+        auto &sp = c->seq_pages[sq];
+        if ((int64_t)sp.size() * P <= s) {
+            sp.push_back(c->free_list.front());
+            c->free_list.pop_front();
+        }
+        p.seq[b] = sq;
+        p.pid[b] = sp[s / P];
+        p.slot[b] = (int32_t)s;
+        c->n_slots[sq] = (int32_t)(s + 1);
+    }
+    KVG_CUDA(launch_append_batch(p, c->n_sm, static_cast<cudaStream_t>(stream)));
+    return KVG_OK;
+}
+
 extern "C" kvg_status kvg_cache_release(kvg_cache *c, int32_t seq, void *stream) {
     if (!c) return fail(KVG_ERR_ARG, "null cache");
     if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d", seq);
@@ -808,13 +865,21 @@ extern "C" kvg_status kvg_verify(kvg_store *s, uint64_t block_id, kvg_cache *c, 
 
 // ------------------------------------------------------------------ decode --
 
-static int split_target_waves() {
-    static int w = [] {
-        const char *e = getenv("KVG_SPLIT_WAVES");
-        int v = e ? atoi(e) : 0;
-        return v > 0 ? v : 16;
-    }();
-    return w;
+// Fills the per-launch batch rows (sequence, pages, prefix sums of tiles) for
+// rows [b0, b0 + nb) and returns the launch's tile count.
+static int64_t fill_rows(const kvg_cache *c, const int32_t *seq_ids, int64_t b0, int32_t nb, int tpp,
+                         int Lrun, BatchRows *rows) {
+    int32_t acc = 0;
+    for (int32_t i = 0; i < nb; ++i) {
+        const int32_t sq = seq_ids[b0 + i];
+        const int32_t np = (int32_t)c->seq_pages[sq].size();
+        rows->seq[i] = sq;
+        rows->npages[i] = np;
+        rows->pref_tiles[i] = acc;
+        acc += np * tpp;
+    }
+    rows->pref_tiles[nb] = acc;
+    return (int64_t)Lrun * c->dims.n_kv_heads * acc;
 }
 
 extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
@@ -829,40 +894,31 @@ extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const in
     if (!decode_supported(d.head_dim, G)) return fail(KVG_ERR_ARG, "unsupported head_dim %d / group %d", d.head_dim, G);
     if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out)) & 15)
         return fail(KVG_ERR_ARG, "q/out must be 16-byte aligned");
-    int64_t max_np = 0, total_np = 0;
-    for (int32_t b = 0; b < B; ++b) {
+    for (int32_t b = 0; b < B; ++b)
         if (seq_ids[b] < 0 || seq_ids[b] >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq id %d", seq_ids[b]);
-        const int64_t np = (int64_t)c->seq_pages[seq_ids[b]].size();
-        max_np = std::max(max_np, np);
-        total_np += np;
-    }
     DeviceGuard g(c->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const int Lrun = layer < 0 ? d.n_layers : 1;
-    const int layer0 = layer < 0 ? 0 : layer;
-    // pages per split: about split_target_waves() CTAs per SM over the whole call
-    const int64_t work = (int64_t)Lrun * d.n_kv_heads * total_np;
-    const int64_t target = (int64_t)c->n_sm * split_target_waves();
-    int64_t pps = std::max<int64_t>(1, (work + target - 1) / target);
-    if (max_np == 0) pps = 1;
-    const int64_t S = std::max<int64_t>(1, (max_np + pps - 1) / pps);
+    const int tpp = (d.page_size + decode_tile_tokens(d.head_dim) - 1) / decode_tile_tokens(d.head_dim);
+    const int w_max = decode_max_warps(d.head_dim, G, c->n_sm);
+    if (w_max <= 0) return fail(KVG_ERR_CUDA, "decode kernel cannot be made resident");
     const int64_t bchunk = std::min<int64_t>(B, kMaxBatchPerLaunch);
-    const size_t units = (size_t)Lrun * bchunk * d.n_kv_heads * S * G;
-    KVG_CUDA(c->part_o.ensure(units * d.head_dim * sizeof(float)));
-    KVG_CUDA(c->part_ml.ensure(units * sizeof(float2)));
+    const size_t slots = (size_t)Lrun * bchunk * d.n_kv_heads + (size_t)w_max;
+    KVG_CUDA(c->part_o.ensure(slots * G * d.head_dim * sizeof(float)));
+    KVG_CUDA(c->part_ml.ensure(slots * G * sizeof(float2)));
     for (int64_t b0 = 0; b0 < B; b0 += kMaxBatchPerLaunch) {
         const int32_t nb = (int32_t)std::min<int64_t>(kMaxBatchPerLaunch, B - b0);
         DecodeParams p{};
+        p.n_tiles = fill_rows(c, seq_ids, b0, nb, tpp, Lrun, &p.rows);
+        p.n_warps = (int32_t)std::min<int64_t>(w_max, std::max<int64_t>(p.n_tiles, 1));
         p.pool = c->pool;
         p.pool_pages = c->n_pages;
         p.n_kv_heads = d.n_kv_heads;
         p.page_size = d.page_size;
         p.n_q_heads = n_q_heads;
-        p.layer0 = layer0;
+        p.layer0 = layer < 0 ? 0 : layer;
         p.n_layers_run = Lrun;
         p.B = nb;
-        p.n_splits = (int32_t)S;
-        p.pages_per_split = (int32_t)pps;
         p.page_table = c->page_table;
         p.page_fill = c->page_fill;
         p.max_pages = c->max_pages;
@@ -872,23 +928,10 @@ extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const in
         p.qscale = scale * 1.4426950408889634f;
         p.part_o = static_cast<float *>(c->part_o.ptr);
         p.part_ml = static_cast<float2 *>(c->part_ml.ptr);
+        p.out = static_cast<__nv_bfloat16 *>(out);
         p.status = c->status;
-        for (int32_t i = 0; i < nb; ++i) {
-            p.rows.seq[i] = seq_ids[b0 + i];
-            p.rows.npages[i] = (int32_t)c->seq_pages[seq_ids[b0 + i]].size();
-        }
         KVG_CUDA(launch_decode(d.head_dim, G, p, st));
-        CombineParams cp{};
-        cp.part_o = p.part_o;
-        cp.part_ml = p.part_ml;
-        cp.out = static_cast<__nv_bfloat16 *>(out);
-        cp.n_kv_heads = d.n_kv_heads;
-        cp.n_q_heads = n_q_heads;
-        cp.n_splits = (int32_t)S;
-        cp.B = nb;
-        cp.q_row_stride_b = B;
-        cp.b0 = (int32_t)b0;
-        KVG_CUDA(launch_combine(d.head_dim, G, cp, Lrun, nb, st));
+        KVG_CUDA(launch_combine(d.head_dim, G, p, st));
     }
     return KVG_OK;
 }
@@ -985,6 +1028,10 @@ bool cache_shape(const kvg_cache *c, CacheShape *out) {
     return true;
 }
 int32_t cache_seq_pages(const kvg_cache *c, int32_t seq) { return (int32_t)c->seq_pages[seq].size(); }
+int64_t cache_fill_rows(const kvg_cache *c, const int32_t *seq_ids, int64_t b0, int32_t nb, int tpp, int Lrun,
+                        BatchRows *rows) {
+    return fill_rows(c, seq_ids, b0, nb, tpp, Lrun, rows);
+}
 void set_last_error(const char *msg) { g_last_error = msg; }
 }  // namespace kvg
 

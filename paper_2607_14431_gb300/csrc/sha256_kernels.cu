@@ -28,11 +28,29 @@ __constant__ uint32_t kH0[8] = {0x6a09e667u, 0xbb67ae85u, 0x3c6ef372u, 0xa54ff53
 
 __device__ __forceinline__ uint32_t rotr(uint32_t x, int n) { return __funnelshift_r(x, x, n); }
 
+// The integer ALU pipe is this kernel's bottleneck while the FMA pipe idles.
+// Additions written as a*one + b and right shifts written as the high word of
+// a*2^(32-n) execute as IMAD on the FMA pipe.  `one` is a kernel argument
+// (always 1) so the compiler cannot fold the multiply back into an add.
+__device__ __forceinline__ uint32_t fadd(uint32_t a, uint32_t b, uint32_t one) {
+    uint32_t d;
+    asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(one), "r"(b));
+    return d;
+}
+template <int N>
+__device__ __forceinline__ uint32_t fshr(uint32_t x, uint32_t one) {
+    uint32_t d;
+    asm("mul.hi.u32 %0, %1, %2;" : "=r"(d) : "r"(x), "r"(one << (32 - N)));
+    return d;
+}
+
 __device__ __forceinline__ uint32_t bswap(uint32_t x) { return __byte_perm(x, 0, 0x0123); }
 
 // One compression of the 16-word block w (FIPS 180-4 sec. 6.2.2), with the
-// message schedule kept as a rolling 16-word window.
-__device__ __forceinline__ void compress(uint32_t st[8], uint32_t w[16]) {
+// message schedule kept as a rolling 16-word window.  Rotations and logic
+// stay on the ALU pipe; additions and the schedule's plain shifts go to the
+// FMA pipe (fadd/fshr), balancing the two.
+__device__ __forceinline__ void compress(uint32_t st[8], uint32_t w[16], uint32_t one) {
     uint32_t a = st[0], b = st[1], c = st[2], d = st[3], e = st[4], f = st[5], g = st[6], h = st[7];
 #pragma unroll
     for (int t = 0; t < 64; ++t) {
@@ -41,24 +59,23 @@ __device__ __forceinline__ void compress(uint32_t st[8], uint32_t w[16]) {
             wt = w[t];
         } else {
             const uint32_t w15 = w[(t - 15) & 15], w2 = w[(t - 2) & 15];
-            const uint32_t s0 = rotr(w15, 7) ^ rotr(w15, 18) ^ (w15 >> 3);
-            const uint32_t s1 = rotr(w2, 17) ^ rotr(w2, 19) ^ (w2 >> 10);
-            wt = w[t & 15] = w[t & 15] + s0 + w[(t - 7) & 15] + s1;
+            const uint32_t s0 = rotr(w15, 7) ^ rotr(w15, 18) ^ fshr<3>(w15, one);
+            const uint32_t s1 = rotr(w2, 17) ^ rotr(w2, 19) ^ fshr<10>(w2, one);
+            wt = w[t & 15] = fadd(fadd(w[t & 15], s0, one), fadd(w[(t - 7) & 15], s1, one), one);
         }
         const uint32_t S1 = rotr(e, 6) ^ rotr(e, 11) ^ rotr(e, 25);
         const uint32_t ch = (e & f) ^ (~e & g);
-        const uint32_t T1 = h + S1 + ch + kK[t] + wt;
+        const uint32_t T1 = fadd(fadd(h, S1, one), fadd(fadd(ch, kK[t], one), wt, one), one);
         const uint32_t S0 = rotr(a, 2) ^ rotr(a, 13) ^ rotr(a, 22);
         const uint32_t maj = (a & b) ^ (a & c) ^ (b & c);
-        const uint32_t T2 = S0 + maj;
         h = g;
         g = f;
         f = e;
-        e = d + T1;
+        e = fadd(d, T1, one);
         d = c;
         c = b;
         b = a;
-        a = T1 + T2;
+        a = fadd(T1, fadd(S0, maj, one), one);
     }
     st[0] += a;
     st[1] += b;
@@ -77,7 +94,7 @@ __device__ __forceinline__ void init_state(uint32_t st[8]) {
 
 // Final block(s) for a message whose last `rem` (< 64) bytes start at `tail`
 // and whose total length is `total_bytes`.
-__device__ void finish(uint32_t st[8], const uint8_t *tail, int rem, uint64_t total_bytes) {
+__device__ void finish(uint32_t st[8], const uint8_t *tail, int rem, uint64_t total_bytes, uint32_t one) {
     uint32_t w[16];
 #pragma unroll
     for (int i = 0; i < 16; ++i) w[i] = 0;
@@ -87,14 +104,14 @@ __device__ void finish(uint32_t st[8], const uint8_t *tail, int rem, uint64_t to
     if (rem < 56) {
         w[14] = (uint32_t)(bits >> 32);
         w[15] = (uint32_t)bits;
-        compress(st, w);
+        compress(st, w, one);
     } else {
-        compress(st, w);
+        compress(st, w, one);
 #pragma unroll
         for (int i = 0; i < 16; ++i) w[i] = 0;
         w[14] = (uint32_t)(bits >> 32);
         w[15] = (uint32_t)bits;
-        compress(st, w);
+        compress(st, w, one);
     }
 }
 
@@ -107,7 +124,7 @@ __device__ __forceinline__ const uint8_t *page_addr(const PageSource &s, int64_t
 
 __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src, int64_t n_pages,
                                                             int64_t leaves_per_page,
-                                                            uint32_t *__restrict__ out) {
+                                                            uint32_t *__restrict__ out, uint32_t one) {
     const int64_t n_leaves = n_pages * leaves_per_page;
     for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < n_leaves;
          idx += (int64_t)gridDim.x * blockDim.x) {
@@ -130,7 +147,7 @@ __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src
                 w[4 * q + 2] = bswap(x.z);
                 w[4 * q + 3] = bswap(x.w);
             }
-            compress(st, w);
+            compress(st, w, one);
         }
         const int rem = (int)(len & 63);
         if (rem == 0) {
@@ -141,9 +158,9 @@ __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src
             const uint64_t bits = len * 8ull;
             w[14] = (uint32_t)(bits >> 32);
             w[15] = (uint32_t)bits;
-            compress(st, w);
+            compress(st, w, one);
         } else {
-            finish(st, leaf + (len & ~63ull), rem, len);
+            finish(st, leaf + (len & ~63ull), rem, len, one);
         }
         uint4 *o = reinterpret_cast<uint4 *>(out + idx * 8);
         o[0] = make_uint4(st[0], st[1], st[2], st[3]);
@@ -157,7 +174,7 @@ __global__ void __launch_bounds__(128) sha256_pages_kernel(const uint32_t *__res
                                                            int64_t n_pages, int64_t m,
                                                            uint8_t *__restrict__ out,
                                                            const uint8_t *__restrict__ expected,
-                                                           DevStatus *status, int32_t seq) {
+                                                           DevStatus *status, int32_t seq, uint32_t one) {
     const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (p >= n_pages) return;
     const uint32_t *lw = leaf_words + p * m * 8;
@@ -176,7 +193,7 @@ __global__ void __launch_bounds__(128) sha256_pages_kernel(const uint32_t *__res
             w[4 * q + 2] = x.z;
             w[4 * q + 3] = x.w;
         }
-        compress(st, w);
+        compress(st, w, one);
     }
     {
         uint32_t w[16];
@@ -188,7 +205,7 @@ __global__ void __launch_bounds__(128) sha256_pages_kernel(const uint32_t *__res
         const uint64_t bits = (uint64_t)m * 32ull * 8ull;
         w[14] = (uint32_t)(bits >> 32);
         w[15] = (uint32_t)bits;
-        compress(st, w);
+        compress(st, w, one);
     }
     uint8_t dg[32];
 #pragma unroll
@@ -217,12 +234,14 @@ __global__ void __launch_bounds__(128) sha256_pages_kernel(const uint32_t *__res
 
 // Streaming single-thread hasher for seg0 || seg1 of arbitrary lengths.
 struct Stream {
+    uint32_t one;
     uint32_t st[8];
     uint32_t w[16];
     int fill;  // bytes in w
     uint64_t total;
 
-    __device__ void init() {
+    __device__ void init(uint32_t one_) {
+        one = one_;
         init_state(st);
         fill = 0;
         total = 0;
@@ -232,7 +251,7 @@ struct Stream {
     __device__ void byte(uint8_t x) {
         w[fill >> 2] |= (uint32_t)x << (24 - 8 * (fill & 3));
         if (++fill == 64) {
-            compress(st, w);
+            compress(st, w, one);
             fill = 0;
 #pragma unroll
             for (int i = 0; i < 16; ++i) w[i] = 0;
@@ -246,7 +265,7 @@ struct Stream {
             const uint32_t *q = reinterpret_cast<const uint32_t *>(ptr + k);
 #pragma unroll
             for (int i = 0; i < 16; ++i) w[i] = bswap(q[i]);
-            compress(st, w);
+            compress(st, w, one);
 #pragma unroll
             for (int i = 0; i < 16; ++i) w[i] = 0;
             k += 64;
@@ -269,10 +288,10 @@ struct Stream {
 
 __global__ void sha256_serial_kernel(const uint8_t *seg0, uint64_t n0, const uint8_t *seg1,
                                      uint64_t n1, uint8_t *out, const uint8_t *expected,
-                                     DevStatus *status) {
+                                     DevStatus *status, uint32_t one) {
     if (threadIdx.x != 0 || blockIdx.x != 0) return;
     Stream s;
-    s.init();
+    s.init(one);
     if (n0) s.feed(seg0, n0);
     if (n1) s.feed(seg1, n1);
     uint8_t dg[32];
@@ -297,9 +316,10 @@ cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_
     const int64_t n = n_pages * m;
     if (n == 0) return cudaSuccess;
     int64_t grid = (n + 127) / 128;
-    const int64_t cap = (int64_t)n_sm * 16;
+    static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 8);
+    const int64_t cap = (int64_t)n_sm * ctas_per_sm;
     if (grid > cap) grid = cap;
-    sha256_leaves_kernel<<<(int)grid, 128, 0, s>>>(src, n_pages, m, leaf_words);
+    sha256_leaves_kernel<<<(int)grid, 128, 0, s>>>(src, n_pages, m, leaf_words, 1u);
     count_launches(1);
     return cudaGetLastError();
 }
@@ -310,7 +330,7 @@ cudaError_t launch_sha256_pages(const uint32_t *leaf_words, int64_t n_pages, int
     if (n_pages == 0) return cudaSuccess;
     sha256_pages_kernel<<<(int)((n_pages + 127) / 128), 128, 0, s>>>(leaf_words, n_pages,
                                                                      leaves_per_page, out,
-                                                                     expected, status, seq);
+                                                                     expected, status, seq, 1u);
     count_launches(1);
     return cudaGetLastError();
 }
@@ -318,7 +338,7 @@ cudaError_t launch_sha256_pages(const uint32_t *leaf_words, int64_t n_pages, int
 cudaError_t launch_sha256_serial(const uint8_t *seg0, uint64_t n0, const uint8_t *seg1, uint64_t n1,
                                  uint8_t *out, const uint8_t *expected, DevStatus *status,
                                  cudaStream_t s) {
-    sha256_serial_kernel<<<1, 32, 0, s>>>(seg0, n0, seg1, n1, out, expected, status);
+    sha256_serial_kernel<<<1, 32, 0, s>>>(seg0, n0, seg1, n1, out, expected, status, 1u);
     count_launches(1);
     return cudaGetLastError();
 }

@@ -77,6 +77,7 @@ _SIGNATURES = {
     "kvg_cache_view_get": ([_vp, _P(kvg_cache_view)], _i32),
     "kvg_cache_seq_info": ([_vp, _i32, _P(_i32), _P(_i32)], _i32),
     "kvg_cache_append": ([_vp, _i32, _vp, _vp, _vp, _i32, _vp], _i32),
+    "kvg_cache_append_batch": ([_vp, _vp, _i32, _vp, _vp, _vp, _vp], _i32),
     "kvg_cache_release": ([_vp, _i32, _vp], _i32),
     "kvg_deposit": ([_vp, _vp, _i32, _i32, _i32, _vp, _P(_u64)], _i32),
     "kvg_graft": ([_vp, _u64, _vp, _i32, _i32, _i64, _u32, _vp, _P(kvg_graft_report)], _i32),
@@ -194,6 +195,11 @@ def kvg_cache_seq_info(cache, seq: int):
 
 def kvg_cache_append(cache, seq: int, k_ptr: int, v_ptr: int, pos_ptr: int, n: int, stream=None):
     _check(lib().kvg_cache_append(cache, seq, k_ptr, v_ptr, pos_ptr, n, _stream(stream)))
+
+
+def kvg_cache_append_batch(cache, seq_ids, k_ptr: int, v_ptr: int, pos_ptr: int, stream=None):
+    ids = (ctypes.c_int32 * len(seq_ids))(*[int(x) for x in seq_ids])
+    _check(lib().kvg_cache_append_batch(cache, ids, len(seq_ids), k_ptr, v_ptr, pos_ptr, _stream(stream)))
 
 
 def kvg_cache_release(cache, seq: int, stream=None):

@@ -1,0 +1,267 @@
+"""Parity at the benchmark's full sizes, in the launch configuration bench.py
+times (its workload classes build the state): bit-exact block bytes, page
+digests, page tables and restored pages against the oracle; attention and
+relocated keys on sampled (sequence, layer, head) outputs the oracle computes
+one by one; the grafted-vs-fresh SHA-256 gate and run-to-run determinism at
+32k context; the deep store's planted needles on every one of 1,000 grafts."""
+import hashlib
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import kvg_synth as syn
+from kvg_testlib import dev_view, need_gpu, tables
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _free_device_memory():
+    """Each workload takes most of the GPU: release what earlier tests cached."""
+    import gc
+    gc.collect()
+    if torch.cuda.is_available():
+        torch.cuda.empty_cache()
+    yield
+    gc.collect()
+    if torch.cuda.is_available():
+        torch.cuda.empty_cache()
+
+
+def _od(oracle, w):
+    return oracle.Dims(w.n_layers, w.n_kv_heads, w.head_dim, w.page_size, w.rope_theta, 0)
+
+
+def _pool_page(cache, w, l, kv, pid):
+    """Bytes of one (layer, K/V) page of the pool, as uint16 [Hkv][P][D]."""
+    v = cache.view
+    pb = w.page_bytes
+    off = ((l * 2 + kv) * v.n_pages + int(pid)) * pb
+    t = dev_view(v.pool + off, pb, torch.int16).cpu().numpy().view(np.uint16)
+    return t.reshape(w.n_kv_heads, w.page_size, w.head_dim)
+
+
+def _sha(t: torch.Tensor) -> bytes:
+    return hashlib.sha256(t.contiguous().view(torch.int16).cpu().numpy().tobytes()).digest()
+
+
+def _close(*objs):
+    for o in objs:
+        o.close()
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+
+
+def test_12b_single_graft_full_size(oracle):
+    kvg = need_gpu()
+    import bench
+    dev = torch.device("cuda", 0)
+    s, side = torch.cuda.Stream(), torch.cuda.Stream()
+    st = bench.Step12B(kvg, dev, s, side)
+    fresh = None
+    try:
+        st.run_step()
+        s.synchronize()
+        kvg.kvg_sync(st.cache.h, s, 60.0)  # every restored page matched its stored digest
+        w, nb, nf, P = st.w, st.nb, st.nf, st.w.page_size
+        kb, vb = syn.as_u16(st.kb), syn.as_u16(st.vb)
+        od = _od(oracle, w)
+        blk = oracle.block_from_kv(od, kb, vb, syn.positions(0, nb))
+        ser = blk.serialize()  # 12,288 page digests computed by the oracle
+        assert kvg.kvg_store_export(st.store.h, st.bid) == ser
+        assert kvg.kvg_store_export(st.hstore.h, st.hbid) == ser
+        # page tables, fills and position tags: the oracle's bookkeeping of the same calls
+        meta = oracle.OracleCache(od, st.cache.view.n_pages, 2, syn.B12_CTX, with_pool=False)
+        meta.append(1, None, None, syn.positions(0, nb))
+        meta.release(1)
+        meta.release(0)
+        meta.graft(0, oracle.BlockMeta(od, syn.positions(0, nb)))
+        meta.append(0, None, None, syn.positions(nb, nf))
+        pt, pf, ps = tables(st.cache)
+        assert np.array_equal(pt, meta.page_table) and np.array_equal(pf, meta.page_fill)
+        assert np.array_equal(ps, meta.positions)
+        # restored pages equal the block's pages: 48 sampled (layer, K/V, page)
+        rng = np.random.default_rng(1)
+        for _ in range(48):
+            l, kv, j = int(rng.integers(w.n_layers)), int(rng.integers(2)), int(rng.integers(nb // P))
+            assert np.array_equal(_pool_page(st.cache, w, l, kv, pt[0, j]), blk.pages[l, kv, j])
+        # decode: sampled heads against fp64 attention over all 32,768 rows
+        kf, vf = st.kf, st.vf
+        for l, h in [(0, 0), (17, 5), (w.n_layers - 1, w.n_q_heads - 1)]:
+            g = h // w.group
+            k = np.concatenate([kb[l, :, g], syn.as_u16(kf[l, :, g])])
+            v = np.concatenate([vb[l, :, g], syn.as_u16(vf[l, :, g])])
+            ref = oracle.attention_head(syn.as_u16(st.q[l, 0, h]), k, v, st.scale)
+            got = oracle.bf16_to_f64(syn.as_u16(st.out[l, 0, h]))
+            assert np.abs(got - ref).max() <= 1e-2
+        # the same 32,768 rows written fresh into other pages: SHA-256-identical output
+        out_grafted = st.out.clone()
+        fresh = kvg.Cache(st.dims, st.cache.view.n_pages, 1, syn.B12_CTX)
+        kvg.kvg_cache_set_free_order(fresh.h, syn.permutation(st.cache.view.n_pages, 5))
+        pb_ = torch.arange(nb, dtype=torch.int32, device=dev)
+        kvg.kvg_cache_append(fresh.h, 0, st.kb.data_ptr(), st.vb.data_ptr(), pb_.data_ptr(), nb, s)
+        kvg.kvg_cache_append(fresh.h, 0, kf.data_ptr(), vf.data_ptr(), st.pf.data_ptr(), nf, s)
+        out_fresh = torch.empty_like(st.q)
+        kvg.kvg_decode_attention(fresh.h, -1, [0], st.q.data_ptr(), w.n_q_heads, out_fresh.data_ptr(),
+                                 st.scale, s)
+        s.synchronize()
+        assert _sha(out_fresh) == _sha(out_grafted)
+        # run-to-run: two more full steps give the same bytes
+        for _ in range(2):
+            st.run_step()
+            s.synchronize()
+            assert _sha(st.out) == _sha(out_grafted)
+    finally:
+        _close(*(x for x in (fresh, st.cache, st.store, st.hstore) if x is not None))
+
+
+def test_31b_relocation_full_size(oracle):
+    kvg = need_gpu()
+    import bench
+    dev = torch.device("cuda", 0)
+    s = torch.cuda.Stream()
+    st = bench.Step31B(kvg, dev, s)
+    try:
+        st.run_step()
+        s.synchronize()
+        kvg.kvg_sync(st.cache.h, s, 60.0)
+        w, nb, P = st.w, st.nb, st.w.page_size
+        pt, pf, ps = tables(st.cache)
+        kb = torch.cat([k for k, _ in st.blk_sample], dim=1)[:, :, 0]  # [L][nb][D], kv head 0
+        vb = torch.cat([v for _, v in st.blk_sample], dim=1)[:, :, 0]
+        # position tags: block tags + delta, then the fresh rows' tags
+        for sq in range(st.B):
+            d = st.deltas[sq]
+            assert np.array_equal(ps[sq, :nb], np.arange(nb) + d)
+            assert np.array_equal(ps[sq, nb:st.ctx], np.arange(nb, st.ctx) + d)
+        assert np.array_equal(ps[st.B, :nb], np.arange(nb) + 4096)  # the timed relocation
+        # relocated keys (kv head 0) within 2e-2 of the fp64 rotation; values bit-exact
+        rng = np.random.default_rng(3)
+        for sq, d in [(3, st.deltas[3]), (1, st.deltas[1]), (0, 0), (st.B, 4096)]:
+            for _ in range(6):
+                l, j = int(rng.integers(w.n_layers)), int(rng.integers(nb // P))
+                kpage = _pool_page(st.cache, w, l, 0, pt[sq, j])[0]
+                vpage = _pool_page(st.cache, w, l, 1, pt[sq, j])[0]
+                rows_k = syn.as_u16(kb[l, j * P:(j + 1) * P])
+                rows_v = syn.as_u16(vb[l, j * P:(j + 1) * P])
+                assert np.array_equal(vpage, rows_v)
+                if d == 0:
+                    assert np.array_equal(kpage, rows_k)
+                else:
+                    ref = oracle.rope_rotate_rows(rows_k, d, w.rope_theta, 0)
+                    assert np.abs(oracle.bf16_to_f64(kpage) - ref).max() <= 2e-2
+        # decode: sampled (sequence, layer) for query head 0 against fp64 attention
+        for sq in (0, 3, 6):
+            fr = [st.fresh[(sq * 7 + i) % len(st.fresh)] for i in range((st.ctx - nb) // st.CHUNK)]
+            for l in (0, w.n_layers - 1):
+                kblk = syn.as_u16(kb[l])
+                if st.deltas[sq]:
+                    kblk = oracle.rope_rotate_rows_bf16(kblk, st.deltas[sq], w.rope_theta, 0)
+                k = np.concatenate([kblk] + [syn.as_u16(f[0][l, :, 0]) for f in fr])
+                v = np.concatenate([syn.as_u16(vb[l])] + [syn.as_u16(f[1][l, :, 0]) for f in fr])
+                ref = oracle.attention_head(syn.as_u16(st.q[l, sq, 0]), k, v, st.scale)
+                got = oracle.bf16_to_f64(syn.as_u16(st.out[l, sq, 0]))
+                assert np.abs(got - ref).max() <= 1e-2
+    finally:
+        _close(st.cache, st.store)
+
+
+def test_batched_library_full_size(oracle):
+    kvg = need_gpu()
+    import bench
+    dev = torch.device("cuda", 0)
+    s = torch.cuda.Stream()
+    st = bench.StepBatched(kvg, dev, s, 4)
+    try:
+        st.run_step()
+        s.synchronize()
+        kvg.kvg_sync(st.cache.h, s, 60.0)
+        w, P, nS = st.w, st.w.page_size, syn.BATCHED_SEQS
+        od = _od(oracle, w)
+        # page tables, fills, positions: the oracle's bookkeeping of the same calls
+        meta = oracle.OracleCache(od, st.cache.view.n_pages, nS + 1, st.max_slots, with_pool=False)
+        for n in st.lens:
+            meta.append(nS, None, None, syn.positions(0, int(n)))
+            meta.release(nS)
+        for sq in range(nS):
+            meta.release(sq)
+            for b in st.ids[sq]:
+                meta.graft(sq, oracle.BlockMeta(od, syn.positions(0, int(st.lens[b]))))
+        posn = st.pos.cpu().numpy()
+        for t in range(st.steps):  # one decode-step row per sequence, in batch order
+            for sq in range(nS):
+                meta.append(sq, None, None, posn[t, sq:sq + 1])
+        pt, pf, ps = tables(st.cache)
+        assert np.array_equal(pt, meta.page_table) and np.array_equal(pf, meta.page_fill)
+        assert np.array_equal(ps, meta.positions)
+        # grafted pages equal the deposited blocks' pages (sampled), incl. ragged tail pages
+        for sq in (0, 13, nS - 1):
+            j0 = 0
+            for b in st.ids[sq]:
+                n = int(st.lens[b])
+                k, v = syn.kv_rows(w, n, w.seed + int(b), "cuda")
+                blk = oracle.block_from_kv(od, syn.as_u16(k), syn.as_u16(v), syn.positions(0, n))
+                for j in (0, blk.n_pages - 1):
+                    for kv in (0, 1):
+                        got = _pool_page(st.cache, w, w.n_layers - 1, kv, pt[sq, j0 + j])
+                        want = blk.pages[w.n_layers - 1, kv, j]
+                        if j == blk.n_pages - 1 and n % P:
+                            # the tail page's fill rows are the block's; later rows
+                            # belong to the decode appends of the last block only
+                            got, want = got[:, :n % P], want[:, :n % P]
+                        assert np.array_equal(got, want)
+                j0 += blk.n_pages
+        # decode after the last step: sampled heads against fp64 attention
+        for sq in (0, nS - 1):
+            for l in (0, w.n_layers - 1):
+                ks, vs = [], []
+                for b in st.ids[sq]:
+                    k, v = syn.kv_rows(w, int(st.lens[b]), w.seed + int(b), "cuda")
+                    ks.append(syn.as_u16(k[l, :, 0]))
+                    vs.append(syn.as_u16(v[l, :, 0]))
+                ks.append(syn.as_u16(st.kd[l, sq::nS, 0]))
+                vs.append(syn.as_u16(st.vd[l, sq::nS, 0]))
+                ref = oracle.attention_head(syn.as_u16(st.q[l, sq, 0]), np.concatenate(ks), np.concatenate(vs),
+                                            st.scale)
+                got = oracle.bf16_to_f64(syn.as_u16(st.out[l, sq, 0]))
+                assert np.abs(got - ref).max() <= 1e-2
+    finally:
+        _close(st.cache, st.store)
+
+
+def test_deep_store_needles_full_size(oracle):
+    kvg = need_gpu()
+    import bench
+    dev = torch.device("cuda", 0)
+    s = torch.cuda.Stream()
+    st = bench.StepDeep(kvg, dev, s)
+    try:
+        w = st.w
+        od = _od(oracle, w)
+        # blocks at several depths: serialized bytes equal the oracle's block
+        for b in (0, 697, st.n_blocks - 1):
+            k, v = st.block_rows(b, dev)
+            blk = oracle.block_from_kv(od, syn.as_u16(k), syn.as_u16(v), syn.positions(0, st.nb))
+            assert kvg.kvg_store_export(st.store.h, b) == blk.serialize()
+        # every one of the 1,000 random grafts reads its own block's needle
+        # (and so not the previous block's: the window really moves)
+        prev = None
+        for _ in range(len(st.order)):
+            b = st.run_step()
+            s.synchronize()
+            assert st.needle_error(b) <= 1e-2, b
+            if prev is not None and st.tag(prev) != st.tag(b):
+                assert float((st.out.float() - st.tag(prev)).abs().max()) > 1e-2
+            prev = b
+        # the needle read matches fp64 attention over the grafted rows (sampled)
+        b = int(st.order[-1])
+        k, v = st.block_rows(b, dev)
+        for l, h in [(0, 0), (1, w.n_q_heads - 1)]:
+            g = h // w.group
+            ref = oracle.attention_head(syn.as_u16(st.q[l, 0, h]), syn.as_u16(k[l, :, g]), syn.as_u16(v[l, :, g]),
+                                        st.scale)
+            assert np.abs(oracle.bf16_to_f64(syn.as_u16(st.out[l, 0, h])) - ref).max() <= 1e-2
+    finally:
+        _close(st.cache, st.store)

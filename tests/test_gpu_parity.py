@@ -338,3 +338,35 @@ def test_host_checks_reject_bad_calls(oracle):
     with pytest.raises(E) as e:
         kvg.kvg_cache_set_free_order(s["src"].h, list(range(s["n_pages"])))  # pages in use
     assert e.value.status == kvg.KVG_ERR_ARG
+
+
+def test_append_batch_matches_oracle(oracle):
+    kvg = need_gpu()
+    w = geometry("d128")
+    dims = dims_for(kvg, w)
+    lens = [63, 64, 1, 130]  # one row lands in a fresh page, one mid-page
+    max_slots = 256
+    n_pages = 20
+    cache = kvg.Cache(dims, n_pages, 5, max_slots)
+    fill_canary(cache)
+    od = oracle_dims(oracle, w)
+    oc = oracle.OracleCache(od, n_pages, 5, max_slots, fill=CANARY)
+    for i, n in enumerate(lens):
+        k, v = _kv(w, n, 90 + i)
+        append(kvg, cache, i, k, v, syn.positions(0, n))
+        oc.append(i, k, v, syn.positions(0, n))
+    seqs = [3, 0, 1, 2]
+    for step in range(3):
+        k, v = _kv(w, len(seqs), 95 + step)  # [L][B][Hkv][D]: one row per sequence
+        pos = np.array([1000 + 10 * step + b for b in range(len(seqs))], np.int32)
+        kd, vd, pd = to_dev(k), to_dev(v), to_dev(pos)
+        kvg.kvg_cache_append_batch(cache.h, seqs, kd.data_ptr(), vd.data_ptr(), pd.data_ptr())
+        torch.cuda.synchronize()
+        oc.append_batch(seqs, k, v, pos)
+    assert np.array_equal(pool_u16(cache, w), oc.pool)
+    pt, pf, ps = tables(cache)
+    assert np.array_equal(pt, oc.page_table) and np.array_equal(pf, oc.page_fill)
+    assert np.array_equal(ps, oc.positions)
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_cache_append_batch(cache.h, [0, 0], kd.data_ptr(), vd.data_ptr(), pd.data_ptr())
+    assert e.value.status == kvg.KVG_ERR_ARG
