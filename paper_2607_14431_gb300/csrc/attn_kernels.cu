@@ -7,26 +7,31 @@
 // rows.  The kernel launches W one-warp CTAs, all co-resident; warp w takes
 // the contiguous range [w*T/W, (w+1)*T/W) of the T tiles, so every warp gets
 // the same share and there is no tail wave.  A warp is an independent
-// pipeline: lane 0 issues bulk asynchronous copies (cp.async.bulk, completion
-// on an mbarrier, bounded wait) of the K and V rows of a tile into a
-// STAGES-deep shared-memory ring, STAGES-1 tiles ahead, across unit
-// boundaries; the 32 lanes consume them:
-//   - lanes form 4 groups of 8; a group owns every 4th row of the tile and
-//     each lane 8*D/64 dimensions in 16-byte chunks j, j+8, ... (a group's 8
-//     lanes read one contiguous 128-byte span: no bank conflicts);
-//   - q.k partial sums are all-reduced over the group with 3 xor shuffles;
-//   - each group keeps an online-softmax state (running max m, sum l, fp32
-//     output o) for all G query heads of the kv head (K/V read once) and
-//     rescales o only when the running max grows (the skipped factor is
-//     exactly 1);
-//   - when the warp leaves a unit it merges its 4 groups in a fixed order and
-//     writes the unit's partial (o, m, l) to slot unit + w.
-// The combine kernel merges, for each unit, the partials of the warps that
-// covered it, in warp order.  Every reduction order is a function of logical
-// token indices and of (T, W) only — never of physical page ids — so results
-// are bitwise reproducible and identical for grafted and freshly written rows.
-// G = 2 fills 2 of 16 rows of an MMA tile; at ~2 flop per byte the CUDA cores
-// keep up with HBM, so the contraction stays on the FMA pipe.
+// pipeline over a STAGES-deep shared-memory ring: for each tile lane 0 issues
+// 2-D tensor copies (TMA, cp.async.bulk.tensor, completion on an mbarrier,
+// bounded wait) of the K and V rows as boxes of 64 columns x TOK rows with the
+// 128-byte swizzle, so the 8-row ldmatrix reads below hit 8 different bank
+// groups; value rows past the page's fill are zeroed after arrival and the
+// scores of those rows are masked.
+//
+// The contractions run on the tensor cores with mma.sync m16n8k16 (bf16 in,
+// fp32 accumulate).  Each tile is bandwidth-bound (~2 flop per byte at G = 2),
+// so the point is not FLOPs but instruction count: a 16-row sub-tile costs
+// D/16 MMAs for q.k and D/16 for p.v instead of ~1,400 scalar instructions.
+//   S[16 tok][8] = K[16][D] . Q^T[D][8]  (A = K rows, B = the G query heads of
+//                                          the kv head, padded with zeros)
+//   O^T[D][8] += V^T[D][16] . P^T[16][8] (A = V rows, transposed by ldmatrix;
+//                                          B = the bf16-rounded weights P)
+// The online softmax is per head in fp32: scores are scaled by scale*log2(e),
+// the running max m is reduced across the 8 lanes holding a head's column, O
+// is rescaled only when m grows (the skipped factor is exactly 1), and the
+// running sum l adds the same bf16-rounded weights the MMA uses.  When the
+// warp leaves a unit it writes that unit's partial (o, m, l) to slot unit + w;
+// the combine kernel merges, for each unit, the partials of the warps that
+// covered it, in warp order.  Every order of operations is a function of
+// logical token indices and of (T, W) only — never of physical page ids — so
+// results are bitwise reproducible and identical for grafted and freshly
+// written rows.
 #include <math.h>
 
 #include "common.cuh"
@@ -39,43 +44,30 @@ template <int D>
 struct TileShape;
 template <>
 struct TileShape<64> {
-    static constexpr int TOK = 32, STAGES = 3;
+    static constexpr int TOK = 64, STAGES = 3;
 };
 template <>
 struct TileShape<128> {
-    static constexpr int TOK = 32, STAGES = 2;
+    static constexpr int TOK = 32, STAGES = 3;
 };
 template <>
 struct TileShape<256> {
-    static constexpr int TOK = 16, STAGES = 2;
+    static constexpr int TOK = 16, STAGES = 3;
 };
 
 template <int D>
 struct Cfg {
     static constexpr int TOK = TileShape<D>::TOK;
     static constexpr int STAGES = TileShape<D>::STAGES;
-    static constexpr int NCH = D / 64;              // 16-byte chunks per lane per row
-    static constexpr int TILE_BYTES = TOK * D * 2;  // one K (or V) tile
-    static constexpr int STAGE_BYTES = 2 * TILE_BYTES;
+    static constexpr int NB = D / 64;                  // 64-column boxes per K (or V) tile
+    static constexpr int BOX = TOK * 128;              // bytes of one box (TOK rows x 128 B)
+    static constexpr int STAGE_BYTES = 2 * NB * BOX;   // K boxes then V boxes
     static constexpr int RING_BYTES = STAGES * STAGE_BYTES;
-    static constexpr int SMEM = RING_BYTES + STAGES * (8 + 4);
+    static constexpr int SMEM = RING_BYTES + STAGES * (8 + 4) + 1024;  // + alignment slack
+    static constexpr int KS = D / 16;                  // k-steps of q.k, m-tiles of p.v
+    static constexpr int SUB = TOK / 16;               // 16-row sub-tiles per tile
+    static_assert(BOX % 1024 == 0, "a swizzle atom is 8 rows of 128 bytes");
 };
-
-__device__ __forceinline__ void unpack8(const uint4 &v, float *f) {
-    const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&v);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const float2 t = __bfloat1622float2(h[i]);
-        f[2 * i] = t.x;
-        f[2 * i + 1] = t.y;
-    }
-}
-
-// Weighted sum x*a + y*b with an operation order that is symmetric in the two
-// operands, so both partners of a shuffle merge compute identical bits.
-__device__ __forceinline__ float wsum(float x, float a, float y, float b) {
-    return __fadd_rn(__fmul_rn(x, a), __fmul_rn(y, b));
-}
 
 // Position of global tile t: unit (lr, b, g) and tile index within the unit.
 struct TilePos {
@@ -109,15 +101,46 @@ __device__ __forceinline__ TilePos locate(const DecodeParams &p, int64_t t) {
 
 __device__ __forceinline__ int64_t warp_start(int64_t w, int64_t T, int64_t W) { return w * T / W; }
 
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+// D += A(16x16, row) . B(16x8, col), bf16 inputs, fp32 accumulators.
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t x) { return __uint_as_float(x << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t x) { return __uint_as_float(x & 0xffff0000u); }
+
 template <int D, int G>
-__global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p) {
+__global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const __grid_constant__ CUtensorMap pool_map) {
     using C = Cfg<D>;
-    constexpr int TOK = C::TOK, STAGES = C::STAGES, NCH = C::NCH;
-    constexpr int TPG = TOK / 4;  // rows per lane group per tile
-    extern __shared__ __align__(128) uint8_t smem[];
+    constexpr int TOK = C::TOK, STAGES = C::STAGES, KS = C::KS, SUB = C::SUB, NB = C::NB, BOX = C::BOX;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    // swizzled boxes must start on a 1024-byte boundary
+    uint8_t *smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
 
     const int lane = threadIdx.x;
-    const int grp = lane >> 3, lj = lane & 7;
+    const int gq = lane >> 2, tq = lane & 3;  // mma fragment coordinates
     const int64_t w = blockIdx.x;
     const int64_t t0 = warp_start(w, p.n_tiles, p.n_warps);
     const int64_t t1 = warp_start(w + 1, p.n_tiles, p.n_warps);
@@ -134,10 +157,10 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p) {
     }
     __syncwarp();
 
-    const int64_t plane_elems = p.pool_pages * (int64_t)p.n_kv_heads * P * D;
-    const __nv_bfloat16 *poolh = reinterpret_cast<const __nv_bfloat16 *>(p.pool);
+    const int64_t plane_rows = p.pool_pages * (int64_t)p.n_kv_heads * P;  // rows per (layer, K/V)
 
-    auto issue = [&](int64_t t, int stg) {  // lane 0
+    // lane 0: arm the stage's barrier and copy the tile's K and V boxes
+    auto issue = [&](int64_t t, int stg) {
         const TilePos tp = locate(p, t);
         const int seq = p.rows.seq[tp.b];
         const int jj = tp.tile / tpp;
@@ -153,60 +176,50 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p) {
         vrs[stg] = vr;
         uint64_t *bar = &bars[stg];
         if (vr > 0) {
-            const uint32_t bytes = (uint32_t)vr * D * 2;
-            mbar_arrive_expect_tx(bar, 2 * bytes);
+            mbar_arrive_expect_tx(bar, (uint32_t)C::STAGE_BYTES);
             const int l = p.layer0 + tp.lr;
-            const __nv_bfloat16 *ks = poolh + (int64_t)(2 * l) * plane_elems +
-                                      ((int64_t)pid * p.n_kv_heads + tp.g) * P * D + (int64_t)k * TOK * D;
+            const int32_t row_k = (int32_t)((2 * l) * plane_rows + ((int64_t)pid * p.n_kv_heads + tp.g) * P +
+                                            (int64_t)k * TOK);
+            const int32_t row_v = (int32_t)(row_k + plane_rows);
             uint8_t *dst = ring + stg * C::STAGE_BYTES;
-            bulk_g2s(dst, ks, bytes, bar);
-            bulk_g2s(dst + C::TILE_BYTES, ks + plane_elems, bytes, bar);
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+                tma_load_2d(dst + b * BOX, &pool_map, 64 * b, row_k, bar);
+                tma_load_2d(dst + (NB + b) * BOX, &pool_map, 64 * b, row_v, bar);
+            }
         } else {
             mbar_arrive(bar);
         }
     };
 
-    float qf[G][NCH][8];
-    float m[G], lsum[G], o[G][NCH][8];
+    uint32_t qb[KS][2];   // B fragments of q (heads gq < G), per k-step
+    float o[KS][4];       // O^T accumulators: dims 16*mt + gq (+8), heads 2*tq (+1)
+    float m[2], lsum[2];  // running max / partial sum of heads 2*tq, 2*tq+1
     int64_t cur_unit = -1;
 
     auto flush = [&](int64_t unit) {
-        // merge the 4 lane groups: (0,1),(2,3) then (01,23)
+        float lt[2];
 #pragma unroll
-        for (int off = 8; off <= 16; off <<= 1) {
-#pragma unroll
-            for (int h = 0; h < G; ++h) {
-                const float mo = __shfl_xor_sync(0xffffffffu, m[h], off);
-                const float lo = __shfl_xor_sync(0xffffffffu, lsum[h], off);
-                const float mn = fmaxf(m[h], mo);
-                const float a = m[h] == -INFINITY ? 0.f : exp2f(m[h] - mn);
-                const float bb = mo == -INFINITY ? 0.f : exp2f(mo - mn);
-                lsum[h] = wsum(lsum[h], a, lo, bb);
-#pragma unroll
-                for (int c = 0; c < NCH; ++c)
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const float oo = __shfl_xor_sync(0xffffffffu, o[h][c][e], off);
-                        o[h][c][e] = wsum(o[h][c][e], a, oo, bb);
-                    }
-                m[h] = mn;
-            }
+        for (int e = 0; e < 2; ++e) {
+            float v = lsum[e];
+            v += __shfl_xor_sync(0xffffffffu, v, 4);
+            v += __shfl_xor_sync(0xffffffffu, v, 8);
+            v += __shfl_xor_sync(0xffffffffu, v, 16);
+            lt[e] = v;
         }
         const int64_t slot = unit + w;
-        if (lane < 8) {
 #pragma unroll
-            for (int h = 0; h < G; ++h) {
+        for (int e = 0; e < 2; ++e) {
+            const int h = 2 * tq + e;
+            if (h < G) {
                 float *dst = p.part_o + (slot * G + h) * D;
 #pragma unroll
-                for (int c = 0; c < NCH; ++c) {
-                    float4 *d4 = reinterpret_cast<float4 *>(dst + 8 * (lj + 8 * c));
-                    d4[0] = make_float4(o[h][c][0], o[h][c][1], o[h][c][2], o[h][c][3]);
-                    d4[1] = make_float4(o[h][c][4], o[h][c][5], o[h][c][6], o[h][c][7]);
+                for (int mt = 0; mt < KS; ++mt) {
+                    dst[16 * mt + gq] = o[mt][e];
+                    dst[16 * mt + gq + 8] = o[mt][2 + e];
                 }
+                if (gq == 0) p.part_ml[slot * G + h] = make_float2(m[e], lt[e]);
             }
-            if (lane == 0)
-#pragma unroll
-                for (int h = 0; h < G; ++h) p.part_ml[slot * G + h] = make_float2(m[h], lsum[h]);
         }
     };
 
@@ -214,26 +227,25 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p) {
         const __nv_bfloat16 *qrow =
             p.q + ((int64_t)(tp.lr * p.q_row_stride_b + p.b0 + tp.b) * p.n_q_heads + tp.g * G) * D;
 #pragma unroll
-        for (int h = 0; h < G; ++h) {
-            m[h] = -INFINITY;
-            lsum[h] = 0.f;
-#pragma unroll
-            for (int c = 0; c < NCH; ++c) {
-                const uint4 v = *reinterpret_cast<const uint4 *>(qrow + h * D + 8 * (lj + 8 * c));
-                unpack8(v, qf[h][c]);
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    qf[h][c][e] *= p.qscale;
-                    o[h][c][e] = 0.f;
-                }
+        for (int ks = 0; ks < KS; ++ks) {
+            if (gq < G) {
+                const uint32_t *q32 = reinterpret_cast<const uint32_t *>(qrow + gq * D + 16 * ks + 2 * tq);
+                qb[ks][0] = q32[0];
+                qb[ks][1] = q32[4];  // dims + 8
+            } else {
+                qb[ks][0] = qb[ks][1] = 0u;
             }
+#pragma unroll
+            for (int c = 0; c < 4; ++c) o[ks][c] = 0.f;
         }
+        m[0] = m[1] = -INFINITY;
+        lsum[0] = lsum[1] = 0.f;
     };
 
-    if (lane == 0) {
+    if (lane == 0)
         for (int i = 0; i < STAGES && t0 + i < t1; ++i) issue(t0 + i, i);
-    }
 
+    const uint32_t ring_s = smem_addr(ring);
     bool alive = true;
     int64_t unit_end = t0;  // first tile past the current unit
     for (int64_t t = t0; t < t1; ++t) {
@@ -254,92 +266,116 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p) {
             break;
         }
         const int vr = vrs[stg];
+        bool zeroed = false;
+        if (vr > 0 && vr < TOK) {
+            // value rows past the fill hold whatever the pool had there: zero
+            // them so their zero weights contribute exactly 0
+            uint4 *vz = reinterpret_cast<uint4 *>(ring + stg * C::STAGE_BYTES + NB * BOX);
+            for (int idx = lane; idx < NB * (TOK - vr) * 8; idx += 32) {
+                const int b = idx / ((TOK - vr) * 8);
+                const int rem = idx - b * (TOK - vr) * 8;
+                vz[(b * BOX + (vr + rem / 8) * 128) / 16 + (rem & 7)] = make_uint4(0, 0, 0, 0);
+            }
+            fence_proxy_async_shared();
+            zeroed = true;
+            __syncwarp();
+        }
         if (vr > 0) {
-            const __nv_bfloat16 *Ks = reinterpret_cast<const __nv_bfloat16 *>(ring + stg * C::STAGE_BYTES);
-            const __nv_bfloat16 *Vs = Ks + TOK * D;
-            float s[TPG][G];
+            const uint32_t ks_base = ring_s + stg * C::STAGE_BYTES;
+            const uint32_t vs_base = ks_base + NB * BOX;
+            // ---- scores S[16 rows][8 heads] per sub-tile
+            float sc[SUB][4];
 #pragma unroll
-            for (int i4 = 0; i4 < TPG; ++i4) {
-                const int ti = i4 * 4 + grp;
-                float acc[G];
+            for (int sb = 0; sb < SUB; ++sb) {
+                float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
+                // lane -> row of its 8x8 matrix (rows +8 for matrices 1,3) and
+                // 16-byte chunk (+1 for matrices 2,3), swizzled: chunk ^ (row & 7)
+                const uint32_t a_row = ks_base + (16 * sb + (lane & 7) + ((lane >> 3) & 1) * 8) * 128;
+                const int a_hi = (lane >> 4) & 1;
 #pragma unroll
-                for (int h = 0; h < G; ++h) acc[h] = 0.f;
-                if (ti < vr) {
-#pragma unroll
-                    for (int c = 0; c < NCH; ++c) {
-                        const uint4 kv = *reinterpret_cast<const uint4 *>(Ks + ti * D + 8 * (lj + 8 * c));
-                        float kf[8];
-                        unpack8(kv, kf);
-#pragma unroll
-                        for (int h = 0; h < G; ++h)
-#pragma unroll
-                            for (int e = 0; e < 8; ++e) acc[h] = fmaf(qf[h][c][e], kf[e], acc[h]);
-                    }
+                for (int ks = 0; ks < KS; ++ks) {
+                    uint32_t a0, a1, a2, a3;
+                    const int chunk = ((ks & 3) << 1) + a_hi;
+                    ldsm_x4(a_row + (ks >> 2) * BOX + ((chunk ^ (lane & 7)) << 4), a0, a1, a2, a3);
+                    if (ks & 1)
+                        mma_bf16(acc1, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+                    else
+                        mma_bf16(acc0, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
                 }
+                const int r0 = 16 * sb + gq, r1 = r0 + 8;
+                sc[sb][0] = r0 < vr ? (acc0[0] + acc1[0]) * p.qscale : -INFINITY;
+                sc[sb][1] = r0 < vr ? (acc0[1] + acc1[1]) * p.qscale : -INFINITY;
+                sc[sb][2] = r1 < vr ? (acc0[2] + acc1[2]) * p.qscale : -INFINITY;
+                sc[sb][3] = r1 < vr ? (acc0[3] + acc1[3]) * p.qscale : -INFINITY;
+            }
+            // ---- online softmax for heads 2*tq (e = 0) and 2*tq+1 (e = 1)
+            float mt_[2] = {-INFINITY, -INFINITY};
 #pragma unroll
-                for (int h = 0; h < G; ++h) {
-                    acc[h] += __shfl_xor_sync(0xffffffffu, acc[h], 4);
-                    acc[h] += __shfl_xor_sync(0xffffffffu, acc[h], 2);
-                    acc[h] += __shfl_xor_sync(0xffffffffu, acc[h], 1);
-                    s[i4][h] = ti < vr ? acc[h] : -INFINITY;
+            for (int sb = 0; sb < SUB; ++sb) {
+                mt_[0] = fmaxf(mt_[0], fmaxf(sc[sb][0], sc[sb][2]));
+                mt_[1] = fmaxf(mt_[1], fmaxf(sc[sb][1], sc[sb][3]));
+            }
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                mt_[e] = fmaxf(mt_[e], __shfl_xor_sync(0xffffffffu, mt_[e], 4));
+                mt_[e] = fmaxf(mt_[e], __shfl_xor_sync(0xffffffffu, mt_[e], 8));
+                mt_[e] = fmaxf(mt_[e], __shfl_xor_sync(0xffffffffu, mt_[e], 16));
+                if (mt_[e] > m[e]) {
+                    const float alpha = exp2f(m[e] - mt_[e]);
+                    lsum[e] *= alpha;
+#pragma unroll
+                    for (int mt = 0; mt < KS; ++mt) {
+                        o[mt][e] *= alpha;
+                        o[mt][2 + e] *= alpha;
+                    }
+                    m[e] = mt_[e];
                 }
             }
 #pragma unroll
-            for (int h = 0; h < G; ++h) {
-                float mt = s[0][h];
+            for (int sb = 0; sb < SUB; ++sb) {
+                // weights, rounded to bf16 exactly as the MMA consumes them
+                const uint32_t p01 = pack_bf16(exp2f(sc[sb][0] - m[0]), exp2f(sc[sb][1] - m[1]));
+                const uint32_t p23 = pack_bf16(exp2f(sc[sb][2] - m[0]), exp2f(sc[sb][3] - m[1]));
+                lsum[0] += bf16_lo(p01) + bf16_lo(p23);
+                lsum[1] += bf16_hi(p01) + bf16_hi(p23);
+                // B fragment of P^T for this lane: tokens 2*tq, 2*tq+1 (+8) of head gq,
+                // held by lanes 4*token + gq/2 in half gq%2 of p01 (p23 for +8)
+                const int src0 = 4 * (2 * tq) + (gq >> 1), src1 = src0 + 4;
+                const uint32_t x0 = __shfl_sync(0xffffffffu, p01, src0);
+                const uint32_t x1 = __shfl_sync(0xffffffffu, p01, src1);
+                const uint32_t y0 = __shfl_sync(0xffffffffu, p23, src0);
+                const uint32_t y1 = __shfl_sync(0xffffffffu, p23, src1);
+                const uint32_t sel = (gq & 1) ? 0x7632u : 0x5410u;
+                uint32_t b0 = __byte_perm(x0, x1, sel);
+                uint32_t b1 = __byte_perm(y0, y1, sel);
+                if (gq >= G) b0 = b1 = 0u;
+                // ---- O^T[D][8] += V^T[D][16 rows] . P^T[16][8]
+                const uint32_t v_row = vs_base + (16 * sb + (lane & 7) + ((lane >> 4) & 1) * 8) * 128;
+                const int v_hi = (lane >> 3) & 1;
 #pragma unroll
-                for (int i4 = 1; i4 < TPG; ++i4) mt = fmaxf(mt, s[i4][h]);
-                if (mt > m[h]) {
-                    const float alpha = exp2f(m[h] - mt);
-                    lsum[h] *= alpha;
-#pragma unroll
-                    for (int c = 0; c < NCH; ++c)
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) o[h][c][e] *= alpha;
-                    m[h] = mt;
-                }
-            }
-#pragma unroll
-            for (int i4 = 0; i4 < TPG; ++i4) {
-                const int ti = i4 * 4 + grp;
-                if (ti < vr) {
-                    float pw[G];
-#pragma unroll
-                    for (int h = 0; h < G; ++h) {
-                        pw[h] = exp2f(s[i4][h] - m[h]);
-                        lsum[h] += pw[h];
-                    }
-#pragma unroll
-                    for (int c = 0; c < NCH; ++c) {
-                        const uint4 vv = *reinterpret_cast<const uint4 *>(Vs + ti * D + 8 * (lj + 8 * c));
-                        float vf[8];
-                        unpack8(vv, vf);
-#pragma unroll
-                        for (int h = 0; h < G; ++h)
-#pragma unroll
-                            for (int e = 0; e < 8; ++e) o[h][c][e] = fmaf(pw[h], vf[e], o[h][c][e]);
-                    }
+                for (int mt = 0; mt < KS; ++mt) {
+                    uint32_t a0, a1, a2, a3;
+                    const int chunk = ((mt & 3) << 1) + v_hi;
+                    ldsm_x4_t(v_row + (mt >> 2) * BOX + ((chunk ^ (lane & 7)) << 4), a0, a1, a2, a3);
+                    mma_bf16(o[mt], a0, a1, a2, a3, b0, b1);
                 }
             }
         }
         __syncwarp();
+        (void)zeroed;
         if (lane == 0 && t + STAGES < t1) issue(t + STAGES, stg);
     }
     if (!alive) {
         // a copy never completed: wait (bounded) on every stage once more so
         // no copy is left writing this CTA's shared memory, then record an
         // empty partial for the unit in progress
-        if (lane == 0)
-            for (int s = 0; s < STAGES; ++s) (void)mbar_wait_bounded(&bars[s], 0);
+        for (int s = 0; s < STAGES; ++s) (void)mbar_wait_bounded(&bars[s], 0);
 #pragma unroll
-        for (int h = 0; h < G; ++h) {
-            m[h] = -INFINITY;
-            lsum[h] = 0.f;
+        for (int mt = 0; mt < KS; ++mt)
 #pragma unroll
-            for (int c = 0; c < NCH; ++c)
-#pragma unroll
-                for (int e = 0; e < 8; ++e) o[h][c][e] = 0.f;
-        }
+            for (int c = 0; c < 4; ++c) o[mt][c] = 0.f;
+        m[0] = m[1] = -INFINITY;
+        lsum[0] = lsum[1] = 0.f;
     }
     if (cur_unit >= 0) flush(cur_unit);
 }
@@ -397,16 +433,41 @@ struct DecodeLaunch {
         }
         return cached;
     }
-    static cudaError_t run(const DecodeParams &p, cudaStream_t s) {
+    static cudaError_t run(const DecodeParams &p, const CUtensorMap &map, cudaStream_t s) {
         if (max_blocks_per_sm() <= 0) return cudaErrorInvalidConfiguration;
         if (p.n_warps <= 0 || p.n_tiles <= 0) return cudaSuccess;
-        decode_kernel<D, G><<<p.n_warps, 32, Cfg<D>::SMEM, s>>>(p);
+        decode_kernel<D, G><<<p.n_warps, 32, Cfg<D>::SMEM, s>>>(p, map);
         count_launches(1);
         return cudaGetLastError();
     }
 };
 
 }  // namespace
+
+cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, uint64_t rows) {
+    typedef CUresult (*EncodeTiled)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                    const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+    static EncodeTiled encode = nullptr;
+    if (!encode) {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e != cudaSuccess) return e;
+        if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorSymbolNotFound;
+        encode = reinterpret_cast<EncodeTiled>(fn);
+    }
+    const int tok = decode_tile_tokens(head_dim);
+    if (tok == 0 || rows == 0 || rows > 0x7fffffffull) return cudaErrorInvalidValue;
+    const cuuint64_t dims[2] = {(cuuint64_t)head_dim, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)head_dim * 2};
+    const cuuint32_t box[2] = {64, (cuuint32_t)tok};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = encode(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pool, dims, strides, box, estr,
+                              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
 
 bool decode_supported(int head_dim, int group) {
     if (head_dim != 64 && head_dim != 128 && head_dim != 256) return false;
@@ -434,9 +495,10 @@ int decode_max_warps(int head_dim, int group, int n_sm) {
     return 0;
 }
 
-cudaError_t launch_decode(int head_dim, int group, const DecodeParams &p, cudaStream_t s) {
+cudaError_t launch_decode(int head_dim, int group, const DecodeParams &p, const CUtensorMap &pool_map,
+                          cudaStream_t s) {
 #define KVG_CASE(DD, GG) \
-    if (head_dim == DD && group == GG) return DecodeLaunch<DD, GG>::run(p, s);
+    if (head_dim == DD && group == GG) return DecodeLaunch<DD, GG>::run(p, pool_map, s);
     KVG_DECODE_CASES(KVG_CASE)
 #undef KVG_CASE
     return cudaErrorInvalidValue;

@@ -4,6 +4,7 @@
 // exports to the host runtime.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -192,7 +193,12 @@ cudaError_t launch_sha256_serial(const uint8_t *seg0, uint64_t n0, const uint8_t
 // combine over every (layer, row, query head).  decode_tile_tokens() is the
 // tile height TOK (tiles per page = ceil(P / TOK)); decode_max_warps() the
 // number of co-resident warps the decode kernel can keep on the device.
-cudaError_t launch_decode(int head_dim, int group, const DecodeParams &p, cudaStream_t s);
+cudaError_t launch_decode(int head_dim, int group, const DecodeParams &p, const CUtensorMap &pool_map,
+                          cudaStream_t s);
+// Tensor map of a cache pool for the decode kernel: a 2-D bf16 tensor of
+// head_dim columns and n_layers*2*n_pages*n_kv_heads*page_size rows, boxes of
+// 64 columns x decode_tile_tokens(head_dim) rows, 128-byte swizzle.
+cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, uint64_t rows);
 cudaError_t launch_combine(int head_dim, int group, const DecodeParams &p, cudaStream_t s);
 bool decode_supported(int head_dim, int group);
 int decode_tile_tokens(int head_dim);
@@ -262,6 +268,22 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
             "r"(smem_addr(dst)),
         "l"(src), "r"(bytes), "r"(smem_addr(bar))
         : "memory");
+}
+
+// 2-D tensor copy (TMA) of one box at column x, row y of `map` into this
+// CTA's shared memory, completing its bytes on `bar`.  x * 2 bytes must be a
+// multiple of 16 (callers use multiples of 64 columns).
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int32_t x, int32_t y,
+                                            uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
+            "r"(smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_shared() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 __device__ __forceinline__ void record_error(DevStatus *st, int32_t code, int32_t detail) {

@@ -43,6 +43,7 @@ struct CacheShape {
     uint8_t *pool;
     int32_t *page_table, *page_fill;
     DevStatus *status;
+    const CUtensorMap *pool_map;
 };
 bool cache_shape(const kvg_cache *c, CacheShape *out);
 int32_t cache_seq_pages(const kvg_cache *c, int32_t seq);
@@ -150,7 +151,7 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
         p.part_ml = part_ml;
         p.out = static_cast<__nv_bfloat16 *>(out);
         p.status = cs.status;
-        cudaError_t e = launch_decode(cs.head_dim, G, p, st);
+        cudaError_t e = launch_decode(cs.head_dim, G, p, *cs.pool_map, st);
         if (e != cudaSuccess) return reject(KVG_ERR_CUDA, std::string("decode launch: ") + cudaGetErrorString(e));
         e = launch_combine(cs.head_dim, G, p, st);
         if (e != cudaSuccess) return reject(KVG_ERR_CUDA, std::string("combine launch: ") + cudaGetErrorString(e));

@@ -424,6 +424,7 @@ struct kvg_cache {
     std::vector<std::vector<int32_t>> seq_pages;
     std::vector<int32_t> n_slots;
     Scratch leaf, part_o, part_ml;
+    CUtensorMap pool_map;  // decode kernel's 2-D view of the pool
 };
 
 extern "C" kvg_status kvg_cache_create(const kvg_dims *dims, int32_t n_pages, int32_t max_seqs,
@@ -469,6 +470,12 @@ extern "C" kvg_status kvg_cache_create(const kvg_dims *dims, int32_t n_pages, in
         cudaMemset(c->positions, 0xFF, pos) != cudaSuccess ||
         cudaMemset(c->status, 0, sizeof(DevStatus)) != cudaSuccess)
         return cleanup(fail(KVG_ERR_CUDA, "cache tables init failed"));
+    const uint64_t pool_rows = (uint64_t)dims->n_layers * 2 * n_pages * dims->n_kv_heads * dims->page_size;
+    if (pool_rows > 0x7fffffffull)
+        return cleanup(fail(KVG_ERR_ARG, "pool of %llu rows exceeds the decode kernel's 2^31-row addressing",
+                            (unsigned long long)pool_rows));
+    if (make_pool_tensor_map(&c->pool_map, c->pool, dims->head_dim, pool_rows) != cudaSuccess)
+        return cleanup(fail(KVG_ERR_CUDA, "tensor map of the pool could not be encoded"));
     for (int32_t i = 0; i < n_pages; ++i) c->free_list.push_back(i);
     c->seq_pages.assign(max_seqs, {});
     c->n_slots.assign(max_seqs, 0);
@@ -930,7 +937,7 @@ extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const in
         p.part_ml = static_cast<float2 *>(c->part_ml.ptr);
         p.out = static_cast<__nv_bfloat16 *>(out);
         p.status = c->status;
-        KVG_CUDA(launch_decode(d.head_dim, G, p, st));
+        KVG_CUDA(launch_decode(d.head_dim, G, p, c->pool_map, st));
         KVG_CUDA(launch_combine(d.head_dim, G, p, st));
     }
     return KVG_OK;
@@ -1019,12 +1026,13 @@ struct CacheShape {
     uint8_t *pool;
     int32_t *page_table, *page_fill;
     DevStatus *status;
+    const CUtensorMap *pool_map;
 };
 bool cache_shape(const kvg_cache *c, CacheShape *out) {
     if (!c || !out) return false;
     *out = CacheShape{c->dims.n_layers, c->dims.n_kv_heads, c->dims.head_dim, c->dims.page_size, c->n_pages,
                       c->max_seqs, c->max_pages, c->device, c->n_sm, c->pool, c->page_table, c->page_fill,
-                      c->status};
+                      c->status, &c->pool_map};
     return true;
 }
 int32_t cache_seq_pages(const kvg_cache *c, int32_t seq) { return (int32_t)c->seq_pages[seq].size(); }
