@@ -69,6 +69,17 @@ def load_traffic():
     return out
 
 
+def aggregate(total_ms: float, steps: int, step_bytes: int, world: int, device) -> tuple:
+    """Whole-job figures of a run on `world` replicas: the slowest rank's time
+    per step (max over ranks) and the bytes every rank processed over it."""
+    if world > 1:
+        t = torch.tensor([total_ms], dtype=torch.float64, device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_step = total_ms / steps
+    return ms_step, world * step_bytes / (ms_step * 1e-3) / 1e9
+
+
 class Clocks:
     """Samples SM clocks and throttle reasons with nvidia-smi during a region."""
     FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
@@ -156,13 +167,14 @@ class Step12B:
                       + 2 * self.q.numel() * 2,
         }
         self.sha_blocks = (blk_pages // 4096) * 65
-        self.phases = ["release", "graft", "append", "verify_join", "decode", "verify"]
+        self.phases = ["release", "graft", "append", "decode", "verify_join", "verify"]
 
     def run_step(self, store=None, bid=None, ev=None):
-        """One step.  The digest check only reads the grafted pages, which the
-        append does not write, so it runs on a side stream, overlapping the
-        HBM-bound append with its ALU-bound hashing; the main stream waits for
-        it before the decode (which would otherwise share SMs with it).
+        """One step.  The digest check only reads the grafted pages, which
+        neither the append nor the decode writes, so it runs on a side stream:
+        its ALU-bound hashing overlaps the HBM-bound append and decode (the
+        kernels' grids are sized so all three fit on an SM together); the main
+        stream waits for it before the step ends.
         ev: optional per-phase timing events (main: 6, side: 2)."""
         kvg, s, side, c = self.kvg, self.stream, self.side, self.cache.h
         store = store or self.store.h
@@ -181,10 +193,10 @@ class Step12B:
         self.ev_verify.record(side)
         kvg.kvg_cache_append(c, 0, self.kf.data_ptr(), self.vf.data_ptr(), self.pf.data_ptr(), self.nf, s)
         if m: m[3].record(s)
-        s.wait_event(self.ev_verify)
-        if m: m[4].record(s)
         kvg.kvg_decode_attention(c, -1, [0], self.q.data_ptr(), self.w.n_q_heads, self.out.data_ptr(),
                                  self.scale, s)
+        if m: m[4].record(s)
+        s.wait_event(self.ev_verify)
         if m: m[5].record(s)
 
 def run_kvg(args, rank, world):
@@ -232,17 +244,12 @@ def run_kvg(args, rank, world):
     clk = clocks.stop()
     total_ms = t_start.elapsed_time(t_end)
     kvg.kvg_sync(st.cache.h, stream, 60.0)  # digest verification of every timed step passed
-    if world > 1:
-        t = torch.tensor([total_ms], device=device)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
-    ms_step = total_ms / K
-    main_idx = {"release": 0, "graft": 1, "append": 2, "verify_join": 3, "decode": 4}
+    step_bytes = sum(st.bytes.values())
+    ms_step, value = aggregate(total_ms, K, step_bytes, world, device)
+    main_idx = {"release": 0, "graft": 1, "append": 2, "decode": 3, "verify_join": 4}
     phase_ms = {p: statistics.mean(evs[k]["main"][i].elapsed_time(evs[k]["main"][i + 1]) for k in range(K))
                 for p, i in main_idx.items()}
     phase_ms["verify"] = statistics.mean(evs[k]["side"][0].elapsed_time(evs[k]["side"][1]) for k in range(K))
-    step_bytes = sum(st.bytes.values())
-    value = world * step_bytes / (ms_step * 1e-3) / 1e9
     deterministic = _sha_tensor(st.out) == first_sha
 
     # e2e: host-store graft, query from pinned host memory, output read back

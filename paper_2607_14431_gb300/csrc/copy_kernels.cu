@@ -16,6 +16,7 @@ namespace {
 
 constexpr int kCopyThreads = 512;
 constexpr int kCopyUnroll = 8;
+constexpr int kRotUnroll = 4;
 
 __device__ __forceinline__ void copy_chunk(uint8_t *__restrict__ dst, const uint8_t *__restrict__ src,
                                            int bytes) {
@@ -76,28 +77,44 @@ __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const ui
     const uint4 *s4 = reinterpret_cast<const uint4 *>(src);
     uint4 *d4 = reinterpret_cast<uint4 *>(dst);
     if (ROT == 1) {
+        // item = (row, pair chunk c < D/16): the 16-byte vectors c and c + D/16
+        // of the row; kRotUnroll items per thread loaded before any is stored
         const int half_vecs = vec_per_row >> 1;
         const int n_items = rows * half_vecs;
-        for (int it = threadIdx.x; it < n_items; it += kCopyThreads) {
-            const int rr = it / half_vecs;
-            const int c = it - rr * half_vecs;
-            const int64_t row_in_page = first_row_in_page + rr;
-            const int64_t tok = page_token0 + (row_in_page % p.page_size);
-            const int lo_i = rr * vec_per_row + c;
-            const int hi_i = lo_i + half_vecs;
-            const uint4 lo = __ldcs(s4 + lo_i);
-            const uint4 hi = __ldcs(s4 + hi_i);
-            if (tok < p.n_tokens) {
-                float a[8], b[8], ra[8], rb[8];
-                unpack8(lo, a);
-                unpack8(hi, b);
+        for (int base = threadIdx.x; base < n_items; base += kCopyThreads * kRotUnroll) {
+            uint4 lo[kRotUnroll], hi[kRotUnroll];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) rot(a[e], b[e], p.cosv[c * 8 + e], p.sinv[c * 8 + e], ra[e], rb[e]);
-                __stcs(d4 + lo_i, pack8(ra));
-                __stcs(d4 + hi_i, pack8(rb));
-            } else {
-                __stcs(d4 + lo_i, lo);
-                __stcs(d4 + hi_i, hi);
+            for (int u = 0; u < kRotUnroll; ++u) {
+                const int it = base + u * kCopyThreads;
+                if (it < n_items) {
+                    const int rr = it / half_vecs;
+                    const int lo_i = rr * vec_per_row + (it - rr * half_vecs);
+                    lo[u] = __ldcs(s4 + lo_i);
+                    hi[u] = __ldcs(s4 + lo_i + half_vecs);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kRotUnroll; ++u) {
+                const int it = base + u * kCopyThreads;
+                if (it < n_items) {
+                    const int rr = it / half_vecs;
+                    const int c = it - rr * half_vecs;
+                    const int lo_i = rr * vec_per_row + c;
+                    const int64_t tok = page_token0 + ((first_row_in_page + rr) % p.page_size);
+                    if (tok < p.n_tokens) {
+                        float a[8], b[8], ra[8], rb[8];
+                        unpack8(lo[u], a);
+                        unpack8(hi[u], b);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e)
+                            rot(a[e], b[e], p.cosv[c * 8 + e], p.sinv[c * 8 + e], ra[e], rb[e]);
+                        __stcs(d4 + lo_i, pack8(ra));
+                        __stcs(d4 + lo_i + half_vecs, pack8(rb));
+                    } else {
+                        __stcs(d4 + lo_i, lo[u]);
+                        __stcs(d4 + lo_i + half_vecs, hi[u]);
+                    }
+                }
             }
         }
     } else {

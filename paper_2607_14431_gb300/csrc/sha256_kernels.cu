@@ -316,7 +316,7 @@ cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_
     const int64_t n = n_pages * m;
     if (n == 0) return cudaSuccess;
     int64_t grid = (n + 127) / 128;
-    static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 8);
+    static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 4);
     const int64_t cap = (int64_t)n_sm * ctas_per_sm;
     if (grid > cap) grid = cap;
     sha256_leaves_kernel<<<(int)grid, 128, 0, s>>>(src, n_pages, m, leaf_words, 1u);

@@ -370,3 +370,22 @@ def test_append_batch_matches_oracle(oracle):
     with pytest.raises(kvg.KvgError) as e:
         kvg.kvg_cache_append_batch(cache.h, [0, 0], kd.data_ptr(), vd.data_ptr(), pd.data_ptr())
     assert e.value.status == kvg.KVG_ERR_ARG
+
+
+def test_sync_times_out_while_the_stream_is_busy_then_succeeds():
+    # host-side failure detection: kvg_sync gives up after its limit and
+    # reports KVG_ERR_TIMEOUT without touching the work in flight
+    kvg = need_gpu()
+    w = geometry("d256")
+    cache = kvg.Cache(dims_for(kvg, w), 600, 1, 64 * 600)
+    k, v = _kv(w, 30000, 111)
+    append(kvg, cache, 0, k, v, syn.positions(0, 30000))
+    q = torch.zeros((w.n_layers, 1, w.n_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    out = torch.empty_like(q)
+    s = torch.cuda.current_stream()
+    for _ in range(200):  # a few ms of queued work
+        kvg.kvg_decode_attention(cache.h, -1, [0], q.data_ptr(), w.n_q_heads, out.data_ptr(), 0.1)
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_sync(cache.h, s, 1e-6)
+    assert e.value.status == kvg.KVG_ERR_TIMEOUT
+    kvg.kvg_sync(cache.h, s, 60.0)
