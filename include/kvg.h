@@ -146,6 +146,18 @@ kvg_status kvg_store_import(kvg_store *store, const void *bytes, uint64_t n_byte
  * dst_bytes >= total_bytes).  Synchronous. */
 kvg_status kvg_store_export(kvg_store *store, uint64_t block_id, void *dst, uint64_t dst_bytes);
 
+/* Writes block `block_id` to the file `path` in the serialized layout above:
+ * one plain file per block, the paper's persistent medium (Sec. 4.4) that is
+ * copied between machines as is (Sec. 4.11).  Synchronous; KVG_ERR_ARG if the
+ * file cannot be written. */
+kvg_status kvg_store_save(kvg_store *store, uint64_t block_id, const char *path);
+
+/* Reads a block file into the store, validating it like kvg_store_import;
+ * with KVG_GRAFT_VERIFY every page digest and the block digest are recomputed
+ * on the GPU and compared (KVG_ERR_DIGEST: the block is not added).
+ * KVG_ERR_FORMAT for a short or malformed file.  Synchronous. */
+kvg_status kvg_store_load(kvg_store *store, const char *path, uint32_t flags, uint64_t *block_id_out);
+
 /* ---------------------------------------------------------------- cache -- */
 
 /* A paged KV cache on `device`: pool bf16 [n_layers][2][n_pages][n_kv_heads]

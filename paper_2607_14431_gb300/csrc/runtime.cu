@@ -410,6 +410,53 @@ extern "C" kvg_status kvg_store_export(kvg_store *s, uint64_t id, void *dst, uin
     return KVG_OK;
 }
 
+extern "C" kvg_status kvg_store_save(kvg_store *s, uint64_t id, const char *path) {
+    if (!s || !path) return fail(KVG_ERR_ARG, "null argument");
+    if (id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)id);
+    const auto &b = s->blocks[id];
+    std::vector<uint8_t> buf;
+    const uint8_t *src = b.host;
+    if (!src) {
+        buf.resize(b.lay.total);
+        kvg_status st = kvg_store_export(s, id, buf.data(), buf.size());
+        if (st != KVG_OK) return st;
+        src = buf.data();
+    } else {
+        DeviceGuard g(s->device);
+        KVG_CUDA(cudaDeviceSynchronize());
+    }
+    FILE *f = fopen(path, "wb");
+    if (!f) return fail(KVG_ERR_ARG, "cannot open %s for writing", path);
+    const size_t w = fwrite(src, 1, b.lay.total, f);
+    const int rc = fclose(f);
+    if (w != b.lay.total || rc != 0) return fail(KVG_ERR_ARG, "short write to %s", path);
+    return KVG_OK;
+}
+
+extern "C" kvg_status kvg_store_load(kvg_store *s, const char *path, uint32_t flags, uint64_t *block_id_out) {
+    if (!s || !path || !block_id_out) return fail(KVG_ERR_ARG, "null argument");
+    FILE *f = fopen(path, "rb");
+    if (!f) return fail(KVG_ERR_ARG, "cannot open %s", path);
+    uint8_t hdr[256];
+    if (fread(hdr, 1, sizeof hdr, f) != sizeof hdr) {
+        fclose(f);
+        return fail(KVG_ERR_FORMAT, "%s: shorter than a block header", path);
+    }
+    uint64_t total = 0;
+    memcpy(&total, hdr + 88, 8);
+    if (memcmp(hdr, "KVGBLK01", 8) != 0 || total < 256 || total > (1ull << 40)) {
+        fclose(f);
+        return fail(KVG_ERR_FORMAT, "%s: not a block file", path);
+    }
+    std::vector<uint8_t> buf(total);
+    memcpy(buf.data(), hdr, 256);
+    const size_t got = fread(buf.data() + 256, 1, total - 256, f);
+    fclose(f);
+    if (got != total - 256) return fail(KVG_ERR_FORMAT, "%s: truncated (%zu of %llu bytes)", path, got + 256,
+                                        (unsigned long long)total);
+    return kvg_store_import(s, buf.data(), total, flags, block_id_out);
+}
+
 // ------------------------------------------------------------------- cache --
 
 struct kvg_cache {

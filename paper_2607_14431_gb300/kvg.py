@@ -71,6 +71,8 @@ _SIGNATURES = {
     "kvg_store_block_info": ([_vp, _u64, _P(kvg_block_info)], _i32),
     "kvg_store_import": ([_vp, _vp, _u64, _u32, _P(_u64)], _i32),
     "kvg_store_export": ([_vp, _u64, _vp, _u64], _i32),
+    "kvg_store_save": ([_vp, _u64, ctypes.c_char_p], _i32),
+    "kvg_store_load": ([_vp, ctypes.c_char_p, _u32, _P(_u64)], _i32),
     "kvg_cache_create": ([_P(kvg_dims), _i32, _i32, _i32, _i32, _P(_vp)], _i32),
     "kvg_cache_destroy": ([_vp], None),
     "kvg_cache_set_free_order": ([_vp, _vp, _i32], _i32),
@@ -164,6 +166,16 @@ def kvg_store_export(store, block_id: int) -> bytes:
     buf = ctypes.create_string_buffer(info.total_bytes)
     _check(lib().kvg_store_export(store, block_id, buf, info.total_bytes))
     return buf.raw
+
+
+def kvg_store_save(store, block_id: int, path: str):
+    _check(lib().kvg_store_save(store, block_id, os.fsencode(path)))
+
+
+def kvg_store_load(store, path: str, flags: int = 0) -> int:
+    out = _u64()
+    _check(lib().kvg_store_load(store, os.fsencode(path), flags, ctypes.byref(out)))
+    return out.value
 
 
 def kvg_cache_create(dims: kvg_dims, n_pages: int, max_seqs: int, max_slots: int, device: int = 0):
