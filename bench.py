@@ -129,7 +129,7 @@ class Clocks:
 class Step12B:
     """Device state and the per-step call sequence for the 12B workload."""
 
-    def __init__(self, kvg, device, stream, side, n_layers=None):
+    def __init__(self, kvg, device, stream, side, n_layers=None, pool_store=False):
         self.kvg = kvg
         self.w = w = syn.B12 if not n_layers else syn.B12.with_layers(n_layers)
         self.dev = device
@@ -141,8 +141,11 @@ class Step12B:
         P = w.page_size
         self.dims = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0)
         n_pages = syn.B12_CTX // P + self.nb // P
-        self.cache = kvg.Cache(self.dims, n_pages, 2, syn.B12_CTX)
-        self.store = kvg.Store(self.dims, kvg.KVG_RESIDENCY_HBM, 4 << 30)
+        self.cache = kvg.Cache(self.dims, n_pages + (self.nb // P if pool_store else 0), 2, syn.B12_CTX)
+        # pool_store: the block lives in the cache's own pool and grafts by
+        # aliasing its pages (no page copy)
+        self.store = (kvg.PoolStore(self.cache, 64 << 20) if pool_store
+                      else kvg.Store(self.dims, kvg.KVG_RESIDENCY_HBM, 4 << 30))
         self.hstore = kvg.Store(self.dims, kvg.KVG_RESIDENCY_PINNED_HOST, 4 << 30)
         with torch.cuda.stream(stream):
             kb, vb = syn.kv_rows(w, self.nb, w.seed, device)
@@ -159,8 +162,9 @@ class Step12B:
         self.kb, self.vb = kb, vb  # the block's rows, kept for parity tests
         self.scale = 1.0 / math.sqrt(w.head_dim)
         blk_pages = w.n_layers * 2 * (self.nb // P) * w.page_bytes
+        self.pool_store = pool_store
         self.bytes = {
-            "graft": 2 * blk_pages,
+            "graft": 0 if pool_store else 2 * blk_pages,
             "verify": blk_pages,
             "append": 2 * w.n_layers * 2 * self.nf * w.n_kv_heads * w.head_dim * 2,
             "decode": w.n_layers * 2 * syn.B12_CTX * w.n_kv_heads * w.head_dim * 2
@@ -210,7 +214,7 @@ def run_kvg(args, rank, world):
     stream = torch.cuda.Stream(device)
     side = torch.cuda.Stream(device)
     hbm_peak, sm_max, peak_kind = load_peaks()
-    st = Step12B(kvg, device, stream, side, args.layers)
+    st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool")
 
     # correctness of the configuration being timed: one verified step
     st.run_step()
@@ -293,7 +297,7 @@ def run_kvg(args, rank, world):
     parts = {}
     for p in st.phases:
         ms = phase_ms[p]
-        if p in ("release", "verify_join"):
+        if p in ("release", "verify_join") or st.bytes.get(p) == 0:
             parts[p] = {"ms": round(ms, 4)}
             continue
         b = st.bytes[p]
@@ -310,7 +314,7 @@ def run_kvg(args, rank, world):
     kernel_of = {"graft": "graft_kernel", "verify": "sha256_leaves_kernel", "append": "append_kernel",
                  "decode": "decode_kernel"}
     # dominant kernel: the longest phase on the step's critical (main-stream) path
-    dom = max(("graft", "append", "decode", "verify"), key=lambda p: phase_ms[p])
+    dom = max(("graft", "append", "decode", "verify"), key=lambda p: phase_ms[p] if st.bytes[p] else 0.0)
     if dom == "verify":
         ops = st.sha_blocks * SHA_OPS_PER_BLOCK
         ach = ops / (phase_ms[dom] * 1e-3) / 1e12
@@ -328,7 +332,8 @@ def run_kvg(args, rank, world):
         "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": f"12b-single-graft: L{st.w.n_layers} Hq16/Hkv8 D256 P64, 8192-token block grafted "
-                               "at own positions (digest-verified) + 24576 fresh tokens, decode 1 token over 32768",
+                               "at own positions (digest-verified) + 24576 fresh tokens, decode 1 token over 32768"
+                               + (" [block in the cache pool: zero-copy graft]" if st.pool_store else ""),
                    "global_batch": world, "seq_len": syn.B12_CTX, "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)"},
         "parts": parts, "roofline": roof, "e2e": e2e, "gpu_launches": int(launches),
@@ -742,6 +747,8 @@ def main():
     ap.add_argument("--layers", type=int, default=0, help="layer count override (small profiling cases)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--config", default="12b", choices=["12b", "31b", "batched", "deep"])
+    ap.add_argument("--store", default="hbm", choices=["hbm", "pool"],
+                    help="12b: block in an HBM store (copying graft) or in the cache pool (zero-copy graft)")
     ap.add_argument("--deep-blocks", type=int, default=syn.DEEP_BLOCKS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()

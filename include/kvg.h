@@ -57,7 +57,7 @@ typedef enum kvg_status {
     KVG_ERR_DEVICE_CHECK = -10 /* a kernel's own bounds/wait check failed */
 } kvg_status;
 
-enum { KVG_RESIDENCY_HBM = 0, KVG_RESIDENCY_PINNED_HOST = 1 };
+enum { KVG_RESIDENCY_HBM = 0, KVG_RESIDENCY_PINNED_HOST = 1, KVG_RESIDENCY_CACHE_POOL = 2 };
 enum { KVG_ROPE_HALF = 0, KVG_ROPE_INTERLEAVED = 1 };
 enum { KVG_GRAFT_VERIFY = 1u, KVG_GRAFT_SYNC = 2u };
 enum { KVG_SHA256_PLAIN = 0, KVG_SHA256_PAGED = 1 };
@@ -99,6 +99,23 @@ typedef struct kvg_cache kvg_cache;
 kvg_status kvg_store_create(const kvg_dims *dims, int32_t residency, uint64_t capacity_bytes,
                             int32_t device, kvg_store **out);
 void kvg_store_destroy(kvg_store *store);
+
+/* A store whose blocks live inside `cache`'s own page pool (residency
+ * KVG_RESIDENCY_CACHE_POOL), for a zero-copy graft.  A deposit copies the rows
+ * into pool pages that the block owns from then on (taken from the cache's
+ * free list for good); an own-position graft then writes only the sequence's
+ * page-table entries, fills and position tags, pointing at the block's full
+ * pages (shared and read-only: appends never write a full page), and copies a
+ * partially filled last page into a page of the sequence, which its appends
+ * fill.  A release never frees a block's pages.  Deposits and grafts must use
+ * this cache; relocation (delta != 0) needs a copying store (KVG_ERR_ARG);
+ * blocks have at most 1024 pages.  capacity_bytes bounds the blocks'
+ * metadata (header, position tags, digests, page ids) kept in HBM.
+ * kvg_store_block_info's `bytes` points at that metadata; export, save and
+ * import produce and accept the same serialized bytes as other stores.
+ * Destroy such a store before its cache; its pages return to the free list
+ * unless a sequence still points at them. */
+kvg_status kvg_store_create_in_cache(kvg_cache *cache, uint64_t capacity_bytes, kvg_store **out);
 
 /* Serialized block layout (little-endian), one contiguous region:
  *   [0, 256)      header: magic "KVGBLK01", u32 version = 1, u32 header bytes
@@ -264,8 +281,10 @@ kvg_status kvg_graft(kvg_store *store, uint64_t block_id, kvg_cache *cache, int3
  * [slot0, slot0 + n_tokens(block)) of `seq` (slot0 page-aligned) on the GPU
  * and compares each page digest with block `block_id`'s stored digest
  * (Sec. 4.11 integrity check, applied to the live copy).  Only meaningful for
- * own-position grafts (relocated key pages differ by design).  Flags and
- * reporting as for kvg_graft (KVG_GRAFT_SYNC waits and fills `report`). */
+ * own-position grafts (relocated key pages differ by design), and only until
+ * rows are appended into a ragged block's last page: its digest covers the
+ * block's zero padding rows, which appends overwrite.  Flags and reporting as
+ * for kvg_graft (KVG_GRAFT_SYNC waits and fills `report`). */
 kvg_status kvg_verify(kvg_store *store, uint64_t block_id, kvg_cache *cache, int32_t seq,
                       int32_t slot0, uint32_t flags, void *stream, kvg_graft_report *report);
 

@@ -364,6 +364,15 @@ class KvgError(Exception):
     pass
 
 
+class PinnedBlock:
+    """A block whose pages live in the cache's own pool (zero-copy graft):
+    pids[j] holds block page j of every layer and K/V."""
+
+    def __init__(self, pids, block: Block):
+        self.pids = list(pids)
+        self.block = block
+
+
 class OracleCache:
     """Paged KV cache.
 
@@ -391,6 +400,7 @@ class OracleCache:
         if fill is not None and self.pool is not None:
             self.pool[...] = fill
         self.free = list(range(n_pages))
+        self.pinned = set()
         self.page_table = np.full((max_seqs, self.max_pages), -1, np.int32)
         self.page_fill = np.zeros((max_seqs, self.max_pages), np.int32)
         self.positions = np.full((max_seqs, max_slots), -1, np.int32)
@@ -481,8 +491,42 @@ class OracleCache:
         for b, sq in enumerate(seq_ids):
             self.append(int(sq), k[:, b:b + 1], v[:, b:b + 1], positions[b:b + 1])
 
+    def pin_block(self, seq: int, slot0: int, n: int) -> PinnedBlock:
+        """Deposit into the pool: the block's pages (as deposit() builds them)
+        are copied into pages taken from the free list for good."""
+        blk = self.deposit(seq, slot0, n)
+        pids = self._take(blk.n_pages)
+        self.pinned |= set(pids)
+        for j, pid in enumerate(pids):
+            self.pool[:, :, pid] = blk.pages[:, :, j]
+        return PinnedBlock(pids, blk)
+
+    def graft_pinned(self, seq: int, pb: PinnedBlock, dst_slot: int = -1):
+        """Own-position graft by aliasing: the sequence's page table points at
+        the block's pages; a partially filled last page is copied into a page
+        of the sequence (its appends fill that page)."""
+        d = self.dims
+        boundary = _round_up(int(self.n_slots[seq]), d.P)
+        if dst_slot < 0:
+            dst_slot = boundary
+        if dst_slot != boundary:
+            raise KvgError("dst_slot must be the next page boundary")
+        n = pb.block.n_tokens
+        if dst_slot + n > self.max_slots:
+            raise KvgError("capacity")
+        pages = list(pb.pids)
+        if n % d.P:
+            pages[-1] = self._take(1)[0]
+            self.pool[:, :, pages[-1]] = self.pool[:, :, pb.pids[-1]]
+        j0 = dst_slot // d.P
+        for j, pid in enumerate(pages):
+            self.page_table[seq, j0 + j] = pid
+            self.page_fill[seq, j0 + j] = min(d.P, n - j * d.P)
+        self.positions[seq, dst_slot:dst_slot + n] = pb.block.positions
+        self.n_slots[seq] = dst_slot + n
+
     def release(self, seq: int):
-        used = [int(p) for p in self.page_table[seq] if p >= 0]
+        used = [int(p) for p in self.page_table[seq] if p >= 0 and int(p) not in self.pinned]
         self.free.extend(used)
         self.page_table[seq] = -1
         self.page_fill[seq] = 0

@@ -100,15 +100,33 @@ struct AppendBatchParams {
 // --------------------------------------------------------------- deposit --
 struct GatherParams {
     const uint8_t *pool;
-    uint8_t *dst;              // block pages region
+    uint8_t *dst;              // block pages region (dst_pids.n == 0), or the pool (dst_pids given)
     uint64_t page_bytes;
     int64_t pool_pages;
     int32_t n_layers, npb, page_base, block_pages;
     int32_t n_kv_heads, page_size, head_dim;
     int64_t n_tokens;          // rows >= n_tokens are written as zero
-    const int32_t *src_pos;    // positions row + slot0
+    const int32_t *src_pos;    // positions row + slot0 (nullable: no position copy)
     int32_t *dst_pos;          // block positions
-    PageList pids;
+    PageList pids;             // source pool pages
+    PageList dst_pids;         // destination pool pages (pool-resident blocks), n = 0 when unused
+};
+
+// Own-position graft by aliasing: page-table entries, fills and position
+// tags of a sequence for a block whose pages already sit in the pool.
+struct AliasParams {
+    const int32_t *src_pos;    // block positions
+    int32_t *table_row;        // page_table row + first page index
+    int32_t *fill_row;         // page_fill row + first page index
+    int32_t *dst_pos;          // positions row + dst slot
+    int64_t n_tokens;
+    int32_t page_size;
+    PageList pids;             // the sequence's pages for the block, in order
+};
+
+struct IntsParams {
+    int32_t *dst;
+    PageList vals;
 };
 
 struct HeaderParams {
@@ -173,6 +191,8 @@ cudaError_t launch_append(const AppendParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_append_batch(const AppendBatchParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_write_header(const HeaderParams &p, cudaStream_t s);
+cudaError_t launch_alias(const AliasParams &p, int n_sm, cudaStream_t s);
+cudaError_t launch_write_ints(const IntsParams &p, cudaStream_t s);
 cudaError_t launch_reset_seq(int32_t *table_row, int32_t *fill_row, int32_t max_pages,
                              int32_t *pos_row, int32_t max_slots, cudaStream_t s);
 

@@ -284,7 +284,8 @@ __global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
     const int64_t tok0 = (int64_t)p.page_base * P;
     int64_t n_meta = (int64_t)p.npb * P;
     if (tok0 + n_meta > p.n_tokens) n_meta = p.n_tokens - tok0;
-    for (int64_t t = gtid; t < n_meta; t += gsz) p.dst_pos[t] = p.src_pos[t];
+    if (p.src_pos)
+        for (int64_t t = gtid; t < n_meta; t += gsz) p.dst_pos[t] = p.src_pos[t];
     for (int64_t idx = gtid; idx < total; idx += gsz) {
         const int64_t page_u = idx / vpp;
         const int64_t off = idx - page_u * vpp;
@@ -299,9 +300,26 @@ __global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
             val = __ldcs(src + off);
         }
         uint4 *dst = reinterpret_cast<uint4 *>(
-            p.dst + ((uint64_t)lkv * p.block_pages + p.page_base + jj) * p.page_bytes);
+            p.dst_pids.n ? p.dst + ((uint64_t)lkv * p.pool_pages + p.dst_pids.pid[jj]) * p.page_bytes
+                         : p.dst + ((uint64_t)lkv * p.block_pages + p.page_base + jj) * p.page_bytes);
         dst[off] = val;
     }
+}
+
+__global__ void __launch_bounds__(256) alias_kernel(const AliasParams p) {
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+    const int64_t P = p.page_size;
+    for (int64_t t = gtid; t < p.n_tokens; t += gsz) p.dst_pos[t] = p.src_pos[t];
+    for (int64_t j = gtid; j < p.pids.n; j += gsz) {
+        p.table_row[j] = p.pids.pid[j];
+        const int64_t f = p.n_tokens - j * P;
+        p.fill_row[j] = (int32_t)(f < P ? f : P);
+    }
+}
+
+__global__ void write_ints_kernel(const IntsParams p) {
+    for (int i = threadIdx.x; i < p.vals.n; i += blockDim.x) p.dst[i] = p.vals.pid[i];
 }
 
 __global__ void write_header_kernel(const HeaderParams p) {
@@ -361,6 +379,18 @@ cudaError_t launch_append_batch(const AppendBatchParams &p, int n_sm, cudaStream
 cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s) {
     const int64_t items = 2ll * p.n_layers * p.npb * (int64_t)(p.page_bytes / 16);
     gather_kernel<<<grid_for(items, 256, n_sm, 8), 256, 0, s>>>(p);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_alias(const AliasParams &p, int n_sm, cudaStream_t s) {
+    alias_kernel<<<grid_for(p.n_tokens > p.pids.n ? p.n_tokens : p.pids.n, 256, n_sm, 1), 256, 0, s>>>(p);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_write_ints(const IntsParams &p, cudaStream_t s) {
+    write_ints_kernel<<<1, 256, 0, s>>>(p);
     count_launches(1);
     return cudaGetLastError();
 }

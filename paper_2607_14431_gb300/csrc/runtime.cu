@@ -185,14 +185,16 @@ struct kvg_store {
     };
     std::vector<Slab> slabs;
     struct Blk {
-        uint8_t *dev;   // device-accessible start of the serialized block
+        uint8_t *dev;   // device-accessible start of the serialized block (pool stores: its metadata)
         uint8_t *host;  // host address (pinned-host store) or nullptr
         BlockLayout lay;
         int64_t min_pos, max_pos;
+        std::vector<int32_t> pids;  // pool stores: the block's pages in the cache pool
     };
     std::vector<Blk> blocks;
     Scratch leaf;
     DevStatus *status = nullptr;
+    kvg_cache *pool_cache = nullptr;  // KVG_RESIDENCY_CACHE_POOL: the cache holding the pages
 };
 
 static kvg_status store_alloc(kvg_store *s, uint64_t bytes, uint8_t **dev, uint8_t **host) {
@@ -215,7 +217,7 @@ static kvg_status store_alloc(kvg_store *s, uint64_t bytes, uint8_t **dev, uint8
     const uint64_t size = std::min<uint64_t>(slab, s->capacity - s->reserved_bytes);
     kvg_store::Slab sl;
     sl.size = size;
-    if (s->residency == KVG_RESIDENCY_HBM) {
+    if (s->residency != KVG_RESIDENCY_PINNED_HOST) {
         cudaError_t e = cudaMalloc(&sl.dev, size);
         if (e != cudaSuccess) {
             cudaGetLastError();
@@ -270,10 +272,13 @@ extern "C" kvg_status kvg_store_create(const kvg_dims *dims, int32_t residency, 
     return KVG_OK;
 }
 
+static void pool_release_blocks(kvg_store *s);
+
 extern "C" void kvg_store_destroy(kvg_store *s) {
     if (!s) return;
     DeviceGuard g(s->device);
     cudaDeviceSynchronize();
+    if (s->pool_cache) pool_release_blocks(s);
     for (auto &sl : s->slabs) {
         if (sl.host)
             cudaFreeHost(sl.host);
@@ -338,6 +343,11 @@ static void minmax_positions(const int32_t *pos, int64_t n, int64_t *mn, int64_t
     *mx = n ? b : 0;
 }
 
+// Pool-resident blocks (KVG_RESIDENCY_CACHE_POOL), defined after kvg_cache.
+static kvg_status pool_export(kvg_store *s, uint64_t id, uint8_t *dst);
+static kvg_status pool_import(kvg_store *s, const uint8_t *h, const BlockLayout &lay, uint32_t flags,
+                              uint64_t *block_id_out);
+
 extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t n_bytes, uint32_t flags,
                                        uint64_t *block_id_out) {
     if (!s || !bytes || !block_id_out) return fail(KVG_ERR_ARG, "null argument");
@@ -371,6 +381,7 @@ extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t
         tot != lay.total || n_bytes < tot)
         return fail(KVG_ERR_FORMAT, "layout fields inconsistent");
     DeviceGuard g(s->device);
+    if (s->pool_cache) return pool_import(s, h, lay, flags, block_id_out);
     uint8_t *dev = nullptr, *host = nullptr;
     kvg_status st = store_alloc(s, lay.total, &dev, &host);
     if (st != KVG_OK) return st;
@@ -403,6 +414,7 @@ extern "C" kvg_status kvg_store_export(kvg_store *s, uint64_t id, void *dst, uin
     if (dst_bytes < b.lay.total) return fail(KVG_ERR_CAPACITY, "destination too small");
     DeviceGuard g(s->device);
     KVG_CUDA(cudaDeviceSynchronize());
+    if (s->pool_cache) return pool_export(s, id, static_cast<uint8_t *>(dst));
     if (b.host)
         memcpy(dst, b.host, b.lay.total);
     else
@@ -472,7 +484,138 @@ struct kvg_cache {
     std::vector<int32_t> n_slots;
     Scratch leaf, part_o, part_ml;
     CUtensorMap pool_map;  // decode kernel's 2-D view of the pool
+    std::vector<uint8_t> pinned;  // per page: owned by a pool-resident store block
+    std::vector<int32_t> alias;   // per pinned page: sequences whose page tables point at it
 };
+
+// ---------------------------------------------- store inside a cache pool --
+
+static std::vector<int32_t> take_pages(kvg_cache *c, int64_t n);
+
+extern "C" kvg_status kvg_store_create_in_cache(kvg_cache *c, uint64_t capacity_bytes, kvg_store **out) {
+    if (!c || !out) return fail(KVG_ERR_ARG, "null argument");
+    *out = nullptr;
+    DeviceGuard g(c->device);
+    kvg_store *s = new kvg_store();
+    s->dims = c->dims;
+    s->residency = KVG_RESIDENCY_CACHE_POOL;
+    s->capacity = capacity_bytes;
+    s->device = c->device;
+    s->n_sm = c->n_sm;
+    s->pool_cache = c;
+    cudaError_t e = cudaMalloc(&s->status, sizeof(DevStatus));
+    if (e != cudaSuccess) {
+        delete s;
+        return cuda_fail(e, "cudaMalloc(status)");
+    }
+    cudaMemset(s->status, 0, sizeof(DevStatus));
+    *out = s;
+    return KVG_OK;
+}
+
+// Metadata region of a pool-resident block: the serialized layout up to
+// pages_off (header, positions, digests), then the block's page ids.
+static uint64_t pool_meta_bytes(const BlockLayout &lay) { return lay.pages_off + 4ull * lay.n_pages; }
+
+// Hashes a pool-resident block's pages (digests into its metadata, or
+// compared with them when verify) and its block digest.
+static kvg_status pool_hash(kvg_store *s, uint8_t *meta, const BlockLayout &lay, bool verify, cudaStream_t st) {
+    kvg_cache *c = s->pool_cache;
+    const uint64_t pb = c->page_bytes;
+    const int64_t m = (int64_t)((pb + kLeafBytes - 1) / kLeafBytes);
+    const int64_t n_pages = (int64_t)s->dims.n_layers * 2 * lay.n_pages;
+    KVG_CUDA(s->leaf.ensure((size_t)n_pages * m * 32));
+    PageSource src{c->pool, pb, reinterpret_cast<const int32_t *>(meta + lay.pages_off), (int32_t)lay.n_pages,
+                   (int64_t)c->n_pages};
+    uint32_t *leaf = static_cast<uint32_t *>(s->leaf.ptr);
+    KVG_CUDA(launch_sha256_leaves(src, n_pages, leaf, s->n_sm, st));
+    uint8_t *dig = meta + lay.dig_off;
+    KVG_CUDA(launch_sha256_pages(leaf, n_pages, m, verify ? nullptr : dig, verify ? dig : nullptr, s->status, -1, st));
+    KVG_CUDA(launch_sha256_serial(meta + lay.pos_off, 4ull * lay.n_tokens, dig, (uint64_t)n_pages * 32,
+                                  verify ? nullptr : meta + 96, verify ? meta + 96 : nullptr, s->status, st));
+    return KVG_OK;
+}
+
+static kvg_status pool_write_pids(uint8_t *meta, const BlockLayout &lay, const std::vector<int32_t> &pids,
+                                  cudaStream_t st) {
+    int32_t *dst = reinterpret_cast<int32_t *>(meta + lay.pages_off);
+    for (size_t base = 0; base < pids.size(); base += kMaxPagesPerLaunch) {
+        IntsParams ip{};
+        ip.dst = dst + base;
+        ip.vals.n = (int32_t)std::min<size_t>(kMaxPagesPerLaunch, pids.size() - base);
+        for (int32_t i = 0; i < ip.vals.n; ++i) ip.vals.pid[i] = pids[base + i];
+        KVG_CUDA(launch_write_ints(ip, st));
+    }
+    return KVG_OK;
+}
+
+static void pool_unpin(kvg_cache *c, const std::vector<int32_t> &pids) {
+    for (int32_t pid : pids) {
+        c->pinned[pid] = 0;
+        c->free_list.push_back(pid);
+    }
+}
+
+// A destroyed pool-resident store gives its pages back unless a sequence
+// still points at them (those stay reserved until the cache is destroyed).
+static void pool_release_blocks(kvg_store *s) {
+    kvg_cache *c = s->pool_cache;
+    for (auto &b : s->blocks)
+        for (int32_t pid : b.pids)
+            if (c->alias[pid] == 0) {
+                c->pinned[pid] = 0;
+                c->free_list.push_back(pid);
+            }
+}
+
+static kvg_status pool_export(kvg_store *s, uint64_t id, uint8_t *dst) {
+    const auto &b = s->blocks[id];
+    kvg_cache *c = s->pool_cache;
+    KVG_CUDA(cudaMemcpy(dst, b.dev, b.lay.pages_off, cudaMemcpyDeviceToHost));
+    const uint64_t pb = c->page_bytes;
+    const int64_t npb = b.lay.n_pages;
+    for (int64_t lkv = 0; lkv < (int64_t)s->dims.n_layers * 2; ++lkv)
+        for (int64_t j = 0; j < npb; ++j)
+            KVG_CUDA(cudaMemcpy(dst + b.lay.pages_off + (uint64_t)(lkv * npb + j) * pb,
+                                c->pool + ((uint64_t)lkv * c->n_pages + b.pids[j]) * pb, pb, cudaMemcpyDeviceToHost));
+    return KVG_OK;
+}
+
+static kvg_status pool_import(kvg_store *s, const uint8_t *h, const BlockLayout &lay, uint32_t flags,
+                              uint64_t *block_id_out) {
+    kvg_cache *c = s->pool_cache;
+    if (lay.n_pages > (int64_t)c->free_list.size()) return fail(KVG_ERR_CAPACITY, "cache pool has too few free pages");
+    uint8_t *meta = nullptr, *host = nullptr;
+    kvg_status st = store_alloc(s, pool_meta_bytes(lay), &meta, &host);
+    if (st != KVG_OK) return st;
+    auto pids = take_pages(c, lay.n_pages);
+    for (int32_t pid : pids) c->pinned[pid] = 1;
+    const uint64_t pb = c->page_bytes;
+    KVG_CUDA(cudaMemcpy(meta, h, lay.pages_off, cudaMemcpyHostToDevice));
+    KVG_CUDA(cudaMemcpy(meta + lay.pages_off, pids.data(), 4 * pids.size(), cudaMemcpyHostToDevice));
+    for (int64_t lkv = 0; lkv < (int64_t)s->dims.n_layers * 2; ++lkv)
+        for (int64_t j = 0; j < lay.n_pages; ++j)
+            KVG_CUDA(cudaMemcpy(c->pool + ((uint64_t)lkv * c->n_pages + pids[j]) * pb,
+                                h + lay.pages_off + (uint64_t)(lkv * lay.n_pages + j) * pb, pb, cudaMemcpyHostToDevice));
+    if (flags & KVG_GRAFT_VERIFY) {
+        KVG_CUDA(cudaMemset(s->status, 0, sizeof(DevStatus)));
+        st = pool_hash(s, meta, lay, true, 0);
+        if (st != KVG_OK) return st;
+        KVG_CUDA(cudaDeviceSynchronize());
+        DevStatus hs;
+        KVG_CUDA(cudaMemcpy(&hs, s->status, sizeof hs, cudaMemcpyDeviceToHost));
+        KVG_CUDA(cudaMemset(s->status, 0, sizeof(DevStatus)));
+        if (hs.n_mismatch) {
+            pool_unpin(c, pids);
+            return fail(KVG_ERR_DIGEST, "import: %d digest mismatches (block not added)", hs.n_mismatch);
+        }
+    }
+    kvg_store::Blk b{meta, nullptr, lay, 0, 0, pids};
+    minmax_positions(reinterpret_cast<const int32_t *>(h + lay.pos_off), lay.n_tokens, &b.min_pos, &b.max_pos);
+    s->blocks.push_back(b);
+    *block_id_out = s->blocks.size() - 1;
+    return KVG_OK;
+}
 
 extern "C" kvg_status kvg_cache_create(const kvg_dims *dims, int32_t n_pages, int32_t max_seqs,
                                        int32_t max_slots, int32_t device, kvg_cache **out) {
@@ -524,6 +667,8 @@ extern "C" kvg_status kvg_cache_create(const kvg_dims *dims, int32_t n_pages, in
     if (make_pool_tensor_map(&c->pool_map, c->pool, dims->head_dim, pool_rows) != cudaSuccess)
         return cleanup(fail(KVG_ERR_CUDA, "tensor map of the pool could not be encoded"));
     for (int32_t i = 0; i < n_pages; ++i) c->free_list.push_back(i);
+    c->pinned.assign(n_pages, 0);
+    c->alias.assign(n_pages, 0);
     c->seq_pages.assign(max_seqs, {});
     c->n_slots.assign(max_seqs, 0);
     if (cudaDeviceSynchronize() != cudaSuccess) return cleanup(fail(KVG_ERR_CUDA, "init sync failed"));
@@ -699,7 +844,12 @@ extern "C" kvg_status kvg_cache_release(kvg_cache *c, int32_t seq, void *stream)
     if (!c) return fail(KVG_ERR_ARG, "null cache");
     if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d", seq);
     DeviceGuard g(c->device);
-    for (int32_t pid : c->seq_pages[seq]) c->free_list.push_back(pid);
+    for (int32_t pid : c->seq_pages[seq]) {
+        if (c->pinned[pid])
+            --c->alias[pid];  // a pool-resident block's page: not the sequence's to free
+        else
+            c->free_list.push_back(pid);
+    }
     c->seq_pages[seq].clear();
     c->n_slots[seq] = 0;
     KVG_CUDA(launch_reset_seq(c->page_table + (int64_t)seq * c->max_pages,
@@ -710,6 +860,61 @@ extern "C" kvg_status kvg_cache_release(kvg_cache *c, int32_t seq, void *stream)
 }
 
 // ----------------------------------------------------------------- deposit --
+
+// Deposit into a pool-resident store: the rows are copied into pool pages
+// that the block owns from then on (taken from the free list for good).
+static kvg_status pool_deposit(kvg_store *s, kvg_cache *c, int32_t seq, int32_t slot0, int32_t n,
+                               const BlockLayout &lay, cudaStream_t st, uint64_t *block_id_out) {
+    if (lay.n_pages > (int64_t)c->free_list.size()) return fail(KVG_ERR_CAPACITY, "cache pool has too few free pages");
+    uint8_t *meta = nullptr, *host = nullptr;
+    kvg_status stt = store_alloc(s, pool_meta_bytes(lay), &meta, &host);
+    if (stt != KVG_OK) return stt;
+    auto pids = take_pages(c, lay.n_pages);
+    for (int32_t pid : pids) c->pinned[pid] = 1;
+    HeaderParams hp;
+    hp.dst = meta;
+    build_header(hp.bytes, s->dims, lay);
+    KVG_CUDA(launch_write_header(hp, st));
+    const int64_t P = c->dims.page_size;
+    const auto &sp = c->seq_pages[seq];
+    const int64_t j_first = slot0 / P;
+    for (int64_t base = 0; base < lay.n_pages; base += kMaxPagesPerLaunch) {
+        GatherParams p{};
+        p.pool = c->pool;
+        p.dst = c->pool;
+        p.page_bytes = c->page_bytes;
+        p.pool_pages = c->n_pages;
+        p.n_layers = c->dims.n_layers;
+        p.npb = (int32_t)std::min<int64_t>(kMaxPagesPerLaunch, lay.n_pages - base);
+        p.page_base = (int32_t)base;
+        p.block_pages = (int32_t)lay.n_pages;
+        p.n_kv_heads = c->dims.n_kv_heads;
+        p.page_size = (int32_t)P;
+        p.head_dim = c->dims.head_dim;
+        p.n_tokens = n;
+        p.src_pos = c->positions + (int64_t)seq * c->max_slots + slot0 + base * P;
+        p.dst_pos = reinterpret_cast<int32_t *>(meta + lay.pos_off) + base * P;
+        p.pids.n = p.npb;
+        p.dst_pids.n = p.npb;
+        for (int32_t i = 0; i < p.npb; ++i) {
+            p.pids.pid[i] = sp[j_first + base + i];
+            p.dst_pids.pid[i] = pids[base + i];
+        }
+        KVG_CUDA(launch_gather(p, s->n_sm, st));
+    }
+    stt = pool_write_pids(meta, lay, pids, st);
+    if (stt != KVG_OK) return stt;
+    stt = pool_hash(s, meta, lay, false, st);
+    if (stt != KVG_OK) return stt;
+    KVG_CUDA(cudaStreamSynchronize(st));
+    kvg_store::Blk b{meta, nullptr, lay, 0, 0, pids};
+    std::vector<int32_t> pos(n);
+    KVG_CUDA(cudaMemcpy(pos.data(), meta + lay.pos_off, 4ull * n, cudaMemcpyDeviceToHost));
+    minmax_positions(pos.data(), n, &b.min_pos, &b.max_pos);
+    s->blocks.push_back(b);
+    *block_id_out = s->blocks.size() - 1;
+    return KVG_OK;
+}
 
 extern "C" kvg_status kvg_deposit(kvg_store *s, const kvg_cache *cc, int32_t seq, int32_t slot0, int32_t n,
                                   void *stream, uint64_t *block_id_out) {
@@ -723,6 +928,10 @@ extern "C" kvg_status kvg_deposit(kvg_store *s, const kvg_cache *cc, int32_t seq
         return fail(KVG_ERR_ARG, "bad range [%d, %d) of %d slots", slot0, slot0 + n, c->n_slots[seq]);
     DeviceGuard g(s->device);
     const BlockLayout lay = layout_for(s->dims, n);
+    if (s->pool_cache) {
+        if (s->pool_cache != c) return fail(KVG_ERR_ARG, "a pool-resident store deposits from its own cache");
+        return pool_deposit(s, c, seq, slot0, n, lay, static_cast<cudaStream_t>(stream), block_id_out);
+    }
     uint8_t *dev = nullptr, *host = nullptr;
     kvg_status stt = store_alloc(s, lay.total, &dev, &host);
     if (stt != KVG_OK) return stt;
@@ -825,6 +1034,65 @@ static kvg_status finish_verify(kvg_cache *c, int32_t seq, uint32_t flags, int32
     return KVG_OK;
 }
 
+// Own-position graft of a pool-resident block by aliasing: the sequence's
+// page table points at the block's full pages (shared, read-only: appends
+// never write a full page); a partially filled last page is copied into a
+// page of the sequence, because the sequence's appends fill it.
+static kvg_status pool_graft(kvg_store *s, const kvg_store::Blk &blk, kvg_cache *c, int32_t seq, int64_t dst,
+                             int64_t delta, uint32_t flags, cudaStream_t st, kvg_graft_report *report) {
+    if (s->pool_cache != c) return fail(KVG_ERR_ARG, "a pool-resident block grafts only into its own cache");
+    if (delta != 0) return fail(KVG_ERR_ARG, "relocation needs a copying store (HBM or pinned host)");
+    const int64_t P = c->dims.page_size, n = blk.lay.n_tokens, npb = blk.lay.n_pages;
+    if (npb > kMaxPagesPerLaunch) return fail(KVG_ERR_ARG, "pool-resident blocks are limited to %d pages", kMaxPagesPerLaunch);
+    const bool partial = n % P != 0;
+    if (partial && c->free_list.empty()) return fail(KVG_ERR_CAPACITY, "out of free pages");
+    std::vector<int32_t> pages(blk.pids);
+    if (partial) pages.back() = take_pages(c, 1)[0];
+    for (int64_t j = 0; j < npb; ++j)
+        if (pages[j] == blk.pids[j]) ++c->alias[pages[j]];
+    auto &sp = c->seq_pages[seq];
+    const int64_t jdst = dst / P;
+    sp.insert(sp.end(), pages.begin(), pages.end());
+    c->n_slots[seq] = (int32_t)(dst + n);
+    if (partial) {
+        GatherParams p{};
+        p.pool = c->pool;
+        p.dst = c->pool;
+        p.page_bytes = c->page_bytes;
+        p.pool_pages = c->n_pages;
+        p.n_layers = c->dims.n_layers;
+        p.npb = 1;
+        p.page_base = (int32_t)(npb - 1);
+        p.block_pages = (int32_t)npb;
+        p.n_kv_heads = c->dims.n_kv_heads;
+        p.page_size = (int32_t)P;
+        p.head_dim = c->dims.head_dim;
+        p.n_tokens = n;
+        p.src_pos = nullptr;
+        p.pids.n = 1;
+        p.pids.pid[0] = blk.pids.back();
+        p.dst_pids.n = 1;
+        p.dst_pids.pid[0] = pages.back();
+        KVG_CUDA(launch_gather(p, c->n_sm, st));
+    }
+    AliasParams ap{};
+    ap.src_pos = reinterpret_cast<const int32_t *>(blk.dev + blk.lay.pos_off);
+    ap.table_row = c->page_table + (int64_t)seq * c->max_pages + jdst;
+    ap.fill_row = c->page_fill + (int64_t)seq * c->max_pages + jdst;
+    ap.dst_pos = c->positions + (int64_t)seq * c->max_slots + dst;
+    ap.n_tokens = n;
+    ap.page_size = (int32_t)P;
+    ap.pids.n = (int32_t)npb;
+    for (int64_t j = 0; j < npb; ++j) ap.pids.pid[j] = pages[j];
+    KVG_CUDA(launch_alias(ap, c->n_sm, st));
+    if (flags & KVG_GRAFT_VERIFY) {
+        kvg_status r = enqueue_verify(s, blk, c, seq, jdst, false, st);
+        if (r != KVG_OK) return r;
+    }
+    return finish_verify(c, seq, flags, (flags & KVG_GRAFT_VERIFY) ? (int32_t)(c->dims.n_layers * 2 * npb) : 0,
+                         st, report);
+}
+
 extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t dst_slot,
                                 int64_t delta, uint32_t flags, void *stream, kvg_graft_report *report) {
     if (!s || !c) return fail(KVG_ERR_ARG, "null argument");
@@ -840,11 +1108,12 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
     if (dst != boundary) return fail(KVG_ERR_ARG, "dst_slot %d is not the next page boundary %lld", dst_slot, (long long)boundary);
     const int64_t n = blk.lay.n_tokens, npb = blk.lay.n_pages;
     if (dst + n > c->max_slots) return fail(KVG_ERR_CAPACITY, "graft past max_slots");
-    if (npb > (int64_t)c->free_list.size()) return fail(KVG_ERR_CAPACITY, "out of free pages");
+    if (!s->pool_cache && npb > (int64_t)c->free_list.size()) return fail(KVG_ERR_CAPACITY, "out of free pages");
     if (blk.min_pos + delta < 0 || blk.max_pos + delta >= (1ll << 31))
         return fail(KVG_ERR_POSITION, "position tags + delta leave [0, 2^31)");
     DeviceGuard g(c->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (s->pool_cache) return pool_graft(s, blk, c, seq, dst, delta, flags, st, report);
     auto pids = take_pages(c, npb);
     auto &sp = c->seq_pages[seq];
     const int64_t jdst = dst / P;

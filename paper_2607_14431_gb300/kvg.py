@@ -20,7 +20,7 @@ KVG_OK = 0
 KVG_ERR_ARG, KVG_ERR_OOM, KVG_ERR_CUDA, KVG_ERR_NOT_FOUND = -1, -2, -3, -4
 KVG_ERR_CAPACITY, KVG_ERR_POSITION, KVG_ERR_DIGEST, KVG_ERR_FORMAT = -5, -6, -7, -8
 KVG_ERR_TIMEOUT, KVG_ERR_DEVICE_CHECK = -9, -10
-KVG_RESIDENCY_HBM, KVG_RESIDENCY_PINNED_HOST = 0, 1
+KVG_RESIDENCY_HBM, KVG_RESIDENCY_PINNED_HOST, KVG_RESIDENCY_CACHE_POOL = 0, 1, 2
 KVG_ROPE_HALF, KVG_ROPE_INTERLEAVED = 0, 1
 KVG_GRAFT_VERIFY, KVG_GRAFT_SYNC = 1, 2
 KVG_SHA256_PLAIN, KVG_SHA256_PAGED = 0, 1
@@ -68,6 +68,7 @@ _P = ctypes.POINTER
 _SIGNATURES = {
     "kvg_store_create": ([_P(kvg_dims), _i32, _u64, _i32, _P(_vp)], _i32),
     "kvg_store_destroy": ([_vp], None),
+    "kvg_store_create_in_cache": ([_vp, _u64, _P(_vp)], _i32),
     "kvg_store_block_info": ([_vp, _u64, _P(kvg_block_info)], _i32),
     "kvg_store_import": ([_vp, _vp, _u64, _u32, _P(_u64)], _i32),
     "kvg_store_export": ([_vp, _u64, _vp, _u64], _i32),
@@ -141,6 +142,12 @@ def make_dims(n_layers, n_kv_heads, head_dim, page_size, rope_theta=10000.0, rop
 def kvg_store_create(dims: kvg_dims, residency: int, capacity_bytes: int, device: int = 0):
     h = _vp()
     _check(lib().kvg_store_create(ctypes.byref(dims), residency, capacity_bytes, device, ctypes.byref(h)))
+    return h
+
+
+def kvg_store_create_in_cache(cache, capacity_bytes: int):
+    h = _vp()
+    _check(lib().kvg_store_create_in_cache(cache, capacity_bytes, ctypes.byref(h)))
     return h
 
 
@@ -293,6 +300,14 @@ class Store:
             self.close()
         except Exception:
             pass
+
+
+class PoolStore(Store):
+    """A store whose blocks live in `cache`'s page pool (zero-copy graft)."""
+
+    def __init__(self, cache: "Cache", capacity_bytes: int):
+        self.dims = cache.dims
+        self.h = kvg_store_create_in_cache(cache.h, capacity_bytes)
 
 
 class Cache:

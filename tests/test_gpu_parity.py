@@ -413,3 +413,77 @@ def test_block_files_round_trip_and_are_verified(oracle, tmp_path):
     with pytest.raises(kvg.KvgError) as e:
         kvg.kvg_store_load(host.h, path, 0)
     assert e.value.status == kvg.KVG_ERR_FORMAT
+
+
+def test_pool_store_zero_copy_graft(oracle):
+    # blocks living in the cache's own pool: a graft writes only the page
+    # table (full pages shared), a ragged last page is copied, two sequences
+    # share the block's pages while their appends diverge
+    kvg = need_gpu()
+    w = geometry("d128")
+    nb, nf = 333, 100
+    k, v = _kv(w, nb + nf, 131)
+    P = w.page_size
+    max_slots = (-(-(nb + nf) // P) + 2) * P
+    n_pages = 40
+    dims = dims_for(kvg, w)
+    perm = syn.permutation(n_pages, 133)
+    cache = kvg.Cache(dims, n_pages, 4, max_slots)
+    fill_canary(cache)
+    kvg.kvg_cache_set_free_order(cache.h, perm)
+    od = oracle_dims(oracle, w)
+    oc = oracle.OracleCache(od, n_pages, 4, max_slots, fill=CANARY)
+    oc.set_free_order(perm)
+    append(kvg, cache, 0, k[:, :nb], v[:, :nb], syn.positions(0, nb))
+    oc.append(0, k[:, :nb], v[:, :nb], syn.positions(0, nb))
+    store = kvg.PoolStore(cache, 64 << 20)
+    bid = kvg.kvg_deposit(store.h, cache.h, 0, 0, nb)
+    opb = oc.pin_block(0, 0, nb)
+    assert kvg.kvg_store_export(store.h, bid) == opb.block.serialize()
+    kvg.kvg_cache_release(cache.h, 0)
+    oc.release(0)
+    for seq in (1, 2):
+        kvg.kvg_graft(store.h, bid, cache.h, seq, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+        oc.graft_pinned(seq, opb)
+    kvg.kvg_verify(store.h, bid, cache.h, 1, 0, kvg.KVG_GRAFT_SYNC)  # before appends fill the last page
+    append(kvg, cache, 1, k[:, nb:], v[:, nb:], syn.positions(nb, nf))
+    oc.append(1, k[:, nb:], v[:, nb:], syn.positions(nb, nf))
+    k2, v2 = _kv(w, 50, 132)
+    append(kvg, cache, 2, k2, v2, syn.positions(nb, 50))
+    oc.append(2, k2, v2, syn.positions(nb, 50))
+    assert np.array_equal(pool_u16(cache, w), oc.pool)
+    pt, pf, ps = tables(cache)
+    assert np.array_equal(pt, oc.page_table) and np.array_equal(pf, oc.page_fill)
+    assert np.array_equal(ps, oc.positions)
+    full = nb // P
+    assert list(pt[1, :full]) == list(pt[2, :full]) == opb.pids[:full]  # shared, not copied
+    assert pt[1, full] != pt[2, full] != opb.pids[full]                 # ragged page copied per sequence
+    # attention over the aliased rows equals attention over the same rows written fresh
+    q = syn.as_u16(syn.queries(w, w.n_layers, 1, 134))
+    fresh = kvg.Cache(dims, n_pages, 1, max_slots)
+    append(kvg, fresh, 0, k, v, syn.positions(0, nb + nf))
+    assert _sha(decode(kvg, cache, w, [1], q)) == _sha(decode(kvg, fresh, w, [0], q))
+    # releases keep the block's pages; a relocating graft needs a copying store
+    kvg.kvg_cache_release(cache.h, 1)
+    kvg.kvg_cache_release(cache.h, 2)
+    oc.release(1)
+    oc.release(2)
+    kvg.kvg_graft(store.h, bid, cache.h, 3, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+    oc.graft_pinned(3, opb)
+    pt, pf, ps = tables(cache)
+    assert np.array_equal(pt, oc.page_table) and np.array_equal(pool_u16(cache, w), oc.pool)
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_graft(store.h, bid, cache.h, 0, -1, 4096)
+    assert e.value.status == kvg.KVG_ERR_ARG
+    # a flipped byte in a shared page is caught by verification of the sequence
+    v_ = cache.view
+    off = ((1 * 2 + 0) * v_.n_pages + opb.pids[2]) * w.page_bytes + 10
+    page = dev_view(v_.pool + off, 16)
+    page[0] ^= 1
+    torch.cuda.synchronize()
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_verify(store.h, bid, cache.h, 3, 0, kvg.KVG_GRAFT_SYNC)
+    assert e.value.status == kvg.KVG_ERR_DIGEST
+    store.close()
+    fresh.close()
+    cache.close()

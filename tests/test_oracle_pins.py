@@ -444,3 +444,26 @@ def test_cache_errors_and_release(oracle):
     assert c.free == [3, 0, 1, 2]
     with pytest.raises(oracle.KvgError):
         c.graft(1, oracle.block_from_kv(d, k, v, syn.positions(2**31 - 10, 40)))
+
+
+def test_pinned_block_graft_aliases_pages(oracle):
+    d = _dims()
+    n = 40  # 2 full pages + 8 rows
+    k, v = _kv(n, 8)
+    c = oracle.OracleCache(d, 12, 3, 64, fill=CANARY)
+    c.append(0, k, v, syn.positions(0, n))
+    pb = c.pin_block(0, 0, n)
+    assert pb.pids == [3, 4, 5]  # taken after the sequence's own pages 0..2
+    c.release(0)
+    assert c.free == [6, 7, 8, 9, 10, 11, 0, 1, 2]  # pinned pages never return
+    c.graft_pinned(1, pb)
+    c.graft_pinned(2, pb)
+    assert list(c.page_table[1, :2]) == list(c.page_table[2, :2]) == [3, 4]  # shared
+    assert c.page_table[1, 2] == 6 and c.page_table[2, 2] == 7            # ragged page copied
+    for sq in (1, 2):
+        kk, vv, pp = c.logical_kv(sq, 1)
+        assert np.array_equal(kk, k[1]) and np.array_equal(vv, v[1]) and np.array_equal(pp, np.arange(n))
+    c.append(1, k[:, :3], v[:, :3], syn.positions(n, 3))
+    assert np.array_equal(c.pool[:, :, 5], pb.block.pages[:, :, 2])  # the block's own page untouched
+    c.release(1)
+    assert 3 not in c.free and 6 in c.free
