@@ -487,3 +487,53 @@ def test_pool_store_zero_copy_graft(oracle):
     store.close()
     fresh.close()
     cache.close()
+
+
+def test_launch_chunking_limits(oracle):
+    # > 1,024 pages per graft / deposit / append (several launches each) and
+    # > 256 decode rows per call (several batch chunks): same bytes, same
+    # attention as the oracle
+    kvg = need_gpu()
+    w = syn.Workload("p8", 1, 2, 1, 64, 8, 10000.0, 0x61)
+    n = 9000  # 1,125 pages of 8 rows
+    k, v = _kv(w, n, 141)
+    P = w.page_size
+    n_pages = 2 * (-(-n // P)) + 4
+    dims = dims_for(kvg, w)
+    src = kvg.Cache(dims, n_pages, 2, n + 2 * P)
+    append(kvg, src, 0, k, v, syn.positions(0, n))
+    store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, 1 << 30)
+    bid = kvg.kvg_deposit(store.h, src.h, 0, 0, n)
+    od = oracle_dims(oracle, w)
+    oblk = oracle.block_from_kv(od, k, v, syn.positions(0, n))
+    assert kvg.kvg_store_export(store.h, bid) == oblk.serialize()
+    dst = kvg.Cache(dims, n_pages, 2, n + 2 * P)
+    fill_canary(dst)
+    oc = oracle.OracleCache(od, n_pages, 2, n + 2 * P, fill=CANARY)
+    kvg.kvg_graft(store.h, bid, dst.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+    oc.graft(0, oblk)
+    kvg.kvg_graft(store.h, bid, dst.h, 1, -1, 77, kvg.KVG_GRAFT_SYNC)
+    oc.graft(1, oblk, delta=77)
+    pool = pool_u16(dst, w)
+    pt, pf, ps = tables(dst)
+    assert np.array_equal(pt, oc.page_table) and np.array_equal(pf, oc.page_fill)
+    assert np.array_equal(ps, oc.positions)
+    assert np.array_equal(pool[:, 1], oc.pool[:, 1])
+    assert np.array_equal(pool[:, 0, pt[0, :(n + P - 1) // P]], oc.pool[:, 0, pt[0, :(n + P - 1) // P]])
+    kg = _logical_k(pool, pt, w, 1, n)
+    k64 = oracle.rope_rotate_rows(k[0], 77, w.rope_theta, 0)
+    assert np.abs(oracle.bf16_to_f64(kg[0]) - k64).max() <= 2e-2
+    # 300 decode rows over the two sequences (rows alternate; 2 batch chunks)
+    ids = [i % 2 for i in range(300)]
+    q = syn.as_u16(syn.queries(w, 1, 300, 142))
+    o = decode(kvg, dst, w, ids, q)
+    scale = 1 / math.sqrt(w.head_dim)
+    kk1, vv1, _ = oc.logical_kv(1, 0)
+    for b in (0, 1, 255, 256, 299):
+        kk, vv = (k[0], v[0]) if ids[b] == 0 else (kk1, vv1)
+        compare_decode(oracle, o[0, b], oracle.gqa_decode(q[0, b], kk, vv, scale))
+    o_noalloc = torch.empty_like(to_dev(q))
+    qd = to_dev(q)
+    kvg.kvg_decode_attention_noalloc(dst.h, -1, ids, qd.data_ptr(), w.n_q_heads, o_noalloc.data_ptr(), scale)
+    torch.cuda.synchronize()
+    assert np.abs(oracle.bf16_to_f64(u16(o_noalloc)) - oracle.bf16_to_f64(o)).max() <= 1e-2
