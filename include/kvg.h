@@ -356,6 +356,13 @@ kvg_status kvg_digest(const void *bytes, uint64_t n, int32_t mode, uint64_t page
  * gets the details), KVG_ERR_DEVICE_CHECK if a kernel's own check failed. */
 kvg_status kvg_sync(kvg_cache *cache, void *stream, double timeout_s, kvg_graft_report *report);
 
+/* Failure-detection self-test: enqueues a kernel whose wait (an mbarrier
+ * that nothing completes — the same bounded wait every kernel uses for its
+ * asynchronous copies) gives up after limit_ns (at most 10 s) and records
+ * KVG_ERR_DEVICE_CHECK in the cache's status word; the next kvg_sync returns
+ * it and the context stays usable.  Nothing faults or hangs. */
+kvg_status kvg_selftest_bounded_wait(kvg_cache *cache, uint64_t limit_ns, void *stream);
+
 const char *kvg_status_string(kvg_status status);
 
 /* Human-readable detail of the last failed call on this host thread (empty if

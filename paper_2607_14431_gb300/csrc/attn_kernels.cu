@@ -159,12 +159,35 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
 
     const int64_t plane_rows = p.pool_pages * (int64_t)p.n_kv_heads * P;  // rows per (layer, K/V)
 
-    // lane 0: arm the stage's barrier and copy the tile's K and V boxes
-    auto issue = [&](int64_t t, int stg) {
-        const TilePos tp = locate(p, t);
-        const int seq = p.rows.seq[tp.b];
-        const int jj = tp.tile / tpp;
-        const int k = tp.tile - jj * tpp;
+    // Lane 0's cursor over the tiles it copies: tiles are issued in order, so
+    // the position advances by one; it is re-located only at a unit boundary.
+    struct Cursor {
+        int64_t t, end;  // next tile to issue; first tile past its unit
+        int lr, b, g, seq, jj, k;
+    } cur;
+    cur.t = t0;
+    cur.end = t0;
+    auto advance_to_unit = [&]() {
+        const TilePos tp = locate(p, cur.t);
+        cur.lr = tp.lr;
+        cur.b = tp.b;
+        cur.g = tp.g;
+        cur.seq = p.rows.seq[tp.b];
+        cur.jj = tp.tile / tpp;
+        cur.k = tp.tile - cur.jj * tpp;
+        cur.end = cur.t - tp.tile + (p.rows.pref_tiles[tp.b + 1] - p.rows.pref_tiles[tp.b]);
+    };
+
+    // lane 0: arm the stage's barrier and copy the next tile's K and V boxes
+    auto issue = [&](int stg) {
+        if (cur.t >= cur.end) advance_to_unit();
+        const int seq = cur.seq, jj = cur.jj, k = cur.k;
+        struct { int lr, g; } tp{cur.lr, cur.g};
+        ++cur.t;
+        if (++cur.k == tpp) {
+            cur.k = 0;
+            ++cur.jj;
+        }
         const int fill = p.page_fill[(int64_t)seq * p.max_pages + jj];
         const int pid = p.page_table[(int64_t)seq * p.max_pages + jj];
         int vr = fill - k * TOK;
@@ -243,7 +266,7 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
     };
 
     if (lane == 0)
-        for (int i = 0; i < STAGES && t0 + i < t1; ++i) issue(t0 + i, i);
+        for (int i = 0; i < STAGES && t0 + i < t1; ++i) issue(i);
 
     const uint32_t ring_s = smem_addr(ring);
     bool alive = true;
@@ -363,7 +386,7 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
         }
         __syncwarp();
         (void)zeroed;
-        if (lane == 0 && t + STAGES < t1) issue(t + STAGES, stg);
+        if (lane == 0 && t + STAGES < t1) issue(stg);
     }
     if (!alive) {
         // a copy never completed: wait (bounded) on every stage once more so

@@ -192,6 +192,9 @@ cudaError_t launch_append_batch(const AppendBatchParams &p, int n_sm, cudaStream
 cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_write_header(const HeaderParams &p, cudaStream_t s);
 cudaError_t launch_alias(const AliasParams &p, int n_sm, cudaStream_t s);
+// A kernel whose mbarrier nothing completes: its bounded wait gives up after
+// limit_ns and records KVG_ERR_DEVICE_CHECK (detail 3) in `status`.
+cudaError_t launch_wait_selftest(DevStatus *status, uint64_t limit_ns, cudaStream_t s);
 cudaError_t launch_write_ints(const IntsParams &p, cudaStream_t s);
 cudaError_t launch_reset_seq(int32_t *table_row, int32_t *fill_row, int32_t max_pages,
                              int32_t *pos_row, int32_t max_slots, cudaStream_t s);
@@ -267,14 +270,16 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
     return t;
 }
 
-// Bounded wait on an mbarrier phase: gives up after ~2 s of wall time and
-// returns false (the caller records KVG_ERR_DEVICE_CHECK and unwinds).
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
+// Bounded wait on an mbarrier phase: gives up after limit_ns of wall time
+// (default ~2 s) and returns false; the caller records KVG_ERR_DEVICE_CHECK
+// in its status word and unwinds instead of hanging the GPU.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity,
+                                                  uint64_t limit_ns = 2000000000ull) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     for (uint32_t it = 0;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 255u) == 255u && global_timer_ns() - t0 > 2000000000ull) return false;
+        if ((it & 255u) == 255u && global_timer_ns() - t0 > limit_ns) return false;
     }
 }
 

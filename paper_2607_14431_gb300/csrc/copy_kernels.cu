@@ -318,6 +318,18 @@ __global__ void __launch_bounds__(256) alias_kernel(const AliasParams p) {
     }
 }
 
+__global__ void wait_selftest_kernel(DevStatus *status, uint64_t limit_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    // no thread arrives and no copy completes: phase 0 never completes
+    const bool ok = mbar_wait_bounded(&bar, 0, limit_ns);
+    if (!ok && threadIdx.x == 0) record_error(status, KVG_ERR_DEVICE_CHECK, 3);
+}
+
 __global__ void write_ints_kernel(const IntsParams p) {
     for (int i = threadIdx.x; i < p.vals.n; i += blockDim.x) p.dst[i] = p.vals.pid[i];
 }
@@ -385,6 +397,12 @@ cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s) {
 
 cudaError_t launch_alias(const AliasParams &p, int n_sm, cudaStream_t s) {
     alias_kernel<<<grid_for(p.n_tokens > p.pids.n ? p.n_tokens : p.pids.n, 256, n_sm, 1), 256, 0, s>>>(p);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_wait_selftest(DevStatus *status, uint64_t limit_ns, cudaStream_t s) {
+    wait_selftest_kernel<<<1, 32, 0, s>>>(status, limit_ns);
     count_launches(1);
     return cudaGetLastError();
 }

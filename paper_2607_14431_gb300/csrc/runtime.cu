@@ -19,9 +19,20 @@
 #include <thread>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "common.cuh"
 
 using namespace kvg;
+
+namespace {
+// NVTX range around each ABI call, so a profiler's timeline names the
+// library call that enqueued each kernel.
+struct Trace {
+    explicit Trace(const char *name) { nvtxRangePushA(name); }
+    ~Trace() { nvtxRangePop(); }
+};
+}  // namespace
 
 namespace kvg {
 static std::atomic<uint64_t> g_launches{0};
@@ -350,6 +361,7 @@ static kvg_status pool_import(kvg_store *s, const uint8_t *h, const BlockLayout 
 
 extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t n_bytes, uint32_t flags,
                                        uint64_t *block_id_out) {
+    Trace trace_("kvg_store_import");
     if (!s || !bytes || !block_id_out) return fail(KVG_ERR_ARG, "null argument");
     const uint8_t *h = static_cast<const uint8_t *>(bytes);
     if (n_bytes < 256 || memcmp(h, "KVGBLK01", 8) != 0) return fail(KVG_ERR_FORMAT, "bad magic");
@@ -408,6 +420,7 @@ extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t
 }
 
 extern "C" kvg_status kvg_store_export(kvg_store *s, uint64_t id, void *dst, uint64_t dst_bytes) {
+    Trace trace_("kvg_store_export");
     if (!s || !dst) return fail(KVG_ERR_ARG, "null argument");
     if (id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)id);
     const auto &b = s->blocks[id];
@@ -423,6 +436,7 @@ extern "C" kvg_status kvg_store_export(kvg_store *s, uint64_t id, void *dst, uin
 }
 
 extern "C" kvg_status kvg_store_save(kvg_store *s, uint64_t id, const char *path) {
+    Trace trace_("kvg_store_save");
     if (!s || !path) return fail(KVG_ERR_ARG, "null argument");
     if (id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)id);
     const auto &b = s->blocks[id];
@@ -446,6 +460,7 @@ extern "C" kvg_status kvg_store_save(kvg_store *s, uint64_t id, const char *path
 }
 
 extern "C" kvg_status kvg_store_load(kvg_store *s, const char *path, uint32_t flags, uint64_t *block_id_out) {
+    Trace trace_("kvg_store_load");
     if (!s || !path || !block_id_out) return fail(KVG_ERR_ARG, "null argument");
     FILE *f = fopen(path, "rb");
     if (!f) return fail(KVG_ERR_ARG, "cannot open %s", path);
@@ -739,6 +754,7 @@ static std::vector<int32_t> take_pages(kvg_cache *c, int64_t n) {
 
 extern "C" kvg_status kvg_cache_append(kvg_cache *c, int32_t seq, const void *k, const void *v,
                                        const int32_t *positions, int32_t n, void *stream) {
+    Trace trace_("kvg_cache_append");
     if (!c) return fail(KVG_ERR_ARG, "null cache");
     if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d", seq);
     if (n < 0) return fail(KVG_ERR_ARG, "negative n");
@@ -790,6 +806,7 @@ extern "C" kvg_status kvg_cache_append(kvg_cache *c, int32_t seq, const void *k,
 
 extern "C" kvg_status kvg_cache_append_batch(kvg_cache *c, const int32_t *seq_ids, int32_t B, const void *k,
                                              const void *v, const int32_t *positions, void *stream) {
+    Trace trace_("kvg_cache_append_batch");
     if (!c || !seq_ids || !k || !v || !positions) return fail(KVG_ERR_ARG, "null argument");
     if (B <= 0 || B > kMaxBatchPerLaunch) return fail(KVG_ERR_ARG, "B must be in [1, %d]", kMaxBatchPerLaunch);
     if ((reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(v)) & 15)
@@ -841,6 +858,7 @@ extern "C" kvg_status kvg_cache_append_batch(kvg_cache *c, const int32_t *seq_id
 }
 
 extern "C" kvg_status kvg_cache_release(kvg_cache *c, int32_t seq, void *stream) {
+    Trace trace_("kvg_cache_release");
     if (!c) return fail(KVG_ERR_ARG, "null cache");
     if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d", seq);
     DeviceGuard g(c->device);
@@ -918,6 +936,7 @@ static kvg_status pool_deposit(kvg_store *s, kvg_cache *c, int32_t seq, int32_t 
 
 extern "C" kvg_status kvg_deposit(kvg_store *s, const kvg_cache *cc, int32_t seq, int32_t slot0, int32_t n,
                                   void *stream, uint64_t *block_id_out) {
+    Trace trace_("kvg_deposit");
     kvg_cache *c = const_cast<kvg_cache *>(cc);
     if (!s || !c || !block_id_out) return fail(KVG_ERR_ARG, "null argument");
     if (!same_geometry(s->dims, c->dims)) return fail(KVG_ERR_ARG, "store and cache geometry differ");
@@ -1095,6 +1114,7 @@ static kvg_status pool_graft(kvg_store *s, const kvg_store::Blk &blk, kvg_cache 
 
 extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t dst_slot,
                                 int64_t delta, uint32_t flags, void *stream, kvg_graft_report *report) {
+    Trace trace_("kvg_graft");
     if (!s || !c) return fail(KVG_ERR_ARG, "null argument");
     if (block_id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)block_id);
     if (!same_geometry(s->dims, c->dims)) return fail(KVG_ERR_ARG, "store and cache geometry differ");
@@ -1167,6 +1187,7 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
 
 extern "C" kvg_status kvg_verify(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t slot0,
                                  uint32_t flags, void *stream, kvg_graft_report *report) {
+    Trace trace_("kvg_verify");
     if (!s || !c) return fail(KVG_ERR_ARG, "null argument");
     if (block_id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)block_id);
     if (!same_geometry(s->dims, c->dims)) return fail(KVG_ERR_ARG, "store and cache geometry differ");
@@ -1208,6 +1229,7 @@ static int64_t fill_rows(const kvg_cache *c, const int32_t *seq_ids, int64_t b0,
 extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
                                            const void *q, int32_t n_q_heads, void *out, float scale,
                                            void *stream) {
+    Trace trace_("kvg_decode_attention");
     if (!c || !seq_ids || !q || !out) return fail(KVG_ERR_ARG, "null argument");
     const kvg_dims &d = c->dims;
     if (layer < -1 || layer >= d.n_layers) return fail(KVG_ERR_ARG, "bad layer %d", layer);
@@ -1269,6 +1291,7 @@ DevStatus *g_digest_status[64] = {};
 
 extern "C" kvg_status kvg_digest(const void *bytes, uint64_t n, int32_t mode, uint64_t page_bytes, uint8_t *out,
                                  void *stream) {
+    Trace trace_("kvg_digest");
     if (!out || (n && !bytes)) return fail(KVG_ERR_ARG, "null argument");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     int dev = 0;
@@ -1300,6 +1323,7 @@ extern "C" kvg_status kvg_digest(const void *bytes, uint64_t n, int32_t mode, ui
 // -------------------------------------------------------------------- misc --
 
 extern "C" kvg_status kvg_sync(kvg_cache *c, void *stream, double timeout_s, kvg_graft_report *report) {
+    Trace trace_("kvg_sync");
     if (!c) return fail(KVG_ERR_ARG, "null cache");
     DeviceGuard g(c->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -1314,6 +1338,14 @@ extern "C" kvg_status kvg_sync(kvg_cache *c, void *stream, double timeout_s, kvg
     }
     if (report) memset(report, 0, sizeof *report);
     return read_status(c, report);
+}
+
+extern "C" kvg_status kvg_selftest_bounded_wait(kvg_cache *c, uint64_t limit_ns, void *stream) {
+    if (!c) return fail(KVG_ERR_ARG, "null cache");
+    if (limit_ns == 0 || limit_ns > 10000000000ull) return fail(KVG_ERR_ARG, "limit must be in (0, 10 s]");
+    DeviceGuard g(c->device);
+    KVG_CUDA(launch_wait_selftest(c->status, limit_ns, static_cast<cudaStream_t>(stream)));
+    return KVG_OK;
 }
 
 extern "C" const char *kvg_status_string(kvg_status s) {

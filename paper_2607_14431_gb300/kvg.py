@@ -89,6 +89,7 @@ _SIGNATURES = {
     "kvg_decode_attention_noalloc": ([_vp, _i32, _vp, _i32, _vp, _i32, _vp, ctypes.c_float, _vp], _i32),
     "kvg_digest": ([_vp, _u64, _i32, _u64, _vp, _vp], _i32),
     "kvg_sync": ([_vp, _vp, ctypes.c_double, _P(kvg_graft_report)], _i32),
+    "kvg_selftest_bounded_wait": ([_vp, _u64, _vp], _i32),
     "kvg_status_string": ([_i32], ctypes.c_char_p),
     "kvg_last_error": ([], ctypes.c_char_p),
     "kvg_version": ([], _u32),
@@ -265,6 +266,10 @@ def kvg_digest(ptr: int, n: int, mode: int, page_bytes: int, out_ptr: int, strea
 def kvg_sync(cache, stream=None, timeout_s: float = 10.0, report: kvg_graft_report | None = None):
     _check(lib().kvg_sync(cache, _stream(stream), timeout_s,
                           ctypes.byref(report) if report is not None else None))
+
+
+def kvg_selftest_bounded_wait(cache, limit_ns: int, stream=None):
+    _check(lib().kvg_selftest_bounded_wait(cache, limit_ns, _stream(stream)))
 
 
 def kvg_status_string(status: int) -> str:

@@ -537,3 +537,22 @@ def test_launch_chunking_limits(oracle):
     kvg.kvg_decode_attention_noalloc(dst.h, -1, ids, qd.data_ptr(), w.n_q_heads, o_noalloc.data_ptr(), scale)
     torch.cuda.synchronize()
     assert np.abs(oracle.bf16_to_f64(u16(o_noalloc)) - oracle.bf16_to_f64(o)).max() <= 1e-2
+
+
+def test_device_wait_gives_up_and_reports(oracle):
+    # every kernel wait on an asynchronous copy is bounded; a wait that nothing
+    # completes gives up, records a device-check status, and the context stays
+    # usable (no trap, no hang)
+    kvg = need_gpu()
+    w = geometry("tiny")
+    cache = kvg.Cache(dims_for(kvg, w), 20, 1, 320)
+    kvg.kvg_selftest_bounded_wait(cache.h, 20_000_000)  # 20 ms
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_sync(cache.h, None, 10.0)
+    assert e.value.status == kvg.KVG_ERR_DEVICE_CHECK
+    kvg.kvg_sync(cache.h, None, 10.0)  # status word cleared
+    k, v = _kv(w, 100, 151)
+    append(kvg, cache, 0, k, v, syn.positions(0, 100))
+    q = syn.as_u16(syn.queries(w, w.n_layers, 1, 152))
+    o = decode(kvg, cache, w, [0], q)
+    compare_decode(oracle, o[0, 0], oracle.gqa_decode(q[0, 0], k[0], v[0], 1 / math.sqrt(w.head_dim)))
