@@ -129,7 +129,7 @@ class Clocks:
 class Step12B:
     """Device state and the per-step call sequence for the 12B workload."""
 
-    def __init__(self, kvg, device, stream, side, n_layers=None, pool_store=False):
+    def __init__(self, kvg, device, stream, side, n_layers=None, pool_store=False, schedule="overlap"):
         self.kvg = kvg
         self.w = w = syn.B12 if not n_layers else syn.B12.with_layers(n_layers)
         self.dev = device
@@ -171,15 +171,31 @@ class Step12B:
                       + 2 * self.q.numel() * 2,
         }
         self.sha_blocks = (blk_pages // 4096) * 65
-        self.phases = ["release", "graft", "append", "decode", "verify_join", "verify"]
+        self.blk_pages = blk_pages
+        # the step's work, whatever the schedule: block bytes copied (read +
+        # write) and hashed, fresh rows read and written, K/V rows decoded
+        self.step_bytes = sum(self.bytes.values())
+        self.schedule = schedule
+        # phase -> (stream, first event, last event) of the per-step events
+        if schedule == "fused":
+            self.bytes["graft_verify"] = self.bytes.pop("graft") or blk_pages
+            self.bytes.pop("verify")
+            self.spans = {"release": ("main", 0, 1), "append": ("main", 1, 2), "graft_join": ("main", 2, 3),
+                          "decode": ("main", 3, 4), "graft_verify": ("side", 0, 1)}
+        else:
+            self.spans = {"release": ("main", 0, 1), "graft": ("main", 1, 2), "append": ("main", 2, 3),
+                          "decode": ("main", 3, 4), "verify_join": ("main", 4, 5), "verify": ("side", 0, 1)}
+        self.phases = list(self.spans)
 
     def run_step(self, store=None, bid=None, ev=None):
-        """One step.  The digest check only reads the grafted pages, which
-        neither the append nor the decode writes, so it runs on a side stream:
-        its ALU-bound hashing overlaps the HBM-bound append and decode (the
-        kernels' grids are sized so all three fit on an SM together); the main
-        stream waits for it before the step ends.
+        """One step.  Schedule "overlap": the graft copies, then the digest
+        check (which only reads the grafted pages, written by neither the
+        append nor the decode) runs on a side stream, its ALU-bound hashing
+        overlapping the HBM-bound append and decode; the main stream waits for
+        it before the step ends.  Schedule "fused": see _run_fused.
         ev: optional per-phase timing events (main: 6, side: 2)."""
+        if self.schedule == "fused":
+            return self._run_fused(store, bid, ev)
         kvg, s, side, c = self.kvg, self.stream, self.side, self.cache.h
         store = store or self.store.h
         bid = self.bid if bid is None else bid
@@ -203,6 +219,32 @@ class Step12B:
         s.wait_event(self.ev_verify)
         if m: m[5].record(s)
 
+    def _run_fused(self, store=None, bid=None, ev=None):
+        """The same step with the digest check folded into the graft: the
+        verified graft (one pass: copy + leaf hashes, then page digests) runs
+        on a side stream while the main stream appends the fresh rows into
+        other pages; the decode waits for both."""
+        kvg, s, side, c = self.kvg, self.stream, self.side, self.cache.h
+        store = store or self.store.h
+        bid = self.bid if bid is None else bid
+        m = ev["main"] if ev else None
+        if m: m[0].record(s)
+        kvg.kvg_cache_release(c, 0, s)
+        if m: m[1].record(s)
+        self.ev_graft.record(s)
+        side.wait_event(self.ev_graft)
+        if ev: ev["side"][0].record(side)
+        kvg.kvg_graft(store, bid, c, 0, -1, 0, kvg.KVG_GRAFT_VERIFY, side)
+        if ev: ev["side"][1].record(side)
+        self.ev_verify.record(side)
+        kvg.kvg_cache_append(c, 0, self.kf.data_ptr(), self.vf.data_ptr(), self.pf.data_ptr(), self.nf, s)
+        if m: m[2].record(s)
+        s.wait_event(self.ev_verify)
+        if m: m[3].record(s)
+        kvg.kvg_decode_attention(c, -1, [0], self.q.data_ptr(), self.w.n_q_heads, self.out.data_ptr(),
+                                 self.scale, s)
+        if m: m[4].record(s)
+
 def run_kvg(args, rank, world):
     from paper_2607_14431_gb300 import build
     build.build()
@@ -214,7 +256,7 @@ def run_kvg(args, rank, world):
     stream = torch.cuda.Stream(device)
     side = torch.cuda.Stream(device)
     hbm_peak, sm_max, peak_kind = load_peaks()
-    st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool")
+    st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool", schedule=args.schedule)
 
     # correctness of the configuration being timed: one verified step
     st.run_step()
@@ -248,12 +290,10 @@ def run_kvg(args, rank, world):
     clk = clocks.stop()
     total_ms = t_start.elapsed_time(t_end)
     kvg.kvg_sync(st.cache.h, stream, 60.0)  # digest verification of every timed step passed
-    step_bytes = sum(st.bytes.values())
+    step_bytes = st.step_bytes
     ms_step, value = aggregate(total_ms, K, step_bytes, world, device)
-    main_idx = {"release": 0, "graft": 1, "append": 2, "decode": 3, "verify_join": 4}
-    phase_ms = {p: statistics.mean(evs[k]["main"][i].elapsed_time(evs[k]["main"][i + 1]) for k in range(K))
-                for p, i in main_idx.items()}
-    phase_ms["verify"] = statistics.mean(evs[k]["side"][0].elapsed_time(evs[k]["side"][1]) for k in range(K))
+    phase_ms = {p: statistics.mean(evs[k][sn][i].elapsed_time(evs[k][sn][j]) for k in range(K))
+                for p, (sn, i, j) in st.spans.items()}
     deterministic = _sha_tensor(st.out) == first_sha
 
     # e2e: host-store graft, query from pinned host memory, output read back
@@ -275,7 +315,7 @@ def run_kvg(args, rank, world):
                 ts.append(time.perf_counter() - t0)
         kvg.kvg_sync(st.cache.h, stream, 60.0)
         e2e_ms = statistics.mean(ts) * 1e3
-        blk_read = st.bytes["verify"]  # block pages read from host memory by the graft
+        blk_read = st.blk_pages  # block pages read from host memory by the graft
         e2e = {"value": round(world * step_bytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
                "ms_per_step": round(e2e_ms, 3),
                "h2d_bytes_per_step": int(blk_read + st.q.numel() * 2),
@@ -295,27 +335,28 @@ def run_kvg(args, rank, world):
 
     traffic = load_traffic()
     parts = {}
+    hashing = ("verify", "graft_verify")
     for p in st.phases:
         ms = phase_ms[p]
-        if p in ("release", "verify_join") or st.bytes.get(p) == 0:
+        if not st.bytes.get(p):
             parts[p] = {"ms": round(ms, 4)}
             continue
         b = st.bytes[p]
         gbs = b / (ms * 1e-3) / 1e9
         parts[p] = {"ms": round(ms, 4), "algorithmic_bytes": b, "gbs": round(gbs, 1)}
-        if p == "verify":
+        if p in hashing:
             ops = st.sha_blocks * SHA_OPS_PER_BLOCK
             alu_peak = 152 * 64 * sm_max * 1e6
             parts[p].update({"gops": round(ops / (ms * 1e-3) / 1e9, 1),
                              "alu_frac": round(ops / (ms * 1e-3) / alu_peak, 3)})
-        else:
+        if p != "verify":
             parts[p]["hbm_frac"] = round(gbs / hbm_peak, 3)
     parts["decode"]["tokens_per_s"] = round(1e3 / phase_ms["decode"], 1)
-    kernel_of = {"graft": "graft_kernel", "verify": "sha256_leaves_kernel", "append": "append_kernel",
-                 "decode": "decode_kernel"}
-    # dominant kernel: the longest phase on the step's critical (main-stream) path
-    dom = max(("graft", "append", "decode", "verify"), key=lambda p: phase_ms[p] if st.bytes[p] else 0.0)
-    if dom == "verify":
+    kernel_of = {"graft": "graft_kernel", "verify": "sha256_leaves_kernel", "append": "append_tma_kernel",
+                 "decode": "decode_kernel", "graft_verify": "graft_verify_kernel"}
+    # dominant kernel: the longest phase that moves or hashes bytes
+    dom = max((p for p in st.phases if st.bytes.get(p)), key=lambda p: phase_ms[p])
+    if dom in hashing:
         ops = st.sha_blocks * SHA_OPS_PER_BLOCK
         ach = ops / (phase_ms[dom] * 1e-3) / 1e12
         peak = 152 * 64 * sm_max * 1e6 / 1e12
@@ -327,13 +368,22 @@ def run_kvg(args, rank, world):
         roof = {"bound": "hbm", "kernel": kernel_of[dom], "achieved": round(ach, 1), "peak": hbm_peak,
                 "unit": "GB/s", "frac": round(ach / hbm_peak, 3), "traffic": traffic.get(kernel_of[dom]),
                 "peak_kind": peak_kind}
+    if st.schedule == "fused":
+        # the append shares HBM with the verified graft running beside it: the
+        # window from the release to the decode's start moves both kernels' bytes
+        win = statistics.mean(evs[k]["main"][1].elapsed_time(evs[k]["main"][3]) for k in range(K))
+        wb = st.bytes["append"] + st.bytes["graft_verify"]
+        roof["concurrent"] = {"kernels": ["append_tma_kernel", "graft_verify_kernel"], "window_ms": round(win, 4),
+                              "bytes": wb, "achieved": round(wb / (win * 1e-3) / 1e9, 1),
+                              "frac": round(wb / (win * 1e-3) / 1e9 / hbm_peak, 3)}
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": f"12b-single-graft: L{st.w.n_layers} Hq16/Hkv8 D256 P64, 8192-token block grafted "
                                "at own positions (digest-verified) + 24576 fresh tokens, decode 1 token over 32768"
-                               + (" [block in the cache pool: zero-copy graft]" if st.pool_store else ""),
+                               + (" [block in the cache pool: zero-copy graft]" if st.pool_store else "")
+                               + (" [verified graft in one pass, beside the append]" if st.schedule == "fused" else ""),
                    "global_batch": world, "seq_len": syn.B12_CTX, "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)"},
         "parts": parts, "roofline": roof, "e2e": e2e, "gpu_launches": int(launches),
@@ -747,6 +797,9 @@ def main():
     ap.add_argument("--layers", type=int, default=0, help="layer count override (small profiling cases)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--config", default="12b", choices=["12b", "31b", "batched", "deep"])
+    ap.add_argument("--schedule", default="fused", choices=["overlap", "fused"],
+                    help="12b step: digest check on a side stream after the graft (overlap) or folded "
+                         "into the graft, which runs beside the append (fused)")
     ap.add_argument("--store", default="hbm", choices=["hbm", "pool"],
                     help="12b: block in an HBM store (copying graft) or in the cache pool (zero-copy graft)")
     ap.add_argument("--deep-blocks", type=int, default=syn.DEEP_BLOCKS)

@@ -266,9 +266,13 @@ typedef struct kvg_graft_report {
  * host-fp64 cos/sin table, rounded to bf16 RNE); value rows and padding rows
  * are copied unchanged.  delta == 0 is the pure copy.
  * Blocks of a pinned-host store are read by the GPU directly from host memory.
- * flags: KVG_GRAFT_VERIFY hashes every page the graft read (delta != 0: the
- * store's pages; delta == 0: the restored cache pages) and compares with the
- * stored digests; KVG_GRAFT_SYNC waits for completion, fills `report`
+ * flags: KVG_GRAFT_VERIFY hashes every page the graft read and compares with
+ * the stored digests.  With delta == 0 this is one pass: each 4 KiB leaf is
+ * read from the store once, written to its cache page and hashed from the same
+ * registers, so the digest covers exactly the restored bytes; with delta != 0
+ * the store's pages are hashed after the copy.  Verifying calls on one cache
+ * (this flag, kvg_verify) share its leaf-digest scratch, so they must not run
+ * concurrently on different streams.  KVG_GRAFT_SYNC waits for completion, fills `report`
  * (nullable) and returns KVG_ERR_DIGEST on a mismatch.  Without SYNC a
  * mismatch surfaces at the next kvg_sync().
  * Errors (no state change): KVG_ERR_NOT_FOUND, KVG_ERR_ARG (geometry or

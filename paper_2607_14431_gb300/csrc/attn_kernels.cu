@@ -467,19 +467,40 @@ struct DecodeLaunch {
 
 }  // namespace
 
-cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, uint64_t rows) {
-    typedef CUresult (*EncodeTiled)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                    const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
-                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-    static EncodeTiled encode = nullptr;
-    if (!encode) {
-        void *fn = nullptr;
+namespace {
+typedef CUresult (*EncodeTiled)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+// The driver's tensor-map encoder, looked up once (thread-safe static init).
+EncodeTiled tensor_map_encoder() {
+    static const EncodeTiled fn = []() -> EncodeTiled {
+        void *f = nullptr;
         cudaDriverEntryPointQueryResult q;
-        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
-        if (e != cudaSuccess) return e;
-        if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorSymbolNotFound;
-        encode = reinterpret_cast<EncodeTiled>(fn);
-    }
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return nullptr;
+        return reinterpret_cast<EncodeTiled>(f);
+    }();
+    return fn;
+}
+}  // namespace
+
+cudaError_t encode_tensor_map(CUtensorMap *out, int rank, void *base, const cuuint64_t *dims,
+                              const cuuint64_t *strides, const cuuint32_t *box) {
+    const EncodeTiled encode = tensor_map_encoder();
+    if (!encode) return cudaErrorSymbolNotFound;
+    const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    const CUresult r = encode(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, base, dims, strides, box, estr,
+                              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, uint64_t rows) {
+    const EncodeTiled encode = tensor_map_encoder();
+    if (!encode) return cudaErrorSymbolNotFound;
     const int tok = decode_tile_tokens(head_dim);
     if (tok == 0 || rows == 0 || rows > 0x7fffffffull) return cudaErrorInvalidValue;
     const cuuint64_t dims[2] = {(cuuint64_t)head_dim, (cuuint64_t)rows};

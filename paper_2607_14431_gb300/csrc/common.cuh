@@ -65,6 +65,23 @@ struct GraftParams {
     PageList pids;
 };
 
+// Position tags (+ delta), page-table entries and fill counts of one graft
+// launch's pages, written grid-stride by every thread of the launch.
+__device__ __forceinline__ void graft_metadata(const GraftParams &p) {
+    const int64_t P = p.page_size;
+    const int64_t tok0 = (int64_t)p.page_base * P;
+    int64_t n_meta = (int64_t)p.npb * P;
+    if (tok0 + n_meta > p.n_tokens) n_meta = p.n_tokens - tok0;
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t t = gtid; t < n_meta; t += gsz) p.dst_pos[t] = (int32_t)((int64_t)p.src_pos[t] + p.delta);
+    for (int64_t j = gtid; j < p.npb; j += gsz) {
+        p.table_row[j] = p.pids.pid[j];
+        const int64_t f = p.n_tokens - (tok0 + j * P);
+        p.fill_row[j] = (int32_t)(f < P ? f : P);
+    }
+}
+
 // ---------------------------------------------------------------- append --
 struct AppendParams {
     const uint16_t *k, *v;     // [L][n][Hkv][D]
@@ -187,6 +204,15 @@ uint64_t launch_count();
 int env_knob(const char *name, int fallback);
 
 cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s);
+// Bulk append by tensor copies, for appends of at least append_tma_rows()
+// rows (16-byte aligned k/v).  Returns cudaErrorNotSupported (nothing
+// launched) when the tensor maps cannot be encoded, so the caller can take
+// launch_append().
+int32_t append_tma_rows(int32_t page_size, int32_t head_dim);
+cudaError_t launch_append_tma(const AppendParams &p, DevStatus *status, int n_sm, cudaStream_t s);
+// Own-position graft (delta 0) fused with the leaf hashes of the copied pages:
+// leaf_words[(block page) * leaves_per_page + leaf] gets the leaf's state words.
+cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int n_sm, cudaStream_t s);
 cudaError_t launch_append(const AppendParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_append_batch(const AppendBatchParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s);
@@ -222,6 +248,10 @@ cudaError_t launch_decode(int head_dim, int group, const DecodeParams &p, const 
 // head_dim columns and n_layers*2*n_pages*n_kv_heads*page_size rows, boxes of
 // 64 columns x decode_tile_tokens(head_dim) rows, 128-byte swizzle.
 cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, uint64_t rows);
+// A rank-`rank` bf16 tensor map (no swizzle, zero fill out of bounds): dims
+// innermost first, byte strides of dims 1.., box extents per dim.
+cudaError_t encode_tensor_map(CUtensorMap *out, int rank, void *base, const cuuint64_t *dims,
+                              const cuuint64_t *strides, const cuuint32_t *box);
 cudaError_t launch_combine(int head_dim, int group, const DecodeParams &p, cudaStream_t s);
 bool decode_supported(int head_dim, int group);
 int decode_tile_tokens(int head_dim);
@@ -305,6 +335,37 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
             "r"(smem_addr(dst)),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
         : "memory");
+}
+
+// 4-D tensor copy (TMA) of one box at coordinates (x, y, z, w) of `map`.
+// x * element size must be a multiple of 16 bytes (callers pass x = 0).
+__device__ __forceinline__ void tma_load_4d(void *dst, const CUtensorMap *map, int32_t x, int32_t y, int32_t z,
+                                            int32_t w, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];" ::
+            "r"(smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(w), "r"(smem_addr(bar))
+        : "memory");
+}
+
+// Bulk (non-tensor) asynchronous copy of this CTA's shared memory to global
+// memory, tracked by the bulk async-group of the issuing thread.  dst/src
+// 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_s2g(void *dst, const void *src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(smem_addr(src)),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Waits until at most N of the thread's bulk groups still read shared memory.
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// Waits until at most N of the thread's bulk groups are still incomplete.
+template <int N>
+__device__ __forceinline__ void bulk_wait() {
+    asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
 }
 
 __device__ __forceinline__ void fence_proxy_async_shared() {

@@ -144,21 +144,7 @@ __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const ui
 template <int ROT>
 __global__ void __launch_bounds__(kCopyThreads) graft_kernel(const GraftParams p) {
     const int64_t P = p.page_size;
-    // metadata: position tags, page table and fill counts of this launch's pages
-    {
-        const int64_t tok0 = (int64_t)p.page_base * P;
-        int64_t n_meta = (int64_t)p.npb * P;
-        if (tok0 + n_meta > p.n_tokens) n_meta = p.n_tokens - tok0;
-        const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-        const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
-        for (int64_t t = gtid; t < n_meta; t += gsz)
-            p.dst_pos[t] = (int32_t)((int64_t)p.src_pos[t] + p.delta);
-        for (int64_t j = gtid; j < p.npb; j += gsz) {
-            p.table_row[j] = p.pids.pid[j];
-            int64_t f = p.n_tokens - (tok0 + j * P);
-            p.fill_row[j] = (int32_t)(f < P ? f : P);
-        }
-    }
+    graft_metadata(p);
     const uint64_t page_bytes = p.page_bytes;
     const int cpp = (int)(page_bytes / (uint64_t)p.chunk_bytes);
     const int64_t n_units = (int64_t)p.n_layers * 2 * p.npb * cpp;
@@ -187,7 +173,8 @@ __global__ void __launch_bounds__(kCopyThreads) graft_kernel(const GraftParams p
 constexpr int kAppendThreads = 256;
 constexpr int kAppendUnroll = 8;
 
-__global__ void __launch_bounds__(kAppendThreads) append_kernel(const AppendParams p) {
+// Position tags, page-table entries and fill counts of one append launch.
+__device__ __forceinline__ void append_metadata(const AppendParams &p) {
     const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
     const int64_t P = p.page_size;
@@ -198,6 +185,13 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(const AppendPara
         const int64_t f = (int64_t)p.slot0 + p.n - pg * P;
         p.fill_row[pg] = (int32_t)(f < P ? f : P);
     }
+}
+
+__global__ void __launch_bounds__(kAppendThreads) append_kernel(const AppendParams p) {
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+    const int64_t P = p.page_size;
+    append_metadata(p);
     const int D = p.head_dim;
     const int vpr = D >> 3;                 // 16-byte vectors per head row
     const int vpt = p.n_kv_heads * vpr;     // vectors per token row
@@ -240,6 +234,105 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(const AppendPara
 
 // One warp per (layer, K/V, batch row): Hkv*D*2 contiguous source bytes to
 // row `row` of each head's slab of the row's page.
+// Bulk append with the copy engine of each SM (TMA) instead of its threads.
+// A job is (layer, K|V, page, kv head, row chunk): a 4-D tensor copy gathers
+// the job's rows of one kv head from k/v [L][n][Hkv][D] (token stride
+// Hkv*D) into a shared-memory stage, where they already have the page's
+// [rows][D] layout, and one bulk copy writes them to the page.  Lane 0 of
+// the one-warp CTA keeps up to kTmaStagesMax stages in flight; the other lanes only
+// write the metadata.  The SM's ALUs stay free for concurrent work (hashing).
+// kTmaSmemBytes is the largest stage budget (KVG_APPEND_TMA_KB tunes it).
+constexpr int kTmaStagesMax = 8;
+constexpr uint32_t kTmaSmemBytes = 192 * 1024;
+
+struct TmaJob {
+    int32_t lkv, jj, h, row_lo, row_hi;  // rows [row_lo, row_hi) of page jj (launch-relative)
+    int64_t tok;                          // source token (row of k/v) of row_lo
+};
+
+__device__ __forceinline__ TmaJob tma_job(const AppendParams &p, int64_t J, int chunks, int pbox) {
+    TmaJob j;
+    const int c = (int)(J % chunks);
+    J /= chunks;
+    j.h = (int32_t)(J % p.n_kv_heads);
+    J /= p.n_kv_heads;
+    j.jj = (int32_t)(J % p.pids.n);
+    j.lkv = (int32_t)(J / p.pids.n);
+    const int64_t P = p.page_size;
+    const int64_t pg = p.page0 + j.jj;
+    int64_t lo = (int64_t)p.slot0 - pg * P, hi = (int64_t)p.slot0 + p.n - pg * P;
+    if (lo < (int64_t)c * pbox) lo = (int64_t)c * pbox;
+    if (hi > (int64_t)(c + 1) * pbox) hi = (int64_t)(c + 1) * pbox;
+    if (hi > P) hi = P;
+    if (hi < lo) hi = lo;
+    j.row_lo = (int32_t)lo;
+    j.row_hi = (int32_t)hi;
+    j.tok = (int64_t)p.row0 + pg * P + lo - p.slot0;
+    return j;
+}
+
+__global__ void __launch_bounds__(32) append_tma_kernel(const AppendParams p,
+                                                        const __grid_constant__ CUtensorMap kmap,
+                                                        const __grid_constant__ CUtensorMap vmap,
+                                                        DevStatus *status, int32_t pbox, int32_t n_stages,
+                                                        uint64_t limit_ns) {
+    extern __shared__ __align__(128) uint8_t stage_mem[];
+    __shared__ __align__(8) uint64_t bars[kTmaStagesMax];
+    append_metadata(p);
+    if (threadIdx.x != 0) return;
+    const int D = p.head_dim;
+    const int64_t P = p.page_size;
+    const int chunks = (int)((P + pbox - 1) / pbox);
+    const int64_t n_jobs = (int64_t)p.n_layers * 2 * p.pids.n * p.n_kv_heads * chunks;
+    if (blockIdx.x >= n_jobs) return;
+    const int64_t K = (n_jobs - blockIdx.x + gridDim.x - 1) / gridDim.x;  // this CTA's jobs
+    const uint32_t stage_bytes = (uint32_t)pbox * D * 2;
+    for (int i = 0; i < n_stages; ++i) mbar_init(&bars[i], 1);
+    fence_mbar_init();
+    auto job = [&](int64_t k) { return tma_job(p, blockIdx.x + k * gridDim.x, chunks, pbox); };
+    auto load = [&](int64_t k) {
+        const TmaJob j = job(k);
+        const int st = (int)(k % n_stages);
+        if (j.row_hi == j.row_lo) {
+            mbar_arrive(&bars[st]);
+            return;
+        }
+        mbar_arrive_expect_tx(&bars[st], stage_bytes);
+        tma_load_4d(stage_mem + (size_t)st * stage_bytes, (j.lkv & 1) ? &vmap : &kmap, 0, j.h, (int32_t)j.tok,
+                    j.lkv >> 1, &bars[st]);
+    };
+    const int64_t pro = K < n_stages ? K : n_stages;
+    for (int64_t k = 0; k < pro; ++k) load(k);
+    int64_t loaded = pro;  // jobs [0, loaded) have a load issued
+    int64_t k = 0;
+    for (; k < K; ++k) {
+        const int st = (int)(k % n_stages);
+        if (!mbar_wait_bounded(&bars[st], (uint32_t)((k / n_stages) & 1), limit_ns)) {
+            record_error(status, KVG_ERR_DEVICE_CHECK, 2);
+            break;
+        }
+        const TmaJob j = job(k);
+        if (j.row_hi > j.row_lo) {
+            fence_proxy_async_shared();
+            uint8_t *dst = p.pool + ((((uint64_t)j.lkv * p.pool_pages + (uint64_t)p.pids.pid[j.jj]) * p.n_kv_heads +
+                                      j.h) * P + j.row_lo) * (uint64_t)D * 2;
+            bulk_s2g(dst, stage_mem + (size_t)st * stage_bytes, (uint32_t)(j.row_hi - j.row_lo) * D * 2);
+        }
+        bulk_commit();
+        // refill the previous job's stage once its store has read it
+        if (k >= 1 && loaded < K) {
+            bulk_wait_read<1>();
+            load(loaded++);
+        }
+    }
+    if (k < K) {
+        // gave up: let the loads still in flight land before the CTA exits
+        for (int64_t m = k + 1; m < loaded; ++m)
+            mbar_wait_bounded(&bars[m % n_stages], (uint32_t)((m / n_stages) & 1), limit_ns);
+    }
+    bulk_wait<0>();
+}
+
 __global__ void __launch_bounds__(kAppendThreads) append_batch_kernel(const AppendBatchParams p) {
     const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
@@ -377,6 +470,53 @@ cudaError_t launch_append(const AppendParams &p, int n_sm, cudaStream_t s) {
     const int64_t rows = 2ll * p.n_layers * p.n;  // one warp each
     static const int ctas_per_sm = env_knob("KVG_APPEND_CTAS_PER_SM", 2);
     append_kernel<<<grid_for(rows, kAppendThreads / 32, n_sm, ctas_per_sm), kAppendThreads, 0, s>>>(p);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+// Rows per tensor copy: a page's rows, at most 256 (the box limit) and at
+// most 48 KiB of one kv head's rows, so that at least four stages fit.
+int32_t append_tma_rows(int32_t page_size, int32_t head_dim) {
+    int32_t r = page_size < 256 ? page_size : 256;
+    const int32_t cap = 49152 / (2 * head_dim);
+    return r < cap ? r : cap;
+}
+
+cudaError_t launch_append_tma(const AppendParams &p, DevStatus *status, int n_sm, cudaStream_t s) {
+    const int pbox = append_tma_rows(p.page_size, p.head_dim);
+    const int D = p.head_dim;
+    const uint32_t stage_bytes = (uint32_t)pbox * D * 2;
+    // 96 KiB of stages per SM keeps HBM busy (6.5 TB/s alone) while leaving
+    // room beside it for concurrent hashing; 192 KiB starves a concurrent
+    // graft + verify of bandwidth, 64 KiB starves the append.
+    static const uint32_t smem_budget =
+        (uint32_t)std::min(std::max(env_knob("KVG_APPEND_TMA_KB", 96), 16), 192) * 1024u;
+    int n_stages = (int)(smem_budget / stage_bytes);
+    if (n_stages > kTmaStagesMax) n_stages = kTmaStagesMax;
+    if (n_stages < 2) return cudaErrorNotSupported;
+    // k and v: 4-D bf16 tensors (D, Hkv, n_rows_total, L); box (D, 1, pbox, 1)
+    CUtensorMap maps[2];
+    const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)p.n_kv_heads, (cuuint64_t)p.n_rows_total,
+                                (cuuint64_t)p.n_layers};
+    const cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)p.n_kv_heads * D * 2,
+                                   (cuuint64_t)p.n_rows_total * p.n_kv_heads * D * 2};
+    const cuuint32_t box[4] = {(cuuint32_t)D, 1, (cuuint32_t)pbox, 1};
+    const uint16_t *src[2] = {p.k, p.v};
+    for (int i = 0; i < 2; ++i)
+        if (encode_tensor_map(&maps[i], 4, const_cast<uint16_t *>(src[i]), dims, strides, box) != cudaSuccess)
+            return cudaErrorNotSupported;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(append_tma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kTmaSmemBytes);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    const int chunks = (p.page_size + pbox - 1) / pbox;
+    const int64_t jobs = 2ll * p.n_layers * p.pids.n * p.n_kv_heads * chunks;
+    const int grid = grid_for(jobs, 1, n_sm, 1);
+    append_tma_kernel<<<grid, 32, (size_t)n_stages * stage_bytes, s>>>(p, maps[0], maps[1], status, pbox, n_stages,
+                                                                      2000000000ull);
     count_launches(1);
     return cudaGetLastError();
 }

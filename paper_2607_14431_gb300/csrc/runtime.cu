@@ -798,7 +798,12 @@ extern "C" kvg_status kvg_cache_append(kvg_cache *c, int32_t seq, const void *k,
         const int64_t last = (s + nr - 1) / P;
         p.pids.n = (int32_t)(last - p.page0 + 1);
         for (int32_t i = 0; i < p.pids.n; ++i) p.pids.pid[i] = sp[p.page0 + i];
-        KVG_CUDA(launch_append(p, c->n_sm, st));
+        // long appends move rows with tensor copies; short ones (a box would
+        // mostly carry rows that are not stored) with a warp per row
+        cudaError_t e = cudaErrorNotSupported;
+        if (nr >= append_tma_rows(p.page_size, p.head_dim)) e = launch_append_tma(p, c->status, c->n_sm, st);
+        if (e == cudaErrorNotSupported) e = launch_append(p, c->n_sm, st);
+        KVG_CUDA(e);
     }
     c->n_slots[seq] = (int32_t)(s0 + n);
     return KVG_OK;
@@ -1166,6 +1171,11 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
         }
     }
     const int32_t *bpos = reinterpret_cast<const int32_t *>(blk.dev + blk.lay.pos_off);
+    // A verified own-position graft reads each page once: the copy and the
+    // leaf hashes are one kernel, and only the page digests follow.
+    const bool fused = (flags & KVG_GRAFT_VERIFY) && delta == 0;
+    const int64_t m = (int64_t)((c->page_bytes + kLeafBytes - 1) / kLeafBytes);
+    if (fused) KVG_CUDA(c->leaf.ensure((size_t)c->dims.n_layers * 2 * npb * m * 32));
     for (int64_t base = 0; base < npb; base += kMaxPagesPerLaunch) {
         p.npb = (int32_t)std::min<int64_t>(kMaxPagesPerLaunch, npb - base);
         p.page_base = (int32_t)base;
@@ -1175,10 +1185,16 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
         p.fill_row = c->page_fill + (int64_t)seq * c->max_pages + jdst + base;
         p.pids.n = p.npb;
         for (int32_t i = 0; i < p.npb; ++i) p.pids.pid[i] = pids[base + i];
-        KVG_CUDA(launch_graft_copy(p, c->n_sm, st));
+        if (fused)
+            KVG_CUDA(launch_graft_verify(p, static_cast<uint32_t *>(c->leaf.ptr), c->n_sm, st));
+        else
+            KVG_CUDA(launch_graft_copy(p, c->n_sm, st));
     }
-    if (flags & KVG_GRAFT_VERIFY) {
-        kvg_status r = enqueue_verify(s, blk, c, seq, jdst, delta != 0, st);
+    if (fused) {
+        KVG_CUDA(launch_sha256_pages(static_cast<const uint32_t *>(c->leaf.ptr), (int64_t)c->dims.n_layers * 2 * npb, m,
+                                     nullptr, blk.dev + blk.lay.dig_off, c->status, seq, st));
+    } else if (flags & KVG_GRAFT_VERIFY) {
+        kvg_status r = enqueue_verify(s, blk, c, seq, jdst, true, st);
         if (r != KVG_OK) return r;
     }
     return finish_verify(c, seq, flags, (flags & KVG_GRAFT_VERIFY) ? (int32_t)(c->dims.n_layers * 2 * npb) : 0,

@@ -122,6 +122,73 @@ __device__ __forceinline__ const uint8_t *page_addr(const PageSource &s, int64_t
     return s.base + ((uint64_t)plane * s.plane_pages + (uint64_t)s.pid[j]) * s.page_bytes;
 }
 
+// SHA-256 of one leaf of `len` bytes (16-byte aligned).  With COPY the leaf
+// is also written to `copy_to`, from the same registers that are hashed, so
+// the bytes written are exactly the bytes whose digest is checked.
+template <bool COPY>
+__device__ __forceinline__ void hash_leaf(const uint8_t *leaf, uint64_t len, uint8_t *copy_to, uint32_t st[8],
+                                          uint32_t one) {
+    const uint4 *v = reinterpret_cast<const uint4 *>(leaf);
+    uint4 *o = reinterpret_cast<uint4 *>(copy_to);
+    init_state(st);
+    const int nfull = (int)(len >> 6);
+    // The next two 64-byte blocks are in flight while the current one is
+    // compressed, so their memory latency (long when other kernels keep HBM
+    // busy) hides behind ~3.4k ALU ops.
+    uint4 n1[4], n2[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        if (nfull > 0) n1[q] = __ldg(v + q);
+        if (nfull > 1) n2[q] = __ldg(v + 4 + q);
+    }
+    for (int blk = 0; blk < nfull; ++blk) {
+        uint32_t w[16];
+        uint4 x[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            x[q] = n1[q];
+            n1[q] = n2[q];
+        }
+        if (blk + 2 < nfull) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) n2[q] = __ldg(v + 4 * (blk + 2) + q);
+        }
+        if (COPY) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) __stcs(o + 4 * blk + q, x[q]);
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            w[4 * q + 0] = bswap(x[q].x);
+            w[4 * q + 1] = bswap(x[q].y);
+            w[4 * q + 2] = bswap(x[q].z);
+            w[4 * q + 3] = bswap(x[q].w);
+        }
+        compress(st, w, one);
+    }
+    const int rem = (int)(len & 63);
+    if (rem == 0) {
+        uint32_t w[16];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) w[q] = 0;
+        w[0] = 0x80000000u;
+        const uint64_t bits = len * 8ull;
+        w[14] = (uint32_t)(bits >> 32);
+        w[15] = (uint32_t)bits;
+        compress(st, w, one);
+    } else {
+        if (COPY)
+            for (int q = 0; q < rem / 16; ++q) o[4 * nfull + q] = v[4 * nfull + q];
+        finish(st, leaf + (len & ~63ull), rem, len, one);
+    }
+}
+
+__device__ __forceinline__ void store_state(uint32_t *out, const uint32_t st[8]) {
+    uint4 *o = reinterpret_cast<uint4 *>(out);
+    o[0] = make_uint4(st[0], st[1], st[2], st[3]);
+    o[1] = make_uint4(st[4], st[5], st[6], st[7]);
+}
+
 __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src, int64_t n_pages,
                                                             int64_t leaves_per_page,
                                                             uint32_t *__restrict__ out, uint32_t one) {
@@ -132,39 +199,35 @@ __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src
         const int64_t i = idx - p * leaves_per_page;
         uint64_t len = src.page_bytes - (uint64_t)i * kLeafBytes;
         if (len > kLeafBytes) len = kLeafBytes;
-        const uint8_t *leaf = page_addr(src, p) + (uint64_t)i * kLeafBytes;
-        const uint4 *v = reinterpret_cast<const uint4 *>(leaf);
         uint32_t st[8];
-        init_state(st);
-        const int nfull = (int)(len >> 6);
-        for (int blk = 0; blk < nfull; ++blk) {
-            uint32_t w[16];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint4 x = __ldg(v + 4 * blk + q);
-                w[4 * q + 0] = bswap(x.x);
-                w[4 * q + 1] = bswap(x.y);
-                w[4 * q + 2] = bswap(x.z);
-                w[4 * q + 3] = bswap(x.w);
-            }
-            compress(st, w, one);
-        }
-        const int rem = (int)(len & 63);
-        if (rem == 0) {
-            uint32_t w[16];
-#pragma unroll
-            for (int q = 0; q < 16; ++q) w[q] = 0;
-            w[0] = 0x80000000u;
-            const uint64_t bits = len * 8ull;
-            w[14] = (uint32_t)(bits >> 32);
-            w[15] = (uint32_t)bits;
-            compress(st, w, one);
-        } else {
-            finish(st, leaf + (len & ~63ull), rem, len, one);
-        }
-        uint4 *o = reinterpret_cast<uint4 *>(out + idx * 8);
-        o[0] = make_uint4(st[0], st[1], st[2], st[3]);
-        o[1] = make_uint4(st[4], st[5], st[6], st[7]);
+        hash_leaf<false>(page_addr(src, p) + (uint64_t)i * kLeafBytes, len, nullptr, st, one);
+        store_state(out + idx * 8, st);
+    }
+}
+
+// Own-position graft with the verification folded into the copy: one thread
+// per 4 KiB leaf reads it from the block once, writes it to its cache page and
+// hashes it (leaf order of a page digest, Sec. 3.2's integrity check).
+__global__ void __launch_bounds__(128) graft_verify_kernel(const GraftParams p, int64_t leaves_per_page,
+                                                           uint32_t *__restrict__ out, uint32_t one) {
+    graft_metadata(p);
+    const uint64_t page_bytes = p.page_bytes;
+    const int64_t n_leaves = (int64_t)p.n_layers * 2 * p.npb * leaves_per_page;
+    for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < n_leaves;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t page_u = idx / leaves_per_page;
+        const int64_t i = idx - page_u * leaves_per_page;
+        const int64_t lkv = page_u / p.npb;
+        const int64_t jj = page_u - lkv * p.npb;
+        const uint64_t off = (uint64_t)i * kLeafBytes;
+        uint64_t len = page_bytes - off;
+        if (len > kLeafBytes) len = kLeafBytes;
+        const int64_t block_page = lkv * p.block_pages + p.page_base + jj;
+        const uint8_t *src = p.src + (uint64_t)block_page * page_bytes + off;
+        uint8_t *dst = p.pool + ((uint64_t)lkv * p.pool_pages + (uint64_t)p.pids.pid[jj]) * page_bytes + off;
+        uint32_t st[8];
+        hash_leaf<true>(src, len, dst, st, one);
+        store_state(out + (block_page * leaves_per_page + i) * 8, st);
     }
 }
 
@@ -316,10 +379,23 @@ cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_
     const int64_t n = n_pages * m;
     if (n == 0) return cudaSuccess;
     int64_t grid = (n + 127) / 128;
-    static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 4);
+    static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 8);
     const int64_t cap = (int64_t)n_sm * ctas_per_sm;
     if (grid > cap) grid = cap;
     sha256_leaves_kernel<<<(int)grid, 128, 0, s>>>(src, n_pages, m, leaf_words, 1u);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int n_sm, cudaStream_t s) {
+    const int64_t m = (int64_t)((p.page_bytes + kLeafBytes - 1) / kLeafBytes);
+    const int64_t n = (int64_t)p.n_layers * 2 * p.npb * m;
+    if (n == 0) return cudaSuccess;
+    int64_t grid = (n + 127) / 128;
+    static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 8);
+    const int64_t cap = (int64_t)n_sm * ctas_per_sm;
+    if (grid > cap) grid = cap;
+    graft_verify_kernel<<<(int)grid, 128, 0, s>>>(p, m, leaf_words, 1u);
     count_launches(1);
     return cudaGetLastError();
 }

@@ -305,6 +305,49 @@ def test_verify_detects_a_flipped_byte(oracle):
     kvg.kvg_sync(s["dst"].h)
 
 
+@pytest.mark.parametrize("hkv,P", [(3, 7), (1, 33), (4, 64)], ids=["2688B_page", "4224B_page", "64KiB_page"])
+def test_fused_verified_graft(oracle, hkv, P):
+    """A verified own-position graft copies and hashes in one pass.  Pages of
+    2,688 B (one short leaf), 4,224 B (a full and a short leaf) and 64 KiB: the
+    restored cache equals the oracle's and the unverified copy's byte for byte;
+    a flipped byte in a short leaf is reported on exactly its page, and the
+    pass still restores the bytes it read."""
+    kvg = need_gpu()
+    w = syn.Workload("odd", 2, 2 * hkv, hkv, 64, P, 10000.0, 0x61 + P)
+    nb = 5 * P + 3
+    s = _build_both(kvg, oracle, w, nb, 0, seed=P, copies=3)
+    rep = kvg.kvg_graft_report()
+    kvg.kvg_graft(s["store"].h, s["bid"], s["dst"].h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC,
+                  report=rep)
+    assert rep.n_mismatch == 0 and rep.n_pages_checked == w.n_layers * 2 * s["oblk"].n_pages
+    kvg.kvg_graft(s["store"].h, s["bid"], s["dst"].h, 1, -1, 0, kvg.KVG_GRAFT_SYNC)
+    s["ocache"].graft(0, s["oblk"])
+    s["ocache"].graft(1, s["oblk"])
+    assert np.array_equal(pool_u16(s["dst"], w), s["ocache"].pool)
+    pt, pf, ps = tables(s["dst"])
+    assert np.array_equal(pt, s["ocache"].page_table) and np.array_equal(ps, s["ocache"].positions)
+    # corrupt the last byte of the last leaf of (layer 1, K, page 4)
+    blob = bytearray(kvg.kvg_store_export(s["store"].h, s["bid"]))
+    info = kvg.kvg_store_block_info(s["store"].h, s["bid"])
+    page_bytes = hkv * P * w.head_dim * 2
+    bad_page = (1 * 2 + 0) * info.n_pages + 4
+    at = info.pages_offset + bad_page * page_bytes + page_bytes - 1
+    blob[at] ^= 0x01
+    bid2 = kvg.kvg_store_import(s["store"].h, bytes(blob), 0)
+    rep2 = kvg.kvg_graft_report()
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_graft(s["store"].h, bid2, s["dst"].h, 2, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC,
+                      report=rep2)
+    assert e.value.status == kvg.KVG_ERR_DIGEST
+    assert rep2.n_mismatch == 1 and rep2.mismatch_pages[0] == bad_page and rep2.seq == 2
+    pool = pool_u16(s["dst"], w)
+    pt, _, _ = tables(s["dst"])
+    pid = int(pt[2, 4])
+    got = pool[1, 0, pid].tobytes()
+    want = bytes(blob[at - page_bytes + 1: at + 1])
+    assert got == want
+
+
 def test_host_checks_reject_bad_calls(oracle):
     kvg = need_gpu()
     w = geometry("tiny")
@@ -338,6 +381,44 @@ def test_host_checks_reject_bad_calls(oracle):
     with pytest.raises(E) as e:
         kvg.kvg_cache_set_free_order(s["src"].h, list(range(s["n_pages"])))  # pages in use
     assert e.value.status == kvg.KVG_ERR_ARG
+
+
+@pytest.mark.parametrize("geo", ["tiny", "g4", "d256"])
+def test_append_sizes_and_offsets(oracle, geo):
+    """Appends of 1, P-1, P, P+1 and 3P+5 rows at ragged slot offsets (rows
+    shorter than a page go through the warp-per-row kernel, longer ones
+    through the tensor-copy kernel), and one long append into a second
+    sequence: pool bytes, page tables, fills and positions equal the
+    oracle's."""
+    kvg = need_gpu()
+    w = geometry(geo)
+    P = w.page_size
+    sizes = [1, P - 1, P, P + 1, 3 * P + 5, 2]
+    total = sum(sizes)
+    k, v = _kv(w, total + 5 * P + 3, 71)
+    max_slots = _slots(w, total + 5 * P + 3)
+    n_pages = 2 * (max_slots // P) + 4
+    dims = dims_for(kvg, w)
+    c = kvg.Cache(dims, n_pages, 2, max_slots)
+    fill_canary(c)
+    kvg.kvg_cache_set_free_order(c.h, syn.permutation(n_pages, 72))
+    oc = oracle.OracleCache(oracle_dims(oracle, w), n_pages, 2, max_slots, fill=CANARY)
+    oc.set_free_order(syn.permutation(n_pages, 72))
+    t = 0
+    for n in sizes:
+        pos = syn.positions(t, n)
+        append(kvg, c, 0, k[:, t:t + n], v[:, t:t + n], pos)
+        oc.append(0, k[:, t:t + n], v[:, t:t + n], pos)
+        t += n
+    n = 5 * P + 3
+    pos = syn.positions(1000, n)
+    append(kvg, c, 1, k[:, t:t + n], v[:, t:t + n], pos)
+    oc.append(1, k[:, t:t + n], v[:, t:t + n], pos)
+    assert np.array_equal(pool_u16(c, w), oc.pool)
+    pt, pf, ps = tables(c)
+    assert np.array_equal(pt, oc.page_table) and np.array_equal(pf, oc.page_fill)
+    assert np.array_equal(ps, oc.positions)
+    kvg.kvg_sync(c.h)
 
 
 def test_append_batch_matches_oracle(oracle):
