@@ -129,7 +129,8 @@ class Clocks:
 class Step12B:
     """Device state and the per-step call sequence for the 12B workload."""
 
-    def __init__(self, kvg, device, stream, side, n_layers=None, pool_store=False, schedule="overlap"):
+    def __init__(self, kvg, device, stream, side, n_layers=None, pool_store=False, schedule="overlap",
+                 swa=None):
         self.kvg = kvg
         self.w = w = syn.B12 if not n_layers else syn.B12.with_layers(n_layers)
         self.dev = device
@@ -163,12 +164,20 @@ class Step12B:
         self.scale = 1.0 / math.sqrt(w.head_dim)
         blk_pages = w.n_layers * 2 * (self.nb // P) * w.page_bytes
         self.pool_store = pool_store
+        # swa = (W, R): sliding-window layers over the full-size cache, every
+        # R-th layer global and the others attending to their last W rows
+        self.swa = swa
+        self.windows = [0] * w.n_layers
+        if swa:
+            W, R = swa
+            self.windows = [0 if (l + 1) % R == 0 else W for l in range(w.n_layers)]
+            kvg.kvg_cache_set_layer_windows(self.cache.h, self.windows)
+        rows_read = sum(min(x, syn.B12_CTX) if x else syn.B12_CTX for x in self.windows)
         self.bytes = {
             "graft": 0 if pool_store else 2 * blk_pages,
             "verify": blk_pages,
             "append": 2 * w.n_layers * 2 * self.nf * w.n_kv_heads * w.head_dim * 2,
-            "decode": w.n_layers * 2 * syn.B12_CTX * w.n_kv_heads * w.head_dim * 2
-                      + 2 * self.q.numel() * 2,
+            "decode": rows_read * 2 * w.n_kv_heads * w.head_dim * 2 + 2 * self.q.numel() * 2,
         }
         self.sha_blocks = (blk_pages // 4096) * 65
         self.blk_pages = blk_pages
@@ -256,7 +265,9 @@ def run_kvg(args, rank, world):
     stream = torch.cuda.Stream(device)
     side = torch.cuda.Stream(device)
     hbm_peak, sm_max, peak_kind = load_peaks()
-    st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool", schedule=args.schedule)
+    swa = tuple(int(x) for x in args.swa.split(":")) if args.swa else None
+    st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool", schedule=args.schedule,
+                 swa=swa)
 
     # correctness of the configuration being timed: one verified step
     st.run_step()
@@ -383,7 +394,9 @@ def run_kvg(args, rank, world):
         "config": {"workload": f"12b-single-graft: L{st.w.n_layers} Hq16/Hkv8 D256 P64, 8192-token block grafted "
                                "at own positions (digest-verified) + 24576 fresh tokens, decode 1 token over 32768"
                                + (" [block in the cache pool: zero-copy graft]" if st.pool_store else "")
-                               + (" [verified graft in one pass, beside the append]" if st.schedule == "fused" else ""),
+                               + (" [verified graft in one pass, beside the append]" if st.schedule == "fused" else "")
+                               + (f" [sliding-window layers: window {st.swa[0]}, every {st.swa[1]}th layer global]"
+                                  if st.swa else ""),
                    "global_batch": world, "seq_len": syn.B12_CTX, "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)"},
         "parts": parts, "roofline": roof, "e2e": e2e, "gpu_launches": int(launches),
@@ -800,6 +813,8 @@ def main():
     ap.add_argument("--schedule", default="fused", choices=["overlap", "fused"],
                     help="12b step: digest check on a side stream after the graft (overlap) or folded "
                          "into the graft, which runs beside the append (fused)")
+    ap.add_argument("--swa", default="", help="12b step with sliding-window layers, 'W:R' (window W, every "
+                                              "R-th layer global), over the full-size cache")
     ap.add_argument("--store", default="hbm", choices=["hbm", "pool"],
                     help="12b: block in an HBM store (copying graft) or in the cache pool (zero-copy graft)")
     ap.add_argument("--deep-blocks", type=int, default=syn.DEEP_BLOCKS)
@@ -822,7 +837,7 @@ def main():
         torch.distributed.init_process_group("nccl")
     line = run_kvg(args, rank, world)
     if rank == 0:
-        if not args.no_cpu_baseline:
+        if not args.no_cpu_baseline and not args.swa:
             line["cpu_baseline"] = cpu_baseline(args.cpu_baseline_layers)
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -193,6 +193,22 @@ void kvg_cache_destroy(kvg_cache *cache);
  * changes any result: attention reduces in logical token order. */
 kvg_status kvg_cache_set_free_order(kvg_cache *cache, const int32_t *order, int32_t n_pages);
 
+/* Sliding-window layers over a full-size cache (Sec. 4.3: a sliding-window
+ * model resumes exactly from a restored block once its windowed layers keep
+ * full-size KV).  Every layer keeps every row, so deposits and grafts stay
+ * byte-exact; decode attention on layer l reads only the last windows[l]
+ * valid rows of each sequence (counted back over its pages' fills, so the
+ * window spans an unfilled tail of a page left by a page-aligned graft), or
+ * every row when windows[l] == 0.  With consecutive position tags over the
+ * valid rows, as after an own-position graft followed by appends, this is the
+ * usual window over positions (query position q sees keys q-W+1 .. q, its
+ * own row appended before the decode).
+ * windows: host array of n_layers values >= 0; n == 0 (windows ignored)
+ * resets every layer to 0.  Takes effect for later decode calls; changes no
+ * cache contents.  Errors: KVG_ERR_ARG (n not 0 or n_layers, a negative
+ * window). */
+kvg_status kvg_cache_set_layer_windows(kvg_cache *cache, const int32_t *windows, int32_t n);
+
 /* Device-side layout, for inspection and for interop with other kernels. */
 typedef struct kvg_cache_view {
     void *pool;            /* bf16 [L][2][n_pages][Hkv][P][D] */
@@ -299,8 +315,10 @@ kvg_status kvg_verify(kvg_store *store, uint64_t block_id, kvg_cache *cache, int
  * g = h / (n_q_heads / n_kv_heads):
  *     o[h] = sum_t softmax_t(scale * q[h] . k_t[g]) v_t[g]
  * over every valid row of the sequence (pages in logical order, rows below
- * their fill), accumulated in fp32 and rounded to bf16 (RNE).  An empty
- * sequence gives o = 0.
+ * their fill) — on a windowed layer (kvg_cache_set_layer_windows) over its
+ * last W valid rows — accumulated in fp32 and rounded to bf16 (RNE).  An
+ * empty sequence gives o = 0.  Layers with different windows run as separate
+ * launches on the stream.
  * q, out: device bf16 [n_layers_run][B][n_q_heads][head_dim] where
  * layer >= 0 runs that layer only (n_layers_run = 1) and layer == -1 runs all
  * layers in one launch.  The reduction order depends only on the logical
@@ -324,7 +342,8 @@ kvg_status kvg_decode_attention(kvg_cache *cache, int32_t layer, const int32_t *
  * (no cudaMalloc, cudaFree or library allocator).  Arguments, results and
  * errors are those of kvg_decode_attention, with these differences:
  *   - the partials take (units + workers) * G * (4 * head_dim + 8) bytes,
- *     units = n_layers_run * min(B, 256) * n_kv_heads, G = n_q_heads /
+ *     units = (layers of one launch: those sharing a window, at most 256)
+ *     * min(B, 256) * n_kv_heads, G = n_q_heads /
  *     n_kv_heads; the number of decode workers (warps) is capped so they fit
  *     in 16 MiB - 256 bytes, and a call that does not fit even with one
  *     worker returns KVG_ERR_CAPACITY with an explanatory kvg_last_error()

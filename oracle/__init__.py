@@ -405,6 +405,7 @@ class OracleCache:
         self.page_fill = np.zeros((max_seqs, self.max_pages), np.int32)
         self.positions = np.full((max_seqs, max_slots), -1, np.int32)
         self.n_slots = np.zeros(max_seqs, np.int32)
+        self.windows = [0] * d.L  # per layer: 0 = global attention, W > 0 = last W valid rows
 
     def set_free_order(self, order):
         if len(self.free) != self.n_pages:
@@ -567,7 +568,20 @@ class OracleCache:
         return (np.ascontiguousarray(np.concatenate(ks)), np.ascontiguousarray(np.concatenate(vs)),
                 np.concatenate(ps))
 
+    def set_layer_windows(self, windows):
+        """Per-layer sliding windows (0 = global) over the full-size cache
+        (Sec. 4.3: windowed layers keep full-size KV so a restored block
+        resumes exactly); [] resets every layer to global."""
+        w = [int(x) for x in windows] or [0] * self.dims.L
+        if len(w) != self.dims.L or min(w) < 0:
+            raise KvgError("need one window >= 0 per layer")
+        self.windows = w
+
     def decode(self, seq: int, layer: int, q: np.ndarray, scale: float) -> np.ndarray:
-        """fp64 decode attention of q[Hq][D] over the sequence's valid rows."""
+        """fp64 decode attention of q[Hq][D] over the sequence's valid rows,
+        or over the last W of them when the layer has a window W > 0."""
         k, v, _ = self.logical_kv(seq, layer)
+        W = self.windows[layer]
+        if W > 0:
+            k, v = k[-W:], v[-W:]
         return gqa_decode(q, k, v, scale)

@@ -12,7 +12,8 @@
 // bounded wait) of the K and V rows as boxes of 64 columns x TOK rows with the
 // 128-byte swizzle, so the 8-row ldmatrix reads below hit 8 different bank
 // groups; value rows past the page's fill are zeroed after arrival and the
-// scores of those rows are masked.
+// scores of those rows are masked; on a sliding-window layer the unit starts
+// at the window's first tile and the rows before the window are masked too.
 //
 // The contractions run on the tensor cores with mma.sync m16n8k16 (bf16 in,
 // fp32 accumulate).  Each tile is bandwidth-bound (~2 flop per byte at G = 2),
@@ -63,7 +64,7 @@ struct Cfg {
     static constexpr int BOX = TOK * 128;              // bytes of one box (TOK rows x 128 B)
     static constexpr int STAGE_BYTES = 2 * NB * BOX;   // K boxes then V boxes
     static constexpr int RING_BYTES = STAGES * STAGE_BYTES;
-    static constexpr int SMEM = RING_BYTES + STAGES * (8 + 4) + 1024;  // + alignment slack
+    static constexpr int SMEM = RING_BYTES + STAGES * (8 + 4 + 4) + 1024;  // + alignment slack
     static constexpr int KS = D / 16;                  // k-steps of q.k, m-tiles of p.v
     static constexpr int SUB = TOK / 16;               // 16-row sub-tiles per tile
     static_assert(BOX % 1024 == 0, "a swizzle atom is 8 rows of 128 bytes");
@@ -149,7 +150,8 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
 
     uint8_t *ring = smem;
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::RING_BYTES);
-    int *vrs = reinterpret_cast<int *>(smem + C::RING_BYTES + STAGES * 8);
+    int *vrs = reinterpret_cast<int *>(smem + C::RING_BYTES + STAGES * 8);  // valid rows [los, vrs) per stage
+    int *los = vrs + STAGES;
     if (lane == 0) {
 #pragma unroll
         for (int s = 0; s < STAGES; ++s) mbar_init(&bars[s], 1);
@@ -164,6 +166,7 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
     struct Cursor {
         int64_t t, end;  // next tile to issue; first tile past its unit
         int lr, b, g, seq, jj, k;
+        int lo;          // rows before the window start in the next tile (its unit's first only)
     } cur;
     cur.t = t0;
     cur.end = t0;
@@ -173,17 +176,20 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
         cur.b = tp.b;
         cur.g = tp.g;
         cur.seq = p.rows.seq[tp.b];
-        cur.jj = tp.tile / tpp;
-        cur.k = tp.tile - cur.jj * tpp;
+        const int tile = tp.tile + p.rows.tile0[tp.b];
+        cur.jj = tile / tpp;
+        cur.k = tile - cur.jj * tpp;
+        cur.lo = tp.tile == 0 ? p.rows.lo[tp.b] : 0;
         cur.end = cur.t - tp.tile + (p.rows.pref_tiles[tp.b + 1] - p.rows.pref_tiles[tp.b]);
     };
 
     // lane 0: arm the stage's barrier and copy the next tile's K and V boxes
     auto issue = [&](int stg) {
         if (cur.t >= cur.end) advance_to_unit();
-        const int seq = cur.seq, jj = cur.jj, k = cur.k;
+        const int seq = cur.seq, jj = cur.jj, k = cur.k, lo = cur.lo;
         struct { int lr, g; } tp{cur.lr, cur.g};
         ++cur.t;
+        cur.lo = 0;
         if (++cur.k == tpp) {
             cur.k = 0;
             ++cur.jj;
@@ -192,15 +198,17 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
         const int pid = p.page_table[(int64_t)seq * p.max_pages + jj];
         int vr = fill - k * TOK;
         vr = vr < 0 ? 0 : (vr > TOK ? TOK : vr);
+        if (lo >= vr) vr = 0;
         if (vr > 0 && (pid < 0 || pid >= p.pool_pages)) {
             record_error(p.status, KVG_ERR_DEVICE_CHECK, 1);
             vr = 0;
         }
         vrs[stg] = vr;
+        los[stg] = lo;
         uint64_t *bar = &bars[stg];
         if (vr > 0) {
             mbar_arrive_expect_tx(bar, (uint32_t)C::STAGE_BYTES);
-            const int l = p.layer0 + tp.lr;
+            const int l = p.layers[tp.lr];
             const int32_t row_k = (int32_t)((2 * l) * plane_rows + ((int64_t)pid * p.n_kv_heads + tp.g) * P +
                                             (int64_t)k * TOK);
             const int32_t row_v = (int32_t)(row_k + plane_rows);
@@ -248,7 +256,7 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
 
     auto begin = [&](const TilePos &tp) {
         const __nv_bfloat16 *qrow =
-            p.q + ((int64_t)(tp.lr * p.q_row_stride_b + p.b0 + tp.b) * p.n_q_heads + tp.g * G) * D;
+            p.q + ((int64_t)(p.qlayers[tp.lr] * p.q_row_stride_b + p.b0 + tp.b) * p.n_q_heads + tp.g * G) * D;
 #pragma unroll
         for (int ks = 0; ks < KS; ++ks) {
             if (gq < G) {
@@ -288,16 +296,19 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
             alive = false;
             break;
         }
-        const int vr = vrs[stg];
+        const int vr = vrs[stg], lo = los[stg];
         bool zeroed = false;
-        if (vr > 0 && vr < TOK) {
-            // value rows past the fill hold whatever the pool had there: zero
-            // them so their zero weights contribute exactly 0
+        if (vr > 0 && (vr < TOK || lo > 0)) {
+            // value rows past the fill hold whatever the pool had there, and
+            // rows before a window's start are outside the attention: zero
+            // both so their zero weights contribute exactly 0
             uint4 *vz = reinterpret_cast<uint4 *>(ring + stg * C::STAGE_BYTES + NB * BOX);
-            for (int idx = lane; idx < NB * (TOK - vr) * 8; idx += 32) {
-                const int b = idx / ((TOK - vr) * 8);
-                const int rem = idx - b * (TOK - vr) * 8;
-                vz[(b * BOX + (vr + rem / 8) * 128) / 16 + (rem & 7)] = make_uint4(0, 0, 0, 0);
+            const int n_out = TOK - vr + lo;  // rows [0, lo) and [vr, TOK)
+            for (int idx = lane; idx < NB * n_out * 8; idx += 32) {
+                const int b = idx / (n_out * 8);
+                const int rem = idx - b * n_out * 8;
+                const int r = rem / 8 < lo ? rem / 8 : vr + (rem / 8 - lo);
+                vz[(b * BOX + r * 128) / 16 + (rem & 7)] = make_uint4(0, 0, 0, 0);
             }
             fence_proxy_async_shared();
             zeroed = true;
@@ -326,10 +337,11 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
                         mma_bf16(acc0, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
                 }
                 const int r0 = 16 * sb + gq, r1 = r0 + 8;
-                sc[sb][0] = r0 < vr ? (acc0[0] + acc1[0]) * p.qscale : -INFINITY;
-                sc[sb][1] = r0 < vr ? (acc0[1] + acc1[1]) * p.qscale : -INFINITY;
-                sc[sb][2] = r1 < vr ? (acc0[2] + acc1[2]) * p.qscale : -INFINITY;
-                sc[sb][3] = r1 < vr ? (acc0[3] + acc1[3]) * p.qscale : -INFINITY;
+                const bool in0 = r0 >= lo && r0 < vr, in1 = r1 >= lo && r1 < vr;
+                sc[sb][0] = in0 ? (acc0[0] + acc1[0]) * p.qscale : -INFINITY;
+                sc[sb][1] = in0 ? (acc0[1] + acc1[1]) * p.qscale : -INFINITY;
+                sc[sb][2] = in1 ? (acc0[2] + acc1[2]) * p.qscale : -INFINITY;
+                sc[sb][3] = in1 ? (acc0[3] + acc1[3]) * p.qscale : -INFINITY;
             }
             // ---- online softmax for heads 2*tq (e = 0) and 2*tq+1 (e = 1)
             float mt_[2] = {-INFINITY, -INFINITY};
@@ -437,7 +449,8 @@ __global__ void __launch_bounds__(D) combine_kernel(const DecodeParams p) {
         }
     }
     const float r = L > 0.f ? __fdiv_rn(O, L) : 0.f;
-    p.out[((int64_t)(lr * p.q_row_stride_b + p.b0 + b) * p.n_q_heads + h) * D + d] = __float2bfloat16_rn(r);
+    p.out[((int64_t)(p.qlayers[lr] * p.q_row_stride_b + p.b0 + b) * p.n_q_heads + h) * D + d] =
+        __float2bfloat16_rn(r);
 }
 
 template <int D, int G>

@@ -16,6 +16,7 @@ namespace kvg {
 // ---------------------------------------------------------------- limits --
 constexpr int kMaxPagesPerLaunch = 1024;  // page ids carried in kernel params
 constexpr int kMaxBatchPerLaunch = 256;   // decode rows carried in kernel params
+constexpr int kMaxLayersPerLaunch = 256;  // decode layers carried in kernel params
 constexpr int kMaxHalfDim = 128;          // head_dim <= 256
 constexpr uint64_t kLeafBytes = KVG_DIGEST_LEAF_BYTES;
 
@@ -170,7 +171,8 @@ struct PageSource {
 // touches, at slot unit + w (unique because both ranges are contiguous).
 struct BatchRows {
     int32_t seq[kMaxBatchPerLaunch];
-    int32_t npages[kMaxBatchPerLaunch];
+    int32_t tile0[kMaxBatchPerLaunch];  // first tile of the row's pages that is read (window start)
+    int32_t lo[kMaxBatchPerLaunch];     // rows of that first tile before the window start
     int32_t pref_tiles[kMaxBatchPerLaunch + 1];  // prefix sums of T_b
 };
 
@@ -178,7 +180,9 @@ struct DecodeParams {
     const uint8_t *pool;
     int64_t pool_pages;
     int32_t n_kv_heads, page_size, n_q_heads;
-    int32_t layer0, n_layers_run, B;
+    int32_t n_layers_run, B;
+    int16_t layers[kMaxLayersPerLaunch];   // run layer lr -> cache layer
+    int16_t qlayers[kMaxLayersPerLaunch];  // run layer lr -> layer index of q and out
     int32_t n_warps;           // W
     int64_t n_tiles;           // T
     const int32_t *page_table;

@@ -16,6 +16,7 @@
 #include <cstdlib>
 #include <mutex>
 #include <string>
+#include <vector>
 
 #include "common.cuh"
 
@@ -47,8 +48,8 @@ struct CacheShape {
 };
 bool cache_shape(const kvg_cache *c, CacheShape *out);
 int32_t cache_seq_pages(const kvg_cache *c, int32_t seq);
-int64_t cache_fill_rows(const kvg_cache *c, const int32_t *seq_ids, int64_t b0, int32_t nb, int tpp, int Lrun,
-                        BatchRows *rows);
+kvg_status cache_plan_decode(const kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
+                             std::vector<DecodeParams> *plan, int64_t *max_units);
 void set_last_error(const char *msg);
 }  // namespace kvg
 
@@ -77,23 +78,24 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
     if (cs.device < 0 || cs.device >= kMaxDevices) return reject(KVG_ERR_ARG, "device ordinal out of range");
     for (int32_t b = 0; b < B; ++b)
         if (seq_ids[b] < 0 || seq_ids[b] >= cs.max_seqs) return reject(KVG_ERR_ARG, "bad seq id");
-    const int Lrun = layer < 0 ? cs.n_layers : 1;
-    const int64_t bchunk = B < kMaxBatchPerLaunch ? B : kMaxBatchPerLaunch;
+    // the launches (as kvg_decode_attention makes them); host memory only
+    std::vector<DecodeParams> plan;
+    int64_t units = 0;
+    const kvg_status pst = cache_plan_decode(c, layer, seq_ids, B, &plan, &units);
+    if (pst != KVG_OK) return pst;
     // partials: (units + workers) slots of G * (4 * head_dim + 8) bytes; the
     // (m, l) part starts 256-byte aligned after o, so keep 256 bytes of slack
     const uint64_t per_slot = (uint64_t)G * ((uint64_t)cs.head_dim * 4 + 8);
     const int64_t cap_slots = (int64_t)((kScratchBytes - 256) / per_slot);
-    const int64_t units = (int64_t)Lrun * bchunk * cs.n_kv_heads;
     if (cap_slots - units < 1) {
         char m[320];
         snprintf(m, sizeof m,
-                 "noalloc decode: %d layer(s) x %lld batch rows x %d kv heads need at least %llu bytes of "
-                 "partials, above the %zu-byte static scratch; use kvg_decode_attention or fewer rows per call",
-                 Lrun, (long long)bchunk, cs.n_kv_heads, (unsigned long long)((units + 1) * per_slot),
-                 kScratchBytes);
+                 "noalloc decode: %lld units (layers x batch rows x kv heads of one launch) need at least %llu "
+                 "bytes of partials, above the %zu-byte static scratch; use kvg_decode_attention or fewer rows "
+                 "per call",
+                 (long long)units, (unsigned long long)((units + 1) * per_slot), kScratchBytes);
         return reject(KVG_ERR_CAPACITY, m);
     }
-    const int tpp = (cs.page_size + decode_tile_tokens(cs.head_dim) - 1) / decode_tile_tokens(cs.head_dim);
 
     int prev = -1;
     cudaGetDevice(&prev);
@@ -127,30 +129,15 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
     float2 *part_ml = reinterpret_cast<float2 *>(static_cast<unsigned char *>(scratch) +
                                                  ((slots * G * cs.head_dim * 4 + 255) / 256) * 256);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    for (int64_t b0 = 0; b0 < B; b0 += kMaxBatchPerLaunch) {
-        const int32_t nb = (int32_t)((B - b0) < kMaxBatchPerLaunch ? (B - b0) : kMaxBatchPerLaunch);
-        DecodeParams p{};
-        p.n_tiles = cache_fill_rows(c, seq_ids, b0, nb, tpp, Lrun, &p.rows);
+    for (DecodeParams &p : plan) {
         p.n_warps = (int32_t)(p.n_tiles < w_cap ? (p.n_tiles > 1 ? p.n_tiles : 1) : w_cap);
-        p.pool = cs.pool;
-        p.pool_pages = cs.n_pages;
-        p.n_kv_heads = cs.n_kv_heads;
-        p.page_size = cs.page_size;
         p.n_q_heads = n_q_heads;
-        p.layer0 = layer < 0 ? 0 : layer;
-        p.n_layers_run = Lrun;
-        p.B = nb;
-        p.page_table = cs.page_table;
-        p.page_fill = cs.page_fill;
-        p.max_pages = cs.max_pages;
         p.q = static_cast<const __nv_bfloat16 *>(q);
         p.q_row_stride_b = B;
-        p.b0 = (int32_t)b0;
         p.qscale = scale * 1.4426950408889634f;
         p.part_o = part_o;
         p.part_ml = part_ml;
         p.out = static_cast<__nv_bfloat16 *>(out);
-        p.status = cs.status;
         cudaError_t e = launch_decode(cs.head_dim, G, p, *cs.pool_map, st);
         if (e != cudaSuccess) return reject(KVG_ERR_CUDA, std::string("decode launch: ") + cudaGetErrorString(e));
         e = launch_combine(cs.head_dim, G, p, st);

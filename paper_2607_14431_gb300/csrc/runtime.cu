@@ -496,7 +496,9 @@ struct kvg_cache {
     DevStatus *status = nullptr;
     std::deque<int32_t> free_list;
     std::vector<std::vector<int32_t>> seq_pages;
+    std::vector<std::vector<int32_t>> seq_fill;  // host copy of page_fill for each sequence's pages
     std::vector<int32_t> n_slots;
+    std::vector<int32_t> layer_window;  // per layer: 0 = global attention, W > 0 = last W tokens
     Scratch leaf, part_o, part_ml;
     CUtensorMap pool_map;  // decode kernel's 2-D view of the pool
     std::vector<uint8_t> pinned;  // per page: owned by a pool-resident store block
@@ -686,6 +688,8 @@ extern "C" kvg_status kvg_cache_create(const kvg_dims *dims, int32_t n_pages, in
     c->alias.assign(n_pages, 0);
     c->seq_pages.assign(max_seqs, {});
     c->n_slots.assign(max_seqs, 0);
+    c->seq_fill.resize(max_seqs);
+    c->layer_window.assign(dims->n_layers, 0);
     if (cudaDeviceSynchronize() != cudaSuccess) return cleanup(fail(KVG_ERR_CUDA, "init sync failed"));
     *out = c;
     return KVG_OK;
@@ -752,6 +756,15 @@ static std::vector<int32_t> take_pages(kvg_cache *c, int64_t n) {
     return v;
 }
 
+// Mirrors on the host the fill counts the kernels write for the pages that
+// hold slots [slot_begin, slot_end) of `seq` (rows below the fill are valid).
+static void note_fills(kvg_cache *c, int32_t seq, int64_t slot_begin, int64_t slot_end) {
+    const int64_t P = c->dims.page_size;
+    auto &f = c->seq_fill[seq];
+    f.resize(c->seq_pages[seq].size(), 0);
+    for (int64_t pg = slot_begin / P; pg * P < slot_end; ++pg) f[pg] = (int32_t)std::min<int64_t>(P, slot_end - pg * P);
+}
+
 extern "C" kvg_status kvg_cache_append(kvg_cache *c, int32_t seq, const void *k, const void *v,
                                        const int32_t *positions, int32_t n, void *stream) {
     Trace trace_("kvg_cache_append");
@@ -806,6 +819,7 @@ extern "C" kvg_status kvg_cache_append(kvg_cache *c, int32_t seq, const void *k,
         KVG_CUDA(e);
     }
     c->n_slots[seq] = (int32_t)(s0 + n);
+    note_fills(c, seq, s0, s0 + n);
     return KVG_OK;
 }
 
@@ -857,6 +871,7 @@ extern "C" kvg_status kvg_cache_append_batch(kvg_cache *c, const int32_t *seq_id
         p.pid[b] = sp[s / P];
         p.slot[b] = (int32_t)s;
         c->n_slots[sq] = (int32_t)(s + 1);
+        note_fills(c, sq, s, s + 1);
     }
     KVG_CUDA(launch_append_batch(p, c->n_sm, static_cast<cudaStream_t>(stream)));
     return KVG_OK;
@@ -874,6 +889,7 @@ extern "C" kvg_status kvg_cache_release(kvg_cache *c, int32_t seq, void *stream)
             c->free_list.push_back(pid);
     }
     c->seq_pages[seq].clear();
+    c->seq_fill[seq].clear();
     c->n_slots[seq] = 0;
     KVG_CUDA(launch_reset_seq(c->page_table + (int64_t)seq * c->max_pages,
                               c->page_fill + (int64_t)seq * c->max_pages, c->max_pages,
@@ -1078,6 +1094,7 @@ static kvg_status pool_graft(kvg_store *s, const kvg_store::Blk &blk, kvg_cache 
     const int64_t jdst = dst / P;
     sp.insert(sp.end(), pages.begin(), pages.end());
     c->n_slots[seq] = (int32_t)(dst + n);
+    note_fills(c, seq, dst, dst + n);
     if (partial) {
         GatherParams p{};
         p.pool = c->pool;
@@ -1144,6 +1161,7 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
     const int64_t jdst = dst / P;
     sp.insert(sp.end(), pids.begin(), pids.end());
     c->n_slots[seq] = (int32_t)(dst + n);
+    note_fills(c, seq, dst, dst + n);
 
     GraftParams p{};
     p.src = blk.dev + blk.lay.pages_off;
@@ -1225,21 +1243,103 @@ extern "C" kvg_status kvg_verify(kvg_store *s, uint64_t block_id, kvg_cache *c, 
 
 // ------------------------------------------------------------------ decode --
 
-// Fills the per-launch batch rows (sequence, pages, prefix sums of tiles) for
-// rows [b0, b0 + nb) and returns the launch's tile count.
-static int64_t fill_rows(const kvg_cache *c, const int32_t *seq_ids, int64_t b0, int32_t nb, int tpp,
-                         int Lrun, BatchRows *rows) {
-    int32_t acc = 0;
-    for (int32_t i = 0; i < nb; ++i) {
-        const int32_t sq = seq_ids[b0 + i];
-        const int32_t np = (int32_t)c->seq_pages[sq].size();
-        rows->seq[i] = sq;
-        rows->npages[i] = np;
-        rows->pref_tiles[i] = acc;
-        acc += np * tpp;
+// First row read by a windowed layer: the last `window` valid rows of the
+// sequence, counted back over its pages' fills (a page's valid rows are
+// [0, fill)).  Returns the page index and the row within it.
+static void window_start(const kvg_cache *c, int32_t seq, int64_t window, int32_t *page, int32_t *row) {
+    const auto &f = c->seq_fill[seq];
+    int64_t acc = 0;
+    for (int64_t j = (int64_t)f.size() - 1; j >= 0; --j) {
+        if (acc + f[j] >= window) {
+            *page = (int32_t)j;
+            *row = (int32_t)(f[j] - (window - acc));
+            return;
+        }
+        acc += f[j];
     }
-    rows->pref_tiles[nb] = acc;
-    return (int64_t)Lrun * c->dims.n_kv_heads * acc;
+    *page = 0;
+    *row = 0;
+}
+
+// The launches of one decode call: the layers run are grouped by their
+// window (one group when no layer is windowed), each group split into
+// launches of at most kMaxLayersPerLaunch layers and kMaxBatchPerLaunch rows.
+// Fills every field but the per-call ones (q, out, scale, heads, scratch,
+// workers); *max_units gets the largest layers x rows x kv heads of a launch.
+static kvg_status plan_decode(const kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
+                              std::vector<DecodeParams> *plan, int64_t *max_units) {
+    const kvg_dims &d = c->dims;
+    const int TOK = decode_tile_tokens(d.head_dim);
+    const int tpp = (d.page_size + TOK - 1) / TOK;
+    // (window, [(cache layer, q layer)]) in order of first appearance
+    std::vector<std::pair<int32_t, std::vector<std::pair<int32_t, int32_t>>>> groups;
+    for (int32_t l = layer < 0 ? 0 : layer; l < (layer < 0 ? d.n_layers : layer + 1); ++l) {
+        const int32_t w = c->layer_window[l];
+        auto it = std::find_if(groups.begin(), groups.end(), [w](const auto &g) { return g.first == w; });
+        if (it == groups.end()) {
+            groups.push_back({w, {}});
+            it = groups.end() - 1;
+        }
+        it->second.push_back({l, layer < 0 ? l : 0});
+    }
+    plan->clear();
+    *max_units = 0;
+    for (const auto &grp : groups) {
+        const int64_t W = grp.first;
+        for (size_t l0 = 0; l0 < grp.second.size(); l0 += kMaxLayersPerLaunch) {
+            const int32_t nl = (int32_t)std::min<size_t>(kMaxLayersPerLaunch, grp.second.size() - l0);
+            for (int64_t b0 = 0; b0 < B; b0 += kMaxBatchPerLaunch) {
+                const int32_t nb = (int32_t)std::min<int64_t>(kMaxBatchPerLaunch, B - b0);
+                plan->emplace_back();
+                DecodeParams &p = plan->back();
+                memset(&p, 0, sizeof p);
+                int32_t acc = 0;
+                for (int32_t i = 0; i < nb; ++i) {
+                    const int32_t sq = seq_ids[b0 + i];
+                    const int32_t np = (int32_t)c->seq_pages[sq].size();
+                    int32_t pg = 0, row = 0;
+                    if (W > 0) window_start(c, sq, W, &pg, &row);
+                    p.rows.seq[i] = sq;
+                    p.rows.tile0[i] = pg * tpp + row / TOK;
+                    p.rows.lo[i] = row % TOK;
+                    p.rows.pref_tiles[i] = acc;
+                    acc += np * tpp - p.rows.tile0[i];
+                }
+                p.rows.pref_tiles[nb] = acc;
+                for (int32_t i = 0; i < nl; ++i) {
+                    p.layers[i] = (int16_t)grp.second[l0 + i].first;
+                    p.qlayers[i] = (int16_t)grp.second[l0 + i].second;
+                }
+                p.n_layers_run = nl;
+                p.n_tiles = (int64_t)nl * d.n_kv_heads * acc;
+                p.B = nb;
+                p.b0 = (int32_t)b0;
+                p.pool = c->pool;
+                p.pool_pages = c->n_pages;
+                p.n_kv_heads = d.n_kv_heads;
+                p.page_size = d.page_size;
+                p.page_table = c->page_table;
+                p.page_fill = c->page_fill;
+                p.max_pages = c->max_pages;
+                p.status = c->status;
+                *max_units = std::max<int64_t>(*max_units, (int64_t)nl * nb * d.n_kv_heads);
+            }
+        }
+    }
+    return KVG_OK;
+}
+
+extern "C" kvg_status kvg_cache_set_layer_windows(kvg_cache *c, const int32_t *windows, int32_t n) {
+    if (!c) return fail(KVG_ERR_ARG, "null cache");
+    if (n == 0) {
+        std::fill(c->layer_window.begin(), c->layer_window.end(), 0);
+        return KVG_OK;
+    }
+    if (!windows || n != c->dims.n_layers) return fail(KVG_ERR_ARG, "need one window per layer (%d)", c->dims.n_layers);
+    for (int32_t l = 0; l < n; ++l)
+        if (windows[l] < 0) return fail(KVG_ERR_ARG, "negative window for layer %d", l);
+    c->layer_window.assign(windows, windows + n);
+    return KVG_OK;
 }
 
 extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
@@ -1259,38 +1359,24 @@ extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const in
         if (seq_ids[b] < 0 || seq_ids[b] >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq id %d", seq_ids[b]);
     DeviceGuard g(c->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const int Lrun = layer < 0 ? d.n_layers : 1;
-    const int tpp = (d.page_size + decode_tile_tokens(d.head_dim) - 1) / decode_tile_tokens(d.head_dim);
     const int w_max = decode_max_warps(d.head_dim, G, c->n_sm);
     if (w_max <= 0) return fail(KVG_ERR_CUDA, "decode kernel cannot be made resident");
-    const int64_t bchunk = std::min<int64_t>(B, kMaxBatchPerLaunch);
-    const size_t slots = (size_t)Lrun * bchunk * d.n_kv_heads + (size_t)w_max;
+    std::vector<DecodeParams> plan;
+    int64_t max_units = 0;
+    kvg_status r = plan_decode(c, layer, seq_ids, B, &plan, &max_units);
+    if (r != KVG_OK) return r;
+    const size_t slots = (size_t)max_units + (size_t)w_max;
     KVG_CUDA(c->part_o.ensure(slots * G * d.head_dim * sizeof(float)));
     KVG_CUDA(c->part_ml.ensure(slots * G * sizeof(float2)));
-    for (int64_t b0 = 0; b0 < B; b0 += kMaxBatchPerLaunch) {
-        const int32_t nb = (int32_t)std::min<int64_t>(kMaxBatchPerLaunch, B - b0);
-        DecodeParams p{};
-        p.n_tiles = fill_rows(c, seq_ids, b0, nb, tpp, Lrun, &p.rows);
+    for (DecodeParams &p : plan) {
         p.n_warps = (int32_t)std::min<int64_t>(w_max, std::max<int64_t>(p.n_tiles, 1));
-        p.pool = c->pool;
-        p.pool_pages = c->n_pages;
-        p.n_kv_heads = d.n_kv_heads;
-        p.page_size = d.page_size;
         p.n_q_heads = n_q_heads;
-        p.layer0 = layer < 0 ? 0 : layer;
-        p.n_layers_run = Lrun;
-        p.B = nb;
-        p.page_table = c->page_table;
-        p.page_fill = c->page_fill;
-        p.max_pages = c->max_pages;
         p.q = static_cast<const __nv_bfloat16 *>(q);
         p.q_row_stride_b = B;
-        p.b0 = (int32_t)b0;
         p.qscale = scale * 1.4426950408889634f;
         p.part_o = static_cast<float *>(c->part_o.ptr);
         p.part_ml = static_cast<float2 *>(c->part_ml.ptr);
         p.out = static_cast<__nv_bfloat16 *>(out);
-        p.status = c->status;
         KVG_CUDA(launch_decode(d.head_dim, G, p, c->pool_map, st));
         KVG_CUDA(launch_combine(d.head_dim, G, p, st));
     }
@@ -1400,9 +1486,9 @@ bool cache_shape(const kvg_cache *c, CacheShape *out) {
     return true;
 }
 int32_t cache_seq_pages(const kvg_cache *c, int32_t seq) { return (int32_t)c->seq_pages[seq].size(); }
-int64_t cache_fill_rows(const kvg_cache *c, const int32_t *seq_ids, int64_t b0, int32_t nb, int tpp, int Lrun,
-                        BatchRows *rows) {
-    return fill_rows(c, seq_ids, b0, nb, tpp, Lrun, rows);
+kvg_status cache_plan_decode(const kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
+                             std::vector<DecodeParams> *plan, int64_t *max_units) {
+    return plan_decode(c, layer, seq_ids, B, plan, max_units);
 }
 void set_last_error(const char *msg) { g_last_error = msg; }
 }  // namespace kvg

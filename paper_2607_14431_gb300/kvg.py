@@ -77,6 +77,7 @@ _SIGNATURES = {
     "kvg_cache_create": ([_P(kvg_dims), _i32, _i32, _i32, _i32, _P(_vp)], _i32),
     "kvg_cache_destroy": ([_vp], None),
     "kvg_cache_set_free_order": ([_vp, _vp, _i32], _i32),
+    "kvg_cache_set_layer_windows": ([_vp, _vp, _i32], _i32),
     "kvg_cache_view_get": ([_vp, _P(kvg_cache_view)], _i32),
     "kvg_cache_seq_info": ([_vp, _i32, _P(_i32), _P(_i32)], _i32),
     "kvg_cache_append": ([_vp, _i32, _vp, _vp, _vp, _i32, _vp], _i32),
@@ -199,6 +200,12 @@ def kvg_cache_destroy(cache):
 def kvg_cache_set_free_order(cache, order):
     arr = (ctypes.c_int32 * len(order))(*[int(x) for x in order])
     _check(lib().kvg_cache_set_free_order(cache, arr, len(order)))
+
+
+def kvg_cache_set_layer_windows(cache, windows):
+    """windows: one int per layer (0 = global attention), or [] to reset."""
+    arr = (ctypes.c_int32 * max(len(windows), 1))(*[int(x) for x in windows])
+    _check(lib().kvg_cache_set_layer_windows(cache, arr, len(windows)))
 
 
 def kvg_cache_view_get(cache) -> kvg_cache_view:

@@ -152,6 +152,93 @@ def test_decode_matches_oracle_and_grafted_equals_fresh(oracle, geo, nb, nf):
         compare_decode(oracle, ol[0, 0], oracle.gqa_decode(q[l, 0], s["k"][l], s["v"][l], scale))
 
 
+def _windows(w):
+    P = w.page_size
+    return [(1, P + 3, 0, 2 * P + 5)[l % 4] for l in range(w.n_layers)]
+
+
+@pytest.mark.parametrize("geo", ["tiny", "d128", "d256", "g4"])
+def test_windowed_decode_matches_oracle(oracle, geo):
+    """Sliding-window layers over a full-size cache: per-layer windows 1,
+    P+3, 0 (global), 2P+5.  Seq 0 holds a ragged grafted block, fresh rows on
+    its last page, a second block grafted at the next page boundary (leaving
+    unfilled rows the window must skip) and more fresh rows; seq 1 one long
+    fresh write; seq 2 three rows.  All layers in one call and one layer at a
+    time match the fp64 oracle; a window of one returns the last value row bit
+    for bit; a grafted sequence equals the same rows written fresh, bit for
+    bit, under the windows."""
+    kvg = need_gpu()
+    w = geometry(geo)
+    P = w.page_size
+    dims = dims_for(kvg, w)
+    od = oracle_dims(oracle, w)
+    na, nb_, nc, nd = 2 * P + 5, P + 2, P + 7, 3
+    k, v = _kv(w, na + nb_ + nc + nd + 5 * P, 81)
+    parts, t = [], 0
+    for n in (na, nb_, nc, nd):
+        parts.append((k[:, t:t + n], v[:, t:t + n], syn.positions(t, n)))
+        t += n
+    n_long = 5 * P
+    k_long, v_long = k[:, t:t + n_long], v[:, t:t + n_long]
+    max_slots = 8 * P + 64
+    n_pages = 64
+    # the two blocks, deposited from a source cache
+    src = kvg.Cache(dims, n_pages, 2, max_slots)
+    store = kvg.Store(dims, 0, HBM_CAP)
+    bids = []
+    for i, (kk, vv, pp) in enumerate((parts[0], parts[2])):
+        append(kvg, src, i, kk, vv, pp)
+        bids.append(kvg.kvg_deposit(store.h, src.h, i, 0, pp.size))
+    c = kvg.Cache(dims, n_pages, 5, max_slots)
+    fill_canary(c)
+    kvg.kvg_cache_set_free_order(c.h, syn.permutation(n_pages, 82))
+    oc = oracle.OracleCache(od, n_pages, 5, max_slots, fill=CANARY)
+    oc.set_free_order(syn.permutation(n_pages, 82))
+    kvg.kvg_graft(store.h, bids[0], c.h, 0, -1, 0, kvg.KVG_GRAFT_SYNC)
+    oc.graft(0, oracle.block_from_kv(od, *parts[0]))
+    append(kvg, c, 0, *parts[1])
+    oc.append(0, *parts[1])
+    kvg.kvg_graft(store.h, bids[1], c.h, 0, -1, 0, kvg.KVG_GRAFT_SYNC)
+    oc.graft(0, oracle.block_from_kv(od, *parts[2]))
+    append(kvg, c, 0, *parts[3])
+    oc.append(0, *parts[3])
+    append(kvg, c, 1, k_long, v_long, syn.positions(0, n_long))
+    oc.append(1, k_long, v_long, syn.positions(0, n_long))
+    append(kvg, c, 2, k[:, :3], v[:, :3], syn.positions(0, 3))
+    oc.append(2, k[:, :3], v[:, :3], syn.positions(0, 3))
+    # grafted (seq 3) and fresh (seq 4) copies of block A + fresh rows
+    kvg.kvg_graft(store.h, bids[0], c.h, 3, -1, 0, kvg.KVG_GRAFT_SYNC)
+    append(kvg, c, 3, *parts[1])
+    append(kvg, c, 4, np.concatenate([parts[0][0], parts[1][0]], 1), np.concatenate([parts[0][1], parts[1][1]], 1),
+           syn.positions(0, na + nb_))
+    wins = _windows(w)
+    kvg.kvg_cache_set_layer_windows(c.h, wins)
+    oc.set_layer_windows(wins)
+    scale = 1.0 / math.sqrt(w.head_dim)
+    rows = [0, 1, 2]
+    q = syn.as_u16(syn.queries(w, w.n_layers, len(rows), 83))
+    o = decode(kvg, c, w, rows, q)
+    G = w.group
+    for l in range(w.n_layers):
+        for b, sq in enumerate(rows):
+            compare_decode(oracle, o[l, b], oc.decode(sq, l, q[l, b], scale))
+            ol = decode(kvg, c, w, [sq], q[l:l + 1, b:b + 1], layer=l)
+            compare_decode(oracle, ol[0, 0], oc.decode(sq, l, q[l, b], scale))
+        if wins[l] == 1:
+            kk, vv, _ = oc.logical_kv(0, l)
+            for h in range(w.n_q_heads):
+                assert np.array_equal(o[l, 0, h], vv[-1, h // G])
+    q2 = syn.as_u16(syn.queries(w, w.n_layers, 1, 84))
+    assert _sha(decode(kvg, c, w, [3], q2)) == _sha(decode(kvg, c, w, [4], q2))
+    # the windows only select rows: resetting them gives global attention again
+    kvg.kvg_cache_set_layer_windows(c.h, [])
+    og = decode(kvg, c, w, [0], q[:, :1])
+    for l in range(w.n_layers):
+        kk, vv, _ = oc.logical_kv(0, l)
+        compare_decode(oracle, og[l, 0], oracle.gqa_decode(q[l, 0], kk, vv, scale))
+    kvg.kvg_sync(c.h)
+
+
 def test_decode_closed_forms(oracle):
     kvg = need_gpu()
     w = geometry("d128")

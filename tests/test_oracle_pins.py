@@ -467,3 +467,64 @@ def test_pinned_block_graft_aliases_pages(oracle):
     assert np.array_equal(c.pool[:, :, 5], pb.block.pages[:, :, 2])  # the block's own page untouched
     c.release(1)
     assert 3 not in c.free and 6 in c.free
+
+
+# --------------------------------------------------------------------------
+# Sliding-window layers over a full-size cache (Sec. 4.3)
+# --------------------------------------------------------------------------
+
+def _stitched(oracle, seed):
+    """Seq 0: a ragged 37-row block grafted, then 20 fresh rows appended on
+    its partly filled last page, then a 21-row block grafted at the next page
+    boundary (a hole of unfilled rows before it), then 5 fresh rows.
+    Returns the cache and the rows written, in order, per layer."""
+    d = _dims()
+    c = oracle.OracleCache(d, 40, 2, 256, fill=CANARY)
+    c.set_free_order(syn.permutation(40, seed))
+    ka, va = _kv(37, seed)
+    kb, vb = _kv(20, seed + 1)
+    kc, vc = _kv(21, seed + 2)
+    kd, vd = _kv(5, seed + 3)
+    c.graft(0, oracle.block_from_kv(d, ka, va, syn.positions(0, 37)))
+    c.append(0, kb, vb, syn.positions(37, 20))
+    c.graft(0, oracle.block_from_kv(d, kc, vc, syn.positions(57, 21)))
+    c.append(0, kd, vd, syn.positions(78, 5))
+    k = np.concatenate([ka, kb, kc, kd], axis=1)
+    v = np.concatenate([va, vb, vc, vd], axis=1)
+    return c, k, v
+
+
+@pytest.mark.parametrize("W", [1, 5, 16, 17, 40, 83, 500])
+def test_window_attends_to_the_last_w_rows_written(oracle, W):
+    c, k, v = _stitched(oracle, 21)
+    q = syn.as_u16(syn.queries(syn.TINY, 2, 1, 22))[:, 0]
+    c.set_layer_windows([W, 0])
+    n = k.shape[1]  # 83 rows written; the hole is not among them
+    assert n == 83
+    got = c.decode(0, 0, q[0], 0.125)
+    want = oracle.gqa_decode(q[0], k[0, -W:], v[0, -W:], 0.125)
+    assert got.tobytes() == want.tobytes()
+    # the other layer stays global
+    assert c.decode(0, 1, q[1], 0.125).tobytes() == oracle.gqa_decode(q[1], k[1], v[1], 0.125).tobytes()
+    if W >= n:
+        c.set_layer_windows([])
+        assert c.decode(0, 0, q[0], 0.125).tobytes() == got.tobytes()
+
+
+def test_window_of_one_returns_the_last_value_row(oracle):
+    c, k, v = _stitched(oracle, 23)
+    c.set_layer_windows([1, 1])
+    q = syn.as_u16(syn.queries(syn.TINY, 2, 1, 24))[:, 0]
+    for l in range(2):
+        o = c.decode(0, l, q[l], 0.125)
+        G = q.shape[1] // v.shape[2]
+        for h in range(q.shape[1]):
+            assert np.array_equal(o[h], oracle.bf16_to_f64(v[l, -1, h // G]))
+
+
+def test_window_settings_are_checked(oracle):
+    c, _, _ = _stitched(oracle, 25)
+    with pytest.raises(oracle.KvgError):
+        c.set_layer_windows([1])
+    with pytest.raises(oracle.KvgError):
+        c.set_layer_windows([-1, 0])

@@ -30,14 +30,17 @@ def _decode_both(kvg, cache, w, seq_ids, q):
     return u16(a), u16(b)
 
 
-@pytest.mark.parametrize("geo,lens", [("tiny", [256]), ("d256", [700, 1300, 65]), ("g4", [333, 1])])
-def test_noalloc_matches_decode_attention_twice(oracle, geo, lens):
+@pytest.mark.parametrize("geo,lens,windowed", [("tiny", [256], False), ("d256", [700, 1300, 65], False),
+                                               ("g4", [333, 1], False), ("d256", [700, 1300, 65], True)])
+def test_noalloc_matches_decode_attention_twice(oracle, geo, lens, windowed):
     kvg = need_gpu()
     w = geometry(geo)
     dims = dims_for(kvg, w)
     P = w.page_size
     max_slots = (max(lens) // P + 2) * P
     cache = kvg.Cache(dims, sum(n // P + 1 for n in lens) + 2, len(lens), max_slots)
+    if windowed:  # sliding-window layers: the same launch plan for both entry points
+        kvg.kvg_cache_set_layer_windows(cache.h, [P + 3] + [0] * (w.n_layers - 1))
     for i, n in enumerate(lens):
         k, v = syn.kv_rows(w, n, 70 + i)
         append(kvg, cache, i, syn.as_u16(k), syn.as_u16(v), syn.positions(0, n))
