@@ -161,6 +161,10 @@ struct PageSource {
     const int32_t *pid;
     int32_t npb;
     int64_t plane_pages;
+    // with pid: leaf digests of page (plane, j) go to page slot
+    // plane * out_plane_stride + out_j0 + j of the output (0: plane * npb + j)
+    int64_t out_plane_stride = 0;
+    int32_t out_j0 = 0;
 };
 
 // --------------------------------------------------------------- decode --

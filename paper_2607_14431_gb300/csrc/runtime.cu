@@ -486,6 +486,8 @@ extern "C" kvg_status kvg_store_load(kvg_store *s, const char *path, uint32_t fl
 
 // ------------------------------------------------------------------- cache --
 
+constexpr int kHostVerifyChunks = 8;  // page-range chunks of a verified host-store graft
+
 struct kvg_cache {
     kvg_dims dims;
     int32_t n_pages = 0, max_seqs = 0, max_slots = 0, max_pages = 0;
@@ -501,6 +503,10 @@ struct kvg_cache {
     std::vector<int32_t> layer_window;  // per layer: 0 = global attention, W > 0 = last W tokens
     Scratch leaf, part_o, part_ml;
     CUtensorMap pool_map;  // decode kernel's 2-D view of the pool
+    // library stream and events for hashing a host-store graft's pages while
+    // the next pages still cross the host link (made on first use)
+    cudaStream_t aux = nullptr;
+    cudaEvent_t aux_ev[kHostVerifyChunks + 1] = {};
     std::vector<uint8_t> pinned;  // per page: owned by a pool-resident store block
     std::vector<int32_t> alias;   // per pinned page: sequences whose page tables point at it
 };
@@ -699,6 +705,9 @@ extern "C" void kvg_cache_destroy(kvg_cache *c) {
     if (!c) return;
     DeviceGuard g(c->device);
     cudaDeviceSynchronize();
+    for (cudaEvent_t &e : c->aux_ev)
+        if (e) cudaEventDestroy(e);
+    if (c->aux) cudaStreamDestroy(c->aux);
     if (c->pool) cudaFree(c->pool);
     if (c->page_table) cudaFree(c->page_table);
     if (c->page_fill) cudaFree(c->page_fill);
@@ -1189,13 +1198,28 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
         }
     }
     const int32_t *bpos = reinterpret_cast<const int32_t *>(blk.dev + blk.lay.pos_off);
-    // A verified own-position graft reads each page once: the copy and the
-    // leaf hashes are one kernel, and only the page digests follow.
-    const bool fused = (flags & KVG_GRAFT_VERIFY) && delta == 0;
+    // A verified own-position graft from an HBM store reads each page once:
+    // the copy and the leaf hashes are one kernel, and only the page digests
+    // follow.  From a pinned-host store the copy instead moves page-range
+    // chunks with the copy kernel (whose wide reads keep the host link at its
+    // limit) and a library stream hashes each chunk's restored pages in HBM
+    // while the next chunk crosses the link.
+    const bool verify0 = (flags & KVG_GRAFT_VERIFY) && delta == 0;
+    const bool piped = verify0 && s->residency == KVG_RESIDENCY_PINNED_HOST;
+    const bool fused = verify0 && !piped;
     const int64_t m = (int64_t)((c->page_bytes + kLeafBytes - 1) / kLeafBytes);
-    if (fused) KVG_CUDA(c->leaf.ensure((size_t)c->dims.n_layers * 2 * npb * m * 32));
-    for (int64_t base = 0; base < npb; base += kMaxPagesPerLaunch) {
-        p.npb = (int32_t)std::min<int64_t>(kMaxPagesPerLaunch, npb - base);
+    if (verify0) KVG_CUDA(c->leaf.ensure((size_t)c->dims.n_layers * 2 * npb * m * 32));
+    int64_t step = kMaxPagesPerLaunch;
+    if (piped) {
+        if (!c->aux) {
+            KVG_CUDA(cudaStreamCreateWithFlags(&c->aux, cudaStreamNonBlocking));
+            for (cudaEvent_t &e : c->aux_ev) KVG_CUDA(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+        }
+        step = std::min<int64_t>(step, (npb + kHostVerifyChunks - 1) / kHostVerifyChunks);
+    }
+    int chunk = 0;
+    for (int64_t base = 0; base < npb; base += step, ++chunk) {
+        p.npb = (int32_t)std::min<int64_t>(step, npb - base);
         p.page_base = (int32_t)base;
         p.src_pos = bpos + base * P;
         p.dst_pos = c->positions + (int64_t)seq * c->max_slots + dst + base * P;
@@ -1207,8 +1231,25 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
             KVG_CUDA(launch_graft_verify(p, static_cast<uint32_t *>(c->leaf.ptr), c->n_sm, st));
         else
             KVG_CUDA(launch_graft_copy(p, c->n_sm, st));
+        if (piped) {
+            // (more than kHostVerifyChunks chunks only past 8 x 1,024 pages per
+            // plane; an event is re-recorded after its wait is enqueued)
+            cudaEvent_t ev = c->aux_ev[chunk % kHostVerifyChunks];
+            KVG_CUDA(cudaEventRecord(ev, st));
+            KVG_CUDA(cudaStreamWaitEvent(c->aux, ev, 0));
+            PageSource src{c->pool, c->page_bytes, c->page_table + (int64_t)seq * c->max_pages + jdst + base, p.npb,
+                           (int64_t)c->n_pages};
+            src.out_plane_stride = npb;
+            src.out_j0 = (int32_t)base;
+            KVG_CUDA(launch_sha256_leaves(src, (int64_t)c->dims.n_layers * 2 * p.npb,
+                                          static_cast<uint32_t *>(c->leaf.ptr), c->n_sm, c->aux));
+        }
     }
-    if (fused) {
+    if (piped) {
+        KVG_CUDA(cudaEventRecord(c->aux_ev[kHostVerifyChunks], c->aux));
+        KVG_CUDA(cudaStreamWaitEvent(st, c->aux_ev[kHostVerifyChunks], 0));
+    }
+    if (verify0) {
         KVG_CUDA(launch_sha256_pages(static_cast<const uint32_t *>(c->leaf.ptr), (int64_t)c->dims.n_layers * 2 * npb, m,
                                      nullptr, blk.dev + blk.lay.dig_off, c->status, seq, st));
     } else if (flags & KVG_GRAFT_VERIFY) {

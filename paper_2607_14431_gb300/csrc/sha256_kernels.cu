@@ -201,7 +201,12 @@ __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src
         if (len > kLeafBytes) len = kLeafBytes;
         uint32_t st[8];
         hash_leaf<false>(page_addr(src, p) + (uint64_t)i * kLeafBytes, len, nullptr, st, one);
-        store_state(out + idx * 8, st);
+        int64_t po = p;
+        if (src.pid && src.out_plane_stride) {
+            const int64_t plane = p / src.npb;
+            po = plane * src.out_plane_stride + src.out_j0 + (p - plane * src.npb);
+        }
+        store_state(out + (po * leaves_per_page + i) * 8, st);
     }
 }
 

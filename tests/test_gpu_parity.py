@@ -435,6 +435,42 @@ def test_fused_verified_graft(oracle, hkv, P):
     assert got == want
 
 
+@pytest.mark.parametrize("geo,nb,bad", [("tiny", 250, (3, 15)), ("d128", 1000, (4, 0)), ("d128", 1000, (5, 9))])
+def test_host_store_verified_graft_reports_the_bad_page(oracle, geo, nb, bad):
+    """A verified graft from a pinned-host store copies page-range chunks and
+    hashes each chunk's restored pages on a second stream: a flipped byte in
+    page (plane, j) is reported as that block page, whichever chunk holds it,
+    and an intact block grafts clean."""
+    kvg = need_gpu()
+    w = geometry(geo)
+    s = _build_both(kvg, oracle, w, nb, 0, seed=61, copies=3)
+    host = kvg.Store(s["dims"], kvg.KVG_RESIDENCY_PINNED_HOST, 1 << 30)
+    blob = bytearray(kvg.kvg_store_export(s["store"].h, s["bid"]))
+    hid = kvg.kvg_store_import(host.h, bytes(blob), kvg.KVG_GRAFT_VERIFY)
+    rep = kvg.kvg_graft_report()
+    kvg.kvg_graft(host.h, hid, s["dst"].h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, report=rep)
+    assert rep.n_mismatch == 0
+    info = kvg.kvg_store_block_info(s["store"].h, s["bid"])
+    page_bytes = w.n_kv_heads * w.page_size * w.head_dim * 2
+    plane, j = bad
+    bad_page = plane * info.n_pages + j
+    blob[info.pages_offset + bad_page * page_bytes + 7] ^= 0x40
+    hid2 = kvg.kvg_store_import(host.h, bytes(blob), 0)
+    rep2 = kvg.kvg_graft_report()
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_graft(host.h, hid2, s["dst"].h, 1, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, report=rep2)
+    assert e.value.status == kvg.KVG_ERR_DIGEST
+    assert rep2.n_mismatch == 1 and rep2.mismatch_pages[0] == bad_page
+    # the intact graft restored the oracle's bytes
+    s["ocache"].graft(0, s["oblk"])
+    pool = pool_u16(s["dst"], w)
+    pt, _, _ = tables(s["dst"])
+    for jj in range(info.n_pages):
+        pid = int(pt[0, jj])
+        assert np.array_equal(pool[:, :, pid], s["ocache"].pool[:, :, int(s["ocache"].page_table[0, jj])])
+    kvg.kvg_sync(s["dst"].h)
+
+
 def test_host_checks_reject_bad_calls(oracle):
     kvg = need_gpu()
     w = geometry("tiny")
