@@ -130,7 +130,7 @@ class Step12B:
     """Device state and the per-step call sequence for the 12B workload."""
 
     def __init__(self, kvg, device, stream, side, n_layers=None, pool_store=False, schedule="overlap",
-                 swa=None):
+                 swa=None, kv="bf16"):
         self.kvg = kvg
         self.w = w = syn.B12 if not n_layers else syn.B12.with_layers(n_layers)
         self.dev = device
@@ -140,7 +140,14 @@ class Step12B:
         self.ev_verify = torch.cuda.Event()
         self.nb, self.nf = syn.B12_BLOCK, syn.B12_CTX - syn.B12_BLOCK
         P = w.page_size
-        self.dims = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0)
+        # kv "e4m3": the cache (and so the block) holds fp8 E4M3 codes with
+        # per-tensor scales; appends quantize the bf16 rows
+        self.kv = kv
+        fp8 = kv == "e4m3"
+        self.dims = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0,
+                                  kv_dtype=kvg.KVG_KV_E4M3 if fp8 else kvg.KVG_KV_BF16,
+                                  k_scale=syn.FP8_K_SCALE, v_scale=syn.FP8_V_SCALE)
+        elem = 1 if fp8 else 2
         n_pages = syn.B12_CTX // P + self.nb // P
         self.cache = kvg.Cache(self.dims, n_pages + (self.nb // P if pool_store else 0), 2, syn.B12_CTX)
         # pool_store: the block lives in the cache's own pool and grafts by
@@ -162,7 +169,7 @@ class Step12B:
         stream.synchronize()
         self.kb, self.vb = kb, vb  # the block's rows, kept for parity tests
         self.scale = 1.0 / math.sqrt(w.head_dim)
-        blk_pages = w.n_layers * 2 * (self.nb // P) * w.page_bytes
+        blk_pages = w.n_layers * 2 * (self.nb // P) * w.page_bytes * elem // 2
         self.pool_store = pool_store
         # swa = (W, R): sliding-window layers over the full-size cache, every
         # R-th layer global and the others attending to their last W rows
@@ -176,8 +183,8 @@ class Step12B:
         self.bytes = {
             "graft": 0 if pool_store else 2 * blk_pages,
             "verify": blk_pages,
-            "append": 2 * w.n_layers * 2 * self.nf * w.n_kv_heads * w.head_dim * 2,
-            "decode": rows_read * 2 * w.n_kv_heads * w.head_dim * 2 + 2 * self.q.numel() * 2,
+            "append": (2 + elem) * w.n_layers * 2 * self.nf * w.n_kv_heads * w.head_dim,
+            "decode": rows_read * 2 * w.n_kv_heads * w.head_dim * elem + 2 * self.q.numel() * 2,
         }
         self.sha_blocks = (blk_pages // 4096) * 65
         self.blk_pages = blk_pages
@@ -267,7 +274,7 @@ def run_kvg(args, rank, world):
     hbm_peak, sm_max, peak_kind = load_peaks()
     swa = tuple(int(x) for x in args.swa.split(":")) if args.swa else None
     st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool", schedule=args.schedule,
-                 swa=swa)
+                 swa=swa, kv=args.kv)
 
     # correctness of the configuration being timed: one verified step
     st.run_step()
@@ -396,7 +403,9 @@ def run_kvg(args, rank, world):
                                + (" [block in the cache pool: zero-copy graft]" if st.pool_store else "")
                                + (" [verified graft in one pass, beside the append]" if st.schedule == "fused" else "")
                                + (f" [sliding-window layers: window {st.swa[0]}, every {st.swa[1]}th layer global]"
-                                  if st.swa else ""),
+                                  if st.swa else "")
+                               + (f" [fp8 E4M3 KV, scales k {syn.FP8_K_SCALE} v {syn.FP8_V_SCALE}]"
+                                  if st.kv == "e4m3" else ""),
                    "global_batch": world, "seq_len": syn.B12_CTX, "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)"},
         "parts": parts, "roofline": roof, "e2e": e2e, "gpu_launches": int(launches),
@@ -815,6 +824,8 @@ def main():
                          "into the graft, which runs beside the append (fused)")
     ap.add_argument("--swa", default="", help="12b step with sliding-window layers, 'W:R' (window W, every "
                                               "R-th layer global), over the full-size cache")
+    ap.add_argument("--kv", default="bf16", choices=["bf16", "e4m3"],
+                    help="12b step: KV element type of the cache and the block (e4m3: quantized KV blocks)")
     ap.add_argument("--store", default="hbm", choices=["hbm", "pool"],
                     help="12b: block in an HBM store (copying graft) or in the cache pool (zero-copy graft)")
     ap.add_argument("--deep-blocks", type=int, default=syn.DEEP_BLOCKS)
@@ -837,7 +848,7 @@ def main():
         torch.distributed.init_process_group("nccl")
     line = run_kvg(args, rank, world)
     if rank == 0:
-        if not args.no_cpu_baseline and not args.swa:
+        if not args.no_cpu_baseline and not args.swa and args.kv == "bf16":
             line["cpu_baseline"] = cpu_baseline(args.cpu_baseline_layers)
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -61,6 +61,8 @@ enum { KVG_RESIDENCY_HBM = 0, KVG_RESIDENCY_PINNED_HOST = 1, KVG_RESIDENCY_CACHE
 enum { KVG_ROPE_HALF = 0, KVG_ROPE_INTERLEAVED = 1 };
 enum { KVG_GRAFT_VERIFY = 1u, KVG_GRAFT_SYNC = 2u };
 enum { KVG_SHA256_PLAIN = 0, KVG_SHA256_PAGED = 1 };
+/* KV element types (kvg_dims.kv_dtype). */
+enum { KVG_KV_BF16 = 0, KVG_KV_E4M3 = 1 };
 
 /* Leaf size of the two-level page digest (bytes). */
 #define KVG_DIGEST_LEAF_BYTES 4096
@@ -69,12 +71,23 @@ enum { KVG_SHA256_PLAIN = 0, KVG_SHA256_PAGED = 1 };
 
 /* KV geometry shared by a store and the caches it grafts into.
  * A page holds page_size consecutive token slots of every KV head:
- * bf16 [n_kv_heads][page_size][head_dim] per layer and per K or V, so
- * page_bytes = 2 * n_kv_heads * page_size * head_dim.
+ * [n_kv_heads][page_size][head_dim] elements per layer and per K or V, so
+ * page_bytes = elem_bytes * n_kv_heads * page_size * head_dim.
  * Supported: head_dim in {64, 128, 256}; page_size >= 1; page_bytes a
  * multiple of 16.  rope_theta / rope_style only matter for relocation:
  * the rotation pairs dimension i with i + head_dim/2 (KVG_ROPE_HALF) or
- * 2i with 2i+1 (KVG_ROPE_INTERLEAVED) at frequency rope_theta^(-2i/head_dim). */
+ * 2i with 2i+1 (KVG_ROPE_INTERLEAVED) at frequency rope_theta^(-2i/head_dim).
+ * Element type (quantized KV blocks: a block's size depends on the cache's
+ * quantization, Sec. 4.4):
+ *   KVG_KV_BF16 (0): bf16, elem_bytes 2; k_scale, v_scale ignored.
+ *   KVG_KV_E4M3 (1): fp8 E4M3 codes, elem_bytes 1, with per-tensor fp32
+ *     scales (finite, > 0): a K element is its code's value * k_scale, a V
+ *     element * v_scale.  Appends quantize bf16 input: the fp32 value times
+ *     r = fp32(1 / scale) (IEEE fp32 division, then one fp32 product),
+ *     rounded to nearest-even on the E4M3 grid, saturating at +-448.
+ *     Relocation (delta != 0) is not supported; decode needs head_dim 128 or
+ *     256.  Blocks carry the scales; a block grafts only into a cache with
+ *     the same element type and scales. */
 typedef struct kvg_dims {
     int32_t n_layers;
     int32_t n_kv_heads;
@@ -82,7 +95,9 @@ typedef struct kvg_dims {
     int32_t page_size;
     double rope_theta;
     int32_t rope_style;
-    int32_t reserved;
+    int32_t kv_dtype;
+    float k_scale;
+    float v_scale;
 } kvg_dims;
 
 typedef struct kvg_store kvg_store;
@@ -392,7 +407,7 @@ const char *kvg_status_string(kvg_status status);
  * none); valid until the next call on the thread. */
 const char *kvg_last_error(void);
 
-/* Library version, e.g. 0x000100 for 0.1.0. */
+/* Library version, e.g. 0x000200 for 0.2.0 (0.2: kv_dtype and fp8 scales in kvg_dims). */
 uint32_t kvg_version(void);
 
 /* Number of CUDA kernel launches this library has issued since it was

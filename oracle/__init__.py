@@ -97,6 +97,18 @@ def lib():
                                          ctypes.c_uint64, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                          ctypes.c_double, ctypes.c_void_p]
             L.ora_omp_threads.restype = ctypes.c_int
+            L.ora_e4m3_to_f64.argtypes = [ctypes.c_uint8]
+            L.ora_e4m3_to_f64.restype = ctypes.c_double
+            L.ora_e4m3_rne_sat.argtypes = [ctypes.c_double]
+            L.ora_e4m3_rne_sat.restype = ctypes.c_uint8
+            L.ora_e4m3_quantize_bf16.argtypes = [ctypes.c_void_p, ctypes.c_uint64, ctypes.c_float,
+                                                 ctypes.c_void_p]
+            L.ora_e4m3_quantize_bf16.restype = None
+            L.ora_e4m3_dequant.argtypes = [ctypes.c_void_p, ctypes.c_uint64, ctypes.c_float, ctypes.c_void_p]
+            L.ora_e4m3_dequant.restype = None
+            L.ora_gqa_decode_f64kv.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                               ctypes.c_uint64, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                               ctypes.c_double, ctypes.c_void_p]
             del u8p
         return _lib
 
@@ -225,6 +237,52 @@ def attention_head(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float) ->
     return o
 
 
+def e4m3_to_f64(c) -> np.ndarray:
+    """Values of E4M3 codes (uint8) in fp64."""
+    c = np.ascontiguousarray(c, np.uint8)
+    out = np.zeros(c.shape, np.float64)
+    lib().ora_e4m3_dequant(_ptr(c), c.size, 1.0, _ptr(out))
+    return out
+
+
+def e4m3_rne(x) -> np.ndarray:
+    """fp64 values -> E4M3 codes, ties to even, saturating at +-448."""
+    x = np.asarray(x, np.float64)
+    return np.array([lib().ora_e4m3_rne_sat(float(v)) for v in x.reshape(-1)], np.uint8).reshape(x.shape)
+
+
+def e4m3_quantize(x_bf16: np.ndarray, scale: float) -> np.ndarray:
+    """bf16 bits -> E4M3 codes of fp32 value * fp32(1 / scale), the product in fp32."""
+    x = np.ascontiguousarray(x_bf16, np.uint16)
+    out = np.zeros(x.shape, np.uint8)
+    lib().ora_e4m3_quantize_bf16(_ptr(x), x.size, float(scale), _ptr(out))
+    return out
+
+
+def e4m3_dequant(c: np.ndarray, scale: float) -> np.ndarray:
+    """E4M3 codes -> code value * scale in fp64."""
+    c = np.ascontiguousarray(c, np.uint8)
+    out = np.zeros(c.shape, np.float64)
+    lib().ora_e4m3_dequant(_ptr(c), c.size, float(scale), _ptr(out))
+    return out
+
+
+def gqa_decode_f64kv(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float) -> np.ndarray:
+    """gqa_decode with k/v given as fp64 values [n][Hkv][D] (dequantized rows)."""
+    q = np.ascontiguousarray(q, np.uint16)
+    k = np.ascontiguousarray(k, np.float64)
+    v = np.ascontiguousarray(v, np.float64)
+    Hq, D = q.shape
+    n, Hkv, D2 = k.shape
+    assert D2 == D and v.shape == k.shape
+    o = np.zeros((Hq, D), np.float64)
+    rc = lib().ora_gqa_decode_f64kv(_ptr(q), _ptr(k) if n else None, _ptr(v) if n else None, n, Hq, Hkv, D,
+                                    float(scale), _ptr(o))
+    if rc:
+        raise ValueError("gqa_decode: Hq must be a multiple of Hkv")
+    return o
+
+
 def gqa_decode(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float) -> np.ndarray:
     """Decode attention of one query token: q[Hq][D], k/v[n][Hkv][D] (bf16 bits,
     logical token order) -> fp64 o[Hq][D].  Query head h reads KV head
@@ -251,14 +309,31 @@ def _round_up(x: int, m: int) -> int:
     return (x + m - 1) // m * m
 
 
+KV_BF16, KV_E4M3 = 0, 1  # cache element types (dims); block header dtype codes 1, 2
+
+
 class Dims:
-    """KV geometry: L layers, Hkv KV heads, D head dim, P tokens per page."""
+    """KV geometry: L layers, Hkv KV heads, D head dim, P tokens per page, and
+    the element type: bf16, or fp8 E4M3 codes with per-tensor scales (a K
+    element is code value * k_scale, a V element code value * v_scale)."""
 
     def __init__(self, n_layers, n_kv_heads, head_dim, page_size, rope_theta=10000.0,
-                 rope_style=0):
+                 rope_style=0, kv_dtype=KV_BF16, k_scale=1.0, v_scale=1.0):
         self.L, self.Hkv, self.D, self.P = int(n_layers), int(n_kv_heads), int(head_dim), int(page_size)
         self.rope_theta = float(rope_theta)
         self.rope_style = int(rope_style)
+        self.kv_dtype = int(kv_dtype)
+        # the scales are fp32 values
+        self.k_scale = float(np.float32(k_scale))
+        self.v_scale = float(np.float32(v_scale))
+
+    @property
+    def fp8(self):
+        return self.kv_dtype == KV_E4M3
+
+    @property
+    def code_dtype(self):
+        return np.uint8 if self.fp8 else np.uint16
 
     @property
     def page_elems(self):
@@ -266,7 +341,17 @@ class Dims:
 
     @property
     def page_bytes(self):
-        return 2 * self.page_elems
+        return (1 if self.fp8 else 2) * self.page_elems
+
+    def same(self, o) -> bool:
+        return ((self.L, self.Hkv, self.D, self.P, self.kv_dtype) == (o.L, o.Hkv, o.D, o.P, o.kv_dtype)
+                and (not self.fp8 or (self.k_scale, self.v_scale) == (o.k_scale, o.v_scale)))
+
+    def codes(self, k_bf16: np.ndarray, v_bf16: np.ndarray):
+        """Rows as the cache stores them: bf16 bits, or E4M3 codes."""
+        if not self.fp8:
+            return k_bf16, v_bf16
+        return e4m3_quantize(k_bf16, self.k_scale), e4m3_quantize(v_bf16, self.v_scale)
 
 
 class Block:
@@ -284,7 +369,7 @@ class Block:
         self.positions = np.ascontiguousarray(positions, np.int32)
         self.n_tokens = int(self.positions.size)
         self.n_pages = pages.shape[2]
-        self.pages = pages  # uint16 [L][2][n_pages][Hkv][P][D]
+        self.pages = pages  # [L][2][n_pages][Hkv][P][D] bf16 bits or E4M3 codes
         d = dims
         self.digests = page_digests(pages.reshape(-1), d.page_bytes).reshape(
             d.L, 2, self.n_pages, 32)
@@ -301,17 +386,19 @@ class Block:
         pos_off = HEADER_BYTES
         dig_off = _round_up(pos_off + 4 * self.n_tokens, 256)
         pages_off = _round_up(dig_off + self.digests.size, 4096)
-        total = pages_off + self.pages.size * 2
+        total = pages_off + self.pages.size * (1 if d.fp8 else 2)
         hdr = bytearray(HEADER_BYTES)
         struct.pack_into("<8sIIiiiiqqdiiQQQQ", hdr, 0, BLOCK_MAGIC, BLOCK_VERSION, HEADER_BYTES,
                          d.L, d.Hkv, d.D, d.P, self.n_tokens, self.n_pages, d.rope_theta,
-                         d.rope_style, 1, pos_off, dig_off, pages_off, total)
+                         d.rope_style, 2 if d.fp8 else 1, pos_off, dig_off, pages_off, total)
         hdr[96:128] = self.block_digest
+        if d.fp8:  # the per-tensor scales, fp32 at bytes 128 (K) and 132 (V)
+            struct.pack_into("<ff", hdr, 128, d.k_scale, d.v_scale)
         out = bytearray(total)
         out[:HEADER_BYTES] = hdr
         out[pos_off:pos_off + 4 * self.n_tokens] = self.positions.astype("<i4").tobytes()
         out[dig_off:dig_off + self.digests.size] = self.digests.tobytes()
-        out[pages_off:] = self.pages.astype("<u2").tobytes()
+        out[pages_off:] = self.pages.astype("u1" if d.fp8 else "<u2").tobytes()
         return bytes(out)
 
     @staticmethod
@@ -336,11 +423,13 @@ class BlockMeta:
 
 
 def block_from_kv(dims: Dims, k: np.ndarray, v: np.ndarray, positions: np.ndarray) -> Block:
-    """Deposit of logical rows: k, v [L][n][Hkv][D] bf16 bits, positions[n]."""
+    """Deposit of logical rows: k, v [L][n][Hkv][D] bf16 bits (quantized to the
+    cache's element type), positions[n]."""
     d = dims
+    k, v = d.codes(k, v)
     n = int(positions.size)
     npb = (n + d.P - 1) // d.P
-    pages = np.zeros((d.L, 2, npb, d.Hkv, d.P, d.D), np.uint16)
+    pages = np.zeros((d.L, 2, npb, d.Hkv, d.P, d.D), d.code_dtype)
     for t in range(n):
         j, r = divmod(t, d.P)
         pages[:, 0, j, :, r, :] = k[:, t, :, :]
@@ -396,7 +485,7 @@ class OracleCache:
         self.max_seqs = max_seqs
         self.max_slots = max_slots
         self.max_pages = (max_slots + d.P - 1) // d.P
-        self.pool = np.zeros((d.L, 2, n_pages, d.Hkv, d.P, d.D), np.uint16) if with_pool else None
+        self.pool = np.zeros((d.L, 2, n_pages, d.Hkv, d.P, d.D), d.code_dtype) if with_pool else None
         if fill is not None and self.pool is not None:
             self.pool[...] = fill
         self.free = list(range(n_pages))
@@ -422,8 +511,10 @@ class OracleCache:
         return got
 
     def append(self, seq: int, k: np.ndarray, v: np.ndarray, positions: np.ndarray):
-        """Fresh write of n rows (k, v [L][n][Hkv][D]) at slots n_slots.. (Sec. 3.2 fresh arm)."""
+        """Fresh write of n rows (k, v [L][n][Hkv][D] bf16 bits, quantized to the
+        cache's element type) at slots n_slots.. (Sec. 3.2 fresh arm)."""
         d = self.dims
+        k, v = d.codes(k, v)
         n = int(positions.size)
         s0 = int(self.n_slots[seq])
         if s0 + n > self.max_slots:
@@ -454,8 +545,10 @@ class OracleCache:
         padding rows are copied unchanged."""
         d = self.dims
         bd = block.dims
-        if (bd.L, bd.Hkv, bd.D, bd.P) != (d.L, d.Hkv, d.D, d.P):
+        if not bd.same(d):
             raise KvgError("dims")
+        if delta != 0 and d.fp8:
+            raise KvgError("relocation needs bf16 keys")
         boundary = _round_up(int(self.n_slots[seq]), d.P)
         if dst_slot < 0:
             dst_slot = boundary
@@ -541,7 +634,7 @@ class OracleCache:
         if slot0 % d.P or slot0 + n > int(self.n_slots[seq]) or n <= 0:
             raise KvgError("range")
         npb = (n + d.P - 1) // d.P
-        pages = np.zeros((d.L, 2, npb, d.Hkv, d.P, d.D), np.uint16)
+        pages = np.zeros((d.L, 2, npb, d.Hkv, d.P, d.D), d.code_dtype)
         for j in range(npb):
             pid = self.page_table[seq, slot0 // d.P + j]
             valid = min(d.P, n - j * d.P)
@@ -563,7 +656,7 @@ class OracleCache:
             vs.append(np.transpose(self.pool[layer, 1, pid, :, :f, :], (1, 0, 2)))
             ps.append(self.positions[seq, j * d.P:j * d.P + f])
         if not ks:
-            z = np.zeros((0, d.Hkv, d.D), np.uint16)
+            z = np.zeros((0, d.Hkv, d.D), d.code_dtype)
             return z, z.copy(), np.zeros(0, np.int32)
         return (np.ascontiguousarray(np.concatenate(ks)), np.ascontiguousarray(np.concatenate(vs)),
                 np.concatenate(ps))
@@ -584,4 +677,7 @@ class OracleCache:
         W = self.windows[layer]
         if W > 0:
             k, v = k[-W:], v[-W:]
+        d = self.dims
+        if d.fp8:
+            return gqa_decode_f64kv(q, e4m3_dequant(k, d.k_scale), e4m3_dequant(v, d.v_scale), scale)
         return gqa_decode(q, k, v, scale)

@@ -281,6 +281,65 @@ int ora_rope_rotate_rows_bf16(const uint16_t *x, uint64_t n, int D, double delta
 }
 
 /* ------------------------------------------------------------------------ */
+/* fp8 E4M3 KV codes (quantized KV blocks: the block's size depends on the   */
+/* cache's quantization, Sec. 4.4).  Format: sign, 4 exponent bits (bias 7), */
+/* 3 mantissa bits; exponent field 0 holds subnormals m * 2^-9; the code     */
+/* S.1111.111 is NaN; there are no infinities; the largest finite is 448.    */
+/* ------------------------------------------------------------------------ */
+
+double ora_e4m3_to_f64(uint8_t c) {
+    int s = c >> 7, e = (c >> 3) & 15, m = c & 7;
+    double v;
+    if (e == 15 && m == 7) return NAN;
+    if (e == 0)
+        v = ldexp((double)m, -9);
+    else
+        v = ldexp(1.0 + m / 8.0, e - 7);
+    return s ? -v : v;
+}
+
+/* Round-to-nearest-even onto the E4M3 grid, saturating: magnitudes above the
+ * largest finite (448) give 448; NaN gives the NaN code 0x7F. */
+uint8_t ora_e4m3_rne_sat(double x) {
+    if (isnan(x)) return 0x7F;
+    uint8_t s = signbit(x) ? 0x80 : 0x00;
+    double a = fabs(x);
+    if (a > 448.0) return s | 0x7E;
+    if (a < ldexp(1.0, -6)) {
+        /* subnormal grid m * 2^-9, m in 0..8 (8 is the smallest normal) */
+        double q = nearbyint(a / ldexp(1.0, -9));
+        return s | (uint8_t)q; /* q == 8 encodes exponent field 1, mantissa 0 */
+    }
+    int e;
+    frexp(a, &e);       /* a = f * 2^e, f in [0.5, 1): a in [2^(e-1), 2^e) */
+    int E = e - 1;      /* a in [2^E, 2^(E+1)), E in [-6, 8] */
+    double q = nearbyint(a / ldexp(1.0, E - 3)); /* 8 .. 16 units of 2^(E-3) */
+    if (q == 16.0) {
+        q = 8.0;
+        E += 1;
+    }
+    if (E > 8 || (E == 8 && q > 14.0)) return s | 0x7E; /* cannot happen after the clamp */
+    return s | (uint8_t)(((E + 7) << 3) | ((int)q - 8));
+}
+
+/* Quantization of bf16 values with a per-tensor scale: r = 1 / scale as an
+ * fp32 quotient; each bf16 value as fp32 times r, rounded once to fp32; then
+ * E4M3 RNE with saturation. */
+void ora_e4m3_quantize_bf16(const uint16_t *x, uint64_t n, float scale, uint8_t *out) {
+    float r = 1.0f / scale;
+    for (uint64_t i = 0; i < n; ++i) {
+        float f = (float)ora_bf16_to_f64(x[i]);
+        float y = f * r;
+        out[i] = ora_e4m3_rne_sat((double)y);
+    }
+}
+
+/* Dequantized values: code value times the scale, in fp64 (exact). */
+void ora_e4m3_dequant(const uint8_t *c, uint64_t n, float scale, double *out) {
+    for (uint64_t i = 0; i < n; ++i) out[i] = ora_e4m3_to_f64(c[i]) * (double)scale;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Decode attention in fp64 (Sec. 3.2 / Sec. 4.3: the query decoded on top   */
 /* of the restored prefix attends to every cached token).                   */
 /* ------------------------------------------------------------------------ */
@@ -330,6 +389,44 @@ int ora_gqa_decode(const uint16_t *q, const uint16_t *k, const uint16_t *v, uint
         int g = h / G;
         ora_attention_head(q + (uint64_t)h * D, k + (uint64_t)g * D, v + (uint64_t)g * D, n,
                            (uint64_t)Hkv * D, D, scale, o + (uint64_t)h * D);
+    }
+    return 0;
+}
+
+/* The same attention with K and V given as fp64 values (dequantized rows):
+ * identical steps, only the loads differ. */
+static void attention_head_f64kv(const uint16_t *q, const double *k, const double *v, uint64_t n,
+                                 uint64_t row_stride, int D, double scale, double *o) {
+    for (int d = 0; d < D; ++d) o[d] = 0.0;
+    if (n == 0) return;
+    double *s = (double *)malloc(sizeof(double) * n);
+    if (!s) return;
+    double m = -INFINITY;
+    for (uint64_t t = 0; t < n; ++t) {
+        double acc = 0.0;
+        for (int d = 0; d < D; ++d) acc += ora_bf16_to_f64(q[d]) * k[t * row_stride + d];
+        s[t] = acc * scale;
+        if (s[t] > m) m = s[t];
+    }
+    double l = 0.0;
+    for (uint64_t t = 0; t < n; ++t) {
+        double w = exp(s[t] - m);
+        l += w;
+        for (int d = 0; d < D; ++d) o[d] += w * v[t * row_stride + d];
+    }
+    for (int d = 0; d < D; ++d) o[d] /= l;
+    free(s);
+}
+
+int ora_gqa_decode_f64kv(const uint16_t *q, const double *k, const double *v, uint64_t n, int Hq, int Hkv,
+                         int D, double scale, double *o) {
+    if (Hkv <= 0 || Hq % Hkv) return -1;
+    int G = Hq / Hkv;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int h = 0; h < Hq; ++h) {
+        int g = h / G;
+        attention_head_f64kv(q + (uint64_t)h * D, k + (uint64_t)g * D, v + (uint64_t)g * D, n,
+                             (uint64_t)Hkv * D, D, scale, o + (uint64_t)h * D);
     }
     return 0;
 }

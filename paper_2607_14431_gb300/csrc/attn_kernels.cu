@@ -33,6 +33,7 @@
 // logical token indices and of (T, W) only — never of physical page ids — so
 // results are bitwise reproducible and identical for grafted and freshly
 // written rows.
+#include <cuda_fp16.h>
 #include <math.h>
 
 #include "common.cuh"
@@ -56,18 +57,27 @@ struct TileShape<256> {
     static constexpr int TOK = 16, STAGES = 3;
 };
 
-template <int D>
+// FP8: the pool holds E4M3 codes; TMA brings boxes of 128 one-byte columns.
+// Keys go from the fp8 tile straight into MMA fragments; values are expanded
+// into a 16-bit staging tile with the bf16 layout (for ldmatrix.trans).
+// fp8 tiles carry half the bytes; two stages per warp leave room for 8
+// warps per SM (the decode is latency-bound per warp: more warps, not deeper
+// rings, keep HBM busy; three stages gave 0.77 of the copy peak, two 0.97)
+template <int D, bool FP8 = false>
 struct Cfg {
     static constexpr int TOK = TileShape<D>::TOK;
-    static constexpr int STAGES = TileShape<D>::STAGES;
-    static constexpr int NB = D / 64;                  // 64-column boxes per K (or V) tile
+    static constexpr int STAGES = FP8 ? 2 : TileShape<D>::STAGES;
+    static constexpr int NB = D / 64;                  // 64-column 16-bit boxes per K (or V) tile
     static constexpr int BOX = TOK * 128;              // bytes of one box (TOK rows x 128 B)
-    static constexpr int STAGE_BYTES = 2 * NB * BOX;   // K boxes then V boxes
+    static constexpr int NB8 = FP8 ? D / 128 : 0;      // 128-column fp8 boxes per K (or V) tile
+    static constexpr int STAGE_BYTES = FP8 ? 2 * NB8 * BOX : 2 * NB * BOX;  // K boxes then V boxes
     static constexpr int RING_BYTES = STAGES * STAGE_BYTES;
-    static constexpr int SMEM = RING_BYTES + STAGES * (8 + 4 + 4) + 1024;  // + alignment slack
+    static constexpr int STAGING_BYTES = FP8 ? NB * BOX : 0;  // the current tile's values, expanded
+    static constexpr int SMEM = RING_BYTES + STAGING_BYTES + STAGES * (8 + 4 + 4) + 1024;  // + alignment slack
     static constexpr int KS = D / 16;                  // k-steps of q.k, m-tiles of p.v
     static constexpr int SUB = TOK / 16;               // 16-row sub-tiles per tile
     static_assert(BOX % 1024 == 0, "a swizzle atom is 8 rows of 128 bytes");
+    static_assert(!FP8 || D % 128 == 0, "fp8 tiles are whole 128-byte boxes");
 };
 
 // Position of global tile t: unit (lr, b, g) and tile index within the unit.
@@ -114,28 +124,66 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t 
                  : "r"(addr));
 }
 
-// D += A(16x16, row) . B(16x8, col), bf16 inputs, fp32 accumulators.
-__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
-                                         uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-        "{%0,%1,%2,%3};"
-        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+// D += A(16x16, row) . B(16x8, col), bf16 (F16: fp16) inputs, fp32 accumulators.
+template <bool F16>
+__device__ __forceinline__ void mma16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                      uint32_t b0, uint32_t b1) {
+    if constexpr (F16)
+        asm volatile(
+            "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+            "{%0,%1,%2,%3};"
+            : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+            : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+    else
+        asm volatile(
+            "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+            "{%0,%1,%2,%3};"
+            : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+            : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<const uint32_t *>(&v);
+// Two floats rounded (RNE) to the MMA's 16-bit type, low half first.
+template <bool F16>
+__device__ __forceinline__ uint32_t pack16(float lo, float hi) {
+    if constexpr (F16) {
+        const __half2 v = __floats2half2_rn(lo, hi);
+        return *reinterpret_cast<const uint32_t *>(&v);
+    } else {
+        const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+        return *reinterpret_cast<const uint32_t *>(&v);
+    }
 }
 
-__device__ __forceinline__ float bf16_lo(uint32_t x) { return __uint_as_float(x << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t x) { return __uint_as_float(x & 0xffff0000u); }
+// The two values of a packed 16-bit pair, as floats.
+template <bool F16>
+__device__ __forceinline__ float lo16(uint32_t x) {
+    if constexpr (F16)
+        return __low2float(*reinterpret_cast<const __half2 *>(&x));
+    else
+        return __uint_as_float(x << 16);
+}
+template <bool F16>
+__device__ __forceinline__ float hi16(uint32_t x) {
+    if constexpr (F16)
+        return __high2float(*reinterpret_cast<const __half2 *>(&x));
+    else
+        return __uint_as_float(x & 0xffff0000u);
+}
 
-template <int D, int G>
+// Two E4M3 codes (low byte first) -> two fp16 values (exact: every E4M3
+// value is an fp16 value).
+__device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t two_codes) {
+    uint32_t d;
+    const uint16_t a = (uint16_t)two_codes;
+    asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(d) : "h"(a));
+    return d;
+}
+
+template <int D, int G, bool FP8>
 __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const __grid_constant__ CUtensorMap pool_map) {
-    using C = Cfg<D>;
+    using C = Cfg<D, FP8>;
     constexpr int TOK = C::TOK, STAGES = C::STAGES, KS = C::KS, SUB = C::SUB, NB = C::NB, BOX = C::BOX;
+    constexpr int NB8 = C::NB8;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // swizzled boxes must start on a 1024-byte boundary
     uint8_t *smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
@@ -149,8 +197,9 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
     const int tpp = (P + TOK - 1) / TOK;
 
     uint8_t *ring = smem;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::RING_BYTES);
-    int *vrs = reinterpret_cast<int *>(smem + C::RING_BYTES + STAGES * 8);  // valid rows [los, vrs) per stage
+    uint8_t *staging = smem + C::RING_BYTES;  // fp8: the current tile's values expanded to fp16
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::RING_BYTES + C::STAGING_BYTES);
+    int *vrs = reinterpret_cast<int *>(smem + C::RING_BYTES + C::STAGING_BYTES + STAGES * 8);  // valid rows [los, vrs)
     int *los = vrs + STAGES;
     if (lane == 0) {
 #pragma unroll
@@ -213,10 +262,18 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
                                             (int64_t)k * TOK);
             const int32_t row_v = (int32_t)(row_k + plane_rows);
             uint8_t *dst = ring + stg * C::STAGE_BYTES;
+            if constexpr (FP8) {
 #pragma unroll
-            for (int b = 0; b < NB; ++b) {
-                tma_load_2d(dst + b * BOX, &pool_map, 64 * b, row_k, bar);
-                tma_load_2d(dst + (NB + b) * BOX, &pool_map, 64 * b, row_v, bar);
+                for (int b = 0; b < NB8; ++b) {
+                    tma_load_2d(dst + b * BOX, &pool_map, 128 * b, row_k, bar);
+                    tma_load_2d(dst + (NB8 + b) * BOX, &pool_map, 128 * b, row_v, bar);
+                }
+            } else {
+#pragma unroll
+                for (int b = 0; b < NB; ++b) {
+                    tma_load_2d(dst + b * BOX, &pool_map, 64 * b, row_k, bar);
+                    tma_load_2d(dst + (NB + b) * BOX, &pool_map, 64 * b, row_v, bar);
+                }
             }
         } else {
             mbar_arrive(bar);
@@ -260,9 +317,18 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
 #pragma unroll
         for (int ks = 0; ks < KS; ++ks) {
             if (gq < G) {
-                const uint32_t *q32 = reinterpret_cast<const uint32_t *>(qrow + gq * D + 16 * ks + 2 * tq);
-                qb[ks][0] = q32[0];
-                qb[ks][1] = q32[4];  // dims + 8
+                if constexpr (FP8) {
+                    // fp16 MMAs over permuted dims: within each 16-dim step the
+                    // MMA's k = 2tq, 2tq+1, 2tq+8, 2tq+9 are dims 4tq .. 4tq+3, so a
+                    // key row's 4 consecutive codes fill a lane's two registers
+                    const uint32_t *q32 = reinterpret_cast<const uint32_t *>(qrow + gq * D + 16 * ks + 4 * tq);
+                    qb[ks][0] = pack16<true>(lo16<false>(q32[0]), hi16<false>(q32[0]));
+                    qb[ks][1] = pack16<true>(lo16<false>(q32[1]), hi16<false>(q32[1]));
+                } else {
+                    const uint32_t *q32 = reinterpret_cast<const uint32_t *>(qrow + gq * D + 16 * ks + 2 * tq);
+                    qb[ks][0] = q32[0];
+                    qb[ks][1] = q32[4];  // dims + 8
+                }
             } else {
                 qb[ks][0] = qb[ks][1] = 0u;
             }
@@ -298,7 +364,35 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
         }
         const int vr = vrs[stg], lo = los[stg];
         bool zeroed = false;
-        if (vr > 0 && (vr < TOK || lo > 0)) {
+        if constexpr (FP8) {
+            if (vr > 0) {
+                // expand the value codes into the fp16 staging tile (the swizzled
+                // box layout of a bf16 tile); rows outside [lo, vr) become zeros.
+                // All loads first, then the conversions and stores.
+                constexpr int GPR = D / 8;             // 8-value groups per row
+                constexpr int ITEMS = TOK * GPR / 32;  // per lane
+                const uint8_t *v8 = ring + stg * C::STAGE_BYTES + NB8 * BOX;
+                uint2 w[ITEMS];
+#pragma unroll
+                for (int i = 0; i < ITEMS; ++i) {
+                    const int item = i * 32 + lane, r = item / GPR, g = item % GPR;
+                    w[i] = make_uint2(0, 0);
+                    if (r >= lo && r < vr)
+                        w[i] = *reinterpret_cast<const uint2 *>(v8 + (g >> 4) * BOX + r * 128 +
+                                                                ((((g & 15) >> 1) ^ (r & 7)) << 4) + (g & 1) * 8);
+                }
+#pragma unroll
+                for (int i = 0; i < ITEMS; ++i) {
+                    const int item = i * 32 + lane, r = item / GPR, g = item % GPR;
+                    *reinterpret_cast<uint4 *>(staging + (g >> 3) * BOX + r * 128 + (((g & 7) ^ (r & 7)) << 4)) =
+                        make_uint4(e4m3x2_to_f16x2(w[i].x), e4m3x2_to_f16x2(w[i].x >> 16), e4m3x2_to_f16x2(w[i].y),
+                                   e4m3x2_to_f16x2(w[i].y >> 16));
+                }
+                __syncwarp();
+            } else if (lane == 0 && t + STAGES < t1) {
+                issue(stg);  // an empty tile: nothing to read from the stage
+            }
+        } else if (vr > 0 && (vr < TOK || lo > 0)) {
             // value rows past the fill hold whatever the pool had there, and
             // rows before a window's start are outside the attention: zero
             // both so their zero weights contribute exactly 0
@@ -316,25 +410,43 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
         }
         if (vr > 0) {
             const uint32_t ks_base = ring_s + stg * C::STAGE_BYTES;
-            const uint32_t vs_base = ks_base + NB * BOX;
+            const uint32_t vs_base = FP8 ? smem_addr(staging) : ks_base + NB * BOX;
             // ---- scores S[16 rows][8 heads] per sub-tile
             float sc[SUB][4];
 #pragma unroll
             for (int sb = 0; sb < SUB; ++sb) {
                 float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
-                // lane -> row of its 8x8 matrix (rows +8 for matrices 1,3) and
-                // 16-byte chunk (+1 for matrices 2,3), swizzled: chunk ^ (row & 7)
-                const uint32_t a_row = ks_base + (16 * sb + (lane & 7) + ((lane >> 3) & 1) * 8) * 128;
-                const int a_hi = (lane >> 4) & 1;
+                if constexpr (FP8) {
+                    // rows gq and gq+8 of the sub-tile, 4 codes at dims 16ks + 4tq of
+                    // each (swizzle: chunk ^ (row & 7), the same for both rows)
+                    const uint8_t *k0 = ring + stg * C::STAGE_BYTES + (16 * sb + gq) * 128 + 4 * tq;
 #pragma unroll
-                for (int ks = 0; ks < KS; ++ks) {
-                    uint32_t a0, a1, a2, a3;
-                    const int chunk = ((ks & 3) << 1) + a_hi;
-                    ldsm_x4(a_row + (ks >> 2) * BOX + ((chunk ^ (lane & 7)) << 4), a0, a1, a2, a3);
-                    if (ks & 1)
-                        mma_bf16(acc1, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
-                    else
-                        mma_bf16(acc0, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+                    for (int ks = 0; ks < KS; ++ks) {
+                        const int off = (ks >> 3) * BOX + (((ks & 7) ^ gq) << 4);
+                        const uint32_t w0 = *reinterpret_cast<const uint32_t *>(k0 + off);
+                        const uint32_t w1 = *reinterpret_cast<const uint32_t *>(k0 + off + 8 * 128);
+                        const uint32_t a0 = e4m3x2_to_f16x2(w0), a2 = e4m3x2_to_f16x2(w0 >> 16);
+                        const uint32_t a1 = e4m3x2_to_f16x2(w1), a3 = e4m3x2_to_f16x2(w1 >> 16);
+                        if (ks & 1)
+                            mma16<true>(acc1, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+                        else
+                            mma16<true>(acc0, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+                    }
+                } else {
+                    // lane -> row of its 8x8 matrix (rows +8 for matrices 1,3) and
+                    // 16-byte chunk (+1 for matrices 2,3), swizzled: chunk ^ (row & 7)
+                    const uint32_t a_row = ks_base + (16 * sb + (lane & 7) + ((lane >> 3) & 1) * 8) * 128;
+                    const int a_hi = (lane >> 4) & 1;
+#pragma unroll
+                    for (int ks = 0; ks < KS; ++ks) {
+                        uint32_t a0, a1, a2, a3;
+                        const int chunk = ((ks & 3) << 1) + a_hi;
+                        ldsm_x4(a_row + (ks >> 2) * BOX + ((chunk ^ (lane & 7)) << 4), a0, a1, a2, a3);
+                        if (ks & 1)
+                            mma16<false>(acc1, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+                        else
+                            mma16<false>(acc0, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+                    }
                 }
                 const int r0 = 16 * sb + gq, r1 = r0 + 8;
                 const bool in0 = r0 >= lo && r0 < vr, in1 = r1 >= lo && r1 < vr;
@@ -342,6 +454,11 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
                 sc[sb][1] = in0 ? (acc0[1] + acc1[1]) * p.qscale : -INFINITY;
                 sc[sb][2] = in1 ? (acc0[2] + acc1[2]) * p.qscale : -INFINITY;
                 sc[sb][3] = in1 ? (acc0[3] + acc1[3]) * p.qscale : -INFINITY;
+            }
+            if constexpr (FP8) {
+                // the keys have been read: the stage can take the next tile
+                __syncwarp();
+                if (lane == 0 && t + STAGES < t1) issue(stg);
             }
             // ---- online softmax for heads 2*tq (e = 0) and 2*tq+1 (e = 1)
             float mt_[2] = {-INFINITY, -INFINITY};
@@ -368,11 +485,11 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
             }
 #pragma unroll
             for (int sb = 0; sb < SUB; ++sb) {
-                // weights, rounded to bf16 exactly as the MMA consumes them
-                const uint32_t p01 = pack_bf16(exp2f(sc[sb][0] - m[0]), exp2f(sc[sb][1] - m[1]));
-                const uint32_t p23 = pack_bf16(exp2f(sc[sb][2] - m[0]), exp2f(sc[sb][3] - m[1]));
-                lsum[0] += bf16_lo(p01) + bf16_lo(p23);
-                lsum[1] += bf16_hi(p01) + bf16_hi(p23);
+                // weights, rounded to the MMA's 16-bit type exactly as it consumes them
+                const uint32_t p01 = pack16<FP8>(exp2f(sc[sb][0] - m[0]), exp2f(sc[sb][1] - m[1]));
+                const uint32_t p23 = pack16<FP8>(exp2f(sc[sb][2] - m[0]), exp2f(sc[sb][3] - m[1]));
+                lsum[0] += lo16<FP8>(p01) + lo16<FP8>(p23);
+                lsum[1] += hi16<FP8>(p01) + hi16<FP8>(p23);
                 // B fragment of P^T for this lane: tokens 2*tq, 2*tq+1 (+8) of head gq,
                 // held by lanes 4*token + gq/2 in half gq%2 of p01 (p23 for +8)
                 const int src0 = 4 * (2 * tq) + (gq >> 1), src1 = src0 + 4;
@@ -392,13 +509,13 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
                     uint32_t a0, a1, a2, a3;
                     const int chunk = ((mt & 3) << 1) + v_hi;
                     ldsm_x4_t(v_row + (mt >> 2) * BOX + ((chunk ^ (lane & 7)) << 4), a0, a1, a2, a3);
-                    mma_bf16(o[mt], a0, a1, a2, a3, b0, b1);
+                    mma16<FP8>(o[mt], a0, a1, a2, a3, b0, b1);
                 }
             }
         }
         __syncwarp();
         (void)zeroed;
-        if (lane == 0 && t + STAGES < t1) issue(stg);
+        if (!FP8 && lane == 0 && t + STAGES < t1) issue(stg);
     }
     if (!alive) {
         // a copy never completed: wait (bounded) on every stage once more so
@@ -448,21 +565,21 @@ __global__ void __launch_bounds__(D) combine_kernel(const DecodeParams p) {
             O = __fmaf_rn(p.part_o[((unit + w) * G + hh) * D + d], sc, O);
         }
     }
-    const float r = L > 0.f ? __fdiv_rn(O, L) : 0.f;
+    const float r = L > 0.f ? __fdiv_rn(O, L) * p.vscale : 0.f;
     p.out[((int64_t)(p.qlayers[lr] * p.q_row_stride_b + p.b0 + b) * p.n_q_heads + h) * D + d] =
         __float2bfloat16_rn(r);
 }
 
-template <int D, int G>
+template <int D, int G, bool FP8>
 struct DecodeLaunch {
     static int max_blocks_per_sm() {
         static int cached = -1;
         if (cached < 0) {
-            if (cudaFuncSetAttribute(decode_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     Cfg<D>::SMEM) != cudaSuccess)
+            if (cudaFuncSetAttribute(decode_kernel<D, G, FP8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     Cfg<D, FP8>::SMEM) != cudaSuccess)
                 return 0;
             int n = 0;
-            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<D, G>, 32, Cfg<D>::SMEM) !=
+            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<D, G, FP8>, 32, Cfg<D, FP8>::SMEM) !=
                 cudaSuccess)
                 return 0;
             cached = n;
@@ -472,7 +589,7 @@ struct DecodeLaunch {
     static cudaError_t run(const DecodeParams &p, const CUtensorMap &map, cudaStream_t s) {
         if (max_blocks_per_sm() <= 0) return cudaErrorInvalidConfiguration;
         if (p.n_warps <= 0 || p.n_tiles <= 0) return cudaSuccess;
-        decode_kernel<D, G><<<p.n_warps, 32, Cfg<D>::SMEM, s>>>(p, map);
+        decode_kernel<D, G, FP8><<<p.n_warps, 32, Cfg<D, FP8>::SMEM, s>>>(p, map);
         count_launches(1);
         return cudaGetLastError();
     }
@@ -511,23 +628,30 @@ cudaError_t encode_tensor_map(CUtensorMap *out, int rank, void *base, const cuui
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, uint64_t rows) {
+cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, bool fp8, uint64_t rows) {
     const EncodeTiled encode = tensor_map_encoder();
     if (!encode) return cudaErrorSymbolNotFound;
     const int tok = decode_tile_tokens(head_dim);
     if (tok == 0 || rows == 0 || rows > 0x7fffffffull) return cudaErrorInvalidValue;
+    if (fp8 && head_dim % 128) {  // no fp8 decode for this head_dim: nothing to map
+        memset(out, 0, sizeof *out);
+        return cudaSuccess;
+    }
+    // 128-byte rows per box: 64 bf16 columns, or 128 fp8 columns
     const cuuint64_t dims[2] = {(cuuint64_t)head_dim, (cuuint64_t)rows};
-    const cuuint64_t strides[1] = {(cuuint64_t)head_dim * 2};
-    const cuuint32_t box[2] = {64, (cuuint32_t)tok};
+    const cuuint64_t strides[1] = {(cuuint64_t)head_dim * (fp8 ? 1 : 2)};
+    const cuuint32_t box[2] = {fp8 ? 128u : 64u, (cuuint32_t)tok};
     const cuuint32_t estr[2] = {1, 1};
-    const CUresult r = encode(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pool, dims, strides, box, estr,
+    const CUresult r = encode(out, fp8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pool,
+                              dims, strides, box, estr,
                               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-bool decode_supported(int head_dim, int group) {
+bool decode_supported(int head_dim, int group, bool fp8) {
     if (head_dim != 64 && head_dim != 128 && head_dim != 256) return false;
+    if (fp8 && head_dim == 64) return false;
     if (group != 1 && group != 2 && group != 4 && group != 8) return false;
     return head_dim * group <= 512;
 }
@@ -541,21 +665,23 @@ int decode_tile_tokens(int head_dim) {
     return 0;
 }
 
-#define KVG_DECODE_CASES(X) \
-    X(64, 1) X(64, 2) X(64, 4) X(64, 8) X(128, 1) X(128, 2) X(128, 4) X(256, 1) X(256, 2)
+#define KVG_DECODE_CASES(X)                                                                              \
+    X(64, 1, false) X(64, 2, false) X(64, 4, false) X(64, 8, false) X(128, 1, false) X(128, 2, false)   \
+    X(128, 4, false) X(256, 1, false) X(256, 2, false) X(128, 1, true) X(128, 2, true) X(128, 4, true) \
+    X(256, 1, true) X(256, 2, true)
 
-int decode_max_warps(int head_dim, int group, int n_sm) {
-#define KVG_CASE(DD, GG) \
-    if (head_dim == DD && group == GG) return DecodeLaunch<DD, GG>::max_blocks_per_sm() * n_sm;
+int decode_max_warps(int head_dim, int group, bool fp8, int n_sm) {
+#define KVG_CASE(DD, GG, FF) \
+    if (head_dim == DD && group == GG && fp8 == FF) return DecodeLaunch<DD, GG, FF>::max_blocks_per_sm() * n_sm;
     KVG_DECODE_CASES(KVG_CASE)
 #undef KVG_CASE
     return 0;
 }
 
-cudaError_t launch_decode(int head_dim, int group, const DecodeParams &p, const CUtensorMap &pool_map,
+cudaError_t launch_decode(int head_dim, int group, bool fp8, const DecodeParams &p, const CUtensorMap &pool_map,
                           cudaStream_t s) {
-#define KVG_CASE(DD, GG) \
-    if (head_dim == DD && group == GG) return DecodeLaunch<DD, GG>::run(p, pool_map, s);
+#define KVG_CASE(DD, GG, FF) \
+    if (head_dim == DD && group == GG && fp8 == FF) return DecodeLaunch<DD, GG, FF>::run(p, pool_map, s);
     KVG_DECODE_CASES(KVG_CASE)
 #undef KVG_CASE
     return cudaErrorInvalidValue;

@@ -98,6 +98,7 @@ struct AppendParams {
     int32_t *pos_row;          // positions row of the sequence
     int32_t *table_row;        // page_table row
     int32_t *fill_row;         // page_fill row
+    float k_inv_scale, v_inv_scale;  // fp8 caches: 1/scale (fp32) of the quantizing append
     PageList pids;             // pages touched: page0 .. page0 + n - 1
 };
 
@@ -110,6 +111,7 @@ struct AppendBatchParams {
     int64_t pool_pages;
     int32_t n_layers, n_kv_heads, page_size, head_dim, B, max_pages, max_slots;
     int32_t *page_table, *page_fill, *positions;  // whole-cache arrays
+    float k_inv_scale, v_inv_scale;  // fp8 caches: 1/scale (fp32) of the quantizing append
     int32_t seq[kMaxBatchPerLaunch];
     int32_t pid[kMaxBatchPerLaunch];
     int32_t slot[kMaxBatchPerLaunch];
@@ -195,7 +197,8 @@ struct DecodeParams {
     const __nv_bfloat16 *q;    // [Lrun][Btot][Hq][D]
     int32_t q_row_stride_b;    // rows of the full batch (B of the whole call)
     int32_t b0;                // first batch row of this launch
-    float qscale;              // softmax scale * log2(e)
+    float qscale;              // softmax scale * log2(e) (* k_scale for fp8 keys)
+    float vscale;              // 1, or v_scale for fp8 values (applied by the combine)
     float *part_o;             // [U + W][G][D]
     float2 *part_ml;           // [U + W][G]
     __nv_bfloat16 *out;        // [Lrun][Btot][Hq][D] (combine)
@@ -218,6 +221,9 @@ cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s);
 // launch_append().
 int32_t append_tma_rows(int32_t page_size, int32_t head_dim);
 cudaError_t launch_append_tma(const AppendParams &p, DevStatus *status, int n_sm, cudaStream_t s);
+// Appends into an fp8 E4M3 cache: bf16 rows quantized with p.k_inv_scale / p.v_inv_scale.
+cudaError_t launch_append_e4m3(const AppendParams &p, int n_sm, cudaStream_t s);
+cudaError_t launch_append_batch_e4m3(const AppendBatchParams &p, int n_sm, cudaStream_t s);
 // Own-position graft (delta 0) fused with the leaf hashes of the copied pages:
 // leaf_words[(block page) * leaves_per_page + leaf] gets the leaf's state words.
 cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int n_sm, cudaStream_t s);
@@ -250,20 +256,20 @@ cudaError_t launch_sha256_serial(const uint8_t *seg0, uint64_t n0, const uint8_t
 // combine over every (layer, row, query head).  decode_tile_tokens() is the
 // tile height TOK (tiles per page = ceil(P / TOK)); decode_max_warps() the
 // number of co-resident warps the decode kernel can keep on the device.
-cudaError_t launch_decode(int head_dim, int group, const DecodeParams &p, const CUtensorMap &pool_map,
+cudaError_t launch_decode(int head_dim, int group, bool fp8, const DecodeParams &p, const CUtensorMap &pool_map,
                           cudaStream_t s);
 // Tensor map of a cache pool for the decode kernel: a 2-D bf16 tensor of
 // head_dim columns and n_layers*2*n_pages*n_kv_heads*page_size rows, boxes of
 // 64 columns x decode_tile_tokens(head_dim) rows, 128-byte swizzle.
-cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, uint64_t rows);
+cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, bool fp8, uint64_t rows);
 // A rank-`rank` bf16 tensor map (no swizzle, zero fill out of bounds): dims
 // innermost first, byte strides of dims 1.., box extents per dim.
 cudaError_t encode_tensor_map(CUtensorMap *out, int rank, void *base, const cuuint64_t *dims,
                               const cuuint64_t *strides, const cuuint32_t *box);
 cudaError_t launch_combine(int head_dim, int group, const DecodeParams &p, cudaStream_t s);
-bool decode_supported(int head_dim, int group);
+bool decode_supported(int head_dim, int group, bool fp8 = false);
 int decode_tile_tokens(int head_dim);
-int decode_max_warps(int head_dim, int group, int n_sm);
+int decode_max_warps(int head_dim, int group, bool fp8, int n_sm);
 
 // ------------------------------------------------------------ PTX helpers --
 #ifdef __CUDACC__

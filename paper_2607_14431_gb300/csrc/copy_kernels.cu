@@ -333,6 +333,109 @@ __global__ void __launch_bounds__(32) append_tma_kernel(const AppendParams p,
     bulk_wait<0>();
 }
 
+// ---- appends into an fp8 E4M3 cache (quantized KV blocks) ----------------
+// Eight bf16 values -> their E4M3 codes: each value in fp32 times the fp32
+// reciprocal of the scale (one rounding), rounded to nearest-even on the E4M3
+// grid with saturation at +-448 (cvt.rn.satfinite); code i lands in byte i.
+__device__ __forceinline__ uint2 e4m3x8(const uint4 x, float inv_scale) {
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+    uint32_t h[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float lo = __fmul_rn(__uint_as_float(w[i] << 16), inv_scale);
+        const float hi = __fmul_rn(__uint_as_float(w[i] & 0xffff0000u), inv_scale);
+        uint16_t c;
+        asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(c) : "f"(hi), "f"(lo));
+        h[i] = c;
+    }
+    return make_uint2(h[0] | (h[1] << 16), h[2] | (h[3] << 16));
+}
+
+// One warp per (layer, K/V, token) row, like append_kernel; 8 values per lane
+// per step (16 bytes in, 8 bytes out).
+__global__ void __launch_bounds__(kAppendThreads) append_e4m3_kernel(const AppendParams p) {
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+    const int64_t P = p.page_size;
+    append_metadata(p);
+    const int D = p.head_dim;
+    const int gpr = D >> 3;               // 8-value groups per head row
+    const int gpt = p.n_kv_heads * gpr;   // groups per token row
+    const int lane = threadIdx.x & 31;
+    const int64_t rows = (int64_t)p.n_layers * 2 * p.n;
+    for (int64_t r = gtid >> 5; r < rows; r += gsz >> 5) {
+        const int64_t lkv = r / p.n;
+        const int t = (int)(r - lkv * p.n);
+        const int l = (int)(lkv >> 1), kv = (int)(lkv & 1);
+        const float inv = kv ? p.v_inv_scale : p.k_inv_scale;
+        const uint4 *src = reinterpret_cast<const uint4 *>(
+            (kv ? p.v : p.k) + ((int64_t)l * p.n_rows_total + p.row0 + t) * p.n_kv_heads * D);
+        const int64_t s = (int64_t)p.slot0 + t;
+        const int64_t pg = s / P;
+        const int pid = p.pids.pid[pg - p.page0];
+        const int64_t row = s - pg * P;
+        uint2 *dst = reinterpret_cast<uint2 *>(p.pool + (((int64_t)lkv * p.pool_pages + pid) * p.n_kv_heads) * P * D +
+                                               row * D);
+        for (int base = lane; base < gpt; base += 32 * kAppendUnroll) {
+            uint4 val[kAppendUnroll];  // the loads first, kAppendUnroll in flight
+#pragma unroll
+            for (int u = 0; u < kAppendUnroll; ++u)
+                if (base + 32 * u < gpt) val[u] = __ldcs(src + base + 32 * u);
+#pragma unroll
+            for (int u = 0; u < kAppendUnroll; ++u) {
+                const int i = base + 32 * u;
+                if (i < gpt) {
+                    const int h = i / gpr, c = i - h * gpr;
+                    __stcs(dst + h * (P * D / 8) + c, e4m3x8(val[u], inv));
+                }
+            }
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kAppendThreads) append_batch_e4m3_kernel(const AppendBatchParams p) {
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+    const int64_t P = p.page_size;
+    for (int64_t b = gtid; b < p.B; b += gsz) {
+        const int64_t s = p.slot[b];
+        const int64_t pg = s / P;
+        p.positions[(int64_t)p.seq[b] * p.max_slots + s] = p.pos[b];
+        p.page_table[(int64_t)p.seq[b] * p.max_pages + pg] = p.pid[b];
+        p.page_fill[(int64_t)p.seq[b] * p.max_pages + pg] = (int32_t)(s - pg * P + 1);
+    }
+    const int D = p.head_dim;
+    const int gpr = D >> 3;
+    const int gpt = p.n_kv_heads * gpr;
+    const int lane = threadIdx.x & 31;
+    const int64_t rows = (int64_t)p.n_layers * 2 * p.B;
+    for (int64_t r = gtid >> 5; r < rows; r += gsz >> 5) {
+        const int64_t lkv = r / p.B;
+        const int b = (int)(r - lkv * p.B);
+        const int l = (int)(lkv >> 1), kv = (int)(lkv & 1);
+        const float inv = kv ? p.v_inv_scale : p.k_inv_scale;
+        const uint4 *src = reinterpret_cast<const uint4 *>((kv ? p.v : p.k) + ((int64_t)l * p.B + b) * p.n_kv_heads * D);
+        const int64_t s = p.slot[b];
+        const int64_t row = s - (s / P) * P;
+        uint2 *dst = reinterpret_cast<uint2 *>(p.pool + (((int64_t)lkv * p.pool_pages + p.pid[b]) * p.n_kv_heads) * P * D +
+                                               row * D);
+        for (int base = lane; base < gpt; base += 32 * kAppendUnroll) {
+            uint4 val[kAppendUnroll];  // the loads first, kAppendUnroll in flight
+#pragma unroll
+            for (int u = 0; u < kAppendUnroll; ++u)
+                if (base + 32 * u < gpt) val[u] = __ldcs(src + base + 32 * u);
+#pragma unroll
+            for (int u = 0; u < kAppendUnroll; ++u) {
+                const int i = base + 32 * u;
+                if (i < gpt) {
+                    const int h = i / gpr, c = i - h * gpr;
+                    __stcs(dst + h * (P * D / 8) + c, e4m3x8(val[u], inv));
+                }
+            }
+        }
+    }
+}
+
 __global__ void __launch_bounds__(kAppendThreads) append_batch_kernel(const AppendBatchParams p) {
     const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
@@ -369,7 +472,7 @@ __global__ void __launch_bounds__(kAppendThreads) append_batch_kernel(const Appe
 
 __global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
     const int64_t P = p.page_size;
-    const int64_t D = p.head_dim;
+    const int64_t row_bytes = (int64_t)(p.page_bytes / ((uint64_t)p.n_kv_heads * P));
     const int64_t vpp = (int64_t)(p.page_bytes >> 4);
     const int64_t total = (int64_t)p.n_layers * 2 * p.npb * vpp;
     const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -384,7 +487,7 @@ __global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
         const int64_t off = idx - page_u * vpp;
         const int64_t lkv = page_u / p.npb;
         const int64_t jj = page_u - lkv * p.npb;
-        const int64_t row = ((off * 16) / (2 * D)) % P;
+        const int64_t row = ((off * 16) / row_bytes) % P;
         const int64_t tok = (p.page_base + jj) * P + row;
         uint4 val = make_uint4(0, 0, 0, 0);
         if (tok < p.n_tokens) {
@@ -517,6 +620,21 @@ cudaError_t launch_append_tma(const AppendParams &p, DevStatus *status, int n_sm
     const int grid = grid_for(jobs, 1, n_sm, 1);
     append_tma_kernel<<<grid, 32, (size_t)n_stages * stage_bytes, s>>>(p, maps[0], maps[1], status, pbox, n_stages,
                                                                       2000000000ull);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append_e4m3(const AppendParams &p, int n_sm, cudaStream_t s) {
+    const int64_t rows = 2ll * p.n_layers * p.n;  // one warp each
+    static const int ctas_per_sm = env_knob("KVG_APPEND_CTAS_PER_SM", 2);
+    append_e4m3_kernel<<<grid_for(rows, kAppendThreads / 32, n_sm, ctas_per_sm), kAppendThreads, 0, s>>>(p);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append_batch_e4m3(const AppendBatchParams &p, int n_sm, cudaStream_t s) {
+    const int64_t rows = 2ll * p.n_layers * p.B;
+    append_batch_e4m3_kernel<<<grid_for(rows, kAppendThreads / 32, n_sm, 8), kAppendThreads, 0, s>>>(p);
     count_launches(1);
     return cudaGetLastError();
 }

@@ -41,6 +41,8 @@ namespace kvg {
 // Read-only views of a cache's geometry and host bookkeeping (runtime.cu).
 struct CacheShape {
     int32_t n_layers, n_kv_heads, head_dim, page_size, n_pages, max_seqs, max_pages, device, n_sm;
+    int32_t kv_dtype;
+    float k_scale, v_scale;
     uint8_t *pool;
     int32_t *page_table, *page_fill;
     DevStatus *status;
@@ -72,7 +74,8 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
     if (n_q_heads <= 0 || n_q_heads % cs.n_kv_heads)
         return reject(KVG_ERR_ARG, "n_q_heads must be a multiple of n_kv_heads");
     const int G = n_q_heads / cs.n_kv_heads;
-    if (!decode_supported(cs.head_dim, G)) return reject(KVG_ERR_ARG, "unsupported head_dim / group");
+    const bool fp8 = cs.kv_dtype == KVG_KV_E4M3;
+    if (!decode_supported(cs.head_dim, G, fp8)) return reject(KVG_ERR_ARG, "unsupported head_dim / group");
     if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out)) & 15)
         return reject(KVG_ERR_ARG, "q/out must be 16-byte aligned");
     if (cs.device < 0 || cs.device >= kMaxDevices) return reject(KVG_ERR_ARG, "device ordinal out of range");
@@ -121,7 +124,7 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
         }
         scratch = g_scratch_dev[cs.device];
     }
-    const int w_max = decode_max_warps(cs.head_dim, G, cs.n_sm);
+    const int w_max = decode_max_warps(cs.head_dim, G, fp8, cs.n_sm);
     if (w_max <= 0) return reject(KVG_ERR_CUDA, "decode kernel cannot be made resident");
     const int64_t w_cap = cap_slots - units < w_max ? cap_slots - units : w_max;
     const size_t slots = (size_t)units + (size_t)w_cap;
@@ -134,11 +137,12 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
         p.n_q_heads = n_q_heads;
         p.q = static_cast<const __nv_bfloat16 *>(q);
         p.q_row_stride_b = B;
-        p.qscale = scale * 1.4426950408889634f;
+        p.qscale = scale * 1.4426950408889634f * (fp8 ? cs.k_scale : 1.f);
+        p.vscale = fp8 ? cs.v_scale : 1.f;
         p.part_o = part_o;
         p.part_ml = part_ml;
         p.out = static_cast<__nv_bfloat16 *>(out);
-        cudaError_t e = launch_decode(cs.head_dim, G, p, *cs.pool_map, st);
+        cudaError_t e = launch_decode(cs.head_dim, G, fp8, p, *cs.pool_map, st);
         if (e != cudaSuccess) return reject(KVG_ERR_CUDA, std::string("decode launch: ") + cudaGetErrorString(e));
         e = launch_combine(cs.head_dim, G, p, st);
         if (e != cudaSuccess) return reject(KVG_ERR_CUDA, std::string("combine launch: ") + cudaGetErrorString(e));

@@ -91,20 +91,28 @@ int sm_count(int dev) {
     return n;
 }
 
+int elem_bytes(const kvg_dims &d) { return d.kv_dtype == KVG_KV_E4M3 ? 1 : 2; }
+
 bool dims_valid(const kvg_dims &d) {
     if (d.n_layers <= 0 || d.n_kv_heads <= 0 || d.page_size <= 0) return false;
     if (d.head_dim != 64 && d.head_dim != 128 && d.head_dim != 256) return false;
     if (d.rope_style != KVG_ROPE_HALF && d.rope_style != KVG_ROPE_INTERLEAVED) return false;
-    const uint64_t pb = 2ull * d.n_kv_heads * d.page_size * d.head_dim;
+    if (d.kv_dtype != KVG_KV_BF16 && d.kv_dtype != KVG_KV_E4M3) return false;
+    if (d.kv_dtype == KVG_KV_E4M3 && !(std::isfinite(d.k_scale) && d.k_scale > 0.f && std::isfinite(d.v_scale) &&
+                                       d.v_scale > 0.f))
+        return false;
+    const uint64_t pb = (uint64_t)elem_bytes(d) * d.n_kv_heads * d.page_size * d.head_dim;
     return pb % 16 == 0 && pb <= (1ull << 31);
 }
 
 bool same_geometry(const kvg_dims &a, const kvg_dims &b) {
+    if (a.kv_dtype != b.kv_dtype) return false;
+    if (a.kv_dtype == KVG_KV_E4M3 && (a.k_scale != b.k_scale || a.v_scale != b.v_scale)) return false;
     return a.n_layers == b.n_layers && a.n_kv_heads == b.n_kv_heads && a.head_dim == b.head_dim &&
            a.page_size == b.page_size;
 }
 
-uint64_t page_bytes_of(const kvg_dims &d) { return 2ull * d.n_kv_heads * d.page_size * d.head_dim; }
+uint64_t page_bytes_of(const kvg_dims &d) { return (uint64_t)elem_bytes(d) * d.n_kv_heads * d.page_size * d.head_dim; }
 
 struct BlockLayout {
     int64_t n_tokens, n_pages;
@@ -140,17 +148,21 @@ void build_header(uint8_t h[256], const kvg_dims &d, const BlockLayout &b) {
     i64 = b.n_pages; memcpy(h + 40, &i64, 8);
     f64 = d.rope_theta; memcpy(h + 48, &f64, 8);
     i32 = d.rope_style; memcpy(h + 56, &i32, 4);
-    i32 = 1; memcpy(h + 60, &i32, 4);
+    i32 = d.kv_dtype == KVG_KV_E4M3 ? 2 : 1; memcpy(h + 60, &i32, 4);  // block dtype code
     u64 = b.pos_off; memcpy(h + 64, &u64, 8);
     u64 = b.dig_off; memcpy(h + 72, &u64, 8);
     u64 = b.pages_off; memcpy(h + 80, &u64, 8);
     u64 = b.total; memcpy(h + 88, &u64, 8);
+    if (d.kv_dtype == KVG_KV_E4M3) {  // per-tensor scales (the digest is written at 96..127 later)
+        memcpy(h + 128, &d.k_scale, 4);
+        memcpy(h + 132, &d.v_scale, 4);
+    }
 }
 
 // Chunk of a page that one CTA copies: <= 64 KiB, divides the page, whole rows.
 int32_t copy_chunk_bytes(const kvg_dims &d) {
     uint64_t c = page_bytes_of(d);
-    const uint64_t row = 2ull * d.head_dim;
+    const uint64_t row = (uint64_t)elem_bytes(d) * d.head_dim;
     while (c > 65536 && c % 2 == 0 && (c / 2) % row == 0 && (c / 2) % 16 == 0) c /= 2;
     return (int32_t)c;
 }
@@ -384,9 +396,16 @@ extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t
     memcpy(&pgo, h + 80, 8);
     memcpy(&tot, h + 88, 8);
     const kvg_dims &d = s->dims;
-    if (ver != 1 || hb != 256 || dtype != 1) return fail(KVG_ERR_FORMAT, "unsupported version/dtype");
+    if (ver != 1 || hb != 256 || (dtype != 1 && dtype != 2)) return fail(KVG_ERR_FORMAT, "unsupported version/dtype");
     if (L != d.n_layers || Hkv != d.n_kv_heads || D != d.head_dim || P != d.page_size)
         return fail(KVG_ERR_FORMAT, "geometry differs from the store's");
+    if (dtype != (d.kv_dtype == KVG_KV_E4M3 ? 2 : 1)) return fail(KVG_ERR_FORMAT, "element type differs from the store's");
+    if (dtype == 2) {
+        float ks, vs;
+        memcpy(&ks, h + 128, 4);
+        memcpy(&vs, h + 132, 4);
+        if (ks != d.k_scale || vs != d.v_scale) return fail(KVG_ERR_FORMAT, "fp8 scales differ from the store's");
+    }
     if (n_tok <= 0 || n_tok > (1ll << 31)) return fail(KVG_ERR_FORMAT, "bad n_tokens");
     const BlockLayout lay = layout_for(d, n_tok);
     if (n_pg != lay.n_pages || po != lay.pos_off || dof != lay.dig_off || pgo != lay.pages_off ||
@@ -687,7 +706,8 @@ extern "C" kvg_status kvg_cache_create(const kvg_dims *dims, int32_t n_pages, in
     if (pool_rows > 0x7fffffffull)
         return cleanup(fail(KVG_ERR_ARG, "pool of %llu rows exceeds the decode kernel's 2^31-row addressing",
                             (unsigned long long)pool_rows));
-    if (make_pool_tensor_map(&c->pool_map, c->pool, dims->head_dim, pool_rows) != cudaSuccess)
+    if (make_pool_tensor_map(&c->pool_map, c->pool, dims->head_dim, dims->kv_dtype == KVG_KV_E4M3, pool_rows) !=
+        cudaSuccess)
         return cleanup(fail(KVG_ERR_CUDA, "tensor map of the pool could not be encoded"));
     for (int32_t i = 0; i < n_pages; ++i) c->free_list.push_back(i);
     c->pinned.assign(n_pages, 0);
@@ -821,10 +841,17 @@ extern "C" kvg_status kvg_cache_append(kvg_cache *c, int32_t seq, const void *k,
         p.pids.n = (int32_t)(last - p.page0 + 1);
         for (int32_t i = 0; i < p.pids.n; ++i) p.pids.pid[i] = sp[p.page0 + i];
         // long appends move rows with tensor copies; short ones (a box would
-        // mostly carry rows that are not stored) with a warp per row
+        // mostly carry rows that are not stored) with a warp per row; an fp8
+        // cache quantizes each row on the way
         cudaError_t e = cudaErrorNotSupported;
-        if (nr >= append_tma_rows(p.page_size, p.head_dim)) e = launch_append_tma(p, c->status, c->n_sm, st);
-        if (e == cudaErrorNotSupported) e = launch_append(p, c->n_sm, st);
+        if (c->dims.kv_dtype == KVG_KV_E4M3) {
+            p.k_inv_scale = 1.0f / c->dims.k_scale;
+            p.v_inv_scale = 1.0f / c->dims.v_scale;
+            e = launch_append_e4m3(p, c->n_sm, st);
+        } else {
+            if (nr >= append_tma_rows(p.page_size, p.head_dim)) e = launch_append_tma(p, c->status, c->n_sm, st);
+            if (e == cudaErrorNotSupported) e = launch_append(p, c->n_sm, st);
+        }
         KVG_CUDA(e);
     }
     c->n_slots[seq] = (int32_t)(s0 + n);
@@ -882,7 +909,13 @@ extern "C" kvg_status kvg_cache_append_batch(kvg_cache *c, const int32_t *seq_id
         c->n_slots[sq] = (int32_t)(s + 1);
         note_fills(c, sq, s, s + 1);
     }
-    KVG_CUDA(launch_append_batch(p, c->n_sm, static_cast<cudaStream_t>(stream)));
+    if (c->dims.kv_dtype == KVG_KV_E4M3) {
+        p.k_inv_scale = 1.0f / c->dims.k_scale;
+        p.v_inv_scale = 1.0f / c->dims.v_scale;
+        KVG_CUDA(launch_append_batch_e4m3(p, c->n_sm, static_cast<cudaStream_t>(stream)));
+    } else {
+        KVG_CUDA(launch_append_batch(p, c->n_sm, static_cast<cudaStream_t>(stream)));
+    }
     return KVG_OK;
 }
 
@@ -1162,6 +1195,7 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
     if (!s->pool_cache && npb > (int64_t)c->free_list.size()) return fail(KVG_ERR_CAPACITY, "out of free pages");
     if (blk.min_pos + delta < 0 || blk.max_pos + delta >= (1ll << 31))
         return fail(KVG_ERR_POSITION, "position tags + delta leave [0, 2^31)");
+    if (delta != 0 && c->dims.kv_dtype != KVG_KV_BF16) return fail(KVG_ERR_ARG, "relocation needs a bf16 cache");
     DeviceGuard g(c->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (s->pool_cache) return pool_graft(s, blk, c, seq, dst, delta, flags, st, report);
@@ -1393,14 +1427,16 @@ extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const in
     if (B <= 0 || B > 4096) return fail(KVG_ERR_ARG, "B must be in [1, 4096]");
     if (n_q_heads <= 0 || n_q_heads % d.n_kv_heads) return fail(KVG_ERR_ARG, "n_q_heads must be a multiple of n_kv_heads");
     const int G = n_q_heads / d.n_kv_heads;
-    if (!decode_supported(d.head_dim, G)) return fail(KVG_ERR_ARG, "unsupported head_dim %d / group %d", d.head_dim, G);
+    const bool fp8 = d.kv_dtype == KVG_KV_E4M3;
+    if (!decode_supported(d.head_dim, G, fp8))
+        return fail(KVG_ERR_ARG, "unsupported head_dim %d / group %d%s", d.head_dim, G, fp8 ? " (fp8)" : "");
     if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out)) & 15)
         return fail(KVG_ERR_ARG, "q/out must be 16-byte aligned");
     for (int32_t b = 0; b < B; ++b)
         if (seq_ids[b] < 0 || seq_ids[b] >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq id %d", seq_ids[b]);
     DeviceGuard g(c->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const int w_max = decode_max_warps(d.head_dim, G, c->n_sm);
+    const int w_max = decode_max_warps(d.head_dim, G, fp8, c->n_sm);
     if (w_max <= 0) return fail(KVG_ERR_CUDA, "decode kernel cannot be made resident");
     std::vector<DecodeParams> plan;
     int64_t max_units = 0;
@@ -1414,11 +1450,12 @@ extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const in
         p.n_q_heads = n_q_heads;
         p.q = static_cast<const __nv_bfloat16 *>(q);
         p.q_row_stride_b = B;
-        p.qscale = scale * 1.4426950408889634f;
+        p.qscale = scale * 1.4426950408889634f * (fp8 ? d.k_scale : 1.f);
+        p.vscale = fp8 ? d.v_scale : 1.f;
         p.part_o = static_cast<float *>(c->part_o.ptr);
         p.part_ml = static_cast<float2 *>(c->part_ml.ptr);
         p.out = static_cast<__nv_bfloat16 *>(out);
-        KVG_CUDA(launch_decode(d.head_dim, G, p, c->pool_map, st));
+        KVG_CUDA(launch_decode(d.head_dim, G, fp8, p, c->pool_map, st));
         KVG_CUDA(launch_combine(d.head_dim, G, p, st));
     }
     return KVG_OK;
@@ -1514,6 +1551,8 @@ namespace kvg {
 // Read-only views used by noalloc.cu.
 struct CacheShape {
     int32_t n_layers, n_kv_heads, head_dim, page_size, n_pages, max_seqs, max_pages, device, n_sm;
+    int32_t kv_dtype;
+    float k_scale, v_scale;
     uint8_t *pool;
     int32_t *page_table, *page_fill;
     DevStatus *status;
@@ -1522,8 +1561,8 @@ struct CacheShape {
 bool cache_shape(const kvg_cache *c, CacheShape *out) {
     if (!c || !out) return false;
     *out = CacheShape{c->dims.n_layers, c->dims.n_kv_heads, c->dims.head_dim, c->dims.page_size, c->n_pages,
-                      c->max_seqs, c->max_pages, c->device, c->n_sm, c->pool, c->page_table, c->page_fill,
-                      c->status, &c->pool_map};
+                      c->max_seqs, c->max_pages, c->device, c->n_sm, c->dims.kv_dtype, c->dims.k_scale,
+                      c->dims.v_scale, c->pool, c->page_table, c->page_fill, c->status, &c->pool_map};
     return true;
 }
 int32_t cache_seq_pages(const kvg_cache *c, int32_t seq) { return (int32_t)c->seq_pages[seq].size(); }
@@ -1534,6 +1573,6 @@ kvg_status cache_plan_decode(const kvg_cache *c, int32_t layer, const int32_t *s
 void set_last_error(const char *msg) { g_last_error = msg; }
 }  // namespace kvg
 
-extern "C" uint32_t kvg_version(void) { return 0x000100u; }
+extern "C" uint32_t kvg_version(void) { return 0x000200u; }
 
 extern "C" uint64_t kvg_launch_count(void) { return kvg::launch_count(); }

@@ -24,6 +24,7 @@ KVG_RESIDENCY_HBM, KVG_RESIDENCY_PINNED_HOST, KVG_RESIDENCY_CACHE_POOL = 0, 1, 2
 KVG_ROPE_HALF, KVG_ROPE_INTERLEAVED = 0, 1
 KVG_GRAFT_VERIFY, KVG_GRAFT_SYNC = 1, 2
 KVG_SHA256_PLAIN, KVG_SHA256_PAGED = 0, 1
+KVG_KV_BF16, KVG_KV_E4M3 = 0, 1
 KVG_REPORT_MAX_PAGES = 64
 
 
@@ -37,7 +38,7 @@ class kvg_dims(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("page_size", ctypes.c_int32),
                 ("rope_theta", ctypes.c_double), ("rope_style", ctypes.c_int32),
-                ("reserved", ctypes.c_int32)]
+                ("kv_dtype", ctypes.c_int32), ("k_scale", ctypes.c_float), ("v_scale", ctypes.c_float)]
 
 
 class kvg_block_info(ctypes.Structure):
@@ -135,8 +136,10 @@ def _stream(stream) -> int:
     return int(getattr(stream, "cuda_stream", stream))
 
 
-def make_dims(n_layers, n_kv_heads, head_dim, page_size, rope_theta=10000.0, rope_style=0) -> kvg_dims:
-    return kvg_dims(n_layers, n_kv_heads, head_dim, page_size, float(rope_theta), rope_style, 0)
+def make_dims(n_layers, n_kv_heads, head_dim, page_size, rope_theta=10000.0, rope_style=0,
+              kv_dtype=KVG_KV_BF16, k_scale=1.0, v_scale=1.0) -> kvg_dims:
+    return kvg_dims(n_layers, n_kv_heads, head_dim, page_size, float(rope_theta), rope_style, kv_dtype,
+                    float(k_scale), float(v_scale))
 
 
 # ---- thin wrappers, same names as the C ABI ---------------------------------

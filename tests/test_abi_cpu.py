@@ -42,9 +42,19 @@ def test_host_checks_reject_bad_geometry_without_a_gpu(lib):
     assert lib.kvg_decode_attention(None, 0, None, 1, None, 4, None, ctypes.c_float(1.0), None) == kvg.KVG_ERR_ARG
 
 
+def test_host_checks_reject_bad_fp8_dims_without_a_gpu(lib):
+    h = ctypes.c_void_p()
+    for ks, vs, dt in [(0.0, 1.0, kvg.KVG_KV_E4M3), (1.0, float("inf"), kvg.KVG_KV_E4M3),
+                       (-0.5, 1.0, kvg.KVG_KV_E4M3), (1.0, 1.0, 7)]:
+        bad = kvg.make_dims(2, 2, 128, 16, kv_dtype=dt, k_scale=ks, v_scale=vs)
+        assert lib.kvg_store_create(ctypes.byref(bad), 0, 1 << 20, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
+        assert lib.kvg_cache_create(ctypes.byref(bad), 4, 1, 64, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
+
+
 def test_struct_layouts_match_header():
     # field offsets the C side relies on
-    assert ctypes.sizeof(kvg.kvg_dims) == 32
+    assert ctypes.sizeof(kvg.kvg_dims) == 40
+    assert (kvg.kvg_dims.kv_dtype.offset, kvg.kvg_dims.k_scale.offset, kvg.kvg_dims.v_scale.offset) == (28, 32, 36)
     assert kvg.kvg_block_info.block_digest.offset == 64
     assert ctypes.sizeof(kvg.kvg_graft_report) == 16 + 4 * kvg.KVG_REPORT_MAX_PAGES
     assert ctypes.sizeof(kvg.kvg_cache_view) == 4 * 8 + 2 * 8 + 4 * 4

@@ -528,3 +528,94 @@ def test_window_settings_are_checked(oracle):
         c.set_layer_windows([1])
     with pytest.raises(oracle.KvgError):
         c.set_layer_windows([-1, 0])
+
+
+# --------------------------------------------------------------------------
+# Quantized KV: fp8 E4M3 codes with per-tensor scales
+# --------------------------------------------------------------------------
+
+def test_e4m3_code_values_match_torch(oracle):
+    codes = np.arange(256, dtype=np.uint8)
+    ours = oracle.e4m3_to_f64(codes)
+    ref = torch.from_numpy(codes.copy()).view(torch.float8_e4m3fn).to(torch.float64).numpy()
+    nan = np.isnan(ref)
+    assert (np.isnan(ours) == nan).all() and nan.sum() == 2  # 0x7F, 0xFF
+    assert np.array_equal(ours[~nan], ref[~nan])
+    assert ours[0x7E] == 448.0 and ours[0x01] == 2.0 ** -9 and ours[0x08] == 2.0 ** -6
+
+
+def test_e4m3_rounding_matches_torch_on_every_bf16_in_range(oracle):
+    bits = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    x = oracle.bf16_to_f64(bits)
+    keep = np.isfinite(x) & (np.abs(x) <= 448.0)
+    x = x[keep]
+    ours = oracle.e4m3_rne(x)
+    ref = torch.from_numpy(x.astype(np.float32)).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    assert np.array_equal(ours, ref)
+
+
+def test_e4m3_saturates_and_keeps_nan(oracle):
+    got = oracle.e4m3_rne(np.array([448.0, 449.0, 464.0, 1e6, -1e6, -500.0, np.nan, 0.0, -0.0]))
+    assert list(got) == [0x7E, 0x7E, 0x7E, 0x7E, 0xFE, 0xFE, 0x7F, 0x00, 0x80]
+
+
+@pytest.mark.parametrize("scale", [0.0625, 0.037, 3.3])
+def test_e4m3_quantize_multiplies_by_the_fp32_reciprocal(oracle, scale):
+    rng = np.random.default_rng(7)
+    x = syn.as_u16(torch.from_numpy(rng.standard_normal(20000).astype(np.float32) * 4).to(torch.bfloat16))
+    q = oracle.e4m3_quantize(x, scale)
+    xf = torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).float()
+    r = torch.tensor(1.0, dtype=torch.float32) / torch.tensor(scale, dtype=torch.float32)
+    y = xf * r
+    ok = (y.abs() <= 448).numpy()
+    ref = y.to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    assert np.array_equal(q[ok], ref[ok])
+    assert (q[~ok] & 0x7F == 0x7E).all()
+
+
+def _fp8_dims(scale_k=0.125, scale_v=0.25):
+    import oracle as o
+    w = syn.TINY
+    return o.Dims(w.n_layers, w.n_kv_heads, w.head_dim, w.page_size, w.rope_theta, 0, o.KV_E4M3, scale_k, scale_v)
+
+
+def test_fp8_block_layout_and_header(oracle):
+    d = _fp8_dims()
+    n = 40
+    k, v = _kv(n, 31)
+    blk = oracle.block_from_kv(d, k, v, syn.positions(0, n))
+    assert blk.pages.dtype == np.uint8 and d.page_bytes == d.page_elems
+    assert np.array_equal(blk.pages[1, 0, 2, 1, 3], oracle.e4m3_quantize(k[1, 2 * 16 + 3, 1], 0.125))
+    assert np.array_equal(blk.pages[0, 1, 0, 0, 5], oracle.e4m3_quantize(v[0, 5, 0], 0.25))
+    ser = blk.serialize()
+    f = struct.unpack_from("<8sIIiiiiqqdiiQQQQ", ser, 0)
+    assert f[11] == 2 and struct.unpack_from("<ff", ser, 128) == (0.125, 0.25)
+    assert len(ser) - f[14] == blk.pages.size  # one byte per element
+    for l in range(d.L):
+        for kv in range(2):
+            for j in range(blk.n_pages):
+                assert blk.digests[l, kv, j].tobytes() == _two_level_hashlib(blk.pages[l, kv, j].tobytes())
+
+
+def test_fp8_decode_equals_bf16_decode_over_the_dequantized_rows(oracle):
+    """With power-of-two scales every dequantized element is exactly a bf16
+    value, so the fp8 cache's attention must equal the bf16 cache's attention
+    over those values, in fp64, bit for bit."""
+    import oracle as o
+    d8 = _fp8_dims(0.125, 0.5)
+    w = syn.TINY
+    d16 = o.Dims(w.n_layers, w.n_kv_heads, w.head_dim, w.page_size, w.rope_theta, 0)
+    n = 70
+    k, v = _kv(n, 33)
+    c8 = o.OracleCache(d8, 12, 1, 128)
+    c8.append(0, k, v, syn.positions(0, n))
+    kq = oracle.bf16_rne(oracle.e4m3_dequant(oracle.e4m3_quantize(k, 0.125), 0.125))
+    vq = oracle.bf16_rne(oracle.e4m3_dequant(oracle.e4m3_quantize(v, 0.5), 0.5))
+    assert np.array_equal(oracle.bf16_to_f64(kq), oracle.e4m3_dequant(oracle.e4m3_quantize(k, 0.125), 0.125))
+    c16 = o.OracleCache(d16, 12, 1, 128)
+    c16.append(0, kq, vq, syn.positions(0, n))
+    q = syn.as_u16(syn.queries(w, 2, 1, 34))[:, 0]
+    for l in range(2):
+        assert c8.decode(0, l, q[l], 0.125).tobytes() == c16.decode(0, l, q[l], 0.125).tobytes()
+    with pytest.raises(o.KvgError):
+        c8.graft(0, c8.deposit(0, 0, 32), delta=5)
