@@ -312,6 +312,23 @@ kvg_status kvg_graft(kvg_store *store, uint64_t block_id, kvg_cache *cache, int3
                      int32_t dst_slot, int64_t delta, uint32_t flags, void *stream,
                      kvg_graft_report *report);
 
+/* A batch of own-position grafts (Sec. 3.2) in one call: graft i installs
+ * block block_ids[i] into sequence seq_ids[i] at that sequence's next page
+ * boundary, in order, exactly as n kvg_graft(delta = 0) calls would (a
+ * sequence may appear several times: its blocks land one after another,
+ * each page-aligned).  The page copies of all grafts run as one launch, so
+ * the GPU stays full across graft boundaries.  block_ids, seq_ids: host
+ * arrays of n (1 <= n <= 4096); each block at most 1,024 pages per (layer,
+ * K/V).  Every argument, capacity and page count is checked first: on an
+ * error nothing is grafted.  Not for pool-resident stores (KVG_ERR_ARG; use
+ * kvg_graft).  flags as for kvg_graft: KVG_GRAFT_VERIFY hashes each graft's
+ * restored pages after the copies; the report's seq is the (last) failing
+ * graft's sequence and mismatch_pages its block page indices.  The call
+ * stages its job table in library-owned pinned memory and waits for the
+ * previous batch's table copy on this cache before reusing it. */
+kvg_status kvg_graft_batch(kvg_store *store, const uint64_t *block_ids, kvg_cache *cache, const int32_t *seq_ids,
+                           int32_t n, uint32_t flags, void *stream, kvg_graft_report *report);
+
 /* Re-checks a grafted range: hashes the cache pages that hold slots
  * [slot0, slot0 + n_tokens(block)) of `seq` (slot0 page-aligned) on the GPU
  * and compares each page digest with block `block_id`'s stored digest

@@ -83,6 +83,36 @@ __device__ __forceinline__ void graft_metadata(const GraftParams &p) {
     }
 }
 
+// ------------------------------------------------------------ graft batch --
+// One block page of a batched graft: its plane-0 bytes in the store, the
+// stride between its (layer, K/V) planes in pages, and its cache page id.
+struct GraftJob {
+    const uint8_t *src;
+    int32_t block_pages;
+    int32_t pid;
+};
+// One graft of a batch: position tags, page-table row and fill row of its
+// destination, and its jobs [first_job, first_job + npb).
+struct GraftMeta {
+    const int32_t *src_pos;
+    int32_t *dst_pos;
+    int32_t *table_row;
+    int32_t *fill_row;
+    int64_t n_tokens;
+    int32_t npb;
+    int32_t first_job;
+};
+struct GraftBatchParams {
+    const GraftJob *jobs;
+    const GraftMeta *metas;
+    int64_t n_jobs;
+    int32_t n_grafts;
+    int32_t n_layers, page_size, chunk_bytes;
+    uint64_t page_bytes;
+    int64_t pool_pages;
+    uint8_t *pool;
+};
+
 // ---------------------------------------------------------------- append --
 struct AppendParams {
     const uint16_t *k, *v;     // [L][n][Hkv][D]
@@ -215,6 +245,8 @@ uint64_t launch_count();
 int env_knob(const char *name, int fallback);
 
 cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s);
+// Own-position copies of a batch of grafts in one launch (jobs, metas in device memory).
+cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s);
 // Bulk append by tensor copies, for appends of at least append_tma_rows()
 // rows (16-byte aligned k/v).  Returns cudaErrorNotSupported (nothing
 // launched) when the tensor maps cannot be encoded, so the caller can take

@@ -556,6 +556,46 @@ int grid_for(int64_t work_items, int per_block, int n_sm, int waves) {
 
 }  // namespace
 
+// A batch of own-position grafts in one launch: every block page of every
+// graft is a job; a unit is a chunk of one (job, layer, K/V) page, so the
+// batch keeps every SM busy to its end instead of draining after each graft.
+__global__ void __launch_bounds__(kCopyThreads) graft_batch_kernel(const GraftBatchParams p) {
+    const uint64_t page_bytes = p.page_bytes;
+    const int64_t cpp = (int64_t)(page_bytes / (uint64_t)p.chunk_bytes);
+    const int64_t per_job = (int64_t)p.n_layers * 2 * cpp;
+    const int64_t n_units = p.n_jobs * per_job;
+    for (int64_t unit = blockIdx.x; unit < n_units; unit += gridDim.x) {
+        const int64_t jb = unit / per_job;
+        const int64_t rem = unit - jb * per_job;
+        const int64_t lkv = rem / cpp;
+        const uint64_t off = (uint64_t)(rem - lkv * cpp) * (uint64_t)p.chunk_bytes;
+        const GraftJob job = p.jobs[jb];
+        const uint8_t *src = job.src + (uint64_t)lkv * job.block_pages * page_bytes + off;
+        uint8_t *dst = p.pool + ((uint64_t)lkv * p.pool_pages + (uint64_t)job.pid) * page_bytes + off;
+        copy_chunk(dst, src, p.chunk_bytes);
+    }
+    // metadata last: the copies start at once and this fills the tail wave
+    const int64_t P = p.page_size;
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
+    for (int32_t g = 0; g < p.n_grafts; ++g) {
+        const GraftMeta m = p.metas[g];
+        for (int64_t t = gtid; t < m.n_tokens; t += gsz) m.dst_pos[t] = m.src_pos[t];
+        for (int64_t j = gtid; j < m.npb; j += gsz) {
+            m.table_row[j] = p.jobs[m.first_job + j].pid;
+            const int64_t f = m.n_tokens - j * P;
+            m.fill_row[j] = (int32_t)(f < P ? f : P);
+        }
+    }
+}
+
+cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s) {
+    const int64_t units = p.n_jobs * p.n_layers * 2 * (int64_t)(p.page_bytes / p.chunk_bytes);
+    graft_batch_kernel<<<grid_for(units, 1, n_sm, 4), kCopyThreads, 0, s>>>(p);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s) {
     const int64_t units = (int64_t)p.n_layers * 2 * p.npb * (int64_t)(p.page_bytes / p.chunk_bytes);
     const int grid = grid_for(units, 1, n_sm, 4);

@@ -16,6 +16,7 @@
 #include <deque>
 #include <mutex>
 #include <string>
+#include <unordered_map>
 #include <thread>
 #include <vector>
 
@@ -506,6 +507,7 @@ extern "C" kvg_status kvg_store_load(kvg_store *s, const char *path, uint32_t fl
 // ------------------------------------------------------------------- cache --
 
 constexpr int kHostVerifyChunks = 8;  // page-range chunks of a verified host-store graft
+constexpr int32_t kMaxGraftsPerBatch = 4096;
 
 struct kvg_cache {
     kvg_dims dims;
@@ -526,6 +528,12 @@ struct kvg_cache {
     // the next pages still cross the host link (made on first use)
     cudaStream_t aux = nullptr;
     cudaEvent_t aux_ev[kHostVerifyChunks + 1] = {};
+    // kvg_graft_batch's job table: staged in pinned host memory, copied to
+    // batch_dev on the call's stream; batch_ev marks when the copy has read it
+    Scratch batch_dev;
+    uint8_t *batch_host = nullptr;
+    size_t batch_host_cap = 0;
+    cudaEvent_t batch_ev = nullptr;
     std::vector<uint8_t> pinned;  // per page: owned by a pool-resident store block
     std::vector<int32_t> alias;   // per pinned page: sequences whose page tables point at it
 };
@@ -728,6 +736,9 @@ extern "C" void kvg_cache_destroy(kvg_cache *c) {
     for (cudaEvent_t &e : c->aux_ev)
         if (e) cudaEventDestroy(e);
     if (c->aux) cudaStreamDestroy(c->aux);
+    if (c->batch_ev) cudaEventDestroy(c->batch_ev);
+    if (c->batch_host) cudaFreeHost(c->batch_host);
+    c->batch_dev.release();
     if (c->pool) cudaFree(c->pool);
     if (c->page_table) cudaFree(c->page_table);
     if (c->page_fill) cudaFree(c->page_fill);
@@ -1292,6 +1303,100 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
     }
     return finish_verify(c, seq, flags, (flags & KVG_GRAFT_VERIFY) ? (int32_t)(c->dims.n_layers * 2 * npb) : 0,
                          st, report);
+}
+
+extern "C" kvg_status kvg_graft_batch(kvg_store *s, const uint64_t *block_ids, kvg_cache *c, const int32_t *seq_ids,
+                                      int32_t n, uint32_t flags, void *stream, kvg_graft_report *report) {
+    Trace trace_("kvg_graft_batch");
+    if (!s || !c || !block_ids || !seq_ids) return fail(KVG_ERR_ARG, "null argument");
+    if (n <= 0 || n > kMaxGraftsPerBatch) return fail(KVG_ERR_ARG, "n must be in [1, %d]", kMaxGraftsPerBatch);
+    if (!same_geometry(s->dims, c->dims)) return fail(KVG_ERR_ARG, "store and cache geometry differ");
+    if (s->device != c->device) return fail(KVG_ERR_ARG, "store and cache on different devices");
+    if (s->pool_cache) return fail(KVG_ERR_ARG, "a pool-resident store grafts with kvg_graft (aliasing)");
+    if (flags & ~(uint32_t)(KVG_GRAFT_VERIFY | KVG_GRAFT_SYNC)) return fail(KVG_ERR_ARG, "unknown flags");
+    const int64_t P = c->dims.page_size;
+    // every check before any state changes: the batch happens whole or not at all
+    std::unordered_map<int32_t, int64_t> slots;
+    int64_t pages = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t seq = seq_ids[i];
+        if (seq < 0 || seq >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq %d (graft %d)", seq, i);
+        if (block_ids[i] >= s->blocks.size())
+            return fail(KVG_ERR_NOT_FOUND, "no block %llu (graft %d)", (unsigned long long)block_ids[i], i);
+        const auto &blk = s->blocks[block_ids[i]];
+        auto it = slots.emplace(seq, (int64_t)c->n_slots[seq]).first;
+        const int64_t dst = (it->second + P - 1) / P * P;
+        if (dst + blk.lay.n_tokens > c->max_slots) return fail(KVG_ERR_CAPACITY, "graft %d past max_slots", i);
+        if (blk.lay.n_pages > kMaxPagesPerLaunch) return fail(KVG_ERR_ARG, "graft %d: block too long for a batch", i);
+        it->second = dst + blk.lay.n_tokens;
+        pages += blk.lay.n_pages;
+    }
+    if (pages > (int64_t)c->free_list.size()) return fail(KVG_ERR_CAPACITY, "out of free pages");
+    DeviceGuard g(c->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // the job table: metas then jobs, in pinned host memory
+    const size_t meta_bytes = (size_t)n * sizeof(GraftMeta);
+    const size_t bytes = meta_bytes + (size_t)pages * sizeof(GraftJob);
+    if (!c->batch_ev) KVG_CUDA(cudaEventCreateWithFlags(&c->batch_ev, cudaEventDisableTiming));
+    KVG_CUDA(cudaEventSynchronize(c->batch_ev));  // the previous batch's copy has read the staging
+    if (bytes > c->batch_host_cap) {
+        if (c->batch_host) cudaFreeHost(c->batch_host);
+        c->batch_host = nullptr;
+        c->batch_host_cap = 0;
+        const size_t want = std::max(bytes, (size_t)1 << 16);
+        KVG_CUDA(cudaHostAlloc(reinterpret_cast<void **>(&c->batch_host), want, cudaHostAllocDefault));
+        c->batch_host_cap = want;
+    }
+    KVG_CUDA(c->batch_dev.ensure(bytes));
+    GraftMeta *metas = reinterpret_cast<GraftMeta *>(c->batch_host);
+    GraftJob *jobs = reinterpret_cast<GraftJob *>(c->batch_host + meta_bytes);
+    std::vector<std::pair<int32_t, int64_t>> verify_at;  // (seq, first page index) per graft
+    int32_t job = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t seq = seq_ids[i];
+        const auto &blk = s->blocks[block_ids[i]];
+        const int64_t nt = blk.lay.n_tokens, npb = blk.lay.n_pages;
+        const int64_t dst = (c->n_slots[seq] + P - 1) / P * P;
+        auto pids = take_pages(c, npb);
+        auto &sp = c->seq_pages[seq];
+        const int64_t jdst = dst / P;
+        sp.insert(sp.end(), pids.begin(), pids.end());
+        c->n_slots[seq] = (int32_t)(dst + nt);
+        note_fills(c, seq, dst, dst + nt);
+        GraftMeta &m = metas[i];
+        m.src_pos = reinterpret_cast<const int32_t *>(blk.dev + blk.lay.pos_off);
+        m.dst_pos = c->positions + (int64_t)seq * c->max_slots + dst;
+        m.table_row = c->page_table + (int64_t)seq * c->max_pages + jdst;
+        m.fill_row = c->page_fill + (int64_t)seq * c->max_pages + jdst;
+        m.n_tokens = nt;
+        m.npb = (int32_t)npb;
+        m.first_job = job;
+        for (int64_t j = 0; j < npb; ++j, ++job)
+            jobs[job] = GraftJob{blk.dev + blk.lay.pages_off + (uint64_t)j * c->page_bytes, (int32_t)npb, pids[j]};
+        verify_at.push_back({seq, jdst});
+    }
+    KVG_CUDA(cudaMemcpyAsync(c->batch_dev.ptr, c->batch_host, bytes, cudaMemcpyHostToDevice, st));
+    KVG_CUDA(cudaEventRecord(c->batch_ev, st));
+    GraftBatchParams p{};
+    p.metas = static_cast<const GraftMeta *>(c->batch_dev.ptr);
+    p.jobs = reinterpret_cast<const GraftJob *>(static_cast<uint8_t *>(c->batch_dev.ptr) + meta_bytes);
+    p.n_jobs = pages;
+    p.n_grafts = n;
+    p.n_layers = c->dims.n_layers;
+    p.page_size = (int32_t)P;
+    p.chunk_bytes = copy_chunk_bytes(c->dims);
+    p.page_bytes = c->page_bytes;
+    p.pool_pages = c->n_pages;
+    p.pool = c->pool;
+    KVG_CUDA(launch_graft_batch(p, c->n_sm, st));
+    if (flags & KVG_GRAFT_VERIFY)
+        for (int32_t i = 0; i < n; ++i) {
+            kvg_status r = enqueue_verify(s, s->blocks[block_ids[i]], c, verify_at[i].first, verify_at[i].second,
+                                          false, st);
+            if (r != KVG_OK) return r;
+        }
+    return finish_verify(c, n == 1 ? seq_ids[0] : -1, flags,
+                         (flags & KVG_GRAFT_VERIFY) ? (int32_t)(c->dims.n_layers * 2 * pages) : 0, st, report);
 }
 
 extern "C" kvg_status kvg_verify(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t slot0,

@@ -79,6 +79,7 @@ _SIGNATURES = {
     "kvg_cache_destroy": ([_vp], None),
     "kvg_cache_set_free_order": ([_vp, _vp, _i32], _i32),
     "kvg_cache_set_layer_windows": ([_vp, _vp, _i32], _i32),
+    "kvg_graft_batch": ([_vp, _vp, _vp, _vp, _i32, _u32, _vp, _vp], _i32),
     "kvg_cache_view_get": ([_vp, _P(kvg_cache_view)], _i32),
     "kvg_cache_seq_info": ([_vp, _i32, _P(_i32), _P(_i32)], _i32),
     "kvg_cache_append": ([_vp, _i32, _vp, _vp, _vp, _i32, _vp], _i32),
@@ -246,6 +247,17 @@ def kvg_graft(store, block_id: int, cache, seq: int, dst_slot: int = -1, delta: 
               stream=None, report: kvg_graft_report | None = None):
     _check(lib().kvg_graft(store, block_id, cache, seq, dst_slot, delta, flags, _stream(stream),
                            ctypes.byref(report) if report is not None else None))
+
+
+def kvg_graft_batch(store, block_ids, cache, seq_ids, flags: int = 0, stream=None,
+                    report: kvg_graft_report | None = None):
+    n = len(block_ids)
+    if len(seq_ids) != n:
+        raise ValueError("block_ids and seq_ids differ in length")
+    ids = (ctypes.c_uint64 * max(n, 1))(*[int(b) for b in block_ids])
+    seqs = (ctypes.c_int32 * max(n, 1))(*[int(x) for x in seq_ids])
+    _check(lib().kvg_graft_batch(store, ids, cache, seqs, n, flags, _stream(stream),
+                                 ctypes.byref(report) if report is not None else None))
 
 
 def kvg_verify(store, block_id: int, cache, seq: int, slot0: int = 0, flags: int = 0, stream=None,

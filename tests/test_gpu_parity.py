@@ -471,6 +471,66 @@ def test_host_store_verified_graft_reports_the_bad_page(oracle, geo, nb, bad):
     kvg.kvg_sync(s["dst"].h)
 
 
+@pytest.mark.parametrize("geo", ["tiny", "d128"])
+def test_graft_batch_equals_sequential_grafts(oracle, geo):
+    """kvg_graft_batch: blocks of several lengths (ragged ones too) into
+    sequences that repeat, stitched page-aligned in call order, in one launch:
+    pool bytes, page tables, fills and positions equal the oracle's sequential
+    grafts; with verification every graft is checked; a batch that does not
+    fit changes nothing."""
+    kvg = need_gpu()
+    w = geometry(geo)
+    P = w.page_size
+    dims = dims_for(kvg, w)
+    od = oracle_dims(oracle, w)
+    lens = [3 * P, 2 * P + 5, P - 3, 4 * P + 1, 7]
+    src = kvg.Cache(dims, 64, 1, 8 * P)
+    store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, HBM_CAP)
+    bids, oblks = [], []
+    for i, n in enumerate(lens):
+        k, v = _kv(w, n, 160 + i)
+        append(kvg, src, 0, k, v, syn.positions(0, n))
+        bids.append(kvg.kvg_deposit(store.h, src.h, 0, 0, n))
+        kvg.kvg_cache_release(src.h, 0)
+        oblks.append(oracle.block_from_kv(od, k, v, syn.positions(0, n)))
+    order = [(0, 2), (1, 0), (0, 1), (4, 2), (3, 1), (4, 0), (2, 2)]  # (block, seq)
+    n_pages = 64
+    max_slots = 16 * P
+    c = kvg.Cache(dims, n_pages, 3, max_slots)
+    fill_canary(c)
+    kvg.kvg_cache_set_free_order(c.h, syn.permutation(n_pages, 170))
+    oc = oracle.OracleCache(od, n_pages, 3, max_slots, fill=CANARY)
+    oc.set_free_order(syn.permutation(n_pages, 170))
+    # a short sequence first, so the first batched graft lands after a ragged page
+    k0, v0 = _kv(w, 3, 171)
+    append(kvg, c, 1, k0, v0, syn.positions(0, 3))
+    oc.append(1, k0, v0, syn.positions(0, 3))
+    rep = kvg.kvg_graft_report()
+    kvg.kvg_graft_batch(store.h, [bids[b] for b, _ in order], c.h, [q for _, q in order],
+                        kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, report=rep)
+    assert rep.n_mismatch == 0
+    assert rep.n_pages_checked == w.n_layers * 2 * sum(oblks[b].n_pages for b, _ in order)
+    for b, q in order:
+        oc.graft(q, oblks[b])
+    assert np.array_equal(pool_u16(c, w), oc.pool)
+    pt, pf, ps = tables(c)
+    assert np.array_equal(pt, oc.page_table) and np.array_equal(pf, oc.page_fill)
+    assert np.array_equal(ps, oc.positions)
+    for q in range(3):
+        assert kvg.kvg_cache_seq_info(c.h, q)[0] == oc.n_slots[q]
+    # too many pages for what is left: refused whole
+    before = pool_u16(c, w).copy()
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_graft_batch(store.h, [bids[3]] * 12, c.h, [0, 1, 2] * 4)
+    assert e.value.status == kvg.KVG_ERR_CAPACITY
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_graft_batch(store.h, [bids[0], 999], c.h, [0, 1])
+    assert e.value.status == kvg.KVG_ERR_NOT_FOUND
+    assert np.array_equal(pool_u16(c, w), before)
+    assert all(kvg.kvg_cache_seq_info(c.h, q)[0] == oc.n_slots[q] for q in range(3))
+    kvg.kvg_sync(c.h)
+
+
 def test_host_checks_reject_bad_calls(oracle):
     kvg = need_gpu()
     w = geometry("tiny")
