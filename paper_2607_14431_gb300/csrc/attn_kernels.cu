@@ -36,6 +36,8 @@
 #include <cuda_fp16.h>
 #include <math.h>
 
+#include <atomic>
+
 #include "common.cuh"
 
 namespace kvg {
@@ -572,19 +574,22 @@ __global__ void __launch_bounds__(D) combine_kernel(const DecodeParams p) {
 
 template <int D, int G, bool FP8>
 struct DecodeLaunch {
+    // The shared-memory attribute is per device: set and cached per device.
     static int max_blocks_per_sm() {
-        static int cached = -1;
-        if (cached < 0) {
-            if (cudaFuncSetAttribute(decode_kernel<D, G, FP8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     Cfg<D, FP8>::SMEM) != cudaSuccess)
-                return 0;
-            int n = 0;
-            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<D, G, FP8>, 32, Cfg<D, FP8>::SMEM) !=
-                cudaSuccess)
-                return 0;
-            cached = n;
-        }
-        return cached;
+        static std::atomic<int> cached[kMaxDevices];  // 0 = not yet known
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
+        int n = cached[dev].load();
+        if (n > 0) return n;
+        if (cudaFuncSetAttribute(decode_kernel<D, G, FP8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 Cfg<D, FP8>::SMEM) != cudaSuccess)
+            return 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<D, G, FP8>, 32, Cfg<D, FP8>::SMEM) !=
+                cudaSuccess ||
+            n <= 0)
+            return 0;
+        cached[dev].store(n);
+        return n;
     }
     static cudaError_t run(const DecodeParams &p, const CUtensorMap &map, cudaStream_t s) {
         if (max_blocks_per_sm() <= 0) return cudaErrorInvalidConfiguration;

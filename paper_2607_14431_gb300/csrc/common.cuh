@@ -17,6 +17,7 @@ namespace kvg {
 constexpr int kMaxPagesPerLaunch = 1024;  // page ids carried in kernel params
 constexpr int kMaxBatchPerLaunch = 256;   // decode rows carried in kernel params
 constexpr int kMaxLayersPerLaunch = 256;  // decode layers carried in kernel params
+constexpr int kMaxDevices = 64;           // per-device caches of launch set-up
 constexpr int kMaxHalfDim = 128;          // head_dim <= 256
 constexpr uint64_t kLeafBytes = KVG_DIGEST_LEAF_BYTES;
 

@@ -8,6 +8,8 @@
 //    streaming cache hint (the data is touched once).
 //  append_kernel: the "fresh" write of prefill-shaped rows into slots.
 //  gather_kernel: deposit, cache pages -> block pages, zeroing padding rows.
+#include <atomic>
+
 #include "common.cuh"
 
 namespace kvg {
@@ -648,12 +650,15 @@ cudaError_t launch_append_tma(const AppendParams &p, DevStatus *status, int n_sm
     for (int i = 0; i < 2; ++i)
         if (encode_tensor_map(&maps[i], 4, const_cast<uint16_t *>(src[i]), dims, strides, box) != cudaSuccess)
             return cudaErrorNotSupported;
-    static bool attr_set = false;
-    if (!attr_set) {
+    // the shared-memory attribute is per device
+    static std::atomic<bool> attr_set[kMaxDevices];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return cudaErrorNotSupported;
+    if (!attr_set[dev].load()) {
         cudaError_t e = cudaFuncSetAttribute(append_tma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)kTmaSmemBytes);
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        attr_set[dev].store(true);
     }
     const int chunks = (p.page_size + pbox - 1) / pbox;
     const int64_t jobs = 2ll * p.n_layers * p.pids.n * p.n_kv_heads * chunks;

@@ -31,9 +31,8 @@ static __device__ __align__(256) unsigned char g_decode_scratch[kScratchBytes];
 // Device address of g_decode_scratch per device ordinal.  In host code the
 // symbol names a host-side stand-in, so the address must come from
 // cudaGetSymbolAddress with that device current.
-constexpr int kMaxDevices = 64;
 std::mutex g_mu;
-void *g_scratch_dev[kMaxDevices] = {};
+void *g_scratch_dev[kvg::kMaxDevices] = {};
 
 }  // namespace
 
