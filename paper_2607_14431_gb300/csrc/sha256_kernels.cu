@@ -200,7 +200,17 @@ __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src
         uint64_t len = src.page_bytes - (uint64_t)i * kLeafBytes;
         if (len > kLeafBytes) len = kLeafBytes;
         uint32_t st[8];
-        hash_leaf<false>(page_addr(src, p) + (uint64_t)i * kLeafBytes, len, nullptr, st, one);
+        bool in_range = true;
+        if (src.pid) {  // page ids come from a device page table: never read outside the pool
+            const int32_t pid = src.pid[p - (p / src.npb) * src.npb];
+            in_range = pid >= 0 && pid < src.plane_pages;
+        }
+        if (in_range) {
+            hash_leaf<false>(page_addr(src, p) + (uint64_t)i * kLeafBytes, len, nullptr, st, one);
+        } else {
+#pragma unroll
+            for (int w = 0; w < 8; ++w) st[w] = 0u;  // no digest of any page: reported as a mismatch
+        }
         int64_t po = p;
         if (src.pid && src.out_plane_stride) {
             const int64_t plane = p / src.npb;

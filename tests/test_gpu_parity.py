@@ -531,6 +531,38 @@ def test_graft_batch_equals_sequential_grafts(oracle, geo):
     kvg.kvg_sync(c.h)
 
 
+def test_corrupt_page_table_entries_are_reported_not_followed(oracle):
+    """A page id outside the pool written into the device page table (through
+    the exported view) is never dereferenced: decode records
+    KVG_ERR_DEVICE_CHECK and skips that page; verification reports that page
+    as a digest mismatch."""
+    kvg = need_gpu()
+    w = geometry("d128")
+    s = _build_both(kvg, oracle, w, 300, 0, seed=181)
+    kvg.kvg_graft(s["store"].h, s["bid"], s["dst"].h, 0, -1, 0, kvg.KVG_GRAFT_SYNC)
+    v = s["dst"].view
+    pt = dev_view(v.page_table, v.max_seqs * v.max_pages * 4, torch.int32).view(v.max_seqs, v.max_pages)
+    good = int(pt[0, 2].item())
+    pt[0, 2] = s["n_pages"] + 7
+    torch.cuda.synchronize()
+    q = syn.as_u16(syn.queries(w, w.n_layers, 1, 182))
+    decode(kvg, s["dst"], w, [0], q)
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_sync(s["dst"].h)
+    assert e.value.status == kvg.KVG_ERR_DEVICE_CHECK
+    rep = kvg.kvg_graft_report()
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_verify(s["store"].h, s["bid"], s["dst"].h, 0, 0, kvg.KVG_GRAFT_SYNC, report=rep)
+    assert e.value.status == kvg.KVG_ERR_DIGEST
+    npb = (300 + w.page_size - 1) // w.page_size
+    assert sorted(rep.mismatch_pages[:rep.n_mismatch]) == [pl * npb + 2 for pl in range(w.n_layers * 2)]
+    # restored, everything is clean again
+    pt[0, 2] = good
+    torch.cuda.synchronize()
+    kvg.kvg_verify(s["store"].h, s["bid"], s["dst"].h, 0, 0, kvg.KVG_GRAFT_SYNC)
+    kvg.kvg_sync(s["dst"].h)
+
+
 def test_host_checks_reject_bad_calls(oracle):
     kvg = need_gpu()
     w = geometry("tiny")
