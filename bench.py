@@ -398,16 +398,9 @@ def run_kvg(args, rank, world):
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": f"12b-single-graft: L{st.w.n_layers} Hq16/Hkv8 D256 P64, 8192-token block grafted "
-                               "at own positions (digest-verified) + 24576 fresh tokens, decode 1 token over 32768"
-                               + (" [block in the cache pool: zero-copy graft]" if st.pool_store else "")
-                               + (" [verified graft in one pass, beside the append]" if st.schedule == "fused" else "")
-                               + (f" [sliding-window layers: window {st.swa[0]}, every {st.swa[1]}th layer global]"
-                                  if st.swa else "")
-                               + (f" [fp8 E4M3 KV, scales k {syn.FP8_K_SCALE} v {syn.FP8_V_SCALE}]"
-                                  if st.kv == "e4m3" else ""),
-                   "global_batch": world, "seq_len": syn.B12_CTX, "parallelism": f"replicas{world}",
-                   "l2": "inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)"},
+        "config": dict(config_12b(st.w.n_layers, world, pool_store=st.pool_store, swa=st.swa, kv=st.kv),
+                       schedule="verified graft in one pass, beside the append" if st.schedule == "fused"
+                       else "graft, then the digest check beside the append and the decode"),
         "parts": parts, "roofline": roof, "e2e": e2e, "gpu_launches": int(launches),
         "clocks": clk, "checks": {"deterministic": deterministic, "digest_verified_steps": K + args.warmup + 1},
     }
@@ -797,6 +790,17 @@ def cpu_baseline(n_layers_sample=48):
                       f"append, fp64 decode of 16 heads over 32768 rows), in 4-layer chunks: {dt:.2f} s"}
 
 
+def config_12b(n_layers=48, world=1, pool_store=False, swa=None, kv="bf16"):
+    """The 12b workload's config entry, shared by both arms of the bench."""
+    return {"workload": f"12b-single-graft: L{n_layers} Hq16/Hkv8 D256 P64, 8192-token block grafted "
+                        "at own positions (digest-verified) + 24576 fresh tokens, decode 1 token over 32768"
+                        + (" [block in the cache pool: zero-copy graft]" if pool_store else "")
+                        + (f" [sliding-window layers: window {swa[0]}, every {swa[1]}th layer global]" if swa else "")
+                        + (f" [fp8 E4M3 KV, scales k {syn.FP8_K_SCALE} v {syn.FP8_V_SCALE}]" if kv == "e4m3" else ""),
+            "global_batch": world, "seq_len": syn.B12_CTX, "parallelism": f"replicas{world}",
+            "l2": "inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)"}
+
+
 def run_reference(args):
     ts, b, cores = [], 0, 1
     for k in range(args.warmup + args.steps):
@@ -807,10 +811,10 @@ def run_reference(args):
     value = b / t / 1e9
     cb = {"value": round(value, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
           "sample": "1 of 48 layers of one 12b step per timed step"}
-    return {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": 0,
+    return {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t * 1e3, 2),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": "12b-single-graft (1-layer sample)"},
+            "data": "synthetic", "config": config_12b(world=args.gpus),
             "cpu_baseline": cb, "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                                         "d2h_bytes_per_step": 0}}
 
