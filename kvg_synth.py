@@ -129,3 +129,30 @@ def deep_plan(seed: int = DEEP.seed, n_grafts: int = DEEP_GRAFTS, n_blocks: int 
 
 def permutation(n: int, seed: int) -> np.ndarray:
     return np.random.default_rng(seed).permutation(n).astype(np.int32)
+
+
+def splitmix64(seed: int, n: int) -> np.ndarray:
+    """The first n outputs of SplitMix64 seeded with `seed` (Steele, Lea and
+    Flood, "Fast splittable pseudorandom number generators", 2014: the state
+    advances by the golden-ratio increment, each output is the state mixed by
+    two xor-shift-multiply rounds).  Integer-only, so the same bytes on every
+    machine and library version."""
+    with np.errstate(over="ignore"):
+        z = (np.uint64(seed & 0xFFFFFFFFFFFFFFFF)
+             + (np.arange(1, n + 1, dtype=np.uint64) * np.uint64(0x9E3779B97F4A7C15)))
+        z = (z ^ (z >> np.uint64(30))) * np.uint64(0xBF58476D1CE4E5B9)
+        z = (z ^ (z >> np.uint64(27))) * np.uint64(0x94D049BB133111EB)
+        return z ^ (z >> np.uint64(31))
+
+
+def portable_bf16(shape, seed: int) -> np.ndarray:
+    """bf16 bit patterns drawn with integer operations only (for stored
+    fixtures that must not depend on a library's random generator): random
+    sign, binade uniform over 2^-4 ... 2^0 (so |x| < 2, the scale of the
+    N(0, 1) workloads), mantissa uniform."""
+    n = int(np.prod(shape))
+    r = splitmix64(seed, n)
+    sign = (r & np.uint64(1)) << np.uint64(15)
+    expo = (np.uint64(123) + (r >> np.uint64(8)) % np.uint64(5)) << np.uint64(7)
+    mant = (r >> np.uint64(16)) & np.uint64(0x7F)
+    return (sign | expo | mant).astype(np.uint16).reshape(shape)

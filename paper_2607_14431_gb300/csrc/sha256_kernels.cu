@@ -394,9 +394,11 @@ cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_
     const int64_t n = n_pages * m;
     if (n == 0) return cudaSuccess;
     int64_t grid = (n + 127) / 128;
-    static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 8);
-    const int64_t cap = (int64_t)n_sm * ctas_per_sm;
-    if (grid > cap) grid = cap;
+    // One CTA per 128 leaves (no grid-stride cap by default): 4 CTAs of
+    // 125 registers are resident per SM and the rest queue, which measured
+    // 2-3% faster than a capped, striding grid.
+    static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 0);
+    if (ctas_per_sm > 0 && grid > (int64_t)n_sm * ctas_per_sm) grid = (int64_t)n_sm * ctas_per_sm;
     sha256_leaves_kernel<<<(int)grid, 128, 0, s>>>(src, n_pages, m, leaf_words, 1u);
     count_launches(1);
     return cudaGetLastError();
@@ -407,9 +409,11 @@ cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int 
     const int64_t n = (int64_t)p.n_layers * 2 * p.npb * m;
     if (n == 0) return cudaSuccess;
     int64_t grid = (n + 127) / 128;
-    static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 8);
-    const int64_t cap = (int64_t)n_sm * ctas_per_sm;
-    if (grid > cap) grid = cap;
+    // One CTA per 128 leaves (no grid-stride cap by default): 4 CTAs of
+    // 125 registers are resident per SM and the rest queue, which measured
+    // 2-3% faster than a capped, striding grid.
+    static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 0);
+    if (ctas_per_sm > 0 && grid > (int64_t)n_sm * ctas_per_sm) grid = (int64_t)n_sm * ctas_per_sm;
     graft_verify_kernel<<<(int)grid, 128, 0, s>>>(p, m, leaf_words, 1u);
     count_launches(1);
     return cudaGetLastError();
