@@ -25,8 +25,10 @@
  *     waiting unless a flag asks for it.  Errors that only the GPU can see
  *     (a digest mismatch, a failed device-side bounds check) are recorded in
  *     the cache's device status word and reported by kvg_sync().
- *   - Element type: bf16 only (raw 16-bit patterns).  Sizes are in elements
- *     unless a name ends in _bytes.
+ *   - Element types: inputs and outputs (k, v, q, out) are bf16 (raw 16-bit
+ *     patterns); a cache and its blocks hold bf16 or, when kvg_dims.kv_dtype
+ *     asks for it, fp8 E4M3 codes.  Sizes are in elements unless a name ends
+ *     in _bytes.
  *   - Ownership: stores, caches and their device memory belong to the
  *     library; buffers passed in (k, v, q, out, positions) belong to the
  *     caller and must stay valid until the enqueued work completes.
@@ -136,12 +138,14 @@ kvg_status kvg_store_create_in_cache(kvg_cache *cache, uint64_t capacity_bytes, 
  *   [0, 256)      header: magic "KVGBLK01", u32 version = 1, u32 header bytes
  *                 = 256, i32 n_layers, n_kv_heads, head_dim, page_size,
  *                 i64 n_tokens, i64 n_pages, f64 rope_theta, i32 rope_style,
- *                 i32 dtype (1 = bf16), u64 positions_offset, digests_offset,
- *                 pages_offset, total_bytes; at byte 96 the 32-byte block
- *                 digest; the rest zero.
+ *                 i32 dtype (1 = bf16, 2 = E4M3), u64 positions_offset,
+ *                 digests_offset, pages_offset, total_bytes; at byte 96 the
+ *                 32-byte block digest; for E4M3 the fp32 k_scale and v_scale
+ *                 at bytes 128 and 132; the rest zero.
  *   positions     int32 [n_tokens] position tags (offset 256)
  *   digests       [n_layers][2][n_pages][32] page digests (256-aligned)
- *   pages         bf16 [n_layers][2][n_pages][n_kv_heads][page_size][head_dim]
+ *   pages         bf16 (or E4M3 codes)
+ *                 [n_layers][2][n_pages][n_kv_heads][page_size][head_dim]
  *                 (4096-aligned), kv 0 = K, 1 = V; token t of the block is row
  *                 t % page_size of page t / page_size; rows past n_tokens in
  *                 the last page are zero.
@@ -192,9 +196,9 @@ kvg_status kvg_store_load(kvg_store *store, const char *path, uint32_t flags, ui
 
 /* ---------------------------------------------------------------- cache -- */
 
-/* A paged KV cache on `device`: pool bf16 [n_layers][2][n_pages][n_kv_heads]
- * [page_size][head_dim] (one page id names the same token rows in every
- * layer), and per sequence a page table, per-page fill counts, position tags
+/* A paged KV cache on `device`: pool of elements (bf16, or E4M3 codes for an
+ * fp8 cache) [n_layers][2][n_pages][n_kv_heads][page_size][head_dim] (one
+ * page id names the same token rows in every layer), and per sequence a page table, per-page fill counts, position tags
  * per slot and a slot high-water mark.  The pool is not initialised.
  * Free pages are handed out from the front of an ordered free list,
  * initially 0, 1, ..., n_pages-1; a released sequence's pages go to its back
@@ -226,7 +230,7 @@ kvg_status kvg_cache_set_layer_windows(kvg_cache *cache, const int32_t *windows,
 
 /* Device-side layout, for inspection and for interop with other kernels. */
 typedef struct kvg_cache_view {
-    void *pool;            /* bf16 [L][2][n_pages][Hkv][P][D] */
+    void *pool;            /* elements [L][2][n_pages][Hkv][P][D] (bf16 or E4M3 codes) */
     int32_t *page_table;   /* int32 [max_seqs][max_pages], -1 = no page */
     int32_t *page_fill;    /* int32 [max_seqs][max_pages], valid rows (a prefix) */
     int32_t *positions;    /* int32 [max_seqs][max_slots], -1 = unwritten */
