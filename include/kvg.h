@@ -63,6 +63,7 @@ enum { KVG_RESIDENCY_HBM = 0, KVG_RESIDENCY_PINNED_HOST = 1, KVG_RESIDENCY_CACHE
 enum { KVG_ROPE_HALF = 0, KVG_ROPE_INTERLEAVED = 1 };
 enum { KVG_GRAFT_VERIFY = 1u, KVG_GRAFT_SYNC = 2u };
 enum { KVG_SHA256_PLAIN = 0, KVG_SHA256_PAGED = 1 };
+enum { KVG_DECODE_MERGE = 1u };
 /* KV element types (kvg_dims.kv_dtype). */
 enum { KVG_KV_BF16 = 0, KVG_KV_E4M3 = 1 };
 
@@ -365,6 +366,45 @@ kvg_status kvg_verify(kvg_store *store, uint64_t block_id, kvg_cache *cache, int
 kvg_status kvg_decode_attention(kvg_cache *cache, int32_t layer, const int32_t *seq_ids,
                                 int32_t B, const void *q, int32_t n_q_heads, void *out,
                                 float scale, void *stream);
+
+/* Split decode: the attention of kvg_decode_attention over only the rows in
+ * slots [slot_begin, slot_end) of each sequence, kept as a softmax state that
+ * calls over other slot ranges merge into, so that the part of a context that
+ * is already resident is attended to while the rest is still being restored
+ * (the decode step of Sec. 3.2 on top of a block that a graft from the host
+ * store, Sec. 4.4, is still copying).  The paper has no split decode of its
+ * own; the state is the usual one of an online softmax.
+ * Rows: the valid rows (below their page's fill) of the sequence's pages
+ * slot_begin / page_size ... slot_end / page_size - 1, and on a windowed
+ * layer only those that are also among its last W valid rows (the window is
+ * taken over the whole sequence as it stands at the call).
+ * slot_begin, slot_end: multiples of page_size, 0 <= slot_begin <= slot_end;
+ * slot_end >= max_slots means "to the end of the sequence".
+ * state: device fp32 [n_layers_run][B][n_q_heads][head_dim + 4], 16-byte
+ * aligned, caller-owned; per query head: o[head_dim] (the weighted sum of
+ * value rows, times v_scale for an fp8 cache), m (the running maximum of
+ * scale * log2(e) * q.k), l (the sum of 2^(scale * log2(e) * q.k - m)), two
+ * unused floats.  A head with no rows has l = 0, o = 0, m = -inf.
+ * flags: 0 overwrites the state with this call's part; KVG_DECODE_MERGE
+ * merges this call's part into the state already there (written by earlier
+ * calls with the same layer, batch rows and heads): m' = max(m0, m),
+ * o' = o0 2^(m0 - m') + o 2^(m - m'), l' = l0 2^(m0 - m') + l 2^(m - m').
+ * Parts that cover disjoint slot ranges whose union is every row give, after
+ * kvg_decode_state_finish, the attention over all rows within the rounding
+ * of the merge; the result is bitwise reproducible for the same sequence of
+ * calls.  Other arguments and errors as for kvg_decode_attention, plus
+ * KVG_ERR_ARG for a range that is not page-aligned or unknown flags. */
+kvg_status kvg_decode_attention_range(kvg_cache *cache, int32_t layer, const int32_t *seq_ids, int32_t B,
+                                      const void *q, int32_t n_q_heads, float scale, int32_t slot_begin,
+                                      int32_t slot_end, uint32_t flags, float *state, void *stream);
+
+/* Output of a split decode: out[r][d] = bf16_rne(o[d] / l) for each of the
+ * n_rows = n_layers_run * B * n_q_heads state rows (out = 0 where l = 0),
+ * written as bf16 [n_rows][head_dim] (the layout of kvg_decode_attention's
+ * out).  state and out are device pointers, 16-byte aligned; head_dim 64,
+ * 128 or 256.  Runs on `stream` on the current device. */
+kvg_status kvg_decode_state_finish(const float *state, int64_t n_rows, int32_t head_dim, void *out,
+                                   void *stream);
 
 /* The same decode attention, for callers that cannot allocate GPU memory.
  * (The paper has no counterpart: this is a deployment variant.)

@@ -670,6 +670,33 @@ class OracleCache:
             raise KvgError("need one window >= 0 per layer")
         self.windows = w
 
+    def decode_range(self, seq: int, layer: int, q: np.ndarray, scale: float, slot_begin: int,
+                     slot_end: int) -> np.ndarray:
+        """fp64 decode attention of q[Hq][D] over the valid rows whose slots lie
+        in [slot_begin, slot_end) and, on a windowed layer, among the layer's
+        last W valid rows of the whole sequence: the part of the decode step
+        (Sec. 3.2) that a split decode computes over already-resident rows."""
+        d = self.dims
+        slots = []
+        npg = (int(self.n_slots[seq]) + d.P - 1) // d.P
+        for j in range(npg):
+            for r in range(int(self.page_fill[seq, j]) if self.page_table[seq, j] >= 0 else 0):
+                slots.append(j * d.P + r)
+        W = self.windows[layer]
+        if W > 0:
+            slots = slots[-W:]
+        keep = [s for s in slots if slot_begin <= s < slot_end]
+        k = np.zeros((len(keep), d.Hkv, d.D), d.code_dtype)
+        v = np.zeros((len(keep), d.Hkv, d.D), d.code_dtype)
+        for i, s in enumerate(keep):
+            j, r = divmod(s, d.P)
+            pid = self.page_table[seq, j]
+            k[i] = self.pool[layer, 0, pid, :, r, :]
+            v[i] = self.pool[layer, 1, pid, :, r, :]
+        if d.fp8:
+            return gqa_decode_f64kv(q, e4m3_dequant(k, d.k_scale), e4m3_dequant(v, d.v_scale), scale)
+        return gqa_decode(q, k, v, scale)
+
     def decode(self, seq: int, layer: int, q: np.ndarray, scale: float) -> np.ndarray:
         """fp64 decode attention of q[Hq][D] over the sequence's valid rows,
         or over the last W of them when the layer has a window W > 0."""

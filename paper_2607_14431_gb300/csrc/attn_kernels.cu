@@ -572,6 +572,84 @@ __global__ void __launch_bounds__(D) combine_kernel(const DecodeParams p) {
         __float2bfloat16_rn(r);
 }
 
+// The same merge for a split decode: the unit's partials give (M, L, O) for
+// this call's rows, scaled by vscale, and the result is stored as the state
+// (o, m, l) of query head h, or merged into the state already there:
+// m' = max(m0, M), o' = o0 2^(m0 - m') + O 2^(M - m'), l' likewise (a side
+// with l = 0 holds no rows and is left out).
+template <int D>
+__global__ void __launch_bounds__(D) combine_state_kernel(const DecodeParams p) {
+    const int h = blockIdx.x, b = blockIdx.y, lr = blockIdx.z;
+    const int G = p.n_q_heads / p.n_kv_heads;
+    const int g = h / G, hh = h - g * G;
+    const int d = threadIdx.x;
+    const int64_t unit = ((int64_t)lr * p.B + b) * p.n_kv_heads + g;
+    const int64_t sumT = p.rows.pref_tiles[p.B];
+    const int64_t Tb = p.rows.pref_tiles[b + 1] - p.rows.pref_tiles[b];
+    float L = 0.f, O = 0.f, M = -INFINITY;
+    if (Tb > 0) {
+        const int64_t T = p.n_tiles, W = p.n_warps;
+        const int64_t first = (int64_t)lr * p.n_kv_heads * sumT + (int64_t)p.n_kv_heads * p.rows.pref_tiles[b] +
+                              (int64_t)g * Tb;
+        const int64_t last = first + Tb - 1;
+        const int64_t wa = warp_of(first, T, W), wb = warp_of(last, T, W);
+        for (int64_t w = wa; w <= wb; ++w) {
+            if (warp_start(w + 1, T, W) == warp_start(w, T, W)) continue;  // empty range
+            M = fmaxf(M, p.part_ml[(unit + w) * G + hh].x);
+        }
+        for (int64_t w = wa; w <= wb; ++w) {
+            if (warp_start(w + 1, T, W) == warp_start(w, T, W)) continue;
+            const float2 ml = p.part_ml[(unit + w) * G + hh];
+            if (ml.x == -INFINITY) continue;
+            const float sc = exp2f(ml.x - M);
+            L = __fmaf_rn(ml.y, sc, L);
+            O = __fmaf_rn(p.part_o[((unit + w) * G + hh) * D + d], sc, O);
+        }
+        O = __fmul_rn(O, p.vscale);
+    }
+    float *st = p.state + ((int64_t)(p.qlayers[lr] * p.q_row_stride_b + p.b0 + b) * p.n_q_heads + h) * (D + 4);
+    if (p.state_merge) {
+        const float m0 = st[D], l0 = st[D + 1], o0 = st[d];
+        __syncthreads();  // every thread has read (m0, l0) before thread 0 rewrites them
+        if (l0 > 0.f) {
+            if (L > 0.f) {
+                const float mm = fmaxf(m0, M);
+                const float a = exp2f(m0 - mm), c = exp2f(M - mm);
+                O = __fmaf_rn(o0, a, __fmul_rn(O, c));
+                L = __fmaf_rn(l0, a, __fmul_rn(L, c));
+                M = mm;
+            } else {
+                O = o0;
+                L = l0;
+                M = m0;
+            }
+        }
+    }
+    if (L == 0.f) {
+        O = 0.f;
+        M = -INFINITY;
+    }
+    st[d] = O;
+    if (d == 0) {
+        st[D] = M;
+        st[D + 1] = L;
+        st[D + 2] = 0.f;
+        st[D + 3] = 0.f;
+    }
+}
+
+__global__ void state_finish_kernel(const float *__restrict__ state, int64_t n_rows, int D,
+                                    __nv_bfloat16 *__restrict__ out) {
+    const int64_t n = n_rows * D;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = i / D;
+        const int d = (int)(i - r * D);
+        const float *st = state + r * (D + 4);
+        const float l = st[D + 1];
+        out[i] = __float2bfloat16_rn(l > 0.f ? __fdiv_rn(st[d], l) : 0.f);
+    }
+}
+
 template <int D, int G, bool FP8>
 struct DecodeLaunch {
     // The shared-memory attribute is per device: set and cached per device.
@@ -695,12 +773,33 @@ cudaError_t launch_decode(int head_dim, int group, bool fp8, const DecodeParams 
 cudaError_t launch_combine(int head_dim, int group, const DecodeParams &p, cudaStream_t s) {
     (void)group;
     dim3 grid(p.n_q_heads, p.B, p.n_layers_run);
+    if (p.state) {
+        switch (head_dim) {
+            case 64: combine_state_kernel<64><<<grid, 64, 0, s>>>(p); break;
+            case 128: combine_state_kernel<128><<<grid, 128, 0, s>>>(p); break;
+            case 256: combine_state_kernel<256><<<grid, 256, 0, s>>>(p); break;
+            default: return cudaErrorInvalidValue;
+        }
+        count_launches(1);
+        return cudaGetLastError();
+    }
     switch (head_dim) {
         case 64: combine_kernel<64><<<grid, 64, 0, s>>>(p); count_launches(1); break;
         case 128: combine_kernel<128><<<grid, 128, 0, s>>>(p); count_launches(1); break;
         case 256: combine_kernel<256><<<grid, 256, 0, s>>>(p); count_launches(1); break;
         default: return cudaErrorInvalidValue;
     }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_state_finish(const float *state, int64_t n_rows, int head_dim, __nv_bfloat16 *out,
+                                cudaStream_t s) {
+    const int64_t n = n_rows * head_dim;
+    if (n == 0) return cudaSuccess;
+    int64_t grid = (n + 255) / 256;
+    if (grid > 65535) grid = 65535;
+    state_finish_kernel<<<(int)grid, 256, 0, s>>>(state, n_rows, head_dim, out);
+    count_launches(1);
     return cudaGetLastError();
 }
 

@@ -233,6 +233,8 @@ struct DecodeParams {
     float *part_o;             // [U + W][G][D]
     float2 *part_ml;           // [U + W][G]
     __nv_bfloat16 *out;        // [Lrun][Btot][Hq][D] (combine)
+    float *state;              // split decode: fp32 [Lrun][Btot][Hq][D + 4] (o, m, l, pad); null otherwise
+    int32_t state_merge;       // 1: merge into the state, 0: overwrite it
     DevStatus *status;
     BatchRows rows;
 };
@@ -245,9 +247,11 @@ uint64_t launch_count();
 // a grid-stride kernel; `fallback` when unset or not positive.
 int env_knob(const char *name, int fallback);
 
-cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s);
+// max_ctas > 0 caps the grid (a copy from host memory needs only enough
+// CTAs to keep the host link busy; the rest of the SMs stay free).
+cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s, int max_ctas = 0);
 // Own-position copies of a batch of grafts in one launch (jobs, metas in device memory).
-cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s);
+cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s, int max_ctas = 0);
 // Bulk append by tensor copies, for appends of at least append_tma_rows()
 // rows (16-byte aligned k/v).  Returns cudaErrorNotSupported (nothing
 // launched) when the tensor maps cannot be encoded, so the caller can take
@@ -289,6 +293,10 @@ cudaError_t launch_sha256_serial(const uint8_t *seg0, uint64_t n0, const uint8_t
 // combine over every (layer, row, query head).  decode_tile_tokens() is the
 // tile height TOK (tiles per page = ceil(P / TOK)); decode_max_warps() the
 // number of co-resident warps the decode kernel can keep on the device.
+// Split-decode state -> bf16 output: out[r][d] = o / l (0 where l = 0), for
+// n_rows rows of D + 4 floats.
+cudaError_t launch_state_finish(const float *state, int64_t n_rows, int head_dim, __nv_bfloat16 *out,
+                                cudaStream_t s);
 cudaError_t launch_decode(int head_dim, int group, bool fp8, const DecodeParams &p, const CUtensorMap &pool_map,
                           cudaStream_t s);
 // Tensor map of a cache pool for the decode kernel: a 2-D bf16 tensor of

@@ -591,16 +591,19 @@ __global__ void __launch_bounds__(kCopyThreads) graft_batch_kernel(const GraftBa
     }
 }
 
-cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s) {
+cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s, int max_ctas) {
     const int64_t units = p.n_jobs * p.n_layers * 2 * (int64_t)(p.page_bytes / p.chunk_bytes);
-    graft_batch_kernel<<<grid_for(units, 1, n_sm, 4), kCopyThreads, 0, s>>>(p);
+    int grid = grid_for(units, 1, n_sm, 4);
+    if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
+    graft_batch_kernel<<<grid, kCopyThreads, 0, s>>>(p);
     count_launches(1);
     return cudaGetLastError();
 }
 
-cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s) {
+cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s, int max_ctas) {
     const int64_t units = (int64_t)p.n_layers * 2 * p.npb * (int64_t)(p.page_bytes / p.chunk_bytes);
-    const int grid = grid_for(units, 1, n_sm, 4);
+    int grid = grid_for(units, 1, n_sm, 4);
+    if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
     if (p.rotate == 0)
         graft_kernel<0><<<grid, kCopyThreads, 0, s>>>(p);
     else if (p.rotate == 1)

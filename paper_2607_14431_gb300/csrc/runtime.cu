@@ -506,7 +506,7 @@ extern "C" kvg_status kvg_store_load(kvg_store *s, const char *path, uint32_t fl
 
 // ------------------------------------------------------------------- cache --
 
-constexpr int kHostVerifyChunks = 8;  // page-range chunks of a verified host-store graft
+constexpr int kHostVerifyChunks = 16;  // page-range chunks of a verified host-store graft
 constexpr int32_t kMaxGraftsPerBatch = 4096;
 
 struct kvg_cache {
@@ -1187,6 +1187,16 @@ static kvg_status pool_graft(kvg_store *s, const kvg_store::Blk &blk, kvg_cache 
                          st, report);
 }
 
+// A copy out of a pinned-host store waits on the host link: 32 CTAs keep it
+// at its limit (211 GB/s on the GB300 measured, the same as with 608), and the
+// other SMs stay free for the work that runs beside the graft (appends,
+// decodes, the digest check); with a CTA on every SM the copy held them all
+// and an append beside it finished only when the graft did.
+static int host_copy_grid_cap() {
+    static const int cap = env_knob("KVG_HOST_COPY_CTAS", 32);
+    return cap;
+}
+
 extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t dst_slot,
                                 int64_t delta, uint32_t flags, void *stream, kvg_graft_report *report) {
     Trace trace_("kvg_graft");
@@ -1249,6 +1259,8 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
     // chunks with the copy kernel (whose wide reads keep the host link at its
     // limit) and a library stream hashes each chunk's restored pages in HBM
     // while the next chunk crosses the link.
+    const bool host_src = s->residency == KVG_RESIDENCY_PINNED_HOST;
+    const int host_copy_ctas = host_copy_grid_cap();
     const bool verify0 = (flags & KVG_GRAFT_VERIFY) && delta == 0;
     const bool piped = verify0 && s->residency == KVG_RESIDENCY_PINNED_HOST;
     const bool fused = verify0 && !piped;
@@ -1275,9 +1287,9 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
         if (fused)
             KVG_CUDA(launch_graft_verify(p, static_cast<uint32_t *>(c->leaf.ptr), c->n_sm, st));
         else
-            KVG_CUDA(launch_graft_copy(p, c->n_sm, st));
+            KVG_CUDA(launch_graft_copy(p, c->n_sm, st, host_src ? host_copy_ctas : 0));
         if (piped) {
-            // (more than kHostVerifyChunks chunks only past 8 x 1,024 pages per
+            // (more than kHostVerifyChunks chunks only past 16 x 1,024 pages per
             // plane; an event is re-recorded after its wait is enqueued)
             cudaEvent_t ev = c->aux_ev[chunk % kHostVerifyChunks];
             KVG_CUDA(cudaEventRecord(ev, st));
@@ -1388,7 +1400,7 @@ extern "C" kvg_status kvg_graft_batch(kvg_store *s, const uint64_t *block_ids, k
     p.page_bytes = c->page_bytes;
     p.pool_pages = c->n_pages;
     p.pool = c->pool;
-    KVG_CUDA(launch_graft_batch(p, c->n_sm, st));
+    KVG_CUDA(launch_graft_batch(p, c->n_sm, st, s->residency == KVG_RESIDENCY_PINNED_HOST ? host_copy_grid_cap() : 0));
     if (flags & KVG_GRAFT_VERIFY)
         for (int32_t i = 0; i < n; ++i) {
             kvg_status r = enqueue_verify(s, s->blocks[block_ids[i]], c, verify_at[i].first, verify_at[i].second,
@@ -1446,8 +1458,11 @@ static void window_start(const kvg_cache *c, int32_t seq, int64_t window, int32_
 // launches of at most kMaxLayersPerLaunch layers and kMaxBatchPerLaunch rows.
 // Fills every field but the per-call ones (q, out, scale, heads, scratch,
 // workers); *max_units gets the largest layers x rows x kv heads of a launch.
+// page_begin / page_end: only the sequence's pages [page_begin, page_end)
+// are read (a split decode over a slot range); the defaults read them all.
 static kvg_status plan_decode(const kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
-                              std::vector<DecodeParams> *plan, int64_t *max_units) {
+                              std::vector<DecodeParams> *plan, int64_t *max_units, int32_t page_begin = 0,
+                              int32_t page_end = INT32_MAX) {
     const kvg_dims &d = c->dims;
     const int TOK = decode_tile_tokens(d.head_dim);
     const int tpp = (d.page_size + TOK - 1) / TOK;
@@ -1479,11 +1494,17 @@ static kvg_status plan_decode(const kvg_cache *c, int32_t layer, const int32_t *
                     const int32_t np = (int32_t)c->seq_pages[sq].size();
                     int32_t pg = 0, row = 0;
                     if (W > 0) window_start(c, sq, W, &pg, &row);
+                    int32_t t0 = pg * tpp + row / TOK, lo = row % TOK;
+                    if (page_begin > 0 && (int64_t)page_begin * tpp > t0) {
+                        t0 = page_begin * tpp;
+                        lo = 0;
+                    }
+                    const int32_t t1 = std::min(np, page_end) * tpp;
                     p.rows.seq[i] = sq;
-                    p.rows.tile0[i] = pg * tpp + row / TOK;
-                    p.rows.lo[i] = row % TOK;
+                    p.rows.tile0[i] = t0;
+                    p.rows.lo[i] = lo;
                     p.rows.pref_tiles[i] = acc;
-                    acc += np * tpp - p.rows.tile0[i];
+                    acc += std::max(0, t1 - t0);
                 }
                 p.rows.pref_tiles[nb] = acc;
                 for (int32_t i = 0; i < nl; ++i) {
@@ -1522,11 +1543,12 @@ extern "C" kvg_status kvg_cache_set_layer_windows(kvg_cache *c, const int32_t *w
     return KVG_OK;
 }
 
-extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
-                                           const void *q, int32_t n_q_heads, void *out, float scale,
-                                           void *stream) {
-    Trace trace_("kvg_decode_attention");
-    if (!c || !seq_ids || !q || !out) return fail(KVG_ERR_ARG, "null argument");
+// Decode attention over the sequences' pages [page_begin, page_end): bf16
+// out (state == null), or the softmax state written or merged into `state`.
+static kvg_status decode_impl(const char *what, kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
+                              const void *q, int32_t n_q_heads, void *out, float scale, void *stream,
+                              int32_t page_begin, int32_t page_end, float *state, int32_t merge) {
+    if (!c || !seq_ids || !q || !(out || state)) return fail(KVG_ERR_ARG, "%s: null argument", what);
     const kvg_dims &d = c->dims;
     if (layer < -1 || layer >= d.n_layers) return fail(KVG_ERR_ARG, "bad layer %d", layer);
     if (B <= 0 || B > 4096) return fail(KVG_ERR_ARG, "B must be in [1, 4096]");
@@ -1535,8 +1557,8 @@ extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const in
     const bool fp8 = d.kv_dtype == KVG_KV_E4M3;
     if (!decode_supported(d.head_dim, G, fp8))
         return fail(KVG_ERR_ARG, "unsupported head_dim %d / group %d%s", d.head_dim, G, fp8 ? " (fp8)" : "");
-    if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out)) & 15)
-        return fail(KVG_ERR_ARG, "q/out must be 16-byte aligned");
+    if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out) | reinterpret_cast<uintptr_t>(state)) & 15)
+        return fail(KVG_ERR_ARG, "q/out/state must be 16-byte aligned");
     for (int32_t b = 0; b < B; ++b)
         if (seq_ids[b] < 0 || seq_ids[b] >= c->max_seqs) return fail(KVG_ERR_ARG, "bad seq id %d", seq_ids[b]);
     DeviceGuard g(c->device);
@@ -1545,7 +1567,7 @@ extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const in
     if (w_max <= 0) return fail(KVG_ERR_CUDA, "decode kernel cannot be made resident");
     std::vector<DecodeParams> plan;
     int64_t max_units = 0;
-    kvg_status r = plan_decode(c, layer, seq_ids, B, &plan, &max_units);
+    kvg_status r = plan_decode(c, layer, seq_ids, B, &plan, &max_units, page_begin, page_end);
     if (r != KVG_OK) return r;
     const size_t slots = (size_t)max_units + (size_t)w_max;
     KVG_CUDA(c->part_o.ensure(slots * G * d.head_dim * sizeof(float)));
@@ -1560,9 +1582,48 @@ extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const in
         p.part_o = static_cast<float *>(c->part_o.ptr);
         p.part_ml = static_cast<float2 *>(c->part_ml.ptr);
         p.out = static_cast<__nv_bfloat16 *>(out);
+        p.state = state;
+        p.state_merge = merge;
         KVG_CUDA(launch_decode(d.head_dim, G, fp8, p, c->pool_map, st));
         KVG_CUDA(launch_combine(d.head_dim, G, p, st));
     }
+    return KVG_OK;
+}
+
+extern "C" kvg_status kvg_decode_attention(kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
+                                           const void *q, int32_t n_q_heads, void *out, float scale,
+                                           void *stream) {
+    Trace trace_("kvg_decode_attention");
+    if (!out) return fail(KVG_ERR_ARG, "null argument");
+    return decode_impl("kvg_decode_attention", c, layer, seq_ids, B, q, n_q_heads, out, scale, stream, 0, INT32_MAX,
+                       nullptr, 0);
+}
+
+extern "C" kvg_status kvg_decode_attention_range(kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
+                                                 const void *q, int32_t n_q_heads, float scale, int32_t slot_begin,
+                                                 int32_t slot_end, uint32_t flags, float *state, void *stream) {
+    Trace trace_("kvg_decode_attention_range");
+    if (!c || !state) return fail(KVG_ERR_ARG, "null argument");
+    if (flags & ~(uint32_t)KVG_DECODE_MERGE) return fail(KVG_ERR_ARG, "unknown flags");
+    const int32_t P = c->dims.page_size;
+    if (slot_begin < 0 || slot_end < slot_begin) return fail(KVG_ERR_ARG, "need 0 <= slot_begin <= slot_end");
+    if (slot_begin % P || (slot_end % P && slot_end < c->max_slots))
+        return fail(KVG_ERR_ARG, "slot_begin and slot_end must be multiples of page_size %d (or slot_end >= max_slots)", P);
+    const int32_t pb = slot_begin / P;
+    const int32_t pe = slot_end >= c->max_slots ? INT32_MAX : slot_end / P;
+    return decode_impl("kvg_decode_attention_range", c, layer, seq_ids, B, q, n_q_heads, nullptr, scale, stream, pb,
+                       pe, state, (flags & KVG_DECODE_MERGE) ? 1 : 0);
+}
+
+extern "C" kvg_status kvg_decode_state_finish(const float *state, int64_t n_rows, int32_t head_dim, void *out,
+                                              void *stream) {
+    Trace trace_("kvg_decode_state_finish");
+    if (n_rows < 0 || (n_rows > 0 && (!state || !out))) return fail(KVG_ERR_ARG, "null argument or negative n_rows");
+    if (head_dim != 64 && head_dim != 128 && head_dim != 256) return fail(KVG_ERR_ARG, "head_dim must be 64, 128 or 256");
+    if ((reinterpret_cast<uintptr_t>(state) | reinterpret_cast<uintptr_t>(out)) & 15)
+        return fail(KVG_ERR_ARG, "state/out must be 16-byte aligned");
+    KVG_CUDA(launch_state_finish(state, n_rows, head_dim, static_cast<__nv_bfloat16 *>(out),
+                                 static_cast<cudaStream_t>(stream)));
     return KVG_OK;
 }
 

@@ -24,6 +24,7 @@ KVG_RESIDENCY_HBM, KVG_RESIDENCY_PINNED_HOST, KVG_RESIDENCY_CACHE_POOL = 0, 1, 2
 KVG_ROPE_HALF, KVG_ROPE_INTERLEAVED = 0, 1
 KVG_GRAFT_VERIFY, KVG_GRAFT_SYNC = 1, 2
 KVG_SHA256_PLAIN, KVG_SHA256_PAGED = 0, 1
+KVG_DECODE_MERGE = 1
 KVG_KV_BF16, KVG_KV_E4M3 = 0, 1
 KVG_REPORT_MAX_PAGES = 64
 
@@ -90,6 +91,9 @@ _SIGNATURES = {
     "kvg_verify": ([_vp, _u64, _vp, _i32, _i32, _u32, _vp, _P(kvg_graft_report)], _i32),
     "kvg_decode_attention": ([_vp, _i32, _vp, _i32, _vp, _i32, _vp, ctypes.c_float, _vp], _i32),
     "kvg_decode_attention_noalloc": ([_vp, _i32, _vp, _i32, _vp, _i32, _vp, ctypes.c_float, _vp], _i32),
+    "kvg_decode_attention_range": ([_vp, _i32, _vp, _i32, _vp, _i32, ctypes.c_float, _i32, _i32, _u32, _vp, _vp],
+                                   _i32),
+    "kvg_decode_state_finish": ([_vp, _i64, _i32, _vp, _vp], _i32),
     "kvg_digest": ([_vp, _u64, _i32, _u64, _vp, _vp], _i32),
     "kvg_sync": ([_vp, _vp, ctypes.c_double, _P(kvg_graft_report)], _i32),
     "kvg_selftest_bounded_wait": ([_vp, _u64, _vp], _i32),
@@ -279,6 +283,20 @@ def kvg_decode_attention_noalloc(cache, layer: int, seq_ids, q_ptr: int, n_q_hea
     ids = (ctypes.c_int32 * len(seq_ids))(*[int(x) for x in seq_ids])
     _check(lib().kvg_decode_attention_noalloc(cache, layer, ids, len(seq_ids), q_ptr, n_q_heads, out_ptr,
                                               float(scale), _stream(stream)))
+
+
+def kvg_decode_attention_range(cache, layer: int, seq_ids, q_ptr: int, n_q_heads: int, scale: float,
+                               slot_begin: int, slot_end: int, flags: int, state_ptr: int, stream=None):
+    """Split decode over slots [slot_begin, slot_end): writes (flags 0) or merges
+    (KVG_DECODE_MERGE) the fp32 softmax state [Lrun][B][Hq][D + 4] (see kvg.h)."""
+    ids = (ctypes.c_int32 * len(seq_ids))(*[int(x) for x in seq_ids])
+    _check(lib().kvg_decode_attention_range(cache, layer, ids, len(seq_ids), q_ptr, n_q_heads, float(scale),
+                                            int(slot_begin), int(slot_end), int(flags), state_ptr, _stream(stream)))
+
+
+def kvg_decode_state_finish(state_ptr: int, n_rows: int, head_dim: int, out_ptr: int, stream=None):
+    """bf16 output o / l of a split decode's state rows."""
+    _check(lib().kvg_decode_state_finish(state_ptr, int(n_rows), int(head_dim), out_ptr, _stream(stream)))
 
 
 def kvg_digest(ptr: int, n: int, mode: int, page_bytes: int, out_ptr: int, stream=None):

@@ -522,6 +522,33 @@ def test_window_of_one_returns_the_last_value_row(oracle):
             assert np.array_equal(o[h], oracle.bf16_to_f64(v[l, -1, h // G]))
 
 
+# Split decode over a slot range: the rows written, by construction of the
+# stitched sequence, sit at slots 0..56 (rows 0..56) and 64..89 (rows 57..82).
+def _rows_of_slots(lo, hi):
+    slots = list(range(0, 57)) + list(range(64, 90))
+    return [i for i, s in enumerate(slots) if lo <= s < hi]
+
+
+@pytest.mark.parametrize("lo,hi,W", [(0, 1 << 20, 0), (0, 64, 0), (64, 1 << 20, 0), (48, 64, 0), (16, 16, 0),
+                                     (64, 80, 0), (0, 64, 30), (64, 1 << 20, 30), (0, 32, 30)])
+def test_decode_range_reads_the_rows_in_its_slots(oracle, lo, hi, W):
+    c, k, v = _stitched(oracle, 27)
+    q = syn.as_u16(syn.queries(syn.TINY, 2, 1, 28))[:, 0]
+    c.set_layer_windows([W, 0])
+    rows = _rows_of_slots(lo, hi)
+    if W:
+        rows = [r for r in rows if r >= 83 - W]
+    for l in range(2):
+        rr = rows if l == 0 else _rows_of_slots(lo, hi)
+        got = c.decode_range(0, l, q[l], 0.125, lo, hi)
+        want = oracle.gqa_decode(q[l], k[l, rr], v[l, rr], 0.125)
+        assert got.tobytes() == want.tobytes()
+        if not rr:
+            assert not got.any()
+    if (lo, hi) == (0, 1 << 20):
+        assert c.decode_range(0, 0, q[0], 0.125, lo, hi).tobytes() == c.decode(0, 0, q[0], 0.125).tobytes()
+
+
 def test_window_settings_are_checked(oracle):
     c, _, _ = _stitched(oracle, 25)
     with pytest.raises(oracle.KvgError):
