@@ -293,7 +293,10 @@ def run_kvg(args, rank, world):
     local = int(os.environ.get("LOCAL_RANK", "0"))
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
-    stream = torch.cuda.Stream(device)
+    # the main stream (append, decode) at the highest priority: the append's
+    # one CTA per SM is placed before the verified graft's queued CTAs, which
+    # shortens the window the two share (measured 6.11 -> 6.01 ms per step)
+    stream = torch.cuda.Stream(device, priority=torch.cuda.Stream.priority_range()[1])
     side = torch.cuda.Stream(device)
     hbm_peak, sm_max, peak_kind = load_peaks()
     swa = tuple(int(x) for x in args.swa.split(":")) if args.swa else None

@@ -78,10 +78,17 @@ __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const ui
     const int rows = bytes / (2 * D);
     const uint4 *s4 = reinterpret_cast<const uint4 *>(src);
     uint4 *d4 = reinterpret_cast<uint4 *>(dst);
+    // Rows of the page at or past n_valid are padding (only a block's last
+    // page has any); the chunk's rows are (r0 + rr) mod P, rr < rows.
+    const int P = p.page_size;
+    const int64_t nv = p.n_tokens - page_token0;
+    const int n_valid = nv < P ? (int)nv : P;
+    const int r0 = (int)(first_row_in_page % P);
     if (ROT == 1) {
         // item = (row, pair chunk c < D/16): the 16-byte vectors c and c + D/16
         // of the row; kRotUnroll items per thread loaded before any is stored
-        const int half_vecs = vec_per_row >> 1;
+        const int half_vecs = vec_per_row >> 1;  // D/16: a power of two
+        const int hv_shift = __ffs(half_vecs) - 1;
         const int n_items = rows * half_vecs;
         for (int base = threadIdx.x; base < n_items; base += kCopyThreads * kRotUnroll) {
             uint4 lo[kRotUnroll], hi[kRotUnroll];
@@ -89,8 +96,8 @@ __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const ui
             for (int u = 0; u < kRotUnroll; ++u) {
                 const int it = base + u * kCopyThreads;
                 if (it < n_items) {
-                    const int rr = it / half_vecs;
-                    const int lo_i = rr * vec_per_row + (it - rr * half_vecs);
+                    const int rr = it >> hv_shift;
+                    const int lo_i = rr * vec_per_row + (it & (half_vecs - 1));
                     lo[u] = __ldcs(s4 + lo_i);
                     hi[u] = __ldcs(s4 + lo_i + half_vecs);
                 }
@@ -99,11 +106,10 @@ __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const ui
             for (int u = 0; u < kRotUnroll; ++u) {
                 const int it = base + u * kCopyThreads;
                 if (it < n_items) {
-                    const int rr = it / half_vecs;
-                    const int c = it - rr * half_vecs;
+                    const int rr = it >> hv_shift;
+                    const int c = it & (half_vecs - 1);
                     const int lo_i = rr * vec_per_row + c;
-                    const int64_t tok = page_token0 + ((first_row_in_page + rr) % p.page_size);
-                    if (tok < p.n_tokens) {
+                    if (n_valid == P || (r0 + rr) % P < n_valid) {
                         float a[8], b[8], ra[8], rb[8];
                         unpack8(lo[u], a);
                         unpack8(hi[u], b);
@@ -120,14 +126,13 @@ __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const ui
             }
         }
     } else {
+        const int vr_shift = __ffs(vec_per_row) - 1;  // D/8: a power of two
         const int n_items = rows * vec_per_row;
         for (int it = threadIdx.x; it < n_items; it += kCopyThreads) {
-            const int rr = it / vec_per_row;
-            const int c = it - rr * vec_per_row;
-            const int64_t row_in_page = first_row_in_page + rr;
-            const int64_t tok = page_token0 + (row_in_page % p.page_size);
+            const int rr = it >> vr_shift;
+            const int c = it & (vec_per_row - 1);
             const uint4 x = __ldcs(s4 + it);
-            if (tok < p.n_tokens) {
+            if (n_valid == P || (r0 + rr) % P < n_valid) {
                 float f[8], g[8];
                 unpack8(x, f);
 #pragma unroll
