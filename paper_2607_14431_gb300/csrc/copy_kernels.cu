@@ -231,7 +231,7 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(const AppendPara
             for (int u = 0; u < kAppendUnroll; ++u) {
                 const int i = base + 32 * u;
                 if (i < vpt) {
-                    const int h = i / vpr, c = i - h * vpr;
+                    const int h = i >> (__ffs(vpr) - 1), c = i & (vpr - 1);  // vpr = D/8, a power of two
                     __stcs(dst + h * head_stride_vec + c, val[u]);
                 }
             }
@@ -392,7 +392,7 @@ __global__ void __launch_bounds__(kAppendThreads) append_e4m3_kernel(const Appen
             for (int u = 0; u < kAppendUnroll; ++u) {
                 const int i = base + 32 * u;
                 if (i < gpt) {
-                    const int h = i / gpr, c = i - h * gpr;
+                    const int h = i >> (__ffs(gpr) - 1), c = i & (gpr - 1);  // gpr = D/8, a power of two
                     __stcs(dst + h * (P * D / 8) + c, e4m3x8(val[u], inv));
                 }
             }
@@ -435,7 +435,7 @@ __global__ void __launch_bounds__(kAppendThreads) append_batch_e4m3_kernel(const
             for (int u = 0; u < kAppendUnroll; ++u) {
                 const int i = base + 32 * u;
                 if (i < gpt) {
-                    const int h = i / gpr, c = i - h * gpr;
+                    const int h = i >> (__ffs(gpr) - 1), c = i & (gpr - 1);  // gpr = D/8, a power of two
                     __stcs(dst + h * (P * D / 8) + c, e4m3x8(val[u], inv));
                 }
             }
@@ -471,7 +471,7 @@ __global__ void __launch_bounds__(kAppendThreads) append_batch_kernel(const Appe
                                                (((int64_t)lkv * p.pool_pages + p.pid[b]) * p.n_kv_heads) * P * D +
                                                row * D);
         for (int i = lane; i < vpt; i += 32) {
-            const int h = i / vpr, c = i - h * vpr;
+            const int h = i >> (__ffs(vpr) - 1), c = i & (vpr - 1);  // vpr = D/8, a power of two
             __stcs(dst + h * head_stride_vec + c, __ldcs(src + i));
         }
     }
