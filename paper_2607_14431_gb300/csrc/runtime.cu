@@ -268,6 +268,18 @@ static kvg_status store_alloc(kvg_store *s, uint64_t bytes, uint8_t **dev, uint8
     return KVG_OK;
 }
 
+// Gives back the most recent allocation of its slab (a block that was not
+// added after all, e.g. an import whose digests did not verify); any other
+// region stays allocated.
+static void store_unalloc(kvg_store *s, const uint8_t *dev, uint64_t bytes) {
+    for (auto &sl : s->slabs) {
+        if (dev >= sl.dev && dev + bytes == sl.dev + sl.used) {
+            sl.used = (uint64_t)(dev - sl.dev);
+            return;
+        }
+    }
+}
+
 extern "C" kvg_status kvg_store_create(const kvg_dims *dims, int32_t residency, uint64_t capacity_bytes,
                                        int32_t device, kvg_store **out) {
     if (!dims || !out) return fail(KVG_ERR_ARG, "null argument");
@@ -429,8 +441,10 @@ extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t
         DevStatus hs;
         KVG_CUDA(cudaMemcpy(&hs, s->status, sizeof hs, cudaMemcpyDeviceToHost));
         KVG_CUDA(cudaMemset(s->status, 0, sizeof(DevStatus)));
-        if (hs.n_mismatch)
+        if (hs.n_mismatch) {
+            store_unalloc(s, dev, lay.total);
             return fail(KVG_ERR_DIGEST, "import: %d digest mismatches (block not added)", hs.n_mismatch);
+        }
     }
     kvg_store::Blk b{dev, host, lay, 0, 0};
     minmax_positions(reinterpret_cast<const int32_t *>(h + lay.pos_off), n_tok, &b.min_pos, &b.max_pos);
@@ -657,6 +671,7 @@ static kvg_status pool_import(kvg_store *s, const uint8_t *h, const BlockLayout 
         KVG_CUDA(cudaMemset(s->status, 0, sizeof(DevStatus)));
         if (hs.n_mismatch) {
             pool_unpin(c, pids);
+            store_unalloc(s, meta, pool_meta_bytes(lay));
             return fail(KVG_ERR_DIGEST, "import: %d digest mismatches (block not added)", hs.n_mismatch);
         }
     }

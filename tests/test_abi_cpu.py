@@ -40,6 +40,11 @@ def test_host_checks_reject_bad_geometry_without_a_gpu(lib):
     assert lib.kvg_store_create(None, 0, 1 << 20, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
     assert lib.kvg_graft(None, 0, None, 0, -1, 0, 0, None, None) == kvg.KVG_ERR_ARG
     assert lib.kvg_decode_attention(None, 0, None, 1, None, 4, None, ctypes.c_float(1.0), None) == kvg.KVG_ERR_ARG
+    assert lib.kvg_decode_attention_range(None, 0, None, 1, None, 4, ctypes.c_float(1.0), 0, 16, 0, None,
+                                          None) == kvg.KVG_ERR_ARG
+    assert lib.kvg_decode_state_finish(None, 4, 96, None, None) == kvg.KVG_ERR_ARG
+    assert lib.kvg_decode_state_finish(None, -1, 64, None, None) == kvg.KVG_ERR_ARG
+    assert lib.kvg_decode_state_finish(None, 0, 64, None, None) == kvg.KVG_OK  # nothing to do
 
 
 def test_host_checks_reject_bad_fp8_dims_without_a_gpu(lib):

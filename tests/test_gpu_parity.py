@@ -392,6 +392,30 @@ def test_verify_detects_a_flipped_byte(oracle):
     kvg.kvg_sync(s["dst"].h)
 
 
+@pytest.mark.parametrize("residency", [0, 1])
+def test_failed_import_gives_back_its_store_space(oracle, residency):
+    """A block whose digests do not verify is not added, and the store space
+    it was copied into is free again: a store with room for exactly one block
+    refuses the corrupted copy and then takes the intact one."""
+    kvg = need_gpu()
+    w = geometry("tiny")
+    s = _build_both(kvg, oracle, w, 100, 0, seed=53)
+    good = kvg.kvg_store_export(s["store"].h, s["bid"])
+    bad = bytearray(good)
+    info = kvg.kvg_store_block_info(s["store"].h, s["bid"])
+    bad[info.pages_offset + 7] ^= 0x01
+    small = kvg.Store(s["dims"], residency, len(good))
+    for _ in range(3):
+        with pytest.raises(kvg.KvgError) as e:
+            kvg.kvg_store_import(small.h, bytes(bad), kvg.KVG_GRAFT_VERIFY)
+        assert e.value.status == kvg.KVG_ERR_DIGEST
+    bid = kvg.kvg_store_import(small.h, good, kvg.KVG_GRAFT_VERIFY)
+    assert kvg.kvg_store_export(small.h, bid) == good
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_store_import(small.h, good, 0)
+    assert e.value.status == kvg.KVG_ERR_CAPACITY
+
+
 @pytest.mark.parametrize("hkv,P", [(3, 7), (1, 33), (4, 64)], ids=["2688B_page", "4224B_page", "64KiB_page"])
 def test_fused_verified_graft(oracle, hkv, P):
     """A verified own-position graft copies and hashes in one pass.  Pages of
@@ -471,11 +495,12 @@ def test_host_store_verified_graft_reports_the_bad_page(oracle, geo, nb, bad):
     kvg.kvg_sync(s["dst"].h)
 
 
-@pytest.mark.parametrize("geo", ["tiny", "d128"])
-def test_graft_batch_equals_sequential_grafts(oracle, geo):
+@pytest.mark.parametrize("geo,residency", [("tiny", 0), ("d128", 0), ("d128", 1)])
+def test_graft_batch_equals_sequential_grafts(oracle, geo, residency):
     """kvg_graft_batch: blocks of several lengths (ragged ones too) into
-    sequences that repeat, stitched page-aligned in call order, in one launch:
-    pool bytes, page tables, fills and positions equal the oracle's sequential
+    sequences that repeat, stitched page-aligned in call order, in one launch
+    (from an HBM store, or from a pinned-host store on a capped grid): pool
+    bytes, page tables, fills and positions equal the oracle's sequential
     grafts; with verification every graft is checked; a batch that does not
     fit changes nothing."""
     kvg = need_gpu()
@@ -485,7 +510,7 @@ def test_graft_batch_equals_sequential_grafts(oracle, geo):
     od = oracle_dims(oracle, w)
     lens = [3 * P, 2 * P + 5, P - 3, 4 * P + 1, 7]
     src = kvg.Cache(dims, 64, 1, 8 * P)
-    store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, HBM_CAP)
+    store = kvg.Store(dims, residency, HBM_CAP)
     bids, oblks = [], []
     for i, n in enumerate(lens):
         k, v = _kv(w, n, 160 + i)
