@@ -50,13 +50,30 @@ template <>
 struct TileShape<64> {
     static constexpr int TOK = 64, STAGES = 3;
 };
+// Tile rows and ring stages per head_dim (compile-time knobs, measured on
+// the GB300 decode of the 31B and 12B shapes): head_dim 128, 64 rows x 2
+// stages, 3 warps per SM (7.11 ms for batch 8 x 65,536 rows x 12 layers,
+// against 7.36 with 32 x 3 and 7.22 with 16 x 2); head_dim 256, 16 rows x 3
+// stages, 4 warps per SM (32 x 2 ties; 16 x 2, 16 x 4, 32 x 3, 64 x 2 slower).
+#ifndef KVG_DEC128_TOK
+#define KVG_DEC128_TOK 64
+#endif
+#ifndef KVG_DEC128_STAGES
+#define KVG_DEC128_STAGES 2
+#endif
+#ifndef KVG_DEC256_TOK
+#define KVG_DEC256_TOK 16
+#endif
+#ifndef KVG_DEC256_STAGES
+#define KVG_DEC256_STAGES 3
+#endif
 template <>
 struct TileShape<128> {
-    static constexpr int TOK = 32, STAGES = 3;
+    static constexpr int TOK = KVG_DEC128_TOK, STAGES = KVG_DEC128_STAGES;
 };
 template <>
 struct TileShape<256> {
-    static constexpr int TOK = 16, STAGES = 3;
+    static constexpr int TOK = KVG_DEC256_TOK, STAGES = KVG_DEC256_STAGES;
 };
 
 // FP8: the pool holds E4M3 codes; TMA brings boxes of 128 one-byte columns.
