@@ -830,6 +830,72 @@ def cpu_baseline(n_layers_sample=48):
                       f"append, fp64 decode of 16 heads over 32768 rows), in 4-layer chunks: {dt:.2f} s"}
 
 
+def run_files(args):
+    """Block files (the paper's persistent medium): the 12B block (3.2 GB) is
+    saved to a file and loaded back, into an HBM store and into a pinned-host
+    store, with and without the digest check, each timed over --steps
+    transfers.  The file stays in the page cache (as in the paper's restore
+    timings); the reads and writes are host-memory copies."""
+    import tempfile
+    from paper_2607_14431_gb300 import build
+    build.build()
+    from paper_2607_14431_gb300 import kvg
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    stream, side = torch.cuda.Stream(device), torch.cuda.Stream(device)
+    st = Step12B(kvg, device, stream, side)
+    digest = bytes(kvg.kvg_store_block_info(st.store.h, st.bid).block_digest)
+    tmp = tempfile.mkdtemp(prefix="kvg_files_")
+    path = os.path.join(tmp, "block.kvg")
+    kvg.kvg_store_save(st.store.h, st.bid, path)
+    size = os.path.getsize(path)
+
+    n = max(3, min(args.steps, 8))
+    parts = {}
+    # one store per residency with room for every load: its first (untimed)
+    # load allocates the bounce buffers; each timed load adds a block (and
+    # allocates that block's slab, which is part of a store's growth)
+    for name, res, flags in (("load_hbm_verified", kvg.KVG_RESIDENCY_HBM, kvg.KVG_GRAFT_VERIFY),
+                             ("load_hbm", kvg.KVG_RESIDENCY_HBM, 0),
+                             ("load_pinned_host_verified", kvg.KVG_RESIDENCY_PINNED_HOST, kvg.KVG_GRAFT_VERIFY),
+                             ("load_pinned_host", kvg.KVG_RESIDENCY_PINNED_HOST, 0)):
+        store = kvg.Store(st.dims, res, (n + 1) * (size + (1 << 20)))
+        kvg.kvg_store_load(store.h, path, flags)
+        ts = []
+        for _ in range(n):
+            t0 = time.perf_counter()
+            bid = kvg.kvg_store_load(store.h, path, flags)
+            ts.append(time.perf_counter() - t0)
+            assert bytes(kvg.kvg_store_block_info(store.h, bid).block_digest) == digest
+        store.close()
+        sec = statistics.median(ts)
+        parts[name] = {"ms": round(sec * 1e3, 2), "gbs": round(size / sec / 1e9, 2)}
+    # saves: each to a new file, removed outside the timed region
+    for name, store, bid in (("save_from_hbm", st.store.h, st.bid), ("save_from_pinned_host", st.hstore.h, st.hbid)):
+        ts = []
+        for k in range(n + 1):
+            out = os.path.join(tmp, f"save{k}.kvg")
+            t0 = time.perf_counter()
+            kvg.kvg_store_save(store, bid, out)
+            if k:
+                ts.append(time.perf_counter() - t0)
+            os.remove(out)
+        sec = statistics.median(ts)
+        parts[name] = {"ms": round(sec * 1e3, 2), "gbs": round(size / sec / 1e9, 2)}
+    os.remove(path)
+    os.rmdir(tmp)
+    v = parts["load_hbm_verified"]
+    line = {"metric": "block file -> HBM store GB/s (digest-verified load of the 12b block, page cache warm)",
+            "value": v["gbs"], "unit": "GB/s", "n_gpus": 1, "steps": n, "warmup": args.warmup,
+            "ms_per_step": v["ms"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "u8", "data": "synthetic",
+            "config": {"workload": f"block files: the 12b block ({size} bytes) saved and loaded back; reads "
+                                   f"in 16 MiB chunks by up to 8 threads, HBM stores through pinned bounce "
+                                   f"buffers", "cores": len(os.sched_getaffinity(0))},
+            "parts": parts}
+    print(json.dumps(line), flush=True)
+
+
 def config_12b(n_layers=48, world=1, pool_store=False, swa=None, kv="bf16"):
     """The 12b workload's config entry, shared by both arms of the bench."""
     return {"workload": f"12b-single-graft: L{n_layers} Hq16/Hkv8 D256 P64, 8192-token block grafted "
@@ -868,7 +934,7 @@ def main():
     ap.add_argument("--cpu-baseline-layers", type=int, default=48)
     ap.add_argument("--layers", type=int, default=0, help="layer count override (small profiling cases)")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--config", default="12b", choices=["12b", "31b", "batched", "deep"])
+    ap.add_argument("--config", default="12b", choices=["12b", "31b", "batched", "deep", "files"])
     ap.add_argument("--schedule", default="fused", choices=["overlap", "fused"],
                     help="12b step: digest check on a side stream after the graft (overlap) or folded "
                          "into the graft, which runs beside the append (fused)")
@@ -888,6 +954,10 @@ def main():
     if args.impl == "reference":
         if rank == 0:
             print(json.dumps(run_reference(args)), flush=True)
+        return
+    if args.config == "files":
+        if rank == 0:
+            run_files(args)
         return
     if args.config != "12b":
         if rank == 0:

@@ -186,13 +186,19 @@ kvg_status kvg_store_export(kvg_store *store, uint64_t block_id, void *dst, uint
 /* Writes block `block_id` to the file `path` in the serialized layout above:
  * one plain file per block, the paper's persistent medium (Sec. 4.4) that is
  * copied between machines as is (Sec. 4.11).  Synchronous; KVG_ERR_ARG if the
- * file cannot be written. */
+ * file cannot be written.  An HBM store's block passes through two of the
+ * store's pinned 16 MiB bounce buffers (allocated by its first file transfer
+ * and kept until kvg_store_destroy), the next chunk's copy to the host
+ * overlapping the current chunk's write. */
 kvg_status kvg_store_save(kvg_store *store, uint64_t block_id, const char *path);
 
 /* Reads a block file into the store, validating it like kvg_store_import;
  * with KVG_GRAFT_VERIFY every page digest and the block digest are recomputed
- * on the GPU and compared (KVG_ERR_DIGEST: the block is not added).
- * KVG_ERR_FORMAT for a short or malformed file.  Synchronous. */
+ * on the GPU and compared (KVG_ERR_DIGEST: the block is not added and its
+ * space is given back).  KVG_ERR_FORMAT for a short or malformed file.
+ * Synchronous.  The file is read in 16 MiB chunks by up to 8 threads: into a
+ * pinned-host store directly, into an HBM store through the store's pinned
+ * bounce buffers, each chunk's copy to HBM overlapping the next reads. */
 kvg_status kvg_store_load(kvg_store *store, const char *path, uint32_t flags, uint64_t *block_id_out);
 
 /* ---------------------------------------------------------------- cache -- */

@@ -8,6 +8,7 @@
 // copy_kernels.cu, sha256_kernels.cu and attn_kernels.cu.
 #include <algorithm>
 #include <atomic>
+#include <cerrno>
 #include <cstdarg>
 #include <chrono>
 #include <cmath>
@@ -19,6 +20,10 @@
 #include <unordered_map>
 #include <thread>
 #include <vector>
+
+#include <fcntl.h>
+#include <sys/stat.h>
+#include <unistd.h>
 
 #include <nvtx3/nvToolsExt.h>
 
@@ -219,6 +224,11 @@ struct kvg_store {
     Scratch leaf;
     DevStatus *status = nullptr;
     kvg_cache *pool_cache = nullptr;  // KVG_RESIDENCY_CACHE_POOL: the cache holding the pages
+    // block-file loads into an HBM store: a pinned bounce slot, a stream and
+    // an event per reader thread (allocated by the first load)
+    std::vector<uint8_t *> bounce;
+    std::vector<cudaStream_t> load_streams;
+    std::vector<cudaEvent_t> load_events;
 };
 
 static kvg_status store_alloc(kvg_store *s, uint64_t bytes, uint8_t **dev, uint8_t **host) {
@@ -323,6 +333,9 @@ extern "C" void kvg_store_destroy(kvg_store *s) {
     }
     s->leaf.release();
     if (s->status) cudaFree(s->status);
+    for (uint8_t *b : s->bounce) cudaFreeHost(b);
+    for (cudaStream_t st : s->load_streams) cudaStreamDestroy(st);
+    for (cudaEvent_t e : s->load_events) cudaEventDestroy(e);
     delete s;
 }
 
@@ -384,11 +397,9 @@ static kvg_status pool_export(kvg_store *s, uint64_t id, uint8_t *dst);
 static kvg_status pool_import(kvg_store *s, const uint8_t *h, const BlockLayout &lay, uint32_t flags,
                               uint64_t *block_id_out);
 
-extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t n_bytes, uint32_t flags,
-                                       uint64_t *block_id_out) {
-    Trace trace_("kvg_store_import");
-    if (!s || !bytes || !block_id_out) return fail(KVG_ERR_ARG, "null argument");
-    const uint8_t *h = static_cast<const uint8_t *>(bytes);
+// Validates a serialized block header against the store's geometry and the
+// bytes available (n_bytes), and gives the block's layout.
+static kvg_status parse_block_header(const kvg_store *s, const uint8_t *h, uint64_t n_bytes, BlockLayout *out) {
     if (n_bytes < 256 || memcmp(h, "KVGBLK01", 8) != 0) return fail(KVG_ERR_FORMAT, "bad magic");
     uint32_t ver, hb;
     int32_t L, Hkv, D, P, style, dtype;
@@ -424,18 +435,18 @@ extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t
     if (n_pg != lay.n_pages || po != lay.pos_off || dof != lay.dig_off || pgo != lay.pages_off ||
         tot != lay.total || n_bytes < tot)
         return fail(KVG_ERR_FORMAT, "layout fields inconsistent");
-    DeviceGuard g(s->device);
-    if (s->pool_cache) return pool_import(s, h, lay, flags, block_id_out);
-    uint8_t *dev = nullptr, *host = nullptr;
-    kvg_status st = store_alloc(s, lay.total, &dev, &host);
-    if (st != KVG_OK) return st;
-    if (host)
-        memcpy(host, h, lay.total);
-    else
-        KVG_CUDA(cudaMemcpy(dev, h, lay.total, cudaMemcpyHostToDevice));
+    *out = lay;
+    return KVG_OK;
+}
+
+// After the block's bytes are in the store: the optional digest check (a
+// block that fails it is not added and its space is given back) and the
+// registration.  positions: host copy of the block's position tags.
+static kvg_status finish_store_add(kvg_store *s, uint8_t *dev, uint8_t *host, const BlockLayout &lay,
+                                   const int32_t *positions, uint32_t flags, uint64_t *block_id_out) {
     if (flags & KVG_GRAFT_VERIFY) {
         KVG_CUDA(cudaMemset(s->status, 0, sizeof(DevStatus)));
-        st = hash_block(s, dev, lay, true, 0);
+        kvg_status st = hash_block(s, dev, lay, true, 0);
         if (st != KVG_OK) return st;
         KVG_CUDA(cudaDeviceSynchronize());
         DevStatus hs;
@@ -447,10 +458,31 @@ extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t
         }
     }
     kvg_store::Blk b{dev, host, lay, 0, 0};
-    minmax_positions(reinterpret_cast<const int32_t *>(h + lay.pos_off), n_tok, &b.min_pos, &b.max_pos);
+    minmax_positions(positions, lay.n_tokens, &b.min_pos, &b.max_pos);
     s->blocks.push_back(b);
     *block_id_out = s->blocks.size() - 1;
     return KVG_OK;
+}
+
+extern "C" kvg_status kvg_store_import(kvg_store *s, const void *bytes, uint64_t n_bytes, uint32_t flags,
+                                       uint64_t *block_id_out) {
+    Trace trace_("kvg_store_import");
+    if (!s || !bytes || !block_id_out) return fail(KVG_ERR_ARG, "null argument");
+    const uint8_t *h = static_cast<const uint8_t *>(bytes);
+    BlockLayout lay;
+    kvg_status pst = parse_block_header(s, h, n_bytes, &lay);
+    if (pst != KVG_OK) return pst;
+    DeviceGuard g(s->device);
+    if (s->pool_cache) return pool_import(s, h, lay, flags, block_id_out);
+    uint8_t *dev = nullptr, *host = nullptr;
+    kvg_status st = store_alloc(s, lay.total, &dev, &host);
+    if (st != KVG_OK) return st;
+    if (host)
+        memcpy(host, h, lay.total);
+    else
+        KVG_CUDA(cudaMemcpy(dev, h, lay.total, cudaMemcpyHostToDevice));
+    return finish_store_add(s, dev, host, lay, reinterpret_cast<const int32_t *>(h + lay.pos_off), flags,
+                            block_id_out);
 }
 
 extern "C" kvg_status kvg_store_export(kvg_store *s, uint64_t id, void *dst, uint64_t dst_bytes) {
@@ -469,53 +501,197 @@ extern "C" kvg_status kvg_store_export(kvg_store *s, uint64_t id, void *dst, uin
     return KVG_OK;
 }
 
+// Block files are read and written in chunks of this size by up to
+// kLoadThreads threads.
+constexpr uint64_t kLoadChunk = 16ull << 20;
+constexpr unsigned kLoadThreads = 8;
+
+static bool pread_full(int fd, uint8_t *dst, uint64_t n, uint64_t off) {
+    while (n) {
+        const ssize_t r = pread(fd, dst, n, (off_t)off);
+        if (r < 0 && errno == EINTR) continue;
+        if (r <= 0) return false;
+        dst += r;
+        off += (uint64_t)r;
+        n -= (uint64_t)r;
+    }
+    return true;
+}
+
+static bool pwrite_full(int fd, const uint8_t *src, uint64_t n, uint64_t off) {
+    while (n) {
+        const ssize_t r = pwrite(fd, src, n, (off_t)off);
+        if (r < 0 && errno == EINTR) continue;
+        if (r <= 0) return false;
+        src += r;
+        off += (uint64_t)r;
+        n -= (uint64_t)r;
+    }
+    return true;
+}
+
+// One pinned bounce slot (kLoadChunk bytes), stream and event per thread of a
+// block-file transfer, kept by the store for later loads and saves.
+static kvg_status ensure_bounce(kvg_store *s, int n_thr) {
+    while ((int)s->bounce.size() < n_thr) {
+        uint8_t *b = nullptr;
+        cudaStream_t st = nullptr;
+        cudaEvent_t ev = nullptr;
+        if (cudaHostAlloc(reinterpret_cast<void **>(&b), kLoadChunk, cudaHostAllocDefault) != cudaSuccess) {
+            cudaGetLastError();
+            return fail(KVG_ERR_OOM, "pinned bounce buffer for block-file transfers");
+        }
+        s->bounce.push_back(b);
+        KVG_CUDA(cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking));
+        s->load_streams.push_back(st);
+        KVG_CUDA(cudaEventCreateWithFlags(&ev, cudaEventDisableTiming));
+        s->load_events.push_back(ev);
+    }
+    return KVG_OK;
+}
+
+static int transfer_threads(uint64_t total) {
+    const int64_t n_chunks = (int64_t)((total + kLoadChunk - 1) / kLoadChunk);
+    const unsigned hc = std::thread::hardware_concurrency();
+    return (int)std::min<int64_t>(std::max<int64_t>(n_chunks, 1), std::max(1u, std::min(hc ? hc : 1u, kLoadThreads)));
+}
+
+// Writes bytes [0, total) of a block to the open file with one writer (writes
+// to one file do not scale with threads): a pinned-host store's bytes
+// directly; an HBM store's through two pinned bounce slots, the next chunk's
+// copy to the host running while the current chunk is written.
+static kvg_status save_streamed(kvg_store *s, int fd, uint64_t total, const uint8_t *dev, const uint8_t *host) {
+    if (host) return pwrite_full(fd, host, total, 0) ? KVG_OK : fail(KVG_ERR_ARG, "short write of a block file");
+    const int64_t n_chunks = (int64_t)((total + kLoadChunk - 1) / kLoadChunk);
+    kvg_status st = ensure_bounce(s, 2);
+    if (st != KVG_OK) return st;
+    auto issue = [&](int64_t i) {
+        const uint64_t off = (uint64_t)i * kLoadChunk;
+        return cudaMemcpyAsync(s->bounce[i & 1], dev + off, std::min<uint64_t>(kLoadChunk, total - off),
+                               cudaMemcpyDeviceToHost, s->load_streams[i & 1]);
+    };
+    KVG_CUDA(issue(0));
+    for (int64_t i = 0; i < n_chunks; ++i) {
+        if (i + 1 < n_chunks) KVG_CUDA(issue(i + 1));
+        KVG_CUDA(cudaStreamSynchronize(s->load_streams[i & 1]));
+        const uint64_t off = (uint64_t)i * kLoadChunk;
+        if (!pwrite_full(fd, s->bounce[i & 1], std::min<uint64_t>(kLoadChunk, total - off), off)) {
+            KVG_CUDA(cudaStreamSynchronize(s->load_streams[(i + 1) & 1]));
+            return fail(KVG_ERR_ARG, "short write of a block file");
+        }
+    }
+    return KVG_OK;
+}
+
 extern "C" kvg_status kvg_store_save(kvg_store *s, uint64_t id, const char *path) {
     Trace trace_("kvg_store_save");
     if (!s || !path) return fail(KVG_ERR_ARG, "null argument");
     if (id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)id);
     const auto &b = s->blocks[id];
-    std::vector<uint8_t> buf;
-    const uint8_t *src = b.host;
-    if (!src) {
-        buf.resize(b.lay.total);
-        kvg_status st = kvg_store_export(s, id, buf.data(), buf.size());
-        if (st != KVG_OK) return st;
-        src = buf.data();
+    DeviceGuard g(s->device);
+    KVG_CUDA(cudaDeviceSynchronize());  // the deposit's kernels have written the block
+    const int fd = open(path, O_WRONLY | O_CREAT | O_TRUNC | O_CLOEXEC, 0644);
+    if (fd < 0) return fail(KVG_ERR_ARG, "cannot open %s for writing", path);
+    kvg_status st = KVG_OK;
+    if (s->pool_cache) {  // pool-resident blocks: gathered into host memory first
+        std::vector<uint8_t> buf(b.lay.total);
+        st = kvg_store_export(s, id, buf.data(), buf.size());
+        if (st == KVG_OK && !pwrite_full(fd, buf.data(), buf.size(), 0)) st = fail(KVG_ERR_ARG, "short write to %s", path);
     } else {
-        DeviceGuard g(s->device);
-        KVG_CUDA(cudaDeviceSynchronize());
+        st = save_streamed(s, fd, b.lay.total, b.dev, b.host);
     }
-    FILE *f = fopen(path, "wb");
-    if (!f) return fail(KVG_ERR_ARG, "cannot open %s for writing", path);
-    const size_t w = fwrite(src, 1, b.lay.total, f);
-    const int rc = fclose(f);
-    if (w != b.lay.total || rc != 0) return fail(KVG_ERR_ARG, "short write to %s", path);
+    if (close(fd) != 0 && st == KVG_OK) st = fail(KVG_ERR_ARG, "short write to %s", path);
+    return st;
+}
+
+// Reads bytes [0, total) of the open block file into the store's space: a
+// pinned-host store receives them directly (reader threads on disjoint
+// chunks); an HBM store through one pinned bounce slot per reader thread,
+// each chunk's copy to HBM on the thread's stream while the next chunk is
+// read.  Every copy has completed when this returns.
+static kvg_status stream_file(kvg_store *s, int fd, uint64_t total, uint8_t *dev, uint8_t *host) {
+    const int64_t n_chunks = (int64_t)((total + kLoadChunk - 1) / kLoadChunk);
+    const int n_thr = transfer_threads(total);
+    if (!host) {
+        kvg_status st = ensure_bounce(s, n_thr);
+        if (st != KVG_OK) return st;
+    }
+    std::atomic<int> bad{0};  // 1: a read failed, 2: a CUDA call failed
+    auto worker = [&](int w) {
+        if (!host && cudaSetDevice(s->device) != cudaSuccess) {
+            bad = 2;
+            return;
+        }
+        for (int64_t i = w; i < n_chunks && bad.load() == 0; i += n_thr) {
+            const uint64_t off = (uint64_t)i * kLoadChunk;
+            const uint64_t len = std::min<uint64_t>(kLoadChunk, total - off);
+            if (host) {
+                if (!pread_full(fd, host + off, len, off)) bad = 1;
+                continue;
+            }
+            // the slot's previous chunk has been copied before it is overwritten
+            if (i >= n_thr && cudaEventSynchronize(s->load_events[w]) != cudaSuccess) {
+                bad = 2;
+                return;
+            }
+            if (!pread_full(fd, s->bounce[w], len, off)) {
+                bad = 1;
+                return;
+            }
+            if (cudaMemcpyAsync(dev + off, s->bounce[w], len, cudaMemcpyHostToDevice, s->load_streams[w]) !=
+                    cudaSuccess ||
+                cudaEventRecord(s->load_events[w], s->load_streams[w]) != cudaSuccess) {
+                bad = 2;
+                return;
+            }
+        }
+    };
+    std::vector<std::thread> threads;
+    for (int w = 1; w < n_thr; ++w) threads.emplace_back(worker, w);
+    worker(0);
+    for (auto &t : threads) t.join();
+    if (!host)
+        for (int w = 0; w < n_thr; ++w) KVG_CUDA(cudaStreamSynchronize(s->load_streams[w]));
+    if (bad.load() == 1) return fail(KVG_ERR_FORMAT, "block file read failed");
+    if (bad.load() == 2) return fail(KVG_ERR_CUDA, "copy of a block-file chunk failed");
     return KVG_OK;
 }
 
 extern "C" kvg_status kvg_store_load(kvg_store *s, const char *path, uint32_t flags, uint64_t *block_id_out) {
     Trace trace_("kvg_store_load");
     if (!s || !path || !block_id_out) return fail(KVG_ERR_ARG, "null argument");
-    FILE *f = fopen(path, "rb");
-    if (!f) return fail(KVG_ERR_ARG, "cannot open %s", path);
+    const int fd = open(path, O_RDONLY | O_CLOEXEC);
+    if (fd < 0) return fail(KVG_ERR_ARG, "cannot open %s", path);
+    struct FdGuard {
+        int fd;
+        ~FdGuard() { close(fd); }
+    } fd_guard{fd};
+    struct stat sb;
+    if (fstat(fd, &sb) != 0) return fail(KVG_ERR_ARG, "cannot stat %s", path);
+    const uint64_t fsize = (uint64_t)sb.st_size;
     uint8_t hdr[256];
-    if (fread(hdr, 1, sizeof hdr, f) != sizeof hdr) {
-        fclose(f);
-        return fail(KVG_ERR_FORMAT, "%s: shorter than a block header", path);
+    if (fsize < 256 || !pread_full(fd, hdr, 256, 0)) return fail(KVG_ERR_FORMAT, "%s: shorter than a block header", path);
+    BlockLayout lay;
+    kvg_status st = parse_block_header(s, hdr, fsize, &lay);
+    if (st != KVG_OK) return st;
+    DeviceGuard g(s->device);
+    if (s->pool_cache) {  // the block's pages go to pool pages: read whole, then the pool import
+        std::vector<uint8_t> buf(lay.total);
+        if (!pread_full(fd, buf.data(), lay.total, 0)) return fail(KVG_ERR_FORMAT, "%s: read failed", path);
+        return pool_import(s, buf.data(), lay, flags, block_id_out);
     }
-    uint64_t total = 0;
-    memcpy(&total, hdr + 88, 8);
-    if (memcmp(hdr, "KVGBLK01", 8) != 0 || total < 256 || total > (1ull << 40)) {
-        fclose(f);
-        return fail(KVG_ERR_FORMAT, "%s: not a block file", path);
+    std::vector<int32_t> pos((size_t)lay.n_tokens);
+    if (!pread_full(fd, reinterpret_cast<uint8_t *>(pos.data()), 4ull * lay.n_tokens, lay.pos_off))
+        return fail(KVG_ERR_FORMAT, "%s: read failed", path);
+    uint8_t *dev = nullptr, *host = nullptr;
+    st = store_alloc(s, lay.total, &dev, &host);
+    if (st != KVG_OK) return st;
+    st = stream_file(s, fd, lay.total, dev, host);
+    if (st != KVG_OK) {
+        store_unalloc(s, dev, lay.total);
+        return st;
     }
-    std::vector<uint8_t> buf(total);
-    memcpy(buf.data(), hdr, 256);
-    const size_t got = fread(buf.data() + 256, 1, total - 256, f);
-    fclose(f);
-    if (got != total - 256) return fail(KVG_ERR_FORMAT, "%s: truncated (%zu of %llu bytes)", path, got + 256,
-                                        (unsigned long long)total);
-    return kvg_store_import(s, buf.data(), total, flags, block_id_out);
+    return finish_store_add(s, dev, host, lay, pos.data(), flags, block_id_out);
 }
 
 // ------------------------------------------------------------------- cache --
