@@ -281,7 +281,16 @@ kvg_status kvg_cache_release(kvg_cache *cache, int32_t seq, void *stream);
  * slot0 + n <= n_slots) with their position tags into a new block of `store`
  * (layout above), computing every page digest and the block digest on the
  * GPU.  Sec. 3.3 deposit; the block is byte-identical to one built from the
- * same rows anywhere else.  KVG_ERR_CAPACITY if the store is full. */
+ * same rows anywhere else.  KVG_ERR_CAPACITY if the store is full.
+ * Ordering: the call returns once the rows are gathered (it reads the
+ * position tags back to bound later relocations).  The page digests follow
+ * on `stream`, so work enqueued later on `stream` (a graft, a verification)
+ * sees the whole block but its block digest, which one serial SHA-256 chain
+ * computes on a library stream; kvg_store_block_info, kvg_store_export and
+ * kvg_store_save wait for it.  A pinned-host store's block is assembled and
+ * hashed in an HBM staging buffer (grown to the largest block deposited into
+ * that store) and copied out: everything but the 256-byte header in `stream`
+ * order, the header after the block digest. */
 kvg_status kvg_deposit(kvg_store *store, const kvg_cache *cache, int32_t seq, int32_t slot0,
                        int32_t n, void *stream, uint64_t *block_id_out);
 

@@ -229,6 +229,13 @@ struct kvg_store {
     std::vector<uint8_t *> bounce;
     std::vector<cudaStream_t> load_streams;
     std::vector<cudaEvent_t> load_events;
+    // deposits: the block digest (one serial SHA-256 chain) runs on its own
+    // stream after the page digests; a pinned-host store's blocks are
+    // assembled and hashed in an HBM staging buffer, then copied out
+    cudaStream_t digest_stream = nullptr;
+    cudaEvent_t pages_done = nullptr, stage_free = nullptr;
+    bool stage_used = false;
+    Scratch stage;
 };
 
 static kvg_status store_alloc(kvg_store *s, uint64_t bytes, uint8_t **dev, uint8_t **host) {
@@ -336,6 +343,10 @@ extern "C" void kvg_store_destroy(kvg_store *s) {
     for (uint8_t *b : s->bounce) cudaFreeHost(b);
     for (cudaStream_t st : s->load_streams) cudaStreamDestroy(st);
     for (cudaEvent_t e : s->load_events) cudaEventDestroy(e);
+    if (s->digest_stream) cudaStreamDestroy(s->digest_stream);
+    if (s->pages_done) cudaEventDestroy(s->pages_done);
+    if (s->stage_free) cudaEventDestroy(s->stage_free);
+    s->stage.release();
     delete s;
 }
 
@@ -379,6 +390,17 @@ static kvg_status hash_block(kvg_store *s, uint8_t *blk_dev, const BlockLayout &
     KVG_CUDA(launch_sha256_serial(blk_dev + lay.pos_off, 4ull * lay.n_tokens, dig,
                                   (uint64_t)n_pages * 32, verify ? nullptr : blk_dev + 96,
                                   verify ? blk_dev + 96 : nullptr, s->status, st));
+    return KVG_OK;
+}
+
+// Zeroes a serialized block's alignment gaps (after the position tags and
+// after the page digests): the layout defines them as zero, and reused
+// memory (a staging buffer, a slab freed and allocated again) is not.
+static kvg_status zero_block_gaps(uint8_t *base, const BlockLayout &lay, int32_t n_layers, cudaStream_t st) {
+    const uint64_t pos_end = lay.pos_off + 4ull * (uint64_t)lay.n_tokens;
+    const uint64_t dig_end = lay.dig_off + (uint64_t)n_layers * 2 * (uint64_t)lay.n_pages * 32;
+    if (lay.dig_off > pos_end) KVG_CUDA(cudaMemsetAsync(base + pos_end, 0, lay.dig_off - pos_end, st));
+    if (lay.pages_off > dig_end) KVG_CUDA(cudaMemsetAsync(base + dig_end, 0, lay.pages_off - dig_end, st));
     return KVG_OK;
 }
 
@@ -1158,6 +1180,8 @@ static kvg_status pool_deposit(kvg_store *s, kvg_cache *c, int32_t seq, int32_t 
     hp.dst = meta;
     build_header(hp.bytes, s->dims, lay);
     KVG_CUDA(launch_write_header(hp, st));
+    stt = zero_block_gaps(meta, lay, s->dims.n_layers, st);
+    if (stt != KVG_OK) return stt;
     const int64_t P = c->dims.page_size;
     const auto &sp = c->seq_pages[seq];
     const int64_t j_first = slot0 / P;
@@ -1216,20 +1240,40 @@ extern "C" kvg_status kvg_deposit(kvg_store *s, const kvg_cache *cc, int32_t seq
         if (s->pool_cache != c) return fail(KVG_ERR_ARG, "a pool-resident store deposits from its own cache");
         return pool_deposit(s, c, seq, slot0, n, lay, static_cast<cudaStream_t>(stream), block_id_out);
     }
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (!s->digest_stream) {
+        KVG_CUDA(cudaStreamCreateWithFlags(&s->digest_stream, cudaStreamNonBlocking));
+        KVG_CUDA(cudaEventCreateWithFlags(&s->pages_done, cudaEventDisableTiming));
+        KVG_CUDA(cudaEventCreateWithFlags(&s->stage_free, cudaEventDisableTiming));
+    }
     uint8_t *dev = nullptr, *host = nullptr;
     kvg_status stt = store_alloc(s, lay.total, &dev, &host);
     if (stt != KVG_OK) return stt;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // where the block is assembled and hashed: in place in an HBM store; for
+    // a pinned-host store in the HBM staging buffer (hashing host memory over
+    // the link is slow), copied out at the end
+    uint8_t *tgt = dev;
+    if (host) {
+        if (s->stage_used) KVG_CUDA(cudaStreamWaitEvent(st, s->stage_free, 0));  // the last deposit's copy-out
+        cudaError_t e = s->stage.ensure(lay.total);
+        if (e != cudaSuccess) {
+            store_unalloc(s, dev, lay.total);
+            return cuda_fail(e, "deposit staging buffer");
+        }
+        tgt = static_cast<uint8_t *>(s->stage.ptr);
+    }
     HeaderParams hp;
-    hp.dst = dev;
+    hp.dst = tgt;
     build_header(hp.bytes, s->dims, lay);
     KVG_CUDA(launch_write_header(hp, st));
+    stt = zero_block_gaps(tgt, lay, s->dims.n_layers, st);
+    if (stt != KVG_OK) return stt;
     const auto &sp = c->seq_pages[seq];
     const int64_t j_first = slot0 / P;
     for (int64_t base = 0; base < lay.n_pages; base += kMaxPagesPerLaunch) {
         GatherParams p{};
         p.pool = c->pool;
-        p.dst = dev + lay.pages_off;
+        p.dst = tgt + lay.pages_off;
         p.page_bytes = c->page_bytes;
         p.pool_pages = c->n_pages;
         p.n_layers = c->dims.n_layers;
@@ -1241,20 +1285,43 @@ extern "C" kvg_status kvg_deposit(kvg_store *s, const kvg_cache *cc, int32_t seq
         p.head_dim = c->dims.head_dim;
         p.n_tokens = n;
         p.src_pos = c->positions + (int64_t)seq * c->max_slots + slot0 + base * P;
-        p.dst_pos = reinterpret_cast<int32_t *>(dev + lay.pos_off) + base * P;
+        p.dst_pos = reinterpret_cast<int32_t *>(tgt + lay.pos_off) + base * P;
         p.pids.n = p.npb;
         for (int32_t i = 0; i < p.npb; ++i) p.pids.pid[i] = sp[j_first + base + i];
         KVG_CUDA(launch_gather(p, s->n_sm, st));
     }
-    stt = hash_block(s, dev, lay, false, st);
-    if (stt != KVG_OK) return stt;
-    KVG_CUDA(cudaStreamSynchronize(st));
-    kvg_store::Blk b{dev, host, lay, 0, 0};
+    // the position tags bound later relocations (host-side checks): read once
     std::vector<int32_t> pos(n);
-    if (host)
-        memcpy(pos.data(), host + lay.pos_off, 4ull * n);
-    else
-        KVG_CUDA(cudaMemcpy(pos.data(), dev + lay.pos_off, 4ull * n, cudaMemcpyDeviceToHost));
+    KVG_CUDA(cudaMemcpyAsync(pos.data(), tgt + lay.pos_off, 4ull * n, cudaMemcpyDeviceToHost, st));
+    KVG_CUDA(cudaStreamSynchronize(st));
+    // page digests on the caller's stream; the block digest (one serial chain
+    // over the position tags and every page digest) on the store's digest
+    // stream, so the call does not wait for it and consecutive deposits
+    // overlap it.  Everything that reads a block digest (block info, export,
+    // save) synchronizes the device first.
+    const kvg_dims &d = s->dims;
+    const uint64_t pb = page_bytes_of(d);
+    const int64_t m = (int64_t)((pb + kLeafBytes - 1) / kLeafBytes);
+    const int64_t n_pages = (int64_t)d.n_layers * 2 * lay.n_pages;
+    KVG_CUDA(s->leaf.ensure((size_t)n_pages * m * 32));
+    PageSource src{tgt + lay.pages_off, pb, nullptr, 1, 0};
+    uint32_t *leaf = static_cast<uint32_t *>(s->leaf.ptr);
+    KVG_CUDA(launch_sha256_leaves(src, n_pages, leaf, s->n_sm, st));
+    KVG_CUDA(launch_sha256_pages(leaf, n_pages, m, tgt + lay.dig_off, nullptr, s->status, -1, st));
+    KVG_CUDA(cudaEventRecord(s->pages_done, st));
+    KVG_CUDA(cudaStreamWaitEvent(s->digest_stream, s->pages_done, 0));
+    KVG_CUDA(launch_sha256_serial(tgt + lay.pos_off, 4ull * n, tgt + lay.dig_off, (uint64_t)n_pages * 32, tgt + 96,
+                                  nullptr, s->status, s->digest_stream));
+    if (host) {
+        // everything but the header follows the page digests on the caller's
+        // stream; the header (with the block digest) follows the digest
+        KVG_CUDA(cudaMemcpyAsync(host + lay.pos_off, tgt + lay.pos_off, lay.total - lay.pos_off,
+                                 cudaMemcpyDeviceToHost, st));
+        KVG_CUDA(cudaMemcpyAsync(host, tgt, lay.pos_off, cudaMemcpyDeviceToHost, s->digest_stream));
+        KVG_CUDA(cudaEventRecord(s->stage_free, s->digest_stream));
+        s->stage_used = true;
+    }
+    kvg_store::Blk b{dev, host, lay, 0, 0};
     minmax_positions(pos.data(), n, &b.min_pos, &b.max_pos);
     s->blocks.push_back(b);
     *block_id_out = s->blocks.size() - 1;

@@ -32,13 +32,19 @@ __device__ __forceinline__ uint32_t rotr(uint32_t x, int n) { return __funnelshi
 // Additions written as a*one + b and right shifts written as the high word of
 // a*2^(32-n) execute as IMAD on the FMA pipe.  `one` is a kernel argument
 // (always 1) so the compiler cannot fold the multiply back into an add.
+// FMA = false: plain additions and shifts (the compiler fuses them into
+// 3-input IADD3 on the ALU pipe) for a serial chain, where the dependency
+// chain's latency, not pipe throughput, sets the pace.
+template <bool FMA = true>
 __device__ __forceinline__ uint32_t fadd(uint32_t a, uint32_t b, uint32_t one) {
+    if (!FMA) return a + b;
     uint32_t d;
     asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(one), "r"(b));
     return d;
 }
-template <int N>
+template <int N, bool FMA = true>
 __device__ __forceinline__ uint32_t fshr(uint32_t x, uint32_t one) {
+    if (!FMA) return x >> N;
     uint32_t d;
     asm("mul.hi.u32 %0, %1, %2;" : "=r"(d) : "r"(x), "r"(one << (32 - N)));
     return d;
@@ -50,6 +56,7 @@ __device__ __forceinline__ uint32_t bswap(uint32_t x) { return __byte_perm(x, 0,
 // message schedule kept as a rolling 16-word window.  Rotations and logic
 // stay on the ALU pipe; additions and the schedule's plain shifts go to the
 // FMA pipe (fadd/fshr), balancing the two.
+template <bool FMA = true>
 __device__ __forceinline__ void compress(uint32_t st[8], uint32_t w[16], uint32_t one) {
     uint32_t a = st[0], b = st[1], c = st[2], d = st[3], e = st[4], f = st[5], g = st[6], h = st[7];
 #pragma unroll
@@ -59,23 +66,23 @@ __device__ __forceinline__ void compress(uint32_t st[8], uint32_t w[16], uint32_
             wt = w[t];
         } else {
             const uint32_t w15 = w[(t - 15) & 15], w2 = w[(t - 2) & 15];
-            const uint32_t s0 = rotr(w15, 7) ^ rotr(w15, 18) ^ fshr<3>(w15, one);
-            const uint32_t s1 = rotr(w2, 17) ^ rotr(w2, 19) ^ fshr<10>(w2, one);
-            wt = w[t & 15] = fadd(fadd(w[t & 15], s0, one), fadd(w[(t - 7) & 15], s1, one), one);
+            const uint32_t s0 = rotr(w15, 7) ^ rotr(w15, 18) ^ fshr<3, FMA>(w15, one);
+            const uint32_t s1 = rotr(w2, 17) ^ rotr(w2, 19) ^ fshr<10, FMA>(w2, one);
+            wt = w[t & 15] = fadd<FMA>(fadd<FMA>(w[t & 15], s0, one), fadd<FMA>(w[(t - 7) & 15], s1, one), one);
         }
         const uint32_t S1 = rotr(e, 6) ^ rotr(e, 11) ^ rotr(e, 25);
         const uint32_t ch = (e & f) ^ (~e & g);
-        const uint32_t T1 = fadd(fadd(h, S1, one), fadd(fadd(ch, kK[t], one), wt, one), one);
+        const uint32_t T1 = fadd<FMA>(fadd<FMA>(h, S1, one), fadd<FMA>(fadd<FMA>(ch, kK[t], one), wt, one), one);
         const uint32_t S0 = rotr(a, 2) ^ rotr(a, 13) ^ rotr(a, 22);
         const uint32_t maj = (a & b) ^ (a & c) ^ (b & c);
         h = g;
         g = f;
         f = e;
-        e = fadd(d, T1, one);
+        e = fadd<FMA>(d, T1, one);
         d = c;
         c = b;
         b = a;
-        a = fadd(T1, fadd(S0, maj, one), one);
+        a = fadd<FMA>(T1, fadd<FMA>(S0, maj, one), one);
     }
     st[0] += a;
     st[1] += b;
@@ -271,7 +278,7 @@ __global__ void __launch_bounds__(128) sha256_pages_kernel(const uint32_t *__res
             w[4 * q + 2] = x.z;
             w[4 * q + 3] = x.w;
         }
-        compress(st, w, one);
+        compress<false>(st, w, one);
     }
     {
         uint32_t w[16];
@@ -283,7 +290,7 @@ __global__ void __launch_bounds__(128) sha256_pages_kernel(const uint32_t *__res
         const uint64_t bits = (uint64_t)m * 32ull * 8ull;
         w[14] = (uint32_t)(bits >> 32);
         w[15] = (uint32_t)bits;
-        compress(st, w, one);
+        compress<false>(st, w, one);
     }
     uint8_t dg[32];
 #pragma unroll
@@ -329,7 +336,7 @@ struct Stream {
     __device__ void byte(uint8_t x) {
         w[fill >> 2] |= (uint32_t)x << (24 - 8 * (fill & 3));
         if (++fill == 64) {
-            compress(st, w, one);
+            compress<false>(st, w, one);
             fill = 0;
 #pragma unroll
             for (int i = 0; i < 16; ++i) w[i] = 0;
@@ -343,7 +350,7 @@ struct Stream {
             const uint32_t *q = reinterpret_cast<const uint32_t *>(ptr + k);
 #pragma unroll
             for (int i = 0; i < 16; ++i) w[i] = bswap(q[i]);
-            compress(st, w, one);
+            compress<false>(st, w, one);
 #pragma unroll
             for (int i = 0; i < 16; ++i) w[i] = 0;
             k += 64;
@@ -364,14 +371,67 @@ struct Stream {
     }
 };
 
-__global__ void sha256_serial_kernel(const uint8_t *seg0, uint64_t n0, const uint8_t *seg1,
-                                     uint64_t n1, uint8_t *out, const uint8_t *expected,
-                                     DevStatus *status, uint32_t one) {
-    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+// SHA-256 of seg0 || seg1: one serial chain, run by lane 0 of one warp.
+// When both segments are 4-byte aligned and seg0's length is a multiple of 4
+// (a block's position tags and page digests are), the 32 lanes load the next
+// 2 KiB of the message (coalesced 4-byte words) while lane 0 compresses the
+// current 2 KiB from shared memory, so the chain never waits on a load;
+// otherwise (any byte alignment) lane 0 streams the bytes itself.
+constexpr int kSerialChunkWords = 512;  // 2 KiB = 32 blocks per chunk
+
+__device__ __forceinline__ uint32_t msg_word(const uint8_t *seg0, uint64_t n0, const uint8_t *seg1, uint64_t i) {
+    const uint64_t off = 4 * i;
+    return off < n0 ? *reinterpret_cast<const uint32_t *>(seg0 + off)
+                    : *reinterpret_cast<const uint32_t *>(seg1 + (off - n0));
+}
+
+__global__ void __launch_bounds__(32) sha256_serial_kernel(const uint8_t *seg0, uint64_t n0, const uint8_t *seg1,
+                                                           uint64_t n1, uint8_t *out, const uint8_t *expected,
+                                                           DevStatus *status, uint32_t one) {
+    __shared__ uint32_t buf[2][kSerialChunkWords];
+    const int lane = threadIdx.x;
+    if (blockIdx.x != 0) return;
+    const uint64_t total = n0 + n1;
+    const bool fast = !((reinterpret_cast<uintptr_t>(seg0) | reinterpret_cast<uintptr_t>(seg1) | n0) & 3);
+    const uint64_t n_chunks = fast ? total / (4 * kSerialChunkWords) : 0;
     Stream s;
-    s.init(one);
-    if (n0) s.feed(seg0, n0);
-    if (n1) s.feed(seg1, n1);
+    if (lane == 0) s.init(one);
+    if (n_chunks) {
+        for (int k = 0; k < kSerialChunkWords / 32; ++k)
+            buf[0][lane + 32 * k] = msg_word(seg0, n0, seg1, lane + 32 * k);
+        __syncwarp();
+        for (uint64_t c = 0; c < n_chunks; ++c) {
+            uint32_t nxt[kSerialChunkWords / 32];
+            const bool more = c + 1 < n_chunks;
+            if (more) {
+#pragma unroll
+                for (int k = 0; k < kSerialChunkWords / 32; ++k)
+                    nxt[k] = msg_word(seg0, n0, seg1, (c + 1) * kSerialChunkWords + lane + 32 * k);
+            }
+            if (lane == 0) {
+                const uint32_t *cur = buf[c & 1];
+                for (int b = 0; b < kSerialChunkWords / 16; ++b) {
+                    uint32_t w[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) w[i] = bswap(cur[16 * b + i]);
+                    compress<false>(s.st, w, one);
+                }
+            }
+            __syncwarp();
+            if (more) {
+#pragma unroll
+                for (int k = 0; k < kSerialChunkWords / 32; ++k) buf[(c + 1) & 1][lane + 32 * k] = nxt[k];
+            }
+            __syncwarp();
+        }
+    }
+    if (lane != 0) return;
+    // the rest of the message (and all of it on the byte path)
+    const uint64_t done = n_chunks * 4 * kSerialChunkWords;
+    s.total = done;
+    if (done < n0) s.feed(seg0 + done, n0 - done);
+    const uint64_t d1 = done > n0 ? done - n0 : 0;
+    if (d1 < n1) s.feed(seg1 + d1, n1 - d1);
     uint8_t dg[32];
     s.final(dg);
     if (out)

@@ -774,6 +774,30 @@ def test_block_file_loads_in_chunks(oracle, tmp_path, residency):
     kvg.kvg_sync(s["dst"].h)
 
 
+@pytest.mark.parametrize("residency", [0, 1])
+def test_consecutive_deposits_serialize_exactly(oracle, residency):
+    """Deposits of different lengths into one store, back to back (a
+    pinned-host store reuses its HBM staging buffer): each block's bytes,
+    including the zero gaps after its position tags and page digests, equal
+    the oracle's serialization, and its block digest is written even though
+    the call does not wait for it."""
+    kvg = need_gpu()
+    w = geometry("d128")
+    lens = [1000, 37, 333, 64]
+    k, v = _kv(w, max(lens), 141)
+    dims = dims_for(kvg, w)
+    od = oracle_dims(oracle, w)
+    src = kvg.Cache(dims, 64, 1, _slots(w, max(lens)))
+    append(kvg, src, 0, k, v, syn.positions(0, max(lens)))
+    store = kvg.Store(dims, residency, HBM_CAP)
+    bids = [kvg.kvg_deposit(store.h, src.h, 0, 0, n) for n in lens]
+    for n, bid in zip(lens, bids):
+        oblk = oracle.block_from_kv(od, np.ascontiguousarray(k[:, :n]), np.ascontiguousarray(v[:, :n]),
+                                    syn.positions(0, n))
+        assert kvg.kvg_store_export(store.h, bid) == oblk.serialize()
+        assert bytes(kvg.kvg_store_block_info(store.h, bid).block_digest) == oblk.block_digest
+
+
 def test_pool_store_zero_copy_graft(oracle):
     # blocks living in the cache's own pool: a graft writes only the page
     # table (full pages shared), a ragged last page is copied, two sequences
