@@ -234,9 +234,17 @@ struct kvg_store {
     // assembled and hashed in an HBM staging buffer, then copied out
     cudaStream_t digest_stream = nullptr;
     cudaEvent_t pages_done = nullptr, stage_free = nullptr;
+    bool pages_recorded = false;  // a deposit's page hashing (which uses `leaf`) may still run
     bool stage_used = false;
     Scratch stage;
 };
+
+// The store's leaf-digest scratch is shared by deposits (which return before
+// their page hashing has run) and verified imports: its next user's stream
+// waits for the last deposit's page hashing.
+static cudaError_t wait_for_leaf_scratch(kvg_store *s, cudaStream_t st) {
+    return s->pages_recorded ? cudaStreamWaitEvent(st, s->pages_done, 0) : cudaSuccess;
+}
 
 static kvg_status store_alloc(kvg_store *s, uint64_t bytes, uint8_t **dev, uint8_t **host) {
     for (auto &sl : s->slabs) {
@@ -380,6 +388,7 @@ static kvg_status hash_block(kvg_store *s, uint8_t *blk_dev, const BlockLayout &
     const uint64_t pb = page_bytes_of(d);
     const int64_t m = (int64_t)((pb + kLeafBytes - 1) / kLeafBytes);
     const int64_t n_pages = (int64_t)d.n_layers * 2 * lay.n_pages;
+    KVG_CUDA(wait_for_leaf_scratch(s, st));
     KVG_CUDA(s->leaf.ensure((size_t)n_pages * m * 32));
     PageSource src{blk_dev + lay.pages_off, pb, nullptr, 1, 0};
     uint32_t *leaf = static_cast<uint32_t *>(s->leaf.ptr);
@@ -786,6 +795,7 @@ static kvg_status pool_hash(kvg_store *s, uint8_t *meta, const BlockLayout &lay,
     const uint64_t pb = c->page_bytes;
     const int64_t m = (int64_t)((pb + kLeafBytes - 1) / kLeafBytes);
     const int64_t n_pages = (int64_t)s->dims.n_layers * 2 * lay.n_pages;
+    KVG_CUDA(wait_for_leaf_scratch(s, st));
     KVG_CUDA(s->leaf.ensure((size_t)n_pages * m * 32));
     PageSource src{c->pool, pb, reinterpret_cast<const int32_t *>(meta + lay.pages_off), (int32_t)lay.n_pages,
                    (int64_t)c->n_pages};
@@ -1303,12 +1313,14 @@ extern "C" kvg_status kvg_deposit(kvg_store *s, const kvg_cache *cc, int32_t seq
     const uint64_t pb = page_bytes_of(d);
     const int64_t m = (int64_t)((pb + kLeafBytes - 1) / kLeafBytes);
     const int64_t n_pages = (int64_t)d.n_layers * 2 * lay.n_pages;
+    KVG_CUDA(wait_for_leaf_scratch(s, st));
     KVG_CUDA(s->leaf.ensure((size_t)n_pages * m * 32));
     PageSource src{tgt + lay.pages_off, pb, nullptr, 1, 0};
     uint32_t *leaf = static_cast<uint32_t *>(s->leaf.ptr);
     KVG_CUDA(launch_sha256_leaves(src, n_pages, leaf, s->n_sm, st));
     KVG_CUDA(launch_sha256_pages(leaf, n_pages, m, tgt + lay.dig_off, nullptr, s->status, -1, st));
     KVG_CUDA(cudaEventRecord(s->pages_done, st));
+    s->pages_recorded = true;
     KVG_CUDA(cudaStreamWaitEvent(s->digest_stream, s->pages_done, 0));
     KVG_CUDA(launch_sha256_serial(tgt + lay.pos_off, 4ull * n, tgt + lay.dig_off, (uint64_t)n_pages * 32, tgt + 96,
                                   nullptr, s->status, s->digest_stream));

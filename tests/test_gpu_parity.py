@@ -798,6 +798,37 @@ def test_consecutive_deposits_serialize_exactly(oracle, residency):
         assert bytes(kvg.kvg_store_block_info(store.h, bid).block_digest) == oblk.block_digest
 
 
+def test_deposit_then_verified_import_on_other_streams(oracle):
+    """A deposit returns before its page hashing runs; a verified import
+    into the same store, issued at once on another stream, and a second
+    deposit on a third stream still see their own leaf digests: all three
+    blocks equal the oracle's and the import verifies."""
+    kvg = need_gpu()
+    w = geometry("d256")
+    n1, n2 = 125 * w.page_size, 40 * w.page_size + 9
+    k, v = _kv(w, n1, 151)
+    dims = dims_for(kvg, w)
+    od = oracle_dims(oracle, w)
+    src = kvg.Cache(dims, 400, 1, _slots(w, n1))
+    append(kvg, src, 0, k, v, syn.positions(0, n1))
+    other = kvg.Store(dims, 0, HBM_CAP)
+    good = kvg.kvg_store_export(other.h, kvg.kvg_deposit(other.h, src.h, 0, 0, n2))
+    store = kvg.Store(dims, 0, HBM_CAP)
+    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+    torch.cuda.synchronize()
+    b1 = kvg.kvg_deposit(store.h, src.h, 0, 0, n1, sa)
+    b2 = kvg.kvg_store_import(store.h, good, kvg.KVG_GRAFT_VERIFY)
+    b3 = kvg.kvg_deposit(store.h, src.h, 0, 0, n2, sb)
+    torch.cuda.synchronize()
+    o1 = oracle.block_from_kv(od, k, v, syn.positions(0, n1)).serialize()
+    o2 = oracle.block_from_kv(od, np.ascontiguousarray(k[:, :n2]), np.ascontiguousarray(v[:, :n2]),
+                              syn.positions(0, n2)).serialize()
+    assert good == o2
+    assert kvg.kvg_store_export(store.h, b1) == o1
+    assert kvg.kvg_store_export(store.h, b2) == o2
+    assert kvg.kvg_store_export(store.h, b3) == o2
+
+
 def test_pool_store_zero_copy_graft(oracle):
     # blocks living in the cache's own pool: a graft writes only the page
     # table (full pages shared), a ragged last page is copied, two sequences
