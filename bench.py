@@ -520,6 +520,50 @@ class Step31B:
                                  self.out.data_ptr(), self.scale, s)
         if m: m[3].record(s)
 
+class StepTiny:
+    """The tiny configuration (2 layers, 4/2 heads, head_dim 64, page 16): a
+    256-token block deposited at positions 0..255; one step = own-position
+    graft with digest verification into an empty sequence + decode of one
+    query token over the 256 rows.  Launch-bound (microseconds), timed for
+    completeness (its parity with the oracle is a test)."""
+
+    def __init__(self, kvg, device, stream):
+        self.kvg, self.stream = kvg, stream
+        self.w = w = syn.TINY
+        P = w.page_size
+        self.nb = syn.TINY_BLOCK
+        self.dims = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0)
+        n_pages = 2 * (self.nb // P) + 2
+        self.cache = kvg.Cache(self.dims, n_pages, 2, self.nb)
+        self.store = kvg.Store(self.dims, kvg.KVG_RESIDENCY_HBM, 16 << 20)
+        c = self.cache.h
+        with torch.cuda.stream(stream):
+            self.k, self.v = syn.kv_rows(w, self.nb, w.seed, device)
+            pos = torch.arange(self.nb, dtype=torch.int32, device=device)
+            kvg.kvg_cache_append(c, 1, self.k.data_ptr(), self.v.data_ptr(), pos.data_ptr(), self.nb, stream)
+            self.bid = kvg.kvg_deposit(self.store.h, c, 1, 0, self.nb, stream)
+            kvg.kvg_cache_release(c, 1, stream)
+            self.q = syn.queries(w, w.n_layers, 1, w.seed, device)
+            self.out = torch.empty_like(self.q)
+        stream.synchronize()
+        self.scale = 1.0 / math.sqrt(w.head_dim)
+        blk = w.n_layers * 2 * (self.nb // P) * w.page_bytes
+        self.bytes = {"graft_verify": 2 * blk, "decode": w.n_layers * 2 * self.nb * w.n_kv_heads * w.head_dim * 2}
+        self.phases = ["release", "graft_verify", "decode"]
+
+    def run_step(self, ev=None):
+        kvg, s, c = self.kvg, self.stream, self.cache.h
+        m = ev["main"] if ev else None
+        if m: m[0].record(s)
+        kvg.kvg_cache_release(c, 0, s)
+        if m: m[1].record(s)
+        kvg.kvg_graft(self.store.h, self.bid, c, 0, -1, 0, kvg.KVG_GRAFT_VERIFY, s)
+        if m: m[2].record(s)
+        kvg.kvg_decode_attention(c, -1, [0], self.q.data_ptr(), self.w.n_q_heads, self.out.data_ptr(),
+                                 self.scale, s)
+        if m: m[3].record(s)
+
+
 class StepBatched:
     """Batched library graft on a layer slice of the 12B shape: a 512-block
     HBM store (lengths U{2048..6144}); 32 sequences each graft 4 distinct
@@ -693,7 +737,9 @@ def run_other(args):
     stream = torch.cuda.Stream(device)
     hbm_peak, sm_max, peak_kind = load_peaks()
     mk = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    if args.config == "31b":
+    if args.config == "tiny":
+        st = StepTiny(kvg, device, stream)
+    elif args.config == "31b":
         st = Step31B(kvg, device, stream, args.layers)
     elif args.config == "batched":
         st = StepBatched(kvg, device, stream, args.layers or 4)
@@ -737,7 +783,16 @@ def run_other(args):
     line = {"metric": METRIC, "unit": "GB/s", "n_gpus": 1, "steps": K, "warmup": args.warmup,
             "ms_per_step": round(ms_step, 4), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16", "data": "synthetic", "parts": parts, "gpu_launches": int(launches), "clocks": clk}
-    if args.config == "31b":
+    if args.config == "tiny":
+        line["value"] = round(step_bytes / (ms_step * 1e-3) / 1e9, 2)
+        line["config"] = {"workload": "tiny: L2 Hq4/Hkv2 D64 P16, 256-token block grafted at own positions "
+                                      "(digest-verified), decode 1 token over 256 rows; launch-bound"}
+        line["parts"]["decode"]["tokens_per_s"] = round(1e3 / statistics.mean(phase_ms["decode"]), 1)
+        first = _sha_tensor(st.out)
+        st.run_step()
+        stream.synchronize()
+        line["checks"] = {"deterministic": _sha_tensor(st.out) == first}
+    elif args.config == "31b":
         line["value"] = round(step_bytes / (ms_step * 1e-3) / 1e9, 2)
         line["config"] = {"workload": f"31b-relocation: L{st.w.n_layers} Hq32/Hkv16 D128 P64 theta 1e6, 16384-token "
                                       "block re-based by delta (0,1,4096,100000 across 8 sequences; 4096 timed), "
@@ -934,7 +989,7 @@ def main():
     ap.add_argument("--cpu-baseline-layers", type=int, default=48)
     ap.add_argument("--layers", type=int, default=0, help="layer count override (small profiling cases)")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--config", default="12b", choices=["12b", "31b", "batched", "deep", "files"])
+    ap.add_argument("--config", default="12b", choices=["12b", "tiny", "31b", "batched", "deep", "files"])
     ap.add_argument("--schedule", default="fused", choices=["overlap", "fused"],
                     help="12b step: digest check on a side stream after the graft (overlap) or folded "
                          "into the graft, which runs beside the append (fused)")
