@@ -1,0 +1,210 @@
+"""GPU edge cases against the CPU oracle: every query-group size the decode
+kernel is built for (bf16 and fp8), one-row pages, a one-token block, the
+largest decode batch, an empty append, and position tags at the top of the
+int32 range."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import kvg_synth as syn
+from kvg_testlib import (CANARY, append, compare_decode, decode, dims_for, fill_canary, need_gpu, oracle_dims,
+                         pool_u16, tables, to_dev)
+
+pytestmark = pytest.mark.gpu
+
+HBM_CAP = 1 << 30
+
+
+def _kv(w, n, seed):
+    k, v = syn.kv_rows(w, n, seed)
+    return syn.as_u16(k), syn.as_u16(v)
+
+
+# (head_dim, group, fp8): every instance of the decode kernel
+BF16_CASES = [(64, 1), (64, 4), (64, 8), (128, 1), (256, 1)]
+FP8_CASES = [(128, 1), (256, 1)]
+
+
+def _sequence_case(kvg, oracle, w, fp8=False, ks=0.0625, vs=0.125):
+    """Two sequences: a ragged block grafted then fresh rows; one row only."""
+    P = w.page_size
+    if fp8:
+        dims = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0,
+                             kv_dtype=kvg.KVG_KV_E4M3, k_scale=ks, v_scale=vs)
+        od = oracle.Dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0, oracle.KV_E4M3, ks, vs)
+    else:
+        dims, od = dims_for(kvg, w), oracle_dims(oracle, w)
+    nb, nf = 3 * P + 5, 2 * P + 3
+    k, v = _kv(w, nb + nf, 171 + w.head_dim + w.n_q_heads)
+    max_slots = 8 * P + 64
+    src = kvg.Cache(dims, 32, 1, max_slots)
+    append(kvg, src, 0, k[:, :nb], v[:, :nb], syn.positions(0, nb))
+    store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, HBM_CAP)
+    bid = kvg.kvg_deposit(store.h, src.h, 0, 0, nb)
+    c = kvg.Cache(dims, 32, 2, max_slots)
+    if fp8:
+        oc = oracle.OracleCache(od, 32, 2, max_slots)
+    else:  # both pools canary-filled, so every byte can be compared
+        fill_canary(c)
+        oc = oracle.OracleCache(od, 32, 2, max_slots, fill=CANARY)
+    kvg.kvg_graft(store.h, bid, c.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+    oc.graft(0, oracle.block_from_kv(od, k[:, :nb], v[:, :nb], syn.positions(0, nb)))
+    append(kvg, c, 0, k[:, nb:], v[:, nb:], syn.positions(nb, nf))
+    oc.append(0, k[:, nb:], v[:, nb:], syn.positions(nb, nf))
+    append(kvg, c, 1, k[:, :1], v[:, :1], syn.positions(0, 1))
+    oc.append(1, k[:, :1], v[:, :1], syn.positions(0, 1))
+    return c, oc, (src, store)
+
+
+@pytest.mark.parametrize("D,G", BF16_CASES, ids=[f"D{d}_G{g}" for d, g in BF16_CASES])
+def test_decode_every_group_size(oracle, D, G):
+    kvg = need_gpu()
+    w = syn.Workload(f"d{D}g{G}", 2, 2 * G, 2, D, 16, 10000.0, 0x61 + G)
+    c, oc, _keep = _sequence_case(kvg, oracle, w)
+    q = syn.as_u16(syn.queries(w, w.n_layers, 2, 172))
+    o = decode(kvg, c, w, [0, 1], q)
+    scale = 1.0 / math.sqrt(D)
+    for l in range(w.n_layers):
+        for b in range(2):
+            compare_decode(oracle, o[l, b], oc.decode(b, l, q[l, b], scale))
+        # one row: the softmax weight is exactly 1, so o is that value row
+        for h in range(w.n_q_heads):
+            assert np.array_equal(o[l, 1, h], oc.pool[l, 1, oc.page_table[1, 0], h // G, 0])
+    kvg.kvg_sync(c.h)
+
+
+@pytest.mark.parametrize("D,G", FP8_CASES, ids=[f"D{d}_G{g}_fp8" for d, g in FP8_CASES])
+def test_fp8_decode_every_group_size(oracle, D, G):
+    kvg = need_gpu()
+    w = syn.Workload(f"f{D}g{G}", 2, 2 * G, 2, D, 64, 10000.0, 0x71 + G)
+    c, oc, _keep = _sequence_case(kvg, oracle, w, fp8=True)
+    q = syn.as_u16(syn.queries(w, w.n_layers, 2, 173))
+    o = decode(kvg, c, w, [0, 1], q)
+    scale = 1.0 / math.sqrt(D)
+    for l in range(w.n_layers):
+        for b in range(2):
+            compare_decode(oracle, o[l, b], oc.decode(b, l, q[l, b], scale))
+    kvg.kvg_sync(c.h)
+
+
+def test_one_row_pages(oracle):
+    """page_size 1: every row its own page; grafts, appends and decode stay
+    bit-exact / within tolerance."""
+    kvg = need_gpu()
+    w = syn.Workload("p1", 2, 4, 2, 64, 1, 10000.0, 0x81)
+    c, oc, _keep = _sequence_case(kvg, oracle, w)
+    assert np.array_equal(pool_u16(c, w), oc.pool)
+    pt, pf, ps = tables(c)
+    assert np.array_equal(pt, oc.page_table) and np.array_equal(pf, oc.page_fill)
+    assert np.array_equal(ps, oc.positions)
+    q = syn.as_u16(syn.queries(w, w.n_layers, 2, 174))
+    o = decode(kvg, c, w, [0, 1], q)
+    for l in range(w.n_layers):
+        for b in range(2):
+            compare_decode(oracle, o[l, b], oc.decode(b, l, q[l, b], 0.125))
+    kvg.kvg_sync(c.h)
+
+
+def test_one_token_block(oracle):
+    """A block of one token: deposited, grafted (verified), decoded: o is its
+    value row bit for bit."""
+    kvg = need_gpu()
+    w = syn.TINY
+    dims, od = dims_for(kvg, w), oracle_dims(oracle, w)
+    k, v = _kv(w, 1, 175)
+    src = kvg.Cache(dims, 4, 1, 64)
+    append(kvg, src, 0, k, v, syn.positions(7, 1))
+    store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, HBM_CAP)
+    bid = kvg.kvg_deposit(store.h, src.h, 0, 0, 1)
+    assert kvg.kvg_store_export(store.h, bid) == oracle.block_from_kv(od, k, v, syn.positions(7, 1)).serialize()
+    c = kvg.Cache(dims, 4, 1, 64)
+    kvg.kvg_graft(store.h, bid, c.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+    assert kvg.kvg_cache_seq_info(c.h, 0) == (1, 1)
+    q = syn.as_u16(syn.queries(w, w.n_layers, 1, 176))
+    o = decode(kvg, c, w, [0], q)
+    for l in range(w.n_layers):
+        for h in range(w.n_q_heads):
+            assert np.array_equal(o[l, 0, h], v[l, 0, h // w.group])
+    kvg.kvg_sync(c.h)
+
+
+def test_largest_decode_batch(oracle):
+    """B = 4096 sequences (16 launches of 256 rows) of 1..19 rows each:
+    sampled rows match the oracle; B = 4097 is refused."""
+    kvg = need_gpu()
+    w = syn.TINY
+    P = w.page_size
+    B = 4096
+    dims, od = dims_for(kvg, w), oracle_dims(oracle, w)
+    c = kvg.Cache(dims, 2 * B + 4, B + 1, 2 * P)
+    oc = oracle.OracleCache(od, 2 * B + 4, B + 1, 2 * P)
+    k, v = _kv(w, P + 3, 177)
+    lens = [1 + (b * 5) % (P + 3) for b in range(B)]
+    kd, vd = to_dev(k), to_dev(v)  # [L][P+3][Hkv][D]: each sequence takes a prefix of rows of every layer
+    for b, n in enumerate(lens):
+        kb = kd[:, :n].contiguous()
+        vb = vd[:, :n].contiguous()
+        pb = to_dev(syn.positions(0, n))
+        kvg.kvg_cache_append(c.h, b, kb.data_ptr(), vb.data_ptr(), pb.data_ptr(), n)
+        del kb, vb, pb  # freed after the call is enqueued: later reuse is ordered after it on this stream
+        if b % 257 == 0 or b == B - 1:
+            oc.append(b, np.ascontiguousarray(k[:, :n]), np.ascontiguousarray(v[:, :n]), syn.positions(0, n))
+    torch.cuda.synchronize()
+    q = syn.as_u16(syn.queries(w, w.n_layers, B, 178))
+    o = decode(kvg, c, w, list(range(B)), q)
+    scale = 1.0 / math.sqrt(w.head_dim)
+    for b in list(range(0, B, 257)) + [B - 1]:
+        for l in range(w.n_layers):
+            compare_decode(oracle, o[l, b], oc.decode(b, l, q[l, b], scale))
+    qd = to_dev(np.zeros((w.n_layers, B + 1, w.n_q_heads, w.head_dim), np.uint16))
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_decode_attention(c.h, -1, list(range(B + 1)), qd.data_ptr(), w.n_q_heads, qd.data_ptr(), scale)
+    assert e.value.status == kvg.KVG_ERR_ARG
+    kvg.kvg_sync(c.h)
+
+
+def test_empty_append_is_a_noop(oracle):
+    kvg = need_gpu()
+    w = syn.TINY
+    c = kvg.Cache(dims_for(kvg, w), 8, 1, 64)
+    k, v = _kv(w, 5, 179)
+    append(kvg, c, 0, k, v, syn.positions(0, 5))
+    before = tables(c)
+    n0 = kvg.kvg_launch_count()
+    kvg.kvg_cache_append(c.h, 0, 0, 0, 0, 0)
+    assert kvg.kvg_launch_count() == n0
+    assert kvg.kvg_cache_seq_info(c.h, 0) == (5, 1)
+    after = tables(c)
+    assert all(np.array_equal(a, b) for a, b in zip(before, after))
+
+
+def test_positions_at_the_top_of_int32(oracle):
+    """Position tags up to 2^31 - 1 graft and relocate; one more is refused."""
+    kvg = need_gpu()
+    w = syn.TINY
+    dims, od = dims_for(kvg, w), oracle_dims(oracle, w)
+    n = 21
+    top = 2**31 - 1
+    pos = np.arange(top - 40, top - 40 + n, dtype=np.int64).astype(np.int32)  # last tag top - 20
+    k, v = _kv(w, n, 180)
+    src = kvg.Cache(dims, 8, 1, 64)
+    append(kvg, src, 0, k, v, pos)
+    store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, HBM_CAP)
+    bid = kvg.kvg_deposit(store.h, src.h, 0, 0, n)
+    c = kvg.Cache(dims, 16, 3, 64)
+    fill_canary(c)
+    oc = oracle.OracleCache(od, 16, 3, 64, fill=CANARY)
+    kvg.kvg_graft(store.h, bid, c.h, 0, -1, 0, kvg.KVG_GRAFT_SYNC)
+    oc.graft(0, oracle.block_from_kv(od, k, v, pos))
+    assert np.array_equal(pool_u16(c, w), oc.pool)  # delta 0: bit-exact
+    kvg.kvg_graft(store.h, bid, c.h, 1, -1, 20, kvg.KVG_GRAFT_SYNC)  # last tag exactly 2^31 - 1
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_graft(store.h, bid, c.h, 2, -1, 21)
+    assert e.value.status == kvg.KVG_ERR_POSITION
+    _, _, ps = tables(c)
+    assert np.array_equal(ps[0, :n], pos)
+    assert int(ps[1, n - 1]) == top and np.array_equal(ps[1, :n], (pos.astype(np.int64) + 20).astype(np.int32))
+    assert kvg.kvg_cache_seq_info(c.h, 2) == (0, 0)
+    kvg.kvg_sync(c.h)
