@@ -568,14 +568,20 @@ static kvg_status ensure_bounce(kvg_store *s, int n_thr) {
         uint8_t *b = nullptr;
         cudaStream_t st = nullptr;
         cudaEvent_t ev = nullptr;
+        // the three are kept together or not at all
         if (cudaHostAlloc(reinterpret_cast<void **>(&b), kLoadChunk, cudaHostAllocDefault) != cudaSuccess) {
             cudaGetLastError();
             return fail(KVG_ERR_OOM, "pinned bounce buffer for block-file transfers");
         }
+        cudaError_t e = cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) {
+            if (st) cudaStreamDestroy(st);
+            cudaFreeHost(b);
+            return cuda_fail(e, "stream or event for block-file transfers");
+        }
         s->bounce.push_back(b);
-        KVG_CUDA(cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking));
         s->load_streams.push_back(st);
-        KVG_CUDA(cudaEventCreateWithFlags(&ev, cudaEventDisableTiming));
         s->load_events.push_back(ev);
     }
     return KVG_OK;
