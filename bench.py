@@ -441,7 +441,8 @@ def run_kvg(args, rank, world):
                        schedule="verified graft in one pass, beside the append" if st.schedule == "fused"
                        else "graft, then the digest check beside the append and the decode"),
         "parts": parts, "roofline": roof, "e2e": e2e, "gpu_launches": int(launches),
-        "clocks": clk, "checks": {"deterministic": deterministic, "digest_verified_steps": K + args.warmup + 1,
+        "clocks": clk, "checks": {"deterministic": deterministic, "out_sha256": first_sha,
+                                  "digest_verified_steps": K + args.warmup + 1,
                                   "e2e_out_max_abs_vs_device_out": e2e_vs_device},
     }
     return line
@@ -959,7 +960,8 @@ def config_12b(n_layers=48, world=1, pool_store=False, swa=None, kv="bf16"):
                         + (f" [sliding-window layers: window {swa[0]}, every {swa[1]}th layer global]" if swa else "")
                         + (f" [fp8 E4M3 KV, scales k {syn.FP8_K_SCALE} v {syn.FP8_V_SCALE}]" if kv == "e4m3" else ""),
             "global_batch": world, "seq_len": syn.B12_CTX, "parallelism": f"replicas{world}",
-            "l2": "inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)"}
+            "l2": "inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)",
+            "seed": hex(syn.B12.seed)}
 
 
 def run_reference(args):
