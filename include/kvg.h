@@ -454,7 +454,10 @@ kvg_status kvg_decode_attention_noalloc(kvg_cache *cache, int32_t layer, const i
 /* ------------------------------------------------------------- digest -- */
 
 /* SHA-256 (FIPS 180-4) on the GPU.
- * KVG_SHA256_PLAIN: out[32] = SHA-256 of bytes[0, n) (one serial chain).
+ * KVG_SHA256_PLAIN: out[32] = SHA-256 of bytes[0, n): one serial chain, run
+ *   by one GPU thread (its 32-lane warp prefetches the message), about
+ *   1.5 us per 64-byte block (~40 MB/s) — meant for short messages such as
+ *   headers and test vectors; page contents use KVG_SHA256_PAGED.
  * KVG_SHA256_PAGED: n must be a multiple of page_bytes; out[32 * i] = the
  *   two-level digest of page i = bytes[i * page_bytes, (i+1) * page_bytes).
  * bytes and out are device pointers (or pinned host memory the GPU can
