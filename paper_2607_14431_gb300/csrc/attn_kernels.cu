@@ -76,6 +76,22 @@ struct TileShape<256> {
     static constexpr int TOK = KVG_DEC256_TOK, STAGES = KVG_DEC256_STAGES;
 };
 
+// fp8 tiles (knobs for head_dim 128 and 256).
+#ifndef KVG_FP8_128_TOK
+#define KVG_FP8_128_TOK 32
+#endif
+#ifndef KVG_FP8_256_TOK
+#define KVG_FP8_256_TOK 16
+#endif
+#ifndef KVG_FP8_STAGES
+#define KVG_FP8_STAGES 2
+#endif
+template <int D>
+struct Fp8TileShape {
+    static constexpr int TOK = D == 256 ? KVG_FP8_256_TOK : (D == 128 ? KVG_FP8_128_TOK : 64);
+    static constexpr int STAGES = KVG_FP8_STAGES;
+};
+
 // FP8: the pool holds E4M3 codes; TMA brings boxes of 128 one-byte columns.
 // Keys go from the fp8 tile straight into MMA fragments; values are expanded
 // into a 16-bit staging tile with the bf16 layout (for ldmatrix.trans).
@@ -84,8 +100,8 @@ struct TileShape<256> {
 // rings, keep HBM busy; three stages gave 0.77 of the copy peak, two 0.97)
 template <int D, bool FP8 = false>
 struct Cfg {
-    static constexpr int TOK = TileShape<D>::TOK;
-    static constexpr int STAGES = FP8 ? 2 : TileShape<D>::STAGES;
+    static constexpr int TOK = FP8 ? Fp8TileShape<D>::TOK : TileShape<D>::TOK;
+    static constexpr int STAGES = FP8 ? Fp8TileShape<D>::STAGES : TileShape<D>::STAGES;
     static constexpr int NB = D / 64;                  // 64-column 16-bit boxes per K (or V) tile
     static constexpr int BOX = TOK * 128;              // bytes of one box (TOK rows x 128 B)
     static constexpr int NB8 = FP8 ? D / 128 : 0;      // 128-column fp8 boxes per K (or V) tile
@@ -731,12 +747,12 @@ cudaError_t encode_tensor_map(CUtensorMap *out, int rank, void *base, const cuui
 cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, bool fp8, uint64_t rows) {
     const EncodeTiled encode = tensor_map_encoder();
     if (!encode) return cudaErrorSymbolNotFound;
-    const int tok = decode_tile_tokens(head_dim);
-    if (tok == 0 || rows == 0 || rows > 0x7fffffffull) return cudaErrorInvalidValue;
     if (fp8 && head_dim % 128) {  // no fp8 decode for this head_dim: nothing to map
         memset(out, 0, sizeof *out);
         return cudaSuccess;
     }
+    const int tok = decode_tile_tokens(head_dim, fp8);  // the box height the kernel for this element type expects
+    if (tok == 0 || rows == 0 || rows > 0x7fffffffull) return cudaErrorInvalidValue;
     // 128-byte rows per box: 64 bf16 columns, or 128 fp8 columns
     const cuuint64_t dims[2] = {(cuuint64_t)head_dim, (cuuint64_t)rows};
     const cuuint64_t strides[1] = {(cuuint64_t)head_dim * (fp8 ? 1 : 2)};
@@ -756,11 +772,11 @@ bool decode_supported(int head_dim, int group, bool fp8) {
     return head_dim * group <= 512;
 }
 
-int decode_tile_tokens(int head_dim) {
+int decode_tile_tokens(int head_dim, bool fp8) {
     switch (head_dim) {
-        case 64: return Cfg<64>::TOK;
-        case 128: return Cfg<128>::TOK;
-        case 256: return Cfg<256>::TOK;
+        case 64: return fp8 ? 0 : Cfg<64>::TOK;
+        case 128: return fp8 ? Cfg<128, true>::TOK : Cfg<128>::TOK;
+        case 256: return fp8 ? Cfg<256, true>::TOK : Cfg<256>::TOK;
     }
     return 0;
 }

@@ -291,7 +291,9 @@ cudaError_t launch_sha256_serial(const uint8_t *seg0, uint64_t n0, const uint8_t
 
 // Persistent decode: p.n_warps one-warp CTAs over p.n_tiles tiles, then the
 // combine over every (layer, row, query head).  decode_tile_tokens() is the
-// tile height TOK (tiles per page = ceil(P / TOK)); decode_max_warps() the
+// tile height TOK of the kernel for that element type (tiles per page =
+// ceil(P / TOK); the host plan and the tensor map's box must use the same
+// one as the kernel); decode_max_warps() the
 // number of co-resident warps the decode kernel can keep on the device.
 // Split-decode state -> bf16 output: out[r][d] = o / l (0 where l = 0), for
 // n_rows rows of D + 4 floats.
@@ -301,7 +303,7 @@ cudaError_t launch_decode(int head_dim, int group, bool fp8, const DecodeParams 
                           cudaStream_t s);
 // Tensor map of a cache pool for the decode kernel: a 2-D bf16 tensor of
 // head_dim columns and n_layers*2*n_pages*n_kv_heads*page_size rows, boxes of
-// 64 columns x decode_tile_tokens(head_dim) rows, 128-byte swizzle.
+// 64 columns x decode_tile_tokens(head_dim, fp8) rows, 128-byte swizzle.
 cudaError_t make_pool_tensor_map(CUtensorMap *out, void *pool, int head_dim, bool fp8, uint64_t rows);
 // A rank-`rank` bf16 tensor map (no swizzle, zero fill out of bounds): dims
 // innermost first, byte strides of dims 1.., box extents per dim.
@@ -309,7 +311,7 @@ cudaError_t encode_tensor_map(CUtensorMap *out, int rank, void *base, const cuui
                               const cuuint64_t *strides, const cuuint32_t *box);
 cudaError_t launch_combine(int head_dim, int group, const DecodeParams &p, cudaStream_t s);
 bool decode_supported(int head_dim, int group, bool fp8 = false);
-int decode_tile_tokens(int head_dim);
+int decode_tile_tokens(int head_dim, bool fp8);
 int decode_max_warps(int head_dim, int group, bool fp8, int n_sm);
 
 // ------------------------------------------------------------ PTX helpers --

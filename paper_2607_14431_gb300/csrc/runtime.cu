@@ -1740,7 +1740,7 @@ static kvg_status plan_decode(const kvg_cache *c, int32_t layer, const int32_t *
                               std::vector<DecodeParams> *plan, int64_t *max_units, int32_t page_begin = 0,
                               int32_t page_end = INT32_MAX) {
     const kvg_dims &d = c->dims;
-    const int TOK = decode_tile_tokens(d.head_dim);
+    const int TOK = decode_tile_tokens(d.head_dim, d.kv_dtype == KVG_KV_E4M3);
     const int tpp = (d.page_size + TOK - 1) / TOK;
     // (window, [(cache layer, q layer)]) in order of first appearance
     std::vector<std::pair<int32_t, std::vector<std::pair<int32_t, int32_t>>>> groups;
