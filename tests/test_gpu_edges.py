@@ -208,3 +208,47 @@ def test_positions_at_the_top_of_int32(oracle):
     assert int(ps[1, n - 1]) == top and np.array_equal(ps[1, :n], (pos.astype(np.int64) + 20).astype(np.int32))
     assert kvg.kvg_cache_seq_info(c.h, 2) == (0, 0)
     kvg.kvg_sync(c.h)
+
+
+_CHILD = r'''
+import hashlib, math, sys
+sys.path.insert(0, sys.argv[1])
+sys.path.insert(0, sys.argv[1] + "/tests")
+import numpy as np, torch
+import kvg_synth as syn
+from kvg_testlib import append, decode, dims_for, need_gpu
+kvg = need_gpu()
+w = syn.Workload("repro", 3, 8, 4, 128, 64, 10000.0, 0x91)
+k, v = syn.kv_rows(w, 1000, w.seed)
+k, v = syn.as_u16(k), syn.as_u16(v)
+dims = dims_for(kvg, w)
+src = kvg.Cache(dims, 64, 1, 1088)
+append(kvg, src, 0, k[:, :600], v[:, :600], syn.positions(0, 600))
+store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, 1 << 28)
+bid = kvg.kvg_deposit(store.h, src.h, 0, 0, 600)
+c = kvg.Cache(dims, 64, 1, 1088)
+kvg.kvg_cache_set_free_order(c.h, syn.permutation(64, int(sys.argv[2])))
+kvg.kvg_graft(store.h, bid, c.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+append(kvg, c, 0, np.ascontiguousarray(k[:, 600:]), np.ascontiguousarray(v[:, 600:]), syn.positions(600, 400))
+q = syn.as_u16(syn.queries(w, w.n_layers, 1, 0x92))
+o = decode(kvg, c, w, [0], q)
+print(hashlib.sha256(o.tobytes()).hexdigest())
+'''
+
+
+def test_outputs_are_identical_across_processes():
+    """The paper's gate is byte equality between separate runs: the same
+    graft + decode, run in two fresh processes (with different physical page
+    placement), gives SHA-256-identical attention output."""
+    import os
+    import subprocess
+    import sys
+    need_gpu()
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    digests = []
+    for placement_seed in (1, 2):
+        r = subprocess.run([sys.executable, "-c", _CHILD, root, str(placement_seed)], capture_output=True, text=True,
+                           timeout=600)
+        assert r.returncode == 0, r.stderr[-2000:]
+        digests.append(r.stdout.strip().splitlines()[-1])
+    assert len(digests[0]) == 64 and digests[0] == digests[1]
