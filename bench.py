@@ -938,6 +938,37 @@ def run_files(args):
             os.remove(out)
         sec = statistics.median(ts)
         parts[name] = {"ms": round(sec * 1e3, 2), "gbs": round(size / sec / 1e9, 2)}
+    # restore latency against block length, the paper's disk-to-GPU restore
+    # table's lengths (its figures include an HTTP round trip): block file ->
+    # HBM store with every digest checked -> verified graft into an empty
+    # sequence of the cache, one block length at a time
+    restore = {}
+    pb = torch.arange(st.nb, dtype=torch.int32, device=device)
+    kvg.kvg_cache_append(st.cache.h, 1, st.kb.data_ptr(), st.vb.data_ptr(), pb.data_ptr(), st.nb, stream)
+    for n_tok in (748, 1495, 2990, 5977):
+        src_store = kvg.Store(st.dims, kvg.KVG_RESIDENCY_HBM, 4 << 30)
+        bid = kvg.kvg_deposit(src_store.h, st.cache.h, 1, 0, n_tok, stream)
+        f = os.path.join(tmp, f"block_{n_tok}.kvg")
+        kvg.kvg_store_save(src_store.h, bid, f)
+        src_store.close()
+        nbytes = os.path.getsize(f)
+        # room for every load: a block takes its own slab, or a share of a 1 GiB one
+        store = kvg.Store(st.dims, kvg.KVG_RESIDENCY_HBM, (n + 1) * max(nbytes + (1 << 20), (1 << 30) + (1 << 20)))
+        kvg.kvg_store_load(store.h, f, kvg.KVG_GRAFT_VERIFY)  # untimed: the store's first transfer
+        ts = []
+        for _ in range(n):
+            kvg.kvg_cache_release(st.cache.h, 0, stream)
+            stream.synchronize()
+            t0 = time.perf_counter()
+            b2 = kvg.kvg_store_load(store.h, f, kvg.KVG_GRAFT_VERIFY)
+            kvg.kvg_graft(store.h, b2, st.cache.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, stream)
+            ts.append(time.perf_counter() - t0)
+        store.close()
+        os.remove(f)
+        restore[str(n_tok)] = {"block_bytes": nbytes, "ms": round(statistics.median(ts) * 1e3, 2)}
+    kvg.kvg_cache_release(st.cache.h, 1, stream)
+    stream.synchronize()
+    parts["restore_from_file_then_graft_verified"] = restore
     os.remove(path)
     os.rmdir(tmp)
     v = parts["load_hbm_verified"]
