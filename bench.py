@@ -879,11 +879,29 @@ def oracle_sample(n_layers_sample: int, chunk: int = 4):
     return total_t, total_b, oracle.omp_threads()
 
 
-def cpu_baseline(n_layers_sample=48):
+def oracle_single_thread(n_layers_sample=2):
+    """The oracle on one host thread (OMP_NUM_THREADS=1 in a fresh
+    interpreter, started by exec, never forked from this CUDA process)."""
+    code = ("import json, sys; sys.path.insert(0, %r); import bench; "
+            "print(json.dumps(bench.oracle_sample(%d)))" % (os.path.dirname(os.path.abspath(__file__)),
+                                                          n_layers_sample))
+    env = dict(os.environ, OMP_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=600)
+    if r.returncode != 0:
+        raise RuntimeError("single-thread oracle run failed: " + r.stderr[-2000:])
+    dt, b, threads = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": round(b / dt / 1e9, 4), "unit": "GB/s", "threads": threads,
+            "sample": f"{n_layers_sample} of 48 layers of one 12b step on one thread: {dt:.2f} s"}
+
+
+def cpu_baseline(n_layers_sample=48, single_thread_layers=2):
     dt, b, cores = oracle_sample(n_layers_sample)
-    return {"value": round(b / dt / 1e9, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
-            "sample": f"{n_layers_sample} of 48 layers of one 12b step (graft, page digests, 24576-row "
-                      f"append, fp64 decode of 16 heads over 32768 rows), in 4-layer chunks: {dt:.2f} s"}
+    out = {"value": round(b / dt / 1e9, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
+           "sample": f"{n_layers_sample} of 48 layers of one 12b step (graft, page digests, 24576-row "
+                     f"append, fp64 decode of 16 heads over 32768 rows), in 4-layer chunks: {dt:.2f} s"}
+    if single_thread_layers > 0:
+        out["single_thread"] = oracle_single_thread(single_thread_layers)
+    return out
 
 
 def run_files(args):
