@@ -1543,16 +1543,25 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
     const int64_t m = (int64_t)((c->page_bytes + kLeafBytes - 1) / kLeafBytes);
     if (verify0) KVG_CUDA(c->leaf.ensure((size_t)c->dims.n_layers * 2 * npb * m * 32));
     int64_t step = kMaxPagesPerLaunch;
+    // piped: the last chunk is short (1/64 of the block, at least a page), so
+    // that the one hash not hidden behind the link transfer is short too
+    int64_t tail = 0;
     if (piped) {
         if (!c->aux) {
             KVG_CUDA(cudaStreamCreateWithFlags(&c->aux, cudaStreamNonBlocking));
             for (cudaEvent_t &e : c->aux_ev) KVG_CUDA(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
         }
-        step = std::min<int64_t>(step, (npb + kHostVerifyChunks - 1) / kHostVerifyChunks);
+        if (npb > kHostVerifyChunks) {
+            tail = std::max<int64_t>(1, npb / 64);
+            step = std::min<int64_t>(step, (npb - tail + kHostVerifyChunks - 2) / (kHostVerifyChunks - 1));
+        } else {
+            step = 1;
+        }
     }
     int chunk = 0;
-    for (int64_t base = 0; base < npb; base += step, ++chunk) {
-        p.npb = (int32_t)std::min<int64_t>(step, npb - base);
+    for (int64_t base = 0; base < npb; base += p.npb, ++chunk) {
+        const int64_t body_end = npb - tail;
+        p.npb = (int32_t)(base < body_end ? std::min<int64_t>(step, body_end - base) : std::min<int64_t>(step, npb - base));
         p.page_base = (int32_t)base;
         p.src_pos = bpos + base * P;
         p.dst_pos = c->positions + (int64_t)seq * c->max_slots + dst + base * P;

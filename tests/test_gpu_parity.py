@@ -459,12 +459,15 @@ def test_fused_verified_graft(oracle, hkv, P):
     assert got == want
 
 
-@pytest.mark.parametrize("geo,nb,bad", [("tiny", 250, (3, 15)), ("d128", 1000, (4, 0)), ("d128", 1000, (5, 9))])
+@pytest.mark.parametrize("geo,nb,bad", [("tiny", 250, (3, 15)), ("d128", 1000, (4, 0)), ("d128", 1000, (5, 9)),
+                                        ("d128", 2583, (5, 40)), ("d128", 2583, (0, 39)), ("d128", 8320, (3, 129)),
+                                        ("d128", 8320, (2, 127))])
 def test_host_store_verified_graft_reports_the_bad_page(oracle, geo, nb, bad):
     """A verified graft from a pinned-host store copies page-range chunks and
     hashes each chunk's restored pages on a second stream: a flipped byte in
-    page (plane, j) is reported as that block page, whichever chunk holds it,
-    and an intact block grafts clean."""
+    page (plane, j) is reported as that block page, whichever chunk holds it
+    (41 and 130 pages: a short last chunk of one and two pages after the
+    equal ones), and an intact block grafts clean."""
     kvg = need_gpu()
     w = geometry(geo)
     s = _build_both(kvg, oracle, w, nb, 0, seed=61, copies=3)
