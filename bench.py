@@ -138,6 +138,10 @@ class Step12B:
         self.side = side
         self.ev_graft = torch.cuda.Event()
         self.ev_verify = torch.cuda.Event()
+        # completion events of a chunked graft (e2e step), created by one record
+        self.chunk_ev = [torch.cuda.Event() for _ in range(16)]
+        for e in self.chunk_ev:
+            e.record(side)
         self.nb, self.nf = syn.B12_BLOCK, syn.B12_CTX - syn.B12_BLOCK
         P = w.page_size
         # kv "e4m3": the cache (and so the block) holds fp8 E4M3 codes with
@@ -242,20 +246,27 @@ class Step12B:
         """The fused step with a split decode, for a block that streams in
         from a pinned-host store: the decode over the fresh rows (slots past
         the block) runs on the main stream right after the append, while the
-        verified graft is still copying the block over the host link; the part
-        over the block's slots merges in once the graft is done."""
+        verified graft is still copying the block over the host link; the
+        rows of each chunk of the graft merge in as soon as the chunk has
+        landed, and the output is finished once the whole block's digests
+        have been checked."""
         kvg, s, side, c = self.kvg, self.stream, self.side, self.cache.h
         kvg.kvg_cache_release(c, 0, s)
         self.ev_graft.record(s)
         side.wait_event(self.ev_graft)
-        kvg.kvg_graft(store, bid, c, 0, -1, 0, kvg.KVG_GRAFT_VERIFY, side)
+        ends = kvg.kvg_graft_chunked(store, bid, c, 0, [e.cuda_event for e in self.chunk_ev],
+                                     flags=kvg.KVG_GRAFT_VERIFY, stream=side)
         self.ev_verify.record(side)
         kvg.kvg_cache_append(c, 0, self.kf.data_ptr(), self.vf.data_ptr(), self.pf.data_ptr(), self.nf, s)
         kvg.kvg_decode_attention_range(c, -1, [0], self.q.data_ptr(), self.w.n_q_heads, self.scale, self.nb,
                                        syn.B12_CTX, 0, self.state.data_ptr(), s)
+        lo = 0
+        for j, hi in enumerate(ends):
+            s.wait_event(self.chunk_ev[j])
+            kvg.kvg_decode_attention_range(c, -1, [0], self.q.data_ptr(), self.w.n_q_heads, self.scale, lo, hi,
+                                           kvg.KVG_DECODE_MERGE, self.state.data_ptr(), s)
+            lo = hi
         s.wait_event(self.ev_verify)
-        kvg.kvg_decode_attention_range(c, -1, [0], self.q.data_ptr(), self.w.n_q_heads, self.scale, 0, self.nb,
-                                       kvg.KVG_DECODE_MERGE, self.state.data_ptr(), s)
         kvg.kvg_decode_state_finish(self.state.data_ptr(), self.q.numel() // self.w.head_dim, self.w.head_dim,
                                     self.out.data_ptr(), s)
 
@@ -373,8 +384,8 @@ def run_kvg(args, rank, world):
         blk_read = st.blk_pages  # block pages read from host memory by the graft
         e2e = {"value": round(world * step_bytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
                "ms_per_step": round(e2e_ms, 3),
-               "schedule": ("verified host-store graft; decode split: fresh rows during the graft, the block's "
-                            "rows after it") if split else "verified host-store graft, then the decode",
+               "schedule": ("verified host-store graft in chunks; decode split: fresh rows during the graft, "
+                            "each chunk's rows as it lands") if split else "verified host-store graft, then the decode",
                "h2d_bytes_per_step": int(blk_read + st.q.numel() * 2),
                "d2h_bytes_per_step": int(st.out.numel() * 2),
                "host_graft_gbs": None}

@@ -332,6 +332,32 @@ kvg_status kvg_graft(kvg_store *store, uint64_t block_id, kvg_cache *cache, int3
                      int32_t dst_slot, int64_t delta, uint32_t flags, void *stream,
                      kvg_graft_report *report);
 
+/* kvg_graft with a completion event per chunk of the copy, for a caller that
+ * works on the restored rows while the rest of the block is still being
+ * copied (Sec. 4.4's restore: a split decode over each chunk's slots with
+ * kvg_decode_attention_range while the next chunk crosses the host link).
+ * Same arguments, checks, effects and errors as kvg_graft, plus:
+ * events: host array of max_events (>= 1) caller-created CUDA events
+ * (cudaEvent_t, on the cache's device; timing may be disabled).  The graft
+ * copies the block in page-range chunks (one chunk for most HBM-store
+ * blocks; up to 16 for a verified graft from a pinned-host store, the last
+ * one short); chunk k of C maps to event k * E / C with E = min(max_events,
+ * C).  On KVG_OK, *n_chunks = E, and for j < E events[j] is recorded on
+ * `stream` once every chunk that maps to j has its rows (all layers, K and V)
+ * and position tags in the cache; chunk_end_slot[j] (host array of at least
+ * E) is the slot just past those rows, so event j covers slots
+ * [dst_slot, chunk_end_slot[j]) and chunk_end_slot[E - 1] = dst_slot +
+ * n_tokens.  An event does not wait for the digest check (KVG_GRAFT_VERIFY):
+ * that verdict covers the whole block and is known only when all of the
+ * call's work on `stream` is done (KVG_GRAFT_SYNC, or kvg_sync), so work
+ * started from an event must not publish its result before then.
+ * KVG_ERR_ARG if events, chunk_end_slot or n_chunks is null, an event is
+ * null, or max_events < 1. */
+kvg_status kvg_graft_chunked(kvg_store *store, uint64_t block_id, kvg_cache *cache, int32_t seq,
+                             int32_t dst_slot, int64_t delta, uint32_t flags, void *stream,
+                             kvg_graft_report *report, void *const *events, int32_t max_events,
+                             int32_t *chunk_end_slot, int32_t *n_chunks);
+
 /* A batch of own-position grafts (Sec. 3.2) in one call: graft i installs
  * block block_ids[i] into sequence seq_ids[i] at that sequence's next page
  * boundary, in order, exactly as n kvg_graft(delta = 0) calls would (a

@@ -1407,8 +1407,27 @@ static kvg_status finish_verify(kvg_cache *c, int32_t seq, uint32_t flags, int32
 // page table points at the block's full pages (shared, read-only: appends
 // never write a full page); a partially filled last page is copied into a
 // page of the sequence, because the sequence's appends fill it.
+// Per-chunk completion events of a graft (kvg_graft_chunked): chunk k of
+// n_chunks maps to event k * n_events / n_chunks, recorded on the graft's
+// stream after the last chunk that maps to it.
+struct ChunkEvents {
+    void *const *events = nullptr;
+    int32_t max_events = 0;
+    int32_t *end_slot = nullptr;
+    int32_t *n_out = nullptr;
+};
+
+// A graft done in one piece (pool-resident blocks): one event, at its end.
+static cudaError_t record_single_chunk(const ChunkEvents &ce, cudaStream_t st, int64_t end_slot) {
+    if (!ce.events) return cudaSuccess;
+    if (ce.n_out) *ce.n_out = 1;
+    ce.end_slot[0] = (int32_t)end_slot;
+    return cudaEventRecord(static_cast<cudaEvent_t>(ce.events[0]), st);
+}
+
 static kvg_status pool_graft(kvg_store *s, const kvg_store::Blk &blk, kvg_cache *c, int32_t seq, int64_t dst,
-                             int64_t delta, uint32_t flags, cudaStream_t st, kvg_graft_report *report) {
+                             int64_t delta, uint32_t flags, cudaStream_t st, kvg_graft_report *report,
+                             const ChunkEvents &ce) {
     if (s->pool_cache != c) return fail(KVG_ERR_ARG, "a pool-resident block grafts only into its own cache");
     if (delta != 0) return fail(KVG_ERR_ARG, "relocation needs a copying store (HBM or pinned host)");
     const int64_t P = c->dims.page_size, n = blk.lay.n_tokens, npb = blk.lay.n_pages;
@@ -1455,6 +1474,7 @@ static kvg_status pool_graft(kvg_store *s, const kvg_store::Blk &blk, kvg_cache 
     ap.pids.n = (int32_t)npb;
     for (int64_t j = 0; j < npb; ++j) ap.pids.pid[j] = pages[j];
     KVG_CUDA(launch_alias(ap, c->n_sm, st));
+    KVG_CUDA(record_single_chunk(ce, st, dst + n));
     if (flags & KVG_GRAFT_VERIFY) {
         kvg_status r = enqueue_verify(s, blk, c, seq, jdst, false, st);
         if (r != KVG_OK) return r;
@@ -1473,9 +1493,9 @@ static int host_copy_grid_cap() {
     return cap;
 }
 
-extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t dst_slot,
-                                int64_t delta, uint32_t flags, void *stream, kvg_graft_report *report) {
-    Trace trace_("kvg_graft");
+static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t dst_slot,
+                             int64_t delta, uint32_t flags, void *stream, kvg_graft_report *report,
+                             const ChunkEvents &ce) {
     if (!s || !c) return fail(KVG_ERR_ARG, "null argument");
     if (block_id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)block_id);
     if (!same_geometry(s->dims, c->dims)) return fail(KVG_ERR_ARG, "store and cache geometry differ");
@@ -1495,7 +1515,7 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
     if (delta != 0 && c->dims.kv_dtype != KVG_KV_BF16) return fail(KVG_ERR_ARG, "relocation needs a bf16 cache");
     DeviceGuard g(c->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (s->pool_cache) return pool_graft(s, blk, c, seq, dst, delta, flags, st, report);
+    if (s->pool_cache) return pool_graft(s, blk, c, seq, dst, delta, flags, st, report, ce);
     auto pids = take_pages(c, npb);
     auto &sp = c->seq_pages[seq];
     const int64_t jdst = dst / P;
@@ -1558,10 +1578,19 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
             step = 1;
         }
     }
-    int chunk = 0;
-    for (int64_t base = 0; base < npb; base += p.npb, ++chunk) {
+    std::vector<std::pair<int64_t, int32_t>> plan;  // (first page, pages) per chunk
+    for (int64_t base = 0; base < npb;) {
         const int64_t body_end = npb - tail;
-        p.npb = (int32_t)(base < body_end ? std::min<int64_t>(step, body_end - base) : std::min<int64_t>(step, npb - base));
+        const int64_t k = base < body_end ? std::min<int64_t>(step, body_end - base) : std::min<int64_t>(step, npb - base);
+        plan.push_back({base, (int32_t)k});
+        base += k;
+    }
+    const int64_t n_chunks = (int64_t)plan.size();
+    const int64_t n_ev = ce.events ? std::min<int64_t>(ce.max_events, n_chunks) : 0;
+    if (ce.n_out) *ce.n_out = (int32_t)n_ev;
+    for (int64_t chunk = 0; chunk < n_chunks; ++chunk) {
+        const int64_t base = plan[chunk].first;
+        p.npb = plan[chunk].second;
         p.page_base = (int32_t)base;
         p.src_pos = bpos + base * P;
         p.dst_pos = c->positions + (int64_t)seq * c->max_slots + dst + base * P;
@@ -1573,6 +1602,13 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
             KVG_CUDA(launch_graft_verify(p, static_cast<uint32_t *>(c->leaf.ptr), c->n_sm, st));
         else
             KVG_CUDA(launch_graft_copy(p, c->n_sm, st, host_src ? host_copy_ctas : 0));
+        if (n_ev > 0) {
+            const int64_t j = chunk * n_ev / n_chunks;
+            if (chunk == n_chunks - 1 || (chunk + 1) * n_ev / n_chunks != j) {
+                KVG_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ce.events[j]), st));
+                ce.end_slot[j] = (int32_t)(dst + std::min<int64_t>((base + p.npb) * P, n));
+            }
+        }
         if (piped) {
             // (more than kHostVerifyChunks chunks only past 16 x 1,024 pages per
             // plane; an event is re-recorded after its wait is enqueued)
@@ -1600,6 +1636,30 @@ extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, i
     }
     return finish_verify(c, seq, flags, (flags & KVG_GRAFT_VERIFY) ? (int32_t)(c->dims.n_layers * 2 * npb) : 0,
                          st, report);
+}
+
+extern "C" kvg_status kvg_graft(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t dst_slot,
+                                int64_t delta, uint32_t flags, void *stream, kvg_graft_report *report) {
+    Trace trace_("kvg_graft");
+    return graft_impl(s, block_id, c, seq, dst_slot, delta, flags, stream, report, ChunkEvents{});
+}
+
+extern "C" kvg_status kvg_graft_chunked(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq,
+                                        int32_t dst_slot, int64_t delta, uint32_t flags, void *stream,
+                                        kvg_graft_report *report, void *const *events, int32_t max_events,
+                                        int32_t *chunk_end_slot, int32_t *n_chunks) {
+    Trace trace_("kvg_graft_chunked");
+    if (!events || max_events < 1 || !chunk_end_slot || !n_chunks)
+        return fail(KVG_ERR_ARG, "events, max_events >= 1, chunk_end_slot and n_chunks are required");
+    for (int32_t i = 0; i < max_events; ++i)
+        if (!events[i]) return fail(KVG_ERR_ARG, "null event %d", i);
+    *n_chunks = 0;
+    ChunkEvents ce;
+    ce.events = events;
+    ce.max_events = max_events;
+    ce.end_slot = chunk_end_slot;
+    ce.n_out = n_chunks;
+    return graft_impl(s, block_id, c, seq, dst_slot, delta, flags, stream, report, ce);
 }
 
 extern "C" kvg_status kvg_graft_batch(kvg_store *s, const uint64_t *block_ids, kvg_cache *c, const int32_t *seq_ids,

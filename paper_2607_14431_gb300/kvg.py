@@ -88,6 +88,8 @@ _SIGNATURES = {
     "kvg_cache_release": ([_vp, _i32, _vp], _i32),
     "kvg_deposit": ([_vp, _vp, _i32, _i32, _i32, _vp, _P(_u64)], _i32),
     "kvg_graft": ([_vp, _u64, _vp, _i32, _i32, _i64, _u32, _vp, _P(kvg_graft_report)], _i32),
+    "kvg_graft_chunked": ([_vp, _u64, _vp, _i32, _i32, _i64, _u32, _vp, _P(kvg_graft_report), _P(_vp), _i32,
+                           _P(_i32), _P(_i32)], _i32),
     "kvg_verify": ([_vp, _u64, _vp, _i32, _i32, _u32, _vp, _P(kvg_graft_report)], _i32),
     "kvg_decode_attention": ([_vp, _i32, _vp, _i32, _vp, _i32, _vp, ctypes.c_float, _vp], _i32),
     "kvg_decode_attention_noalloc": ([_vp, _i32, _vp, _i32, _vp, _i32, _vp, ctypes.c_float, _vp], _i32),
@@ -251,6 +253,24 @@ def kvg_graft(store, block_id: int, cache, seq: int, dst_slot: int = -1, delta: 
               stream=None, report: kvg_graft_report | None = None):
     _check(lib().kvg_graft(store, block_id, cache, seq, dst_slot, delta, flags, _stream(stream),
                            ctypes.byref(report) if report is not None else None))
+
+
+def kvg_graft_chunked(store, block_id: int, cache, seq: int, events, dst_slot: int = -1, delta: int = 0,
+                      flags: int = 0, stream=None, report: kvg_graft_report | None = None):
+    """kvg_graft with a completion event per chunk.  events: a list of CUDA
+    event handles (ints, e.g. torch.cuda.Event().cuda_event after a record,
+    or from cudaEventCreate).  Returns [chunk_end_slot[j] for j < n_chunks]:
+    events[j] covers the rows of slots [dst_slot, chunk_end_slot[j])."""
+    n = len(events)
+    if n < 1:
+        raise ValueError("at least one event")
+    ev = (_vp * n)(*[int(e) for e in events])
+    ends = (ctypes.c_int32 * n)()
+    nc = ctypes.c_int32(0)
+    _check(lib().kvg_graft_chunked(store, block_id, cache, seq, dst_slot, delta, flags, _stream(stream),
+                                   ctypes.byref(report) if report is not None else None, ev, n, ends,
+                                   ctypes.byref(nc)))
+    return [int(ends[j]) for j in range(nc.value)]
 
 
 def kvg_graft_batch(store, block_ids, cache, seq_ids, flags: int = 0, stream=None,

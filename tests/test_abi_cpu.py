@@ -39,6 +39,15 @@ def test_host_checks_reject_bad_geometry_without_a_gpu(lib):
     assert lib.kvg_store_create(ctypes.byref(good), 7, 1 << 20, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
     assert lib.kvg_store_create(None, 0, 1 << 20, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
     assert lib.kvg_graft(None, 0, None, 0, -1, 0, 0, None, None) == kvg.KVG_ERR_ARG
+    ends, nc = (ctypes.c_int32 * 2)(), ctypes.c_int32(-1)
+    no_events = (ctypes.c_void_p * 2)()
+    assert lib.kvg_graft_chunked(None, 0, None, 0, -1, 0, 0, None, None, None, 2, ends,
+                                 ctypes.byref(nc)) == kvg.KVG_ERR_ARG  # no event array
+    assert lib.kvg_graft_chunked(None, 0, None, 0, -1, 0, 0, None, None, no_events, 2, ends,
+                                 ctypes.byref(nc)) == kvg.KVG_ERR_ARG  # null events
+    assert "event" in kvg.kvg_last_error()
+    assert lib.kvg_graft_chunked(None, 0, None, 0, -1, 0, 0, None, None, no_events, 0, ends,
+                                 ctypes.byref(nc)) == kvg.KVG_ERR_ARG  # max_events < 1
     assert lib.kvg_decode_attention(None, 0, None, 1, None, 4, None, ctypes.c_float(1.0), None) == kvg.KVG_ERR_ARG
     assert lib.kvg_decode_attention_range(None, 0, None, 1, None, 4, ctypes.c_float(1.0), 0, 16, 0, None,
                                           None) == kvg.KVG_ERR_ARG

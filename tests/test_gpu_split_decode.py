@@ -209,3 +209,82 @@ def test_split_decode_host_checks():
     # slot_end at or past max_slots means "to the end", page-aligned or not
     kvg.kvg_decode_attention_range(c.h, -1, [0], q.data_ptr(), w.n_q_heads, 0.125, 0, 4 * P + 3, 0, st.data_ptr())
     torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("residency,n_pages_block", [(1, 41), (1, 130), (0, 41)])
+def test_chunked_graft_feeds_a_pipelined_split_decode(oracle, residency, n_pages_block):
+    """kvg_graft_chunked (verified) on a side stream, and on the main stream:
+    the fresh rows appended and decoded into a state, then each chunk's
+    slots merged in as soon as its event fires.  The output equals, bit for
+    bit, the same parts merged in the same order after a synchronous graft
+    (so no part read rows that had not landed yet: the destination starts
+    as canary bytes), and the oracle within 1e-2.  The chunk ends are page-aligned, increasing and
+    end at the block's length; a pinned-host store's verified graft uses
+    several chunks (the last one short), an HBM store's one."""
+    kvg = need_gpu()
+    w = geometry("d128")
+    P = w.page_size
+    nb, nf = n_pages_block * P, 3 * P + 11
+    dims = dims_for(kvg, w)
+    od = oracle_dims(oracle, w)
+    k, v = _kv(w, nb + nf, 91)
+    pos = syn.positions(0, nb + nf)
+    max_slots = nb + nf + 2 * P
+    n_pages = max_slots // P + 4
+    src = kvg.Cache(dims, n_pages, 1, max_slots)
+    append(kvg, src, 0, k[:, :nb], v[:, :nb], pos[:nb])
+    store = kvg.Store(dims, residency, 1 << 30)
+    bid = kvg.kvg_deposit(store.h, src.h, 0, 0, nb)
+    torch.cuda.synchronize()
+    q = syn.as_u16(syn.queries(w, w.n_layers, 1, 92))
+    qd = to_dev(q)
+    kf, vf, pf = to_dev(np.ascontiguousarray(k[:, nb:])), to_dev(np.ascontiguousarray(v[:, nb:])), to_dev(pos[nb:])
+    scale = 1.0 / math.sqrt(w.head_dim)
+
+    def run(chunked, same_ends=None):
+        c = kvg.Cache(dims, n_pages, 1, max_slots)
+        fill_canary(c)
+        kvg.kvg_cache_set_free_order(c.h, syn.permutation(n_pages, 93))
+        main, side = torch.cuda.Stream(), torch.cuda.Stream()
+        state = torch.full((w.n_layers, 1, w.n_q_heads, w.head_dim + 4), float("nan"), dtype=torch.float32,
+                           device="cuda")
+        out = torch.empty_like(qd)
+        torch.cuda.synchronize()
+        if chunked:
+            events = [torch.cuda.Event() for _ in range(16)]
+            for e in events:
+                e.record(side)  # creates the event
+            ends = kvg.kvg_graft_chunked(store.h, bid, c.h, 0, [e.cuda_event for e in events],
+                                         flags=kvg.KVG_GRAFT_VERIFY, stream=side)
+        else:
+            kvg.kvg_graft(store.h, bid, c.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+            ends = same_ends  # the same parts, merged in the same order
+        kvg.kvg_cache_append(c.h, 0, kf.data_ptr(), vf.data_ptr(), pf.data_ptr(), nf, main)
+        kvg.kvg_decode_attention_range(c.h, -1, [0], qd.data_ptr(), w.n_q_heads, scale, nb, max_slots, 0,
+                                       state.data_ptr(), main)
+        lo = 0
+        for j, hi in enumerate(ends):
+            if chunked:
+                main.wait_event(events[j])
+            kvg.kvg_decode_attention_range(c.h, -1, [0], qd.data_ptr(), w.n_q_heads, scale, lo, hi,
+                                           kvg.KVG_DECODE_MERGE, state.data_ptr(), main)
+            lo = hi
+        main.wait_stream(side)  # the digest verdict covers the whole block
+        kvg.kvg_decode_state_finish(state.data_ptr(), w.n_layers * w.n_q_heads, w.head_dim, out.data_ptr(), main)
+        kvg.kvg_sync(c.h, main, 60.0)  # raises on a digest mismatch
+        torch.cuda.synchronize()
+        return u16(out), ends, c
+
+    got, ends, c = run(True)
+    assert 1 <= len(ends) <= 16 and ends[-1] == nb
+    assert all(e % P == 0 for e in ends) and all(a < b for a, b in zip(ends, ends[1:]))
+    if residency == kvg.KVG_RESIDENCY_PINNED_HOST:
+        assert len(ends) > 1 and ends[-1] - ends[-2] <= ends[0]
+    else:
+        assert ends == [nb]
+    want, _, _ = run(False, ends)
+    assert np.array_equal(got, want)
+    oc = oracle.OracleCache(od, n_pages, 1, max_slots)
+    oc.append(0, k, v, pos)
+    o_ref = np.stack([oc.decode(0, l, q[l, 0], scale) for l in range(w.n_layers)])[:, None]
+    compare_decode(oracle, got, o_ref)
