@@ -341,7 +341,7 @@ kvg_status kvg_graft(kvg_store *store, uint64_t block_id, kvg_cache *cache, int3
  * (cudaEvent_t, on the cache's device; timing may be disabled).  The graft
  * copies the block in page-range chunks (one chunk for most HBM-store
  * blocks; up to 16 for a verified graft from a pinned-host store, the last
- * one short); chunk k of C maps to event k * E / C with E = min(max_events,
+ * two short); chunk k of C maps to event k * E / C with E = min(max_events,
  * C).  On KVG_OK, *n_chunks = E, and for j < E events[j] is recorded on
  * `stream` once every chunk that maps to j has its rows (all layers, K and V)
  * and position tags in the cache; chunk_end_slot[j] (host array of at least

@@ -1563,27 +1563,36 @@ static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int3
     const int64_t m = (int64_t)((c->page_bytes + kLeafBytes - 1) / kLeafBytes);
     if (verify0) KVG_CUDA(c->leaf.ensure((size_t)c->dims.n_layers * 2 * npb * m * 32));
     int64_t step = kMaxPagesPerLaunch;
-    // piped: the last chunk is short (1/64 of the block, at least a page), so
-    // that the one hash not hidden behind the link transfer is short too
-    int64_t tail = 0;
+    // piped: equal chunks, then two short ones (3/128 and 1/128 of the block,
+    // at least three pages and one): a chunk is hashed while the next one
+    // crosses the link, and only the last chunk's hash and the page digests
+    // follow the transfer, so each chunk's hash must fit in the next one's copy
+    std::vector<int64_t> tails;
     if (piped) {
         if (!c->aux) {
             KVG_CUDA(cudaStreamCreateWithFlags(&c->aux, cudaStreamNonBlocking));
             for (cudaEvent_t &e : c->aux_ev) KVG_CUDA(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
         }
         if (npb > kHostVerifyChunks) {
-            tail = std::max<int64_t>(1, npb / 64);
-            step = std::min<int64_t>(step, (npb - tail + kHostVerifyChunks - 2) / (kHostVerifyChunks - 1));
+            const int64_t t1 = std::min<int64_t>(std::max<int64_t>(1, npb / 128), kMaxPagesPerLaunch / 3);
+            tails = {3 * t1, t1};
+            const int64_t body = npb - 4 * t1;
+            step = std::min<int64_t>(step, (body + kHostVerifyChunks - 3) / (kHostVerifyChunks - 2));
         } else {
             step = 1;
         }
     }
     std::vector<std::pair<int64_t, int32_t>> plan;  // (first page, pages) per chunk
-    for (int64_t base = 0; base < npb;) {
-        const int64_t body_end = npb - tail;
-        const int64_t k = base < body_end ? std::min<int64_t>(step, body_end - base) : std::min<int64_t>(step, npb - base);
+    int64_t tail_pages = 0;
+    for (int64_t t : tails) tail_pages += t;
+    for (int64_t base = 0; base < npb - tail_pages;) {
+        const int64_t k = std::min<int64_t>(step, npb - tail_pages - base);
         plan.push_back({base, (int32_t)k});
         base += k;
+    }
+    for (int64_t t : tails) {
+        const int64_t base = plan.empty() ? 0 : plan.back().first + plan.back().second;
+        plan.push_back({base, (int32_t)t});
     }
     const int64_t n_chunks = (int64_t)plan.size();
     const int64_t n_ev = ce.events ? std::min<int64_t>(ce.max_events, n_chunks) : 0;

@@ -466,8 +466,8 @@ def test_host_store_verified_graft_reports_the_bad_page(oracle, geo, nb, bad):
     """A verified graft from a pinned-host store copies page-range chunks and
     hashes each chunk's restored pages on a second stream: a flipped byte in
     page (plane, j) is reported as that block page, whichever chunk holds it
-    (41 and 130 pages: a short last chunk of one and two pages after the
-    equal ones), and an intact block grafts clean."""
+    (41 and 130 pages: after the equal chunks, a chunk of three pages and
+    one of one), and an intact block grafts clean."""
     kvg = need_gpu()
     w = geometry(geo)
     s = _build_both(kvg, oracle, w, nb, 0, seed=61, copies=3)
