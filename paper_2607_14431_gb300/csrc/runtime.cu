@@ -1554,7 +1554,8 @@ static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int3
     // follow.  From a pinned-host store the copy instead moves page-range
     // chunks with the copy kernel (whose wide reads keep the host link at its
     // limit) and a library stream hashes each chunk's restored pages in HBM
-    // while the next chunk crosses the link.
+    // while the next chunk crosses the link; the last, short chunk goes
+    // through the one-pass kernel.
     const bool host_src = s->residency == KVG_RESIDENCY_PINNED_HOST;
     const int host_copy_ctas = host_copy_grid_cap();
     const bool verify0 = (flags & KVG_GRAFT_VERIFY) && delta == 0;
@@ -1607,7 +1608,10 @@ static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int3
         p.fill_row = c->page_fill + (int64_t)seq * c->max_pages + jdst + base;
         p.pids.n = p.npb;
         for (int32_t i = 0; i < p.npb; ++i) p.pids.pid[i] = pids[base + i];
-        if (fused)
+        // piped: the last (short) chunk is copied and hashed in one pass, so
+        // its hash needs no second read after it has crossed the link
+        const bool one_pass = fused || (piped && chunk == n_chunks - 1);
+        if (one_pass)
             KVG_CUDA(launch_graft_verify(p, static_cast<uint32_t *>(c->leaf.ptr), c->n_sm, st));
         else
             KVG_CUDA(launch_graft_copy(p, c->n_sm, st, host_src ? host_copy_ctas : 0));
@@ -1618,7 +1622,7 @@ static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int3
                 ce.end_slot[j] = (int32_t)(dst + std::min<int64_t>((base + p.npb) * P, n));
             }
         }
-        if (piped) {
+        if (piped && !one_pass) {
             // (more than kHostVerifyChunks chunks only past 16 x 1,024 pages per
             // plane; an event is re-recorded after its wait is enqueued)
             cudaEvent_t ev = c->aux_ev[chunk % kHostVerifyChunks];
