@@ -885,7 +885,13 @@ def test_pool_store_zero_copy_graft(oracle):
     kvg.kvg_cache_release(cache.h, 2)
     oc.release(1)
     oc.release(2)
-    kvg.kvg_graft(store.h, bid, cache.h, 3, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+    # (through kvg_graft_chunked: a pool-resident block grafts in one piece, one event)
+    evs = [torch.cuda.Event() for _ in range(3)]
+    for e in evs:
+        e.record()
+    ends = kvg.kvg_graft_chunked(store.h, bid, cache.h, 3, [e.cuda_event for e in evs],
+                                 flags=kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+    assert ends == [nb] and evs[0].query()
     oc.graft_pinned(3, opb)
     pt, pf, ps = tables(cache)
     assert np.array_equal(pt, oc.page_table) and np.array_equal(pool_u16(cache, w), oc.pool)
