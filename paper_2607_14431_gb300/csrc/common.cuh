@@ -249,7 +249,11 @@ int env_knob(const char *name, int fallback);
 
 // max_ctas > 0 caps the grid (a copy from host memory needs only enough
 // CTAs to keep the host link busy; the rest of the SMs stay free).
-cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s, int max_ctas = 0);
+// max_ctas > 0: a host-mapped source, read by at most max_ctas CTAs of
+// graft_kernel.  Otherwise the shared-memory staged graft runs when the unit
+// fits its stages (its bounded waits record into `status`).
+cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s, int max_ctas = 0,
+                              DevStatus *status = nullptr);
 // Own-position copies of a batch of grafts in one launch (jobs, metas in device memory).
 cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s, int max_ctas = 0);
 // Bulk append by tensor copies, for appends of at least append_tma_rows()

@@ -553,6 +553,147 @@ __global__ void reset_seq_kernel(int32_t *table_row, int32_t *fill_row, int32_t 
     for (int64_t s = gtid; s < max_slots; s += gsz) pos_row[s] = -1;
 }
 
+// ---- graft through shared-memory stages (HBM sources) ---------------------
+// A persistent CTA per SM streams its units (chunks of block pages, as in
+// graft_kernel) through a ring of shared-memory stages: thread 0 brings a
+// unit in with one bulk copy (cp.async.bulk, mbarrier completion), the CTA
+// re-rotates the valid key rows in place when the graft relocates, and
+// thread 0 writes the stage to the cache page with one bulk copy.  The loads
+// of later units are in flight meanwhile, so the copy does not depend on
+// registers for its bytes in flight.  Rows, rounding and operation order of
+// the rotation are those of rotate_chunk.
+constexpr int kTmaGraftThreads = 256;
+
+template <int ROT>
+__device__ __forceinline__ void rotate_stage(uint8_t *stage, int bytes, int64_t first_row_in_page,
+                                             int64_t page_token0, const GraftParams &p, const float *cs) {
+    const int D = p.head_dim;
+    const int vec_per_row = D >> 3;
+    const int rows = bytes / (2 * D);
+    uint4 *v4 = reinterpret_cast<uint4 *>(stage);
+    const int P = p.page_size;
+    const int64_t nv = p.n_tokens - page_token0;
+    const int n_valid = nv < P ? (int)nv : P;
+    const int r0 = (int)(first_row_in_page % P);
+    if (ROT == 1) {
+        const int half_vecs = vec_per_row >> 1;
+        const int hv_shift = __ffs(half_vecs) - 1;
+        const int n_items = rows * half_vecs;
+        for (int it = threadIdx.x; it < n_items; it += blockDim.x) {
+            const int rr = it >> hv_shift;
+            if (n_valid < P && (r0 + rr) % P >= n_valid) continue;  // padding row: unchanged
+            const int c = it & (half_vecs - 1);
+            const int lo_i = rr * vec_per_row + c;
+            float a[8], b[8], ra[8], rb[8];
+            unpack8(v4[lo_i], a);
+            unpack8(v4[lo_i + half_vecs], b);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) rot(a[e], b[e], cs[c * 8 + e], cs[kMaxHalfDim + c * 8 + e], ra[e], rb[e]);
+            v4[lo_i] = pack8(ra);
+            v4[lo_i + half_vecs] = pack8(rb);
+        }
+    } else {
+        const int vr_shift = __ffs(vec_per_row) - 1;
+        const int n_items = rows * vec_per_row;
+        for (int it = threadIdx.x; it < n_items; it += blockDim.x) {
+            const int rr = it >> vr_shift;
+            if (n_valid < P && (r0 + rr) % P >= n_valid) continue;
+            const int c = it & (vec_per_row - 1);
+            float f[8], g[8];
+            unpack8(v4[it], f);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int i = c * 4 + e;
+                rot(f[2 * e], f[2 * e + 1], cs[i], cs[kMaxHalfDim + i], g[2 * e], g[2 * e + 1]);
+            }
+            v4[it] = pack8(g);
+        }
+    }
+}
+
+template <int ROT>
+__global__ void __launch_bounds__(kTmaGraftThreads) graft_tma_kernel(const GraftParams p, DevStatus *status,
+                                                                     int32_t n_stages, uint64_t limit_ns) {
+    extern __shared__ __align__(128) uint8_t stage_mem[];
+    __shared__ __align__(8) uint64_t bars[kTmaStagesMax];
+    __shared__ float cs[2 * kMaxHalfDim];
+    graft_metadata(p);
+    const uint64_t page_bytes = p.page_bytes;
+    const uint32_t cb = (uint32_t)p.chunk_bytes;
+    const int cpp = (int)(page_bytes / cb);
+    const int64_t n_units = (int64_t)p.n_layers * 2 * p.npb * cpp;
+    if ((int64_t)blockIdx.x >= n_units) return;  // the whole CTA
+    const int64_t K = (n_units - blockIdx.x + gridDim.x - 1) / gridDim.x;  // this CTA's units
+    if (ROT != 0)
+        for (int i = threadIdx.x; i < p.head_dim / 2; i += blockDim.x) {
+            cs[i] = p.cosv[i];
+            cs[kMaxHalfDim + i] = p.sinv[i];
+        }
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < n_stages; ++i) mbar_init(&bars[i], 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    struct Unit {
+        const uint8_t *src;
+        uint8_t *dst;
+        int64_t lkv, jj;
+        uint64_t off;
+    };
+    auto unit = [&](int64_t k) {
+        const int64_t u = (int64_t)blockIdx.x + k * gridDim.x;
+        const int64_t page_u = u / cpp;
+        Unit r;
+        r.off = (uint64_t)(u - page_u * cpp) * cb;
+        r.lkv = page_u / p.npb;
+        r.jj = page_u - r.lkv * p.npb;
+        r.src = p.src + ((uint64_t)r.lkv * p.block_pages + p.page_base + r.jj) * page_bytes + r.off;
+        r.dst = p.pool + ((uint64_t)r.lkv * p.pool_pages + p.pids.pid[r.jj]) * page_bytes + r.off;
+        return r;
+    };
+    auto load = [&](int64_t k) {  // thread 0
+        const int st = (int)(k % n_stages);
+        mbar_arrive_expect_tx(&bars[st], cb);
+        bulk_g2s(stage_mem + (size_t)st * cb, unit(k).src, cb, &bars[st]);
+    };
+    const int64_t pro = K < n_stages ? K : n_stages;
+    if (threadIdx.x == 0)
+        for (int64_t k = 0; k < pro; ++k) load(k);
+    int64_t loaded = pro;  // thread 0's count of units whose load is issued
+    int64_t k = 0;
+    for (; k < K; ++k) {
+        const int st = (int)(k % n_stages);
+        const bool ok = mbar_wait_bounded(&bars[st], (uint32_t)((k / n_stages) & 1), limit_ns);
+        if (__syncthreads_or(!ok)) {
+            if (threadIdx.x == 0) record_error(status, KVG_ERR_DEVICE_CHECK, 3);
+            break;
+        }
+        const Unit u = unit(k);
+        uint8_t *stage = stage_mem + (size_t)st * cb;
+        if (ROT != 0 && !(u.lkv & 1)) {
+            rotate_stage<ROT>(stage, (int)cb, (int64_t)(u.off / (uint64_t)(2 * p.head_dim)),
+                              (int64_t)(p.page_base + u.jj) * p.page_size, p, cs);
+            fence_proxy_async_shared();  // this thread's writes, before the bulk copy reads them
+            __syncthreads();
+        }
+        if (threadIdx.x == 0) {
+            bulk_s2g(u.dst, stage, cb);
+            bulk_commit();
+            // refill the previous unit's stage once its store has read it
+            if (k >= 1 && loaded < K) {
+                bulk_wait_read<1>();
+                load(loaded++);
+            }
+        }
+    }
+    if (threadIdx.x == 0) {
+        if (k < K)  // gave up: let the loads still in flight land before the CTA exits
+            for (int64_t m = k; m < loaded; ++m)
+                mbar_wait_bounded(&bars[m % n_stages], (uint32_t)((m / n_stages) & 1), limit_ns);
+        bulk_wait<0>();
+    }
+}
+
 int grid_for(int64_t work_items, int per_block, int n_sm, int waves) {
     int64_t g = (work_items + per_block - 1) / per_block;
     const int64_t cap = (int64_t)n_sm * waves;
@@ -605,7 +746,60 @@ cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t
     return cudaGetLastError();
 }
 
-cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s, int max_ctas) {
+// Shared-memory stage budget of graft_tma_kernel (KVG_GRAFT_TMA_KB, 0 turns
+// the staged graft off).  Three 64 KiB stages measured best: the 31B
+// relocation 2.38 ms against 3.08 ms with two, and 32 KiB units (four or six
+// stages) 2.51-2.56 ms, 16 KiB units 4.3 ms.
+static int graft_tma_budget() {
+    static const int kb = [] {
+        const char *e = getenv("KVG_GRAFT_TMA_KB");
+        return e ? atoi(e) : 192;
+    }();
+    return kb;
+}
+
+// The staged graft for HBM sources: one persistent CTA per SM; -1 if the
+// unit does not fit twice in the stage budget (then graft_kernel runs).
+static cudaError_t launch_graft_tma(const GraftParams &p, DevStatus *status, int n_sm, cudaStream_t s) {
+    const int64_t units = (int64_t)p.n_layers * 2 * p.npb * (int64_t)(p.page_bytes / p.chunk_bytes);
+    const uint32_t budget = (uint32_t)std::min(graft_tma_budget(), 200) * 1024u;
+    int n_stages = (int)(budget / (uint32_t)p.chunk_bytes);
+    if (n_stages > kTmaStagesMax) n_stages = kTmaStagesMax;
+    if (n_stages < 2 || units == 0) return cudaErrorNotSupported;
+    static std::atomic<bool> attr_set[kMaxDevices][3];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return cudaErrorNotSupported;
+    const size_t smem = (size_t)n_stages * p.chunk_bytes;
+    const int r = p.rotate;
+    if (!attr_set[dev][r].load()) {
+        cudaError_t e = r == 0 ? cudaFuncSetAttribute(graft_tma_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                      200 * 1024)
+                      : r == 1 ? cudaFuncSetAttribute(graft_tma_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                      200 * 1024)
+                               : cudaFuncSetAttribute(graft_tma_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                      200 * 1024);
+        if (e != cudaSuccess) return e;
+        attr_set[dev][r].store(true);
+    }
+    const int grid = grid_for(units, 1, n_sm, 1);
+    const uint64_t limit_ns = 2000000000ull;
+    if (r == 0)
+        graft_tma_kernel<0><<<grid, kTmaGraftThreads, smem, s>>>(p, status, n_stages, limit_ns);
+    else if (r == 1)
+        graft_tma_kernel<1><<<grid, kTmaGraftThreads, smem, s>>>(p, status, n_stages, limit_ns);
+    else
+        graft_tma_kernel<2><<<grid, kTmaGraftThreads, smem, s>>>(p, status, n_stages, limit_ns);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s, int max_ctas, DevStatus *status) {
+    // HBM sources go through shared-memory stages; a host-mapped source is
+    // read by a capped grid of graft_kernel (the host link bounds it)
+    if (max_ctas == 0 && status && graft_tma_budget() > 0) {
+        const cudaError_t e = launch_graft_tma(p, status, n_sm, s);
+        if (e != cudaErrorNotSupported) return e;
+    }
     const int64_t units = (int64_t)p.n_layers * 2 * p.npb * (int64_t)(p.page_bytes / p.chunk_bytes);
     int grid = grid_for(units, 1, n_sm, 4);
     if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;

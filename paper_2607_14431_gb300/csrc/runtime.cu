@@ -1614,7 +1614,7 @@ static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int3
         if (one_pass)
             KVG_CUDA(launch_graft_verify(p, static_cast<uint32_t *>(c->leaf.ptr), c->n_sm, st));
         else
-            KVG_CUDA(launch_graft_copy(p, c->n_sm, st, host_src ? host_copy_ctas : 0));
+            KVG_CUDA(launch_graft_copy(p, c->n_sm, st, host_src ? host_copy_ctas : 0, c->status));
         if (n_ev > 0) {
             const int64_t j = chunk * n_ev / n_chunks;
             if (chunk == n_chunks - 1 || (chunk + 1) * n_ev / n_chunks != j) {
