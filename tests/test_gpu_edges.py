@@ -252,3 +252,52 @@ def test_outputs_are_identical_across_processes():
         assert r.returncode == 0, r.stderr[-2000:]
         digests.append(r.stdout.strip().splitlines()[-1])
     assert len(digests[0]) == 64 and digests[0] == digests[1]
+
+
+_RELOC_CHILD = r'''
+import hashlib, sys
+sys.path.insert(0, sys.argv[1])
+sys.path.insert(0, sys.argv[1] + "/tests")
+import numpy as np, torch
+import kvg_synth as syn
+from kvg_testlib import append, dims_for, fill_canary, need_gpu, pool_u16
+kvg = need_gpu()
+out = []
+for style in (0, 1):
+    w = syn.Workload("reloc", 3, 8, 4, 128, 64, 1e6, 0x93)
+    nb = 1000
+    k, v = syn.kv_rows(w, nb, w.seed)
+    k, v = syn.as_u16(k), syn.as_u16(v)
+    dims = dims_for(kvg, w, style)
+    src = kvg.Cache(dims, 40, 1, 1088)
+    append(kvg, src, 0, k, v, syn.positions(0, nb))
+    store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, 1 << 28)
+    bid = kvg.kvg_deposit(store.h, src.h, 0, 0, nb)
+    c = kvg.Cache(dims, 40, 2, 1088)
+    fill_canary(c)  # pages no graft writes hold known bytes
+    kvg.kvg_graft(store.h, bid, c.h, 0, -1, 4096, kvg.KVG_GRAFT_SYNC)
+    kvg.kvg_graft(store.h, bid, c.h, 1, -1, 0, kvg.KVG_GRAFT_SYNC)
+    torch.cuda.synchronize()
+    out.append(hashlib.sha256(pool_u16(c, w).tobytes()).hexdigest())
+print(" ".join(out))
+'''
+
+
+def test_staged_and_register_grafts_write_identical_bytes():
+    """An HBM-store graft runs through shared-memory stages by default and
+    through registers with KVG_GRAFT_TMA_KB=0 (the pinned-host path): the
+    relocated (delta 4096, half-split and interleaved) and own-position
+    grafts of a ragged 1,000-token block leave byte-identical pools."""
+    import os
+    import subprocess
+    import sys
+    need_gpu()
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    digests = []
+    for kb in ("192", "0"):
+        env = dict(os.environ, KVG_GRAFT_TMA_KB=kb)
+        r = subprocess.run([sys.executable, "-c", _RELOC_CHILD, root], capture_output=True, text=True, timeout=600,
+                           env=env)
+        assert r.returncode == 0, r.stderr[-2000:]
+        digests.append(r.stdout.strip().splitlines()[-1])
+    assert len(digests[0]) == 2 * 64 + 1 and digests[0] == digests[1]
