@@ -301,3 +301,48 @@ def test_staged_and_register_grafts_write_identical_bytes():
         assert r.returncode == 0, r.stderr[-2000:]
         digests.append(r.stdout.strip().splitlines()[-1])
     assert len(digests[0]) == 2 * 64 + 1 and digests[0] == digests[1]
+
+
+def test_graft_of_pages_too_large_for_two_stages(oracle):
+    """page_size 1023 (2 kv heads, head_dim 128): a page of 523,776 bytes
+    halves once into 261,888-byte units (its rows do not halve again), more
+    than two shared-memory stages hold, so the HBM-store graft takes the
+    register copy instead.  The own-position graft of a ragged two-page block
+    is bit-exact with the oracle (every pool byte, tables, positions); a
+    relocated one (delta 4096, both RoPE styles) keeps values and padding
+    bit-exact and keys within 2e-2 of the fp64 rotation."""
+    kvg = need_gpu()
+    w = syn.Workload("p1023", 2, 4, 2, 128, 1023, 10000.0, 0x95)
+    P = w.page_size
+    nb = P + 500
+    k, v = _kv(w, nb, 176)
+    max_slots, n_pages = 4 * P, 8
+    for style in (0, 1):
+        dims, od = dims_for(kvg, w, style), oracle_dims(oracle, w, style)
+        src = kvg.Cache(dims, n_pages, 1, max_slots)
+        append(kvg, src, 0, k, v, syn.positions(0, nb))
+        store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, HBM_CAP)
+        bid = kvg.kvg_deposit(store.h, src.h, 0, 0, nb)
+        c = kvg.Cache(dims, n_pages, 2, max_slots)
+        fill_canary(c)
+        oc = oracle.OracleCache(od, n_pages, 2, max_slots, fill=CANARY)
+        oblk = oracle.block_from_kv(od, k, v, syn.positions(0, nb))
+        kvg.kvg_graft(store.h, bid, c.h, 0, -1, 0, kvg.KVG_GRAFT_SYNC)
+        oc.graft(0, oblk)
+        assert np.array_equal(pool_u16(c, w), oc.pool)
+        kvg.kvg_graft(store.h, bid, c.h, 1, -1, 4096, kvg.KVG_GRAFT_SYNC)
+        oc.graft(1, oblk, delta=4096)
+        pool = pool_u16(c, w)
+        pt, pf, ps = tables(c)
+        assert np.array_equal(pt, oc.page_table) and np.array_equal(pf, oc.page_fill)
+        assert np.array_equal(ps, oc.positions)
+        assert np.array_equal(pool[:, 1], oc.pool[:, 1])  # values
+        k64 = np.stack([oracle.rope_rotate_rows(k[l], 4096, w.rope_theta, style) for l in range(w.n_layers)])
+        kg = np.empty_like(k)
+        for t in range(nb):
+            j, r = divmod(t, P)
+            kg[:, t] = pool[:, 0, pt[1, j], :, r, :]
+        assert np.abs(oracle.bf16_to_f64(kg) - k64).max() <= 2e-2
+        j, r = divmod(nb, P)  # padding rows of the last page: copied unchanged (zeros)
+        assert not pool[:, 0, pt[1, j], :, r:, :].any()
+        kvg.kvg_sync(c.h)
