@@ -810,12 +810,14 @@ def run_other(args):
                                       "block re-based by delta (0,1,4096,100000 across 8 sequences; 4096 timed), "
                                       "decode batch 8 over 65536-token contexts"}
         line["parts"]["decode"]["tokens_per_s"] = round(st.B * 1e3 / statistics.mean(phase_ms["decode"]), 1)
+        line["roofline"] = _part_roofline(line["parts"], "decode", "decode_kernel", hbm_peak, peak_kind)
     elif args.config == "batched":
         line["value"] = round(step_bytes / (ms_step * 1e-3) / 1e9, 2)
         line["config"] = {"workload": f"batched-library: L{st.w.n_layers} slice of 12b, 32 seqs x 4 blocks "
                                       "U{2048..6144} from a 512-block HBM store, then 64 decode steps (batch 32)"}
         line["parts"]["decode_steps"]["tokens_per_s"] = round(
             syn.BATCHED_SEQS * st.steps * 1e3 / statistics.mean(phase_ms["decode_steps"]), 1)
+        line["roofline"] = _part_roofline(line["parts"], "decode_steps", "decode_kernel", hbm_peak, peak_kind)
     else:
         g = np.array(phase_ms["host_graft"])
         depth = np.array(blocks, dtype=np.float64)
@@ -847,6 +849,15 @@ def run_other(args):
             errs.append(st.needle_error(b))
         line["checks"] = {"needle_max_abs_err": max(errs), "needles_checked": len(errs)}
     print(json.dumps(line), flush=True)
+
+
+def _part_roofline(parts, part, kernel, hbm_peak, peak_kind):
+    """Roofline object of a workload's longest part (HBM-bound): its
+    algorithmic bytes over its CUDA-event time against the measured copy
+    peak; no ncu traffic is kept for these workloads."""
+    p = parts[part]
+    return {"bound": "hbm", "kernel": kernel, "part": part, "achieved": p["gbs"], "peak": round(hbm_peak, 1),
+            "unit": "GB/s", "frac": p["hbm_frac"], "traffic": None, "peak_kind": peak_kind}
 
 
 def _sha_tensor(t):
