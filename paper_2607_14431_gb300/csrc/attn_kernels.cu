@@ -267,6 +267,12 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
         cur.end = cur.t - tp.tile + (p.rows.pref_tiles[tp.b + 1] - p.rows.pref_tiles[tp.b]);
     };
 
+    // The page-table entry and fill of the next tile to issue are loaded one
+    // issue ahead (lane 0's registers), so their latency hides behind a
+    // tile's compute instead of stalling the warp at the issue.
+    struct PageAhead {
+        int seq = -1, jj = -1, fill = 0, pid = -1;
+    } ahead;
     // lane 0: arm the stage's barrier and copy the next tile's K and V boxes
     auto issue = [&](int stg) {
         if (cur.t >= cur.end) advance_to_unit();
@@ -278,8 +284,29 @@ __global__ void __launch_bounds__(32) decode_kernel(const DecodeParams p, const 
             cur.k = 0;
             ++cur.jj;
         }
-        const int fill = p.page_fill[(int64_t)seq * p.max_pages + jj];
-        const int pid = p.page_table[(int64_t)seq * p.max_pages + jj];
+        int fill, pid;
+        if (!FP8 && ahead.seq == seq && ahead.jj == jj) {
+            fill = ahead.fill;
+            pid = ahead.pid;
+        } else {
+            fill = p.page_fill[(int64_t)seq * p.max_pages + jj];
+            pid = p.page_table[(int64_t)seq * p.max_pages + jj];
+        }
+        // the next tile of this unit (same page, or the next one); the fp8
+        // kernel issues in mid-tile and measured no faster with it
+        if constexpr (!FP8) {
+            if (cur.t < cur.end && cur.jj != jj) {
+                ahead.seq = cur.seq;
+                ahead.jj = cur.jj;
+                ahead.fill = p.page_fill[(int64_t)cur.seq * p.max_pages + cur.jj];
+                ahead.pid = p.page_table[(int64_t)cur.seq * p.max_pages + cur.jj];
+            } else if (cur.jj == jj) {
+                ahead.seq = seq;
+                ahead.jj = jj;
+                ahead.fill = fill;
+                ahead.pid = pid;
+            }
+        }
         int vr = fill - k * TOK;
         vr = vr < 0 ? 0 : (vr > TOK ? TOK : vr);
         if (lo >= vr) vr = 0;
