@@ -211,8 +211,9 @@ def test_split_decode_host_checks():
     torch.cuda.synchronize()
 
 
-@pytest.mark.parametrize("residency,n_pages_block", [(1, 41), (1, 130), (0, 41)])
-def test_chunked_graft_feeds_a_pipelined_split_decode(oracle, residency, n_pages_block):
+@pytest.mark.parametrize("residency,n_pages_block,n_events", [(1, 41, 16), (1, 130, 16), (0, 41, 16), (1, 41, 4),
+                                                                (1, 130, 1)])
+def test_chunked_graft_feeds_a_pipelined_split_decode(oracle, residency, n_pages_block, n_events):
     """kvg_graft_chunked (verified) on a side stream, and on the main stream:
     the fresh rows appended and decoded into a state, then each chunk's
     slots merged in as soon as its event fires.  The output equals, bit for
@@ -220,7 +221,8 @@ def test_chunked_graft_feeds_a_pipelined_split_decode(oracle, residency, n_pages
     (so no part read rows that had not landed yet: the destination starts
     as canary bytes), and the oracle within 1e-2.  The chunk ends are page-aligned, increasing and
     end at the block's length; a pinned-host store's verified graft uses
-    several chunks (the last one short), an HBM store's one."""
+    several chunks (the last one short), an HBM store's one; with fewer
+    events than chunks (4, or 1) consecutive chunks share an event."""
     kvg = need_gpu()
     w = geometry("d128")
     P = w.page_size
@@ -251,7 +253,7 @@ def test_chunked_graft_feeds_a_pipelined_split_decode(oracle, residency, n_pages
         out = torch.empty_like(qd)
         torch.cuda.synchronize()
         if chunked:
-            events = [torch.cuda.Event() for _ in range(16)]
+            events = [torch.cuda.Event() for _ in range(n_events)]
             for e in events:
                 e.record(side)  # creates the event
             ends = kvg.kvg_graft_chunked(store.h, bid, c.h, 0, [e.cuda_event for e in events],
@@ -276,10 +278,12 @@ def test_chunked_graft_feeds_a_pipelined_split_decode(oracle, residency, n_pages
         return u16(out), ends, c
 
     got, ends, c = run(True)
-    assert 1 <= len(ends) <= 16 and ends[-1] == nb
+    assert 1 <= len(ends) <= n_events and ends[-1] == nb
     assert all(e % P == 0 for e in ends) and all(a < b for a, b in zip(ends, ends[1:]))
-    if residency == kvg.KVG_RESIDENCY_PINNED_HOST:
-        assert len(ends) > 1 and ends[-1] - ends[-2] <= ends[0]
+    if residency == kvg.KVG_RESIDENCY_PINNED_HOST and n_events == 16:
+        assert len(ends) > 1 and ends[-1] - ends[-2] <= ends[0]  # the last chunk is short
+    elif residency == kvg.KVG_RESIDENCY_PINNED_HOST:
+        assert len(ends) == n_events  # fewer events than chunks: chunks share events
     else:
         assert ends == [nb]
     want, _, _ = run(False, ends)
