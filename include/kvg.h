@@ -203,13 +203,18 @@ kvg_status kvg_store_load(kvg_store *store, const char *path, uint32_t flags, ui
 
 /* ---------------------------------------------------------------- cache -- */
 
-/* A paged KV cache on `device`: pool of elements (bf16, or E4M3 codes for an
+/* A paged KV cache on `device`: the "fresh inference context" a block is
+ * installed into (Sec. 3.2: a fresh process or serving slot whose live
+ * context holds the restored prefix at [0, N); Sec. 3.3: the serving side of
+ * the deposit/graft cycle).  Pool of elements (bf16, or E4M3 codes for an
  * fp8 cache) [n_layers][2][n_pages][n_kv_heads][page_size][head_dim] (one
  * page id names the same token rows in every layer), and per sequence a page table, per-page fill counts, position tags
  * per slot and a slot high-water mark.  The pool is not initialised.
  * Free pages are handed out from the front of an ordered free list,
  * initially 0, 1, ..., n_pages-1; a released sequence's pages go to its back
- * in page-table order.  max_slots bounds one sequence's slots. */
+ * in page-table order.  max_slots bounds one sequence's slots.  The first
+ * cache created on a device also makes the 16 MiB static scratch of
+ * kvg_decode_attention_noalloc resident there (KVG_ERR_CUDA if that fails). */
 kvg_status kvg_cache_create(const kvg_dims *dims, int32_t n_pages, int32_t max_seqs,
                             int32_t max_slots, int32_t device, kvg_cache **out);
 void kvg_cache_destroy(kvg_cache *cache);
@@ -272,7 +277,10 @@ kvg_status kvg_cache_append_batch(kvg_cache *cache, const int32_t *seq_ids, int3
                                   const void *v, const int32_t *positions, void *stream);
 
 /* Returns the sequence's pages to the free list and clears its page table,
- * fills and position tags. */
+ * fills and position tags: the serving slot is empty again, ready for the
+ * next graft into a fresh context (Sec. 3.2; Sec. 4.4, where the movable
+ * window swaps which block is resident in the live prefix).  Enqueued on
+ * `stream`; the host bookkeeping changes at once. */
 kvg_status kvg_cache_release(kvg_cache *cache, int32_t seq, void *stream);
 
 /* ----------------------------------------------------------- deposit -- */
@@ -465,9 +473,12 @@ kvg_status kvg_decode_state_finish(const float *state, int64_t n_rows, int32_t h
  *     in 16 MiB - 256 bytes, and a call that does not fit even with one
  *     worker returns KVG_ERR_CAPACITY with an explanatory kvg_last_error()
  *     and enqueues nothing;
- *   - the first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress, with that device current); make that first call
- *     before any stream capture;
+ *   - the array's device address is looked up (cudaGetSymbolAddress, with
+ *     the device current) by kvg_cache_create, once per device: that is when
+ *     the module holding the array is made resident on the device and its
+ *     16 MiB are taken, also under lazy module loading.  This entry point
+ *     itself only reads the stored address, so its first call allocates
+ *     nothing either;
  *   - every call on a device shares the one array, and the array keeps the
  *     previous call's contents (each partial the call reads is first written
  *     by the same call, so nothing needs clearing): calls whose GPU work
@@ -494,7 +505,10 @@ kvg_status kvg_digest(const void *bytes, uint64_t n, int32_t mode, uint64_t page
 /* --------------------------------------------------------------- misc -- */
 
 /* Waits (up to timeout_s seconds, polling) for `stream`, then reads and clears
- * the cache's device status word.  Returns KVG_ERR_TIMEOUT if the stream is
+ * the cache's device status word.  This is where the outcome of the
+ * asynchronous digest gate arrives on the host: a graft is accepted only
+ * when every restored page's SHA-256 matches the deposited one (Sec. 3.2's
+ * byte-equality test; Sec. 4.11's per-block integrity check).  Returns KVG_ERR_TIMEOUT if the stream is
  * still busy, KVG_ERR_DIGEST after a failed verification (report, nullable,
  * gets the details), KVG_ERR_DEVICE_CHECK if a kernel's own check failed. */
 kvg_status kvg_sync(kvg_cache *cache, void *stream, double timeout_s, kvg_graft_report *report);
@@ -506,6 +520,10 @@ kvg_status kvg_sync(kvg_cache *cache, void *stream, double timeout_s, kvg_graft_
  * it and the context stays usable.  Nothing faults or hangs. */
 kvg_status kvg_selftest_bounded_wait(kvg_cache *cache, uint64_t limit_ns, void *stream);
 
+/* Name of a status code (a static string; "unknown status" for values not
+ * in kvg_status).  The codes are the failure modes of the problem statement:
+ * digest mismatch (Sec. 3.2, Sec. 4.11), position tags out of range after a
+ * re-base (Sec. 4.2), a block that does not fit the cache (Sec. 3.3). */
 const char *kvg_status_string(kvg_status status);
 
 /* Human-readable detail of the last failed call on this host thread (empty if

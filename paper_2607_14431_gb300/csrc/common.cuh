@@ -9,6 +9,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <vector>
+
 #include "kvg.h"
 
 namespace kvg {
@@ -317,6 +319,29 @@ cudaError_t launch_combine(int head_dim, int group, const DecodeParams &p, cudaS
 bool decode_supported(int head_dim, int group, bool fp8 = false);
 int decode_tile_tokens(int head_dim, bool fp8);
 int decode_max_warps(int head_dim, int group, bool fp8, int n_sm);
+
+// ------------------------------------- runtime.cu <-> noalloc.cu interface --
+// Read-only view of a cache's geometry and device buffers (runtime.cu fills
+// it; noalloc.cu reads it).  One definition here, included by both files.
+struct CacheShape {
+    int32_t n_layers, n_kv_heads, head_dim, page_size, n_pages, max_seqs, max_pages, device, n_sm;
+    int32_t kv_dtype;
+    float k_scale, v_scale;
+    uint8_t *pool;
+    int32_t *page_table, *page_fill;
+    DevStatus *status;
+    const CUtensorMap *pool_map;
+};
+bool cache_shape(const kvg_cache *c, CacheShape *out);
+int32_t cache_seq_pages(const kvg_cache *c, int32_t seq);
+kvg_status cache_plan_decode(const kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
+                             std::vector<DecodeParams> *plan, int64_t *max_units);
+void set_last_error(const char *msg);
+// Looks up the device address of the allocation-free decode's static scratch
+// on the current device (once per device) and so makes the module that
+// holds it resident there; called by kvg_cache_create with the cache's
+// device current.  Returns cudaSuccess or the lookup's error.
+cudaError_t noalloc_prepare_device(int device);
 
 // ------------------------------------------------------------ PTX helpers --
 #ifdef __CUDACC__

@@ -37,21 +37,21 @@ void *g_scratch_dev[kvg::kMaxDevices] = {};
 }  // namespace
 
 namespace kvg {
-// Read-only views of a cache's geometry and host bookkeeping (runtime.cu).
-struct CacheShape {
-    int32_t n_layers, n_kv_heads, head_dim, page_size, n_pages, max_seqs, max_pages, device, n_sm;
-    int32_t kv_dtype;
-    float k_scale, v_scale;
-    uint8_t *pool;
-    int32_t *page_table, *page_fill;
-    DevStatus *status;
-    const CUtensorMap *pool_map;
-};
-bool cache_shape(const kvg_cache *c, CacheShape *out);
-int32_t cache_seq_pages(const kvg_cache *c, int32_t seq);
-kvg_status cache_plan_decode(const kvg_cache *c, int32_t layer, const int32_t *seq_ids, int32_t B,
-                             std::vector<DecodeParams> *plan, int64_t *max_units);
-void set_last_error(const char *msg);
+cudaError_t noalloc_prepare_device(int device) {
+    if (device < 0 || device >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (g_scratch_dev[device]) return cudaSuccess;
+    void *p = nullptr;
+    // with the device current: resolves (and, under lazy module loading,
+    // loads) this file's module on it, which places the array in its memory
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_decode_scratch);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return e;
+    }
+    g_scratch_dev[device] = p;
+    return cudaSuccess;
+}
 }  // namespace kvg
 
 using namespace kvg;
@@ -111,18 +111,12 @@ extern "C" kvg_status kvg_decode_attention_noalloc(kvg_cache *c, int32_t layer, 
     } restore{prev, cs.device};
     void *scratch = nullptr;
     {
-        // first call on a device: look up the array's device address with
-        // that device current (no allocation happens here)
+        // the address was looked up when the cache was created on this
+        // device (kvg_cache_create); this call only reads it
         std::lock_guard<std::mutex> lk(g_mu);
-        if (!g_scratch_dev[cs.device]) {
-            cudaError_t e = cudaGetSymbolAddress(&g_scratch_dev[cs.device], g_decode_scratch);
-            if (e != cudaSuccess) {
-                g_scratch_dev[cs.device] = nullptr;
-                return reject(KVG_ERR_CUDA, std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e));
-            }
-        }
         scratch = g_scratch_dev[cs.device];
     }
+    if (!scratch) return reject(KVG_ERR_CUDA, "static decode scratch was not set up on the cache's device");
     const int w_max = decode_max_warps(cs.head_dim, G, fp8, cs.n_sm);
     if (w_max <= 0) return reject(KVG_ERR_CUDA, "decode kernel cannot be made resident");
     const int64_t w_cap = cap_slots - units < w_max ? cap_slots - units : w_max;

@@ -946,6 +946,10 @@ extern "C" kvg_status kvg_cache_create(const kvg_dims *dims, int32_t n_pages, in
     if (make_pool_tensor_map(&c->pool_map, c->pool, dims->head_dim, dims->kv_dtype == KVG_KV_E4M3, pool_rows) !=
         cudaSuccess)
         return cleanup(fail(KVG_ERR_CUDA, "tensor map of the pool could not be encoded"));
+    // the allocation-free decode's static scratch becomes resident on this
+    // device now, while the caller expects allocations, not at its first call
+    if (cudaError_t ne = noalloc_prepare_device(device); ne != cudaSuccess)
+        return cleanup(fail(KVG_ERR_CUDA, "static decode scratch lookup: %s", cudaGetErrorString(ne)));
     for (int32_t i = 0; i < n_pages; ++i) c->free_list.push_back(i);
     c->pinned.assign(n_pages, 0);
     c->alias.assign(n_pages, 0);
@@ -2072,16 +2076,7 @@ extern "C" const char *kvg_status_string(kvg_status s) {
 extern "C" const char *kvg_last_error(void) { return g_last_error.c_str(); }
 
 namespace kvg {
-// Read-only views used by noalloc.cu.
-struct CacheShape {
-    int32_t n_layers, n_kv_heads, head_dim, page_size, n_pages, max_seqs, max_pages, device, n_sm;
-    int32_t kv_dtype;
-    float k_scale, v_scale;
-    uint8_t *pool;
-    int32_t *page_table, *page_fill;
-    DevStatus *status;
-    const CUtensorMap *pool_map;
-};
+// Read-only views used by noalloc.cu (CacheShape is declared in common.cuh).
 bool cache_shape(const kvg_cache *c, CacheShape *out) {
     if (!c || !out) return false;
     *out = CacheShape{c->dims.n_layers, c->dims.n_kv_heads, c->dims.head_dim, c->dims.page_size, c->n_pages,
