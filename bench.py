@@ -38,7 +38,13 @@ import torch  # noqa: E402
 import kvg_synth as syn  # noqa: E402
 
 METRIC = ("graft GB/s (HBM & host→HBM) + decode-attn tokens/s @32k grafted, % roofline")
-SHA_OPS_PER_BLOCK = 1400  # fused 32-bit ops per SHA-256 compression (rotate, 3-input logic/add = 1)
+# ALU-pipe instructions per SHA-256 compression in graft_verify_kernel: the
+# kernel's own mix as ncu counts it (sm__inst_executed_pipe_alu over the
+# compressions of one launch, 4-layer 12b slice): 951 on the ALU pipe (funnel
+# shifts, 3-input logic), 739 on the FMA pipe (the additions and plain shifts
+# issued as IMADs), 47 other; 1,737 in all.  The ALU pipe is the binding one.
+SHA_ALU_OPS_PER_COMPRESSION = 951
+ALU_LANES_PER_SM = 64  # 4 SM sub-partitions x 16 ALU-pipe lanes
 
 
 def load_peaks():
@@ -187,22 +193,28 @@ class Step12B:
             self.windows = [0 if (l + 1) % R == 0 else W for l in range(w.n_layers)]
             kvg.kvg_cache_set_layer_windows(self.cache.h, self.windows)
         rows_read = sum(min(x, syn.B12_CTX) if x else syn.B12_CTX for x in self.windows)
+        # HBM algorithmic bytes of each phase: the graft copies the block
+        # (read + write); the digest check hashes the block's bytes, which
+        # must be read once from HBM only when no copy reads them (the
+        # zero-copy graft); the append reads the fresh rows and writes them;
+        # the decode reads every valid K/V row once
         self.bytes = {
             "graft": 0 if pool_store else 2 * blk_pages,
-            "verify": blk_pages,
+            "verify": blk_pages if pool_store else 0,
             "append": (2 + elem) * w.n_layers * 2 * self.nf * w.n_kv_heads * w.head_dim,
             "decode": rows_read * 2 * w.n_kv_heads * w.head_dim * elem + 2 * self.q.numel() * 2,
         }
+        # bytes the digest check hashes (not HBM traffic of their own when a
+        # copy reads them) and its SHA-256 compressions (65 per 4 KiB leaf)
+        self.hashed_bytes = blk_pages
         self.sha_blocks = (blk_pages // 4096) * 65
         self.blk_pages = blk_pages
-        # the step's work, whatever the schedule: block bytes copied (read +
-        # write) and hashed, fresh rows read and written, K/V rows decoded
+        # the step's HBM algorithmic bytes, whatever the schedule
         self.step_bytes = sum(self.bytes.values())
         self.schedule = schedule
         # phase -> (stream, first event, last event) of the per-step events
         if schedule == "fused":
-            self.bytes["graft_verify"] = self.bytes.pop("graft") or blk_pages
-            self.bytes.pop("verify")
+            self.bytes["graft_verify"] = self.bytes.pop("graft") + self.bytes.pop("verify")
             self.spans = {"release": ("main", 0, 1), "append": ("main", 1, 2), "graft_join": ("main", 2, 3),
                           "decode": ("main", 3, 4), "graft_verify": ("side", 0, 1)}
         else:
@@ -310,6 +322,7 @@ def run_kvg(args, rank, world):
     stream = torch.cuda.Stream(device, priority=torch.cuda.Stream.priority_range()[1])
     side = torch.cuda.Stream(device)
     hbm_peak, sm_max, peak_kind = load_peaks()
+    n_sm = torch.cuda.get_device_properties(device).multi_processor_count
     swa = tuple(int(x) for x in args.swa.split(":")) if args.swa else None
     st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool", schedule=args.schedule,
                  swa=swa, kv=args.kv)
@@ -404,33 +417,36 @@ def run_kvg(args, rank, world):
     traffic = load_traffic()
     parts = {}
     hashing = ("verify", "graft_verify")
+    alu_peak = n_sm * ALU_LANES_PER_SM * sm_max * 1e6  # ALU-pipe ops per second at the max SM clock
     for p in st.phases:
         ms = phase_ms[p]
-        if not st.bytes.get(p):
+        if not st.bytes.get(p) and p not in hashing:
             parts[p] = {"ms": round(ms, 4)}
             continue
-        b = st.bytes[p]
-        gbs = b / (ms * 1e-3) / 1e9
-        parts[p] = {"ms": round(ms, 4), "algorithmic_bytes": b, "gbs": round(gbs, 1)}
+        b = st.bytes.get(p, 0)
+        parts[p] = {"ms": round(ms, 4), "algorithmic_bytes": b}
+        if b:
+            gbs = b / (ms * 1e-3) / 1e9
+            parts[p].update({"gbs": round(gbs, 1), "hbm_frac": round(gbs / hbm_peak, 3)})
         if p in hashing:
-            ops = st.sha_blocks * SHA_OPS_PER_BLOCK
-            alu_peak = 152 * 64 * sm_max * 1e6
-            parts[p].update({"gops": round(ops / (ms * 1e-3) / 1e9, 1),
+            ops = st.sha_blocks * SHA_ALU_OPS_PER_COMPRESSION
+            parts[p].update({"hashed_bytes": st.hashed_bytes,
+                             "hashed_gbs": round(st.hashed_bytes / (ms * 1e-3) / 1e9, 1),
+                             "compressions": st.sha_blocks,
+                             "alu_ops_per_compression": SHA_ALU_OPS_PER_COMPRESSION,
+                             "alu_tops": round(ops / (ms * 1e-3) / 1e12, 3),
                              "alu_frac": round(ops / (ms * 1e-3) / alu_peak, 3)})
-        if p != "verify":
-            parts[p]["hbm_frac"] = round(gbs / hbm_peak, 3)
     parts["decode"]["tokens_per_s"] = round(1e3 / phase_ms["decode"], 1)
     kernel_of = {"graft": "graft_kernel", "verify": "sha256_leaves_kernel", "append": "append_tma_kernel",
                  "decode": "decode_kernel", "graft_verify": "graft_verify_kernel"}
     # dominant kernel: the longest phase that moves or hashes bytes
-    dom = max((p for p in st.phases if st.bytes.get(p)), key=lambda p: phase_ms[p])
+    dom = max((p for p in st.phases if st.bytes.get(p) or p in hashing), key=lambda p: phase_ms[p])
     if dom in hashing:
-        ops = st.sha_blocks * SHA_OPS_PER_BLOCK
+        ops = st.sha_blocks * SHA_ALU_OPS_PER_COMPRESSION
         ach = ops / (phase_ms[dom] * 1e-3) / 1e12
-        peak = 152 * 64 * sm_max * 1e6 / 1e12
-        roof = {"bound": "alu", "kernel": kernel_of[dom], "achieved": round(ach, 3), "peak": round(peak, 3),
-                "unit": "Top/s", "frac": round(ach / peak, 3), "traffic": traffic.get(kernel_of[dom]),
-                "peak_kind": "derived: 152 SMs x 64 int32 lanes x max SM clock"}
+        roof = {"bound": "alu", "kernel": kernel_of[dom], "achieved": round(ach, 3), "peak": round(alu_peak / 1e12, 3),
+                "unit": "Top/s", "frac": round(ach / (alu_peak / 1e12), 3), "traffic": traffic.get(kernel_of[dom]),
+                "peak_kind": f"derived: {n_sm} SMs x {ALU_LANES_PER_SM} ALU-pipe lanes x max SM clock"}
     else:
         ach = st.bytes[dom] / (phase_ms[dom] * 1e-3) / 1e9
         roof = {"bound": "hbm", "kernel": kernel_of[dom], "achieved": round(ach, 1), "peak": hbm_peak,
@@ -463,17 +479,14 @@ def run_kvg(args, rank, world):
 # The other workloads (run with --config; the default line is the 12B step)
 # --------------------------------------------------------------------------
 
-def _gen_chunks(w, n_chunks, rows, seed, device):
-    """A small pool of distinct prefill-shaped K/V chunks [L][rows][Hkv][D]."""
-    return [syn.kv_rows(w, rows, seed + 17 * c, device) for c in range(n_chunks)]
-
-
 class Step31B:
     """31B-class relocation: a 16,384-token block deposited at positions
     0..16,383; 8 sequences hold it re-based by delta in {0, 1, 4096, 100000}
     followed by 49,152 fresh rows (65,536-token contexts).  One step =
     relocating graft (delta 4096) of the block into a spare sequence + decode
-    of one token for the 8 sequences over all 60 layers."""
+    of one token for the 8 sequences over all 60 layers.  Every chunk of rows
+    (the block's and each sequence's fresh rows) is its own N(0, 1) draw, so
+    no two slot ranges hold the same K/V."""
 
     CHUNK = 2048
 
@@ -490,26 +503,25 @@ class Step31B:
         self.store = kvg.Store(self.dims, kvg.KVG_RESIDENCY_HBM, blk_bytes + (64 << 20))
         c = self.cache.h
         with torch.cuda.stream(stream):
-            # the block: written fresh into the spare sequence, deposited, released
-            # (generated one chunk at a time: the cache leaves little room)
-            self.blk_sample = []
+            # the block: written fresh into the spare sequence, deposited,
+            # released; then every sequence's relocated graft and its fresh
+            # rows.  Rows are generated one chunk at a time (the cache leaves
+            # little room) on this stream, which also frees them.
             for i in range(self.nb // self.CHUNK):
-                k, v = syn.kv_rows(w, self.CHUNK, w.seed + 17 * i, device)
+                k, v = self.block_rows(i, device)
                 pos = torch.arange(i * self.CHUNK, (i + 1) * self.CHUNK, dtype=torch.int32, device=device)
                 kvg.kvg_cache_append(c, self.B, k.data_ptr(), v.data_ptr(), pos.data_ptr(), self.CHUNK, stream)
-                self.blk_sample.append((k[:, :, :1].clone(), v[:, :, :1].clone()))  # kv head 0 only
-                stream.synchronize()
                 del k, v, pos
             self.bid = kvg.kvg_deposit(self.store.h, c, self.B, 0, self.nb, stream)
             kvg.kvg_cache_release(c, self.B, stream)
-            self.fresh = _gen_chunks(w, 4, self.CHUNK, w.seed + 1000, device)
             for sq in range(self.B):
                 kvg.kvg_graft(self.store.h, self.bid, c, sq, -1, self.deltas[sq], 0, stream)
-                for i in range((self.ctx - self.nb) // self.CHUNK):
-                    k, v = self.fresh[(sq * 7 + i) % len(self.fresh)]
+                for i in range(self.n_fresh_chunks):
+                    k, v = self.fresh_rows(sq, i, device)
                     p0 = self.deltas[sq] + self.nb + i * self.CHUNK
                     pos = torch.arange(p0, p0 + self.CHUNK, dtype=torch.int32, device=device)
                     kvg.kvg_cache_append(c, sq, k.data_ptr(), v.data_ptr(), pos.data_ptr(), self.CHUNK, stream)
+                    del k, v, pos
             self.q = syn.queries(w, w.n_layers, self.B, w.seed, device)
             self.out = torch.empty_like(self.q)
         stream.synchronize()
@@ -519,6 +531,18 @@ class Step31B:
                       "decode": self.B * w.n_layers * 2 * self.ctx * w.n_kv_heads * w.head_dim * 2
                                 + 2 * self.q.numel() * 2}
         self.phases = ["release", "relocate", "decode"]
+
+    @property
+    def n_fresh_chunks(self):
+        return (self.ctx - self.nb) // self.CHUNK
+
+    def block_rows(self, i, device):
+        """K, V of the block's chunk i (rows i*CHUNK ...), bf16 [L][CHUNK][Hkv][D]."""
+        return syn.kv_rows(self.w, self.CHUNK, self.w.seed + 17 * i, device)
+
+    def fresh_rows(self, sq, i, device):
+        """K, V of sequence sq's fresh chunk i (slots nb + i*CHUNK ...)."""
+        return syn.kv_rows(self.w, self.CHUNK, self.w.seed + 100_000 + 64 * sq + i, device)
 
     def run_step(self, ev=None):
         kvg, s, c = self.kvg, self.stream, self.cache.h
@@ -896,7 +920,9 @@ def oracle_sample(n_layers_sample: int, chunk: int = 4):
             cache.decode(0, l, q[l, 0], scale)
         total_t += time.perf_counter() - t0
         blk_pages = w.n_layers * 2 * (nb // w.page_size) * w.page_bytes
-        total_b += 2 * blk_pages + blk_pages + 2 * w.n_layers * 2 * nf * w.n_kv_heads * w.head_dim * 2 \
+        # HBM algorithmic bytes, as the GPU step counts them: block copied,
+        # fresh rows read and written, every row decoded (hashing adds none)
+        total_b += 2 * blk_pages + 2 * w.n_layers * 2 * nf * w.n_kv_heads * w.head_dim * 2 \
             + w.n_layers * 2 * syn.B12_CTX * w.n_kv_heads * w.head_dim * 2
     return total_t, total_b, oracle.omp_threads()
 

@@ -4,6 +4,7 @@ its C ABI, the oracle on the CPU), each fed the same seeded bytes."""
 from __future__ import annotations
 
 import math
+import os
 
 import numpy as np
 import pytest
@@ -105,10 +106,54 @@ def decode(kvg, cache, w, seq_ids, q: np.ndarray, layer=-1) -> np.ndarray:
     return u16(out)
 
 
-def compare_decode(oracle, o_gpu_bits: np.ndarray, o_ref: np.ndarray, tol=1e-2):
+# Decode gate (paper Sec. 3.2 for the attention being computed; Sec. 4.1 for
+# the byte-exact regime it is checked in).  Three bounds, all on one output
+# (every query head of one (layer, batch row)):
+#   * max |got - ref| <= 1e-2, the stated tolerance for bf16 outputs;
+#   * max |got - ref| / max |ref| <= REL_TOL.  The kernel's only rounding
+#     steps that matter are the softmax weights, rounded to bf16 before the
+#     P.V product (relative error <= 2^-9 each, uniform, so a weighted error
+#     of ~2^-9/sqrt(3) of the output's own scale, ~4 sigma at the maximum of
+#     a few thousand elements), and the output's bf16 rounding (<= 2^-9 of
+#     the element).  Together ~3.6e-3 of max |ref| at every context length
+#     from 2 to 65,536 rows (a numpy model of these roundings on N(0, 1)
+#     rows); REL_TOL = 2^-7 leaves a factor ~2 of margin.  Dropping 1% of a
+#     32k context's rows moves the output by ~1e-1 of max |ref| (0.1%: 3e-2),
+#     so a partial-context bug fails this bound;
+#   * the fraction of elements equal to bf16_rne(ref) >= RNE_FLOOR (checked
+#     on outputs of >= 256 elements).  The same model gives 0.52-0.81 (most
+#     rounding boundaries lie farther from the exact value than the weights'
+#     error); dropping 1% (0.1%) of the rows leaves ~0.02 (~0.08).
+REL_TOL = 2.0 ** -7
+RNE_FLOOR = 0.35
+# Keys and the query re-rotated by RoPE (relocation, Sec. 4.2) and rounded to
+# bf16 before the score, compared with the un-rotated reference: each score
+# gains an error of ~1.6e-3, the model's maximum becomes ~5.4e-3 of max |ref|
+# and the RNE match 0.40-0.48.
+REL_TOL_RELOCATED = 2.0 ** -6
+RNE_FLOOR_RELOCATED = 0.25
+
+
+def compare_decode(oracle, o_gpu_bits: np.ndarray, o_ref: np.ndarray, tol=1e-2, rel=REL_TOL, floor=RNE_FLOOR,
+                   what=""):
+    """Checks one decode output against the fp64 oracle with the three bounds
+    above; returns (max-abs error, relative error, RNE-match fraction).  With
+    KVG_DECODE_GATE_LOG set, appends the figures to that file."""
     got = oracle.bf16_to_f64(o_gpu_bits)
-    err = np.abs(got - o_ref).max() if got.size else 0.0
+    if not got.size:
+        return 0.0, 0.0, 1.0
+    err = float(np.abs(got - o_ref).max())
+    top = float(np.abs(o_ref).max())
+    relerr = err / top if top > 0 else (0.0 if err == 0 else math.inf)
     rne = oracle.bf16_rne(o_ref)
-    match = float((rne == o_gpu_bits).mean()) if got.size else 1.0
-    assert err <= tol, f"max-abs error {err} > {tol}"
-    return err, match
+    match = float((rne == o_gpu_bits).mean())
+    log = os.environ.get("KVG_DECODE_GATE_LOG")
+    if log:
+        with open(log, "a") as f:
+            f.write(f"{what or os.environ.get('PYTEST_CURRENT_TEST', '?')}\t{got.size}\t{err:.3e}\t"
+                    f"{relerr:.3e}\t{match:.4f}\n")
+    assert err <= tol, f"{what}: max-abs error {err} > {tol}"
+    assert relerr <= rel, f"{what}: relative error {relerr:.3e} > {rel:.3e} (max |ref| {top:.3e})"
+    if got.size >= 256:
+        assert match >= floor, f"{what}: RNE match {match:.3f} < {floor}"
+    return err, relerr, match

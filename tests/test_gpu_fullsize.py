@@ -1,9 +1,11 @@
 """Parity at the benchmark's full sizes, in the launch configuration bench.py
 times (its workload classes build the state): bit-exact block bytes, page
-digests, page tables and restored pages against the oracle; attention and
-relocated keys on sampled (sequence, layer, head) outputs the oracle computes
-one by one; the grafted-vs-fresh SHA-256 gate and run-to-run determinism at
-32k context; the deep store's planted needles on every one of 1,000 grafts."""
+digests, page tables and restored pages against the oracle; attention on
+every query head of two layers (of several sequences where there are
+several), through the decode gate of kvg_testlib.compare_decode, and
+relocated keys on sampled pages; the grafted-vs-fresh SHA-256 gate and
+run-to-run determinism at 32k context; the deep store's planted needles on
+every one of 1,000 grafts."""
 import hashlib
 import math
 
@@ -12,7 +14,7 @@ import pytest
 import torch
 
 import kvg_synth as syn
-from kvg_testlib import dev_view, need_gpu, tables
+from kvg_testlib import compare_decode, dev_view, need_gpu, tables
 
 pytestmark = pytest.mark.gpu
 
@@ -87,15 +89,15 @@ def test_12b_single_graft_full_size(oracle):
         for _ in range(48):
             l, kv, j = int(rng.integers(w.n_layers)), int(rng.integers(2)), int(rng.integers(nb // P))
             assert np.array_equal(_pool_page(st.cache, w, l, kv, pt[0, j]), blk.pages[l, kv, j])
-        # decode: sampled heads against fp64 attention over all 32,768 rows
+        # decode: every query head of two layers against fp64 attention over
+        # all 32,768 rows, through the decode gate
         kf, vf = st.kf, st.vf
-        for l, h in [(0, 0), (17, 5), (w.n_layers - 1, w.n_q_heads - 1)]:
-            g = h // w.group
-            k = np.concatenate([kb[l, :, g], syn.as_u16(kf[l, :, g])])
-            v = np.concatenate([vb[l, :, g], syn.as_u16(vf[l, :, g])])
-            ref = oracle.attention_head(syn.as_u16(st.q[l, 0, h]), k, v, st.scale)
-            got = oracle.bf16_to_f64(syn.as_u16(st.out[l, 0, h]))
-            assert np.abs(got - ref).max() <= 1e-2
+        rows = {}
+        for l in (0, 17, w.n_layers - 1):
+            rows[l] = (np.concatenate([kb[l], syn.as_u16(kf[l])]), np.concatenate([vb[l], syn.as_u16(vf[l])]))
+        for l in (0, w.n_layers - 1):
+            ref = oracle.gqa_decode(syn.as_u16(st.q[l, 0]), rows[l][0], rows[l][1], st.scale)
+            compare_decode(oracle, syn.as_u16(st.out[l, 0]), ref, what=f"12b layer {l}")
         # the same 32,768 rows written fresh into other pages: SHA-256-identical output
         out_grafted = st.out.clone()
         fresh = kvg.Cache(st.dims, st.cache.view.n_pages, 1, syn.B12_CTX)
@@ -116,8 +118,8 @@ def test_12b_single_graft_full_size(oracle):
         # the end-to-end form: verified graft from the pinned-host store (16
         # chunks on a capped grid) with the split decode (fresh rows while the
         # block streams in, the block's rows merged after): digests verified,
-        # restored pages bit-exact, sampled heads within 1e-2 of fp64, bitwise
-        # reproducible
+        # restored pages bit-exact, every head of two layers through the decode
+        # gate, bitwise reproducible
         st.run_step_split(st.hstore.h, st.hbid)
         s.synchronize()
         kvg.kvg_sync(st.cache.h, s, 60.0)
@@ -126,18 +128,38 @@ def test_12b_single_graft_full_size(oracle):
             l, kv, j = int(rng.integers(w.n_layers)), int(rng.integers(2)), int(rng.integers(nb // P))
             assert np.array_equal(_pool_page(st.cache, w, l, kv, pt[0, j]), blk.pages[l, kv, j])
         out_split = st.out.clone()
-        for l, h in [(0, 0), (23, 9), (w.n_layers - 1, w.n_q_heads - 1)]:
-            g = h // w.group
-            k = np.concatenate([kb[l, :, g], syn.as_u16(kf[l, :, g])])
-            v = np.concatenate([vb[l, :, g], syn.as_u16(vf[l, :, g])])
-            ref = oracle.attention_head(syn.as_u16(st.q[l, 0, h]), k, v, st.scale)
-            assert np.abs(oracle.bf16_to_f64(syn.as_u16(out_split[l, 0, h])) - ref).max() <= 1e-2
+        for l in (17, w.n_layers - 1):
+            ref = oracle.gqa_decode(syn.as_u16(st.q[l, 0]), rows[l][0], rows[l][1], st.scale)
+            compare_decode(oracle, syn.as_u16(out_split[l, 0]), ref, what=f"12b split layer {l}")
         assert float((out_split.float() - out_grafted.float()).abs().max()) <= 1e-2
         st.run_step_split(st.hstore.h, st.hbid)
         s.synchronize()
         assert _sha(st.out) == _sha(out_split)
     finally:
         _close(*(x for x in (fresh, st.cache, st.store, st.hstore) if x is not None))
+
+
+def _rows31(st, dev, layers, seqs):
+    """Host copies (uint16 [len(layers)][rows][Hkv][D]) of the K/V rows the
+    31B workload wrote: the block's rows (as deposited) and each listed
+    sequence's fresh rows, regenerated chunk by chunk from their seeds."""
+    li = torch.tensor(layers, device=dev)
+    kb, vb = [], []
+    for i in range(st.nb // st.CHUNK):
+        k, v = st.block_rows(i, dev)
+        kb.append(syn.as_u16(k.index_select(0, li)))
+        vb.append(syn.as_u16(v.index_select(0, li)))
+        del k, v
+    fresh = {}
+    for sq in seqs:
+        kf, vf = [], []
+        for i in range(st.n_fresh_chunks):
+            k, v = st.fresh_rows(sq, i, dev)
+            kf.append(syn.as_u16(k.index_select(0, li)))
+            vf.append(syn.as_u16(v.index_select(0, li)))
+            del k, v
+        fresh[sq] = (np.concatenate(kf, axis=1), np.concatenate(vf, axis=1))
+    return np.concatenate(kb, axis=1), np.concatenate(vb, axis=1), fresh
 
 
 def test_31b_relocation_full_size(oracle):
@@ -152,41 +174,51 @@ def test_31b_relocation_full_size(oracle):
         kvg.kvg_sync(st.cache.h, s, 60.0)
         w, nb, P = st.w, st.nb, st.w.page_size
         pt, pf, ps = tables(st.cache)
-        kb = torch.cat([k for k, _ in st.blk_sample], dim=1)[:, :, 0]  # [L][nb][D], kv head 0
-        vb = torch.cat([v for _, v in st.blk_sample], dim=1)[:, :, 0]
         # position tags: block tags + delta, then the fresh rows' tags
         for sq in range(st.B):
             d = st.deltas[sq]
             assert np.array_equal(ps[sq, :nb], np.arange(nb) + d)
             assert np.array_equal(ps[sq, nb:st.ctx], np.arange(nb, st.ctx) + d)
         assert np.array_equal(ps[st.B, :nb], np.arange(nb) + 4096)  # the timed relocation
-        # relocated keys (kv head 0) within 2e-2 of the fp64 rotation; values bit-exact
+        sample_layers = [0, 29, w.n_layers - 1]
+        seqs = [0, 1, 3, 6]  # delta 0, 1, 100000, 4096
+        kb, vb, fresh = _rows31(st, dev, sample_layers, seqs)
+        # relocated keys (every kv head) within 2e-2 of the fp64 rotation;
+        # values and delta-0 keys bit-exact
         rng = np.random.default_rng(3)
         for sq, d in [(3, st.deltas[3]), (1, st.deltas[1]), (0, 0), (st.B, 4096)]:
             for _ in range(6):
-                l, j = int(rng.integers(w.n_layers)), int(rng.integers(nb // P))
-                kpage = _pool_page(st.cache, w, l, 0, pt[sq, j])[0]
-                vpage = _pool_page(st.cache, w, l, 1, pt[sq, j])[0]
-                rows_k = syn.as_u16(kb[l, j * P:(j + 1) * P])
-                rows_v = syn.as_u16(vb[l, j * P:(j + 1) * P])
+                li, j = int(rng.integers(len(sample_layers))), int(rng.integers(nb // P))
+                l = sample_layers[li]
+                kpage = _pool_page(st.cache, w, l, 0, pt[sq, j])
+                vpage = _pool_page(st.cache, w, l, 1, pt[sq, j])
+                rows_k = kb[li, j * P:(j + 1) * P].transpose(1, 0, 2)  # [Hkv][P][D]
+                rows_v = vb[li, j * P:(j + 1) * P].transpose(1, 0, 2)
                 assert np.array_equal(vpage, rows_v)
                 if d == 0:
                     assert np.array_equal(kpage, rows_k)
                 else:
                     ref = oracle.rope_rotate_rows(rows_k, d, w.rope_theta, 0)
                     assert np.abs(oracle.bf16_to_f64(kpage) - ref).max() <= 2e-2
-        # decode: sampled (sequence, layer) for query head 0 against fp64 attention
-        for sq in (0, 3, 6):
-            fr = [st.fresh[(sq * 7 + i) % len(st.fresh)] for i in range((st.ctx - nb) // st.CHUNK)]
-            for l in (0, w.n_layers - 1):
-                kblk = syn.as_u16(kb[l])
-                if st.deltas[sq]:
-                    kblk = oracle.rope_rotate_rows_bf16(kblk, st.deltas[sq], w.rope_theta, 0)
-                k = np.concatenate([kblk] + [syn.as_u16(f[0][l, :, 0]) for f in fr])
-                v = np.concatenate([syn.as_u16(vb[l])] + [syn.as_u16(f[1][l, :, 0]) for f in fr])
-                ref = oracle.attention_head(syn.as_u16(st.q[l, sq, 0]), k, v, st.scale)
-                got = oracle.bf16_to_f64(syn.as_u16(st.out[l, sq, 0]))
-                assert np.abs(got - ref).max() <= 1e-2
+        # the fresh rows landed where the oracle's bookkeeping puts them (one
+        # sampled page per sampled sequence and layer)
+        for sq in seqs:
+            j = nb // P + int(rng.integers((st.ctx - nb) // P))
+            t0 = j * P - nb
+            for li, l in enumerate(sample_layers):
+                assert np.array_equal(_pool_page(st.cache, w, l, 0, pt[sq, j]),
+                                      fresh[sq][0][li, t0:t0 + P].transpose(1, 0, 2))
+        # decode: every query head of two layers of four sequences against
+        # fp64 attention over all 65,536 rows, through the decode gate
+        for sq in seqs:
+            d = st.deltas[sq]
+            for li in (0, len(sample_layers) - 1):
+                l = sample_layers[li]
+                kblk = kb[li] if d == 0 else oracle.rope_rotate_rows_bf16(kb[li], d, w.rope_theta, 0)
+                k = np.concatenate([kblk, fresh[sq][0][li]])
+                v = np.concatenate([vb[li], fresh[sq][1][li]])
+                ref = oracle.gqa_decode(syn.as_u16(st.q[l, sq]), k, v, st.scale)
+                compare_decode(oracle, syn.as_u16(st.out[l, sq]), ref, what=f"31b seq {sq} layer {l}")
     finally:
         _close(st.cache, st.store)
 
@@ -236,20 +268,19 @@ def test_batched_library_full_size(oracle):
                             got, want = got[:, :n % P], want[:, :n % P]
                         assert np.array_equal(got, want)
                 j0 += blk.n_pages
-        # decode after the last step: sampled heads against fp64 attention
-        for sq in (0, nS - 1):
+        # decode after the last step: every query head of two layers of three
+        # sequences against fp64 attention, through the decode gate
+        for sq in (0, 13, nS - 1):
             for l in (0, w.n_layers - 1):
                 ks, vs = [], []
                 for b in st.ids[sq]:
                     k, v = syn.kv_rows(w, int(st.lens[b]), w.seed + int(b), "cuda")
-                    ks.append(syn.as_u16(k[l, :, 0]))
-                    vs.append(syn.as_u16(v[l, :, 0]))
-                ks.append(syn.as_u16(st.kd[l, sq::nS, 0]))
-                vs.append(syn.as_u16(st.vd[l, sq::nS, 0]))
-                ref = oracle.attention_head(syn.as_u16(st.q[l, sq, 0]), np.concatenate(ks), np.concatenate(vs),
-                                            st.scale)
-                got = oracle.bf16_to_f64(syn.as_u16(st.out[l, sq, 0]))
-                assert np.abs(got - ref).max() <= 1e-2
+                    ks.append(syn.as_u16(k[l]))
+                    vs.append(syn.as_u16(v[l]))
+                ks.append(syn.as_u16(st.kd[l, sq::nS]))
+                vs.append(syn.as_u16(st.vd[l, sq::nS]))
+                ref = oracle.gqa_decode(syn.as_u16(st.q[l, sq]), np.concatenate(ks), np.concatenate(vs), st.scale)
+                compare_decode(oracle, syn.as_u16(st.out[l, sq]), ref, what=f"batched seq {sq} layer {l}")
     finally:
         _close(st.cache, st.store)
 
@@ -281,10 +312,8 @@ def test_deep_store_needles_full_size(oracle):
         # the needle read matches fp64 attention over the grafted rows (sampled)
         b = int(st.order[-1])
         k, v = st.block_rows(b, dev)
-        for l, h in [(0, 0), (1, w.n_q_heads - 1)]:
-            g = h // w.group
-            ref = oracle.attention_head(syn.as_u16(st.q[l, 0, h]), syn.as_u16(k[l, :, g]), syn.as_u16(v[l, :, g]),
-                                        st.scale)
-            assert np.abs(oracle.bf16_to_f64(syn.as_u16(st.out[l, 0, h])) - ref).max() <= 1e-2
+        for l in range(w.n_layers):
+            ref = oracle.gqa_decode(syn.as_u16(st.q[l, 0]), syn.as_u16(k[l]), syn.as_u16(v[l]), st.scale)
+            compare_decode(oracle, syn.as_u16(st.out[l, 0]), ref, what=f"deep block {b} layer {l}")
     finally:
         _close(st.cache, st.store)

@@ -1,8 +1,10 @@
 """GPU parity: the CUDA library (through its C ABI) against the CPU oracle on
 the same seeded inputs.  Graft, page tables, positions, block bytes and
 digests must match bit for bit; decode attention within 1e-2 max-abs of the
-fp64 oracle (bf16 out, fp32 accumulate); relocated keys within 2e-2 of the
-fp64 rotation; grafted-vs-fresh attention outputs SHA-256-identical."""
+fp64 oracle (bf16 out, fp32 accumulate), within 2^-7 of its largest element
+and with at least 35% of elements equal to the oracle's bf16 rounding
+(kvg_testlib.compare_decode); relocated keys within 2e-2 of the fp64
+rotation; grafted-vs-fresh attention outputs SHA-256-identical."""
 import hashlib
 import math
 
@@ -11,8 +13,8 @@ import pytest
 import torch
 
 import kvg_synth as syn
-from kvg_testlib import (CANARY, append, compare_decode, decode, dev_view, dims_for, fill_canary,
-                         geometry, need_gpu, oracle_dims, pool_u16, tables, to_dev, u16)
+from kvg_testlib import (CANARY, REL_TOL_RELOCATED, RNE_FLOOR_RELOCATED, append, compare_decode, decode, dev_view,
+                         dims_for, fill_canary, geometry, need_gpu, oracle_dims, pool_u16, tables, to_dev, u16)
 
 pytestmark = pytest.mark.gpu
 
@@ -355,7 +357,14 @@ def test_relocated_decode_is_delta_invariant_within_tolerance(oracle):
         qd = np.stack([oracle.rope_rotate_rows_bf16(q0[l], delta, w.rope_theta, 0) for l in range(w.n_layers)])
         o = decode(kvg, s["dst"], w, [seq], qd)
         for l in range(w.n_layers):
-            compare_decode(oracle, o[l, 0], ref[l])
+            # the same query over the keys as the cache holds them (rotated,
+            # rounded to bf16): only the kernel's own rounding remains
+            kr = s["k"][l] if delta == 0 else oracle.rope_rotate_rows_bf16(s["k"][l], delta, w.rope_theta, 0)
+            compare_decode(oracle, o[l, 0], oracle.gqa_decode(qd[l, 0], kr, s["v"][l], scale), what=f"reloc {delta}")
+            # against the un-rotated fp64 reference: q and k also carry the
+            # bf16 rounding of their rotation
+            compare_decode(oracle, o[l, 0], ref[l], rel=REL_TOL_RELOCATED, floor=RNE_FLOOR_RELOCATED,
+                           what=f"reloc-invariance {delta}")
 
 
 # ------------------------------------------------------- integrity & errors
@@ -959,7 +968,9 @@ def test_launch_chunking_limits(oracle):
     qd = to_dev(q)
     kvg.kvg_decode_attention_noalloc(dst.h, -1, ids, qd.data_ptr(), w.n_q_heads, o_noalloc.data_ptr(), scale)
     torch.cuda.synchronize()
-    assert np.abs(oracle.bf16_to_f64(u16(o_noalloc)) - oracle.bf16_to_f64(o)).max() <= 1e-2
+    # the same plan and worker count (the static scratch's cap does not bind
+    # at 256 rows per launch here), so the same bytes
+    assert np.array_equal(u16(o_noalloc), o)
 
 
 def test_device_wait_gives_up_and_reports(oracle):
