@@ -20,6 +20,7 @@ replica (weak scaling); there is no data-path collective.
 from __future__ import annotations
 
 import argparse
+import gc
 import json
 import math
 import os
@@ -323,6 +324,7 @@ def run_kvg(args, rank, world):
     side = torch.cuda.Stream(device)
     hbm_peak, sm_max, peak_kind = load_peaks()
     n_sm = torch.cuda.get_device_properties(device).multi_processor_count
+    alu_peak = n_sm * ALU_LANES_PER_SM * sm_max * 1e6  # ALU-pipe ops per second at the max SM clock
     swa = tuple(int(x) for x in args.swa.split(":")) if args.swa else None
     st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool", schedule=args.schedule,
                  swa=swa, kv=args.kv)
@@ -364,6 +366,34 @@ def run_kvg(args, rank, world):
     phase_ms = {p: statistics.mean(evs[k][sn][i].elapsed_time(evs[k][sn][j]) for k in range(K))
                 for p, (sn, i, j) in st.spans.items()}
     deterministic = _sha_tensor(st.out) == first_sha
+
+    # each graft form alone (CUDA events, median of 8 after 3 untimed): the
+    # plain own-position graft (HBM-bound) and the verified one (ALU-bound)
+    alone = {}
+    if not st.pool_store:
+        for name, flags in (("graft_alone", 0), ("graft_verify_alone", kvg.KVG_GRAFT_VERIFY)):
+            g0, g1 = mk(), mk()
+            gts = []
+            clk_g = None
+            for k in range(11):
+                if k == 3:
+                    clk_g = Clocks(local)
+                kvg.kvg_cache_release(st.cache.h, 0, stream)
+                g0.record(stream)
+                kvg.kvg_graft(st.store.h, st.bid, st.cache.h, 0, -1, 0, flags, stream)
+                g1.record(stream)
+                stream.synchronize()
+                if k >= 3:
+                    gts.append(g0.elapsed_time(g1))
+            ms = statistics.median(gts)
+            b = 2 * st.blk_pages
+            alone[name] = {"ms": round(ms, 4), "algorithmic_bytes": b, "gbs": round(b / (ms * 1e-3) / 1e9, 1),
+                           "hbm_frac": round(b / (ms * 1e-3) / 1e9 / hbm_peak, 3), "clocks": clk_g.stop()}
+            if flags:
+                ops = st.sha_blocks * SHA_ALU_OPS_PER_COMPRESSION
+                alone[name].update({"alu_tops": round(ops / (ms * 1e-3) / 1e12, 3),
+                                    "alu_frac": round(ops / (ms * 1e-3) / alu_peak, 3)})
+        kvg.kvg_sync(st.cache.h, stream, 60.0)
 
     # e2e: host-store graft, query from pinned host memory, output read back.
     # With the fused schedule the decode is split: the part over the fresh
@@ -413,11 +443,14 @@ def run_kvg(args, rank, world):
             stream.synchronize()
             gts.append(e0.elapsed_time(e1))
         e2e["host_graft_gbs"] = round(blk_read / (statistics.median(gts) * 1e-3) / 1e9, 2)
+        # the host link's ceiling in the same run: pinned cudaMemcpyAsync H2D of 1 GiB
+        h2d = measure_h2d(device, 1 << 30, 5)
+        e2e["h2d_ceiling_gbs"] = round(h2d, 2)
+        e2e["host_graft_link_frac"] = round(e2e["host_graft_gbs"] / h2d, 3)
 
     traffic = load_traffic()
     parts = {}
     hashing = ("verify", "graft_verify")
-    alu_peak = n_sm * ALU_LANES_PER_SM * sm_max * 1e6  # ALU-pipe ops per second at the max SM clock
     for p in st.phases:
         ms = phase_ms[p]
         if not st.bytes.get(p) and p not in hashing:
@@ -467,7 +500,7 @@ def run_kvg(args, rank, world):
         "config": dict(config_12b(st.w.n_layers, world, pool_store=st.pool_store, swa=st.swa, kv=st.kv),
                        schedule="verified graft in one pass, beside the append" if st.schedule == "fused"
                        else "graft, then the digest check beside the append and the decode"),
-        "parts": parts, "roofline": roof, "e2e": e2e, "gpu_launches": int(launches),
+        "parts": parts, "alone": alone, "roofline": roof, "e2e": e2e, "gpu_launches": int(launches),
         "clocks": clk, "checks": {"deterministic": deterministic, "out_sha256": first_sha,
                                   "digest_verified_steps": K + args.warmup + 1,
                                   "e2e_out_max_abs_vs_device_out": e2e_vs_device},
@@ -604,9 +637,12 @@ class StepBatched:
     """Batched library graft on a layer slice of the 12B shape: a 512-block
     HBM store (lengths U{2048..6144}); 32 sequences each graft 4 distinct
     blocks at their own positions (page-aligned, stitched), then 64 decode
-    steps append one row per sequence and decode all 32."""
+    steps append one row per sequence and decode all 32.  consecutive=True:
+    blocks 2-4 of each sequence are re-based by the tokens already in it, so
+    its position tags run without a gap (the same single batched call, with
+    per-graft deltas; their keys are rotated during the copy)."""
 
-    def __init__(self, kvg, device, stream, n_layers=4):
+    def __init__(self, kvg, device, stream, n_layers=4, consecutive=False):
         self.kvg, self.stream = kvg, stream
         self.w = w = syn.BATCHED.with_layers(n_layers or 4)
         P = w.page_size
@@ -652,6 +688,15 @@ class StepBatched:
         self.batch_seqs = [sq for sq in range(nS) for _ in self.ids[sq]]
         self.step_k = [self.kd[:, t * nS:(t + 1) * nS].contiguous() for t in range(self.steps)]
         self.step_v = [self.vd[:, t * nS:(t + 1) * nS].contiguous() for t in range(self.steps)]
+        self.set_consecutive(consecutive)
+
+    def set_consecutive(self, consecutive):
+        """Own positions (False) or blocks 2-4 of each sequence re-based by the
+        tokens already in it (True), from the next step on."""
+        nS = syn.BATCHED_SEQS
+        self.consecutive = consecutive
+        self.batch_deltas = ([int(sum(int(self.lens[b]) for b in self.ids[sq][:i])) for sq in range(nS)
+                              for i in range(len(self.ids[sq]))] if consecutive else None)
 
     def run_step(self, ev=None):
         kvg, s, c = self.kvg, self.stream, self.cache.h
@@ -661,7 +706,7 @@ class StepBatched:
         for sq in range(nS):
             kvg.kvg_cache_release(c, sq, s)
         # the 128 grafts (4 stitched blocks per sequence) in one batched call
-        kvg.kvg_graft_batch(self.store.h, self.batch_bids, c, self.batch_seqs, 0, s)
+        kvg.kvg_graft_batch(self.store.h, self.batch_bids, c, self.batch_seqs, 0, s, deltas=self.batch_deltas)
         if m: m[1].record(s)
         seqs = list(range(nS))
         for t in range(self.steps):
@@ -764,32 +809,35 @@ def measure_h2d(device, nbytes=32 << 20, reps=20):
     return nbytes * reps / (e0.elapsed_time(e1) * 1e-3) / 1e9
 
 
-def run_other(args):
-    from paper_2607_14431_gb300 import build
-    build.build()
-    from paper_2607_14431_gb300 import kvg
-    torch.cuda.set_device(0)
-    device = torch.device("cuda", 0)
+def measure_other(kvg, device, config, steps, warmup, layers=0, deep_blocks=syn.DEEP_BLOCKS,
+                  consecutive=False, st=None):
+    """Builds (unless st is given) and times one of the other workloads;
+    returns its JSON line (with the set-up time and the clocks of its own
+    timed region)."""
     stream = torch.cuda.Stream(device)
     hbm_peak, sm_max, peak_kind = load_peaks()
     mk = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    if args.config == "tiny":
+    t_setup = time.perf_counter()
+    if st is not None:
+        st.stream = stream
+    elif config == "tiny":
         st = StepTiny(kvg, device, stream)
-    elif args.config == "31b":
-        st = Step31B(kvg, device, stream, args.layers)
-    elif args.config == "batched":
-        st = StepBatched(kvg, device, stream, args.layers or 4)
+    elif config == "31b":
+        st = Step31B(kvg, device, stream, layers)
+    elif config == "batched":
+        st = StepBatched(kvg, device, stream, layers or 4, consecutive=consecutive)
     else:
-        st = StepDeep(kvg, device, stream, args.deep_blocks)
+        st = StepDeep(kvg, device, stream, deep_blocks)
+    setup_s = time.perf_counter() - t_setup
     st.run_step()
     kvg.kvg_sync(st.cache.h, stream, 60.0)
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         st.run_step()
     stream.synchronize()
-    K = args.steps
+    K = steps
     n_ev = len(st.phases) + 1
     evs = [{"main": [mk() for _ in range(n_ev)]} for _ in range(K)]
-    clocks = Clocks(0)
+    clocks = Clocks(device.index or 0)
     launches0 = kvg.kvg_launch_count()
     t0, t1 = mk(), mk()
     blocks = []
@@ -816,10 +864,11 @@ def run_other(args):
             gbs = st.bytes[p] / (ms * 1e-3) / 1e9
             parts[p].update({"algorithmic_bytes": st.bytes[p], "gbs": round(gbs, 1),
                              "hbm_frac": round(gbs / hbm_peak, 3)})
-    line = {"metric": METRIC, "unit": "GB/s", "n_gpus": 1, "steps": K, "warmup": args.warmup,
+    line = {"metric": METRIC, "unit": "GB/s", "n_gpus": 1, "steps": K, "warmup": warmup,
             "ms_per_step": round(ms_step, 4), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "bf16", "data": "synthetic", "parts": parts, "gpu_launches": int(launches), "clocks": clk}
-    if args.config == "tiny":
+            "dtype": "bf16", "data": "synthetic", "parts": parts, "gpu_launches": int(launches), "clocks": clk,
+            "setup_s": round(setup_s, 1)}
+    if config == "tiny":
         line["value"] = round(step_bytes / (ms_step * 1e-3) / 1e9, 2)
         line["config"] = {"workload": "tiny: L2 Hq4/Hkv2 D64 P16, 256-token block grafted at own positions "
                                       "(digest-verified), decode 1 token over 256 rows; launch-bound"}
@@ -828,17 +877,19 @@ def run_other(args):
         st.run_step()
         stream.synchronize()
         line["checks"] = {"deterministic": _sha_tensor(st.out) == first}
-    elif args.config == "31b":
+    elif config == "31b":
         line["value"] = round(step_bytes / (ms_step * 1e-3) / 1e9, 2)
         line["config"] = {"workload": f"31b-relocation: L{st.w.n_layers} Hq32/Hkv16 D128 P64 theta 1e6, 16384-token "
                                       "block re-based by delta (0,1,4096,100000 across 8 sequences; 4096 timed), "
                                       "decode batch 8 over 65536-token contexts"}
         line["parts"]["decode"]["tokens_per_s"] = round(st.B * 1e3 / statistics.mean(phase_ms["decode"]), 1)
         line["roofline"] = _part_roofline(line["parts"], "decode", "decode_kernel", hbm_peak, peak_kind)
-    elif args.config == "batched":
+    elif config == "batched":
         line["value"] = round(step_bytes / (ms_step * 1e-3) / 1e9, 2)
         line["config"] = {"workload": f"batched-library: L{st.w.n_layers} slice of 12b, 32 seqs x 4 blocks "
-                                      "U{2048..6144} from a 512-block HBM store, then 64 decode steps (batch 32)"}
+                                      "U{2048..6144} from a 512-block HBM store, then 64 decode steps (batch 32)"
+                                      + (" [blocks 2-4 re-based to consecutive positions]" if st.consecutive
+                                         else "")}
         line["parts"]["decode_steps"]["tokens_per_s"] = round(
             syn.BATCHED_SEQS * st.steps * 1e3 / statistics.mean(phase_ms["decode_steps"]), 1)
         line["roofline"] = _part_roofline(line["parts"], "decode_steps", "decode_kernel", hbm_peak, peak_kind)
@@ -872,7 +923,76 @@ def run_other(args):
             stream.synchronize()
             errs.append(st.needle_error(b))
         line["checks"] = {"needle_max_abs_err": max(errs), "needles_checked": len(errs)}
+    line["_step"] = st
+    return line
+
+
+def run_other(args):
+    from paper_2607_14431_gb300 import build
+    build.build()
+    from paper_2607_14431_gb300 import kvg
+    torch.cuda.set_device(0)
+    line = measure_other(kvg, torch.device("cuda", 0), args.config, args.steps, args.warmup, args.layers,
+                         args.deep_blocks, args.consecutive)
+    line.pop("_step")
     print(json.dumps(line), flush=True)
+
+
+def _close_step(st):
+    for name in ("cache", "store", "hstore"):
+        o = getattr(st, name, None)
+        if o is not None:
+            o.close()
+    torch.cuda.synchronize()
+
+
+def _compact(line, keep_parts):
+    """The figures of a workload line that the default line carries."""
+    out = {"workload": line["config"]["workload"], "value": line["value"], "unit": line["unit"],
+           "ms_per_step": line["ms_per_step"], "steps": line["steps"], "warmup": line["warmup"],
+           "setup_s": line["setup_s"], "clocks": line["clocks"],
+           "parts": {p: line["parts"][p] for p in keep_parts if p in line["parts"]}}
+    for k in ("roofline", "latency_ms", "checks"):
+        if k in line:
+            out[k] = line[k]
+    return out
+
+
+def run_workloads(args):
+    """The other four workloads, each built, timed (with its own clock
+    record) and freed in turn, for the default line's `workloads` object.
+    The 31B workload runs at its full 60 layers, the batched library at its
+    4-layer slice (own positions, then re-based to consecutive positions),
+    the deep store with its full 1,394 blocks and 1,000 random grafts."""
+    from paper_2607_14431_gb300 import kvg
+    device = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
+    out = {}
+    t_all = time.perf_counter()
+    plan = [("tiny", dict(steps=20, warmup=5), ("graft_verify", "decode")),
+            ("31b", dict(steps=5, warmup=3, layers=args.workload_31b_layers), ("relocate", "decode")),
+            ("batched", dict(steps=3, warmup=3), ("graft", "decode_steps")),
+            ("deep", dict(steps=syn.DEEP_GRAFTS, warmup=5), ("host_graft", "decode"))]
+    for name, kw, keep in plan:
+        try:
+            line = measure_other(kvg, device, name, kw["steps"], kw["warmup"], kw.get("layers", 0))
+            st = line.pop("_step")
+            out[name] = _compact(line, keep)
+            if name == "batched":
+                # the same store and sequences, blocks 2-4 re-based by the
+                # tokens before them (per-graft deltas in the one batched call)
+                st.set_consecutive(True)
+                line = measure_other(kvg, device, name, kw["steps"], kw["warmup"], st=st)
+                line.pop("_step")
+                line["setup_s"] = 0.0
+                out["batched_consecutive"] = _compact(line, keep)
+            _close_step(st)
+            del st, line
+        except Exception as e:  # reported in the line, never hidden
+            out[name] = {"error": f"{type(e).__name__}: {e}"[:300]}
+        gc.collect()
+        torch.cuda.empty_cache()
+    out["total_s"] = round(time.perf_counter() - t_all, 1)
+    return out
 
 
 def _part_roofline(parts, part, kernel, hbm_peak, peak_kind):
@@ -1099,7 +1219,13 @@ def main():
     ap.add_argument("--store", default="hbm", choices=["hbm", "pool"],
                     help="12b: block in an HBM store (copying graft) or in the cache pool (zero-copy graft)")
     ap.add_argument("--deep-blocks", type=int, default=syn.DEEP_BLOCKS)
+    ap.add_argument("--consecutive", action="store_true",
+                    help="batched: re-base blocks 2-4 of each sequence so its position tags are consecutive")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="12b: leave out the other four workloads (tiny, 31b, batched, deep) from the line")
+    ap.add_argument("--workload-31b-layers", type=int, default=0,
+                    help="layers of the 31b workload in the default line (0: all 60)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -1122,6 +1248,11 @@ def main():
         torch.distributed.init_process_group("nccl")
     line = run_kvg(args, rank, world)
     if rank == 0:
+        default_step = not (args.swa or args.kv != "bf16" or args.store != "hbm" or args.layers)
+        if world == 1 and default_step and not args.no_workloads:
+            gc.collect()
+            torch.cuda.empty_cache()
+            line["workloads"] = run_workloads(args)
         if not args.no_cpu_baseline and not args.swa and args.kv == "bf16":
             line["cpu_baseline"] = cpu_baseline(args.cpu_baseline_layers)
         print(json.dumps(line), flush=True)

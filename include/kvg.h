@@ -366,22 +366,32 @@ kvg_status kvg_graft_chunked(kvg_store *store, uint64_t block_id, kvg_cache *cac
                              kvg_graft_report *report, void *const *events, int32_t max_events,
                              int32_t *chunk_end_slot, int32_t *n_chunks);
 
-/* A batch of own-position grafts (Sec. 3.2) in one call: graft i installs
- * block block_ids[i] into sequence seq_ids[i] at that sequence's next page
- * boundary, in order, exactly as n kvg_graft(delta = 0) calls would (a
- * sequence may appear several times: its blocks land one after another,
- * each page-aligned).  The page copies of all grafts run as one launch, so
- * the GPU stays full across graft boundaries.  block_ids, seq_ids: host
- * arrays of n (1 <= n <= 4096); each block at most 1,024 pages per (layer,
- * K/V).  Every argument, capacity and page count is checked first: on an
- * error nothing is grafted.  Not for pool-resident stores (KVG_ERR_ARG; use
- * kvg_graft).  flags as for kvg_graft: KVG_GRAFT_VERIFY hashes each graft's
- * restored pages after the copies; the report's seq is the (last) failing
- * graft's sequence and mismatch_pages its block page indices.  The call
- * stages its job table in library-owned pinned memory and waits for the
- * previous batch's table copy on this cache before reusing it. */
+/* A batch of grafts in one call: graft i installs block block_ids[i] into
+ * sequence seq_ids[i] at that sequence's next page boundary, in order,
+ * exactly as n kvg_graft calls with delta = deltas[i] would (a sequence may
+ * appear several times: its blocks land one after another, each
+ * page-aligned).  deltas: host array of n, or NULL for own-position grafts
+ * throughout (Sec. 3.2).  A nonzero delta re-bases that graft (Sec. 4.2):
+ * position tags + delta, keys rotated with the same fp32 cos/sin and the
+ * same operation order as kvg_graft, so the restored bytes equal those of a
+ * kvg_graft with that delta.  With deltas equal to the tokens already in the
+ * sequence, a sequence's blocks get consecutive position tags (the
+ * sequential composition of Sec. 4.8 at the KV level).  The page copies of
+ * all grafts run as one launch, so the GPU stays full across graft
+ * boundaries.  block_ids, seq_ids: host arrays of n (1 <= n <= 4096); each
+ * block at most 1,024 pages per (layer, K/V).  Every argument, capacity,
+ * page count and position range is checked first: on an error nothing is
+ * grafted (KVG_ERR_POSITION when tags + delta leave [0, 2^31), KVG_ERR_ARG
+ * for a nonzero delta on an fp8 cache).  Not for pool-resident stores
+ * (KVG_ERR_ARG; use kvg_graft).  flags as for kvg_graft: KVG_GRAFT_VERIFY
+ * hashes each own-position graft's restored pages, and each re-based
+ * graft's stored pages, after the copies; the report's seq is the (last)
+ * failing graft's sequence and mismatch_pages its block page indices.  The
+ * call stages its job table in library-owned pinned memory and waits for
+ * the previous batch's table copy on this cache before reusing it. */
 kvg_status kvg_graft_batch(kvg_store *store, const uint64_t *block_ids, kvg_cache *cache, const int32_t *seq_ids,
-                           int32_t n, uint32_t flags, void *stream, kvg_graft_report *report);
+                           const int64_t *deltas, int32_t n, uint32_t flags, void *stream,
+                           kvg_graft_report *report);
 
 /* Re-checks a grafted range: hashes the cache pages that hold slots
  * [slot0, slot0 + n_tokens(block)) of `seq` (slot0 page-aligned) on the GPU

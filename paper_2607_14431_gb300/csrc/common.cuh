@@ -93,24 +93,34 @@ struct GraftJob {
     const uint8_t *src;
     int32_t block_pages;
     int32_t pid;
+    int32_t meta;      // the graft this page belongs to
+    int32_t page;      // its page index within the block
 };
 // One graft of a batch: position tags, page-table row and fill row of its
-// destination, and its jobs [first_job, first_job + npb).
+// destination, and its jobs [first_job, first_job + npb).  A graft re-based
+// by delta != 0 has the cos/sin table trig (>= 0) of the batch's tables.
 struct GraftMeta {
     const int32_t *src_pos;
     int32_t *dst_pos;
     int32_t *table_row;
     int32_t *fill_row;
     int64_t n_tokens;
+    int64_t delta;
     int32_t npb;
     int32_t first_job;
+    int32_t trig;      // -1: own position (byte copy)
+    int32_t pad_;
 };
 struct GraftBatchParams {
     const GraftJob *jobs;
     const GraftMeta *metas;
+    // rotation tables of the re-based grafts: table t holds cos(delta w_i)
+    // for i < head_dim / 2, then sin(delta w_i), as fp32
+    const float *trig;
     int64_t n_jobs;
     int32_t n_grafts;
     int32_t n_layers, page_size, chunk_bytes;
+    int32_t n_kv_heads, head_dim;
     uint64_t page_bytes;
     int64_t pool_pages;
     uint8_t *pool;
@@ -257,7 +267,10 @@ int env_knob(const char *name, int fallback);
 cudaError_t launch_graft_copy(const GraftParams &p, int n_sm, cudaStream_t s, int max_ctas = 0,
                               DevStatus *status = nullptr);
 // Own-position copies of a batch of grafts in one launch (jobs, metas in device memory).
-cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s, int max_ctas = 0);
+// rotate: 0 when every graft of the batch is at its own position, else the
+// cache's RoPE pairing (1 half-split, 2 interleaved) for its re-based grafts.
+cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s, int max_ctas = 0,
+                               int rotate = 0);
 // Bulk append by tensor copies, for appends of at least append_tma_rows()
 // rows (16-byte aligned k/v).  Returns cudaErrorNotSupported (nothing
 // launched) when the tensor maps cannot be encoded, so the caller can take

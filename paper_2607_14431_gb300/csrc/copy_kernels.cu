@@ -65,23 +65,37 @@ __device__ __forceinline__ void rot(float a, float b, float c, float s, float &r
     rb = __fmaf_rn(a, s, __fmul_rn(b, c));
 }
 
+// cos/sin of a re-basing: from the launch's parameters (one graft per
+// launch) or from a table in global memory (a batch of grafts).
+struct ParamTrig {
+    const GraftParams &p;
+    __device__ __forceinline__ float c(int i) const { return p.cosv[i]; }
+    __device__ __forceinline__ float s(int i) const { return p.sinv[i]; }
+};
+struct TableTrig {
+    const float *cs;  // cos[half] then sin[half]
+    int half;
+    __device__ __forceinline__ float c(int i) const { return __ldg(cs + i); }
+    __device__ __forceinline__ float s(int i) const { return __ldg(cs + half + i); }
+};
+
 // Key chunk re-based by delta: rows of head_dim elements; half-split pairs
 // (i, i + D/2) live in two 16-byte vectors of the same row, interleaved pairs
 // (2i, 2i+1) inside one vector.  Rows whose token index is >= n_tokens are
 // padding and are copied unchanged.
-template <int ROT>
+template <int ROT, class Trig>
 __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const uint8_t *__restrict__ src,
-                                             int bytes, int64_t first_row_in_page,
-                                             int64_t page_token0, const GraftParams &p) {
-    const int D = p.head_dim;
+                                             int bytes, int64_t first_row_in_page, int64_t page_token0,
+                                             int head_dim, int page_size, int64_t n_tokens, const Trig &trig) {
+    const int D = head_dim;
     const int vec_per_row = D >> 3;
     const int rows = bytes / (2 * D);
     const uint4 *s4 = reinterpret_cast<const uint4 *>(src);
     uint4 *d4 = reinterpret_cast<uint4 *>(dst);
     // Rows of the page at or past n_valid are padding (only a block's last
     // page has any); the chunk's rows are (r0 + rr) mod P, rr < rows.
-    const int P = p.page_size;
-    const int64_t nv = p.n_tokens - page_token0;
+    const int P = page_size;
+    const int64_t nv = n_tokens - page_token0;
     const int n_valid = nv < P ? (int)nv : P;
     const int r0 = (int)(first_row_in_page % P);
     if (ROT == 1) {
@@ -115,7 +129,7 @@ __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const ui
                         unpack8(hi[u], b);
 #pragma unroll
                         for (int e = 0; e < 8; ++e)
-                            rot(a[e], b[e], p.cosv[c * 8 + e], p.sinv[c * 8 + e], ra[e], rb[e]);
+                            rot(a[e], b[e], trig.c(c * 8 + e), trig.s(c * 8 + e), ra[e], rb[e]);
                         __stcs(d4 + lo_i, pack8(ra));
                         __stcs(d4 + lo_i + half_vecs, pack8(rb));
                     } else {
@@ -138,7 +152,7 @@ __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const ui
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     const int i = c * 4 + e;
-                    rot(f[2 * e], f[2 * e + 1], p.cosv[i], p.sinv[i], g[2 * e], g[2 * e + 1]);
+                    rot(f[2 * e], f[2 * e + 1], trig.c(i), trig.s(i), g[2 * e], g[2 * e + 1]);
                 }
                 __stcs(d4 + it, pack8(g));
             } else {
@@ -168,7 +182,7 @@ __global__ void __launch_bounds__(kCopyThreads) graft_kernel(const GraftParams p
             copy_chunk(dst, src, p.chunk_bytes);
         } else {
             rotate_chunk<ROT>(dst, src, p.chunk_bytes, (int64_t)(off / row_bytes),
-                              (int64_t)(p.page_base + jj) * P, p);
+                              (int64_t)(p.page_base + jj) * P, p.head_dim, p.page_size, p.n_tokens, ParamTrig{p});
         }
     }
 }
@@ -704,14 +718,18 @@ int grid_for(int64_t work_items, int per_block, int n_sm, int waves) {
 
 }  // namespace
 
-// A batch of own-position grafts in one launch: every block page of every
-// graft is a job; a unit is a chunk of one (job, layer, K/V) page, so the
-// batch keeps every SM busy to its end instead of draining after each graft.
+// A batch of grafts in one launch: every block page of every graft is a job;
+// a unit is a chunk of one (job, layer, K/V) page, so the batch keeps every
+// SM busy to its end instead of draining after each graft.  ROT > 0: some
+// grafts are re-based (their key chunks rotate with their own cos/sin table,
+// as the single-graft kernels do; values and own-position grafts copy).
+template <int ROT>
 __global__ void __launch_bounds__(kCopyThreads) graft_batch_kernel(const GraftBatchParams p) {
     const uint64_t page_bytes = p.page_bytes;
     const int64_t cpp = (int64_t)(page_bytes / (uint64_t)p.chunk_bytes);
     const int64_t per_job = (int64_t)p.n_layers * 2 * cpp;
     const int64_t n_units = p.n_jobs * per_job;
+    const int row_bytes = 2 * p.head_dim;
     for (int64_t unit = blockIdx.x; unit < n_units; unit += gridDim.x) {
         const int64_t jb = unit / per_job;
         const int64_t rem = unit - jb * per_job;
@@ -720,7 +738,15 @@ __global__ void __launch_bounds__(kCopyThreads) graft_batch_kernel(const GraftBa
         const GraftJob job = p.jobs[jb];
         const uint8_t *src = job.src + (uint64_t)lkv * job.block_pages * page_bytes + off;
         uint8_t *dst = p.pool + ((uint64_t)lkv * p.pool_pages + (uint64_t)job.pid) * page_bytes + off;
-        copy_chunk(dst, src, p.chunk_bytes);
+        const int32_t trig = ROT != 0 && !(lkv & 1) ? p.metas[job.meta].trig : -1;
+        if (trig < 0) {
+            copy_chunk(dst, src, p.chunk_bytes);
+        } else {
+            const int half = p.head_dim >> 1;
+            rotate_chunk<ROT>(dst, src, p.chunk_bytes, (int64_t)(off / row_bytes), (int64_t)job.page * p.page_size,
+                              p.head_dim, p.page_size, p.metas[job.meta].n_tokens,
+                              TableTrig{p.trig + (int64_t)trig * 2 * half, half});
+        }
     }
     // metadata last: the copies start at once and this fills the tail wave
     const int64_t P = p.page_size;
@@ -728,7 +754,7 @@ __global__ void __launch_bounds__(kCopyThreads) graft_batch_kernel(const GraftBa
     const int64_t gsz = (int64_t)gridDim.x * blockDim.x;
     for (int32_t g = 0; g < p.n_grafts; ++g) {
         const GraftMeta m = p.metas[g];
-        for (int64_t t = gtid; t < m.n_tokens; t += gsz) m.dst_pos[t] = m.src_pos[t];
+        for (int64_t t = gtid; t < m.n_tokens; t += gsz) m.dst_pos[t] = (int32_t)((int64_t)m.src_pos[t] + m.delta);
         for (int64_t j = gtid; j < m.npb; j += gsz) {
             m.table_row[j] = p.jobs[m.first_job + j].pid;
             const int64_t f = m.n_tokens - j * P;
@@ -737,11 +763,16 @@ __global__ void __launch_bounds__(kCopyThreads) graft_batch_kernel(const GraftBa
     }
 }
 
-cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s, int max_ctas) {
+cudaError_t launch_graft_batch(const GraftBatchParams &p, int n_sm, cudaStream_t s, int max_ctas, int rotate) {
     const int64_t units = p.n_jobs * p.n_layers * 2 * (int64_t)(p.page_bytes / p.chunk_bytes);
     int grid = grid_for(units, 1, n_sm, 4);
     if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
-    graft_batch_kernel<<<grid, kCopyThreads, 0, s>>>(p);
+    if (rotate == 0)
+        graft_batch_kernel<0><<<grid, kCopyThreads, 0, s>>>(p);
+    else if (rotate == 1)
+        graft_batch_kernel<1><<<grid, kCopyThreads, 0, s>>>(p);
+    else
+        graft_batch_kernel<2><<<grid, kCopyThreads, 0, s>>>(p);
     count_launches(1);
     return cudaGetLastError();
 }

@@ -1497,6 +1497,20 @@ static int host_copy_grid_cap() {
     return cap;
 }
 
+// cos and sin of delta * w_i, w_i = theta^(-2i/D), i < D/2 (Sec. 4.2's
+// re-basing of a block by delta positions): fp64 on the host, rounded to the
+// fp32 the kernels rotate with.  One function for every graft path, so a
+// re-based block gets the same bytes whichever entry point grafts it.
+static void rope_table(const kvg_dims &d, int64_t delta, float *cosv, float *sinv) {
+    const int half = d.head_dim / 2;
+    for (int i = 0; i < half; ++i) {
+        const double w = std::pow(d.rope_theta, -2.0 * i / d.head_dim);
+        const double a = (double)delta * w;
+        cosv[i] = (float)std::cos(a);
+        sinv[i] = (float)std::sin(a);
+    }
+}
+
 static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t dst_slot,
                              int64_t delta, uint32_t flags, void *stream, kvg_graft_report *report,
                              const ChunkEvents &ce) {
@@ -1542,15 +1556,8 @@ static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int3
     p.delta = delta;
     p.rotate = 0;
     if (delta != 0) {
-        const kvg_dims &sd = s->dims;
-        p.rotate = sd.rope_style == KVG_ROPE_HALF ? 1 : 2;
-        const int half = sd.head_dim / 2;
-        for (int i = 0; i < half; ++i) {
-            const double w = std::pow(sd.rope_theta, -2.0 * i / sd.head_dim);
-            const double a = (double)delta * w;
-            p.cosv[i] = (float)std::cos(a);
-            p.sinv[i] = (float)std::sin(a);
-        }
+        p.rotate = s->dims.rope_style == KVG_ROPE_HALF ? 1 : 2;
+        rope_table(s->dims, delta, p.cosv, p.sinv);
     }
     const int32_t *bpos = reinterpret_cast<const int32_t *>(blk.dev + blk.lay.pos_off);
     // A verified own-position graft from an HBM store reads each page once:
@@ -1680,7 +1687,8 @@ extern "C" kvg_status kvg_graft_chunked(kvg_store *s, uint64_t block_id, kvg_cac
 }
 
 extern "C" kvg_status kvg_graft_batch(kvg_store *s, const uint64_t *block_ids, kvg_cache *c, const int32_t *seq_ids,
-                                      int32_t n, uint32_t flags, void *stream, kvg_graft_report *report) {
+                                      const int64_t *deltas, int32_t n, uint32_t flags, void *stream,
+                                      kvg_graft_report *report) {
     Trace trace_("kvg_graft_batch");
     if (!s || !c || !block_ids || !seq_ids) return fail(KVG_ERR_ARG, "null argument");
     if (n <= 0 || n > kMaxGraftsPerBatch) return fail(KVG_ERR_ARG, "n must be in [1, %d]", kMaxGraftsPerBatch);
@@ -1702,15 +1710,32 @@ extern "C" kvg_status kvg_graft_batch(kvg_store *s, const uint64_t *block_ids, k
         const int64_t dst = (it->second + P - 1) / P * P;
         if (dst + blk.lay.n_tokens > c->max_slots) return fail(KVG_ERR_CAPACITY, "graft %d past max_slots", i);
         if (blk.lay.n_pages > kMaxPagesPerLaunch) return fail(KVG_ERR_ARG, "graft %d: block too long for a batch", i);
+        const int64_t delta = deltas ? deltas[i] : 0;
+        if (blk.min_pos + delta < 0 || blk.max_pos + delta >= (1ll << 31))
+            return fail(KVG_ERR_POSITION, "graft %d: position tags + delta leave [0, 2^31)", i);
+        if (delta != 0 && c->dims.kv_dtype != KVG_KV_BF16)
+            return fail(KVG_ERR_ARG, "graft %d: relocation needs a bf16 cache", i);
         it->second = dst + blk.lay.n_tokens;
         pages += blk.lay.n_pages;
     }
     if (pages > (int64_t)c->free_list.size()) return fail(KVG_ERR_CAPACITY, "out of free pages");
     DeviceGuard g(c->device);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    // the job table: metas then jobs, in pinned host memory
+    // one cos/sin table per distinct nonzero delta, in order of first use
+    std::vector<int64_t> table_delta;
+    std::vector<int32_t> trig_of(n, -1);
+    for (int32_t i = 0; i < n; ++i) {
+        const int64_t delta = deltas ? deltas[i] : 0;
+        if (delta == 0) continue;
+        auto f = std::find(table_delta.begin(), table_delta.end(), delta);
+        trig_of[i] = (int32_t)(f - table_delta.begin());
+        if (f == table_delta.end()) table_delta.push_back(delta);
+    }
+    const int half = c->dims.head_dim / 2;
+    // the job table: metas, jobs, then the cos/sin tables, in pinned host memory
     const size_t meta_bytes = (size_t)n * sizeof(GraftMeta);
-    const size_t bytes = meta_bytes + (size_t)pages * sizeof(GraftJob);
+    const size_t trig_off = (meta_bytes + (size_t)pages * sizeof(GraftJob) + 15) / 16 * 16;
+    const size_t bytes = trig_off + table_delta.size() * 2 * half * sizeof(float);
     if (!c->batch_ev) KVG_CUDA(cudaEventCreateWithFlags(&c->batch_ev, cudaEventDisableTiming));
     KVG_CUDA(cudaEventSynchronize(c->batch_ev));  // the previous batch's copy has read the staging
     if (bytes > c->batch_host_cap) {
@@ -1743,30 +1768,44 @@ extern "C" kvg_status kvg_graft_batch(kvg_store *s, const uint64_t *block_ids, k
         m.table_row = c->page_table + (int64_t)seq * c->max_pages + jdst;
         m.fill_row = c->page_fill + (int64_t)seq * c->max_pages + jdst;
         m.n_tokens = nt;
+        m.delta = deltas ? deltas[i] : 0;
         m.npb = (int32_t)npb;
         m.first_job = job;
+        m.trig = trig_of[i];
+        m.pad_ = 0;
         for (int64_t j = 0; j < npb; ++j, ++job)
-            jobs[job] = GraftJob{blk.dev + blk.lay.pages_off + (uint64_t)j * c->page_bytes, (int32_t)npb, pids[j]};
+            jobs[job] = GraftJob{blk.dev + blk.lay.pages_off + (uint64_t)j * c->page_bytes, (int32_t)npb, pids[j], i,
+                                 (int32_t)j};
         verify_at.push_back({seq, jdst});
     }
+    float *trig = reinterpret_cast<float *>(c->batch_host + trig_off);
+    for (size_t t = 0; t < table_delta.size(); ++t)
+        rope_table(c->dims, table_delta[t], trig + t * 2 * half, trig + t * 2 * half + half);
     KVG_CUDA(cudaMemcpyAsync(c->batch_dev.ptr, c->batch_host, bytes, cudaMemcpyHostToDevice, st));
     KVG_CUDA(cudaEventRecord(c->batch_ev, st));
     GraftBatchParams p{};
     p.metas = static_cast<const GraftMeta *>(c->batch_dev.ptr);
     p.jobs = reinterpret_cast<const GraftJob *>(static_cast<uint8_t *>(c->batch_dev.ptr) + meta_bytes);
+    p.trig = reinterpret_cast<const float *>(static_cast<uint8_t *>(c->batch_dev.ptr) + trig_off);
     p.n_jobs = pages;
     p.n_grafts = n;
     p.n_layers = c->dims.n_layers;
     p.page_size = (int32_t)P;
     p.chunk_bytes = copy_chunk_bytes(c->dims);
+    p.n_kv_heads = c->dims.n_kv_heads;
+    p.head_dim = c->dims.head_dim;
     p.page_bytes = c->page_bytes;
     p.pool_pages = c->n_pages;
     p.pool = c->pool;
-    KVG_CUDA(launch_graft_batch(p, c->n_sm, st, s->residency == KVG_RESIDENCY_PINNED_HOST ? host_copy_grid_cap() : 0));
+    const int rotate = table_delta.empty() ? 0 : c->dims.rope_style == KVG_ROPE_HALF ? 1 : 2;
+    KVG_CUDA(launch_graft_batch(p, c->n_sm, st, s->residency == KVG_RESIDENCY_PINNED_HOST ? host_copy_grid_cap() : 0,
+                                rotate));
+    // verification: own-position grafts hash their restored pages; re-based
+    // ones hash the stored pages (their key pages differ by design)
     if (flags & KVG_GRAFT_VERIFY)
         for (int32_t i = 0; i < n; ++i) {
             kvg_status r = enqueue_verify(s, s->blocks[block_ids[i]], c, verify_at[i].first, verify_at[i].second,
-                                          false, st);
+                                          trig_of[i] >= 0, st);
             if (r != KVG_OK) return r;
         }
     return finish_verify(c, n == 1 ? seq_ids[0] : -1, flags,

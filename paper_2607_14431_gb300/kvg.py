@@ -80,7 +80,7 @@ _SIGNATURES = {
     "kvg_cache_destroy": ([_vp], None),
     "kvg_cache_set_free_order": ([_vp, _vp, _i32], _i32),
     "kvg_cache_set_layer_windows": ([_vp, _vp, _i32], _i32),
-    "kvg_graft_batch": ([_vp, _vp, _vp, _vp, _i32, _u32, _vp, _vp], _i32),
+    "kvg_graft_batch": ([_vp, _vp, _vp, _vp, _vp, _i32, _u32, _vp, _vp], _i32),
     "kvg_cache_view_get": ([_vp, _P(kvg_cache_view)], _i32),
     "kvg_cache_seq_info": ([_vp, _i32, _P(_i32), _P(_i32)], _i32),
     "kvg_cache_append": ([_vp, _i32, _vp, _vp, _vp, _i32, _vp], _i32),
@@ -274,13 +274,15 @@ def kvg_graft_chunked(store, block_id: int, cache, seq: int, events, dst_slot: i
 
 
 def kvg_graft_batch(store, block_ids, cache, seq_ids, flags: int = 0, stream=None,
-                    report: kvg_graft_report | None = None):
+                    report: kvg_graft_report | None = None, deltas=None):
+    """deltas: None (every graft at its own position) or one int per graft."""
     n = len(block_ids)
-    if len(seq_ids) != n:
-        raise ValueError("block_ids and seq_ids differ in length")
+    if len(seq_ids) != n or (deltas is not None and len(deltas) != n):
+        raise ValueError("block_ids, seq_ids and deltas differ in length")
     ids = (ctypes.c_uint64 * max(n, 1))(*[int(b) for b in block_ids])
     seqs = (ctypes.c_int32 * max(n, 1))(*[int(x) for x in seq_ids])
-    _check(lib().kvg_graft_batch(store, ids, cache, seqs, n, flags, _stream(stream),
+    ds = None if deltas is None else (ctypes.c_int64 * max(n, 1))(*[int(d) for d in deltas])
+    _check(lib().kvg_graft_batch(store, ids, cache, seqs, ds, n, flags, _stream(stream),
                                  ctypes.byref(report) if report is not None else None))
 
 

@@ -223,12 +223,16 @@ def test_31b_relocation_full_size(oracle):
         _close(st.cache, st.store)
 
 
-def test_batched_library_full_size(oracle):
+@pytest.mark.parametrize("consecutive", [False, True])
+def test_batched_library_full_size(oracle, consecutive):
+    """The batched library at its 4-layer slice; consecutive: blocks 2-4 of
+    every sequence re-based by the tokens before them (per-graft deltas in
+    the one batched call)."""
     kvg = need_gpu()
     import bench
     dev = torch.device("cuda", 0)
     s = torch.cuda.Stream()
-    st = bench.StepBatched(kvg, dev, s, 4)
+    st = bench.StepBatched(kvg, dev, s, 4, consecutive=consecutive)
     try:
         st.run_step()
         s.synchronize()
@@ -240,10 +244,15 @@ def test_batched_library_full_size(oracle):
         for n in st.lens:
             meta.append(nS, None, None, syn.positions(0, int(n)))
             meta.release(nS)
+        delta_of = {}
         for sq in range(nS):
             meta.release(sq)
+            run = 0
             for b in st.ids[sq]:
-                meta.graft(sq, oracle.BlockMeta(od, syn.positions(0, int(st.lens[b]))))
+                d = run if consecutive else 0
+                delta_of[(sq, int(b))] = d
+                meta.graft(sq, oracle.BlockMeta(od, syn.positions(0, int(st.lens[b]))), delta=d)
+                run += int(st.lens[b])
         posn = st.pos.cpu().numpy()
         for t in range(st.steps):  # one decode-step row per sequence, in batch order
             for sq in range(nS):
@@ -258,6 +267,7 @@ def test_batched_library_full_size(oracle):
                 n = int(st.lens[b])
                 k, v = syn.kv_rows(w, n, w.seed + int(b), "cuda")
                 blk = oracle.block_from_kv(od, syn.as_u16(k), syn.as_u16(v), syn.positions(0, n))
+                d = delta_of[(sq, int(b))]
                 for j in (0, blk.n_pages - 1):
                     for kv in (0, 1):
                         got = _pool_page(st.cache, w, w.n_layers - 1, kv, pt[sq, j0 + j])
@@ -266,7 +276,11 @@ def test_batched_library_full_size(oracle):
                             # the tail page's fill rows are the block's; later rows
                             # belong to the decode appends of the last block only
                             got, want = got[:, :n % P], want[:, :n % P]
-                        assert np.array_equal(got, want)
+                        if kv == 0 and d:
+                            ref = oracle.rope_rotate_rows(want, d, w.rope_theta, 0)
+                            assert np.abs(oracle.bf16_to_f64(got) - ref).max() <= 2e-2
+                        else:
+                            assert np.array_equal(got, want)
                 j0 += blk.n_pages
         # decode after the last step: every query head of two layers of three
         # sequences against fp64 attention, through the decode gate
@@ -275,12 +289,15 @@ def test_batched_library_full_size(oracle):
                 ks, vs = [], []
                 for b in st.ids[sq]:
                     k, v = syn.kv_rows(w, int(st.lens[b]), w.seed + int(b), "cuda")
-                    ks.append(syn.as_u16(k[l]))
+                    kl = syn.as_u16(k[l])
+                    d = delta_of[(sq, int(b))]
+                    ks.append(oracle.rope_rotate_rows_bf16(kl, d, w.rope_theta, 0) if d else kl)
                     vs.append(syn.as_u16(v[l]))
                 ks.append(syn.as_u16(st.kd[l, sq::nS]))
                 vs.append(syn.as_u16(st.vd[l, sq::nS]))
                 ref = oracle.gqa_decode(syn.as_u16(st.q[l, sq]), np.concatenate(ks), np.concatenate(vs), st.scale)
-                compare_decode(oracle, syn.as_u16(st.out[l, sq]), ref, what=f"batched seq {sq} layer {l}")
+                compare_decode(oracle, syn.as_u16(st.out[l, sq]), ref,
+                               what=f"batched{' consecutive' if consecutive else ''} seq {sq} layer {l}")
     finally:
         _close(st.cache, st.store)
 

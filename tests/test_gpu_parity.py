@@ -568,6 +568,95 @@ def test_graft_batch_equals_sequential_grafts(oracle, geo, residency):
     kvg.kvg_sync(c.h)
 
 
+@pytest.mark.parametrize("geo,style", [("d128", 0), ("d128", 1), ("d256", 0), ("tiny", 0)])
+def test_relocate_to_consecutive_composition(oracle, geo, style):
+    """Sequential composition at the KV level (Sec. 4.8), re-basing blocks
+    (Sec. 4.2): four blocks deposited at their own positions [0, N_b) go into
+    one sequence, each at the next page boundary; block 1 at its own
+    positions, block b > 1 re-based by delta = the tokens already present, so
+    the position tags run 0 .. sum(N) - 1 without a gap.  One
+    kvg_graft_batch call with per-graft deltas and four kvg_graft calls give
+    the same pool bytes; page tables, fills and tags equal the oracle's;
+    values and padding are bit-exact, re-based keys within 2e-2 of the fp64
+    rotation; the decode over the composed sequence passes the decode gate
+    against the oracle's cache built with the same deltas; verification of
+    every graft passes (re-based ones hash their stored pages)."""
+    kvg = need_gpu()
+    w = geometry(geo)
+    P = w.page_size
+    dims = dims_for(kvg, w, style)
+    od = oracle_dims(oracle, w, style)
+    lens = [3 * P + 7, 2 * P, P - 5, 2 * P + 1]
+    src = kvg.Cache(dims, 32, 1, 8 * P)
+    store = kvg.Store(dims, 0, HBM_CAP)
+    bids, oblks, rows = [], [], []
+    for i, n in enumerate(lens):
+        k, v = _kv(w, n, 310 + i)
+        append(kvg, src, 0, k, v, syn.positions(0, n))
+        bids.append(kvg.kvg_deposit(store.h, src.h, 0, 0, n))
+        kvg.kvg_cache_release(src.h, 0)
+        oblks.append(oracle.block_from_kv(od, k, v, syn.positions(0, n)))
+        rows.append((k, v))
+    deltas = [int(sum(lens[:i])) for i in range(len(lens))]
+    n_pages, max_slots = 48, 16 * P
+    caches = []
+    for _ in range(2):
+        c = kvg.Cache(dims, n_pages, 2, max_slots)
+        fill_canary(c)
+        kvg.kvg_cache_set_free_order(c.h, syn.permutation(n_pages, 320))
+        caches.append(c)
+    flags = kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC
+    rep = kvg.kvg_graft_report()
+    kvg.kvg_graft_batch(store.h, bids, caches[0].h, [1] * 4, flags, report=rep, deltas=deltas)
+    assert rep.n_mismatch == 0 and rep.n_pages_checked == w.n_layers * 2 * sum(b.n_pages for b in oblks)
+    for b, d in zip(bids, deltas):
+        kvg.kvg_graft(store.h, b, caches[1].h, 1, -1, d, flags)
+    pool = pool_u16(caches[0], w)
+    assert np.array_equal(pool, pool_u16(caches[1], w))
+    oc = oracle.OracleCache(od, n_pages, 2, max_slots, fill=CANARY)
+    oc.set_free_order(syn.permutation(n_pages, 320))
+    for blk, d in zip(oblks, deltas):
+        oc.graft(1, blk, delta=d)
+    pt, pf, ps = tables(caches[0])
+    assert np.array_equal(pt, oc.page_table) and np.array_equal(pf, oc.page_fill)
+    assert np.array_equal(ps, oc.positions)
+    # the position tags of the valid rows run 0 .. sum(N) - 1
+    valid = np.concatenate([np.arange(j * P, j * P + pf[1, j]) for j in range(int((pt[1] >= 0).sum()))])
+    assert np.array_equal(ps[1, valid], np.arange(sum(lens)))
+    # values, padding rows and untouched pages bit-exact; re-based keys
+    # within 2e-2 of the fp64 rotation
+    assert np.array_equal(pool[:, 1], oc.pool[:, 1])
+    j0 = 0
+    mask = np.ones(pool[:, 0].shape, bool)
+    for (k, _), n, d in zip(rows, lens, deltas):
+        kg = np.stack([np.stack([pool[l, 0, pt[1, j0 + t // P], :, t % P] for t in range(n)]) for l in range(w.n_layers)])
+        if d == 0:
+            assert np.array_equal(kg, k)
+        else:
+            k64 = np.stack([oracle.rope_rotate_rows(k[l], d, w.rope_theta, style) for l in range(w.n_layers)])
+            assert np.abs(oracle.bf16_to_f64(kg) - k64).max() <= 2e-2
+        for t in range(n):
+            mask[:, pt[1, j0 + t // P], :, t % P] = False
+        j0 += -(-n // P)
+    assert np.array_equal(pool[:, 0][mask], oc.pool[:, 0][mask])
+    # decode over the composed sequence against the oracle's cache
+    q = syn.as_u16(syn.queries(w, w.n_layers, 1, 330))
+    scale = 1 / math.sqrt(w.head_dim)
+    o = decode(kvg, caches[0], w, [1], q)
+    assert np.array_equal(o, decode(kvg, caches[1], w, [1], q))
+    for l in range(w.n_layers):
+        compare_decode(oracle, o[l, 0], oc.decode(1, l, q[l, 0], scale), what=f"consecutive {geo} layer {l}")
+    # a delta that pushes a tag out of [0, 2^31): refused whole
+    before = pool_u16(caches[0], w).copy()
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_graft_batch(store.h, bids[:2], caches[0].h, [0, 0], deltas=[0, 2 ** 31 - lens[1] + 1])
+    assert e.value.status == kvg.KVG_ERR_POSITION
+    assert np.array_equal(pool_u16(caches[0], w), before)
+    assert kvg.kvg_cache_seq_info(caches[0].h, 0)[0] == 0
+    for c in caches:
+        kvg.kvg_sync(c.h)
+
+
 def test_corrupt_page_table_entries_are_reported_not_followed(oracle):
     """A page id outside the pool written into the device page table (through
     the exported view) is never dereferenced: decode records
