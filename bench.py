@@ -104,6 +104,11 @@ class Clocks:
                  "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
+            # the sampler must be live before the region it records starts
+            t_end = time.perf_counter() + 3.0
+            while not self.samples and time.perf_counter() < t_end and self.proc.poll() is None:
+                time.sleep(0.005)
+            self.n_before = len(self.samples)
         except Exception:
             self.proc = None
 
@@ -120,10 +125,13 @@ class Clocks:
         except Exception:
             self.proc.kill()
         self.t.join(timeout=2)
-        sm = [float(s[0]) for s in self.samples if len(s) >= 7 and s[0].replace(".", "").isdigit()]
-        mx = [float(s[1]) for s in self.samples if len(s) >= 7 and s[1].replace(".", "").isdigit()]
+        # the samples taken during the region (the one that proved the
+        # sampler live came before it)
+        rows = self.samples[self.n_before:] or self.samples[-1:]
+        sm = [float(s[0]) for s in rows if len(s) >= 7 and s[0].replace(".", "").isdigit()]
+        mx = [float(s[1]) for s in rows if len(s) >= 7 and s[1].replace(".", "").isdigit()]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for s in self.samples if len(s) >= 7 for i in range(4)
+        reasons = sorted({names[i] for s in rows if len(s) >= 7 for i in range(4)
                           if s[3 + i].lower() == "active"})
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
                 "reasons": reasons, "samples": len(sm)}
@@ -367,7 +375,7 @@ def run_kvg(args, rank, world):
                 for p, (sn, i, j) in st.spans.items()}
     deterministic = _sha_tensor(st.out) == first_sha
 
-    # each graft form alone (CUDA events, median of 8 after 3 untimed): the
+    # each graft form alone (CUDA events, median of 40 after 3 untimed): the
     # plain own-position graft (HBM-bound) and the verified one (ALU-bound)
     alone = {}
     if not st.pool_store:
@@ -375,7 +383,7 @@ def run_kvg(args, rank, world):
             g0, g1 = mk(), mk()
             gts = []
             clk_g = None
-            for k in range(11):
+            for k in range(43):
                 if k == 3:
                     clk_g = Clocks(local)
                 kvg.kvg_cache_release(st.cache.h, 0, stream)
@@ -968,7 +976,7 @@ def run_workloads(args):
     device = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
     out = {}
     t_all = time.perf_counter()
-    plan = [("tiny", dict(steps=20, warmup=5), ("graft_verify", "decode")),
+    plan = [("tiny", dict(steps=500, warmup=5), ("graft_verify", "decode")),
             ("31b", dict(steps=5, warmup=3, layers=args.workload_31b_layers), ("relocate", "decode")),
             ("batched", dict(steps=3, warmup=3), ("graft", "decode_steps")),
             ("deep", dict(steps=syn.DEEP_GRAFTS, warmup=5), ("host_graft", "decode"))]

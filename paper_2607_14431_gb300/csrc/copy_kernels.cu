@@ -67,16 +67,33 @@ __device__ __forceinline__ void rot(float a, float b, float c, float s, float &r
 
 // cos/sin of a re-basing: from the launch's parameters (one graft per
 // launch) or from a table in global memory (a batch of grafts).
+// load<N>(i0, c, s) gives cos and sin of pairs i0 .. i0 + N - 1 (N = 4 or 8,
+// i0 a multiple of N).
 struct ParamTrig {
     const GraftParams &p;
-    __device__ __forceinline__ float c(int i) const { return p.cosv[i]; }
-    __device__ __forceinline__ float s(int i) const { return p.sinv[i]; }
+    template <int N>
+    __device__ __forceinline__ void load(int i0, float *c, float *s) const {
+#pragma unroll
+        for (int e = 0; e < N; ++e) {
+            c[e] = p.cosv[i0 + e];
+            s[e] = p.sinv[i0 + e];
+        }
+    }
 };
 struct TableTrig {
-    const float *cs;  // cos[half] then sin[half]
+    const float *cs;  // cos[half] then sin[half], 16-byte aligned, half a multiple of 4
     int half;
-    __device__ __forceinline__ float c(int i) const { return __ldg(cs + i); }
-    __device__ __forceinline__ float s(int i) const { return __ldg(cs + half + i); }
+    template <int N>
+    __device__ __forceinline__ void load(int i0, float *c, float *s) const {
+        const float4 *c4 = reinterpret_cast<const float4 *>(cs + i0);
+        const float4 *s4 = reinterpret_cast<const float4 *>(cs + half + i0);
+#pragma unroll
+        for (int q = 0; q < N / 4; ++q) {
+            const float4 x = __ldg(c4 + q), y = __ldg(s4 + q);
+            c[4 * q] = x.x, c[4 * q + 1] = x.y, c[4 * q + 2] = x.z, c[4 * q + 3] = x.w;
+            s[4 * q] = y.x, s[4 * q + 1] = y.y, s[4 * q + 2] = y.z, s[4 * q + 3] = y.w;
+        }
+    }
 };
 
 // Key chunk re-based by delta: rows of head_dim elements; half-split pairs
@@ -124,12 +141,12 @@ __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const ui
                     const int c = it & (half_vecs - 1);
                     const int lo_i = rr * vec_per_row + c;
                     if (n_valid == P || (r0 + rr) % P < n_valid) {
-                        float a[8], b[8], ra[8], rb[8];
+                        float a[8], b[8], ra[8], rb[8], cv[8], sv[8];
                         unpack8(lo[u], a);
                         unpack8(hi[u], b);
+                        trig.template load<8>(c * 8, cv, sv);
 #pragma unroll
-                        for (int e = 0; e < 8; ++e)
-                            rot(a[e], b[e], trig.c(c * 8 + e), trig.s(c * 8 + e), ra[e], rb[e]);
+                        for (int e = 0; e < 8; ++e) rot(a[e], b[e], cv[e], sv[e], ra[e], rb[e]);
                         __stcs(d4 + lo_i, pack8(ra));
                         __stcs(d4 + lo_i + half_vecs, pack8(rb));
                     } else {
@@ -147,13 +164,11 @@ __device__ __forceinline__ void rotate_chunk(uint8_t *__restrict__ dst, const ui
             const int c = it & (vec_per_row - 1);
             const uint4 x = __ldcs(s4 + it);
             if (n_valid == P || (r0 + rr) % P < n_valid) {
-                float f[8], g[8];
+                float f[8], g[8], cv[4], sv[4];
                 unpack8(x, f);
+                trig.template load<4>(c * 4, cv, sv);
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int i = c * 4 + e;
-                    rot(f[2 * e], f[2 * e + 1], trig.c(i), trig.s(i), g[2 * e], g[2 * e + 1]);
-                }
+                for (int e = 0; e < 4; ++e) rot(f[2 * e], f[2 * e + 1], cv[e], sv[e], g[2 * e], g[2 * e + 1]);
                 __stcs(d4 + it, pack8(g));
             } else {
                 __stcs(d4 + it, x);
