@@ -568,8 +568,9 @@ def test_graft_batch_equals_sequential_grafts(oracle, geo, residency):
     kvg.kvg_sync(c.h)
 
 
-@pytest.mark.parametrize("geo,style", [("d128", 0), ("d128", 1), ("d256", 0), ("tiny", 0)])
-def test_relocate_to_consecutive_composition(oracle, geo, style):
+@pytest.mark.parametrize("geo,style,residency", [("d128", 0, 0), ("d128", 1, 0), ("d256", 0, 0), ("tiny", 0, 0),
+                                                 ("d128", 0, 1)])
+def test_relocate_to_consecutive_composition(oracle, geo, style, residency):
     """Sequential composition at the KV level (Sec. 4.8), re-basing blocks
     (Sec. 4.2): four blocks deposited at their own positions [0, N_b) go into
     one sequence, each at the next page boundary; block 1 at its own
@@ -580,7 +581,8 @@ def test_relocate_to_consecutive_composition(oracle, geo, style):
     values and padding are bit-exact, re-based keys within 2e-2 of the fp64
     rotation; the decode over the composed sequence passes the decode gate
     against the oracle's cache built with the same deltas; verification of
-    every graft passes (re-based ones hash their stored pages)."""
+    every graft passes (re-based ones hash their stored pages).  From an HBM
+    store, and from a pinned-host store (read over the host link)."""
     kvg = need_gpu()
     w = geometry(geo)
     P = w.page_size
@@ -588,7 +590,7 @@ def test_relocate_to_consecutive_composition(oracle, geo, style):
     od = oracle_dims(oracle, w, style)
     lens = [3 * P + 7, 2 * P, P - 5, 2 * P + 1]
     src = kvg.Cache(dims, 32, 1, 8 * P)
-    store = kvg.Store(dims, 0, HBM_CAP)
+    store = kvg.Store(dims, residency, HBM_CAP)
     bids, oblks, rows = [], [], []
     for i, n in enumerate(lens):
         k, v = _kv(w, n, 310 + i)
