@@ -810,10 +810,12 @@ def graft_latencies(kvg, st, stream, blocks, hold_cycles=2_000_000):
     launch latency."""
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     out = []
+    hold = getattr(torch.cuda, "_sleep", None)  # a private torch helper: without it, no hold
     with torch.cuda.stream(stream):
         for b in blocks:
             kvg.kvg_cache_release(st.cache.h, 0, stream)
-            torch.cuda._sleep(hold_cycles)
+            if hold is not None:
+                hold(hold_cycles)
             e0.record(stream)
             kvg.kvg_graft(st.store.h, int(b), st.cache.h, 0, -1, 0, 0, stream)
             e1.record(stream)

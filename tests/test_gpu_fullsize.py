@@ -260,6 +260,19 @@ def test_batched_library_full_size(oracle, consecutive):
         pt, pf, ps = tables(st.cache)
         assert np.array_equal(pt, meta.page_table) and np.array_equal(pf, meta.page_fill)
         assert np.array_equal(ps, meta.positions)
+        if not consecutive:
+            # every page of all 128 grafts: the batch again, digest-verified
+            # (each restored page's SHA-256 against the block's stored digest)
+            # before any decode-step row lands in a ragged tail page
+            for sq in range(nS):
+                kvg.kvg_cache_release(st.cache.h, sq, s)
+            rep = kvg.kvg_graft_report()
+            kvg.kvg_graft_batch(st.store.h, st.batch_bids, st.cache.h, st.batch_seqs,
+                                kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, s, report=rep)
+            n_blk_pages = sum(-(-int(st.lens[b]) // P) for sq in range(nS) for b in st.ids[sq])
+            assert rep.n_mismatch == 0 and rep.n_pages_checked == w.n_layers * 2 * n_blk_pages
+            st.run_step()  # back to the state after a full step
+            s.synchronize()
         # grafted pages equal the deposited blocks' pages (sampled), incl. ragged tail pages
         for sq in (0, 13, nS - 1):
             j0 = 0
@@ -316,12 +329,16 @@ def test_deep_store_needles_full_size(oracle):
             k, v = st.block_rows(b, dev)
             blk = oracle.block_from_kv(od, syn.as_u16(k), syn.as_u16(v), syn.positions(0, st.nb))
             assert kvg.kvg_store_export(st.store.h, b) == blk.serialize()
-        # every one of the 1,000 random grafts reads its own block's needle
-        # (and so not the previous block's: the window really moves)
+        # every one of the 1,000 random grafts: every restored page's SHA-256
+        # equals the block's stored page digest (the block bytes, pinned to
+        # the oracle above), and the decode reads its own block's needle (and
+        # so not the previous block's: the window really moves)
         prev = None
+        rep = kvg.kvg_graft_report()
         for _ in range(len(st.order)):
             b = st.run_step()
-            s.synchronize()
+            kvg.kvg_verify(st.store.h, b, st.cache.h, 0, 0, kvg.KVG_GRAFT_SYNC, s, report=rep)
+            assert rep.n_mismatch == 0 and rep.n_pages_checked == w.n_layers * 2 * (st.nb // w.page_size), b
             assert st.needle_error(b) <= 1e-2, b
             if prev is not None and st.tag(prev) != st.tag(b):
                 assert float((st.out.float() - st.tag(prev)).abs().max()) > 1e-2
