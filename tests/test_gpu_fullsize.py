@@ -260,19 +260,6 @@ def test_batched_library_full_size(oracle, consecutive):
         pt, pf, ps = tables(st.cache)
         assert np.array_equal(pt, meta.page_table) and np.array_equal(pf, meta.page_fill)
         assert np.array_equal(ps, meta.positions)
-        if not consecutive:
-            # every page of all 128 grafts: the batch again, digest-verified
-            # (each restored page's SHA-256 against the block's stored digest)
-            # before any decode-step row lands in a ragged tail page
-            for sq in range(nS):
-                kvg.kvg_cache_release(st.cache.h, sq, s)
-            rep = kvg.kvg_graft_report()
-            kvg.kvg_graft_batch(st.store.h, st.batch_bids, st.cache.h, st.batch_seqs,
-                                kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, s, report=rep)
-            n_blk_pages = sum(-(-int(st.lens[b]) // P) for sq in range(nS) for b in st.ids[sq])
-            assert rep.n_mismatch == 0 and rep.n_pages_checked == w.n_layers * 2 * n_blk_pages
-            st.run_step()  # back to the state after a full step
-            s.synchronize()
         # grafted pages equal the deposited blocks' pages (sampled), incl. ragged tail pages
         for sq in (0, 13, nS - 1):
             j0 = 0
@@ -311,6 +298,17 @@ def test_batched_library_full_size(oracle, consecutive):
                 ref = oracle.gqa_decode(syn.as_u16(st.q[l, sq]), np.concatenate(ks), np.concatenate(vs), st.scale)
                 compare_decode(oracle, syn.as_u16(st.out[l, sq]), ref,
                                what=f"batched{' consecutive' if consecutive else ''} seq {sq} layer {l}")
+        if not consecutive:
+            # every page of all 128 grafts: the batch again, digest-verified
+            # (each restored page's SHA-256 against the block's stored digest)
+            # before any decode-step row lands in a ragged tail page
+            for sq in range(nS):
+                kvg.kvg_cache_release(st.cache.h, sq, s)
+            rep = kvg.kvg_graft_report()
+            kvg.kvg_graft_batch(st.store.h, st.batch_bids, st.cache.h, st.batch_seqs,
+                                kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, s, report=rep)
+            n_blk_pages = sum(-(-int(st.lens[b]) // P) for sq in range(nS) for b in st.ids[sq])
+            assert rep.n_mismatch == 0 and rep.n_pages_checked == w.n_layers * 2 * n_blk_pages
     finally:
         _close(st.cache, st.store)
 
