@@ -650,11 +650,12 @@ class StepBatched:
     its position tags run without a gap (the same single batched call, with
     per-graft deltas; their keys are rotated during the copy)."""
 
-    def __init__(self, kvg, device, stream, n_layers=4, consecutive=False):
+    def __init__(self, kvg, device, stream, n_layers=4, consecutive=False, n_store=syn.BATCHED_STORE):
         self.kvg, self.stream = kvg, stream
         self.w = w = syn.BATCHED.with_layers(n_layers or 4)
         P = w.page_size
-        self.lens, self.ids = syn.batched_plan()
+        self.lens, self.ids = syn.batched_plan(n_store=n_store)
+        self.n_store = n_store
         nS = syn.BATCHED_SEQS
         self.steps = syn.BATCHED_STEPS
         self.dims = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, P, w.rope_theta, 0)
@@ -850,7 +851,7 @@ def measure_h2d(device, nbytes=32 << 20, reps=20):
 
 
 def measure_other(kvg, device, config, steps, warmup, layers=0, deep_blocks=syn.DEEP_BLOCKS,
-                  consecutive=False, st=None):
+                  consecutive=False, st=None, batched_store=syn.BATCHED_STORE):
     """Builds (unless st is given) and times one of the other workloads;
     returns its JSON line (with the set-up time and the clocks of its own
     timed region)."""
@@ -865,7 +866,7 @@ def measure_other(kvg, device, config, steps, warmup, layers=0, deep_blocks=syn.
     elif config == "31b":
         st = Step31B(kvg, device, stream, layers)
     elif config == "batched":
-        st = StepBatched(kvg, device, stream, layers or 4, consecutive=consecutive)
+        st = StepBatched(kvg, device, stream, layers or 4, consecutive=consecutive, n_store=batched_store)
     else:
         st = StepDeep(kvg, device, stream, deep_blocks)
     setup_s = time.perf_counter() - t_setup
@@ -927,7 +928,8 @@ def measure_other(kvg, device, config, steps, warmup, layers=0, deep_blocks=syn.
     elif config == "batched":
         line["value"] = round(step_bytes / (ms_step * 1e-3) / 1e9, 2)
         line["config"] = {"workload": f"batched-library: L{st.w.n_layers} slice of 12b, 32 seqs x 4 blocks "
-                                      "U{2048..6144} from a 512-block HBM store, then 64 decode steps (batch 32)"
+                                      f"U{{2048..6144}} from a {st.n_store}-block HBM store, then 64 decode steps "
+                                      "(batch 32)"
                                       + (" [blocks 2-4 re-based to consecutive positions]" if st.consecutive
                                          else "")}
         line["parts"]["decode_steps"]["tokens_per_s"] = round(
@@ -990,7 +992,7 @@ def run_other(args):
     from paper_2607_14431_gb300 import kvg
     torch.cuda.set_device(0)
     line = measure_other(kvg, torch.device("cuda", 0), args.config, args.steps, args.warmup, args.layers,
-                         args.deep_blocks, args.consecutive)
+                         args.deep_blocks, args.consecutive, batched_store=args.batched_store)
     line.pop("_step")
     print(json.dumps(line), flush=True)
 
@@ -1276,6 +1278,8 @@ def main():
     ap.add_argument("--store", default="hbm", choices=["hbm", "pool"],
                     help="12b: block in an HBM store (copying graft) or in the cache pool (zero-copy graft)")
     ap.add_argument("--deep-blocks", type=int, default=syn.DEEP_BLOCKS)
+    ap.add_argument("--batched-store", type=int, default=syn.BATCHED_STORE,
+                    help="batched: blocks in the store (512; fewer for small profiling cases)")
     ap.add_argument("--consecutive", action="store_true",
                     help="batched: re-base blocks 2-4 of each sequence so its position tags are consecutive")
     ap.add_argument("--no-cpu-baseline", action="store_true")

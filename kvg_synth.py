@@ -111,12 +111,13 @@ def positions(start: int, n: int) -> np.ndarray:
     return np.arange(start, start + n, dtype=np.int32)
 
 
-def batched_plan(seed: int = BATCHED.seed):
-    """Per sequence: 4 distinct block ids from the 512-block store and the
-    store's block lengths, U{2048..6144} each."""
+def batched_plan(seed: int = BATCHED.seed, n_store: int = BATCHED_STORE):
+    """Per sequence: 4 distinct block ids from the n_store-block store (512 in
+    the workload; fewer for small profiling cases) and the store's block
+    lengths, U{2048..6144} each."""
     rng = np.random.default_rng(seed)
-    lens = rng.integers(BATCHED_LEN_RANGE[0], BATCHED_LEN_RANGE[1] + 1, size=BATCHED_STORE)
-    ids = np.stack([rng.choice(BATCHED_STORE, BATCHED_BLOCKS_PER_SEQ, replace=False)
+    lens = rng.integers(BATCHED_LEN_RANGE[0], BATCHED_LEN_RANGE[1] + 1, size=n_store)
+    ids = np.stack([rng.choice(n_store, BATCHED_BLOCKS_PER_SEQ, replace=False)
                     for _ in range(BATCHED_SEQS)])
     return lens.astype(np.int64), ids.astype(np.int64)
 

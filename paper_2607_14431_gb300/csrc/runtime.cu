@@ -763,6 +763,10 @@ struct kvg_cache {
     cudaEvent_t batch_ev = nullptr;
     std::vector<uint8_t> pinned;  // per page: owned by a pool-resident store block
     std::vector<int32_t> alias;   // per pinned page: sequences whose page tables point at it
+    // cos/sin tables of the deltas grafts have used (cos[D/2] then sin[D/2]),
+    // so a batch that re-bases many grafts does not recompute them each call
+    std::unordered_map<int64_t, std::vector<float>> rope_memo;
+    double rope_memo_theta = 0.0;  // the RoPE base the memo's tables were made with
 };
 
 // ---------------------------------------------- store inside a cache pool --
@@ -1511,6 +1515,24 @@ static void rope_table(const kvg_dims &d, int64_t delta, float *cosv, float *sin
     }
 }
 
+// rope_table for dims d (a store's; head_dim equal to the cache's),
+// remembered per delta on the cache: at most 4,096 tables are kept, and the
+// memo is cleared when it would grow past that or when d's RoPE base differs
+// from the one its tables were made with.
+static const float *rope_table_memo(kvg_cache *c, const kvg_dims &d, int64_t delta) {
+    if (c->rope_memo_theta != d.rope_theta) {
+        c->rope_memo.clear();
+        c->rope_memo_theta = d.rope_theta;
+    }
+    auto it = c->rope_memo.find(delta);
+    if (it != c->rope_memo.end()) return it->second.data();
+    if (c->rope_memo.size() >= 4096) c->rope_memo.clear();
+    const int half = d.head_dim / 2;
+    std::vector<float> t((size_t)2 * half);
+    rope_table(d, delta, t.data(), t.data() + half);
+    return c->rope_memo.emplace(delta, std::move(t)).first->second.data();
+}
+
 static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int32_t seq, int32_t dst_slot,
                              int64_t delta, uint32_t flags, void *stream, kvg_graft_report *report,
                              const ChunkEvents &ce) {
@@ -1780,7 +1802,7 @@ extern "C" kvg_status kvg_graft_batch(kvg_store *s, const uint64_t *block_ids, k
     }
     float *trig = reinterpret_cast<float *>(c->batch_host + trig_off);
     for (size_t t = 0; t < table_delta.size(); ++t)
-        rope_table(c->dims, table_delta[t], trig + t * 2 * half, trig + t * 2 * half + half);
+        memcpy(trig + t * 2 * half, rope_table_memo(c, s->dims, table_delta[t]), (size_t)2 * half * sizeof(float));
     KVG_CUDA(cudaMemcpyAsync(c->batch_dev.ptr, c->batch_host, bytes, cudaMemcpyHostToDevice, st));
     KVG_CUDA(cudaEventRecord(c->batch_ev, st));
     GraftBatchParams p{};
@@ -1797,7 +1819,8 @@ extern "C" kvg_status kvg_graft_batch(kvg_store *s, const uint64_t *block_ids, k
     p.page_bytes = c->page_bytes;
     p.pool_pages = c->n_pages;
     p.pool = c->pool;
-    const int rotate = table_delta.empty() ? 0 : c->dims.rope_style == KVG_ROPE_HALF ? 1 : 2;
+    // the store's RoPE pairing and base, as kvg_graft uses them
+    const int rotate = table_delta.empty() ? 0 : s->dims.rope_style == KVG_ROPE_HALF ? 1 : 2;
     KVG_CUDA(launch_graft_batch(p, c->n_sm, st, s->residency == KVG_RESIDENCY_PINNED_HOST ? host_copy_grid_cap() : 0,
                                 rotate));
     // verification: own-position grafts hash their restored pages; re-based
