@@ -145,10 +145,15 @@ def test_fp8_deposit_graft_verify_bit_exact(oracle, geo, ks, vs):
         with pytest.raises(kvg.KvgError) as e:
             kvg.kvg_graft(store.h, bid2, dst.h, 1, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, report=rep2)
         assert e.value.status == kvg.KVG_ERR_DIGEST and rep2.mismatch_pages[0] == bad_page
-        # relocation needs bf16 keys
+        # relocation needs bf16 keys, in a single graft and in a batch (which
+        # then grafts nothing, not even its own-position member)
         with pytest.raises(kvg.KvgError) as e:
             kvg.kvg_graft(store.h, bid, dst.h, 2, -1, 5, 0)
         assert e.value.status == kvg.KVG_ERR_ARG
+        with pytest.raises(kvg.KvgError) as e:
+            kvg.kvg_graft_batch(store.h, [bid, bid], dst.h, [2, 2], deltas=[0, 5])
+        assert e.value.status == kvg.KVG_ERR_ARG
+        assert kvg.kvg_cache_seq_info(dst.h, 2)[0] == 0
         kvg.kvg_sync(dst.h)
     # element type and scales are part of the geometry
     bf16 = kvg.make_dims(w.n_layers, w.n_kv_heads, w.head_dim, w.page_size, w.rope_theta, 0)
