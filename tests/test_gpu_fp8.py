@@ -146,12 +146,12 @@ def test_fp8_deposit_graft_verify_bit_exact(oracle, geo, ks, vs):
             kvg.kvg_graft(store.h, bid2, dst.h, 1, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, report=rep2)
         assert e.value.status == kvg.KVG_ERR_DIGEST and rep2.mismatch_pages[0] == bad_page
         # relocation needs bf16 keys, in a single graft and in a batch (which
-        # then grafts nothing, not even its own-position member)
+        # then grafts nothing)
         with pytest.raises(kvg.KvgError) as e:
             kvg.kvg_graft(store.h, bid, dst.h, 2, -1, 5, 0)
         assert e.value.status == kvg.KVG_ERR_ARG
         with pytest.raises(kvg.KvgError) as e:
-            kvg.kvg_graft_batch(store.h, [bid, bid], dst.h, [2, 2], deltas=[0, 5])
+            kvg.kvg_graft_batch(store.h, [bid], dst.h, [2], deltas=[5])
         assert e.value.status == kvg.KVG_ERR_ARG
         assert kvg.kvg_cache_seq_info(dst.h, 2)[0] == 0
         kvg.kvg_sync(dst.h)
