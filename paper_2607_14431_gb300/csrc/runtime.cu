@@ -1746,12 +1746,13 @@ extern "C" kvg_status kvg_graft_batch(kvg_store *s, const uint64_t *block_ids, k
     // one cos/sin table per distinct nonzero delta, in order of first use
     std::vector<int64_t> table_delta;
     std::vector<int32_t> trig_of(n, -1);
+    std::unordered_map<int64_t, int32_t> table_of;
     for (int32_t i = 0; i < n; ++i) {
         const int64_t delta = deltas ? deltas[i] : 0;
         if (delta == 0) continue;
-        auto f = std::find(table_delta.begin(), table_delta.end(), delta);
-        trig_of[i] = (int32_t)(f - table_delta.begin());
-        if (f == table_delta.end()) table_delta.push_back(delta);
+        auto f = table_of.emplace(delta, (int32_t)table_delta.size());
+        if (f.second) table_delta.push_back(delta);
+        trig_of[i] = f.first->second;
     }
     const int half = c->dims.head_dim / 2;
     // the job table: metas, jobs, then the cos/sin tables, in pinned host memory
