@@ -1314,7 +1314,8 @@ def main():
             gc.collect()
             torch.cuda.empty_cache()
             line["workloads"] = run_workloads(args)
-        if not args.no_cpu_baseline and not args.swa and args.kv == "bf16":
+        # the CPU baseline runs at N = 1 only (at N > 1 the other ranks would wait on it)
+        if world == 1 and not args.no_cpu_baseline and not args.swa and args.kv == "bf16":
             line["cpu_baseline"] = cpu_baseline(args.cpu_baseline_layers)
         print(json.dumps(line), flush=True)
     if world > 1:
