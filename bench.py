@@ -39,12 +39,6 @@ import torch  # noqa: E402
 import kvg_synth as syn  # noqa: E402
 
 METRIC = ("graft GB/s (HBM & host→HBM) + decode-attn tokens/s @32k grafted, % roofline")
-# ALU-pipe instructions per SHA-256 compression in graft_verify_kernel: the
-# kernel's own mix as ncu counts it (sm__inst_executed_pipe_alu over the
-# compressions of one launch, 4-layer 12b slice): 951 on the ALU pipe (funnel
-# shifts, 3-input logic), 739 on the FMA pipe (the additions and plain shifts
-# issued as IMADs), 47 other; 1,737 in all.  The ALU pipe is the binding one.
-SHA_ALU_OPS_PER_COMPRESSION = 951
 ALU_LANES_PER_SM = 64  # 4 SM sub-partitions x 16 ALU-pipe lanes
 
 
@@ -57,9 +51,11 @@ def load_peaks():
         return 6800.0, 2070.0, "fallback"
 
 
-def load_traffic():
-    """Per-launch DRAM bytes from the committed ncu summary, keyed by kernel,
-    kept only while the kernel source is unchanged since the capture."""
+def load_ncu_figures():
+    """Per-kernel figures from the committed ncu summary
+    (profiles/ncu_traffic.txt: DRAM bytes per launch, and for the hashing
+    kernel its ALU-pipe instructions per SHA-256 compression), kept only
+    while the kernel's source file is unchanged since the capture."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
     out = {}
     if not os.path.exists(path):
@@ -72,8 +68,20 @@ def load_traffic():
         parts = dict(kv.split("=", 1) for kv in line.split())
         src = os.path.join(ROOT, "paper_2607_14431_gb300", "csrc", parts["source"])
         if os.path.exists(src) and hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] == parts["sha"]:
-            out[parts["kernel"]] = float(parts["bytes_per_launch"])
+            out[parts["kernel"]] = {k: float(v) for k, v in parts.items() if k not in ("kernel", "source", "sha")}
     return out
+
+
+def load_traffic():
+    """Per-launch DRAM bytes from the committed ncu summary, keyed by kernel."""
+    return {k: v["bytes_per_launch"] for k, v in load_ncu_figures().items() if "bytes_per_launch" in v}
+
+
+def sha_alu_ops_per_compression():
+    """ALU-pipe instructions per SHA-256 compression of graft_verify_kernel,
+    the kernel's own instruction mix as ncu counted it (None once the
+    kernel's source has changed since that capture)."""
+    return load_ncu_figures().get("graft_verify_kernel", {}).get("alu_inst_per_compression")
 
 
 def aggregate(total_ms: float, steps: int, step_bytes: int, world: int, device) -> tuple:
@@ -333,6 +341,7 @@ def run_kvg(args, rank, world):
     hbm_peak, sm_max, peak_kind = load_peaks()
     n_sm = torch.cuda.get_device_properties(device).multi_processor_count
     alu_peak = n_sm * ALU_LANES_PER_SM * sm_max * 1e6  # ALU-pipe ops per second at the max SM clock
+    alu_per_c = sha_alu_ops_per_compression()
     swa = tuple(int(x) for x in args.swa.split(":")) if args.swa else None
     st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool", schedule=args.schedule,
                  swa=swa, kv=args.kv)
@@ -397,8 +406,8 @@ def run_kvg(args, rank, world):
             b = 2 * st.blk_pages
             alone[name] = {"ms": round(ms, 4), "algorithmic_bytes": b, "gbs": round(b / (ms * 1e-3) / 1e9, 1),
                            "hbm_frac": round(b / (ms * 1e-3) / 1e9 / hbm_peak, 3), "clocks": clk_g.stop()}
-            if flags:
-                ops = st.sha_blocks * SHA_ALU_OPS_PER_COMPRESSION
+            if flags and alu_per_c:
+                ops = st.sha_blocks * alu_per_c
                 alone[name].update({"alu_tops": round(ops / (ms * 1e-3) / 1e12, 3),
                                     "alu_frac": round(ops / (ms * 1e-3) / alu_peak, 3)})
         kvg.kvg_sync(st.cache.h, stream, 60.0)
@@ -470,20 +479,20 @@ def run_kvg(args, rank, world):
             gbs = b / (ms * 1e-3) / 1e9
             parts[p].update({"gbs": round(gbs, 1), "hbm_frac": round(gbs / hbm_peak, 3)})
         if p in hashing:
-            ops = st.sha_blocks * SHA_ALU_OPS_PER_COMPRESSION
             parts[p].update({"hashed_bytes": st.hashed_bytes,
                              "hashed_gbs": round(st.hashed_bytes / (ms * 1e-3) / 1e9, 1),
-                             "compressions": st.sha_blocks,
-                             "alu_ops_per_compression": SHA_ALU_OPS_PER_COMPRESSION,
-                             "alu_tops": round(ops / (ms * 1e-3) / 1e12, 3),
-                             "alu_frac": round(ops / (ms * 1e-3) / alu_peak, 3)})
+                             "compressions": st.sha_blocks, "alu_ops_per_compression": alu_per_c})
+            if alu_per_c:
+                ops = st.sha_blocks * alu_per_c
+                parts[p].update({"alu_tops": round(ops / (ms * 1e-3) / 1e12, 3),
+                                 "alu_frac": round(ops / (ms * 1e-3) / alu_peak, 3)})
     parts["decode"]["tokens_per_s"] = round(1e3 / phase_ms["decode"], 1)
     kernel_of = {"graft": "graft_kernel", "verify": "sha256_leaves_kernel", "append": "append_tma_kernel",
                  "decode": "decode_kernel", "graft_verify": "graft_verify_kernel"}
     # dominant kernel: the longest phase that moves or hashes bytes
     dom = max((p for p in st.phases if st.bytes.get(p) or p in hashing), key=lambda p: phase_ms[p])
-    if dom in hashing:
-        ops = st.sha_blocks * SHA_ALU_OPS_PER_COMPRESSION
+    if dom in hashing and alu_per_c:
+        ops = st.sha_blocks * alu_per_c
         ach = ops / (phase_ms[dom] * 1e-3) / 1e12
         roof = {"bound": "alu", "kernel": kernel_of[dom], "achieved": round(ach, 3), "peak": round(alu_peak / 1e12, 3),
                 "unit": "Top/s", "frac": round(ach / (alu_peak / 1e12), 3), "traffic": traffic.get(kernel_of[dom]),
