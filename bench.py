@@ -77,11 +77,11 @@ def load_traffic():
     return {k: v["bytes_per_launch"] for k, v in load_ncu_figures().items() if "bytes_per_launch" in v}
 
 
-def sha_alu_ops_per_compression():
-    """ALU-pipe instructions per SHA-256 compression of graft_verify_kernel,
-    the kernel's own instruction mix as ncu counted it (None once the
+def sha_alu_ops_per_compression(kernel="graft_verify_ring_kernel"):
+    """ALU-pipe instructions per SHA-256 compression of the verified graft's
+    kernel, its own instruction mix as ncu counted it (None once the
     kernel's source has changed since that capture)."""
-    return load_ncu_figures().get("graft_verify_kernel", {}).get("alu_inst_per_compression")
+    return load_ncu_figures().get(kernel, {}).get("alu_inst_per_compression")
 
 
 def aggregate(total_ms: float, steps: int, step_bytes: int, world: int, device) -> tuple:
@@ -341,10 +341,13 @@ def run_kvg(args, rank, world):
     hbm_peak, sm_max, peak_kind = load_peaks()
     n_sm = torch.cuda.get_device_properties(device).multi_processor_count
     alu_peak = n_sm * ALU_LANES_PER_SM * sm_max * 1e6  # ALU-pipe ops per second at the max SM clock
-    alu_per_c = sha_alu_ops_per_compression()
     swa = tuple(int(x) for x in args.swa.split(":")) if args.swa else None
     st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool", schedule=args.schedule,
                  swa=swa, kv=args.kv)
+    # the verified graft runs graft_verify_ring_kernel for a full wave of it
+    # (five 128-leaf CTAs on every SM) or more, else graft_verify_kernel
+    gv_kernel = "graft_verify_ring_kernel" if st.sha_blocks // 65 >= n_sm * 5 * 128 else "graft_verify_kernel"
+    alu_per_c = sha_alu_ops_per_compression(gv_kernel)
 
     # correctness of the configuration being timed: one verified step
     st.run_step()
@@ -488,7 +491,7 @@ def run_kvg(args, rank, world):
                                  "alu_frac": round(ops / (ms * 1e-3) / alu_peak, 3)})
     parts["decode"]["tokens_per_s"] = round(1e3 / phase_ms["decode"], 1)
     kernel_of = {"graft": "graft_kernel", "verify": "sha256_leaves_kernel", "append": "append_tma_kernel",
-                 "decode": "decode_kernel", "graft_verify": "graft_verify_kernel"}
+                 "decode": "decode_kernel", "graft_verify": gv_kernel}
     # dominant kernel: the longest phase that moves or hashes bytes
     dom = max((p for p in st.phases if st.bytes.get(p) or p in hashing), key=lambda p: phase_ms[p])
     if dom in hashing and alu_per_c:
@@ -507,7 +510,7 @@ def run_kvg(args, rank, world):
         # window from the release to the decode's start moves both kernels' bytes
         win = statistics.mean(evs[k]["main"][1].elapsed_time(evs[k]["main"][3]) for k in range(K))
         wb = st.bytes["append"] + st.bytes["graft_verify"]
-        roof["concurrent"] = {"kernels": ["append_tma_kernel", "graft_verify_kernel"], "window_ms": round(win, 4),
+        roof["concurrent"] = {"kernels": ["append_tma_kernel", gv_kernel], "window_ms": round(win, 4),
                               "bytes": wb, "achieved": round(wb / (win * 1e-3) / 1e9, 1),
                               "frac": round(wb / (win * 1e-3) / 1e9 / hbm_peak, 3)}
     line = {

@@ -129,6 +129,77 @@ __device__ __forceinline__ const uint8_t *page_addr(const PageSource &s, int64_t
     return s.base + ((uint64_t)plane * s.plane_pages + (uint64_t)s.pid[j]) * s.page_bytes;
 }
 
+// 16-byte asynchronous copy global -> this thread's shared memory (LDGSTS,
+// L1 bypassed); completion is tracked by the thread's cp.async groups.
+__device__ __forceinline__ void cp_async16(void *smem_dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(smem_dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// SHA-256 of one leaf that is also copied to `copy_to`, from the same
+// registers that are hashed, so the bytes written are exactly the bytes whose
+// digest is checked.  The leaf's next R 64-byte blocks are in flight through
+// a ring of this thread's shared memory (ring: R x 64 contiguous bytes), not
+// held in registers, so their latency (long when other kernels keep HBM
+// busy) hides behind the compressions without costing registers.  (A layout
+// with the 32 lanes' vectors side by side, free of bank conflicts, measured
+// slower in the 12b step: 6.05 against 5.94 ms.)
+template <int R>
+__device__ __forceinline__ void hash_leaf_ring(const uint8_t *leaf, uint64_t len, uint8_t *copy_to, uint32_t st[8],
+                                               uint32_t one, uint4 *ring) {
+    const uint4 *v = reinterpret_cast<const uint4 *>(leaf);
+    uint4 *o = reinterpret_cast<uint4 *>(copy_to);
+    init_state(st);
+    const int nfull = (int)(len >> 6);
+#pragma unroll
+    for (int b = 0; b < R; ++b) {
+        if (b < nfull)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) cp_async16(ring + 4 * b + q, v + 4 * b + q);
+        cp_async_commit();  // one group per block, empty or not, so the count stays uniform
+    }
+    for (int blk = 0; blk < nfull; ++blk) {
+        cp_async_wait<R - 1>();  // block blk has landed
+        const int slot = blk % R;
+        uint32_t w[16];
+        uint4 x[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) x[q] = ring[4 * slot + q];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            w[4 * q + 0] = bswap(x[q].x);
+            w[4 * q + 1] = bswap(x[q].y);
+            w[4 * q + 2] = bswap(x[q].z);
+            w[4 * q + 3] = bswap(x[q].w);
+        }
+        // the slot is free once its words are in registers: refill it
+        if (blk + R < nfull)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) cp_async16(ring + 4 * slot + q, v + 4 * (blk + R) + q);
+        cp_async_commit();
+#pragma unroll
+        for (int q = 0; q < 4; ++q) __stcs(o + 4 * blk + q, x[q]);
+        compress(st, w, one);
+    }
+    cp_async_wait<0>();
+    const int rem = (int)(len & 63);
+    if (rem == 0) {
+        uint32_t w[16];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) w[q] = 0;
+        w[0] = 0x80000000u;
+        const uint64_t bits = len * 8ull;
+        w[14] = (uint32_t)(bits >> 32);
+        w[15] = (uint32_t)bits;
+        compress(st, w, one);
+    } else {
+        for (int q = 0; q < rem / 16; ++q) o[4 * nfull + q] = v[4 * nfull + q];
+        finish(st, leaf + (len & ~63ull), rem, len, one);
+    }
+}
+
 // SHA-256 of one leaf of `len` bytes (16-byte aligned).  With COPY the leaf
 // is also written to `copy_to`, from the same registers that are hashed, so
 // the bytes written are exactly the bytes whose digest is checked.
@@ -224,6 +295,43 @@ __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src
             po = plane * src.out_plane_stride + src.out_j0 + (p - plane * src.npb);
         }
         store_state(out + (po * leaves_per_page + i) * 8, st);
+    }
+}
+
+// graft_verify_kernel with each thread keeping its leaf's next
+// kGraftVerifyRing blocks in flight through its own slots of shared memory
+// instead of two blocks in registers; the registers that frees let five CTAs
+// of 128 threads stay resident per SM (96 registers).  Used for launches of
+// at least one full wave of it (five CTAs on every SM): beside a concurrent
+// append the 12b step's window shortens (step 5.94 against 6.01 ms; alone
+// the same 3.12 ms; rings of two or four blocks, or six CTAs at 80
+// registers, measured slower in the step).  For smaller launches each leaf's
+// chain latency decides and the register form is faster (the tiny verified
+// graft 0.099 against 0.133 ms).
+constexpr int kGraftVerifyRing = 3;
+__global__ void __launch_bounds__(128, 5) graft_verify_ring_kernel(const GraftParams p, int64_t leaves_per_page,
+                                                                   uint32_t *__restrict__ out, uint32_t one) {
+    constexpr int R = kGraftVerifyRing;
+    extern __shared__ __align__(16) uint4 ring_mem[];
+    graft_metadata(p);
+    const uint64_t page_bytes = p.page_bytes;
+    const int64_t n_leaves = (int64_t)p.n_layers * 2 * p.npb * leaves_per_page;
+    uint4 *ring = ring_mem + threadIdx.x * 4 * R;
+    for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < n_leaves;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t page_u = idx / leaves_per_page;
+        const int64_t i = idx - page_u * leaves_per_page;
+        const int64_t lkv = page_u / p.npb;
+        const int64_t jj = page_u - lkv * p.npb;
+        const uint64_t off = (uint64_t)i * kLeafBytes;
+        uint64_t len = page_bytes - off;
+        if (len > kLeafBytes) len = kLeafBytes;
+        const int64_t block_page = lkv * p.block_pages + p.page_base + jj;
+        const uint8_t *src = p.src + (uint64_t)block_page * page_bytes + off;
+        uint8_t *dst = p.pool + ((uint64_t)lkv * p.pool_pages + (uint64_t)p.pids.pid[jj]) * page_bytes + off;
+        uint32_t st[8];
+        hash_leaf_ring<R>(src, len, dst, st, one, ring);
+        store_state(out + (block_page * leaves_per_page + i) * 8, st);
     }
 }
 
@@ -469,12 +577,19 @@ cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int 
     const int64_t n = (int64_t)p.n_layers * 2 * p.npb * m;
     if (n == 0) return cudaSuccess;
     int64_t grid = (n + 127) / 128;
-    // One CTA per 128 leaves (no grid-stride cap by default): 4 CTAs of
-    // 125 registers are resident per SM and the rest queue, which measured
-    // 2-3% faster than a capped, striding grid.
+    // One CTA per 128 leaves (no grid-stride cap by default): four CTAs of
+    // the register form (125 registers) or five of the ring form (96) are
+    // resident per SM and the rest queue.
     static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 0);
     if (ctas_per_sm > 0 && grid > (int64_t)n_sm * ctas_per_sm) grid = (int64_t)n_sm * ctas_per_sm;
-    graft_verify_kernel<<<(int)grid, 128, 0, s>>>(p, m, leaf_words, 1u);
+    // a full wave of the ring form (five CTAs on every SM) or more: the ring
+    // form; fewer leaves: the register form (see graft_verify_ring_kernel)
+    if (n >= (int64_t)n_sm * 5 * 128 && grid > (int64_t)n_sm * 4) {
+        const size_t smem = (size_t)128 * kGraftVerifyRing * 64;  // 24 KiB of ring slots per CTA
+        graft_verify_ring_kernel<<<(int)grid, 128, smem, s>>>(p, m, leaf_words, 1u);
+    } else {
+        graft_verify_kernel<<<(int)grid, 128, 0, s>>>(p, m, leaf_words, 1u);
+    }
     count_launches(1);
     return cudaGetLastError();
 }
