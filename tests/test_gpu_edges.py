@@ -346,3 +346,49 @@ def test_graft_of_pages_too_large_for_two_stages(oracle):
         j, r = divmod(nb, P)  # padding rows of the last page: copied unchanged (zeros)
         assert not pool[:, 0, pt[1, j], :, r:, :].any()
         kvg.kvg_sync(c.h)
+
+
+def test_large_verified_graft_with_ragged_leaves(oracle):
+    """A verified graft large enough for the shared-memory ring form of the
+    one-pass kernel (a full wave of it: 98,304 leaves here) on pages of 4,224
+    bytes, so every page has a full 4 KiB leaf and a 128-byte one: the
+    deposited block equals the oracle's (49,152 page digests), the graft
+    restores every pool byte as the oracle's cache holds it and checks every
+    page, and a flipped byte is reported at its page."""
+    kvg = need_gpu()
+    w = syn.Workload("ragleaf", 24, 2, 1, 64, 33, 10000.0, 0x7A)  # page: 1 x 33 x 64 x 2 = 4,224 bytes
+    P = w.page_size
+    npb = 1024
+    n = npb * P
+    k, v = syn.kv_rows(w, n, w.seed)
+    k, v = syn.as_u16(k), syn.as_u16(v)
+    dims = dims_for(kvg, w)
+    src = kvg.Cache(dims, npb + 2, 1, n + P)
+    append(kvg, src, 0, k, v, syn.positions(0, n))
+    store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, 1 << 30)
+    bid = kvg.kvg_deposit(store.h, src.h, 0, 0, n)
+    od = oracle_dims(oracle, w)
+    blk = oracle.block_from_kv(od, k, v, syn.positions(0, n))
+    ser = blk.serialize()
+    assert kvg.kvg_store_export(store.h, bid) == ser
+    src.close()
+    dst = kvg.Cache(dims, npb + 2, 1, n + P)
+    fill_canary(dst)
+    oc = oracle.OracleCache(od, npb + 2, 1, n + P, fill=CANARY)
+    rep = kvg.kvg_graft_report()
+    kvg.kvg_graft(store.h, bid, dst.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, report=rep)
+    assert rep.n_mismatch == 0 and rep.n_pages_checked == w.n_layers * 2 * npb
+    oc.graft(0, blk)
+    assert np.array_equal(pool_u16(dst, w), oc.pool)
+    # one flipped byte in the short leaf of page (plane 37, page 700)
+    info = kvg.kvg_store_block_info(store.h, bid)
+    bad = bytearray(ser)
+    bad_page = 37 * npb + 700
+    bad[info.pages_offset + bad_page * w.page_bytes + 4096 + 77] ^= 0x10
+    bid2 = kvg.kvg_store_import(store.h, bytes(bad), 0)
+    kvg.kvg_cache_release(dst.h, 0)
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_graft(store.h, bid2, dst.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, report=rep)
+    assert e.value.status == kvg.KVG_ERR_DIGEST
+    assert rep.n_mismatch == 1 and rep.mismatch_pages[0] == bad_page
+    kvg.kvg_sync(dst.h)
