@@ -345,8 +345,12 @@ def run_kvg(args, rank, world):
     st = Step12B(kvg, device, stream, side, args.layers, pool_store=args.store == "pool", schedule=args.schedule,
                  swa=swa, kv=args.kv)
     # the verified graft runs graft_verify_ring_kernel for a full wave of it
-    # (five 128-leaf CTAs on every SM) or more, else graft_verify_kernel
-    gv_kernel = "graft_verify_ring_kernel" if st.sha_blocks // 65 >= n_sm * 5 * 128 else "graft_verify_kernel"
+    # (five 128-leaf CTAs on every SM) or more on a bf16 cache, else
+    # graft_verify_kernel; the append is append_tma_kernel (bf16) or
+    # append_e4m3_kernel (fp8)
+    gv_kernel = ("graft_verify_ring_kernel" if st.kv == "bf16" and st.sha_blocks // 65 >= n_sm * 5 * 128
+                 else "graft_verify_kernel")
+    app_kernel = "append_tma_kernel" if st.kv == "bf16" else "append_e4m3_kernel"
     alu_per_c = sha_alu_ops_per_compression(gv_kernel)
 
     # correctness of the configuration being timed: one verified step
@@ -468,7 +472,8 @@ def run_kvg(args, rank, world):
         e2e["h2d_ceiling_gbs"] = round(h2d, 2)
         e2e["host_graft_link_frac"] = round(e2e["host_graft_gbs"] / h2d, 3)
 
-    traffic = load_traffic()
+    # per-launch DRAM bytes from ncu are for the 48-layer launches
+    traffic = load_traffic() if st.w.n_layers == syn.B12.n_layers else {}
     parts = {}
     hashing = ("verify", "graft_verify")
     for p in st.phases:
@@ -490,7 +495,7 @@ def run_kvg(args, rank, world):
                 parts[p].update({"alu_tops": round(ops / (ms * 1e-3) / 1e12, 3),
                                  "alu_frac": round(ops / (ms * 1e-3) / alu_peak, 3)})
     parts["decode"]["tokens_per_s"] = round(1e3 / phase_ms["decode"], 1)
-    kernel_of = {"graft": "graft_kernel", "verify": "sha256_leaves_kernel", "append": "append_tma_kernel",
+    kernel_of = {"graft": "graft_kernel", "verify": "sha256_leaves_kernel", "append": app_kernel,
                  "decode": "decode_kernel", "graft_verify": gv_kernel}
     if st.schedule == "fused":
         # The verified graft and the append run side by side on two streams
@@ -502,14 +507,15 @@ def run_kvg(args, rank, world):
         # each kernel's own figures beside it.
         win = statistics.mean(evs[k]["main"][1].elapsed_time(evs[k]["main"][3]) for k in range(K))
         wb = st.bytes["append"] + st.bytes["graft_verify"]
-        tr = [traffic.get("append_tma_kernel"), traffic.get(gv_kernel)]
+        # (ncu traffic is kept for the bf16 step's kernels only)
+        tr = [traffic.get(app_kernel), traffic.get(gv_kernel)] if st.kv == "bf16" else [None]
         gv = parts["graft_verify"]
-        roof = {"bound": "hbm", "kernel": f"append_tma_kernel || {gv_kernel}",
+        roof = {"bound": "hbm", "kernel": f"{app_kernel} || {gv_kernel}",
                 "achieved": round(wb / (win * 1e-3) / 1e9, 1), "peak": hbm_peak, "unit": "GB/s",
                 "frac": round(wb / (win * 1e-3) / 1e9 / hbm_peak, 3),
                 "traffic": sum(tr) if all(t is not None for t in tr) else None, "peak_kind": peak_kind,
                 "window_ms": round(win, 4), "algorithmic_bytes": wb,
-                "members": {"append_tma_kernel": {k: parts["append"][k] for k in ("ms", "gbs", "hbm_frac")},
+                "members": {app_kernel: {k: parts["append"][k] for k in ("ms", "gbs", "hbm_frac")},
                             gv_kernel: {k: gv[k] for k in ("ms", "gbs", "hbm_frac", "alu_tops", "alu_frac") if k in gv}}}
     else:
         # dominant kernel: the longest phase that moves or hashes bytes
@@ -1261,7 +1267,8 @@ def config_12b(n_layers=48, world=1, pool_store=False, swa=None, kv="bf16"):
                         + (f" [sliding-window layers: window {swa[0]}, every {swa[1]}th layer global]" if swa else "")
                         + (f" [fp8 E4M3 KV, scales k {syn.FP8_K_SCALE} v {syn.FP8_V_SCALE}]" if kv == "e4m3" else ""),
             "global_batch": world, "seq_len": syn.B12_CTX, "parallelism": f"replicas{world}",
-            "l2": "inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)",
+            "l2": ("inputs larger than L2 (3 GiB block, 9.7 GB fresh rows, 12.9 GB cache)" if kv == "bf16" else
+                   "inputs larger than L2 (1.6 GB fp8 block, 9.7 GB bf16 fresh rows, 6.4 GB fp8 cache)"),
             "seed": hex(syn.B12.seed)}
 
 

@@ -1644,8 +1644,13 @@ static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int3
         // piped: the last (short) chunk is copied and hashed in one pass, so
         // its hash needs no second read after it has crossed the link
         const bool one_pass = fused || (piped && chunk == n_chunks - 1);
+        // the ring form for bf16 caches only: it shortens the window it shares
+        // with the bf16 append (a shared-memory-staged kernel), but starves
+        // beside the fp8 append (a register kernel: the SMs it runs on are set
+        // up without room for the ring's shared memory)
         if (one_pass)
-            KVG_CUDA(launch_graft_verify(p, static_cast<uint32_t *>(c->leaf.ptr), c->n_sm, st));
+            KVG_CUDA(launch_graft_verify(p, static_cast<uint32_t *>(c->leaf.ptr), c->n_sm, st,
+                                         c->dims.kv_dtype == KVG_KV_BF16));
         else
             KVG_CUDA(launch_graft_copy(p, c->n_sm, st, host_src ? host_copy_ctas : 0, c->status));
         if (n_ev > 0) {

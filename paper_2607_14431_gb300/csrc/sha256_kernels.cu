@@ -572,7 +572,7 @@ cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_
     return cudaGetLastError();
 }
 
-cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int n_sm, cudaStream_t s) {
+cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int n_sm, cudaStream_t s, bool ring_ok) {
     const int64_t m = (int64_t)((p.page_bytes + kLeafBytes - 1) / kLeafBytes);
     const int64_t n = (int64_t)p.n_layers * 2 * p.npb * m;
     if (n == 0) return cudaSuccess;
@@ -582,9 +582,12 @@ cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int 
     // resident per SM and the rest queue.
     static const int ctas_per_sm = env_knob("KVG_SHA_CTAS_PER_SM", 0);
     if (ctas_per_sm > 0 && grid > (int64_t)n_sm * ctas_per_sm) grid = (int64_t)n_sm * ctas_per_sm;
-    // a full wave of the ring form (five CTAs on every SM) or more: the ring
-    // form; fewer leaves: the register form (see graft_verify_ring_kernel)
-    if (n >= (int64_t)n_sm * 5 * 128 && grid > (int64_t)n_sm * 4) {
+    // a full wave of the ring form (five CTAs on every SM) or more, where the
+    // caller allows it: the ring form; otherwise the register form (see
+    // graft_verify_ring_kernel).  KVG_SHA_REGISTER_FORM=1 keeps the register
+    // form for every size.
+    static const bool regs_only = env_knob("KVG_SHA_REGISTER_FORM", 0) > 0;
+    if (ring_ok && !regs_only && n >= (int64_t)n_sm * 5 * 128 && grid > (int64_t)n_sm * 4) {
         const size_t smem = (size_t)128 * kGraftVerifyRing * 64;  // 24 KiB of ring slots per CTA
         graft_verify_ring_kernel<<<(int)grid, 128, smem, s>>>(p, m, leaf_words, 1u);
     } else {
