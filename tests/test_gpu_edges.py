@@ -392,3 +392,44 @@ def test_large_verified_graft_with_ragged_leaves(oracle):
     assert e.value.status == kvg.KVG_ERR_DIGEST
     assert rep.n_mismatch == 1 and rep.mismatch_pages[0] == bad_page
     kvg.kvg_sync(dst.h)
+
+
+def test_graft_batch_host_checks_change_nothing(oracle):
+    """kvg_graft_batch's host checks: an empty or oversized batch, a bad
+    sequence id, an unknown block, a delta pushing a tag out of range, and a
+    pool-resident store are all refused with their status before any work,
+    and the cache is unchanged (no pages taken, no tags written)."""
+    kvg = need_gpu()
+    w = syn.TINY
+    dims = dims_for(kvg, w)
+    src = kvg.Cache(dims, 40, 1, 512)
+    k, v = _kv(w, 100, 0x51)
+    append(kvg, src, 0, k, v, syn.positions(0, 100))
+    store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, 1 << 24)
+    bid = kvg.kvg_deposit(store.h, src.h, 0, 0, 100)
+    c = kvg.Cache(dims, 40, 2, 512)
+    fill_canary(c)
+    before = pool_u16(c, w).copy()
+    cases = [
+        (lambda: kvg.kvg_graft_batch(store.h, [bid] * 4097, c.h, [0] * 4097), kvg.KVG_ERR_ARG),
+        (lambda: kvg.kvg_graft_batch(store.h, [bid], c.h, [2]), kvg.KVG_ERR_ARG),
+        (lambda: kvg.kvg_graft_batch(store.h, [bid, bid + 7], c.h, [0, 1]), kvg.KVG_ERR_NOT_FOUND),
+        (lambda: kvg.kvg_graft_batch(store.h, [bid, bid], c.h, [0, 1], deltas=[3, -4]), kvg.KVG_ERR_POSITION),
+        (lambda: kvg.kvg_graft_batch(store.h, [bid, bid], c.h, [0, 1], deltas=[0, 2 ** 31 - 50]),
+         kvg.KVG_ERR_POSITION),
+    ]
+    pool_store = kvg.PoolStore(src, 1 << 22)
+    pbid = kvg.kvg_deposit(pool_store.h, src.h, 0, 0, 100)
+    cases.append((lambda: kvg.kvg_graft_batch(pool_store.h, [pbid], src.h, [0]), kvg.KVG_ERR_ARG))
+    for call, status in cases:
+        with pytest.raises(kvg.KvgError) as e:
+            call()
+        assert e.value.status == status, (e.value.status, status)
+    assert kvg.kvg_cache_seq_info(c.h, 0) == (0, 0) and kvg.kvg_cache_seq_info(c.h, 1) == (0, 0)
+    assert np.array_equal(pool_u16(c, w), before)
+    pt, pf, ps = tables(c)
+    assert (pt == -1).all() and (pf == 0).all() and (ps == -1).all()
+    # and the same batch with valid arguments then works
+    kvg.kvg_graft_batch(store.h, [bid, bid], c.h, [0, 1], kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, deltas=[0, 9])
+    assert kvg.kvg_cache_seq_info(c.h, 1)[0] == 100
+    kvg.kvg_sync(c.h)
