@@ -9,8 +9,8 @@ import pytest
 import torch
 
 import kvg_synth as syn
-from kvg_testlib import (CANARY, append, compare_decode, decode, dims_for, fill_canary, need_gpu, oracle_dims,
-                         pool_u16, tables, to_dev)
+from kvg_testlib import (CANARY, append, compare_decode, decode, dims_for, fill_canary, geometry, need_gpu,
+                         oracle_dims, pool_u16, tables, to_dev, u16)
 
 pytestmark = pytest.mark.gpu
 
@@ -433,3 +433,51 @@ def test_graft_batch_host_checks_change_nothing(oracle):
     kvg.kvg_graft_batch(store.h, [bid, bid], c.h, [0, 1], kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC, deltas=[0, 9])
     assert kvg.kvg_cache_seq_info(c.h, 1)[0] == 100
     kvg.kvg_sync(c.h)
+
+
+def test_two_caches_on_two_streams_match_serial(oracle):
+    """Different caches are independent: the same deposit / verified graft /
+    append / decode sequence issued on two caches from two streams at once,
+    each with its own store, gives the same bytes as the sequence run alone,
+    and the oracle's decode through the gate."""
+    kvg = need_gpu()
+    w = geometry("d256")
+    P = w.page_size
+    dims = dims_for(kvg, w)
+    nb, nf = 5 * P + 9, 3 * P + 1
+    k, v = _kv(w, nb + nf, 0x2C)
+    q = syn.as_u16(syn.queries(w, w.n_layers, 1, 0x2D))
+    scale = 1.0 / math.sqrt(w.head_dim)
+
+    def run(stream, sync_each=False):
+        src = kvg.Cache(dims, 16, 1, 16 * P)
+        store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, 1 << 26)
+        dst = kvg.Cache(dims, 16, 1, 16 * P)
+        # k, v arguments are [L][n][Hkv][D] for the n rows appended
+        kd, vd = to_dev(np.ascontiguousarray(k[:, :nb])), to_dev(np.ascontiguousarray(v[:, :nb]))
+        pos = to_dev(syn.positions(0, nb))
+        h = stream.cuda_stream
+        kvg.kvg_cache_append(src.h, 0, kd.data_ptr(), vd.data_ptr(), pos.data_ptr(), nb, h)
+        bid = kvg.kvg_deposit(store.h, src.h, 0, 0, nb, h)
+        kvg.kvg_graft(store.h, bid, dst.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY, h)
+        kf, vf = to_dev(np.ascontiguousarray(k[:, nb:])), to_dev(np.ascontiguousarray(v[:, nb:]))
+        pf = to_dev(syn.positions(nb, nf))
+        kvg.kvg_cache_append(dst.h, 0, kf.data_ptr(), vf.data_ptr(), pf.data_ptr(), nf, h)
+        qd = to_dev(q)
+        out = torch.empty_like(qd)
+        kvg.kvg_decode_attention(dst.h, -1, [0], qd.data_ptr(), w.n_q_heads, out.data_ptr(), scale, h)
+        return out, (src, store, dst, kd, vd, pos, kf, vf, pf, qd)
+
+    s0 = torch.cuda.Stream()
+    ref, keep0 = run(s0)
+    s0.synchronize()
+    ref = u16(ref)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    o1, keep1 = run(s1)
+    o2, keep2 = run(s2)
+    torch.cuda.synchronize()
+    for keep in (keep0, keep1, keep2):
+        kvg.kvg_sync(keep[2].h)
+    assert np.array_equal(u16(o1), ref) and np.array_equal(u16(o2), ref)
+    for l in range(w.n_layers):
+        compare_decode(oracle, ref[l, 0], oracle.gqa_decode(q[l, 0], k[l], v[l], scale), what=f"two streams l {l}")
