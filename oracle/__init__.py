@@ -180,9 +180,14 @@ def bf16_rne(x) -> np.ndarray:
 
 
 def bf16_to_f64(b) -> np.ndarray:
-    """bf16 bits -> exact fp64 value."""
+    """bf16 bits -> exact fp64 value.
+
+    Signalling-NaN patterns become quiet NaNs in the widening cast; numpy
+    reports that as an invalid-value warning, which is expected here.
+    """
     b = np.asarray(b, np.uint16)
-    return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    with np.errstate(invalid="ignore"):
+        return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
 
 
 def rope_rotate_rows(x: np.ndarray, delta: float, theta: float, style: int = 0) -> np.ndarray:
