@@ -88,7 +88,7 @@ def test_gpu_plain_digest_matches_fips_examples(spec, msg, digest):
 
 
 @pytest.mark.gpu
-def test_gpu_tiny_ragged_case_matches_golden(oracle):
+def test_gpu_tiny_ragged_case_matches_golden(oracle, tmp_path):
     from kvg_testlib import append, compare_decode, decode, need_gpu, tables
     import kvg_synth as syn
     kvg = need_gpu()
@@ -104,6 +104,16 @@ def test_gpu_tiny_ragged_case_matches_golden(oracle):
     bid = kvg.kvg_deposit(store.h, src.h, 0, 0, g.N_BLOCK)
     blk = kvg.kvg_store_export(store.h, bid)
     assert hashlib.sha256(blk).hexdigest() == case["block_sha256"]
+    # the block file written on this machine holds the bytes whose SHA-256
+    # the oracle computed on another one (Sec. 4.11: a block copied between
+    # machines is checked by its digest), and loads back with every digest
+    # checked
+    path = str(tmp_path / "golden_block.kvg")
+    kvg.kvg_store_save(store.h, bid, path)
+    with open(path, "rb") as f:
+        assert hashlib.sha256(f.read()).hexdigest() == case["block_sha256"]
+    host = kvg.Store(dims, kvg.KVG_RESIDENCY_PINNED_HOST, 1 << 26)
+    assert kvg.kvg_store_export(host.h, kvg.kvg_store_load(host.h, path, kvg.KVG_GRAFT_VERIFY)) == blk
 
     dst = kvg.Cache(dims, 8, 1, 64)
     kvg.kvg_graft(store.h, bid, dst.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
