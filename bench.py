@@ -453,6 +453,9 @@ def run_kvg(args, rank, world):
                "ms_per_step": round(e2e_ms, 3),
                "schedule": ("verified host-store graft in chunks; decode split: fresh rows during the graft, "
                             "each chunk's rows as it lands") if split else "verified host-store graft, then the decode",
+               "inputs": ("host to device each step: the stored block (pinned-host store) and the query; "
+                          "device to host: the output; the fresh rows stay in HBM (the model's own prefill "
+                          "writes them on the GPU)"),
                "h2d_bytes_per_step": int(blk_read + st.q.numel() * 2),
                "d2h_bytes_per_step": int(st.out.numel() * 2),
                "host_graft_gbs": None}
