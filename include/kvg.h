@@ -508,7 +508,10 @@ kvg_status kvg_decode_attention_noalloc(kvg_cache *cache, int32_t layer, const i
  * KVG_SHA256_PAGED: n must be a multiple of page_bytes; out[32 * i] = the
  *   two-level digest of page i = bytes[i * page_bytes, (i+1) * page_bytes).
  * bytes and out are device pointers (or pinned host memory the GPU can
- * reach).  Uses the library's per-device scratch (leaf digests). */
+ * reach).  Paged calls use the library's per-device scratch (leaf digests):
+ * each one's stream first waits for the previous paged call on the device,
+ * so calls on different streams run one after another on the GPU, in the
+ * order they were made (calls from several host threads take a lock). */
 kvg_status kvg_digest(const void *bytes, uint64_t n, int32_t mode, uint64_t page_bytes,
                       uint8_t *out, void *stream);
 

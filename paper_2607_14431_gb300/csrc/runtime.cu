@@ -2063,6 +2063,10 @@ namespace {
 std::mutex g_digest_mu;
 Scratch g_digest_leaf[64];
 DevStatus *g_digest_status[64] = {};
+// Paged digests share the device's leaf scratch: each call's stream waits for
+// the previous call's last kernel (recorded here), so calls on different
+// streams run one after the other on the GPU instead of racing on it.
+cudaEvent_t g_digest_done[64] = {};
 }  // namespace
 
 extern "C" kvg_status kvg_digest(const void *bytes, uint64_t n, int32_t mode, uint64_t page_bytes, uint8_t *out,
@@ -2088,11 +2092,20 @@ extern "C" kvg_status kvg_digest(const void *bytes, uint64_t n, int32_t mode, ui
         KVG_CUDA(cudaMalloc(&g_digest_status[dev], sizeof(DevStatus)));
         KVG_CUDA(cudaMemset(g_digest_status[dev], 0, sizeof(DevStatus)));
     }
+    if (!g_digest_done[dev]) {
+        KVG_CUDA(cudaEventCreateWithFlags(&g_digest_done[dev], cudaEventDisableTiming));
+    } else {
+        const size_t need = (size_t)n_pages * m * 32;
+        // a larger scratch replaces the old one: the previous call must be done with it
+        if (need > g_digest_leaf[dev].cap) KVG_CUDA(cudaEventSynchronize(g_digest_done[dev]));
+        KVG_CUDA(cudaStreamWaitEvent(st, g_digest_done[dev], 0));
+    }
     KVG_CUDA(g_digest_leaf[dev].ensure((size_t)n_pages * m * 32));
     PageSource src{static_cast<const uint8_t *>(bytes), page_bytes, nullptr, 1, 0};
     uint32_t *leaf = static_cast<uint32_t *>(g_digest_leaf[dev].ptr);
     KVG_CUDA(launch_sha256_leaves(src, n_pages, leaf, sm_count(dev), st));
     KVG_CUDA(launch_sha256_pages(leaf, n_pages, m, out, nullptr, g_digest_status[dev], -1, st));
+    KVG_CUDA(cudaEventRecord(g_digest_done[dev], st));
     return KVG_OK;
 }
 

@@ -481,3 +481,28 @@ def test_two_caches_on_two_streams_match_serial(oracle):
     assert np.array_equal(u16(o1), ref) and np.array_equal(u16(o2), ref)
     for l in range(w.n_layers):
         compare_decode(oracle, ref[l, 0], oracle.gqa_decode(q[l, 0], k[l], v[l], scale), what=f"two streams l {l}")
+
+
+@pytest.mark.gpu
+def test_paged_digests_on_two_streams_match_the_oracle(oracle):
+    """Paged digests share the device's leaf scratch: two calls launched
+    back to back on two streams (the second larger than the first, so the
+    scratch may have to grow) each give the oracle's page digests."""
+    kvg = need_gpu()
+    pb = 262144
+    rng = np.random.default_rng(77)
+    sizes = (128, 256)  # pages of 256 KiB
+    host = [rng.integers(0, 256, n * pb, dtype=np.uint8) for n in sizes]
+    want = [oracle.page_digests(h, pb) for h in host]
+    bufs = [torch.from_numpy(h).cuda() for h in host]
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    for rep in range(3):
+        outs = [torch.zeros(n * 32, dtype=torch.uint8, device="cuda") for n in sizes]
+        torch.cuda.synchronize()
+        order = (0, 1) if rep % 2 == 0 else (1, 0)
+        for i in order:
+            kvg.kvg_digest(bufs[i].data_ptr(), bufs[i].numel(), kvg.KVG_SHA256_PAGED, pb, outs[i].data_ptr(),
+                           streams[i])
+        torch.cuda.synchronize()
+        for i, n in enumerate(sizes):
+            assert np.array_equal(outs[i].cpu().numpy().reshape(n, 32), want[i]), (rep, i)
