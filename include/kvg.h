@@ -421,7 +421,11 @@ kvg_status kvg_verify(kvg_store *store, uint64_t block_id, kvg_cache *cache, int
  * token index, never on physical page placement, so results are bitwise
  * reproducible and identical for grafted and freshly written rows.
  * n_q_heads must be a multiple of n_kv_heads with group size in {1, 2, 4, 8}
- * and group * head_dim <= 512.  B <= 4096. */
+ * and group * head_dim <= 512.  B <= 4096.
+ * The split-K partials live in per-cache scratch shared by every decode of
+ * the cache (this call and kvg_decode_attention_range): a decode enqueued on
+ * another stream than the previous one first waits on the GPU for that one,
+ * so decodes of one cache on several streams run one after another. */
 kvg_status kvg_decode_attention(kvg_cache *cache, int32_t layer, const int32_t *seq_ids,
                                 int32_t B, const void *q, int32_t n_q_heads, void *out,
                                 float scale, void *stream);

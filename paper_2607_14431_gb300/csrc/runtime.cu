@@ -750,6 +750,12 @@ struct kvg_cache {
     std::vector<int32_t> n_slots;
     std::vector<int32_t> layer_window;  // per layer: 0 = global attention, W > 0 = last W tokens
     Scratch leaf, part_o, part_ml;
+    // the split-K partials are shared by every decode of the cache: a decode
+    // on another stream than the previous one waits for that one's last
+    // kernel (part_ev, recorded after each decode) instead of racing on them
+    cudaEvent_t part_ev = nullptr;
+    cudaStream_t part_stream = nullptr;
+    bool part_used = false;
     CUtensorMap pool_map;  // decode kernel's 2-D view of the pool
     // library stream and events for hashing a host-store graft's pages while
     // the next pages still cross the host link (made on first use)
@@ -974,6 +980,7 @@ extern "C" void kvg_cache_destroy(kvg_cache *c) {
         if (e) cudaEventDestroy(e);
     if (c->aux) cudaStreamDestroy(c->aux);
     if (c->batch_ev) cudaEventDestroy(c->batch_ev);
+    if (c->part_ev) cudaEventDestroy(c->part_ev);
     if (c->batch_host) cudaFreeHost(c->batch_host);
     c->batch_dev.release();
     if (c->pool) cudaFree(c->pool);
@@ -2000,6 +2007,8 @@ static kvg_status decode_impl(const char *what, kvg_cache *c, int32_t layer, con
     kvg_status r = plan_decode(c, layer, seq_ids, B, &plan, &max_units, page_begin, page_end);
     if (r != KVG_OK) return r;
     const size_t slots = (size_t)max_units + (size_t)w_max;
+    if (!c->part_ev) KVG_CUDA(cudaEventCreateWithFlags(&c->part_ev, cudaEventDisableTiming));
+    if (c->part_used && st != c->part_stream) KVG_CUDA(cudaStreamWaitEvent(st, c->part_ev, 0));
     KVG_CUDA(c->part_o.ensure(slots * G * d.head_dim * sizeof(float)));
     KVG_CUDA(c->part_ml.ensure(slots * G * sizeof(float2)));
     for (DecodeParams &p : plan) {
@@ -2017,6 +2026,9 @@ static kvg_status decode_impl(const char *what, kvg_cache *c, int32_t layer, con
         KVG_CUDA(launch_decode(d.head_dim, G, fp8, p, c->pool_map, st));
         KVG_CUDA(launch_combine(d.head_dim, G, p, st));
     }
+    KVG_CUDA(cudaEventRecord(c->part_ev, st));
+    c->part_stream = st;
+    c->part_used = true;
     return KVG_OK;
 }
 

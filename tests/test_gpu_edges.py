@@ -506,3 +506,51 @@ def test_paged_digests_on_two_streams_match_the_oracle(oracle):
         torch.cuda.synchronize()
         for i, n in enumerate(sizes):
             assert np.array_equal(outs[i].cpu().numpy().reshape(n, 32), want[i]), (rep, i)
+
+
+@pytest.mark.gpu
+def test_decodes_of_one_cache_on_two_streams_match_serial(oracle):
+    """Decodes of one cache share its split-K scratch: a long decode (32
+    sequences of 4,096 rows, two layers: 512 MiB of K/V) and a second one
+    with other queries and the batch rows in reverse order, launched back to
+    back on two streams, each give the bytes they give one after the other
+    on one stream."""
+    kvg = need_gpu()
+    w = geometry("d256")
+    P = w.page_size
+    dims = dims_for(kvg, w)
+    n_seq, n = 32, 64 * P
+    k, v = _kv(w, n, 0x31)
+    cache = kvg.Cache(dims, n_seq * (n // P), n_seq, n)
+    kd, vd = to_dev(k), to_dev(v)
+    pos = to_dev(syn.positions(0, n))
+    h = torch.cuda.current_stream().cuda_stream
+    for s in range(n_seq):
+        kvg.kvg_cache_append(cache.h, s, kd.data_ptr(), vd.data_ptr(), pos.data_ptr(), n, h)
+    qa = syn.as_u16(syn.queries(w, w.n_layers, n_seq, 0x32))
+    qb = syn.as_u16(syn.queries(w, w.n_layers, n_seq, 0x33))
+    qa_d, qb_d = to_dev(qa), to_dev(qb)
+    seqs_a, seqs_b = list(range(n_seq)), list(range(n_seq))[::-1]
+    scale = 1.0 / math.sqrt(w.head_dim)
+
+    def dec(q_d, seqs, stream):
+        out = torch.empty_like(q_d)
+        kvg.kvg_decode_attention(cache.h, -1, seqs, q_d.data_ptr(), w.n_q_heads, out.data_ptr(), scale,
+                                 stream.cuda_stream)
+        return out
+
+    torch.cuda.synchronize()
+    s0 = torch.cuda.Stream()
+    ra, rb = dec(qa_d, seqs_a, s0), dec(qb_d, seqs_b, s0)
+    s0.synchronize()
+    ref_a, ref_b = u16(ra), u16(rb)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    for rep in range(3):
+        oa = dec(qa_d, seqs_a, s1)
+        ob = dec(qb_d, seqs_b, s2)
+        torch.cuda.synchronize()
+        assert np.array_equal(u16(oa), ref_a) and np.array_equal(u16(ob), ref_b), rep
+    kvg.kvg_sync(cache.h)
+    for l in range(w.n_layers):
+        compare_decode(oracle, ref_a[l, 0], oracle.gqa_decode(qa[l, 0], k[l], v[l], scale), what=f"stream a l {l}")
+        compare_decode(oracle, ref_b[l, 0], oracle.gqa_decode(qb[l, 0], k[l], v[l], scale), what=f"stream b l {l}")
