@@ -280,7 +280,10 @@ kvg_status kvg_cache_append_batch(kvg_cache *cache, const int32_t *seq_ids, int3
  * fills and position tags: the serving slot is empty again, ready for the
  * next graft into a fresh context (Sec. 3.2; Sec. 4.4, where the movable
  * window swaps which block is resident in the live prefix).  Enqueued on
- * `stream`; the host bookkeeping changes at once. */
+ * `stream`; the host bookkeeping changes at once, so the next graft or
+ * append may be given these pages: work on other streams that still reads
+ * them must be ordered before that call's stream (an event), as on one
+ * stream it is by itself. */
 kvg_status kvg_cache_release(kvg_cache *cache, int32_t seq, void *stream);
 
 /* ----------------------------------------------------------- deposit -- */
