@@ -201,6 +201,18 @@ kvg_status kvg_store_save(kvg_store *store, uint64_t block_id, const char *path)
  * bounce buffers, each chunk's copy to HBM overlapping the next reads. */
 kvg_status kvg_store_load(kvg_store *store, const char *path, uint32_t flags, uint64_t *block_id_out);
 
+/* Readies a pinned-host store's block for a later graft (Sec. 4.4's restore
+ * from a deep store, where the next block to restore is known ahead): enqueues
+ * on `stream` one 4-byte read per host page of the block, which makes the GPU
+ * resolve the address translations of all its pages.  A graft reads a block
+ * at the host link's rate only when they are resolved; the GPU keeps those of
+ * the last several GB of host memory it touched, so a graft of a block not
+ * read recently otherwise takes up to about three times as long.  Issue it
+ * on a stream other than the graft's while the previous graft runs (one
+ * small read per host page).  No effect on HBM and cache-pool stores.
+ * Errors: KVG_ERR_ARG (null store), KVG_ERR_NOT_FOUND. */
+kvg_status kvg_store_prefetch(kvg_store *store, uint64_t block_id, void *stream);
+
 /* ---------------------------------------------------------------- cache -- */
 
 /* A paged KV cache on `device`: the "fresh inference context" a block is

@@ -290,6 +290,10 @@ cudaError_t launch_append_batch(const AppendBatchParams &p, int n_sm, cudaStream
 cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_write_header(const HeaderParams &p, cudaStream_t s);
 cudaError_t launch_alias(const AliasParams &p, int n_sm, cudaStream_t s);
+// One 4-byte load per `stride` bytes of [base, base + bytes) (base 4-byte
+// aligned, stride a multiple of 4): resolves the GPU's address translations
+// of the pages of a block in pinned host memory ahead of its graft.
+cudaError_t launch_touch(const uint8_t *base, uint64_t bytes, uint32_t stride, int n_sm, cudaStream_t s);
 // A kernel whose mbarrier nothing completes: its bounded wait gives up after
 // limit_ns and records KVG_ERR_DEVICE_CHECK (detail 3) in `status`.
 cudaError_t launch_wait_selftest(DevStatus *status, uint64_t limit_ns, cudaStream_t s);

@@ -550,6 +550,20 @@ __global__ void __launch_bounds__(256) alias_kernel(const AliasParams p) {
     }
 }
 
+// One 4-byte load per `stride` bytes of [base, base + bytes): each load makes
+// the GPU resolve the address translation of one host page, so a later graft
+// that streams the block finds them resolved.  The values are discarded
+// (sink is written only if the loads' xor hits a constant, and the launcher
+// passes null).
+__global__ void __launch_bounds__(256) touch_kernel(const uint8_t *base, uint64_t n_loads, uint32_t stride,
+                                                    uint32_t *sink) {
+    uint32_t acc = 0;
+    for (uint64_t i = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x; i < n_loads;
+         i += (uint64_t)gridDim.x * blockDim.x)
+        acc ^= __ldcv(reinterpret_cast<const uint32_t *>(base + i * stride));
+    if (acc == 0x9e3779b9u && sink) *sink = acc;
+}
+
 __global__ void wait_selftest_kernel(DevStatus *status, uint64_t limit_ns) {
     __shared__ __align__(8) uint64_t bar;
     if (threadIdx.x == 0) {
@@ -948,6 +962,14 @@ cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s) {
 
 cudaError_t launch_alias(const AliasParams &p, int n_sm, cudaStream_t s) {
     alias_kernel<<<grid_for(p.n_tokens > p.pids.n ? p.n_tokens : p.pids.n, 256, n_sm, 1), 256, 0, s>>>(p);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_touch(const uint8_t *base, uint64_t bytes, uint32_t stride, int n_sm, cudaStream_t s) {
+    const uint64_t n_loads = bytes / stride + (bytes % stride >= 4 ? 1 : 0);  // every load fits in [base, +bytes)
+    if (n_loads == 0) return cudaSuccess;
+    touch_kernel<<<grid_for((int64_t)n_loads, 256, n_sm, 2), 256, 0, s>>>(base, n_loads, stride, nullptr);
     count_launches(1);
     return cudaGetLastError();
 }

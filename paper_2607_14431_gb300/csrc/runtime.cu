@@ -380,6 +380,20 @@ extern "C" kvg_status kvg_store_block_info(kvg_store *s, uint64_t id, kvg_block_
     return KVG_OK;
 }
 
+extern "C" kvg_status kvg_store_prefetch(kvg_store *s, uint64_t id, void *stream) {
+    Trace trace_("kvg_store_prefetch");
+    if (!s) return fail(KVG_ERR_ARG, "null store");
+    if (id >= s->blocks.size()) return fail(KVG_ERR_NOT_FOUND, "no block %llu", (unsigned long long)id);
+    if (s->residency != KVG_RESIDENCY_PINNED_HOST) return KVG_OK;  // HBM and pool blocks need no translations
+    const auto &b = s->blocks[id];
+    DeviceGuard g(s->device);
+    // one load per host page (the system page size, at least 4 KiB): the
+    // block starts 4 KiB-aligned in its slab and its size is a multiple of 16
+    static const uint32_t stride = (uint32_t)std::max<long>(4096, sysconf(_SC_PAGESIZE));
+    KVG_CUDA(launch_touch(b.dev, b.lay.total, stride, s->n_sm, static_cast<cudaStream_t>(stream)));
+    return KVG_OK;
+}
+
 // Hashes every page of a block (contiguous pages region) and its block digest
 // against `expected` digests (nullable: then writes them), on stream st.
 static kvg_status hash_block(kvg_store *s, uint8_t *blk_dev, const BlockLayout &lay, bool verify,

@@ -76,6 +76,7 @@ _SIGNATURES = {
     "kvg_store_export": ([_vp, _u64, _vp, _u64], _i32),
     "kvg_store_save": ([_vp, _u64, ctypes.c_char_p], _i32),
     "kvg_store_load": ([_vp, ctypes.c_char_p, _u32, _P(_u64)], _i32),
+    "kvg_store_prefetch": ([_vp, _u64, _vp], _i32),
     "kvg_cache_create": ([_P(kvg_dims), _i32, _i32, _i32, _i32, _P(_vp)], _i32),
     "kvg_cache_destroy": ([_vp], None),
     "kvg_cache_set_free_order": ([_vp, _vp, _i32], _i32),
@@ -195,6 +196,10 @@ def kvg_store_load(store, path: str, flags: int = 0) -> int:
     out = _u64()
     _check(lib().kvg_store_load(store, os.fsencode(path), flags, ctypes.byref(out)))
     return out.value
+
+
+def kvg_store_prefetch(store, block_id: int, stream=None):
+    _check(lib().kvg_store_prefetch(store, block_id, _stream(stream)))
 
 
 def kvg_cache_create(dims: kvg_dims, n_pages: int, max_seqs: int, max_slots: int, device: int = 0):

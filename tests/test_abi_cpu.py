@@ -39,6 +39,7 @@ def test_host_checks_reject_bad_geometry_without_a_gpu(lib):
     assert lib.kvg_store_create(ctypes.byref(good), 7, 1 << 20, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
     assert lib.kvg_store_create(None, 0, 1 << 20, 0, ctypes.byref(h)) == kvg.KVG_ERR_ARG
     assert lib.kvg_graft(None, 0, None, 0, -1, 0, 0, None, None) == kvg.KVG_ERR_ARG
+    assert lib.kvg_store_prefetch(None, 0, None) == kvg.KVG_ERR_ARG
     ends, nc = (ctypes.c_int32 * 2)(), ctypes.c_int32(-1)
     no_events = (ctypes.c_void_p * 2)()
     assert lib.kvg_graft_chunked(None, 0, None, 0, -1, 0, 0, None, None, None, 2, ends,

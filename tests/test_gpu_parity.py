@@ -811,6 +811,30 @@ def test_sync_times_out_while_the_stream_is_busy_then_succeeds():
     kvg.kvg_sync(cache.h, s, 60.0)
 
 
+@pytest.mark.parametrize("residency", [0, 1])
+def test_prefetch_then_graft_is_bit_exact(oracle, residency):
+    """kvg_store_prefetch only reads: a pinned-host block prefetched on a
+    side stream, then grafted on another, restores the oracle's bytes; on an
+    HBM store the call does nothing; an unknown block is KVG_ERR_NOT_FOUND."""
+    kvg = need_gpu()
+    w = geometry("d128")
+    s = _build_both(kvg, oracle, w, 300, 0, residency=residency, seed=131)
+    side, main = torch.cuda.Stream(), torch.cuda.Stream()
+    ev = torch.cuda.Event()
+    kvg.kvg_store_prefetch(s["store"].h, s["bid"], side)
+    ev.record(side)
+    main.wait_event(ev)
+    kvg.kvg_graft(s["store"].h, s["bid"], s["dst"].h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY, main)
+    main.synchronize()
+    kvg.kvg_sync(s["dst"].h, main)
+    s["ocache"].graft(0, s["oblk"])
+    assert np.array_equal(pool_u16(s["dst"], w), s["ocache"].pool)
+    assert kvg.kvg_store_export(s["store"].h, s["bid"]) == s["oblk"].serialize()
+    with pytest.raises(kvg.KvgError) as e:
+        kvg.kvg_store_prefetch(s["store"].h, s["bid"] + 1, side)
+    assert e.value.status == kvg.KVG_ERR_NOT_FOUND
+
+
 def test_block_files_round_trip_and_are_verified(oracle, tmp_path):
     # a block is a plain file: saved, copied, loaded elsewhere with its digests
     # checked (Sec. 4.4, Sec. 4.11)
