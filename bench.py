@@ -1105,7 +1105,8 @@ def run_workloads(args):
     plan = [("tiny", dict(steps=500, warmup=5), ("graft_verify", "decode")),
             ("31b", dict(steps=5, warmup=3, layers=args.workload_31b_layers), ("relocate", "decode")),
             ("batched", dict(steps=3, warmup=3), ("graft", "decode_steps")),
-            ("deep", dict(steps=syn.DEEP_GRAFTS, warmup=5), ("host_graft", "host_graft_gpu", "decode"))]
+            ("deep", dict(steps=syn.DEEP_GRAFTS, warmup=5),
+             ("host_graft", "host_graft_no_prefetch", "host_graft_gpu", "decode"))]
     for name, kw, keep in plan:
         try:
             line = measure_other(kvg, device, name, kw["steps"], kw["warmup"], kw.get("layers", 0))
