@@ -267,6 +267,223 @@ __device__ __forceinline__ void store_state(uint32_t *out, const uint32_t st[8])
     o[1] = make_uint4(st[4], st[5], st[6], st[7]);
 }
 
+// ---- two-warp form, for launches too small to fill the GPU ---------------
+// When there are few chains, each one's latency decides, and a thread that
+// both expands the message schedule and runs the rounds issues ~27
+// instructions a round from one warp.  Here a 64-thread CTA works on 32
+// chains (lane c of both warps on chain c): warp 1 loads each chain's next
+// 64-byte block, expands its schedule and leaves K[t] + W[t] in shared
+// memory; warp 0 runs the 64 rounds from there.  The rounds' warp then
+// issues ~18 instructions a round on its own scheduler: ~1,775 cycles per
+// block against ~2,480 (a probe over 256 blocks per chain, same digests).
+// Two buffers change hands through named barriers: 1 + b (buffer b full,
+// warp 1 arrives, warp 0 waits) and 3 + b (buffer b free again, warp 0
+// arrives, warp 1 waits).  Both warps run the same number of blocks, with
+// every lane taking part (lanes past the last chain hash zeros and store
+// nothing), so every arrival meets its wait.
+constexpr int kSplitChains = 32;
+
+__device__ __forceinline__ void bar_sync_pair(int id) { asm volatile("bar.sync %0, 64;" ::"r"(id) : "memory"); }
+__device__ __forceinline__ void bar_arrive_pair(int id) { asm volatile("bar.arrive %0, 64;" ::"r"(id) : "memory"); }
+
+// Warp 1: the message schedule of block w plus the round constants, into
+// column `lane` of kw[64][32] (plain ALU arithmetic: this warp's scheduler
+// has nothing else to issue).
+__device__ __forceinline__ void split_expand(uint32_t (*kw)[kSplitChains], uint32_t w[16], int lane) {
+#pragma unroll
+    for (int t = 0; t < 64; ++t) {
+        uint32_t wt;
+        if (t < 16) {
+            wt = w[t];
+        } else {
+            const uint32_t w15 = w[(t - 15) & 15], w2 = w[(t - 2) & 15];
+            const uint32_t s0 = rotr(w15, 7) ^ rotr(w15, 18) ^ (w15 >> 3);
+            const uint32_t s1 = rotr(w2, 17) ^ rotr(w2, 19) ^ (w2 >> 10);
+            wt = w[t & 15] = w[t & 15] + s0 + w[(t - 7) & 15] + s1;
+        }
+        kw[t][lane] = wt + kK[t];
+    }
+}
+
+// Warp 0: the 64 rounds of one block from kw (FIPS 180-4 sec. 6.2.2 step 3,
+// with h + K[t] + W[t] taken whole from shared memory) and the feed-forward.
+// The additions off the last step go to the FMA pipe (fadd), so the ALU pipe
+// carries the rotations and logic.
+__device__ __forceinline__ void split_rounds(uint32_t st[8], const uint32_t (*kw)[kSplitChains], int lane,
+                                             uint32_t one) {
+    uint32_t a = st[0], b = st[1], c = st[2], d = st[3], e = st[4], f = st[5], g = st[6], h = st[7];
+#pragma unroll
+    for (int t = 0; t < 64; ++t) {
+        const uint32_t k = kw[t][lane];
+        const uint32_t S1 = rotr(e, 6) ^ rotr(e, 11) ^ rotr(e, 25);
+        const uint32_t ch = (e & f) ^ (~e & g);
+        const uint32_t S0 = rotr(a, 2) ^ rotr(a, 13) ^ rotr(a, 22);
+        const uint32_t maj = (a & b) ^ (a & c) ^ (b & c);
+        const uint32_t hkc = fadd(fadd(h, k, one), ch, one);  // h + K[t] + W[t] + Ch
+        const uint32_t T1 = fadd(hkc, S1, one);
+        const uint32_t ne = fadd(fadd(d, hkc, one), S1, one);  // d + T1
+        h = g;
+        g = f;
+        f = e;
+        e = ne;
+        d = c;
+        c = b;
+        b = a;
+        a = T1 + S0 + maj;
+    }
+    st[0] += a;
+    st[1] += b;
+    st[2] += c;
+    st[3] += d;
+    st[4] += e;
+    st[5] += f;
+    st[6] += g;
+    st[7] += h;
+}
+
+// Warp 0's side of a chain of n_blocks blocks: state from H0 to the digest.
+__device__ __forceinline__ void split_consume(uint32_t st[8], uint32_t (*kw)[64][kSplitChains], int n_blocks,
+                                              int lane, uint32_t one) {
+    init_state(st);
+    for (int blk = 0; blk < n_blocks; ++blk) {
+        const int buf = blk & 1;
+        bar_sync_pair(1 + buf);
+        split_rounds(st, kw[buf], lane, one);
+        if (blk + 2 < n_blocks) bar_arrive_pair(3 + buf);
+    }
+}
+
+// Warp 1 hands over block blk (its 16 words in w) through buffer blk & 1.
+__device__ __forceinline__ void split_hand_over(uint32_t (*kw)[64][kSplitChains], uint32_t w[16], int blk, int lane) {
+    const int buf = blk & 1;
+    if (blk >= 2) bar_sync_pair(3 + buf);
+    split_expand(kw[buf], w, lane);
+    __threadfence_block();
+    bar_arrive_pair(1 + buf);
+}
+
+// The padding block of a message of `bytes` bytes (a multiple of 64).
+__device__ __forceinline__ void padding_block(uint32_t w[16], uint64_t bytes) {
+#pragma unroll
+    for (int q = 0; q < 16; ++q) w[q] = 0;
+    w[0] = 0x80000000u;
+    const uint64_t bits = bytes * 8ull;
+    w[14] = (uint32_t)(bits >> 32);
+    w[15] = (uint32_t)bits;
+}
+
+// Warp 1's side of a whole 4 KiB leaf at v (nullptr: zeros), also written to
+// o when COPY (the bytes written are the bytes hashed): 64 data blocks, the
+// next two in flight, then the padding block.
+template <bool COPY>
+__device__ __forceinline__ void split_produce_leaf(uint32_t (*kw)[64][kSplitChains], const uint4 *v, uint4 *o,
+                                                   int lane) {
+    constexpr int kData = (int)(kLeafBytes / 64);
+    uint4 n1[4], n2[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        n1[q] = v ? __ldg(v + q) : make_uint4(0, 0, 0, 0);
+        n2[q] = v ? __ldg(v + 4 + q) : make_uint4(0, 0, 0, 0);
+    }
+    for (int blk = 0; blk < kData; ++blk) {
+        uint4 x[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            x[q] = n1[q];
+            n1[q] = n2[q];
+        }
+        if (v && blk + 2 < kData) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) n2[q] = __ldg(v + 4 * (blk + 2) + q);
+        }
+        if (COPY && o) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) __stcs(o + 4 * blk + q, x[q]);
+        }
+        uint32_t w[16];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            w[4 * q + 0] = bswap(x[q].x);
+            w[4 * q + 1] = bswap(x[q].y);
+            w[4 * q + 2] = bswap(x[q].z);
+            w[4 * q + 3] = bswap(x[q].w);
+        }
+        split_hand_over(kw, w, blk, lane);
+    }
+    uint32_t w[16];
+    padding_block(w, kLeafBytes);
+    split_hand_over(kw, w, kData, lane);
+}
+
+constexpr int kSplitLeafBlocks = (int)(kLeafBytes / 64) + 1;
+
+// graft_verify_kernel's work in the two-warp form, for pages made of whole
+// 4 KiB leaves and launches of at most one such CTA per SM.
+__global__ void __launch_bounds__(64) graft_verify_split_kernel(const GraftParams p, int64_t leaves_per_page,
+                                                                uint32_t *__restrict__ out, uint32_t one) {
+    __shared__ __align__(16) uint32_t kw[2][64][kSplitChains];
+    graft_metadata(p);
+    const int lane = threadIdx.x & 31;
+    const uint64_t page_bytes = p.page_bytes;
+    const int64_t n_leaves = (int64_t)p.n_layers * 2 * p.npb * leaves_per_page;
+    const int64_t idx = (int64_t)blockIdx.x * kSplitChains + lane;
+    const bool valid = idx < n_leaves;
+    const int64_t page_u = idx / leaves_per_page;
+    const int64_t i = idx - page_u * leaves_per_page;
+    const int64_t lkv = page_u / p.npb;
+    const int64_t jj = page_u - lkv * p.npb;
+    const int64_t block_page = lkv * p.block_pages + p.page_base + jj;
+    if (threadIdx.x >= 32) {
+        const uint64_t off = (uint64_t)i * kLeafBytes;
+        const uint4 *v = valid ? reinterpret_cast<const uint4 *>(p.src + (uint64_t)block_page * page_bytes + off)
+                               : nullptr;
+        uint4 *o = valid ? reinterpret_cast<uint4 *>(p.pool + ((uint64_t)lkv * p.pool_pages +
+                                                               (uint64_t)p.pids.pid[jj]) * page_bytes + off)
+                         : nullptr;
+        split_produce_leaf<true>(kw, v, o, lane);
+    } else {
+        uint32_t st[8];
+        split_consume(st, kw, kSplitLeafBlocks, lane, one);
+        if (valid) store_state(out + (block_page * leaves_per_page + i) * 8, st);
+    }
+}
+
+// sha256_leaves_kernel's work in the two-warp form (whole 4 KiB leaves).
+__global__ void __launch_bounds__(64) sha256_leaves_split_kernel(const PageSource src, int64_t n_pages,
+                                                                 int64_t leaves_per_page,
+                                                                 uint32_t *__restrict__ out, uint32_t one) {
+    __shared__ __align__(16) uint32_t kw[2][64][kSplitChains];
+    const int lane = threadIdx.x & 31;
+    const int64_t idx = (int64_t)blockIdx.x * kSplitChains + lane;
+    const bool valid = idx < n_pages * leaves_per_page;
+    const int64_t p = idx / leaves_per_page;
+    const int64_t i = idx - p * leaves_per_page;
+    bool in_range = valid;
+    if (valid && src.pid) {  // page ids come from a device page table: never read outside the pool
+        const int32_t pid = src.pid[p - (p / src.npb) * src.npb];
+        in_range = pid >= 0 && pid < src.plane_pages;
+    }
+    if (threadIdx.x >= 32) {
+        const uint4 *v = in_range ? reinterpret_cast<const uint4 *>(page_addr(src, p) + (uint64_t)i * kLeafBytes)
+                                  : nullptr;
+        split_produce_leaf<false>(kw, v, nullptr, lane);
+    } else {
+        uint32_t st[8];
+        split_consume(st, kw, kSplitLeafBlocks, lane, one);
+        if (!valid) return;
+        if (!in_range) {
+#pragma unroll
+            for (int w = 0; w < 8; ++w) st[w] = 0u;  // no digest of any page: reported as a mismatch
+        }
+        int64_t po = p;
+        if (src.pid && src.out_plane_stride) {
+            const int64_t plane = p / src.npb;
+            po = plane * src.out_plane_stride + src.out_j0 + (p - plane * src.npb);
+        }
+        store_state(out + (po * leaves_per_page + i) * 8, st);
+    }
+}
+
 __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src, int64_t n_pages,
                                                             int64_t leaves_per_page,
                                                             uint32_t *__restrict__ out, uint32_t one) {
@@ -361,6 +578,35 @@ __global__ void __launch_bounds__(128) graft_verify_kernel(const GraftParams p, 
     }
 }
 
+// Page p's digest (the state words, big-endian) written to out and/or
+// compared with expected; a mismatch is recorded in the status word.
+__device__ __forceinline__ void page_verdict(int64_t p, const uint32_t st[8], uint8_t *__restrict__ out,
+                                             const uint8_t *__restrict__ expected, DevStatus *status, int32_t seq) {
+    uint8_t dg[32];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        dg[4 * k + 0] = (uint8_t)(st[k] >> 24);
+        dg[4 * k + 1] = (uint8_t)(st[k] >> 16);
+        dg[4 * k + 2] = (uint8_t)(st[k] >> 8);
+        dg[4 * k + 3] = (uint8_t)st[k];
+    }
+    if (out) {
+#pragma unroll
+        for (int k = 0; k < 32; ++k) out[p * 32 + k] = dg[k];
+    }
+    if (expected) {
+        bool same = true;
+#pragma unroll
+        for (int k = 0; k < 32; ++k) same &= dg[k] == expected[p * 32 + k];
+        if (!same) {
+            const int slot = atomicAdd(&status->n_mismatch, 1);
+            if (slot < KVG_REPORT_MAX_PAGES) status->list[slot] = (int32_t)p;
+            status->seq = seq;
+            atomicCAS(&status->err, 0, (int32_t)KVG_ERR_DIGEST);
+        }
+    }
+}
+
 // Page digest from its leaf digests: the message is the leaf digests' bytes,
 // i.e. (big-endian) exactly the 8 state words of each leaf in order.
 __global__ void __launch_bounds__(128) sha256_pages_kernel(const uint32_t *__restrict__ leaf_words,
@@ -400,28 +646,60 @@ __global__ void __launch_bounds__(128) sha256_pages_kernel(const uint32_t *__res
         w[15] = (uint32_t)bits;
         compress<false>(st, w, one);
     }
-    uint8_t dg[32];
+    page_verdict(p, st, out, expected, status, seq);
+}
+
+// sha256_pages_kernel in the two-warp form: warp 1 feeds each page's leaf
+// digests (already big-endian words) and the final block.
+__global__ void __launch_bounds__(64) sha256_pages_split_kernel(const uint32_t *__restrict__ leaf_words,
+                                                                int64_t n_pages, int64_t m,
+                                                                uint8_t *__restrict__ out,
+                                                                const uint8_t *__restrict__ expected,
+                                                                DevStatus *status, int32_t seq, uint32_t one) {
+    __shared__ __align__(16) uint32_t kw[2][64][kSplitChains];
+    const int lane = threadIdx.x & 31;
+    const int64_t p = (int64_t)blockIdx.x * kSplitChains + lane;
+    const bool valid = p < n_pages;
+    const int64_t nwords = m * 8;
+    const int nfull = (int)(nwords / 16);
+    const int remw = (int)(nwords - (int64_t)nfull * 16);  // 0 or 8
+    if (threadIdx.x >= 32) {
+        const uint32_t *lw = leaf_words + (valid ? p : 0) * m * 8;
+        uint4 nx[4];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-        dg[4 * k + 0] = (uint8_t)(st[k] >> 24);
-        dg[4 * k + 1] = (uint8_t)(st[k] >> 16);
-        dg[4 * k + 2] = (uint8_t)(st[k] >> 8);
-        dg[4 * k + 3] = (uint8_t)st[k];
-    }
-    if (out) {
+        for (int q = 0; q < 4; ++q)
+            nx[q] = valid && nfull > 0 ? reinterpret_cast<const uint4 *>(lw)[q] : make_uint4(0, 0, 0, 0);
+        for (int blk = 0; blk < nfull; ++blk) {
+            uint4 x[4];
 #pragma unroll
-        for (int k = 0; k < 32; ++k) out[p * 32 + k] = dg[k];
-    }
-    if (expected) {
-        bool same = true;
+            for (int q = 0; q < 4; ++q) x[q] = nx[q];
+            if (valid && blk + 1 < nfull) {
 #pragma unroll
-        for (int k = 0; k < 32; ++k) same &= dg[k] == expected[p * 32 + k];
-        if (!same) {
-            const int slot = atomicAdd(&status->n_mismatch, 1);
-            if (slot < KVG_REPORT_MAX_PAGES) status->list[slot] = (int32_t)p;
-            status->seq = seq;
-            atomicCAS(&status->err, 0, (int32_t)KVG_ERR_DIGEST);
+                for (int q = 0; q < 4; ++q) nx[q] = reinterpret_cast<const uint4 *>(lw + (blk + 1) * 16)[q];
+            }
+            uint32_t w[16];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                w[4 * q + 0] = x[q].x;
+                w[4 * q + 1] = x[q].y;
+                w[4 * q + 2] = x[q].z;
+                w[4 * q + 3] = x[q].w;
+            }
+            split_hand_over(kw, w, blk, lane);
         }
+        uint32_t w[16];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) w[q] = 0;
+        for (int q = 0; q < remw; ++q) w[q] = valid ? lw[nfull * 16 + q] : 0u;
+        w[remw] = 0x80000000u;
+        const uint64_t bits = (uint64_t)m * 32ull * 8ull;
+        w[14] = (uint32_t)(bits >> 32);
+        w[15] = (uint32_t)bits;
+        split_hand_over(kw, w, nfull, lane);
+    } else {
+        uint32_t st[8];
+        split_consume(st, kw, nfull + 1, lane, one);
+        if (valid) page_verdict(p, st, out, expected, status, seq);
     }
 }
 
@@ -556,11 +834,34 @@ __global__ void __launch_bounds__(32) sha256_serial_kernel(const uint8_t *seg0, 
 
 }  // namespace
 
+// The two-warp form is used for pages of whole 4 KiB leaves when a launch has
+// at most one of its 32-chain CTAs per SM (leaves, 32 * n_sm) or four (page
+// digests, which read their input from L2); beyond that the one-warp forms
+// keep more chains going per SM.  KVG_SHA_NO_SPLIT=1 turns it off.
+static bool split_off() {
+    static const bool off = env_knob("KVG_SHA_NO_SPLIT", 0) > 0;
+    return off;
+}
+
+static int current_sm_count() {
+    static int cache[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    if (!cache[dev]) cudaDeviceGetAttribute(&cache[dev], cudaDevAttrMultiProcessorCount, dev);
+    return cache[dev];
+}
+
 cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_t *leaf_words,
                                  int n_sm, cudaStream_t s) {
     const int64_t m = (int64_t)((src.page_bytes + kLeafBytes - 1) / kLeafBytes);
     const int64_t n = n_pages * m;
     if (n == 0) return cudaSuccess;
+    if (!split_off() && src.page_bytes % kLeafBytes == 0 && n <= (int64_t)n_sm * kSplitChains) {
+        sha256_leaves_split_kernel<<<(int)((n + kSplitChains - 1) / kSplitChains), 64, 0, s>>>(src, n_pages, m,
+                                                                                             leaf_words, 1u);
+        count_launches(1);
+        return cudaGetLastError();
+    }
     int64_t grid = (n + 127) / 128;
     // One CTA per 128 leaves (no grid-stride cap by default): 4 CTAs of
     // 125 registers are resident per SM and the rest queue, which measured
@@ -576,6 +877,11 @@ cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int 
     const int64_t m = (int64_t)((p.page_bytes + kLeafBytes - 1) / kLeafBytes);
     const int64_t n = (int64_t)p.n_layers * 2 * p.npb * m;
     if (n == 0) return cudaSuccess;
+    if (!split_off() && p.page_bytes % kLeafBytes == 0 && n <= (int64_t)n_sm * kSplitChains) {
+        graft_verify_split_kernel<<<(int)((n + kSplitChains - 1) / kSplitChains), 64, 0, s>>>(p, m, leaf_words, 1u);
+        count_launches(1);
+        return cudaGetLastError();
+    }
     int64_t grid = (n + 127) / 128;
     // One CTA per 128 leaves (no grid-stride cap by default): four CTAs of
     // the register form (125 registers) or five of the ring form (96) are
@@ -601,6 +907,12 @@ cudaError_t launch_sha256_pages(const uint32_t *leaf_words, int64_t n_pages, int
                                 uint8_t *out, const uint8_t *expected, DevStatus *status,
                                 int32_t seq, cudaStream_t s) {
     if (n_pages == 0) return cudaSuccess;
+    if (!split_off() && n_pages <= (int64_t)current_sm_count() * 4 * kSplitChains) {
+        sha256_pages_split_kernel<<<(int)((n_pages + kSplitChains - 1) / kSplitChains), 64, 0, s>>>(
+            leaf_words, n_pages, leaves_per_page, out, expected, status, seq, 1u);
+        count_launches(1);
+        return cudaGetLastError();
+    }
     sha256_pages_kernel<<<(int)((n_pages + 127) / 128), 128, 0, s>>>(leaf_words, n_pages,
                                                                      leaves_per_page, out,
                                                                      expected, status, seq, 1u);
