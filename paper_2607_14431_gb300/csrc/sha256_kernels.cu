@@ -523,8 +523,9 @@ __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src
 // append the 12b step's window shortens (step 5.94 against 6.01 ms; alone
 // the same 3.12 ms; rings of two or four blocks, or six CTAs at 80
 // registers, measured slower in the step).  For smaller launches each leaf's
-// chain latency decides and the register form is faster (the tiny verified
-// graft 0.099 against 0.133 ms).
+// chain latency decides: the register form is faster there (the tiny
+// verified graft 0.099 against 0.133 ms), and the two-warp form faster still
+// for launches of up to 32 leaves per SM (0.071 ms).
 constexpr int kGraftVerifyRing = 3;
 __global__ void __launch_bounds__(128, 5) graft_verify_ring_kernel(const GraftParams p, int64_t leaves_per_page,
                                                                    uint32_t *__restrict__ out, uint32_t one) {
