@@ -520,9 +520,10 @@ kvg_status kvg_decode_attention_noalloc(kvg_cache *cache, int32_t layer, const i
 /* ------------------------------------------------------------- digest -- */
 
 /* SHA-256 (FIPS 180-4) on the GPU.
- * KVG_SHA256_PLAIN: out[32] = SHA-256 of bytes[0, n): one serial chain, run
- *   by one GPU thread (its 32-lane warp prefetches the message), about
- *   1.5 us per 64-byte block (~40 MB/s) — meant for short messages such as
+ * KVG_SHA256_PLAIN: out[32] = SHA-256 of bytes[0, n): one serial chain (one
+ *   warp expands each block's message schedule while another runs the
+ *   rounds when bytes is 4-byte aligned), about 0.85 us per 64-byte block
+ *   (~75 MB/s; 1.5 us unaligned) — meant for short messages such as
  *   headers and test vectors; page contents use KVG_SHA256_PAGED.
  * KVG_SHA256_PAGED: n must be a multiple of page_bytes; out[32 * i] = the
  *   two-level digest of page i = bytes[i * page_bytes, (i+1) * page_bytes).

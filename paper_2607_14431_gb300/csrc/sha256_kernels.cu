@@ -833,6 +833,66 @@ __global__ void __launch_bounds__(32) sha256_serial_kernel(const uint8_t *seg0, 
     }
 }
 
+// sha256_serial_kernel's whole 64-byte blocks in the two-warp form: every
+// lane of both warps runs the same chain (lane 0's result is kept), warp 1
+// reads the message two blocks ahead, warp 0 runs the rounds; lane 0 of
+// warp 0 then finishes the tail and the padding with the byte-wise hasher.
+// For 4-byte aligned segments with seg0's length a multiple of 4.
+__global__ void __launch_bounds__(64) sha256_serial_split_kernel(const uint8_t *seg0, uint64_t n0, const uint8_t *seg1,
+                                                                 uint64_t n1, int32_t n_blocks, uint8_t *out,
+                                                                 const uint8_t *expected, DevStatus *status,
+                                                                 uint32_t one) {
+    __shared__ __align__(16) uint32_t kw[2][64][kSplitChains];
+    const int lane = threadIdx.x & 31;
+    if (blockIdx.x != 0) return;
+    if (threadIdx.x >= 32) {
+        uint32_t n1w[16], n2w[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            n1w[i] = n_blocks > 0 ? msg_word(seg0, n0, seg1, (uint64_t)i) : 0u;
+            n2w[i] = n_blocks > 1 ? msg_word(seg0, n0, seg1, 16ull + i) : 0u;
+        }
+        for (int blk = 0; blk < n_blocks; ++blk) {
+            uint32_t w[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                w[i] = bswap(n1w[i]);
+                n1w[i] = n2w[i];
+            }
+            if (blk + 2 < n_blocks) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) n2w[i] = msg_word(seg0, n0, seg1, 16ull * (blk + 2) + i);
+            }
+            split_hand_over(kw, w, blk, lane);
+        }
+        return;
+    }
+    uint32_t st[8];
+    split_consume(st, kw, n_blocks, lane, one);
+    if (lane != 0) return;
+    Stream s;
+    s.init(one);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s.st[i] = st[i];
+    const uint64_t done = 64ull * (uint64_t)n_blocks;
+    s.total = done;
+    if (done < n0) s.feed(seg0 + done, n0 - done);
+    const uint64_t d1 = done > n0 ? done - n0 : 0;
+    if (d1 < n1) s.feed(seg1 + d1, n1 - d1);
+    uint8_t dg[32];
+    s.final(dg);
+    if (out)
+        for (int k = 0; k < 32; ++k) out[k] = dg[k];
+    if (expected) {
+        bool same = true;
+        for (int k = 0; k < 32; ++k) same &= dg[k] == expected[k];
+        if (!same) {
+            atomicAdd(&status->n_mismatch, 1);
+            atomicCAS(&status->err, 0, (int32_t)KVG_ERR_DIGEST);
+        }
+    }
+}
+
 }  // namespace
 
 // The two-warp form is used for pages of whole 4 KiB leaves when a launch has
@@ -924,7 +984,13 @@ cudaError_t launch_sha256_pages(const uint32_t *leaf_words, int64_t n_pages, int
 cudaError_t launch_sha256_serial(const uint8_t *seg0, uint64_t n0, const uint8_t *seg1, uint64_t n1,
                                  uint8_t *out, const uint8_t *expected, DevStatus *status,
                                  cudaStream_t s) {
-    sha256_serial_kernel<<<1, 32, 0, s>>>(seg0, n0, seg1, n1, out, expected, status, 1u);
+    const bool aligned = !((reinterpret_cast<uintptr_t>(seg0) | reinterpret_cast<uintptr_t>(seg1) | n0) & 3);
+    const uint64_t n_blocks = (n0 + n1) / 64;
+    if (!split_off() && aligned && n_blocks >= 1 && n_blocks < (1ull << 30)) {
+        sha256_serial_split_kernel<<<1, 64, 0, s>>>(seg0, n0, seg1, n1, (int32_t)n_blocks, out, expected, status, 1u);
+    } else {
+        sha256_serial_kernel<<<1, 32, 0, s>>>(seg0, n0, seg1, n1, out, expected, status, 1u);
+    }
     count_launches(1);
     return cudaGetLastError();
 }
