@@ -554,3 +554,67 @@ def test_decodes_of_one_cache_on_two_streams_match_serial(oracle):
     for l in range(w.n_layers):
         compare_decode(oracle, ref_a[l, 0], oracle.gqa_decode(qa[l, 0], k[l], v[l], scale), what=f"stream a l {l}")
         compare_decode(oracle, ref_b[l, 0], oracle.gqa_decode(qb[l, 0], k[l], v[l], scale), what=f"stream b l {l}")
+
+
+_DIGEST_CHILD = r'''
+import sys
+sys.path.insert(0, sys.argv[1])
+sys.path.insert(0, sys.argv[1] + "/tests")
+import numpy as np, torch
+import kvg_synth as syn
+from kvg_testlib import append, dims_for, need_gpu, geometry
+kvg = need_gpu()
+rng = np.random.default_rng(91)
+out = []
+# paged digests of a small launch: 96 pages of 4 KiB and 40 pages of 64 KiB
+for n, pb in ((96, 4096), (40, 65536)):
+    buf = torch.from_numpy(rng.integers(0, 256, n * pb, dtype=np.uint8)).cuda()
+    o = torch.zeros(n * 32, dtype=torch.uint8, device="cuda")
+    kvg.kvg_digest(buf.data_ptr(), buf.numel(), kvg.KVG_SHA256_PAGED, pb, o.data_ptr())
+    out.append(bytes(o.cpu().numpy()).hex())
+# a plain digest of 100,000 bytes
+buf = torch.from_numpy(rng.integers(0, 256, 100000, dtype=np.uint8)).cuda()
+o = torch.zeros(32, dtype=torch.uint8, device="cuda")
+kvg.kvg_digest(buf.data_ptr(), buf.numel(), kvg.KVG_SHA256_PLAIN, 0, o.data_ptr())
+out.append(bytes(o.cpu().numpy()).hex())
+# a deposit and a verified graft of a 100-token block (tiny geometry: 4 KiB pages)
+w = geometry("tiny")
+k, v = syn.kv_rows(w, 100, 0x77)
+dims = dims_for(kvg, w)
+src = kvg.Cache(dims, 32, 1, 256)
+append(kvg, src, 0, syn.as_u16(k), syn.as_u16(v), syn.positions(0, 100))
+store = kvg.Store(dims, kvg.KVG_RESIDENCY_HBM, 1 << 24)
+bid = kvg.kvg_deposit(store.h, src.h, 0, 0, 100)
+out.append(kvg.kvg_store_export(store.h, bid).hex())
+dst = kvg.Cache(dims, 32, 1, 256)
+kvg.kvg_graft(store.h, bid, dst.h, 0, -1, 0, kvg.KVG_GRAFT_VERIFY | kvg.KVG_GRAFT_SYNC)
+print("\n".join(out))
+'''
+
+
+def test_two_warp_and_one_warp_hashing_agree_with_the_oracle(oracle):
+    """Small launches hash in the two-warp form; KVG_SHA_NO_SPLIT=1 keeps the
+    one-warp forms.  Both give the oracle's page digests, plain digest and
+    deposited block (whose page and block digests they compute), and a
+    verified graft of the block passes in both."""
+    import os
+    import subprocess
+    import sys
+    need_gpu()
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    res = []
+    for off in ("0", "1"):
+        env = dict(os.environ, KVG_SHA_NO_SPLIT=off)
+        r = subprocess.run([sys.executable, "-c", _DIGEST_CHILD, root], capture_output=True, text=True, timeout=600,
+                           env=env)
+        assert r.returncode == 0, r.stderr[-2000:]
+        res.append(r.stdout.strip().splitlines()[-4:])
+    assert res[0] == res[1]
+    rng = np.random.default_rng(91)
+    for got, (n, pb) in zip(res[0][:2], ((96, 4096), (40, 65536))):
+        assert bytes.fromhex(got) == oracle.page_digests(rng.integers(0, 256, n * pb, dtype=np.uint8), pb).tobytes()
+    assert bytes.fromhex(res[0][2]) == oracle.sha256(rng.integers(0, 256, 100000, dtype=np.uint8).tobytes())
+    w = geometry("tiny")
+    k, v = syn.kv_rows(w, 100, 0x77)
+    blk = oracle.block_from_kv(oracle_dims(oracle, w), syn.as_u16(k), syn.as_u16(v), syn.positions(0, 100))
+    assert bytes.fromhex(res[0][3]) == blk.serialize()
