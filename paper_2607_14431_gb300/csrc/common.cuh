@@ -283,8 +283,10 @@ cudaError_t launch_append_batch_e4m3(const AppendBatchParams &p, int n_sm, cudaS
 // Own-position graft (delta 0) fused with the leaf hashes of the copied pages:
 // leaf_words[(block page) * leaves_per_page + leaf] gets the leaf's state words.
 // ring_ok: a launch of a full wave or more may take the shared-memory ring form.
+// split_ok: a small launch may take the two-warp form (not for blocks read
+// from pinned host memory, whose loads are too slow for it).
 cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int n_sm, cudaStream_t s,
-                                bool ring_ok = true);
+                                bool ring_ok = true, bool split_ok = true);
 cudaError_t launch_append(const AppendParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_append_batch(const AppendBatchParams &p, int n_sm, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams &p, int n_sm, cudaStream_t s);

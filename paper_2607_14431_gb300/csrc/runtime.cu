@@ -1671,7 +1671,7 @@ static kvg_status graft_impl(kvg_store *s, uint64_t block_id, kvg_cache *c, int3
         // up without room for the ring's shared memory)
         if (one_pass)
             KVG_CUDA(launch_graft_verify(p, static_cast<uint32_t *>(c->leaf.ptr), c->n_sm, st,
-                                         c->dims.kv_dtype == KVG_KV_BF16));
+                                         c->dims.kv_dtype == KVG_KV_BF16, !host_src));
         else
             KVG_CUDA(launch_graft_copy(p, c->n_sm, st, host_src ? host_copy_ctas : 0, c->status));
         if (n_ev > 0) {

@@ -525,7 +525,7 @@ __global__ void __launch_bounds__(128) sha256_leaves_kernel(const PageSource src
 // registers, measured slower in the step).  For smaller launches each leaf's
 // chain latency decides: the register form is faster there (the tiny
 // verified graft 0.099 against 0.133 ms), and the two-warp form faster still
-// for launches of up to 32 leaves per SM (0.071 ms).
+// for launches of up to 64 leaves per SM (0.071 ms).
 constexpr int kGraftVerifyRing = 3;
 __global__ void __launch_bounds__(128, 5) graft_verify_ring_kernel(const GraftParams p, int64_t leaves_per_page,
                                                                    uint32_t *__restrict__ out, uint32_t one) {
@@ -896,12 +896,25 @@ __global__ void __launch_bounds__(64) sha256_serial_split_kernel(const uint8_t *
 }  // namespace
 
 // The two-warp form is used for pages of whole 4 KiB leaves when a launch has
-// at most one of its 32-chain CTAs per SM (leaves, 32 * n_sm) or four (page
-// digests, which read their input from L2); beyond that the one-warp forms
-// keep more chains going per SM.  KVG_SHA_NO_SPLIT=1 turns it off.
+// at most two of its 32-chain CTAs per SM (leaves) or four (page digests,
+// which read their input from L2); beyond that the one-warp forms keep more
+// chains going per SM.  KVG_SHA_NO_SPLIT=1 turns it off.
 static bool split_off() {
     static const bool off = env_knob("KVG_SHA_NO_SPLIT", 0) > 0;
     return off;
+}
+
+// Leaves per SM up to which a leaf-hashing launch takes the two-warp form:
+// two of its CTAs per SM (four warps, one per scheduler).  A verified graft
+// of 16 to 64 leaves per SM took 0.082-0.083 ms in it against 0.117 in the
+// one-warp form; at 96 and 128 leaves per SM 0.130-0.137 against 0.118-0.121.
+// A verified graft from pinned host memory keeps the one-warp form: its leaf
+// loads outlast the rounds of a block in the two-warp form (the last chunk of
+// the 12B block's host-store graft, 40 leaves per SM, made the e2e step
+// 15.73-15.83 ms instead of 15.63-15.71).
+static int split_leaves_per_sm() {
+    static const int v = env_knob("KVG_SHA_SPLIT_LEAVES_PER_SM", 2 * kSplitChains);
+    return v;
 }
 
 static int current_sm_count() {
@@ -917,7 +930,7 @@ cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_
     const int64_t m = (int64_t)((src.page_bytes + kLeafBytes - 1) / kLeafBytes);
     const int64_t n = n_pages * m;
     if (n == 0) return cudaSuccess;
-    if (!split_off() && src.page_bytes % kLeafBytes == 0 && n <= (int64_t)n_sm * kSplitChains) {
+    if (!split_off() && src.page_bytes % kLeafBytes == 0 && n <= (int64_t)n_sm * split_leaves_per_sm()) {
         sha256_leaves_split_kernel<<<(int)((n + kSplitChains - 1) / kSplitChains), 64, 0, s>>>(src, n_pages, m,
                                                                                              leaf_words, 1u);
         count_launches(1);
@@ -934,11 +947,12 @@ cudaError_t launch_sha256_leaves(const PageSource &src, int64_t n_pages, uint32_
     return cudaGetLastError();
 }
 
-cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int n_sm, cudaStream_t s, bool ring_ok) {
+cudaError_t launch_graft_verify(const GraftParams &p, uint32_t *leaf_words, int n_sm, cudaStream_t s, bool ring_ok,
+                                bool split_ok) {
     const int64_t m = (int64_t)((p.page_bytes + kLeafBytes - 1) / kLeafBytes);
     const int64_t n = (int64_t)p.n_layers * 2 * p.npb * m;
     if (n == 0) return cudaSuccess;
-    if (!split_off() && p.page_bytes % kLeafBytes == 0 && n <= (int64_t)n_sm * kSplitChains) {
+    if (split_ok && !split_off() && p.page_bytes % kLeafBytes == 0 && n <= (int64_t)n_sm * split_leaves_per_sm()) {
         graft_verify_split_kernel<<<(int)((n + kSplitChains - 1) / kSplitChains), 64, 0, s>>>(p, m, leaf_words, 1u);
         count_launches(1);
         return cudaGetLastError();
