@@ -134,6 +134,23 @@ REL_TOL_RELOCATED = 2.0 ** -6
 RNE_FLOOR_RELOCATED = 0.25
 
 
+def check_rotation_rounding(oracle, got, ref, min_exact=0.999):
+    """Relocated keys against the fp64 rotation `ref`: the kernel rotates in
+    fp32 (cos/sin of the fp64 angle rounded to fp32), so its bf16 result
+    `got` (uint16 bits) is the correctly rounded fp64 value except where the
+    fp32 error straddles a rounding boundary.  There it is one bf16 step away
+    (same sign), or, where the pair's two products nearly cancel, within the
+    fp32 error of the products, 2^-21 of the rows' largest magnitude."""
+    rne = oracle.bf16_rne(ref)
+    g = np.asarray(got, np.uint16)
+    exact = g == rne
+    steps = np.abs((g & 0x7FFF).astype(np.int32) - (rne & 0x7FFF).astype(np.int32))
+    off = int((~exact).sum())
+    assert off <= max(2, (1.0 - min_exact) * exact.size), (off, exact.size)
+    near = np.abs(oracle.bf16_to_f64(g) - ref) <= 2.0 ** -21 * np.abs(ref).max()
+    assert np.all(exact | ((steps == 1) & ((g & 0x8000) == (rne & 0x8000))) | near)
+
+
 def compare_decode(oracle, o_gpu_bits: np.ndarray, o_ref: np.ndarray, tol=1e-2, rel=REL_TOL, floor=RNE_FLOOR,
                    what=""):
     """Checks one decode output against the fp64 oracle with the three bounds

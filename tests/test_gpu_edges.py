@@ -9,7 +9,8 @@ import pytest
 import torch
 
 import kvg_synth as syn
-from kvg_testlib import (CANARY, append, compare_decode, decode, dims_for, fill_canary, geometry, need_gpu,
+from kvg_testlib import (CANARY, append, check_rotation_rounding, compare_decode, decode, dims_for, fill_canary, geometry,
+                         need_gpu,
                          oracle_dims, pool_u16, tables, to_dev, u16)
 
 pytestmark = pytest.mark.gpu
@@ -343,6 +344,7 @@ def test_graft_of_pages_too_large_for_two_stages(oracle):
             j, r = divmod(t, P)
             kg[:, t] = pool[:, 0, pt[1, j], :, r, :]
         assert np.abs(oracle.bf16_to_f64(kg) - k64).max() <= 2e-2
+        check_rotation_rounding(oracle, kg, k64)
         j, r = divmod(nb, P)  # padding rows of the last page: copied unchanged (zeros)
         assert not pool[:, 0, pt[1, j], :, r:, :].any()
         kvg.kvg_sync(c.h)

@@ -14,7 +14,7 @@ import pytest
 import torch
 
 import kvg_synth as syn
-from kvg_testlib import compare_decode, dev_view, need_gpu, tables
+from kvg_testlib import check_rotation_rounding, compare_decode, dev_view, need_gpu, tables
 
 pytestmark = pytest.mark.gpu
 
@@ -200,6 +200,7 @@ def test_31b_relocation_full_size(oracle):
                 else:
                     ref = oracle.rope_rotate_rows(rows_k, d, w.rope_theta, 0)
                     assert np.abs(oracle.bf16_to_f64(kpage) - ref).max() <= 2e-2
+                    check_rotation_rounding(oracle, kpage, ref)
         # the fresh rows landed where the oracle's bookkeeping puts them (one
         # sampled page per sampled sequence and layer)
         for sq in seqs:
@@ -279,6 +280,7 @@ def test_batched_library_full_size(oracle, consecutive):
                         if kv == 0 and d:
                             ref = oracle.rope_rotate_rows(want, d, w.rope_theta, 0)
                             assert np.abs(oracle.bf16_to_f64(got) - ref).max() <= 2e-2
+                            check_rotation_rounding(oracle, got, ref)
                         else:
                             assert np.array_equal(got, want)
                 j0 += blk.n_pages

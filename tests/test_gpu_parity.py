@@ -13,7 +13,8 @@ import pytest
 import torch
 
 import kvg_synth as syn
-from kvg_testlib import (CANARY, REL_TOL_RELOCATED, RNE_FLOOR_RELOCATED, append, compare_decode, decode, dev_view,
+from kvg_testlib import (CANARY, REL_TOL_RELOCATED, RNE_FLOOR_RELOCATED, append, check_rotation_rounding, compare_decode,
+                         decode, dev_view,
                          dims_for, fill_canary, geometry, need_gpu, oracle_dims, pool_u16, tables, to_dev, u16)
 
 pytestmark = pytest.mark.gpu
@@ -335,6 +336,7 @@ def test_relocated_graft_within_tolerance(oracle, geo, style):
                         for l in range(w.n_layers)])
         err = np.abs(oracle.bf16_to_f64(kg) - k64).max()
         assert err <= 2e-2, err
+        check_rotation_rounding(oracle, kg, k64)  # finer than the tolerance
         # bytes outside every key row ever rotated (released pages keep theirs) equal the oracle's
         for t in range(nb):
             j, r = divmod(t, w.page_size)
@@ -637,6 +639,7 @@ def test_relocate_to_consecutive_composition(oracle, geo, style, residency):
         else:
             k64 = np.stack([oracle.rope_rotate_rows(k[l], d, w.rope_theta, style) for l in range(w.n_layers)])
             assert np.abs(oracle.bf16_to_f64(kg) - k64).max() <= 2e-2
+            check_rotation_rounding(oracle, kg, k64)
         for t in range(n):
             mask[:, pt[1, j0 + t // P], :, t % P] = False
         j0 += -(-n // P)
@@ -1070,6 +1073,7 @@ def test_launch_chunking_limits(oracle):
     kg = _logical_k(pool, pt, w, 1, n)
     k64 = oracle.rope_rotate_rows(k[0], 77, w.rope_theta, 0)
     assert np.abs(oracle.bf16_to_f64(kg[0]) - k64).max() <= 2e-2
+    check_rotation_rounding(oracle, kg[0], k64)
     # 300 decode rows over the two sequences (rows alternate; 2 batch chunks)
     ids = [i % 2 for i in range(300)]
     q = syn.as_u16(syn.queries(w, 1, 300, 142))

@@ -16,7 +16,8 @@ import pytest
 import torch
 
 import kvg_synth as syn
-from kvg_testlib import (CANARY, append, compare_decode, decode, dev_view, dims_for, fill_canary, need_gpu,
+from kvg_testlib import (CANARY, append, check_rotation_rounding, compare_decode, decode, dev_view, dims_for,
+                         fill_canary, need_gpu,
                          oracle_dims, pool_u16, tables, to_dev, u16)
 
 pytestmark = pytest.mark.gpu
@@ -123,6 +124,7 @@ def test_random_scenario_matches_oracle(oracle, seed):
                         for l in range(L)])
         ref = np.stack([oracle.rope_rotate_rows(krows[b][l], delta, w.rope_theta, style) for l in range(L)])
         assert np.abs(oracle.bf16_to_f64(got) - ref).max() <= 2e-2, (sq, b, delta)
+        check_rotation_rounding(oracle, got, ref)
         for t in range(n):
             mask[:, pt[sq, (dst + t) // P], :, (dst + t) % P] = False
     assert np.array_equal(pool[:, 0][mask], oc.pool[:, 0][mask])
