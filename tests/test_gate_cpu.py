@@ -8,11 +8,16 @@ is where the gate's bounds come from (2^-7 relative, RNE-match floor 0.35),
 checked at a 4,096-row and a 32,768-row context.  The partial-context
 mistakes stay within the stated 1e-2 max-abs tolerance, which alone would
 pass them.  (A single wrong row out of thousands moves the output by less
-than the rounding does; the byte-exact pool comparisons catch those.)"""
+than the rounding does; the byte-exact pool comparisons catch those.)
+
+The re-basing check (kvg_testlib.check_rotation_rounding) likewise accepts a
+numpy model of the kernel's fp32 rotation and refuses planted mistakes:
+rotation by -delta, frequencies off by one index, the other pairing, and
+cos/sin rounded to bf16 (which the 2e-2 max-abs gate alone would pass)."""
 import numpy as np
 import pytest
 
-from kvg_testlib import RNE_FLOOR, REL_TOL, compare_decode
+from kvg_testlib import RNE_FLOOR, REL_TOL, check_rotation_rounding, compare_decode
 
 
 def _rows(oracle, rng, n, hkv, d):
@@ -67,3 +72,54 @@ def test_gate_passes_the_kernels_rounding_and_refuses_planted_mistakes(oracle, n
         with pytest.raises(AssertionError):
             compare_decode(oracle, bits(o), ref, what=name)
     assert blind >= 2
+
+
+def _fp32(x):
+    return np.asarray(x, np.float64).astype(np.float32).astype(np.float64)
+
+
+def _rotation_model(oracle, k_bits, delta, theta, style, sin_sign=1.0, freq_shift=0, trig_bf16=False):
+    """numpy model of the kernel's re-basing of bf16 key rows: cos/sin of the
+    fp64 angle delta * theta^(-2i/D) rounded to fp32, a' = fma(a, c, -(b s)),
+    b' = fma(a, s, b c) in fp32, then bf16 RNE; pairs (i, i + D/2) for style
+    0, (2i, 2i + 1) for style 1.  The keyword arguments plant mistakes."""
+    x = oracle.bf16_to_f64(k_bits)
+    d = x.shape[-1]
+    half = d // 2
+    ang = delta * theta ** (-2.0 * np.arange(half) / d)
+    rnd = (lambda t: oracle.bf16_to_f64(oracle.bf16_rne(t))) if trig_bf16 else _fp32
+    c, s = rnd(np.cos(ang)), rnd(np.sin(ang)) * sin_sign
+    if freq_shift:
+        c, s = np.roll(c, freq_shift), np.roll(s, freq_shift)
+    a, b = (x[..., :half], x[..., half:]) if style == 0 else (x[..., 0::2], x[..., 1::2])
+    ra = _fp32(a * c - _fp32(b * s))
+    rb = _fp32(a * s + _fp32(b * c))
+    out = np.empty_like(x)
+    if style == 0:
+        out[..., :half], out[..., half:] = ra, rb
+    else:
+        out[..., 0::2], out[..., 1::2] = ra, rb
+    return oracle.bf16_rne(out)
+
+
+@pytest.mark.parametrize("style", [0, 1])
+@pytest.mark.parametrize("delta,theta", [(1, 1e6), (4096, 1e6), (100000, 1e4)])
+def test_rotation_check_passes_fp32_rotation_and_refuses_planted_mistakes(oracle, style, delta, theta):
+    """kvg_testlib.check_rotation_rounding (used on every re-based key the GPU
+    writes) accepts a model of the kernel's fp32 arithmetic and refuses
+    plausible mistakes, including ones the 2e-2 max-abs gate would pass
+    (cos/sin rounded to bf16 instead of fp32)."""
+    rng = np.random.default_rng(delta + style)
+    k = oracle.bf16_rne(rng.standard_normal((512, 128)))
+    ref = oracle.rope_rotate_rows(k, delta, theta, style)
+    check_rotation_rounding(oracle, _rotation_model(oracle, k, delta, theta, style), ref)
+    planted = {"rotation by -delta": dict(sin_sign=-1.0), "frequency index off by one": dict(freq_shift=1),
+               "cos/sin rounded to bf16": dict(trig_bf16=True)}
+    for what, kw in planted.items():
+        bad = _rotation_model(oracle, k, delta, theta, style, **kw)
+        with pytest.raises(AssertionError):
+            check_rotation_rounding(oracle, bad, ref)
+    bf = _rotation_model(oracle, k, delta, theta, style, trig_bf16=True)
+    assert np.abs(oracle.bf16_to_f64(bf) - ref).max() <= 2e-2  # the coarse gate alone would pass it
+    with pytest.raises(AssertionError):  # the other pairing
+        check_rotation_rounding(oracle, _rotation_model(oracle, k, delta, theta, 1 - style), ref)
