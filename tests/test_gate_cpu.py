@@ -123,3 +123,20 @@ def test_rotation_check_passes_fp32_rotation_and_refuses_planted_mistakes(oracle
     assert np.abs(oracle.bf16_to_f64(bf) - ref).max() <= 2e-2  # the coarse gate alone would pass it
     with pytest.raises(AssertionError):  # the other pairing
         check_rotation_rounding(oracle, _rotation_model(oracle, k, delta, theta, 1 - style), ref)
+
+
+def test_max_abs_bound_allows_the_outputs_own_rounding_only(oracle):
+    """The max-abs bound is 1e-2 beyond half a bf16 step of the reference:
+    a correctly rounded output passes at any magnitude (|ref| ~ 5, where a
+    bf16 step is 2^-5 and the rounding alone can exceed 1e-2), while an
+    error of 0.015 on top of the rounding fails at |ref| ~ 0.5."""
+    rng = np.random.default_rng(11)
+    ref = 5.0 + rng.uniform(-0.9, 0.9, (4, 128))
+    rounded = oracle.bf16_rne(ref)
+    assert np.abs(oracle.bf16_to_f64(rounded) - ref).max() > 1e-2  # the rounding alone
+    compare_decode(oracle, rounded, ref, what="correctly rounded, |ref| ~ 5")
+    small = 0.5 + rng.uniform(-0.2, 0.2, (4, 128))
+    off = small.copy()
+    off[1, 7] += 0.015
+    with pytest.raises(AssertionError, match="max-abs"):
+        compare_decode(oracle, oracle.bf16_rne(off), small, rel=1.0, floor=0.0, what="0.015 off at |ref| ~ 0.5")

@@ -10,6 +10,7 @@ gate, whole and split at a random page boundary into two merged parts
 scenarios (own-position grafts and appends).  The scenarios are drawn from
 fixed seeds, so a failure names a case that reproduces."""
 import math
+import os
 
 import numpy as np
 import pytest
@@ -24,7 +25,8 @@ pytestmark = pytest.mark.gpu
 
 # (head_dim, query group) pairs the decode kernel is built for (bf16)
 GROUPS = {64: (1, 2, 4, 8), 128: (1, 2, 4), 256: (1, 2)}
-N_CASES = 64
+# KVG_RANDOM_CASES widens the draw for a longer soak (default 64)
+N_CASES = int(os.environ.get("KVG_RANDOM_CASES", "64"))
 
 
 def _case(seed):
