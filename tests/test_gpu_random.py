@@ -27,6 +27,7 @@ pytestmark = pytest.mark.gpu
 GROUPS = {64: (1, 2, 4, 8), 128: (1, 2, 4), 256: (1, 2)}
 # KVG_RANDOM_CASES widens the draw for a longer soak (default 64)
 N_CASES = int(os.environ.get("KVG_RANDOM_CASES", "64"))
+N_FP8_CASES = int(os.environ.get("KVG_RANDOM_FP8_CASES", "16"))
 
 
 def _case(seed):
@@ -165,7 +166,7 @@ def test_random_scenario_matches_oracle(oracle, seed):
 FP8_GROUPS = {128: (1, 2, 4), 256: (1, 2)}
 
 
-@pytest.mark.parametrize("seed", range(16))
+@pytest.mark.parametrize("seed", range(N_FP8_CASES))
 def test_random_fp8_scenario_matches_oracle(oracle, seed):
     """The same for fp8 E4M3 caches with random per-tensor scales: own-position
     grafts and appends only (relocation needs bf16 keys); pool codes, tables
