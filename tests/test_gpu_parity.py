@@ -836,6 +836,13 @@ def test_prefetch_then_graft_is_bit_exact(oracle, residency):
     with pytest.raises(kvg.KvgError) as e:
         kvg.kvg_store_prefetch(s["store"].h, s["bid"] + 1, side)
     assert e.value.status == kvg.KVG_ERR_NOT_FOUND
+    # a block held in a cache's own pool needs no translations: nothing to do
+    pc = kvg.Cache(s["dims"], 64, 1, 1024)
+    append(kvg, pc, 0, s["k"][:, :100], s["v"][:, :100], syn.positions(0, 100))
+    pool = kvg.PoolStore(pc, 1 << 26)
+    pbid = kvg.kvg_deposit(pool.h, pc.h, 0, 0, 100)
+    kvg.kvg_store_prefetch(pool.h, pbid, side)
+    side.synchronize()
 
 
 def test_block_files_round_trip_and_are_verified(oracle, tmp_path):
